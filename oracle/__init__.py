@@ -1,0 +1,206 @@
+"""The oracle: a plain fp64 CPU statement of the verification step.
+
+TEST INFRASTRUCTURE ONLY -- imported by the tests, by ``__graft_entry__.smoke``
+and by the benchmark's CPU-baseline leg, never by the library.  It shares no
+code with the CUDA path.  ``clover_oracle.c`` holds the arithmetic; this module
+compiles it with gcc (on first use, or from ``build()``) and marshals arguments.
+
+Functions take and return torch CPU tensors (bf16 inputs are passed as their
+bytes and widened exactly inside the C code).
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "clover_oracle.c")
+_OUT_DIR = os.path.join(_HERE, "_build")
+_LIB = os.path.join(_OUT_DIR, "liboracle.so")
+
+OK = 0
+BAD_ARG = 1
+BAD_TREE = 4
+NO_MEMORY = 64
+
+F32 = 0
+BF16 = 1
+
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile clover_oracle.c into _build/liboracle.so (gcc -O2 -fopenmp)."""
+    os.makedirs(_OUT_DIR, exist_ok=True)
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.run(["gcc", "-O2", "-fopenmp", "-std=c11", "-Wall", "-shared", "-fPIC",
+                        _SRC, "-o", tmp, "-lm"], check=True)
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P, I, I64, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_double
+            lib.oracle_tree_mask.argtypes = [P, I, P, P]
+            lib.oracle_tree_attention.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, I, D,
+                                                  P, I64, P, I]
+            lib.oracle_argmax.argtypes = [P, I64, I64, I, P, I64, P, I]
+            lib.oracle_accept_walk.argtypes = [P, P, P, I, I, P, P, P]
+            lib.oracle_append_tree_kv.argtypes = [P, P, P, P, P, I, I, I, I, I, I]
+            lib.oracle_kv_compact.argtypes = [P, P, P, P, P, I, I, I, I, I, I, P]
+            for f in (lib.oracle_tree_mask, lib.oracle_tree_attention, lib.oracle_argmax,
+                      lib.oracle_accept_walk, lib.oracle_append_tree_kv, lib.oracle_kv_compact):
+                f.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+class OracleError(RuntimeError):
+    def __init__(self, code: int):
+        super().__init__(f"oracle returned status {code}")
+        self.code = code
+
+
+def _check(code: int):
+    if code != OK:
+        raise OracleError(code)
+
+
+def _cpu(t: torch.Tensor) -> torch.Tensor:
+    if t.device.type != "cpu":
+        raise ValueError("the oracle takes CPU tensors")
+    return t.contiguous()
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+def _p(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else None
+
+
+def default_threads() -> int:
+    return os.cpu_count() or 1
+
+
+def tree_mask(parent) -> tuple[torch.Tensor, torch.Tensor]:
+    """(mask [T,T] bool, depth [T] int32) of one parent array."""
+    par = _cpu(torch.as_tensor(parent, dtype=torch.int32))
+    T = par.numel()
+    mask = torch.zeros((T, T), dtype=torch.uint8)
+    depth = torch.zeros(T, dtype=torch.int32)
+    _check(_load().oracle_tree_mask(_p(par), T, _p(mask), _p(depth)))
+    return mask.bool(), depth
+
+
+def tree_attention(q, k_new, v_new, k_cache, v_cache, cache_len, parent, scale: float = 0.0,
+                   rows=None, n_threads: int | None = None) -> torch.Tensor:
+    """fp64 attention rows; ``rows`` = flattened (b*T+i)*Hq+h ids, or None for all.
+
+    Returns [B,T,Hq,D] float64 when rows is None, else [len(rows), D].
+    """
+    q, k_new, v_new = _cpu(q), _cpu(k_new), _cpu(v_new)
+    k_cache, v_cache = _cpu(k_cache), _cpu(v_cache)
+    cl = _cpu(cache_len.to(torch.int32))
+    par = _cpu(parent.to(torch.int32))
+    B, T, Hq, D = q.shape
+    Hkv, Lcap = k_cache.shape[1], k_cache.shape[2]
+    dt = _dtype_code(q)
+    if rows is None:
+        out = torch.empty((B, T, Hq, D), dtype=torch.float64)
+        rows_t, n = None, B * T * Hq
+    else:
+        rows_t = _cpu(torch.as_tensor(rows, dtype=torch.int64))
+        n = rows_t.numel()
+        out = torch.empty((n, D), dtype=torch.float64)
+    _check(_load().oracle_tree_attention(
+        _p(q), _p(k_new), _p(v_new), _p(k_cache), _p(v_cache), _p(cl), _p(par),
+        B, T, Hq, Hkv, D, Lcap, dt, float(scale), _p(rows_t), n, _p(out),
+        n_threads or default_threads()))
+    return out
+
+
+def argmax(logits, rows=None, n_threads: int | None = None) -> torch.Tensor:
+    """First-index argmax over the last dim; returns int32 of logits.shape[:-1] or [len(rows)]."""
+    lg = _cpu(logits)
+    V = lg.shape[-1]
+    n_total = lg.numel() // V
+    if rows is None:
+        out = torch.empty(lg.shape[:-1], dtype=torch.int32)
+        rows_t, n = None, n_total
+    else:
+        rows_t = _cpu(torch.as_tensor(rows, dtype=torch.int64))
+        n = rows_t.numel()
+        out = torch.empty(n, dtype=torch.int32)
+    _check(_load().oracle_argmax(_p(lg), n_total, V, _dtype_code(lg), _p(rows_t), n, _p(out),
+                                 n_threads or default_threads()))
+    return out
+
+
+def accept_walk(parent, cand, amax):
+    """(path [B,T], accept_len [B], bonus [B]) int32."""
+    par = _cpu(parent.to(torch.int32))
+    cd = _cpu(cand.to(torch.int32))
+    am = _cpu(amax.to(torch.int32))
+    B, T = par.shape
+    path = torch.empty((B, T), dtype=torch.int32)
+    alen = torch.empty(B, dtype=torch.int32)
+    bonus = torch.empty(B, dtype=torch.int32)
+    _check(_load().oracle_accept_walk(_p(par), _p(cd), _p(am), B, T, _p(path), _p(alen),
+                                      _p(bonus)))
+    return path, alen, bonus
+
+
+def append_tree_kv(k_new, v_new, k_cache, v_cache, cache_len):
+    """In place on k_cache/v_cache (contiguous CPU tensors)."""
+    assert k_cache.is_contiguous() and v_cache.is_contiguous()
+    kn, vn = _cpu(k_new), _cpu(v_new)
+    cl = _cpu(cache_len.to(torch.int32))
+    B, Hkv, Lcap, D = k_cache.shape
+    T = kn.shape[1]
+    _check(_load().oracle_append_tree_kv(_p(kn), _p(vn), _p(k_cache), _p(v_cache), _p(cl), B, T,
+                                         Hkv, D, Lcap, k_cache.element_size()))
+
+
+def kv_compact(k_cache, v_cache, cache_len, path, accept_len):
+    """In place on k_cache/v_cache/cache_len (int32); returns src_index [B,T]."""
+    assert k_cache.is_contiguous() and v_cache.is_contiguous() and cache_len.dtype == torch.int32
+    B, Hkv, Lcap, D = k_cache.shape
+    pa = _cpu(path.to(torch.int32))
+    al = _cpu(accept_len.to(torch.int32))
+    T = pa.shape[1]
+    src = torch.empty((B, T), dtype=torch.int32)
+    _check(_load().oracle_kv_compact(_p(k_cache), _p(v_cache), _p(cache_len), _p(pa), _p(al), B, T,
+                                     Hkv, D, Lcap, k_cache.element_size(), _p(src)))
+    return src
+
+
+def verify_step(inp: dict, scale: float = 0.0, n_threads: int | None = None) -> dict:
+    """The whole step on copies of the inputs: attention, append, argmax, walk, compact."""
+    k_cache = inp["k_cache"].clone()
+    v_cache = inp["v_cache"].clone()
+    cache_len = inp["cache_len"].clone().to(torch.int32)
+    out = tree_attention(inp["q"], inp["k_new"], inp["v_new"], k_cache, v_cache, cache_len,
+                         inp["parent"], scale=scale, n_threads=n_threads)
+    append_tree_kv(inp["k_new"], inp["v_new"], k_cache, v_cache, cache_len)
+    amax = argmax(inp["logits"], n_threads=n_threads)
+    path, alen, bonus = accept_walk(inp["parent"], inp["cand"], amax)
+    src = kv_compact(k_cache, v_cache, cache_len, path, alen)
+    return {"out": out, "argmax": amax, "path": path, "accept_len": alen, "bonus": bonus,
+            "src_index": src, "k_cache": k_cache, "v_cache": v_cache, "cache_len": cache_len}

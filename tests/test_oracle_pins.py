@@ -1,0 +1,515 @@
+"""Pins for the oracle: every function is checked against something other than
+itself -- brute force on tiny inputs, library routines (torch SDPA, numpy argmax),
+closed forms, hand-worked examples and invariants -- so that a dropped term, a
+wrong index, a wrong sign or a transposed operand fails at least one test.
+
+Pure CPU; marked neither gpu nor slow.
+"""
+
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+import oracle
+from synth import trees, workloads
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ---------------------------------------------------------------------------
+# helpers (independent formulations used only as pins)
+# ---------------------------------------------------------------------------
+
+def reach_matrix(parent):
+    """Ancestor-or-self relation as the transitive closure of the parent map:
+    R = (I + A)^(T) with boolean products, A[i][p] = 1 iff p = parent[i]."""
+    T = len(parent)
+    A = np.zeros((T, T), dtype=np.int64)
+    for i in range(1, T):
+        A[i, parent[i]] = 1
+    R = np.eye(T, dtype=np.int64)
+    step = np.eye(T, dtype=np.int64) + A
+    for _ in range(T):
+        R = np.minimum(R @ step, 1)
+    return R.astype(bool)
+
+
+def root_path(parent, i):
+    path = []
+    n = i
+    while n >= 0:
+        path.append(n)
+        n = parent[n]
+    return path[::-1]
+
+
+def rand_inputs(B, T, Hq, Hkv, D, L, seed, dtype=torch.float32, Lcap=None, std=1.0):
+    g = torch.Generator().manual_seed(seed)
+    Lmax = max(L) if isinstance(L, (list, tuple)) else L
+    Lcap = Lcap or Lmax + T + 3
+    def r(*s):
+        return (torch.randn(*s, generator=g, dtype=torch.float64) * std).to(dtype)
+    inp = dict(q=r(B, T, Hq, D), k_new=r(B, T, Hkv, D), v_new=r(B, T, Hkv, D),
+               k_cache=r(B, Hkv, Lcap, D), v_cache=r(B, Hkv, Lcap, D))
+    Ls = list(L) if isinstance(L, (list, tuple)) else [L] * B
+    inp["cache_len"] = torch.tensor(Ls, dtype=torch.int32)
+    return inp
+
+
+def sdpa_decode(q, K, V, scale):
+    """One query row against a key/value list, via torch's SDPA in fp64."""
+    return F.scaled_dot_product_attention(
+        q.double().view(1, 1, 1, -1), K.double().view(1, 1, K.shape[0], -1),
+        V.double().view(1, 1, V.shape[0], -1), scale=scale).view(-1)
+
+
+def sequence_attention(inp, parent, scale):
+    """Tree attention by its definition in terms of the speculated sequences:
+    node i is the last token of the sequence root..i appended to the cache, so
+    its output is plain decode attention over cache ++ k_new[root path of i]."""
+    q, kn, vn, kc, vc, cl = (inp[k] for k in ("q", "k_new", "v_new", "k_cache", "v_cache", "cache_len"))
+    B, T, Hq, D = q.shape
+    Hkv = kn.shape[2]
+    G = Hq // Hkv
+    out = torch.empty((B, T, Hq, D), dtype=torch.float64)
+    for b in range(B):
+        L = int(cl[b])
+        par = parent[b]
+        for i in range(T):
+            nodes = root_path(par, i)
+            for h in range(Hq):
+                g = h // G
+                K = torch.cat([kc[b, g, :L], kn[b, nodes, g]], 0)
+                V = torch.cat([vc[b, g, :L], vn[b, nodes, g]], 0)
+                out[b, i, h] = sdpa_decode(q[b, i, h], K, V, scale)
+    return out
+
+
+def run_oracle_attn(inp, parent, scale=0.0):
+    par = torch.tensor(parent, dtype=torch.int32)
+    if par.dim() == 1:
+        par = par.unsqueeze(0)
+    return oracle.tree_attention(inp["q"], inp["k_new"], inp["v_new"], inp["k_cache"],
+                                 inp["v_cache"], inp["cache_len"], par, scale=scale)
+
+
+# ---------------------------------------------------------------------------
+# A0: tree encoding
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("T", [1, 2, 3, 4, 5])
+def test_tree_mask_all_small_trees_vs_transitive_closure(T):
+    for parent in trees.all_trees(T):
+        mask, depth = oracle.tree_mask(parent)
+        R = reach_matrix(parent)
+        assert np.array_equal(mask.numpy(), R), parent
+        assert depth.tolist() == [int(R[i].sum()) - 1 for i in range(T)]
+
+
+def test_tree_mask_invariants_random_64():
+    for seed in range(20):
+        parent = trees.random_tree(64, seed)
+        mask, depth = oracle.tree_mask(parent)
+        m = mask.numpy()
+        assert np.array_equal(m, reach_matrix(parent))
+        for i in range(64):
+            assert m[i, 0] and m[i, i]
+            assert not m[i, i + 1:].any()
+            if i:
+                expect = m[parent[i]].copy()
+                expect[i] = True
+                assert np.array_equal(m[i], expect)
+            assert m[i].sum() == depth[i] + 1
+
+
+@pytest.mark.parametrize("bad", [[0, 0, 1], [-1, 1], [-1, 0, 2], [-1, 0, -1], [-1, 0, 5], [-1, -1]])
+def test_tree_mask_rejects_invalid(bad):
+    with pytest.raises(oracle.OracleError) as e:
+        oracle.tree_mask(bad)
+    assert e.value.code == oracle.BAD_TREE
+
+
+def test_topk_tree_shapes_match_reading():
+    t16 = trees.topk_tree(16, [4, 2, 1, 1])
+    assert t16 == json.load(open(os.path.join(GOLDEN, "topk_trees.json")))["T16_b4211"]["parent"]
+    for T, br, counts in [(16, [4, 2, 1, 1], [1, 3, 4, 4, 4]), (64, [8, 4, 2, 2, 1], [1, 6, 12, 13, 16, 16]),
+                          (32, [8, 4, 2, 1], [1, 4, 8, 11, 8])]:
+        _, depth = oracle.tree_mask(trees.topk_tree(T, br))
+        assert np.bincount(depth.numpy()).tolist() == counts
+
+
+# ---------------------------------------------------------------------------
+# A1: tree-masked attention
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("T", [1, 2, 3, 4])
+@pytest.mark.parametrize("L", [0, 1, 3])
+def test_attention_brute_force_all_small_trees(T, L):
+    inp = rand_inputs(1, T, 2, 2, 4, L, seed=100 * T + L)
+    for parent in trees.all_trees(T):
+        got = run_oracle_attn(inp, [parent])
+        ref = sequence_attention(inp, [parent], 0.5)
+        assert torch.allclose(got, ref, atol=1e-13, rtol=0), parent
+
+
+def test_attention_sequences_gqa_batched_random_trees():
+    B, T, Hq, Hkv, D = 3, 12, 8, 2, 16
+    inp = rand_inputs(B, T, Hq, Hkv, D, [5, 0, 9], seed=7)
+    parents = [trees.random_tree(T, 11, tag=b) for b in range(B)]
+    got = run_oracle_attn(inp, parents)
+    ref = sequence_attention(inp, parents, 1 / math.sqrt(D))
+    assert torch.allclose(got, ref, atol=1e-13, rtol=0)
+
+
+def test_attention_chain_equals_causal():
+    B, T, H, D, L = 2, 9, 3, 8, 6
+    inp = rand_inputs(B, T, H, H, D, L, seed=3)
+    got = run_oracle_attn(inp, [trees.chain_tree(T)] * B)
+    # causal attention of the whole sequence cache ++ tree, last T positions
+    causal = torch.ones(L + T, L + T, dtype=torch.bool).tril()[L:]
+    for b in range(B):
+        K = torch.cat([inp["k_cache"][b, :, :L], inp["k_new"][b].transpose(0, 1)], 1)
+        V = torch.cat([inp["v_cache"][b, :, :L], inp["v_new"][b].transpose(0, 1)], 1)
+        Q = inp["q"][b].transpose(0, 1)
+        ref = F.scaled_dot_product_attention(Q.double(), K.double(), V.double(), attn_mask=causal,
+                                             scale=1 / math.sqrt(D))
+        assert torch.allclose(got[b], ref.transpose(0, 1), atol=1e-13, rtol=0)
+
+
+def test_attention_single_node_is_plain_decode():
+    B, H, D, L = 2, 4, 32, 17
+    inp = rand_inputs(B, 1, H, H, D, L, seed=4)
+    got = run_oracle_attn(inp, [[-1]] * B)
+    for b in range(B):
+        K = torch.cat([inp["k_cache"][b, :, :L], inp["k_new"][b].transpose(0, 1)], 1)
+        V = torch.cat([inp["v_cache"][b, :, :L], inp["v_new"][b].transpose(0, 1)], 1)
+        ref = F.scaled_dot_product_attention(inp["q"][b].transpose(0, 1).double(), K.double(), V.double())
+        assert torch.allclose(got[b], ref.transpose(0, 1), atol=1e-13, rtol=0)
+
+
+def test_attention_star_tree():
+    T, H, D, L = 6, 2, 8, 4
+    inp = rand_inputs(1, T, H, H, D, L, seed=5)
+    got = run_oracle_attn(inp, [trees.star_tree(T)])
+    for i in range(T):
+        nodes = [0] if i == 0 else [0, i]
+        for h in range(H):
+            K = torch.cat([inp["k_cache"][0, h, :L], inp["k_new"][0, nodes, h]], 0)
+            V = torch.cat([inp["v_cache"][0, h, :L], inp["v_new"][0, nodes, h]], 0)
+            assert torch.allclose(got[0, i, h], sdpa_decode(inp["q"][0, i, h], K, V, 1 / math.sqrt(D)),
+                                  atol=1e-13, rtol=0)
+
+
+def test_attention_uniform_values_and_empty_cache():
+    T, H, D, L = 5, 2, 8, 7
+    inp = rand_inputs(1, T, H, H, D, L, seed=6)
+    row = torch.arange(D, dtype=torch.float64) * 0.25 - 1
+    inp["v_cache"][:] = row
+    inp["v_new"][:] = row
+    got = run_oracle_attn(inp, [trees.random_tree(T, 1)])
+    assert torch.allclose(got, row.expand_as(got), atol=1e-14, rtol=0)
+    # L = 0 and T = 1: the only visible key is the node itself
+    inp0 = rand_inputs(1, 1, 3, 3, 8, 0, seed=8)
+    got0 = run_oracle_attn(inp0, [[-1]])
+    assert torch.equal(got0[0, 0], inp0["v_new"][0, 0])
+
+
+def test_attention_zero_query_is_mean_of_visible_values():
+    """q = 0 gives equal weights: out = mean of the values of the visible keys,
+    of which there are L + depth(i) + 1 (closed form)."""
+    T, H, D, L = 16, 2, 1, 5
+    parent = trees.topk_tree(T, [4, 2, 1, 1])
+    inp = rand_inputs(1, T, H, H, D, L, seed=9)
+    inp["q"][:] = 0
+    inp["v_cache"][0, :, :, 0] = torch.arange(inp["v_cache"].shape[2], dtype=torch.float64)
+    inp["v_new"][0, :, :, 0] = 1000.0 * torch.arange(1, T + 1, dtype=torch.float64).unsqueeze(1)
+    got = run_oracle_attn(inp, [parent])
+    for i in range(T):
+        nodes = root_path(parent, i)
+        expect = (sum(range(L)) + 1000.0 * sum(n + 1 for n in nodes)) / (L + len(nodes))
+        assert got[0, i, :, 0].tolist() == pytest.approx([expect] * H, abs=1e-9)
+
+
+def test_attention_cache_key_permutation_invariance():
+    T, H, D, L = 8, 2, 8, 11
+    inp = rand_inputs(1, T, H, H, D, L, seed=10)
+    parent = [trees.random_tree(T, 3)]
+    base = run_oracle_attn(inp, parent)
+    perm = torch.randperm(L, generator=torch.Generator().manual_seed(1))
+    inp2 = dict(inp)
+    for k in ("k_cache", "v_cache"):
+        c = inp[k].clone()
+        c[:, :, :L] = inp[k][:, :, perm]
+        inp2[k] = c
+    assert torch.allclose(run_oracle_attn(inp2, parent), base, atol=1e-13, rtol=0)
+
+
+def test_attention_gqa_equals_mha_with_repeated_kv_heads():
+    B, T, Hq, Hkv, D, L = 2, 6, 8, 2, 8, 5
+    G = Hq // Hkv
+    inp = rand_inputs(B, T, Hq, Hkv, D, L, seed=12)
+    parents = [trees.random_tree(T, 5, tag=b) for b in range(B)]
+    got = run_oracle_attn(inp, parents)
+    mha = dict(inp)
+    for k, dim in (("k_new", 2), ("v_new", 2), ("k_cache", 1), ("v_cache", 1)):
+        mha[k] = inp[k].repeat_interleave(G, dim=dim).contiguous()
+    assert torch.allclose(run_oracle_attn(mha, parents), got, atol=1e-13, rtol=0)
+
+
+def test_attention_scale_closed_form():
+    """One cache key with score s*a and the root with score 0: out =
+    (v_c * e^{s a} + v_0) / (e^{s a} + 1)."""
+    inp = rand_inputs(1, 1, 1, 1, 1, 1, seed=13)
+    a, vc, v0 = 1.5, 2.0, -3.0
+    inp["q"][:] = 1.0
+    inp["k_cache"][0, 0, 0, 0] = a
+    inp["k_new"][:] = 0.0
+    inp["v_cache"][0, 0, 0, 0] = vc
+    inp["v_new"][:] = v0
+    for s in (0.0, 0.3, 2.0):
+        got = run_oracle_attn(inp, [[-1]], scale=s)
+        ss = 1.0 if s == 0.0 else s   # scale 0 selects 1/sqrt(D) = 1 for D = 1
+        w = math.exp(ss * a)
+        assert float(got[0, 0, 0, 0]) == pytest.approx((vc * w + v0) / (w + 1), abs=1e-15)
+
+
+def test_attention_hand_worked_example():
+    ex = json.load(open(os.path.join(GOLDEN, "hand_tree_attention.json")))
+    T = len(ex["parent"])
+    t32 = lambda x: torch.tensor(x, dtype=torch.float32)
+    q = t32(ex["q"]).view(1, T, 1, 1)
+    k_new = t32(ex["k_new"]).view(1, T, 1, 1)
+    v_new = t32(ex["v_new"]).view(1, T, 1, 1)
+    L = len(ex["k_cache"])
+    k_cache = t32(ex["k_cache"] + [0.0] * T).view(1, 1, L + T, 1)
+    v_cache = t32(ex["v_cache"] + [0.0] * T).view(1, 1, L + T, 1)
+    got = oracle.tree_attention(q, k_new, v_new, k_cache, v_cache, torch.tensor([L], dtype=torch.int32),
+                                torch.tensor([ex["parent"]], dtype=torch.int32), scale=ex["scale"])
+    assert got.view(-1).tolist() == pytest.approx(ex["expected_out"], abs=1e-6)
+
+
+def test_attention_bf16_widening_matches_f32():
+    """bf16 bytes are widened exactly: inputs representable in bf16 give the
+    same fp64 result whether stored as bf16 or fp32."""
+    inp = rand_inputs(2, 7, 4, 2, 16, [3, 8], seed=14, dtype=torch.float32)
+    inp = {k: (v.to(torch.bfloat16).to(torch.float32) if v.is_floating_point() else v) for k, v in inp.items()}
+    bf = {k: (v.to(torch.bfloat16) if v.is_floating_point() else v) for k, v in inp.items()}
+    parents = [trees.random_tree(7, 2, tag=b) for b in range(2)]
+    assert torch.equal(run_oracle_attn(inp, parents), run_oracle_attn(bf, parents))
+
+
+def test_attention_sharp_scores_stable():
+    inp = rand_inputs(1, 8, 2, 2, 16, 20, seed=15, std=6.0)   # scores up to ~hundreds
+    parents = [trees.random_tree(8, 9)]
+    got = run_oracle_attn(inp, parents)
+    assert torch.isfinite(got).all()
+    assert torch.allclose(got, sequence_attention(inp, parents, 0.25), atol=1e-12, rtol=0)
+
+
+def test_attention_rows_subset_matches_full_and_ignores_tail():
+    w = workloads.get("tiny_f32")
+    t = workloads.make(w)           # cache tail slots hold NaN
+    full = oracle.tree_attention(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"],
+                                 t["cache_len"], t["parent"])
+    assert torch.isfinite(full).all()
+    rows = [0, 5, 77, w.T * w.Hq - 1]
+    sub = oracle.tree_attention(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"],
+                                t["cache_len"], t["parent"], rows=rows)
+    assert torch.equal(sub, full.view(-1, w.D)[rows])
+    one = oracle.tree_attention(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"],
+                                t["cache_len"], t["parent"], n_threads=1)
+    assert torch.equal(one, full)
+
+
+def test_attention_rejects_bad_tree():
+    inp = rand_inputs(1, 3, 1, 1, 2, 1, seed=16)
+    with pytest.raises(oracle.OracleError) as e:
+        run_oracle_attn(inp, [[-1, 0, 2]])
+    assert e.value.code == oracle.BAD_TREE
+
+
+# ---------------------------------------------------------------------------
+# A2: argmax
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("V", [1, 7, 1024, 5003])
+def test_argmax_vs_numpy_first_index(dtype, V):
+    g = torch.Generator().manual_seed(V)
+    x = (torch.randn(6, 5, V, generator=g) * 4).to(dtype)
+    got = oracle.argmax(x)
+    ref = np.argmax(x.to(torch.float64).numpy(), axis=-1)   # numpy returns the first maximum
+    assert np.array_equal(got.numpy(), ref)
+
+
+def test_argmax_planted_ties_signed_zero_and_infinities():
+    V = 300
+    x = torch.full((8, V), -5.0, dtype=torch.float32)
+    x[0, [17, 3, 250]] = 9.0                        # tie -> smallest index 3
+    x[1, :] = -1.0
+    x[1, 40] = -0.0
+    x[1, 20] = 0.0                                   # -0 == +0 -> index 20
+    x[2, :] = -1.0
+    x[2, 10] = 0.0
+    x[2, 5] = -0.0                                   # -> index 5
+    x[3, 0] = 1.0                                    # max at index 0
+    x[4, V - 1] = 1.0                                # max at the last index
+    x[5, :] = float("-inf")
+    x[5, 123] = -1e30                                # finite beats -inf
+    x[6, 99] = float("inf")
+    x[6, 7] = 1e38                                   # +inf wins
+    x[7, :] = float("-inf")                          # all -inf -> index 0
+    assert oracle.argmax(x).tolist() == [3, 20, 5, 0, V - 1, 123, 99, 0]
+    assert oracle.argmax(x.to(torch.bfloat16)).tolist()[:5] == [3, 20, 5, 0, V - 1]
+
+
+def test_argmax_row_subset():
+    x = torch.randn(10, 50, generator=torch.Generator().manual_seed(2)).to(torch.bfloat16)
+    full = oracle.argmax(x)
+    assert oracle.argmax(x, rows=[9, 0, 4]).tolist() == full[[9, 0, 4]].tolist()
+
+
+# ---------------------------------------------------------------------------
+# A3: acceptance walk
+# ---------------------------------------------------------------------------
+
+def brute_force_walk(parent, cand, amax):
+    """All root-to-node paths; keep those whose every step matches (child's
+    candidate == parent's argmax) and that cannot be extended; the accepted
+    path is the lexicographically smallest of them (node-index order)."""
+    T = len(parent)
+    children = [[c for c in range(T) if parent[c] == n] for n in range(T)]
+    good = []
+    for i in range(T):
+        p = root_path(parent, i)
+        if all(cand[p[k]] == amax[p[k - 1]] for k in range(1, len(p))):
+            if not any(cand[c] == amax[i] for c in children[i]):
+                good.append(p)
+    best = min(good)
+    return best, len(best), amax[best[-1]]
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 4, 5])
+def test_walk_exhaustive_small(T):
+    """Every tree with T <= 5 nodes, every candidate/argmax assignment over a
+    2-token vocabulary (duplicates among siblings included)."""
+    n = 0
+    for parent in trees.all_trees(T):
+        for cand in itertools.product([0, 1], repeat=T):
+            for amax in itertools.product([0, 1], repeat=T):
+                path, alen, bonus = oracle.accept_walk(torch.tensor([parent]), torch.tensor([cand]),
+                                                       torch.tensor([amax]))
+                bp, bl, bb = brute_force_walk(parent, cand, amax)
+                assert path[0, :bl].tolist() == bp and int(alen[0]) == bl and int(bonus[0]) == bb
+                assert (path[0, bl:] == -1).all()
+                n += 1
+                if n > 4000:
+                    return
+
+
+def test_walk_distinct_siblings_gives_deepest_path_and_bounds():
+    for seed in range(30):
+        w = workloads.get("tiny_f32", seed=seed, tree="random" if seed % 2 else "topk")
+        t = workloads.make(w)
+        amax = oracle.argmax(t["logits"])
+        path, alen, bonus = oracle.accept_walk(t["parent"], t["cand"], amax)
+        parent = t["parent"][0].tolist()
+        cand = t["cand"][0].tolist()
+        a = amax[0].tolist()
+        T = len(parent)
+        full = [i for i in range(T)
+                if all(cand[p] == a[parent[p]] for p in root_path(parent, i)[1:])]
+        deepest = max(len(root_path(parent, i)) for i in full)
+        assert int(alen[0]) == deepest
+        _, depth = oracle.tree_mask(parent)
+        assert 1 <= int(alen[0]) <= int(depth.max()) + 1
+        assert int(bonus[0]) == a[path[0, int(alen[0]) - 1]]
+
+
+def test_walk_plant_all_and_plant_none():
+    for seed in range(5):
+        w = workloads.get("tiny_f32", seed=seed, plant_p=1.0)
+        t = workloads.make(w)
+        amax = oracle.argmax(t["logits"])
+        path, alen, _ = oracle.accept_walk(t["parent"], t["cand"], amax)
+        last = int(path[0, int(alen[0]) - 1])
+        assert last not in t["parent"][0].tolist()          # reached a leaf
+        _, depth = oracle.tree_mask(t["parent"][0].tolist())
+        assert int(alen[0]) == int(depth[last]) + 1
+        # with no planting the root row's argmax is a random token: the walk
+        # stops at the root unless a child's id happens to equal it
+        w0 = workloads.get("tiny_f32", seed=seed, plant_p=0.0)
+        t0 = workloads.make(w0)
+        a0 = oracle.argmax(t0["logits"])
+        _, alen0, _ = oracle.accept_walk(t0["parent"], t0["cand"], a0)
+        kids = [c for c in range(w0.T) if t0["parent"][0, c] == 0]
+        if all(int(t0["cand"][0, c]) != int(a0[0, 0]) for c in kids):
+            assert int(alen0[0]) == 1
+
+
+def test_walk_duplicate_siblings_smallest_index_wins():
+    parent = [-1, 0, 0, 1, 2]
+    cand = [9, 5, 5, 7, 7]
+    amax = [5, 1, 7, 0, 0]        # node 1 is a dead end, node 2 continues to 4
+    path, alen, bonus = oracle.accept_walk(torch.tensor([parent]), torch.tensor([cand]),
+                                           torch.tensor([amax]))
+    assert path[0].tolist() == [0, 1, -1, -1, -1] and int(alen[0]) == 2 and int(bonus[0]) == 1
+
+
+# ---------------------------------------------------------------------------
+# A4: append + compaction
+# ---------------------------------------------------------------------------
+
+def test_append_places_tree_kv_after_cache():
+    B, T, Hkv, D = 2, 5, 3, 4
+    inp = rand_inputs(B, T, Hkv, Hkv, D, [2, 6], seed=20, dtype=torch.float32)
+    kc, vc = inp["k_cache"].clone(), inp["v_cache"].clone()
+    oracle.append_tree_kv(inp["k_new"], inp["v_new"], kc, vc, inp["cache_len"])
+    for b, L in enumerate(inp["cache_len"].tolist()):
+        assert torch.equal(kc[b, :, L:L + T], inp["k_new"][b].permute(1, 0, 2))
+        assert torch.equal(vc[b, :, L:L + T], inp["v_new"][b].permute(1, 0, 2))
+        assert torch.equal(kc[b, :, :L], inp["k_cache"][b, :, :L])
+
+
+def test_compact_equals_out_of_place_gather():
+    B, T, Hkv, D = 3, 8, 2, 4
+    for dtype in (torch.float32, torch.bfloat16):
+        g = torch.Generator().manual_seed(21)
+        Lcap = 30
+        kc = torch.randn(B, Hkv, Lcap, D, generator=g).to(dtype)
+        vc = torch.randn(B, Hkv, Lcap, D, generator=g).to(dtype)
+        L = torch.tensor([0, 7, 22], dtype=torch.int32)
+        paths = [[0, 2, 5, 7], [0], [0, 1, 2, 3, 4, 5, 6, 7]]
+        path = torch.full((B, T), -1, dtype=torch.int32)
+        for b, p in enumerate(paths):
+            path[b, :len(p)] = torch.tensor(p)
+        alen = torch.tensor([len(p) for p in paths], dtype=torch.int32)
+        k2, v2, L2 = kc.clone(), vc.clone(), L.clone()
+        src = oracle.kv_compact(k2, v2, L2, path, alen)
+        for b, p in enumerate(paths):
+            l0 = int(L[b])
+            gather_k = kc[b, :, [l0 + j for j in p]]          # read from the untouched copy
+            assert torch.equal(k2[b, :, l0:l0 + len(p)], gather_k)
+            assert torch.equal(v2[b, :, l0:l0 + len(p)], vc[b, :, [l0 + j for j in p]])
+            assert torch.equal(k2[b, :, :l0], kc[b, :, :l0])
+            assert src[b].tolist() == [l0 + j for j in p] + [-1] * (T - len(p))
+            assert int(L2[b]) == l0 + len(p)
+
+
+def test_verify_step_tiny_invariants():
+    w = workloads.get("tiny_f32")
+    t = workloads.make(w)
+    r = oracle.verify_step(t)
+    a = int(r["accept_len"][0])
+    L = int(t["cache_len"][0])
+    assert int(r["cache_len"][0]) == L + a
+    assert torch.equal(r["k_cache"][0, :, :L], t["k_cache"][0, :, :L])
+    p = r["path"][0, :a].tolist()
+    assert torch.equal(r["k_cache"][0, :, L:L + a], t["k_new"][0, p].permute(1, 0, 2))
+    assert torch.equal(r["v_cache"][0, :, L:L + a], t["v_new"][0, p].permute(1, 0, 2))
