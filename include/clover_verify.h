@@ -1,0 +1,171 @@
+/*
+ * clover_verify.h -- C ABI of the GB300 (sm_103a) verification step of
+ * Clover-style tree speculative decoding (arXiv 2405.00263).
+ *
+ * One verification step (Section 2.1, "verification phase"): the base model
+ * scores all T speculated tokens, arranged as a token tree, in one pass.  The
+ * library provides the data-parallel hot path of that pass:
+ *
+ *   clover_verify_attn    tree-masked attention of the T tree queries against
+ *                         the committed KV cache plus the T new keys
+ *                         (Section 2.2, Tree Attention);
+ *   clover_verify_accept  per-node argmax of the logits and the greedy walk
+ *                         that selects the accepted path (Section 2.1; the
+ *                         tokens/step metric of Section 4.1);
+ *   clover_kv_compact     moves the accepted nodes' K/V to the front of the
+ *                         tree slots (an engine step the paper leaves implicit).
+ *
+ * Conventions shared by every entry point
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *     never allocates, frees or retains them.  Tensors are dense row-major.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t passed as void*;
+ *     NULL = the legacy default stream).  The return value reports errors
+ *     found on the host before anything is launched (and launch failures);
+ *     nothing is launched when it is not CLOVER_OK.
+ *   - Errors found on the device (an invalid parent array, a cache that is too
+ *     small, an invalid path) are OR-ed into `*status` (a device int32 the
+ *     caller zeroes; may be NULL).  Kernels never trap and never wait without
+ *     a bound; outputs are unspecified when a status bit is set.
+ *   - Token tree: parent[b][0] == -1 (node 0 is the root) and
+ *     0 <= parent[b][i] < i for i >= 1, so nodes are topologically numbered.
+ *     Node i attends to node j iff j is i or an ancestor of i (the tree's
+ *     topology as the attention mask, Section 2.2).
+ *   - Limits: 1 <= T <= 64, D in {64, 128}, Hq a multiple of Hkv (query head h
+ *     reads KV head h / (Hq/Hkv)), cache_len[b] + T <= Lcap.
+ */
+#ifndef CLOVER_VERIFY_H
+#define CLOVER_VERIFY_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define CLOVER_API __attribute__((visibility("default")))
+#else
+#define CLOVER_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    CLOVER_OK = 0,
+    CLOVER_ERR_INVALID_ARG = 1,  /* bad size, NULL or misaligned pointer, short workspace */
+    CLOVER_ERR_UNSUPPORTED = 2,  /* outside the limits above (T > 64, D not 64/128, ...) */
+    CLOVER_ERR_BAD_TREE = 4,     /* device: parent array is not a topologically numbered tree */
+    CLOVER_ERR_CAPACITY = 8,     /* device: cache_len[b] < 0 or cache_len[b] + T > Lcap */
+    CLOVER_ERR_CUDA = 16,        /* a CUDA launch or query failed */
+    CLOVER_ERR_TIMEOUT = 32      /* reserved: a bounded device wait gave up */
+} clover_status;
+
+typedef enum {
+    CLOVER_F32 = 0,   /* float32 storage, fp32 arithmetic (no TF32) */
+    CLOVER_BF16 = 1   /* bfloat16 storage, fp32 accumulation, bf16 output (round to nearest even) */
+} clover_dtype;
+
+/* Version of this ABI (incremented on any incompatible change). */
+CLOVER_API int clover_abi_version(void);
+
+/* Short English name of a status code (static storage). */
+CLOVER_API const char *clover_status_string(int status);
+
+/*
+ * Bytes of device workspace clover_verify_attn needs for these sizes
+ * (split-KV partial results and per-head arrival counters).  Returns 0 when
+ * the sizes are outside the limits.
+ */
+CLOVER_API size_t clover_verify_attn_workspace_size(int B, int T, int Hq, int Hkv, int D, int Lcap,
+                                         clover_dtype dtype);
+
+/*
+ * Tree-masked attention of one verification step (Section 2.1 verification
+ * phase; Section 2.2 Tree Attention with the tree topology as the mask).
+ *
+ * For every sequence b, node i and query head h (g = h / (Hq/Hkv)):
+ *   out[b,i,h,:] = softmax_j(scale * q[b,i,h,:] . key_j) . value_j
+ * over the keys j = cache slots 0..cache_len[b]-1 of KV head g, and the tree
+ * nodes m that are i or an ancestor of i (key k_new[b,m,g,:], value v_new[b,m,g,:]).
+ *
+ *   q        [B,T,Hq,D]      dtype   query rows of the tree nodes (positions already applied)
+ *   k_new    [B,T,Hkv,D]     dtype   keys of the tree nodes
+ *   v_new    [B,T,Hkv,D]     dtype   values of the tree nodes
+ *   k_cache  [B,Hkv,Lcap,D]  dtype   in/out: slots [0, cache_len[b]) are read;
+ *   v_cache  [B,Hkv,Lcap,D]  dtype   slots [cache_len[b], cache_len[b]+T) receive
+ *                                    k_new/v_new of nodes 0..T-1 (the append)
+ *   cache_len[B]             int32   committed length of each sequence (read only)
+ *   parent   [B,T]           int32   the token tree (see conventions)
+ *   out      [B,T,Hq,D]      dtype   attention output
+ *   scale                    float   softmax scale; <= 0 selects 1/sqrt(D)
+ *   workspace, ws_bytes              device scratch of at least
+ *                                    clover_verify_attn_workspace_size(...) bytes,
+ *                                    16-byte aligned.  It must be zero-filled before
+ *                                    its first use; every call leaves it ready for the
+ *                                    next one.  Calls sharing a workspace must not
+ *                                    overlap on the device.
+ *   status                           device int32 error bits (may be NULL)
+ * q, k_new, v_new, caches and out must be 16-byte aligned.
+ */
+CLOVER_API clover_status clover_verify_attn(const void *q, const void *k_new, const void *v_new,
+                                 void *k_cache, void *v_cache, const int32_t *cache_len,
+                                 const int32_t *parent, void *out,
+                                 int B, int T, int Hq, int Hkv, int D, int Lcap,
+                                 clover_dtype dtype, float scale,
+                                 void *workspace, size_t ws_bytes,
+                                 int32_t *status, void *stream);
+
+/* Bytes of device workspace clover_verify_accept needs (0 outside the limits). */
+CLOVER_API size_t clover_verify_accept_workspace_size(int B, int T, int V, clover_dtype dtype);
+
+/*
+ * Per-node greedy token and acceptance walk (Section 2.1: the base model
+ * rejects wrong speculations; Section 1: outputs stay those of the base model;
+ * Section 4.1: tokens/step is the accepted length).
+ *
+ *   logits   [B,T,V]  dtype  base-model logits at every tree node (any alignment)
+ *   cand     [B,T]    int32  candidate token of every node; cand[b][0] (the root,
+ *                            already emitted by the base model) is not checked
+ *   parent   [B,T]    int32  the token tree
+ *   argmax_out [B,T]  int32  smallest index v with logits[b,i,v] equal to the row
+ *                            maximum (-0 == +0)
+ *   path_out [B,T]    int32  accepted nodes from the root: path[0] = 0 and
+ *                            path[k+1] = the smallest-index child c of path[k]
+ *                            with cand[c] == argmax[path[k]]; padded with -1
+ *   accept_len [B]    int32  number of accepted nodes (1 .. depth+1)
+ *   bonus_token [B]   int32  argmax at the last accepted node (the next root)
+ *   workspace, ws_bytes      >= clover_verify_accept_workspace_size(...) bytes,
+ *                            8-byte aligned, zero-filled before first use; left
+ *                            ready for the next call.  Calls sharing it must not
+ *                            overlap on the device.
+ */
+CLOVER_API clover_status clover_verify_accept(const void *logits, const int32_t *cand, const int32_t *parent,
+                                   int B, int T, int V, clover_dtype dtype,
+                                   int32_t *argmax_out, int32_t *path_out,
+                                   int32_t *accept_len, int32_t *bonus_token,
+                                   void *workspace, size_t ws_bytes,
+                                   int32_t *status, void *stream);
+
+/*
+ * Commit the accepted path to the cache (no counterpart in the paper, which
+ * leaves the engine's cache handling implicit).  For every sequence b with
+ * L = cache_len[b] and a = accept_len[b]:
+ *   cache[b,g,L+j,:] <- cache[b,g,L+path[b][j],:]  for j < a, every KV head g,
+ * for K and V, with the result of copying in increasing j (all reads happen
+ * before any write); slots < L are not touched.
+ *   k_cache, v_cache [B,Hkv,Lcap,D] dtype  in place, 16-byte aligned
+ *   cache_len [B]        int32   length before the step (read only)
+ *   path, accept_len             as produced by clover_verify_accept
+ *   new_cache_len [B]    int32   out: L + a.  Must not overlap cache_len.
+ *   src_index_out [B,T]  int32   out: L + path[b][j] for j < a, else -1 (may be NULL)
+ */
+CLOVER_API clover_status clover_kv_compact(void *k_cache, void *v_cache, const int32_t *cache_len,
+                                const int32_t *path, const int32_t *accept_len,
+                                int32_t *new_cache_len, int32_t *src_index_out,
+                                int B, int T, int Hkv, int D, int Lcap, clover_dtype dtype,
+                                int32_t *status, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CLOVER_VERIFY_H */

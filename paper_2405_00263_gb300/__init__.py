@@ -1,0 +1,10 @@
+"""GB300 (sm_103a) verification step of Clover-style tree speculative decoding.
+
+The compute lives in libclover_verify.so (CUDA kernels behind a C ABI, see
+include/clover_verify.h); this package builds it in-tree and binds it with the
+same names.  There is no CPU fallback.
+"""
+
+from .api import (  # noqa: F401
+    BF16, F32, OK, CloverError, VerifyStep, clover_abi_version, clover_kv_compact, clover_verify_accept,
+    clover_verify_accept_workspace_size, clover_verify_attn, clover_verify_attn_workspace_size, dtype_code)

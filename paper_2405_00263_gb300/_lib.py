@@ -1,0 +1,65 @@
+"""ctypes loader of libclover_verify.so and the raw C signatures.
+
+The library is built in-tree (``paper_2405_00263_gb300/_build``) by
+``paper_2405_00263_gb300.build.build()``.  There is no fallback: if the shared
+library is missing, loading raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+from . import build as _build
+
+_lock = threading.Lock()
+_lib = None
+
+# Every symbol include/clover_verify.h declares.
+EXPORTS = (
+    "clover_abi_version",
+    "clover_status_string",
+    "clover_verify_attn_workspace_size",
+    "clover_verify_attn",
+    "clover_verify_accept_workspace_size",
+    "clover_verify_accept",
+    "clover_kv_compact",
+)
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = False):
+    """The loaded CDLL with argtypes set.  Raises if the library was not built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = library_path()
+        if not os.path.exists(path):
+            if not build_if_missing:
+                raise RuntimeError(
+                    f"libclover_verify.so is not built ({path}); run "
+                    "`python -c 'import __graft_entry__ as g; g.build()'` first")
+            _build.build()
+        lib = ctypes.CDLL(path)
+        P, I, Z, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
+        lib.clover_abi_version.argtypes = []
+        lib.clover_abi_version.restype = I
+        lib.clover_status_string.argtypes = [I]
+        lib.clover_status_string.restype = ctypes.c_char_p
+        lib.clover_verify_attn_workspace_size.argtypes = [I, I, I, I, I, I, I]
+        lib.clover_verify_attn_workspace_size.restype = Z
+        lib.clover_verify_attn.argtypes = [P, P, P, P, P, P, P, P, I, I, I, I, I, I, I, F, P, Z, P, P]
+        lib.clover_verify_attn.restype = I
+        lib.clover_verify_accept_workspace_size.argtypes = [I, I, I, I]
+        lib.clover_verify_accept_workspace_size.restype = Z
+        lib.clover_verify_accept.argtypes = [P, P, P, I, I, I, I, P, P, P, P, P, Z, P, P]
+        lib.clover_verify_accept.restype = I
+        lib.clover_kv_compact.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P, P]
+        lib.clover_kv_compact.restype = I
+        _lib = lib
+        return lib

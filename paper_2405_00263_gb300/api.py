@@ -1,0 +1,192 @@
+"""Python binding of the C ABI, with the same names.
+
+Each function only checks and marshals its torch arguments (device, dtype,
+shape, contiguity) and calls the library; every step of the computation runs
+in the CUDA kernels.  Tensors must live on the current CUDA device; the stream
+defaults to torch's current stream.
+"""
+
+from __future__ import annotations
+
+import ctypes
+
+import torch
+
+from . import _lib
+
+OK = 0
+ERR_INVALID_ARG = 1
+ERR_UNSUPPORTED = 2
+ERR_BAD_TREE = 4
+ERR_CAPACITY = 8
+ERR_CUDA = 16
+ERR_TIMEOUT = 32
+
+F32 = 0
+BF16 = 1
+
+
+class CloverError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        lib = _lib.load()
+        super().__init__(f"{where}: {lib.clover_status_string(code).decode()} (status {code})")
+        self.code = code
+
+
+def dtype_code(dt: torch.dtype) -> int:
+    if dt == torch.float32:
+        return F32
+    if dt == torch.bfloat16:
+        return BF16
+    raise TypeError(f"unsupported dtype {dt}: float32 or bfloat16")
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(*tensors):
+    dev = None
+    for t in tensors:
+        if t is None:
+            continue
+        if not t.is_cuda:
+            raise ValueError("all tensors must be CUDA tensors")
+        if not t.is_contiguous():
+            raise ValueError("all tensors must be contiguous")
+        if dev is None:
+            dev = t.device
+        elif t.device != dev:
+            raise ValueError("all tensors must be on one device")
+    return dev
+
+
+def _check(t, shape, dtype, name):
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: expected shape {tuple(shape)}, got {tuple(t.shape)}")
+    if t.dtype != dtype:
+        raise ValueError(f"{name}: expected {dtype}, got {t.dtype}")
+
+
+def clover_abi_version() -> int:
+    return _lib.load().clover_abi_version()
+
+
+def clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, Lcap, dtype) -> int:
+    code = dtype if isinstance(dtype, int) else dtype_code(dtype)
+    return int(_lib.load().clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, Lcap, code))
+
+
+def clover_verify_accept_workspace_size(B, T, V, dtype) -> int:
+    code = dtype if isinstance(dtype, int) else dtype_code(dtype)
+    return int(_lib.load().clover_verify_accept_workspace_size(B, T, V, code))
+
+
+def clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, scale=0.0,
+                       workspace=None, status=None, stream=None):
+    """Tree-masked attention; appends k_new/v_new at cache slots [L, L+T)."""
+    B, T, Hq, D = q.shape
+    Hkv, Lcap = k_cache.shape[1], k_cache.shape[2]
+    dt = q.dtype
+    _check(k_new, (B, T, Hkv, D), dt, "k_new")
+    _check(v_new, (B, T, Hkv, D), dt, "v_new")
+    _check(k_cache, (B, Hkv, Lcap, D), dt, "k_cache")
+    _check(v_cache, (B, Hkv, Lcap, D), dt, "v_cache")
+    _check(cache_len, (B,), torch.int32, "cache_len")
+    _check(parent, (B, T), torch.int32, "parent")
+    _check(out, (B, T, Hq, D), dt, "out")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, workspace, status)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    code = _lib.load().clover_verify_attn(
+        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(cache_len), _ptr(parent),
+        _ptr(out), B, T, Hq, Hkv, D, Lcap, dtype_code(dt), float(scale), _ptr(workspace), ws_bytes,
+        _ptr(status), _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_verify_attn")
+
+
+def clover_verify_accept(logits, cand, parent, argmax_out, path_out, accept_len, bonus_token,
+                         workspace, status=None, stream=None):
+    """Per-node argmax and the greedy acceptance walk."""
+    B, T, V = logits.shape
+    _check(cand, (B, T), torch.int32, "cand")
+    _check(parent, (B, T), torch.int32, "parent")
+    _check(argmax_out, (B, T), torch.int32, "argmax_out")
+    _check(path_out, (B, T), torch.int32, "path_out")
+    _check(accept_len, (B,), torch.int32, "accept_len")
+    _check(bonus_token, (B,), torch.int32, "bonus_token")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(logits, cand, parent, argmax_out, path_out, accept_len, bonus_token, workspace, status)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    code = _lib.load().clover_verify_accept(
+        _ptr(logits), _ptr(cand), _ptr(parent), B, T, V, dtype_code(logits.dtype), _ptr(argmax_out),
+        _ptr(path_out), _ptr(accept_len), _ptr(bonus_token), _ptr(workspace), ws_bytes, _ptr(status),
+        _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_verify_accept")
+
+
+def clover_kv_compact(k_cache, v_cache, cache_len, path, accept_len, new_cache_len, src_index_out=None,
+                      status=None, stream=None):
+    """Moves the accepted nodes' K/V to slots [L, L+a); new_cache_len = L + a."""
+    B, Hkv, Lcap, D = k_cache.shape
+    T = path.shape[1]
+    _check(v_cache, (B, Hkv, Lcap, D), k_cache.dtype, "v_cache")
+    _check(cache_len, (B,), torch.int32, "cache_len")
+    _check(path, (B, T), torch.int32, "path")
+    _check(accept_len, (B,), torch.int32, "accept_len")
+    _check(new_cache_len, (B,), torch.int32, "new_cache_len")
+    if src_index_out is not None:
+        _check(src_index_out, (B, T), torch.int32, "src_index_out")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(k_cache, v_cache, cache_len, path, accept_len, new_cache_len, src_index_out, status)
+    code = _lib.load().clover_kv_compact(
+        _ptr(k_cache), _ptr(v_cache), _ptr(cache_len), _ptr(path), _ptr(accept_len), _ptr(new_cache_len),
+        _ptr(src_index_out), B, T, Hkv, D, Lcap, dtype_code(k_cache.dtype), _ptr(status), _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_kv_compact")
+
+
+class VerifyStep:
+    """Device buffers for repeated verification steps of one shape.
+
+    Owns the two zero-initialised workspaces and the output tensors; ``run``
+    issues the three library calls in order on one stream.
+    """
+
+    def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda"):
+        self.shape = dict(B=B, T=T, Hq=Hq, Hkv=Hkv, D=D, Lcap=Lcap, V=V)
+        self.dtype = dtype
+        dev = torch.device(device)
+        ws_a = clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, Lcap, dtype)
+        ws_b = clover_verify_accept_workspace_size(B, T, V, dtype)
+        self.ws_attn = torch.zeros(max(ws_a, 16), dtype=torch.uint8, device=dev) if ws_a else None
+        self.ws_accept = torch.zeros(max(ws_b, 16), dtype=torch.uint8, device=dev)
+        self.out = torch.empty((B, T, Hq, D), dtype=dtype, device=dev)
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.argmax = torch.empty((B, T), **i32)
+        self.path = torch.empty((B, T), **i32)
+        self.accept_len = torch.empty((B,), **i32)
+        self.bonus = torch.empty((B,), **i32)
+        self.new_cache_len = torch.empty((B,), **i32)
+        self.src_index = torch.empty((B, T), **i32)
+        self.status = torch.zeros((1,), **i32)
+
+    def run(self, q, k_new, v_new, k_cache, v_cache, cache_len, parent, cand, logits, scale=0.0,
+            stream=None):
+        clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
+                           workspace=self.ws_attn, status=self.status, stream=stream)
+        clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
+                             self.ws_accept, status=self.status, stream=stream)
+        clover_kv_compact(k_cache, v_cache, cache_len, self.path, self.accept_len, self.new_cache_len,
+                          self.src_index, status=self.status, stream=stream)

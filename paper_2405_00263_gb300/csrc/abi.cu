@@ -1,0 +1,189 @@
+// extern "C" entry points of libclover_verify.so: host-side validation, launch
+// planning and dispatch to the kernels.  Declarations and the full contract of
+// each call are in include/clover_verify.h.
+#include <math.h>
+
+#include "common.cuh"
+
+namespace clover {
+int fma_row_tile();
+cudaError_t launch_tree_attn_fma(const AttnArgs &a, cudaStream_t stream);
+void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk);
+size_t accept_workspace_bytes(int B, int T, int V, int dtype);
+cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T, int V,
+                          int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len, int32_t *bonus,
+                          void *workspace, int32_t *status, cudaStream_t stream);
+cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const int32_t *cache_len, const int32_t *path,
+                              const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index, int B, int T,
+                              int Hkv, int D, int Lcap, int dtype, int32_t *status, cudaStream_t stream);
+
+namespace {
+
+constexpr int kAbiVersion = 1;
+constexpr int kTargetAttnCtas = 2 * 152;   // two resident attention CTAs per SM on a 152-SM GPU
+constexpr int kMinKeysPerSplit = 256;
+constexpr int kMaxSplits = 64;
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct AttnPlan {
+    int row_tile, row_tiles, n_split;
+    size_t o_bytes, ml_bytes, counter_bytes, total;
+};
+
+clover_status check_attn_sizes(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
+    if (B < 0 || T < 1 || Hq < 1 || Hkv < 1 || Lcap < 1) return CLOVER_ERR_INVALID_ARG;
+    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
+    if (T > kMaxTreeNodes || (D != 64 && D != 128) || Hq % Hkv != 0) return CLOVER_ERR_UNSUPPORTED;
+    if (Lcap < T) return CLOVER_ERR_INVALID_ARG;
+    if (B > 65535 || Hkv > 65535) return CLOVER_ERR_UNSUPPORTED;
+    return CLOVER_OK;
+}
+
+AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap) {
+    AttnPlan p;
+    const int G = Hq / Hkv;
+    p.row_tile = fma_row_tile();
+    p.row_tiles = (T * G + p.row_tile - 1) / p.row_tile;
+    const long base = (long)(B > 0 ? B : 1) * Hkv * p.row_tiles;
+    int n = (int)((kTargetAttnCtas + base - 1) / base);
+    const int by_len = (Lcap + kMinKeysPerSplit - 1) / kMinKeysPerSplit;
+    if (n > by_len) n = by_len;
+    if (n > kMaxSplits) n = kMaxSplits;
+    if (n < 1) n = 1;
+    p.n_split = n;
+    const size_t heads = (size_t)(B > 0 ? B : 1) * Hkv * p.row_tiles;
+    if (n == 1) {
+        p.o_bytes = p.ml_bytes = p.counter_bytes = p.total = 0;
+    } else {
+        p.o_bytes = round_up(sizeof(float) * heads * n * p.row_tile * D, 256);
+        p.ml_bytes = round_up(sizeof(float) * heads * n * p.row_tile * 2, 256);
+        p.counter_bytes = round_up(sizeof(unsigned) * heads, 256);
+        p.total = p.o_bytes + p.ml_bytes + p.counter_bytes;
+    }
+    return p;
+}
+
+clover_status from_cuda(cudaError_t e) { return e == cudaSuccess ? CLOVER_OK : CLOVER_ERR_CUDA; }
+
+}  // namespace
+}  // namespace clover
+
+using namespace clover;
+
+extern "C" {
+
+int clover_abi_version(void) { return kAbiVersion; }
+
+const char *clover_status_string(int status) {
+    switch (status) {
+        case CLOVER_OK: return "ok";
+        case CLOVER_ERR_INVALID_ARG: return "invalid argument";
+        case CLOVER_ERR_UNSUPPORTED: return "unsupported size or type";
+        case CLOVER_ERR_BAD_TREE: return "parent array is not a topologically numbered tree";
+        case CLOVER_ERR_CAPACITY: return "cache length out of range or cache too small";
+        case CLOVER_ERR_CUDA: return "CUDA error";
+        case CLOVER_ERR_TIMEOUT: return "device wait timed out";
+        default: return "several errors (bitwise OR of codes)";
+    }
+}
+
+size_t clover_verify_attn_workspace_size(int B, int T, int Hq, int Hkv, int D, int Lcap, clover_dtype dtype) {
+    if (check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype) != CLOVER_OK) return 0;
+    return plan_attn(B, T, Hq, Hkv, D, Lcap).total;
+}
+
+clover_status clover_verify_attn(const void *q, const void *k_new, const void *v_new, void *k_cache,
+                                 void *v_cache, const int32_t *cache_len, const int32_t *parent, void *out,
+                                 int B, int T, int Hq, int Hkv, int D, int Lcap, clover_dtype dtype,
+                                 float scale, void *workspace, size_t ws_bytes, int32_t *status,
+                                 void *stream) {
+    const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype);
+    if (s != CLOVER_OK) return s;
+    if (B == 0) return CLOVER_OK;
+    if (!q || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !parent || !out)
+        return CLOVER_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache) ||
+        !aligned16(out))
+        return CLOVER_ERR_INVALID_ARG;
+    if (!(scale == scale) || isinf(scale)) return CLOVER_ERR_INVALID_ARG;
+    const AttnPlan p = plan_attn(B, T, Hq, Hkv, D, Lcap);
+    if (ws_bytes < p.total || (p.total > 0 && (!workspace || !aligned16(workspace)))) return CLOVER_ERR_INVALID_ARG;
+
+    AttnArgs a;
+    a.q = q;
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_len = cache_len;
+    a.parent = parent;
+    a.out = out;
+    a.B = B;
+    a.T = T;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.D = D;
+    a.Lcap = Lcap;
+    a.G = Hq / Hkv;
+    a.dtype = dtype;
+    const float sc = scale > 0.f ? scale : 1.f / sqrtf((float)D);
+    a.scale_log2 = sc * 1.4426950408889634f;
+    a.rows = T * a.G;
+    a.row_tile = p.row_tile;
+    a.row_tiles = p.row_tiles;
+    a.n_split = p.n_split;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    a.part_o = p.total ? reinterpret_cast<float *>(ws) : nullptr;
+    a.part_ml = p.total ? reinterpret_cast<float *>(ws + p.o_bytes) : nullptr;
+    a.counters = p.total ? reinterpret_cast<unsigned *>(ws + p.o_bytes + p.ml_bytes) : nullptr;
+    a.status = status;
+    return from_cuda(launch_tree_attn_fma(a, static_cast<cudaStream_t>(stream)));
+}
+
+size_t clover_verify_accept_workspace_size(int B, int T, int V, clover_dtype dtype) {
+    if (B < 0 || T < 1 || T > kMaxTreeNodes || V < 1) return 0;
+    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return 0;
+    return accept_workspace_bytes(B > 0 ? B : 1, T, V, dtype);
+}
+
+clover_status clover_verify_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
+                                   int V, clover_dtype dtype, int32_t *argmax_out, int32_t *path_out,
+                                   int32_t *accept_len, int32_t *bonus_token, void *workspace, size_t ws_bytes,
+                                   int32_t *status, void *stream) {
+    if (B < 0 || T < 1 || V < 1) return CLOVER_ERR_INVALID_ARG;
+    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
+    if (T > kMaxTreeNodes) return CLOVER_ERR_UNSUPPORTED;
+    if (B == 0) return CLOVER_OK;
+    if ((long)B * T > 0x7FFFFFFFL) return CLOVER_ERR_UNSUPPORTED;
+    if (!logits || !cand || !parent || !argmax_out || !path_out || !accept_len || !bonus_token)
+        return CLOVER_ERR_INVALID_ARG;
+    const size_t need = accept_workspace_bytes(B, T, V, dtype);
+    if (ws_bytes < need || !workspace || (reinterpret_cast<uintptr_t>(workspace) & 7u)) return CLOVER_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(logits) % (dtype == CLOVER_F32 ? 4 : 2)) return CLOVER_ERR_INVALID_ARG;
+    return from_cuda(launch_accept(logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
+                                   bonus_token, workspace, status, static_cast<cudaStream_t>(stream)));
+}
+
+clover_status clover_kv_compact(void *k_cache, void *v_cache, const int32_t *cache_len, const int32_t *path,
+                                const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index_out, int B,
+                                int T, int Hkv, int D, int Lcap, clover_dtype dtype, int32_t *status,
+                                void *stream) {
+    if (B < 0 || T < 1 || Hkv < 1 || Lcap < 1) return CLOVER_ERR_INVALID_ARG;
+    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
+    if (T > kMaxTreeNodes || (D != 64 && D != 128)) return CLOVER_ERR_UNSUPPORTED;
+    if (Lcap < T) return CLOVER_ERR_INVALID_ARG;
+    if (B > 65535 || Hkv > 65535) return CLOVER_ERR_UNSUPPORTED;
+    if (B == 0) return CLOVER_OK;
+    if (!k_cache || !v_cache || !cache_len || !path || !accept_len || !new_cache_len) return CLOVER_ERR_INVALID_ARG;
+    if (!aligned16(k_cache) || !aligned16(v_cache)) return CLOVER_ERR_INVALID_ARG;
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(cache_len), a1 = a0 + sizeof(int32_t) * (size_t)B;
+    const uintptr_t b0 = reinterpret_cast<uintptr_t>(new_cache_len), b1 = b0 + sizeof(int32_t) * (size_t)B;
+    if (a0 < b1 && b0 < a1) return CLOVER_ERR_INVALID_ARG;      // lengths are read by every CTA: no aliasing
+    return from_cuda(launch_kv_compact(k_cache, v_cache, cache_len, path, accept_len, new_cache_len, src_index_out,
+                                       B, T, Hkv, D, Lcap, dtype, status, static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

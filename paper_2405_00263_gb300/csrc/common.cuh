@@ -1,0 +1,146 @@
+// Shared device helpers and launch-argument structs of the verification kernels.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "clover_verify.h"
+
+namespace clover {
+
+constexpr int kMaxTreeNodes = 64;   // one 64-bit ancestor mask per node
+
+// Everything clover_verify_attn's kernels need, already validated on the host.
+struct AttnArgs {
+    const void *q, *k_new, *v_new;
+    void *k_cache, *v_cache;
+    const int32_t *cache_len, *parent;
+    void *out;
+    int B, T, Hq, Hkv, D, Lcap, G;
+    int dtype;             // clover_dtype
+    float scale_log2;      // softmax scale * log2(e): scores are kept in base 2
+    int rows;              // T * G query rows per KV head
+    int row_tile;          // rows per CTA
+    int row_tiles;         // ceil(rows / row_tile)
+    int n_split;           // cache key ranges per (sequence, KV head, row tile)
+    float *part_o;         // [B, Hkv, row_tiles, n_split, row_tile, D]
+    float *part_ml;        // [B, Hkv, row_tiles, n_split, row_tile, 2]  (max, sum)
+    unsigned *counters;    // [B, Hkv, row_tiles]
+    int32_t *status;
+};
+
+__device__ __forceinline__ void report(int32_t *status, int bits) {
+    if (status) atomicOr(status, bits);
+}
+
+__device__ __forceinline__ float bf16_bits_to_float(uint16_t h) {
+    return __uint_as_float(static_cast<uint32_t>(h) << 16);
+}
+
+// Eight consecutive elements (16 bytes of bf16 or two 16-byte loads of fp32) -> fp32.
+template <typename T>
+struct Vec8;
+
+template <>
+struct Vec8<float> {
+    static __device__ __forceinline__ void load(const float *p, float (&v)[8]) {
+        const float4 a = *reinterpret_cast<const float4 *>(p);
+        const float4 b = *reinterpret_cast<const float4 *>(p + 4);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+};
+
+template <>
+struct Vec8<__nv_bfloat16> {
+    static __device__ __forceinline__ void load(const __nv_bfloat16 *p, float (&v)[8]) {
+        const uint4 a = *reinterpret_cast<const uint4 *>(p);
+        const uint32_t w[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            v[2 * k] = __uint_as_float(w[k] << 16);
+            v[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+        }
+    }
+};
+
+__device__ __forceinline__ float to_float(float x) { return x; }
+__device__ __forceinline__ float to_float(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <typename T>
+__device__ __forceinline__ T from_float(float x);
+template <>
+__device__ __forceinline__ float from_float<float>(float x) { return x; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(float x) { return __float2bfloat16_rn(x); }
+
+// Ancestor-or-self bitmask of every tree node, by pointer jumping, computed by
+// one warp: lane l owns nodes l and l + 32.  After round k each node's mask
+// covers its 2^k nearest ancestors; six rounds cover depth 63.  Invalid parent
+// arrays set *bad (masks are then only self bits and must not be trusted).
+__device__ __forceinline__ void tree_masks_warp(const int32_t *parent, int T, uint64_t *anc,
+                                                bool *bad) {
+    const int lane = threadIdx.x & 31;
+    uint64_t m[2];
+    int up[2];
+    bool invalid = false;
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int i = lane + 32 * k;
+        int p = -1;
+        if (i < T) {
+            p = __ldg(parent + i);
+            if (i == 0 ? (p != -1) : (p < 0 || p >= i)) invalid = true;
+        }
+        if (i >= T || invalid) p = -1;
+        m[k] = (i < T) ? (1ull << i) : 0ull;
+        up[k] = p;
+    }
+    const bool any_bad = __any_sync(0xffffffffu, invalid);
+    if (!any_bad) {
+#pragma unroll
+        for (int round = 0; round < 6; ++round) {
+            uint64_t nm[2];
+            int nu[2];
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const int u = up[k] < 0 ? 0 : up[k];
+                // fetch mask and pointer of node u (held by lane u & 31, slot u >> 5)
+                const uint64_t m0 = __shfl_sync(0xffffffffu, m[0], u & 31);
+                const uint64_t m1 = __shfl_sync(0xffffffffu, m[1], u & 31);
+                const int u0 = __shfl_sync(0xffffffffu, up[0], u & 31);
+                const int u1 = __shfl_sync(0xffffffffu, up[1], u & 31);
+                const uint64_t mu = (u >> 5) ? m1 : m0;
+                const int uu = (u >> 5) ? u1 : u0;
+                nm[k] = up[k] < 0 ? m[k] : (m[k] | mu);
+                nu[k] = up[k] < 0 ? -1 : uu;
+            }
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                m[k] = nm[k];
+                up[k] = nu[k];
+            }
+        }
+    }
+    if (lane < T) anc[lane] = m[0];
+    if (lane + 32 < T) anc[lane + 32] = m[1];
+    if (lane == 0) *bad = any_bad;
+}
+
+// Raises a kernel's dynamic shared memory limit once per device.  Launchers
+// call it before every launch; only the first call on a device reaches the
+// driver, so launches captured into a CUDA graph after a first eager launch
+// issue no attribute call.
+template <typename Kernel>
+cudaError_t ensure_smem_attr(Kernel kernel, size_t bytes, unsigned char (&done)[64]) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 64 && done[dev]) return cudaSuccess;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess && dev < 64) done[dev] = 1;
+    return e;
+}
+
+}  // namespace clover

@@ -1,0 +1,102 @@
+// Commit of the accepted path to the KV cache: for sequence b with committed
+// length L and accepted nodes path[0..a-1], the K/V rows at slots L + path[j]
+// (where the attention kernel appended the tree's K/V) move to slots L + j.
+// The paper leaves this engine step implicit; the result is that of copying in
+// increasing j, which equals a gather because path[j] >= j.
+//
+// One CTA per (KV head, sequence) stages the a accepted rows of K and V in
+// shared memory and only then writes them, so a row that is both a source and
+// a destination is read before it is overwritten.  The CTA of head 0 also
+// writes the source slot indices and the new length.
+#include "common.cuh"
+
+namespace clover {
+namespace {
+
+constexpr int kThreads = 128;
+
+__global__ void __launch_bounds__(kThreads) kv_compact_kernel(
+    uint8_t *k_cache, uint8_t *v_cache, const int32_t *cache_len, const int32_t *path,
+    const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index, int T, int Hkv,
+    int row_bytes, int Lcap, int32_t *status) {
+    extern __shared__ uint4 stage[];          // [2][T][row_bytes / 16]
+    __shared__ int s_src[kMaxTreeNodes];
+    __shared__ int s_ok;
+    const int g = blockIdx.x;
+    const int b = blockIdx.y;
+    const int L = __ldg(cache_len + b);
+    const int a = __ldg(accept_len + b);
+    if (threadIdx.x == 0) {
+        int ok = (a >= 1 && a <= T) ? 1 : 0;
+        if (L < 0 || L + T > Lcap) {
+            ok = 0;
+            if (g == 0) report(status, CLOVER_ERR_CAPACITY);
+        }
+        s_ok = ok;
+    }
+    __syncthreads();
+    if (!s_ok) {
+        if (g == 0 && threadIdx.x == 0 && (a < 1 || a > T)) report(status, CLOVER_ERR_INVALID_ARG);
+        return;
+    }
+    if (threadIdx.x < 32) {
+        bool bad = false;
+        for (int j = threadIdx.x; j < a; j += 32) {
+            const int p = __ldg(path + (size_t)b * T + j);
+            if (p < 0 || p >= T) bad = true;
+            s_src[j] = (p < 0 || p >= T) ? j : p;
+        }
+        bad = __any_sync(0xffffffffu, bad);
+        if (threadIdx.x == 0 && bad) report(status, CLOVER_ERR_INVALID_ARG);
+        __syncwarp();
+        if (g == 0) {
+            if (src_index)
+                for (int j = threadIdx.x; j < T; j += 32) src_index[(size_t)b * T + j] = (j < a) ? L + s_src[j] : -1;
+            if (threadIdx.x == 0) new_cache_len[b] = L + a;
+        }
+    }
+    __syncthreads();
+
+    const int units = row_bytes / 16;
+    const size_t head_base = ((size_t)b * Hkv + g) * Lcap;
+    const uint4 *ks = reinterpret_cast<const uint4 *>(k_cache);
+    const uint4 *vs = reinterpret_cast<const uint4 *>(v_cache);
+    for (int e = threadIdx.x; e < a * units; e += kThreads) {
+        const int j = e / units;
+        const int u = e % units;
+        const size_t src = (head_base + L + s_src[j]) * units + u;
+        stage[e] = ks[src];
+        stage[T * units + e] = vs[src];
+    }
+    __syncthreads();
+    uint4 *kd = reinterpret_cast<uint4 *>(k_cache);
+    uint4 *vd = reinterpret_cast<uint4 *>(v_cache);
+    for (int e = threadIdx.x; e < a * units; e += kThreads) {
+        const int j = e / units;
+        const int u = e % units;
+        const size_t dst = (head_base + L + j) * units + u;
+        kd[dst] = stage[e];
+        vd[dst] = stage[T * units + e];
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const int32_t *cache_len, const int32_t *path,
+                              const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index, int B,
+                              int T, int Hkv, int D, int Lcap, int dtype, int32_t *status,
+                              cudaStream_t stream) {
+    const int row_bytes = D * (dtype == CLOVER_F32 ? 4 : 2);
+    const size_t smem = (size_t)2 * T * row_bytes;
+    static unsigned char done[64];
+    cudaError_t e = ensure_smem_attr(kv_compact_kernel, (size_t)2 * kMaxTreeNodes * 128 * 4, done);
+    if (e != cudaSuccess) return e;
+    dim3 grid(Hkv, B);
+    kv_compact_kernel<<<grid, kThreads, smem, stream>>>(static_cast<uint8_t *>(k_cache),
+                                                        static_cast<uint8_t *>(v_cache), cache_len, path,
+                                                        accept_len, new_cache_len, src_index, T, Hkv,
+                                                        row_bytes, Lcap, status);
+    return cudaGetLastError();
+}
+
+}  // namespace clover

@@ -1,0 +1,120 @@
+"""The C ABI library without a GPU: it builds, loads, exports every symbol the
+header declares, and its host-side validation rejects bad arguments before
+anything is launched."""
+
+import ctypes
+import os
+import re
+
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2405_00263_gb300 import _lib, build
+    build.build()
+    return _lib.load()
+
+
+def declared_symbols():
+    names = []
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            names += re.findall(r"CLOVER_API\s+[\w\s\*]*?\b(clover_\w+)\s*\(", text)
+    return names
+
+
+def test_exports_every_declared_symbol(lib):
+    from paper_2405_00263_gb300 import _lib
+    names = declared_symbols()
+    assert len(names) >= 7
+    assert set(names) == set(_lib.EXPORTS)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_version_and_status_strings(lib):
+    assert lib.clover_abi_version() == 1
+    assert lib.clover_status_string(0) == b"ok"
+    assert b"tree" in lib.clover_status_string(4)
+
+
+def test_workspace_sizes(lib):
+    ws = lib.clover_verify_attn_workspace_size
+    assert ws(1, 16, 8, 8, 64, 192, 0) == 0              # short cache: one split, no workspace
+    big = ws(1, 64, 32, 32, 128, 4160, 1)
+    assert big > 0 and big % 256 == 0
+    assert ws(1, 65, 8, 8, 64, 192, 0) == 0              # T > 64 unsupported
+    assert ws(1, 16, 8, 8, 96, 192, 0) == 0              # D = 96 unsupported
+    assert ws(1, 16, 6, 4, 64, 192, 0) == 0              # Hq not a multiple of Hkv
+    acc = lib.clover_verify_accept_workspace_size
+    assert acc(1, 64, 125696, 1) >= 8 * 64 + 4 * 65
+    assert acc(1, 0, 10, 1) == 0 and acc(1, 4, 0, 1) == 0
+
+
+def _attn(lib, **kw):
+    p = dict(q=16, k_new=16, v_new=16, kc=16, vc=16, cl=16, par=16, out=16, B=1, T=4, Hq=2, Hkv=2, D=64,
+             Lcap=64, dt=1, scale=0.0, ws=None, wsb=0, st=None)
+    p.update(kw)
+    P = ctypes.c_void_p
+    return lib.clover_verify_attn(P(p["q"]), P(p["k_new"]), P(p["v_new"]), P(p["kc"]), P(p["vc"]), P(p["cl"]),
+                                  P(p["par"]), P(p["out"]), p["B"], p["T"], p["Hq"], p["Hkv"], p["D"], p["Lcap"],
+                                  p["dt"], p["scale"], P(p["ws"]), p["wsb"], P(p["st"]), None)
+
+
+def test_attn_host_validation(lib):
+    # every case below returns before any CUDA call
+    assert _attn(lib, T=65) == 2
+    assert _attn(lib, D=80) == 2
+    assert _attn(lib, Hq=3, Hkv=2) == 2
+    assert _attn(lib, T=0) == 1
+    assert _attn(lib, dt=7) == 1
+    assert _attn(lib, Lcap=3) == 1
+    assert _attn(lib, q=None) == 1
+    assert _attn(lib, out=8) == 1                          # misaligned
+    assert _attn(lib, scale=float("nan")) == 1
+    assert _attn(lib, B=0) == 0                            # empty batch: nothing to do
+    assert _attn(lib, B=1, T=64, Hq=32, Hkv=32, D=128, Lcap=8192, ws=None, wsb=0) == 1   # workspace missing
+
+
+def test_accept_and_compact_host_validation(lib):
+    P = ctypes.c_void_p
+    acc = lambda B, T, V, ws, wsb, lg=16: lib.clover_verify_accept(
+        P(lg), P(16), P(16), B, T, V, 1, P(16), P(16), P(16), P(16), P(ws), wsb, None, None)
+    assert acc(1, 65, 10, 16, 1 << 20) == 2
+    assert acc(1, 4, 0, 16, 1 << 20) == 1
+    assert acc(1, 4, 10, 16, 0) == 1                       # workspace too small
+    assert acc(1, 4, 10, 16, 1 << 20, lg=17) == 1          # logits misaligned for bf16
+    assert acc(0, 4, 10, None, 0) == 0
+    cmp = lambda cl, ncl, B=2, T=4, D=64: lib.clover_kv_compact(
+        P(16), P(16), P(cl), P(16), P(16), P(ncl), None, B, T, 2, D, 64, 1, None, None)
+    assert cmp(1024, 1024) == 1                            # new length aliases the old one
+    assert cmp(1024, 1028) == 1                            # partial overlap
+    assert cmp(1024, 2048, D=32) == 2
+    assert cmp(1024, 2048, T=65) == 2
+    assert cmp(1024, 2048, B=0) == 0
+
+
+def test_python_binding_rejects_cpu_tensors(lib):
+    import paper_2405_00263_gb300 as pkg
+    x = torch.zeros(1, 4, 2, 64, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        pkg.clover_verify_attn(x, x, x, torch.zeros(1, 2, 64, 64, dtype=torch.bfloat16),
+                               torch.zeros(1, 2, 64, 64, dtype=torch.bfloat16), torch.zeros(1, dtype=torch.int32),
+                               torch.zeros(1, 4, dtype=torch.int32), x.clone())
+
+
+def test_oracle_and_library_share_no_code():
+    """The oracle is plain C with its own definitions; the library sources never
+    include or import anything under oracle/, and the oracle never reads csrc/."""
+    csrc = os.path.join(ROOT, "paper_2405_00263_gb300", "csrc")
+    for fn in os.listdir(csrc):
+        assert "oracle" not in open(os.path.join(csrc, fn)).read().lower(), fn
+    for fn in ("api.py", "_lib.py", "build.py", "__init__.py"):
+        assert "import oracle" not in open(os.path.join(ROOT, "paper_2405_00263_gb300", fn)).read()
+    src = open(os.path.join(ROOT, "oracle", "clover_oracle.c")).read()
+    assert "#include \"" not in src and "clover_verify.h" not in src

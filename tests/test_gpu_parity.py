@@ -1,0 +1,219 @@
+"""GPU parity: the CUDA path through the C ABI against the oracle on the same
+seeded inputs.  Attention within max-abs 1e-4 (fp32) / 2e-2 (bf16) of the fp64
+oracle; argmax, path, accepted length, bonus token, source indices, new cache
+lengths and committed cache bytes bit-exact."""
+
+import pytest
+import torch
+
+import oracle
+import paper_2405_00263_gb300 as pkg
+from synth import workloads
+from tests.gpu_util import ATOL, compare_full, run_gpu, to_dev
+
+pytestmark = pytest.mark.gpu
+
+SMALL = {
+    "tiny": ("tiny_f32", {}),
+    "f32_d128_splits_raggedV": ("tiny_f32", dict(D=128, L=1000, Hq=4, Hkv=4, V=5003)),
+    "f32_gqa_T64": ("tiny_f32", dict(T=64, Hq=16, Hkv=2, branching=(8, 4, 2, 2, 1), L=200)),
+    "bf16_d64_gqa_raggedV": ("7b_l2048", dict(B=2, T=16, Hq=8, Hkv=2, D=64, L=777, V=4099,
+                                               branching=(4, 2, 1, 1))),
+    "bf16_chain": ("7b_l2048", dict(T=64, Hq=4, Hkv=4, L=300, V=2048, tree="chain")),
+    "bf16_star": ("7b_l2048", dict(T=40, Hq=4, Hkv=4, L=129, V=2048, tree="star")),
+    "bf16_random_trees": ("7b_l2048", dict(B=3, T=37, Hq=4, Hkv=4, L=513, V=2048, tree="random")),
+    "bf16_single_node": ("7b_l2048", dict(B=2, T=1, Hq=4, Hkv=4, L=1500, V=3000, branching=())),
+    "bf16_empty_cache": ("7b_l2048", dict(T=16, Hq=4, Hkv=4, L=0, V=2048, branching=(4, 2, 1, 1))),
+    "bf16_ragged_batch": ("7b_batched", dict(B=5, Hq=8, Hkv=8, L_range=(0, 700), V=3001)),
+    "bf16_sharp_scores": ("7b_l2048", dict(T=64, Hq=4, Hkv=2, L=900, V=2048, qkv_std=1.5)),
+    "bf16_gqa8_T64": ("100b_gqa", dict(B=1, Hq=16, Hkv=2, L=640, V=2048)),
+}
+
+
+@pytest.mark.parametrize("case", sorted(SMALL))
+def test_small_step_matches_oracle(case, cuda):
+    name, over = SMALL[case]
+    w = workloads.get(name, **over)
+    host = workloads.make(w)
+    t = to_dev(host, cuda)
+    step = run_gpu(t)
+    compare_full(host, step, t)
+
+
+def test_scale_argument(cuda):
+    w = workloads.get("tiny_f32", L=300)
+    host = workloads.make(w)
+    t = to_dev(host, cuda)
+    step = run_gpu(t, scale=0.37)
+    compare_full(host, step, t, scale=0.37)
+
+
+def test_repeated_calls_reuse_workspace(cuda):
+    """Counters in the workspaces are reset by every call: a second step on
+    fresh copies of the inputs gives the same bytes."""
+    w = workloads.get("7b_l2048", T=64, Hq=8, Hkv=8, L=1800, V=5000)
+    host = workloads.make(w)
+    t1 = to_dev(host, cuda)
+    step = run_gpu(t1)
+    first = [x.clone() for x in (step.out, step.argmax, step.path, step.accept_len, step.bonus)]
+    for _ in range(3):
+        t2 = to_dev(host, cuda)
+        run_gpu(t2, step=step)
+        again = (step.out, step.argmax, step.path, step.accept_len, step.bonus)
+        for a, b in zip(first, again):
+            assert torch.equal(a, b)
+    compare_full(host, step, t2)
+
+
+FULL = ["7b_l2048", "7b_l4096", "7b_l16384", "7b_batched", "100b_gqa"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_workloads(name, cuda):
+    """The workloads at their full sizes: attention on sampled rows (the
+    oracle computes them one by one), argmax / walk / indices everywhere, the
+    tree slots of the cache everywhere, and the committed prefix untouched."""
+    w = workloads.get(name)
+    t = workloads.make(w, device=cuda)
+    host = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in t.items()}
+    kc0, vc0 = t["k_cache"].clone(), t["v_cache"].clone()
+    step = run_gpu(t)
+    assert int(step.status.item()) == 0
+
+    B, T, Hq, D = w.B, w.T, w.Hq, w.D
+    n_rows = B * T * Hq
+    g = torch.Generator().manual_seed(0)
+    rows = sorted(set([0, n_rows - 1] + torch.randint(0, n_rows, (46,), generator=g).tolist()))
+    ref = oracle.tree_attention(host["q"], host["k_new"], host["v_new"], host["k_cache"], host["v_cache"],
+                                host["cache_len"], host["parent"], rows=rows)
+    got = step.out.view(-1, D)[rows].double().cpu()
+    err = (got - ref).abs().max().item()
+    assert err <= ATOL[torch.bfloat16], err
+
+    amax = oracle.argmax(host["logits"])
+    assert torch.equal(step.argmax.cpu(), amax)
+    path, alen, bonus = oracle.accept_walk(host["parent"], host["cand"], amax)
+    assert torch.equal(step.path.cpu(), path)
+    assert torch.equal(step.accept_len.cpu(), alen)
+    assert torch.equal(step.bonus.cpu(), bonus)
+    L = host["cache_len"]
+    assert torch.equal(step.new_cache_len.cpu(), L + alen)
+
+    # expected tree slots: the oracle's append + compaction on an empty cache of T slots
+    zk = torch.zeros((B, w.Hkv, T, D), dtype=host["k_new"].dtype)
+    zv = torch.zeros_like(zk)
+    zl = torch.zeros(B, dtype=torch.int32)
+    oracle.append_tree_kv(host["k_new"], host["v_new"], zk, zv, zl)
+    src = oracle.kv_compact(zk, zv, zl, path, alen)
+    assert torch.equal(step.src_index.cpu(), torch.where(src >= 0, src + L.unsqueeze(1), src))
+    for b in range(B):
+        l0, a = int(L[b]), int(alen[b])
+        assert torch.equal(t["k_cache"][b, :, l0:l0 + a].cpu().view(torch.int16), zk[b, :, :a].view(torch.int16))
+        assert torch.equal(t["v_cache"][b, :, l0:l0 + a].cpu().view(torch.int16), zv[b, :, :a].view(torch.int16))
+        assert torch.equal(t["k_cache"][b, :, :l0].view(torch.int16), kc0[b, :, :l0].view(torch.int16))
+        assert torch.equal(t["v_cache"][b, :, :l0].view(torch.int16), vc0[b, :, :l0].view(torch.int16))
+
+
+# ---------------------------------------------------------------------------
+# edge cases
+# ---------------------------------------------------------------------------
+
+def _accept_only(logits, cand, parent, cuda):
+    B, T, V = logits.shape
+    ws = torch.zeros(pkg.clover_verify_accept_workspace_size(B, T, V, logits.dtype), dtype=torch.uint8, device=cuda)
+    i32 = dict(dtype=torch.int32, device=cuda)
+    out = dict(argmax=torch.empty((B, T), **i32), path=torch.empty((B, T), **i32),
+               alen=torch.empty(B, **i32), bonus=torch.empty(B, **i32), status=torch.zeros(1, **i32))
+    pkg.clover_verify_accept(logits.to(cuda), cand.to(cuda), parent.to(cuda), out["argmax"], out["path"],
+                             out["alen"], out["bonus"], ws, status=out["status"])
+    torch.cuda.synchronize()
+    return {k: v.cpu() for k, v in out.items()}
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_argmax_ties_signed_zero_infinities(dtype, cuda):
+    B, T, V = 2, 8, 125696
+    g = torch.Generator().manual_seed(5)
+    x = (torch.randn(B, T, V, generator=g) * 4).to(dtype)
+    x[0, 0, [70000, 3, 125695]] = 40.0                   # three-way tie
+    x[0, 1] = -1.0
+    x[0, 1, 9000] = -0.0
+    x[0, 1, 8999] = 0.0                                  # -0 == +0
+    x[0, 2] = float("-inf")                              # all -inf -> 0
+    x[0, 3, V - 1] = 100.0                               # last index
+    x[0, 4, 0] = 100.0                                   # first index
+    x[0, 5, 77] = float("inf")
+    x[0, 6] = 0.0                                        # all equal -> 0
+    x[1, :, 1000:2000] = 50.0                            # long runs of ties in every row
+    parent = torch.tensor([[-1, 0, 1, 2, 3, 4, 5, 6]] * B, dtype=torch.int32)
+    cand = torch.zeros((B, T), dtype=torch.int32)
+    r = _accept_only(x, cand, parent, cuda)
+    amax = oracle.argmax(x)
+    assert torch.equal(r["argmax"], amax)
+    assert amax[0, :7].tolist() == [3, 8999, 0, V - 1, 0, 77, 0] and amax[1].tolist() == [1000] * T
+
+
+def test_argmax_unaligned_rows(cuda):
+    """V odd: bf16 rows start off 16-byte boundaries; every split point is exercised."""
+    for V in (1, 7, 1001, 40001):
+        g = torch.Generator().manual_seed(V)
+        x = (torch.randn(3, 5, V, generator=g) * 4).to(torch.bfloat16)
+        parent = torch.tensor([[-1, 0, 0, 1, 2]] * 3, dtype=torch.int32)
+        cand = torch.randint(0, V, (3, 5), generator=g, dtype=torch.int32)
+        r = _accept_only(x, cand, parent, cuda)
+        amax = oracle.argmax(x)
+        assert torch.equal(r["argmax"], amax), V
+        path, alen, bonus = oracle.accept_walk(parent, cand, amax)
+        assert torch.equal(r["path"], path) and torch.equal(r["alen"], alen) and torch.equal(r["bonus"], bonus)
+
+
+def test_walk_duplicates_and_deep_chain(cuda):
+    V = 16
+    parent = torch.tensor([[-1, 0, 0, 1, 2] + [-1] * 59,
+                           [-1] + list(range(63))], dtype=torch.int32)
+    parent[0, 5:] = 0                                    # extra root children
+    cand = torch.zeros((2, 64), dtype=torch.int32)
+    cand[0, :5] = torch.tensor([9, 5, 5, 7, 7])
+    cand[0, 5:] = torch.arange(59) % 3 + 10
+    logits = torch.zeros((2, 64, V), dtype=torch.float32)
+    logits[0, 0, 5] = 1.0                                # root argmax 5: nodes 1 and 2 both match
+    logits[0, 1, 1] = 1.0
+    logits[0, 2, 7] = 1.0
+    logits[1, :, 3] = 1.0                                # chain: every node predicts 3
+    cand[1, 1:] = 3
+    r = _accept_only(logits, cand, parent, cuda)
+    amax = oracle.argmax(logits)
+    path, alen, bonus = oracle.accept_walk(parent, cand, amax)
+    assert torch.equal(r["path"], path) and torch.equal(r["alen"], alen) and torch.equal(r["bonus"], bonus)
+    assert int(alen[0]) == 2 and int(alen[1]) == 64
+
+
+def test_bad_tree_reports_status(cuda):
+    w = workloads.get("7b_l2048", T=8, Hq=4, Hkv=4, L=300, V=1000, branching=(2, 2, 1))
+    host = workloads.make(w)
+    host["parent"][0, 5] = 6                             # a node whose parent comes after it
+    t = to_dev(host, cuda)
+    step = run_gpu(t)
+    assert int(step.status.item()) & pkg.api.ERR_BAD_TREE
+
+
+def test_capacity_reports_status(cuda):
+    w = workloads.get("7b_l2048", T=8, Hq=4, Hkv=4, L=300, V=1000, branching=(2, 2, 1))
+    host = workloads.make(w)
+    host["cache_len"][0] = host["Lcap"] - w.T + 1
+    t = to_dev(host, cuda)
+    step = run_gpu(t)
+    assert int(step.status.item()) & pkg.api.ERR_CAPACITY
+
+
+def test_host_errors_raise(cuda):
+    w = workloads.get("tiny_f32")
+    t = to_dev(workloads.make(w), cuda)
+    out = torch.empty_like(t["q"])
+    with pytest.raises(pkg.CloverError):
+        pkg.clover_verify_attn(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"],
+                               t["parent"], out, scale=float("inf"))
+    new_len = t["cache_len"]
+    with pytest.raises(pkg.CloverError):   # new length may not alias the old one
+        pkg.clover_kv_compact(t["k_cache"], t["v_cache"], t["cache_len"], torch.zeros_like(t["parent"]),
+                              torch.ones_like(t["cache_len"]), new_len)
