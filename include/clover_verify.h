@@ -56,7 +56,8 @@ typedef enum {
     CLOVER_ERR_BAD_TREE = 4,     /* device: parent array is not a topologically numbered tree */
     CLOVER_ERR_CAPACITY = 8,     /* device: cache_len[b] < 0 or cache_len[b] + T > Lcap */
     CLOVER_ERR_CUDA = 16,        /* a CUDA launch or query failed */
-    CLOVER_ERR_TIMEOUT = 32      /* reserved: a bounded device wait gave up */
+    CLOVER_ERR_TIMEOUT = 32,     /* reserved: a bounded device wait gave up */
+    CLOVER_ERR_SCRATCH_LIMIT = 64 /* clover_verify_attn_noalloc: scratch need exceeds its static buffer */
 } clover_status;
 
 typedef enum {
@@ -163,6 +164,48 @@ CLOVER_API clover_status clover_kv_compact(void *k_cache, void *v_cache, const i
                                 int32_t *new_cache_len, int32_t *src_index_out,
                                 int B, int T, int Hkv, int D, int Lcap, clover_dtype dtype,
                                 int32_t *status, void *stream);
+
+/*
+ * Bytes of the static device scratch buffer behind clover_verify_attn_noalloc.
+ */
+#define CLOVER_NOALLOC_SCRATCH_BYTES ((size_t)8 << 20)
+
+/*
+ * clover_verify_attn without a caller-provided workspace.  The paper has no
+ * counterpart; this entry point exists for deployment.
+ *
+ * Who needs it: callers that cannot allocate device memory themselves.  Two
+ * examples are a plugin inside a serving process whose memory manager has
+ * already reserved the free HBM for its own pool, and latency-critical code
+ * that must not make a call that may synchronise the device (cudaMalloc can).
+ * Such callers cannot supply the workspace clover_verify_attn asks for.
+ *
+ * Behaviour: the same computation, arguments and results as clover_verify_attn
+ * (inputs and outputs are still caller-owned device memory).  The split-KV
+ * scratch lives in one file-scope static device array of
+ * CLOVER_NOALLOC_SCRATCH_BYTES (8 MiB).  Every GPU that loads the library holds
+ * that array until the process exits.  This call allocates nothing: it calls no
+ * cudaMalloc, cudaFree or allocating library routine.
+ *   - The first call on a device looks up the array's device address with that
+ *     device current (cudaGetSymbolAddress) and caches it.  Make this first call
+ *     before any stream capture that contains later calls.
+ *   - Each call clears the part of the array that must start at zero (the
+ *     arrival counters) with an asynchronous memset on `stream`, then launches.
+ *     The rest of the array keeps the previous call's contents, which are
+ *     overwritten before they are read.
+ *   - All calls on a device share the one array: calls whose executions
+ *     overlap on the GPU (on any streams) race and give wrong results.
+ *     Serialise them.
+ *   - Sizes whose scratch need (clover_verify_attn_workspace_size) exceeds the
+ *     buffer are rejected with CLOVER_ERR_SCRATCH_LIMIT before anything is
+ *     launched; other errors are those of clover_verify_attn.
+ */
+CLOVER_API clover_status clover_verify_attn_noalloc(const void *q, const void *k_new, const void *v_new,
+                                                    void *k_cache, void *v_cache, const int32_t *cache_len,
+                                                    const int32_t *parent, void *out,
+                                                    int B, int T, int Hq, int Hkv, int D, int Lcap,
+                                                    clover_dtype dtype, float scale,
+                                                    int32_t *status, void *stream);
 
 #ifdef __cplusplus
 }

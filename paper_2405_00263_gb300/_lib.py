@@ -25,7 +25,12 @@ EXPORTS = (
     "clover_verify_accept_workspace_size",
     "clover_verify_accept",
     "clover_kv_compact",
+    "clover_verify_attn_noalloc",
 )
+
+# Bytes of the static scratch buffer behind clover_verify_attn_noalloc
+# (CLOVER_NOALLOC_SCRATCH_BYTES in include/clover_verify.h).
+NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
 def library_path() -> str:
@@ -61,5 +66,7 @@ def load(build_if_missing: bool = False):
         lib.clover_verify_accept.restype = I
         lib.clover_kv_compact.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P, P]
         lib.clover_kv_compact.restype = I
+        lib.clover_verify_attn_noalloc.argtypes = [P, P, P, P, P, P, P, P, I, I, I, I, I, I, I, F, P, P]
+        lib.clover_verify_attn_noalloc.restype = I
         _lib = lib
         return lib

@@ -21,6 +21,7 @@ ERR_BAD_TREE = 4
 ERR_CAPACITY = 8
 ERR_CUDA = 16
 ERR_TIMEOUT = 32
+ERR_SCRATCH_LIMIT = 64
 
 F32 = 0
 BF16 = 1
@@ -111,6 +112,31 @@ def clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out
         _ptr(status), _stream(stream))
     if code != OK:
         raise CloverError(code, "clover_verify_attn")
+
+
+def clover_verify_attn_noalloc(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, scale=0.0,
+                               status=None, stream=None):
+    """clover_verify_attn for callers that cannot allocate device memory: the
+    scratch is a static 8 MiB device buffer inside the library, shared by every
+    call on a device (calls that overlap on the GPU race)."""
+    B, T, Hq, D = q.shape
+    Hkv, Lcap = k_cache.shape[1], k_cache.shape[2]
+    dt = q.dtype
+    _check(k_new, (B, T, Hkv, D), dt, "k_new")
+    _check(v_new, (B, T, Hkv, D), dt, "v_new")
+    _check(k_cache, (B, Hkv, Lcap, D), dt, "k_cache")
+    _check(v_cache, (B, Hkv, Lcap, D), dt, "v_cache")
+    _check(cache_len, (B,), torch.int32, "cache_len")
+    _check(parent, (B, T), torch.int32, "parent")
+    _check(out, (B, T, Hq, D), dt, "out")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, status)
+    code = _lib.load().clover_verify_attn_noalloc(
+        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(cache_len), _ptr(parent),
+        _ptr(out), B, T, Hq, Hkv, D, Lcap, dtype_code(dt), float(scale), _ptr(status), _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_verify_attn_noalloc")
 
 
 def clover_verify_accept(logits, cand, parent, argmax_out, path_out, accept_len, bonus_token,

@@ -3,6 +3,8 @@
 // each call are in include/clover_verify.h.
 #include <math.h>
 
+#include <atomic>
+
 #include "common.cuh"
 
 namespace clover {
@@ -86,6 +88,7 @@ const char *clover_status_string(int status) {
         case CLOVER_ERR_CAPACITY: return "cache length out of range or cache too small";
         case CLOVER_ERR_CUDA: return "CUDA error";
         case CLOVER_ERR_TIMEOUT: return "device wait timed out";
+        case CLOVER_ERR_SCRATCH_LIMIT: return "scratch need exceeds the static buffer of clover_verify_attn_noalloc";
         default: return "several errors (bitwise OR of codes)";
     }
 }
@@ -187,3 +190,69 @@ clover_status clover_kv_compact(void *k_cache, void *v_cache, const int32_t *cac
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free attention: the split-KV scratch of clover_verify_attn lives in
+// a static device array instead of a caller-provided workspace.
+// ---------------------------------------------------------------------------
+
+namespace clover {
+namespace {
+
+static_assert(CLOVER_NOALLOC_SCRATCH_BYTES % 256 == 0, "scratch size must keep 256-byte alignment");
+
+// Resident on every device that loads this library, until the process exits.
+static __device__ __align__(256) unsigned char g_attn_scratch[CLOVER_NOALLOC_SCRATCH_BYTES];
+
+// Device address of g_attn_scratch per device, looked up once with that device current.
+constexpr int kMaxDevices = 64;
+std::atomic<void *> g_attn_scratch_addr[kMaxDevices];
+
+cudaError_t attn_scratch_address(void **addr) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    void *p = g_attn_scratch_addr[dev].load(std::memory_order_acquire);
+    if (p == nullptr) {
+        e = cudaGetSymbolAddress(&p, g_attn_scratch);
+        if (e != cudaSuccess) return e;
+        g_attn_scratch_addr[dev].store(p, std::memory_order_release);
+    }
+    *addr = p;
+    return cudaSuccess;
+}
+
+}  // namespace
+}  // namespace clover
+
+extern "C" clover_status clover_verify_attn_noalloc(const void *q, const void *k_new, const void *v_new,
+                                                    void *k_cache, void *v_cache, const int32_t *cache_len,
+                                                    const int32_t *parent, void *out, int B, int T, int Hq,
+                                                    int Hkv, int D, int Lcap, clover_dtype dtype, float scale,
+                                                    int32_t *status, void *stream) {
+    using namespace clover;
+    const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype);
+    if (s != CLOVER_OK) return s;
+    if (B == 0) return CLOVER_OK;
+    // the argument checks of clover_verify_attn, repeated so that nothing (not
+    // even the counter memset) is issued for a call it would reject
+    if (!q || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !parent || !out)
+        return CLOVER_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache) ||
+        !aligned16(out))
+        return CLOVER_ERR_INVALID_ARG;
+    if (!(scale == scale) || isinf(scale)) return CLOVER_ERR_INVALID_ARG;
+    const AttnPlan p = plan_attn(B, T, Hq, Hkv, D, Lcap);
+    if (p.total > CLOVER_NOALLOC_SCRATCH_BYTES) return CLOVER_ERR_SCRATCH_LIMIT;
+
+    void *scratch = nullptr;
+    if (attn_scratch_address(&scratch) != cudaSuccess) return CLOVER_ERR_CUDA;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (p.counter_bytes > 0 &&
+        cudaMemsetAsync(static_cast<uint8_t *>(scratch) + p.o_bytes + p.ml_bytes, 0, p.counter_bytes, st) !=
+            cudaSuccess)
+        return CLOVER_ERR_CUDA;
+    return clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, B, T, Hq, Hkv, D, Lcap,
+                              dtype, scale, scratch, CLOVER_NOALLOC_SCRATCH_BYTES, status, stream);
+}

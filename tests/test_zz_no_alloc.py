@@ -1,0 +1,95 @@
+"""The allocation-free attention entry point, called through the C ABI.
+
+Some callers of this library cannot allocate device memory (a plugin whose host
+process has already reserved the free HBM for its own pool, or code that must
+not make a call that may synchronise the device).  clover_verify_attn_noalloc
+serves them by keeping its split-KV scratch in a static device buffer.  This
+test checks that it gives the same results as clover_verify_attn with a
+caller-provided workspace, on two calls in a row (the second call finds the
+buffer holding the first call's contents), and that a size whose scratch need
+exceeds the buffer is refused before anything runs.
+
+The file is named so that pytest collects it last.
+"""
+
+import ctypes
+
+import pytest
+import torch
+
+import paper_2405_00263_gb300 as pkg
+from paper_2405_00263_gb300 import _lib
+from synth import workloads
+
+pytestmark = pytest.mark.gpu
+
+ATOL_BF16 = 2e-2
+
+
+def _p(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else None
+
+
+def _call_noalloc(lib, t, out, status, stream):
+    B, T, Hq, D = t["q"].shape
+    Hkv, Lcap = t["k_cache"].shape[1], t["k_cache"].shape[2]
+    return lib.clover_verify_attn_noalloc(
+        _p(t["q"]), _p(t["k_new"]), _p(t["v_new"]), _p(t["k_cache"]), _p(t["v_cache"]), _p(t["cache_len"]),
+        _p(t["parent"]), _p(out), B, T, Hq, Hkv, D, Lcap, pkg.BF16, 0.0, _p(status),
+        ctypes.c_void_p(stream.cuda_stream))
+
+
+def test_noalloc_matches_workspace_entry_point_on_two_calls(cuda):
+    lib = _lib.load(build_if_missing=True)
+    w = workloads.get("7b_l2048")
+    base = workloads.make(w, device=cuda)
+    B, T, Hq, Hkv, D, Lcap = w.B, w.T, w.Hq, w.Hkv, w.D, base["Lcap"]
+    need = pkg.clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, Lcap, torch.bfloat16)
+    assert 0 < need <= _lib.NOALLOC_SCRATCH_BYTES       # this shape does use scratch
+    stream = torch.cuda.current_stream()
+
+    # the existing entry point with a caller-provided, zero-filled workspace
+    ref = {k: (v.clone() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
+    out_ref = torch.empty_like(ref["q"])
+    ws = torch.zeros(need, dtype=torch.uint8, device=cuda)
+    st_ref = torch.zeros(1, dtype=torch.int32, device=cuda)
+    pkg.clover_verify_attn(ref["q"], ref["k_new"], ref["v_new"], ref["k_cache"], ref["v_cache"], ref["cache_len"],
+                           ref["parent"], out_ref, workspace=ws, status=st_ref)
+    torch.cuda.synchronize()
+    assert int(st_ref.item()) == 0
+
+    for call in range(2):
+        t = {k: (v.clone() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
+        out = torch.full_like(t["q"], float("nan"))
+        st = torch.zeros(1, dtype=torch.int32, device=cuda)
+        code = _call_noalloc(lib, t, out, st, stream)
+        assert code == 0, lib.clover_status_string(code)
+        torch.cuda.synchronize()
+        assert int(st.item()) == 0, f"call {call}: device status {int(st.item())}"
+        err = (out.float() - out_ref.float()).abs().max().item()
+        assert err <= ATOL_BF16, f"call {call}: max-abs difference {err}"
+        # the tree K/V append is the same as well
+        L = int(base["cache_len"][0])
+        assert torch.equal(t["k_cache"][:, :, :L + T], ref["k_cache"][:, :, :L + T])
+        assert torch.equal(t["v_cache"][:, :, :L + T], ref["v_cache"][:, :, :L + T])
+
+
+def test_noalloc_rejects_scratch_beyond_its_buffer():
+    """Host-side refusal: nothing is launched, so no GPU work is needed here,
+    but the check lives with the GPU test of the entry point."""
+    lib = _lib.load(build_if_missing=True)
+    shape = None
+    for Hkv in (150, 300, 600, 1200, 2400):
+        for Lcap in (4096, 65536):
+            if lib.clover_verify_attn_workspace_size(1, 64, Hkv, Hkv, 128, Lcap, pkg.BF16) > _lib.NOALLOC_SCRATCH_BYTES:
+                shape = (Hkv, Lcap)
+                break
+        if shape:
+            break
+    assert shape is not None
+    Hkv, Lcap = shape
+    P = ctypes.c_void_p
+    code = lib.clover_verify_attn_noalloc(P(256), P(256), P(256), P(256), P(256), P(256), P(256), P(256),
+                                          1, 64, Hkv, Hkv, 128, Lcap, pkg.BF16, 0.0, None, None)
+    assert code == pkg.api.ERR_SCRATCH_LIMIT
+    assert b"static buffer" in lib.clover_status_string(code)
