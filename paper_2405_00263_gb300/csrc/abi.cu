@@ -9,7 +9,9 @@
 
 namespace clover {
 int fma_row_tile();
+int tc_row_tile();
 cudaError_t launch_tree_attn_fma(const AttnArgs &a, cudaStream_t stream);
+cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream);
 void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk);
 size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T, int V,
@@ -22,16 +24,19 @@ cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const int32_t *cache
 namespace {
 
 constexpr int kAbiVersion = 1;
-constexpr int kTargetAttnCtas = 2 * 152;   // two resident attention CTAs per SM on a 152-SM GPU
+constexpr int kSms = 152;                  // SMs of a GB300 (planning constant; any GPU runs the plan)
+constexpr int kTargetAttnCtas = 2 * kSms;  // FMA path: two resident CTAs per SM
 constexpr int kMinKeysPerSplit = 256;
 constexpr int kMaxSplits = 64;
+constexpr int kTcMinRows = 16;             // query rows per KV head from which the tensor-core path is used
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct AttnPlan {
-    int row_tile, row_tiles, n_split;
+    bool tc;                 // tensor-core (tcgen05) kernel, else the FMA kernel
+    int row_tile, row_tiles, n_split, slot_rows;
     size_t o_bytes, ml_bytes, counter_bytes, total;
 };
 
@@ -44,24 +49,41 @@ clover_status check_attn_sizes(int B, int T, int Hq, int Hkv, int D, int Lcap, i
     return CLOVER_OK;
 }
 
-AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap) {
+// Kernel choice, split count and workspace layout for one shape.  bf16 with at
+// least kTcMinRows query rows per KV head runs on the tensor cores with one CTA
+// per SM (splits chosen so that one wave fills the SMs); everything else runs
+// on the FMA kernel with two CTAs per SM.
+AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
     AttnPlan p;
     const int G = Hq / Hkv;
-    p.row_tile = fma_row_tile();
-    p.row_tiles = (T * G + p.row_tile - 1) / p.row_tile;
-    const long base = (long)(B > 0 ? B : 1) * Hkv * p.row_tiles;
-    int n = (int)((kTargetAttnCtas + base - 1) / base);
+    const int rows = T * G;
+    const long Bp = B > 0 ? B : 1;
     const int by_len = (Lcap + kMinKeysPerSplit - 1) / kMinKeysPerSplit;
+    int n;
+    p.tc = (dtype == CLOVER_BF16) && rows >= kTcMinRows;
+    if (p.tc) {
+        p.row_tile = tc_row_tile();
+        p.row_tiles = (rows + p.row_tile - 1) / p.row_tile;
+        p.slot_rows = rows < p.row_tile ? rows : p.row_tile;
+        const long base = Bp * Hkv * p.row_tiles;
+        n = base >= kSms ? 1 : (int)(kSms / base);
+    } else {
+        p.row_tile = fma_row_tile();
+        p.row_tiles = (rows + p.row_tile - 1) / p.row_tile;
+        p.slot_rows = p.row_tile;
+        const long base = Bp * Hkv * p.row_tiles;
+        n = (int)((kTargetAttnCtas + base - 1) / base);
+    }
     if (n > by_len) n = by_len;
     if (n > kMaxSplits) n = kMaxSplits;
     if (n < 1) n = 1;
     p.n_split = n;
-    const size_t heads = (size_t)(B > 0 ? B : 1) * Hkv * p.row_tiles;
+    const size_t heads = (size_t)Bp * Hkv * p.row_tiles;
     if (n == 1) {
         p.o_bytes = p.ml_bytes = p.counter_bytes = p.total = 0;
     } else {
-        p.o_bytes = round_up(sizeof(float) * heads * n * p.row_tile * D, 256);
-        p.ml_bytes = round_up(sizeof(float) * heads * n * p.row_tile * 2, 256);
+        p.o_bytes = round_up(sizeof(float) * heads * n * p.slot_rows * D, 256);
+        p.ml_bytes = round_up(sizeof(float) * heads * n * p.slot_rows * 2, 256);
         p.counter_bytes = round_up(sizeof(unsigned) * heads, 256);
         p.total = p.o_bytes + p.ml_bytes + p.counter_bytes;
     }
@@ -95,7 +117,7 @@ const char *clover_status_string(int status) {
 
 size_t clover_verify_attn_workspace_size(int B, int T, int Hq, int Hkv, int D, int Lcap, clover_dtype dtype) {
     if (check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype) != CLOVER_OK) return 0;
-    return plan_attn(B, T, Hq, Hkv, D, Lcap).total;
+    return plan_attn(B, T, Hq, Hkv, D, Lcap, dtype).total;
 }
 
 clover_status clover_verify_attn(const void *q, const void *k_new, const void *v_new, void *k_cache,
@@ -112,7 +134,7 @@ clover_status clover_verify_attn(const void *q, const void *k_new, const void *v
         !aligned16(out))
         return CLOVER_ERR_INVALID_ARG;
     if (!(scale == scale) || isinf(scale)) return CLOVER_ERR_INVALID_ARG;
-    const AttnPlan p = plan_attn(B, T, Hq, Hkv, D, Lcap);
+    const AttnPlan p = plan_attn(B, T, Hq, Hkv, D, Lcap, dtype);
     if (ws_bytes < p.total || (p.total > 0 && (!workspace || !aligned16(workspace)))) return CLOVER_ERR_INVALID_ARG;
 
     AttnArgs a;
@@ -138,12 +160,14 @@ clover_status clover_verify_attn(const void *q, const void *k_new, const void *v
     a.row_tile = p.row_tile;
     a.row_tiles = p.row_tiles;
     a.n_split = p.n_split;
+    a.slot_rows = p.slot_rows;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     a.part_o = p.total ? reinterpret_cast<float *>(ws) : nullptr;
     a.part_ml = p.total ? reinterpret_cast<float *>(ws + p.o_bytes) : nullptr;
     a.counters = p.total ? reinterpret_cast<unsigned *>(ws + p.o_bytes + p.ml_bytes) : nullptr;
     a.status = status;
-    return from_cuda(launch_tree_attn_fma(a, static_cast<cudaStream_t>(stream)));
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    return from_cuda(p.tc ? launch_tree_attn_tc(a, st) : launch_tree_attn_fma(a, st));
 }
 
 size_t clover_verify_accept_workspace_size(int B, int T, int V, clover_dtype dtype) {
@@ -243,7 +267,7 @@ extern "C" clover_status clover_verify_attn_noalloc(const void *q, const void *k
         !aligned16(out))
         return CLOVER_ERR_INVALID_ARG;
     if (!(scale == scale) || isinf(scale)) return CLOVER_ERR_INVALID_ARG;
-    const AttnPlan p = plan_attn(B, T, Hq, Hkv, D, Lcap);
+    const AttnPlan p = plan_attn(B, T, Hq, Hkv, D, Lcap, dtype);
     if (p.total > CLOVER_NOALLOC_SCRATCH_BYTES) return CLOVER_ERR_SCRATCH_LIMIT;
 
     void *scratch = nullptr;

@@ -10,10 +10,10 @@
 // Grid: one CTA per (logit row, vocabulary chunk).  Each CTA reduces its chunk
 // with 16-byte loads to a packed 64-bit key (order-preserving value bits in the
 // high word, bit-inverted index in the low word) so that one unsigned max
-// gives "largest value, then smallest index".  The last chunk of a row to
-// finish (per-row arrival counter) merges the chunk keys and writes the
-// argmax; the last row of a sequence to finish runs the walk for that sequence
-// in one warp.  Counters are reset by the CTAs that complete them.
+// gives "largest value, then smallest index", and folds it into the row's key
+// with a 64-bit atomic max.  The CTA that finishes the last chunk of a
+// sequence (per-sequence arrival counter) decodes the argmax of every node and
+// runs the walk in one warp; it also resets the keys and the counter.
 #include "common.cuh"
 
 namespace clover {
@@ -109,27 +109,33 @@ struct AcceptArgs {
     const int32_t *cand, *parent;
     int B, T, V, n_chunks, chunk;
     int32_t *argmax_out, *path_out, *accept_len, *bonus;
-    uint64_t *keys;          // [B*T, n_chunks]
-    unsigned *row_count;     // [B*T]
-    unsigned *seq_count;     // [B]
+    unsigned long long *row_key;   // [B*T] running packed maximum of each logit row
+    unsigned *seq_count;           // [B] chunks of the sequence's rows finished
     int32_t *status;
 };
 
-// Greedy walk of sequence b by one warp: lane l owns nodes l and l + 32.
+// Argmax of every node of sequence b from the merged row keys, then the greedy
+// walk, by one warp: lane l owns nodes l and l + 32.  The walk reads the argmax
+// of the current node from registers (warp shuffles), so each step costs no
+// memory round trip.  The row keys and the counter are reset for the next call.
 __device__ void accept_walk_warp(const AcceptArgs &a, int b) {
     const int lane = threadIdx.x & 31;
     const int T = a.T;
     const int32_t *par = a.parent + (size_t)b * T;
     const int32_t *cd = a.cand + (size_t)b * T;
-    const int32_t *am = a.argmax_out + (size_t)b * T;
-    int p[2], c[2];
+    int p[2], c[2], am[2];
     bool invalid = false;
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
         const int i = lane + 32 * k;
         p[k] = -2;
         c[k] = 0;
+        am[k] = 0;
         if (i < T) {
+            const unsigned long long key = __ldcg(a.row_key + (size_t)b * T + i);
+            am[k] = (int)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+            a.argmax_out[(size_t)b * T + i] = am[k];
+            a.row_key[(size_t)b * T + i] = 0ull;                      // ready for the next call
             p[k] = __ldg(par + i);
             c[k] = __ldg(cd + i);
             if (i == 0 ? (p[k] != -1) : (p[k] < 0 || p[k] >= i)) invalid = true;
@@ -140,12 +146,17 @@ __device__ void accept_walk_warp(const AcceptArgs &a, int b) {
     __syncwarp();
     int cur = 0, len = 1;
     if (lane == 0) path[0] = 0;
+    auto argmax_of = [&](int node) {
+        const int lo = __shfl_sync(0xffffffffu, am[0], node & 31);
+        const int hi = __shfl_sync(0xffffffffu, am[1], node & 31);
+        return (node >> 5) ? hi : lo;
+    };
     if (__any_sync(0xffffffffu, invalid)) {
         if (lane == 0) report(a.status, CLOVER_ERR_BAD_TREE);
     } else {
         // at most T - 1 steps: every step moves to a larger node index
         for (int step = 1; step < T; ++step) {
-            const int want = __ldcg(am + cur);
+            const int want = argmax_of(cur);
             const unsigned lo = __ballot_sync(0xffffffffu, p[0] == cur && c[0] == want);
             const unsigned hi = __ballot_sync(0xffffffffu, p[1] == cur && c[1] == want);
             const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
@@ -155,16 +166,18 @@ __device__ void accept_walk_warp(const AcceptArgs &a, int b) {
             ++len;
         }
     }
+    const int bonus = argmax_of(cur);
     if (lane == 0) {
         a.accept_len[b] = len;
-        a.bonus[b] = __ldcg(am + cur);
+        a.bonus[b] = bonus;
+        a.seq_count[b] = 0u;                                       // ready for the next call
     }
 }
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
     __shared__ uint64_t s_red[kThreads / 32];
-    __shared__ int s_row_last, s_seq_last;
+    __shared__ int s_seq_last;
     const int row = blockIdx.x;               // b * T + i
     const int chunk_id = blockIdx.y;
     const int b = row / a.T;
@@ -187,34 +200,19 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
     }
     best = block_max(best, s_red);
 
-    if (a.n_chunks > 1) {
-        if (threadIdx.x == 0) {
-            a.keys[(size_t)row * a.n_chunks + chunk_id] = best;
-            __threadfence();
-            const unsigned prev = atomicAdd(a.row_count + row, 1u);
-            s_row_last = (prev == (unsigned)a.n_chunks - 1u);
-        }
-        __syncthreads();
-        if (!s_row_last) return;
-        if (threadIdx.x == 0) {
-            __threadfence();
-            best = 0ull;
-            for (int k = 0; k < a.n_chunks; ++k) best = umax64(best, __ldcg(a.keys + (size_t)row * a.n_chunks + k));
-            a.row_count[row] = 0u;
-        }
-    }
+    // fold this chunk into the row's key, then count the chunk as done for the
+    // sequence; the CTA finishing the sequence's last chunk runs the walk
     if (threadIdx.x == 0) {
-        a.argmax_out[row] = (int32_t)(0xFFFFFFFFu - (uint32_t)(best & 0xFFFFFFFFull));
+        atomicMax(a.row_key + row, static_cast<unsigned long long>(best));
         __threadfence();
         const unsigned prev = atomicAdd(a.seq_count + b, 1u);
-        s_seq_last = (prev == (unsigned)a.T - 1u);
+        s_seq_last = (prev == (unsigned)(a.T * a.n_chunks) - 1u);
     }
     __syncthreads();
     if (!s_seq_last) return;
     if (threadIdx.x < 32) {
         __threadfence();
         accept_walk_warp(a, b);
-        if (threadIdx.x == 0) a.seq_count[b] = 0u;
     }
 }
 
@@ -235,11 +233,9 @@ void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk) {
 }
 
 size_t accept_workspace_bytes(int B, int T, int V, int dtype) {
-    int n, c;
-    accept_plan(B, T, V, dtype, &n, &c);
-    const size_t keys = sizeof(uint64_t) * (size_t)B * T * n;
-    const size_t counters = sizeof(unsigned) * ((size_t)B * T + B);
-    return keys + counters;
+    (void)V;
+    (void)dtype;
+    return sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * (size_t)B;
 }
 
 cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
@@ -257,9 +253,8 @@ cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t
     a.path_out = path_out;
     a.accept_len = accept_len;
     a.bonus = bonus;
-    a.keys = static_cast<uint64_t *>(workspace);
-    a.row_count = reinterpret_cast<unsigned *>(a.keys + (size_t)B * T * a.n_chunks);
-    a.seq_count = a.row_count + (size_t)B * T;
+    a.row_key = static_cast<unsigned long long *>(workspace);
+    a.seq_count = reinterpret_cast<unsigned *>(a.row_key + (size_t)B * T);
     a.status = status;
     dim3 grid(B * T, a.n_chunks);
     if (dtype == CLOVER_F32) accept_kernel<float><<<grid, kThreads, 0, stream>>>(a);

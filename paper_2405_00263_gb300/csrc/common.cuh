@@ -24,8 +24,9 @@ struct AttnArgs {
     int row_tile;          // rows per CTA
     int row_tiles;         // ceil(rows / row_tile)
     int n_split;           // cache key ranges per (sequence, KV head, row tile)
-    float *part_o;         // [B, Hkv, row_tiles, n_split, row_tile, D]
-    float *part_ml;        // [B, Hkv, row_tiles, n_split, row_tile, 2]  (max, sum)
+    int slot_rows;         // rows of one partial-result slot (<= row_tile)
+    float *part_o;         // [B, Hkv, row_tiles, n_split, slot_rows, D]
+    float *part_ml;        // [B, Hkv, row_tiles, n_split, slot_rows, 2]  (max, sum)
     unsigned *counters;    // [B, Hkv, row_tiles]
     int32_t *status;
 };

@@ -24,38 +24,36 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
     __shared__ int s_ok;
     const int g = blockIdx.x;
     const int b = blockIdx.y;
+    // the length, the accepted count and the whole path row are loaded at once
     const int L = __ldg(cache_len + b);
     const int a = __ldg(accept_len + b);
-    if (threadIdx.x == 0) {
-        int ok = (a >= 1 && a <= T) ? 1 : 0;
-        if (L < 0 || L + T > Lcap) {
-            ok = 0;
-            if (g == 0) report(status, CLOVER_ERR_CAPACITY);
-        }
-        s_ok = ok;
-    }
-    __syncthreads();
-    if (!s_ok) {
-        if (g == 0 && threadIdx.x == 0 && (a < 1 || a > T)) report(status, CLOVER_ERR_INVALID_ARG);
-        return;
-    }
     if (threadIdx.x < 32) {
-        bool bad = false;
-        for (int j = threadIdx.x; j < a; j += 32) {
-            const int p = __ldg(path + (size_t)b * T + j);
-            if (p < 0 || p >= T) bad = true;
-            s_src[j] = (p < 0 || p >= T) ? j : p;
+        int p0 = -1, p1 = -1;
+        if (threadIdx.x < T) p0 = __ldg(path + (size_t)b * T + threadIdx.x);
+        if (threadIdx.x + 32 < T) p1 = __ldg(path + (size_t)b * T + threadIdx.x + 32);
+        const bool len_ok = (a >= 1 && a <= T);
+        const bool cap_ok = (L >= 0 && L + T <= Lcap);
+        const int j0 = threadIdx.x, j1 = threadIdx.x + 32;
+        const bool bad0 = j0 < a && (p0 < 0 || p0 >= T);
+        const bool bad1 = j1 < a && (p1 < 0 || p1 >= T);
+        const bool bad_path = __any_sync(0xffffffffu, bad0 || bad1);
+        s_src[j0] = bad0 ? j0 : p0;
+        s_src[j1] = bad1 ? j1 : p1;
+        if (threadIdx.x == 0) {
+            s_ok = len_ok && cap_ok;
+            if (g == 0 && !cap_ok) report(status, CLOVER_ERR_CAPACITY);
+            if (g == 0 && (!len_ok || bad_path)) report(status, CLOVER_ERR_INVALID_ARG);
         }
-        bad = __any_sync(0xffffffffu, bad);
-        if (threadIdx.x == 0 && bad) report(status, CLOVER_ERR_INVALID_ARG);
-        __syncwarp();
-        if (g == 0) {
-            if (src_index)
-                for (int j = threadIdx.x; j < T; j += 32) src_index[(size_t)b * T + j] = (j < a) ? L + s_src[j] : -1;
+        if (g == 0 && len_ok && cap_ok) {
+            if (src_index) {
+                if (j0 < T) src_index[(size_t)b * T + j0] = (j0 < a) ? L + s_src[j0] : -1;
+                if (j1 < T) src_index[(size_t)b * T + j1] = (j1 < a) ? L + s_src[j1] : -1;
+            }
             if (threadIdx.x == 0) new_cache_len[b] = L + a;
         }
     }
     __syncthreads();
+    if (!s_ok) return;
 
     const int units = row_bytes / 16;
     const size_t head_base = ((size_t)b * Hkv + g) * Lcap;

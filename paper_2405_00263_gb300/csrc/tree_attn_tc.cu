@@ -1,0 +1,553 @@
+// Tree-masked split-KV attention on the 5th-generation tensor cores (tcgen05,
+// sm_103a) for bf16 inputs.
+//
+// The operation is the tree attention of the verification phase (Sections 2.1
+// and 2.2 of the Clover paper): every tree node attends to all committed cache
+// keys and to the tree nodes on its own root path (the tree topology as mask).
+//
+// One CTA per (row tile of up to 128 query rows, cache-key split, sequence x
+// KV head).  The T*G query rows of a KV head (row i*G + hh = node i, query head
+// g*G + hh) share every K/V tile, so per 64-key tile:
+//   S  = Q K^T        tcgen05.mma M=128 N=64 K=D  (Q, K K-major in smem, S in TMEM)
+//   P  = 2^(S*c - m)  online softmax in registers, bf16 P to smem
+//   O += P V          tcgen05.mma M=128 N=D K=64  (V MN-major in smem, O in TMEM)
+// O stays in TMEM for the whole key range.  Each row keeps a reference max m;
+// P is taken relative to it, and m (with O and the row sum) is only moved when
+// a tile's max exceeds it by more than 2^8, so O is rarely rescaled.
+// Warp roles (192 threads): warp q in 0-3 runs the softmax, rescales and the
+// epilogue of TMEM lanes 32q.. (the lanes warp q may access); warp 4 issues the
+// TMA loads of K/V tiles (4-stage ring, 128-byte swizzle) and appends the tree
+// K/V to the cache; warp 5 allocates TMEM and issues the MMAs from one thread.
+// The split that owns the last cache range also takes the tile of T tree keys
+// (read from k_new/v_new) under the ancestor bitmask.  Splits are merged by the
+// CTA that arrives last at a per-head counter, as in the FMA kernel.
+// Every mbarrier wait is bounded; on a timeout the CTA reports
+// CLOVER_ERR_TIMEOUT, winds down, waits (bounded) for its copies in flight and
+// frees its TMEM.
+#include "common.cuh"
+#include "tc_ptx.cuh"
+#include "tmap_host.cuh"
+
+namespace clover {
+namespace {
+
+using namespace tc;
+
+constexpr int BM = 128;                 // query rows per CTA (MMA M)
+constexpr int BN = 64;                  // keys per tile
+constexpr int NS = 4;                   // K/V pipeline stages
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 256;     // S: 2 x 64 columns, O: D columns
+constexpr float kRescale = 8.0f;        // move the reference max only past 2^8 growth
+constexpr uint64_t kWaitNs = 500ull * 1000 * 1000;   // 0.5 s per wait
+
+template <int D>
+struct TcSmem {
+    static constexpr int DH = D / 64;                // 128-byte column blocks per row
+    static constexpr int q_bytes = BM * D * 2;       // [DH][BM][128 B]
+    static constexpr int kv_bytes = BN * D * 2;      // one stage of K or V: [DH][BN][128 B]
+    static constexpr int p_bytes = BM * BN * 2;      // [BM][128 B]
+    static constexpr int q_off = 0;
+    static constexpr int k_off = q_off + q_bytes;
+    static constexpr int v_off = k_off + NS * kv_bytes;
+    static constexpr int p_off = v_off + NS * kv_bytes;
+    static constexpr int bar_off = p_off + 2 * p_bytes;
+    static constexpr int n_bars = 2 * NS + 9;
+    static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, last, bad flags
+    static constexpr int anc_off = misc_off + 16;                  // ancestor masks [64]
+    static constexpr int total = anc_off + kMaxTreeNodes * 8;
+    static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
+};
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
+                        const __grid_constant__ CUtensorMap tm_kn, const __grid_constant__ CUtensorMap tm_vn,
+                        const AttnArgs a) {
+    using S = TcSmem<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sQ = sm + S::q_off;
+    uint8_t *sK = sm + S::k_off;
+    uint8_t *sV = sm + S::v_off;
+    uint8_t *sP = sm + S::p_off;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sm + S::bar_off);
+    uint64_t *kv_full = bars;
+    uint64_t *kv_empty = bars + NS;
+    uint64_t *s_full = bars + 2 * NS;
+    uint64_t *s_empty = s_full + 2;
+    uint64_t *p_full = s_empty + 2;
+    uint64_t *o_full = p_full + 2;
+    uint64_t *mma_done = o_full + 2;
+    uint32_t *s_tmem = reinterpret_cast<uint32_t *>(sm + S::misc_off);
+    volatile int *s_abort = reinterpret_cast<volatile int *>(sm + S::misc_off + 4);
+    int *s_last = reinterpret_cast<int *>(sm + S::misc_off + 8);
+    bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 12);
+    uint64_t *s_anc = reinterpret_cast<uint64_t *>(sm + S::anc_off);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int rt = blockIdx.x;
+    const int split = blockIdx.y;
+    const int bg = blockIdx.z;
+    const int b = bg / a.Hkv;
+    const int g = bg % a.Hkv;
+    const bool tree_cta = (split == a.n_split - 1);
+    const int rows_here = min(BM, a.rows - rt * BM);
+    const int q_act = (rows_here + 31) >> 5;        // TMEM lane quadrants holding real rows
+
+    int L = __ldg(a.cache_len + b);
+    const bool cap_bad = (L < 0 || L + a.T > a.Lcap);
+    if (cap_bad) {
+        if (threadIdx.x == 0 && split == 0 && rt == 0 && g == 0) report(a.status, CLOVER_ERR_CAPACITY);
+        L = L < 0 ? 0 : a.Lcap - a.T;
+    }
+    const int chunk = (((L + a.n_split - 1) / a.n_split) + BN - 1) / BN * BN;
+    const int kbeg = min(L, split * chunk);
+    const int kend = min(L, kbeg + chunk);
+    const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
+    const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
+
+    // ---------------------------------------------------------------- setup
+    // The producer warp initialises the barriers and issues the first NS tile
+    // loads at once (the stages start empty), so they overlap the Q load and
+    // the TMEM allocation.
+    auto issue_tile = [&](int j) {
+        const int s = j % NS;
+        mbar_arrive_expect_tx(&kv_full[s], 2 * S::kv_bytes);
+        uint8_t *kdst = sK + s * S::kv_bytes;
+        uint8_t *vdst = sV + s * S::kv_bytes;
+        if (j < n_cache_tiles) {
+            const int key0 = kbeg + j * BN;
+#pragma unroll
+            for (int dh = 0; dh < S::DH; ++dh) {
+                tma_load_3d(kdst + dh * BN * 128, &tm_kc, &kv_full[s], dh * 64, key0, bg);
+                tma_load_3d(vdst + dh * BN * 128, &tm_vc, &kv_full[s], dh * 64, key0, bg);
+            }
+        } else {
+#pragma unroll
+            for (int dh = 0; dh < S::DH; ++dh) {
+                tma_load_3d(kdst + dh * BN * 128, &tm_kn, &kv_full[s], dh * 64, g, b * a.T);
+                tma_load_3d(vdst + dh * BN * 128, &tm_vn, &kv_full[s], dh * 64, g, b * a.T);
+            }
+        }
+    };
+    int producer_issued = 0;
+    if (warp == kProducerWarp) {
+        if (lane == 0) {
+            for (int i = 0; i < NS; ++i) {
+                mbar_init(&kv_full[i], 1);
+                mbar_init(&kv_empty[i], 1);
+            }
+            for (int i = 0; i < 2; ++i) {
+                mbar_init(&s_full[i], 1);
+                mbar_init(&s_empty[i], q_act);
+                mbar_init(&p_full[i], q_act);
+                mbar_init(&o_full[i], 1);
+            }
+            mbar_init(mma_done, 1);
+            *s_abort = 0;
+            *s_bad = false;
+            fence_barrier_init();
+            prefetch_tensormap(&tm_kc);
+            prefetch_tensormap(&tm_vc);
+            prefetch_tensormap(&tm_kn);
+            prefetch_tensormap(&tm_vn);
+            for (; producer_issued < min(NS, n_tiles); ++producer_issued) issue_tile(producer_issued);
+        }
+        __syncwarp();
+        if (tree_cta) tree_masks_warp(a.parent + (size_t)b * a.T, a.T, s_anc, s_bad);
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(s_tmem, kTmemCols);
+        tmem_relinquish();
+    }
+    if (warp < 4) {
+        // Q tile -> shared memory in the 128-byte-swizzled K-major layout; rows
+        // past this tile's real rows are zero.  All loads of a thread are
+        // issued before its stores.
+        const __nv_bfloat16 *q = static_cast<const __nv_bfloat16 *>(a.q);
+        constexpr int chunks_per_row = S::DH * 8;
+        constexpr int per_thread = BM * chunks_per_row / 128;
+        uint4 v[per_thread];
+#pragma unroll
+        for (int k = 0; k < per_thread; ++k) {
+            const int c = threadIdx.x + 128 * k;
+            const int r = c / chunks_per_row;
+            const int j = c % chunks_per_row;
+            const int R = rt * BM + r;
+            v[k] = make_uint4(0, 0, 0, 0);
+            if (r < rows_here) {
+                const int i = R / a.G;
+                const int h = g * a.G + (R % a.G);
+                v[k] = __ldg(reinterpret_cast<const uint4 *>(q + ((size_t)(b * a.T + i) * a.Hq + h) * D + (j >> 3) * 64 +
+                                                             (j & 7) * 8));
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < per_thread; ++k) {
+            const int c = threadIdx.x + 128 * k;
+            const int r = c / chunks_per_row;
+            const int j = c % chunks_per_row;
+            *reinterpret_cast<uint4 *>(sQ + (j >> 3) * (BM * 128) + r * 128 + (((j & 7) ^ (r & 7)) << 4)) = v[k];
+        }
+        fence_proxy_async_smem();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *s_tmem;
+    const uint32_t tS = tmem;                 // S tiles: columns [0, 2*BN)
+    const uint32_t tO = tmem + 2 * BN;        // O: columns [2*BN, 2*BN + D)
+
+    // ------------------------------------------------------ TMA producer warp
+    if (warp == kProducerWarp) {
+        if (lane == 0) {
+            for (int j = producer_issued; j < n_tiles; ++j) {
+                const int s = j % NS;
+                if (!mbar_wait(&kv_empty[s], ((j / NS) - 1) & 1, kWaitNs)) {
+                    *s_abort = 1;
+                    break;
+                }
+                if (*s_abort) break;
+                issue_tile(j);
+                producer_issued = j + 1;
+            }
+        }
+        __syncwarp();
+        // append the tree K/V to cache slots [L, L+T) (one CTA per sequence and head)
+        if (tree_cta && rt == 0 && !cap_bad) {
+            const __nv_bfloat16 *kn = static_cast<const __nv_bfloat16 *>(a.k_new);
+            const __nv_bfloat16 *vn = static_cast<const __nv_bfloat16 *>(a.v_new);
+            __nv_bfloat16 *kc = static_cast<__nv_bfloat16 *>(a.k_cache);
+            __nv_bfloat16 *vc = static_cast<__nv_bfloat16 *>(a.v_cache);
+            constexpr int per_row = D / 8;
+            for (int e = lane; e < a.T * per_row; e += 32) {
+                const int m = e / per_row;
+                const int c = (e % per_row) * 8;
+                const size_t src = ((size_t)(b * a.T + m) * a.Hkv + g) * D + c;
+                const size_t dst = ((size_t)(b * a.Hkv + g) * a.Lcap + L + m) * D + c;
+                *reinterpret_cast<uint4 *>(kc + dst) = __ldg(reinterpret_cast<const uint4 *>(kn + src));
+                *reinterpret_cast<uint4 *>(vc + dst) = __ldg(reinterpret_cast<const uint4 *>(vn + src));
+            }
+        }
+    }
+
+    // --------------------------------------------------------- MMA issuer warp
+    if (warp == kMmaWarp && lane == 0) {
+        const uint32_t idS = idesc_bf16(BM, BN, false, false);
+        const uint32_t idO = idesc_bf16(BM, D, false, true);
+        const uint32_t q_base = smem_u32(sQ);
+        bool ok = true;
+        auto issue_s = [&](int j) -> bool {
+            const int s = j % NS;
+            const int sb = j & 1;
+            if (!mbar_wait(&kv_full[s], (j / NS) & 1, kWaitNs)) return false;
+            if (j >= 2 && !mbar_wait(&s_empty[sb], ((j >> 1) - 1) & 1, kWaitNs)) return false;
+            tc_fence_after();
+            const uint32_t k_base = smem_u32(sK + s * S::kv_bytes);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k) {
+                const uint64_t ad = sdesc_sw128(q_base + (k >> 2) * (BM * 128) + (k & 3) * 32, 16, 1024);
+                const uint64_t bd = sdesc_sw128(k_base + (k >> 2) * (BN * 128) + (k & 3) * 32, 16, 1024);
+                mma_bf16(tS + sb * BN, ad, bd, idS, k > 0 ? 1u : 0u);
+            }
+            mma_commit(&s_full[sb]);
+            return true;
+        };
+        if (n_tiles > 0) ok = issue_s(0);
+        for (int j = 0; ok && j < n_tiles; ++j) {
+            if (*s_abort) {
+                ok = false;
+                break;
+            }
+            if (j + 1 < n_tiles && !(ok = issue_s(j + 1))) break;
+            const int s = j % NS;
+            const int sb = j & 1;
+            if (!mbar_wait(&p_full[sb], (j >> 1) & 1, kWaitNs)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t p_base = smem_u32(sP + sb * S::p_bytes);
+            const uint32_t v_base = smem_u32(sV + s * S::kv_bytes);
+#pragma unroll
+            for (int k = 0; k < BN / 16; ++k) {
+                const uint64_t ad = sdesc_sw128(p_base + k * 32, 16, 1024);
+                const uint64_t bd = sdesc_sw128(v_base + k * 16 * 128, BN * 128, 1024);
+                mma_bf16(tO, ad, bd, idO, (j > 0 || k > 0) ? 1u : 0u);
+            }
+            mma_commit(&o_full[sb]);
+            mma_commit(&kv_empty[s]);
+        }
+        if (!ok) *s_abort = 1;
+        mma_commit(mma_done);
+    }
+
+    // ------------------------------------------------------------ softmax warps
+    // Warp q owns TMEM lanes 32q.. = tile rows; it reads S, writes P, keeps the
+    // row's reference max m_ref and sum l, and rescales its O row in TMEM when
+    // m_ref has to move.
+    const int quad = warp & 3;
+    const bool softmax_warp = warp < 4 && quad < q_act;
+    const int r = quad * 32 + lane;
+    const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
+    float m_ref = -INFINITY, l_run = 0.f;
+    bool o_ready = false;
+    if (softmax_warp) {
+        const int R = rt * BM + r;
+        const int node = (r < rows_here) ? R / a.G : 0;
+        const uint64_t anc = tree_cta ? s_anc[node] : 0ull;
+        const float sc = a.scale_log2;
+        for (int j = 0; j < n_tiles; ++j) {
+            const int sb = j & 1;
+            const uint32_t ph = (j >> 1) & 1;
+            const bool got = __all_sync(0xffffffffu, mbar_wait(&s_full[sb], ph, kWaitNs));
+            if (!got || __any_sync(0xffffffffu, *s_abort != 0)) {
+                *s_abort = 1;
+                break;
+            }
+            tc_fence_after();
+            float sv[64];
+            tmem_ld32(tS + lane_base + sb * BN, *reinterpret_cast<float(*)[32]>(sv));
+            tmem_ld32(tS + lane_base + sb * BN + 32, *reinterpret_cast<float(*)[32]>(sv + 32));
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s_empty[sb]);
+
+            const bool tree_tile = (j == n_cache_tiles);
+            const int key0 = kbeg + j * BN;
+            const int n_valid = tree_tile ? a.T : min(BN, kend - key0);
+            if (tree_tile || n_valid < BN) {
+#pragma unroll
+                for (int c = 0; c < 64; ++c) {
+                    const bool ok = tree_tile ? ((anc >> c) & 1ull) != 0 : (c < n_valid);
+                    sv[c] = ok ? sv[c] : -INFINITY;
+                }
+            }
+            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int c = 0; c < 64; ++c) mx4[c & 3] = fmaxf(mx4[c & 3], sv[c]);
+            const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * sc;   // sc > 0
+
+            // move the reference max when this tile exceeds it by more than 2^8
+            const bool move = (mx > m_ref + kRescale);
+            if (j == 0) {
+                m_ref = mx;
+            } else if (__any_sync(0xffffffffu, move)) {
+                // O must hold every earlier tile before it is rescaled
+                const bool got_o =
+                    __all_sync(0xffffffffu, mbar_wait(&o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, kWaitNs));
+                if (!got_o) {
+                    *s_abort = 1;
+                    break;
+                }
+                tc_fence_after();
+                const float f = move ? ex2_approx(m_ref - mx) : 1.f;
+                l_run *= f;
+                if (move) m_ref = mx;
+#pragma unroll 1
+                for (int cc = 0; cc < D / 32; ++cc) {
+                    float x[32];
+                    tmem_ld32(tO + lane_base + cc * 32, x);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) x[c] *= f;
+                    tmem_st32(tO + lane_base + cc * 32, x);
+                }
+                tmem_wait_st();
+                tc_fence_before();
+            }
+            const float ref = (m_ref == -INFINITY) ? 0.f : m_ref;
+            float sum4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int c = 0; c < 64; ++c) {
+                sv[c] = ex2_approx(fmaf(sv[c], sc, -ref));
+                sum4[c & 3] += sv[c];
+            }
+            l_run += (sum4[0] + sum4[1]) + (sum4[2] + sum4[3]);
+            // value rows of keys past the valid ones may hold anything (even NaN): zero them
+            if (n_valid < BN) {
+                uint4 *vrows = reinterpret_cast<uint4 *>(sV + (j % NS) * S::kv_bytes);
+                const int n_zero = (BN - n_valid) * S::DH * 8;
+                for (int e = r; e < n_zero; e += q_act * 32) {
+                    const int row = n_valid + e / (S::DH * 8);
+                    const int rest = e % (S::DH * 8);
+                    vrows[(rest >> 3) * (BN * 8) + row * 8 + (rest & 7)] = make_uint4(0, 0, 0, 0);
+                }
+            }
+            // the P buffer of tile j was read by the P.V product of tile j-2
+            if (j >= 2) {
+                const bool free_p = __all_sync(0xffffffffu, mbar_wait(&o_full[sb], ((j >> 1) - 1) & 1, kWaitNs));
+                if (!free_p) {
+                    *s_abort = 1;
+                    break;
+                }
+            }
+            // P row r (64 keys = 128 bytes, eight swizzled 16-byte chunks)
+            uint8_t *prow = sP + sb * S::p_bytes + r * 128;
+#pragma unroll
+            for (int qd = 0; qd < 8; ++qd) {
+                uint4 w;
+                w.x = pack_bf16x2(sv[qd * 8 + 0], sv[qd * 8 + 1]);
+                w.y = pack_bf16x2(sv[qd * 8 + 2], sv[qd * 8 + 3]);
+                w.z = pack_bf16x2(sv[qd * 8 + 4], sv[qd * 8 + 5]);
+                w.w = pack_bf16x2(sv[qd * 8 + 6], sv[qd * 8 + 7]);
+                *reinterpret_cast<uint4 *>(prow + ((qd ^ (r & 7)) << 4)) = w;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&p_full[sb]);
+        }
+        // the last P.V product completes O
+        if (n_tiles > 0 && !__any_sync(0xffffffffu, *s_abort != 0)) {
+            const int jl = n_tiles - 1;
+            o_ready = __all_sync(0xffffffffu, mbar_wait(&o_full[jl & 1], (jl >> 1) & 1, kWaitNs));
+            if (!o_ready) *s_abort = 1;
+            tc_fence_after();
+        }
+    }
+
+    // ------------------------------------------------------------- epilogue
+    __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(a.out);
+    const bool row_ok = softmax_warp && r < rows_here;
+    const int slot_rows = a.slot_rows;
+    const size_t head_tile = (size_t)bg * a.row_tiles + rt;
+    const size_t slot = head_tile * a.n_split + split;
+    if (softmax_warp && o_ready) {
+        const float inv = (a.n_split == 1) ? 1.f / l_run : 1.f;
+        const int R = rt * BM + r;
+        const int i = row_ok ? R / a.G : 0;
+        const int h = row_ok ? g * a.G + (R % a.G) : 0;
+#pragma unroll 1
+        for (int cc = 0; cc < D / 32; ++cc) {
+            float x[32];
+            tmem_ld32(tO + lane_base + cc * 32, x);
+            tmem_wait_ld();
+            if (!row_ok) continue;
+            if (a.n_split == 1) {
+                __nv_bfloat16 *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D + cc * 32;
+#pragma unroll
+                for (int c = 0; c < 32; c += 8) {
+                    uint4 w;
+                    w.x = pack_bf16x2(x[c] * inv, x[c + 1] * inv);
+                    w.y = pack_bf16x2(x[c + 2] * inv, x[c + 3] * inv);
+                    w.z = pack_bf16x2(x[c + 4] * inv, x[c + 5] * inv);
+                    w.w = pack_bf16x2(x[c + 6] * inv, x[c + 7] * inv);
+                    *reinterpret_cast<uint4 *>(dst + c) = w;
+                }
+            } else {
+                float *po = a.part_o + (slot * slot_rows + r) * D + cc * 32;
+#pragma unroll
+                for (int c = 0; c < 32; c += 4)
+                    *reinterpret_cast<float4 *>(po + c) = make_float4(x[c], x[c + 1], x[c + 2], x[c + 3]);
+            }
+        }
+    } else if (row_ok && a.n_split > 1) {
+        // no tiles here (or an abort): an empty partial
+        float *po = a.part_o + (slot * slot_rows + r) * D;
+        for (int c = 0; c < D; c += 4) *reinterpret_cast<float4 *>(po + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    if (row_ok && a.n_split > 1) {
+        a.part_ml[(slot * slot_rows + r) * 2] = m_ref;
+        a.part_ml[(slot * slot_rows + r) * 2 + 1] = l_run;
+    }
+
+    // every TMEM access and MMA is finished before TMEM is released
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        if (lane == 0) mbar_wait(mma_done, 0, kWaitNs);
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+    if (*s_abort) {
+        // wind down: report and wait (bounded) for the loads still in flight;
+        // still take part in the split merge so the workspace counters reset
+        if (threadIdx.x == 0) report(a.status, CLOVER_ERR_TIMEOUT);
+        if (warp == kProducerWarp && lane == 0)
+            for (int j = max(0, producer_issued - NS); j < producer_issued; ++j)
+                mbar_wait(&kv_full[j % NS], (j / NS) & 1, kWaitNs);
+    }
+    if (tree_cta && rt == 0 && threadIdx.x == 0 && *s_bad) report(a.status, CLOVER_ERR_BAD_TREE);
+    if (a.n_split == 1) return;
+
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const unsigned prev = atomicAdd(a.counters + head_tile, 1u);
+        *s_last = (prev == (unsigned)a.n_split - 1u);
+    }
+    __syncthreads();
+    if (!*s_last) return;
+    __threadfence();
+
+    // last CTA of this (sequence, head, row tile): merge the n_split partials
+    const float *po_all = a.part_o + head_tile * a.n_split * slot_rows * D;
+    const float *pml_all = a.part_ml + head_tile * a.n_split * slot_rows * 2;
+    for (int e = threadIdx.x; e < rows_here * (D / 4); e += kThreads) {
+        const int rr = e / (D / 4);
+        const int c4 = (e % (D / 4)) * 4;
+        float M = -INFINITY;
+        for (int sp = 0; sp < a.n_split; ++sp) M = fmaxf(M, __ldcg(pml_all + ((size_t)sp * slot_rows + rr) * 2));
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        float lsum = 0.f;
+        for (int sp = 0; sp < a.n_split; ++sp) {
+            const float ms = __ldcg(pml_all + ((size_t)sp * slot_rows + rr) * 2);
+            const float ls = __ldcg(pml_all + ((size_t)sp * slot_rows + rr) * 2 + 1);
+            const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+            lsum += w * ls;
+            const float4 x = __ldcg(reinterpret_cast<const float4 *>(po_all + ((size_t)sp * slot_rows + rr) * D + c4));
+            acc.x = fmaf(w, x.x, acc.x);
+            acc.y = fmaf(w, x.y, acc.y);
+            acc.z = fmaf(w, x.z, acc.z);
+            acc.w = fmaf(w, x.w, acc.w);
+        }
+        const float inv = 1.f / lsum;
+        const int R = rt * BM + rr;
+        const int i = R / a.G;
+        const int h = g * a.G + (R % a.G);
+        uint2 w2;
+        w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+        w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+        *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c4) = w2;
+    }
+    if (threadIdx.x == 0) a.counters[head_tile] = 0u;   // ready for the next call
+}
+
+template <int D>
+cudaError_t launch(const AttnArgs &a, cudaStream_t stream) {
+    CUtensorMap kc, vc, kn, vn;
+    const uint64_t e = 2;
+    if (!make_tmap_bf16_3d(&kc, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
+        !make_tmap_bf16_3d(&vc, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
+        !make_tmap_bf16_3d(&kn, a.k_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) ||
+        !make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN))
+        return cudaErrorInvalidValue;
+    static unsigned char done[64];
+    auto kernel = tree_attn_tc_kernel<D>;
+    cudaError_t err = ensure_smem_attr(kernel, TcSmem<D>::alloc, done);
+    if (err != cudaSuccess) return err;
+    dim3 grid(a.row_tiles, a.n_split, a.B * a.Hkv);
+    kernel<<<grid, kThreads, TcSmem<D>::alloc, stream>>>(kc, vc, kn, vn, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int tc_row_tile() { return BM; }
+
+cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream) {
+    return a.D == 64 ? launch<64>(a, stream) : launch<128>(a, stream);
+}
+
+}  // namespace clover

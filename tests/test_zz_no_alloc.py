@@ -79,17 +79,17 @@ def test_noalloc_rejects_scratch_beyond_its_buffer():
     but the check lives with the GPU test of the entry point."""
     lib = _lib.load(build_if_missing=True)
     shape = None
-    for Hkv in (150, 300, 600, 1200, 2400):
-        for Lcap in (4096, 65536):
-            if lib.clover_verify_attn_workspace_size(1, 64, Hkv, Hkv, 128, Lcap, pkg.BF16) > _lib.NOALLOC_SCRATCH_BYTES:
-                shape = (Hkv, Lcap)
-                break
-        if shape:
-            break
+    for dt in (pkg.BF16, pkg.F32):
+        for Hkv in (1, 2, 3, 4, 150, 300, 600):
+            for G in (1, 2):
+                for Lcap in (4096, 65536):
+                    need = lib.clover_verify_attn_workspace_size(1, 64, G * Hkv, Hkv, 128, Lcap, dt)
+                    if need > _lib.NOALLOC_SCRATCH_BYTES and shape is None:
+                        shape = (G * Hkv, Hkv, Lcap, dt)
     assert shape is not None
-    Hkv, Lcap = shape
+    Hq, Hkv, Lcap, dt = shape
     P = ctypes.c_void_p
     code = lib.clover_verify_attn_noalloc(P(256), P(256), P(256), P(256), P(256), P(256), P(256), P(256),
-                                          1, 64, Hkv, Hkv, 128, Lcap, pkg.BF16, 0.0, None, None)
+                                          1, 64, Hq, Hkv, 128, Lcap, dt, 0.0, None, None)
     assert code == pkg.api.ERR_SCRATCH_LIMIT
     assert b"static buffer" in lib.clover_status_string(code)
