@@ -73,8 +73,9 @@ CLOVER_API const char *clover_status_string(int status);
 
 /*
  * Bytes of device workspace clover_verify_attn needs for these sizes
- * (split-KV partial results and per-head arrival counters).  Returns 0 when
- * the sizes are outside the limits.
+ * (split-KV partial results and per-head arrival counters).  0 when none is
+ * needed (the bf16 tensor-core path merges its splits on chip) and when the
+ * sizes are outside the limits.
  */
 CLOVER_API size_t clover_verify_attn_workspace_size(int B, int T, int Hq, int Hkv, int D, int Lcap,
                                          clover_dtype dtype);

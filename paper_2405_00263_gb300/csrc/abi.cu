@@ -50,9 +50,9 @@ clover_status check_attn_sizes(int B, int T, int Hq, int Hkv, int D, int Lcap, i
 }
 
 // Kernel choice, split count and workspace layout for one shape.  bf16 with at
-// least kTcMinRows query rows per KV head runs on the tensor cores with one CTA
-// per SM (splits chosen so that one wave fills the SMs); everything else runs
-// on the FMA kernel with two CTAs per SM.
+// least kTcMinRows query rows per KV head runs on the tensor cores (one CTA per
+// SM, splits merged on chip, no workspace); everything else runs on the FMA
+// kernel with two CTAs per SM and merges splits through the workspace.
 AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
     AttnPlan p;
     const int G = Hq / Hkv;
@@ -62,11 +62,15 @@ AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
     int n;
     p.tc = (dtype == CLOVER_BF16) && rows >= kTcMinRows;
     if (p.tc) {
+        // the tensor-core kernel picks its split count at launch (one wave of
+        // thread-block clusters) and merges splits in distributed shared memory:
+        // it needs no workspace
         p.row_tile = tc_row_tile();
         p.row_tiles = (rows + p.row_tile - 1) / p.row_tile;
         p.slot_rows = rows < p.row_tile ? rows : p.row_tile;
-        const long base = Bp * Hkv * p.row_tiles;
-        n = base >= kSms ? 1 : (int)(kSms / base);
+        p.n_split = 1;
+        p.o_bytes = p.ml_bytes = p.counter_bytes = p.total = 0;
+        return p;
     } else {
         p.row_tile = fma_row_tile();
         p.row_tiles = (rows + p.row_tile - 1) / p.row_tile;

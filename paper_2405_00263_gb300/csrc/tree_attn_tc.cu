@@ -16,11 +16,15 @@
 // a tile's max exceeds it by more than 2^8, so O is rarely rescaled.
 // Warp roles (192 threads): warp q in 0-3 runs the softmax, rescales and the
 // epilogue of TMEM lanes 32q.. (the lanes warp q may access); warp 4 issues the
-// TMA loads of K/V tiles (4-stage ring, 128-byte swizzle) and appends the tree
-// K/V to the cache; warp 5 allocates TMEM and issues the MMAs from one thread.
+// TMA loads of Q and of the K/V tiles (4-stage ring, 128-byte swizzle) and
+// appends the tree K/V to the cache; warp 5 allocates TMEM and issues the MMAs
+// from one thread.
 // The split that owns the last cache range also takes the tile of T tree keys
-// (read from k_new/v_new) under the ancestor bitmask.  Splits are merged by the
-// CTA that arrives last at a per-head counter, as in the FMA kernel.
+// (read from k_new/v_new) under the ancestor bitmask.  The n_split CTAs of a
+// (sequence, head, row tile) form one thread-block cluster: each leaves its
+// partial (m, l, O) in its own shared memory and each merges a share of the
+// rows by reading all partials over distributed shared memory, so no partial
+// result touches global memory.
 // Every mbarrier wait is bounded; on a timeout the CTA reports
 // CLOVER_ERR_TIMEOUT, winds down, waits (bounded) for its copies in flight and
 // frees its TMEM.
@@ -39,6 +43,7 @@ constexpr int NS = 4;                   // K/V pipeline stages
 constexpr int kProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kThreads = 192;
+constexpr int kMaxCluster = 8;          // portable cluster size: splits per head
 constexpr uint32_t kTmemCols = 256;     // S: 2 x 64 columns, O: D columns
 constexpr float kRescale = 8.0f;        // move the reference max only past 2^8 growth
 constexpr uint64_t kWaitNs = 500ull * 1000 * 1000;   // 0.5 s per wait
@@ -54,11 +59,17 @@ struct TcSmem {
     static constexpr int v_off = k_off + NS * kv_bytes;
     static constexpr int p_off = v_off + NS * kv_bytes;
     static constexpr int bar_off = p_off + 2 * p_bytes;
-    static constexpr int n_bars = 2 * NS + 9;
-    static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, last, bad flags
+    static constexpr int n_bars = 2 * NS + 12;
+    static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad flags
     static constexpr int anc_off = misc_off + 16;                  // ancestor masks [64]
-    static constexpr int total = anc_off + kMaxTreeNodes * 8;
+    static constexpr int mw_off = anc_off + kMaxTreeNodes * 8;     // merge weights [BM][kMaxCluster + 1]
+    static constexpr int total = mw_off + BM * (kMaxCluster + 1) * 4;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
+    // after the key loop the K/V ring holds this CTA's partial O (fp32, rows padded
+    // to D + 4 floats) and the P area its (m, l) pairs
+    static constexpr int po_stride = D + 4;
+    static_assert(BM * po_stride * 4 <= 2 * NS * kv_bytes, "partial O must fit in the K/V ring");
+    static_assert(BM * 8 <= 2 * p_bytes, "partial (m, l) must fit in the P area");
 };
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -70,7 +81,7 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                         const __grid_constant__ CUtensorMap tm_kn, const __grid_constant__ CUtensorMap tm_vn,
-                        const AttnArgs a) {
+                        const __grid_constant__ CUtensorMap tm_q, const AttnArgs a) {
     using S = TcSmem<D>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -86,11 +97,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t *p_full = s_empty + 2;
     uint64_t *o_full = p_full + 2;
     uint64_t *mma_done = o_full + 2;
+    uint64_t *q_full = mma_done + 1;
+    uint64_t *m_ready = q_full + 1;           // partials of all cluster CTAs are in place
+    uint64_t *m_done = m_ready + 1;           // all cluster CTAs have read this CTA's partial
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(sm + S::misc_off);
     volatile int *s_abort = reinterpret_cast<volatile int *>(sm + S::misc_off + 4);
-    int *s_last = reinterpret_cast<int *>(sm + S::misc_off + 8);
-    bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 12);
+    bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 8);
     uint64_t *s_anc = reinterpret_cast<uint64_t *>(sm + S::anc_off);
+    float *merge_w = reinterpret_cast<float *>(sm + S::mw_off);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -99,7 +113,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int bg = blockIdx.z;
     const int b = bg / a.Hkv;
     const int g = bg % a.Hkv;
-    const bool tree_cta = (split == a.n_split - 1);
+    const int n_split = a.n_split;
+    const bool tree_cta = (split == n_split - 1);
     const int rows_here = min(BM, a.rows - rt * BM);
     const int q_act = (rows_here + 31) >> 5;        // TMEM lane quadrants holding real rows
 
@@ -109,16 +124,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (threadIdx.x == 0 && split == 0 && rt == 0 && g == 0) report(a.status, CLOVER_ERR_CAPACITY);
         L = L < 0 ? 0 : a.Lcap - a.T;
     }
-    const int chunk = (((L + a.n_split - 1) / a.n_split) + BN - 1) / BN * BN;
+    const int chunk = (((L + n_split - 1) / n_split) + BN - 1) / BN * BN;
     const int kbeg = min(L, split * chunk);
     const int kend = min(L, kbeg + chunk);
     const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
     const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
 
     // ---------------------------------------------------------------- setup
-    // The producer warp initialises the barriers and issues the first NS tile
-    // loads at once (the stages start empty), so they overlap the Q load and
-    // the TMEM allocation.
+    // The producer warp initialises the barriers and issues the Q load and the
+    // first NS tile loads at once (the stages start empty), so they overlap the
+    // TMEM allocation.
     auto issue_tile = [&](int j) {
         const int s = j % NS;
         mbar_arrive_expect_tx(&kv_full[s], 2 * S::kv_bytes);
@@ -153,6 +168,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_init(&o_full[i], 1);
             }
             mbar_init(mma_done, 1);
+            mbar_init(q_full, 1);
+            mbar_init(m_ready, n_split);
+            mbar_init(m_done, n_split);
             *s_abort = 0;
             *s_bad = false;
             fence_barrier_init();
@@ -160,6 +178,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             prefetch_tensormap(&tm_vc);
             prefetch_tensormap(&tm_kn);
             prefetch_tensormap(&tm_vn);
+            if (a.q_box_nodes > 0) {
+                // Q rows (node, head in group) of this tile: box (64 d, G heads, q_box_nodes nodes)
+                mbar_arrive_expect_tx(q_full, S::DH * a.G * a.q_box_nodes * 128);
+#pragma unroll
+                for (int dh = 0; dh < S::DH; ++dh)
+                    tma_load_3d(sQ + dh * (BM * 128), &tm_q, q_full, dh * 64, g * a.G, b * a.T + rt * a.q_box_nodes);
+            } else {
+                mbar_arrive(q_full);
+            }
             for (; producer_issued < min(NS, n_tiles); ++producer_issued) issue_tile(producer_issued);
         }
         __syncwarp();
@@ -169,10 +196,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_alloc(s_tmem, kTmemCols);
         tmem_relinquish();
     }
-    if (warp < 4) {
-        // Q tile -> shared memory in the 128-byte-swizzled K-major layout; rows
-        // past this tile's real rows are zero.  All loads of a thread are
-        // issued before its stores.
+    if (warp < 4 && a.q_box_nodes == 0) {
+        // Q tile by threads (group sizes that do not divide the tile): 128-byte
+        // swizzled K-major layout, rows past this tile's real rows zero
         const __nv_bfloat16 *q = static_cast<const __nv_bfloat16 *>(a.q);
         constexpr int chunks_per_row = S::DH * 8;
         constexpr int per_thread = BM * chunks_per_row / 128;
@@ -201,7 +227,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_proxy_async_smem();
     }
     tc_fence_before();
-    __syncthreads();
+    if (n_split > 1) cluster_sync_all();      // every CTA's barriers exist before any remote arrive
+    else __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *s_tmem;
     const uint32_t tS = tmem;                 // S tiles: columns [0, 2*BN)
@@ -245,7 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t idS = idesc_bf16(BM, BN, false, false);
         const uint32_t idO = idesc_bf16(BM, D, false, true);
         const uint32_t q_base = smem_u32(sQ);
-        bool ok = true;
+        bool ok = mbar_wait(q_full, 0, kWaitNs);
         auto issue_s = [&](int j) -> bool {
             const int s = j % NS;
             const int sb = j & 1;
@@ -262,7 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_commit(&s_full[sb]);
             return true;
         };
-        if (n_tiles > 0) ok = issue_s(0);
+        if (ok && n_tiles > 0) ok = issue_s(0);
         for (int j = 0; ok && j < n_tiles; ++j) {
             if (*s_abort) {
                 ok = false;
@@ -417,23 +444,37 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // ------------------------------------------------------------- epilogue
+    tc_fence_before();
+    __syncthreads();                          // every role is out of its key loop
+    if (*s_abort && warp == kProducerWarp && lane == 0) {
+        // wind down: wait (bounded) for the loads still in flight before the
+        // K/V ring is reused below
+        for (int j = max(0, producer_issued - NS); j < producer_issued; ++j)
+            mbar_wait(&kv_full[j % NS], (j / NS) & 1, kWaitNs);
+    }
+    __syncthreads();
+    tc_fence_after();
     __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(a.out);
     const bool row_ok = softmax_warp && r < rows_here;
-    const int slot_rows = a.slot_rows;
-    const size_t head_tile = (size_t)bg * a.row_tiles + rt;
-    const size_t slot = head_tile * a.n_split + split;
-    if (softmax_warp && o_ready) {
-        const float inv = (a.n_split == 1) ? 1.f / l_run : 1.f;
+    float *part_o = reinterpret_cast<float *>(sK);   // [BM][D + 4] fp32, this CTA's partial
+    float2 *part_ml = reinterpret_cast<float2 *>(sP); // [BM] (m, l)
+    if (softmax_warp) {
         const int R = rt * BM + r;
         const int i = row_ok ? R / a.G : 0;
         const int h = row_ok ? g * a.G + (R % a.G) : 0;
+        const float inv = (n_split == 1 && o_ready) ? 1.f / l_run : 1.f;
 #pragma unroll 1
         for (int cc = 0; cc < D / 32; ++cc) {
             float x[32];
-            tmem_ld32(tO + lane_base + cc * 32, x);
-            tmem_wait_ld();
+            if (o_ready) {
+                tmem_ld32(tO + lane_base + cc * 32, x);
+                tmem_wait_ld();
+            } else {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) x[c] = 0.f;
+            }
             if (!row_ok) continue;
-            if (a.n_split == 1) {
+            if (n_split == 1) {
                 __nv_bfloat16 *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D + cc * 32;
 #pragma unroll
                 for (int c = 0; c < 32; c += 8) {
@@ -445,20 +486,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     *reinterpret_cast<uint4 *>(dst + c) = w;
                 }
             } else {
-                float *po = a.part_o + (slot * slot_rows + r) * D + cc * 32;
+                float *po = part_o + r * S::po_stride + cc * 32;
 #pragma unroll
                 for (int c = 0; c < 32; c += 4)
                     *reinterpret_cast<float4 *>(po + c) = make_float4(x[c], x[c + 1], x[c + 2], x[c + 3]);
             }
         }
-    } else if (row_ok && a.n_split > 1) {
-        // no tiles here (or an abort): an empty partial
-        float *po = a.part_o + (slot * slot_rows + r) * D;
-        for (int c = 0; c < D; c += 4) *reinterpret_cast<float4 *>(po + c) = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    if (row_ok && a.n_split > 1) {
-        a.part_ml[(slot * slot_rows + r) * 2] = m_ref;
-        a.part_ml[(slot * slot_rows + r) * 2 + 1] = l_run;
+        if (row_ok) part_ml[r] = make_float2(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f);
     }
 
     // every TMEM access and MMA is finished before TMEM is released
@@ -470,75 +504,162 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
-    if (*s_abort) {
-        // wind down: report and wait (bounded) for the loads still in flight;
-        // still take part in the split merge so the workspace counters reset
-        if (threadIdx.x == 0) report(a.status, CLOVER_ERR_TIMEOUT);
-        if (warp == kProducerWarp && lane == 0)
-            for (int j = max(0, producer_issued - NS); j < producer_issued; ++j)
-                mbar_wait(&kv_full[j % NS], (j / NS) & 1, kWaitNs);
-    }
     if (tree_cta && rt == 0 && threadIdx.x == 0 && *s_bad) report(a.status, CLOVER_ERR_BAD_TREE);
-    if (a.n_split == 1) return;
-
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        const unsigned prev = atomicAdd(a.counters + head_tile, 1u);
-        *s_last = (prev == (unsigned)a.n_split - 1u);
-    }
-    __syncthreads();
-    if (!*s_last) return;
-    __threadfence();
-
-    // last CTA of this (sequence, head, row tile): merge the n_split partials
-    const float *po_all = a.part_o + head_tile * a.n_split * slot_rows * D;
-    const float *pml_all = a.part_ml + head_tile * a.n_split * slot_rows * 2;
-    for (int e = threadIdx.x; e < rows_here * (D / 4); e += kThreads) {
-        const int rr = e / (D / 4);
-        const int c4 = (e % (D / 4)) * 4;
-        float M = -INFINITY;
-        for (int sp = 0; sp < a.n_split; ++sp) M = fmaxf(M, __ldcg(pml_all + ((size_t)sp * slot_rows + rr) * 2));
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        float lsum = 0.f;
-        for (int sp = 0; sp < a.n_split; ++sp) {
-            const float ms = __ldcg(pml_all + ((size_t)sp * slot_rows + rr) * 2);
-            const float ls = __ldcg(pml_all + ((size_t)sp * slot_rows + rr) * 2 + 1);
-            const float w = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-            lsum += w * ls;
-            const float4 x = __ldcg(reinterpret_cast<const float4 *>(po_all + ((size_t)sp * slot_rows + rr) * D + c4));
-            acc.x = fmaf(w, x.x, acc.x);
-            acc.y = fmaf(w, x.y, acc.y);
-            acc.z = fmaf(w, x.z, acc.z);
-            acc.w = fmaf(w, x.w, acc.w);
+    if (n_split > 1) {
+        // -------------------------------------------- split merge over DSMEM
+        // announce this CTA's partial to every CTA of the cluster
+        if (threadIdx.x < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_ready), threadIdx.x));
+        const bool ready = __syncthreads_and(mbar_wait_cluster(m_ready, 0, kWaitNs));
+        if (ready) {
+            // this CTA merges rows [r0, r1) of the tile
+            const int per = (rows_here + n_split - 1) / n_split;
+            const int r0 = split * per;
+            const int r1 = min(rows_here, r0 + per);
+            const uint32_t ml_base = smem_u32(part_ml);
+            const uint32_t o_base = smem_u32(part_o);
+            for (int rr = r0 + threadIdx.x; rr < r1; rr += kThreads) {
+                float m[kMaxCluster], l[kMaxCluster];
+                float M = -INFINITY;
+                for (int k = 0; k < n_split; ++k) {
+                    const float2 v = ld_dsmem_f2(mapa_shared(ml_base + rr * 8, k));
+                    m[k] = v.x;
+                    l[k] = v.y;
+                    M = fmaxf(M, v.x);
+                }
+                float lsum = 0.f;
+                for (int k = 0; k < n_split; ++k) {
+                    const float w = (m[k] == -INFINITY) ? 0.f : exp2f(m[k] - M);
+                    merge_w[rr * (kMaxCluster + 1) + k] = w;
+                    lsum += w * l[k];
+                }
+                merge_w[rr * (kMaxCluster + 1) + kMaxCluster] = 1.f / lsum;
+            }
+            __syncthreads();
+            for (int e = threadIdx.x; e < (r1 - r0) * (D / 4); e += kThreads) {
+                const int rr = r0 + e / (D / 4);
+                const int c4 = (e % (D / 4)) * 4;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int k = 0; k < n_split; ++k) {
+                    const float w = merge_w[rr * (kMaxCluster + 1) + k];
+                    const float4 x = ld_dsmem_f4(mapa_shared(o_base + (rr * S::po_stride + c4) * 4, k));
+                    acc.x = fmaf(w, x.x, acc.x);
+                    acc.y = fmaf(w, x.y, acc.y);
+                    acc.z = fmaf(w, x.z, acc.z);
+                    acc.w = fmaf(w, x.w, acc.w);
+                }
+                const float inv = merge_w[rr * (kMaxCluster + 1) + kMaxCluster];
+                const int R = rt * BM + rr;
+                const int i = R / a.G;
+                const int h = g * a.G + (R % a.G);
+                uint2 w2;
+                w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+                w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+                *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c4) = w2;
+            }
+        } else {
+            *s_abort = 1;
         }
-        const float inv = 1.f / lsum;
-        const int R = rt * BM + rr;
-        const int i = R / a.G;
-        const int h = g * a.G + (R % a.G);
-        uint2 w2;
-        w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-        w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-        *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c4) = w2;
+        // this CTA has finished reading every partial; wait until every CTA
+        // has finished reading this one's before its shared memory goes away
+        __syncthreads();
+        if (threadIdx.x < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_done), threadIdx.x));
+        if (!__syncthreads_and(mbar_wait_cluster(m_done, 0, kWaitNs))) *s_abort = 1;
     }
-    if (threadIdx.x == 0) a.counters[head_tile] = 0u;   // ready for the next call
+    if (*s_abort && threadIdx.x == 0) report(a.status, CLOVER_ERR_TIMEOUT);
+}
+
+struct TcLaunchCache {
+    int sms = 0;
+    int max_clusters[kMaxCluster + 1] = {0};   // co-resident clusters per cluster size (0: not queried)
+};
+
+template <int D>
+int max_active_clusters(int n, int dev, TcLaunchCache &cache) {
+    if (cache.max_clusters[n] == 0) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(1, n, n);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = TcSmem<D>::alloc;
+        cudaLaunchAttribute attr;
+        attr.id = cudaLaunchAttributeClusterDimension;
+        attr.val.clusterDim.x = 1;
+        attr.val.clusterDim.y = n;
+        attr.val.clusterDim.z = 1;
+        cfg.attrs = &attr;
+        cfg.numAttrs = 1;
+        int num = 0;
+        if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D>, &cfg) != cudaSuccess) {
+            cudaGetLastError();
+            num = -1;
+        }
+        cache.max_clusters[n] = num > 0 ? num : -1;
+    }
+    (void)dev;
+    return cache.max_clusters[n];
 }
 
 template <int D>
-cudaError_t launch(const AttnArgs &a, cudaStream_t stream) {
-    CUtensorMap kc, vc, kn, vn;
+cudaError_t launch(AttnArgs a, cudaStream_t stream) {
+    static unsigned char done[64];
+    static TcLaunchCache caches[64];
+    auto kernel = tree_attn_tc_kernel<D>;
+    cudaError_t err = ensure_smem_attr(kernel, TcSmem<D>::alloc, done);
+    if (err != cudaSuccess) return err;
+    int dev = 0;
+    if ((err = cudaGetDevice(&dev)) != cudaSuccess) return err;
+    TcLaunchCache &cache = caches[dev < 64 ? dev : 63];
+    if (cache.sms == 0 && (err = cudaDeviceGetAttribute(&cache.sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return err;
+
+    // splits per head: as many as fill the SMs in one wave of clusters
+    const long base = (long)a.B * a.Hkv * a.row_tiles;
+    const int by_len = (a.Lcap + 255) / 256;
+    int n = 1;
+    for (int c = kMaxCluster; c >= 2; --c) {
+        if (c > by_len || base * c > cache.sms) continue;
+        if (max_active_clusters<D>(c, dev, cache) >= base) {
+            n = c;
+            break;
+        }
+    }
+    a.n_split = n;
+
+    // Q tile by TMA when a tile holds whole nodes: box (64 d, G heads, nodes)
+    const int G = a.G;
+    int box_nodes = 0;
+    if (a.rows <= BM) box_nodes = a.T;
+    else if (BM % G == 0) box_nodes = BM / G;
+    if (G > 256 || box_nodes > 256) box_nodes = 0;
+    a.q_box_nodes = box_nodes;
+
+    CUtensorMap kc, vc, kn, vn, qm;
     const uint64_t e = 2;
     if (!make_tmap_bf16_3d(&kc, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
         !make_tmap_bf16_3d(&vc, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
         !make_tmap_bf16_3d(&kn, a.k_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) ||
         !make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN))
         return cudaErrorInvalidValue;
-    static unsigned char done[64];
-    auto kernel = tree_attn_tc_kernel<D>;
-    cudaError_t err = ensure_smem_attr(kernel, TcSmem<D>::alloc, done);
+    if (box_nodes > 0) {
+        if (!make_tmap_bf16_3d(&qm, a.q, D, a.Hq, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hq * D * e, 64, G, box_nodes))
+            return cudaErrorInvalidValue;
+    } else {
+        qm = kn;   // unused
+    }
+
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.row_tiles, n, a.B * a.Hkv);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = TcSmem<D>::alloc;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 1;
+    attr.val.clusterDim.y = n;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = n > 1 ? 1 : 0;
+    err = cudaLaunchKernelEx(&cfg, kernel, kc, vc, kn, vn, qm, a);
     if (err != cudaSuccess) return err;
-    dim3 grid(a.row_tiles, a.n_split, a.B * a.Hkv);
-    kernel<<<grid, kThreads, TcSmem<D>::alloc, stream>>>(kc, vc, kn, vn, a);
     return cudaGetLastError();
 }
 

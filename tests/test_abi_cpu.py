@@ -46,8 +46,9 @@ def test_version_and_status_strings(lib):
 def test_workspace_sizes(lib):
     ws = lib.clover_verify_attn_workspace_size
     assert ws(1, 16, 8, 8, 64, 192, 0) == 0              # short cache: one split, no workspace
-    big = ws(1, 64, 32, 32, 128, 4160, 1)
+    big = ws(1, 64, 32, 32, 128, 4160, 0)                # fp32: CUDA-core split-KV merge
     assert big > 0 and big % 256 == 0
+    assert ws(1, 64, 32, 32, 128, 4160, 1) == 0          # bf16: tensor-core path merges on chip
     assert ws(1, 65, 8, 8, 64, 192, 0) == 0              # T > 64 unsupported
     assert ws(1, 16, 8, 8, 96, 192, 0) == 0              # D = 96 unsupported
     assert ws(1, 16, 6, 4, 64, 192, 0) == 0              # Hq not a multiple of Hkv
@@ -78,7 +79,8 @@ def test_attn_host_validation(lib):
     assert _attn(lib, out=8) == 1                          # misaligned
     assert _attn(lib, scale=float("nan")) == 1
     assert _attn(lib, B=0) == 0                            # empty batch: nothing to do
-    assert _attn(lib, B=1, T=64, Hq=32, Hkv=32, D=128, Lcap=8192, ws=None, wsb=0) == 1   # workspace missing
+    # fp32 needs a split-KV workspace at this size: refused before launch when it is missing
+    assert _attn(lib, B=1, T=64, Hq=32, Hkv=32, D=128, Lcap=8192, dt=0, ws=None, wsb=0) == 1
 
 
 def test_accept_and_compact_host_validation(lib):
