@@ -186,11 +186,14 @@ def clover_kv_compact(k_cache, v_cache, cache_len, path, accept_len, new_cache_l
 class VerifyStep:
     """Device buffers for repeated verification steps of one shape.
 
-    Owns the two zero-initialised workspaces and the output tensors; ``run``
-    issues the three library calls in order on one stream.
+    Owns the two zero-initialised workspaces and the output tensors.  ``run``
+    issues the three library calls: the attention on ``stream`` and, at the
+    same time, the argmax/acceptance walk on a side stream (the two read
+    disjoint inputs); the compaction follows on ``stream`` once both are done.
+    With ``concurrent=False`` all three run in order on ``stream``.
     """
 
-    def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda"):
+    def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda", concurrent=True):
         self.shape = dict(B=B, T=T, Hq=Hq, Hkv=Hkv, D=D, Lcap=Lcap, V=V)
         self.dtype = dtype
         dev = torch.device(device)
@@ -207,12 +210,59 @@ class VerifyStep:
         self.new_cache_len = torch.empty((B,), **i32)
         self.src_index = torch.empty((B, T), **i32)
         self.status = torch.zeros((1,), **i32)
+        # the accept call gets its own status word so that the two concurrent
+        # calls never update one word at the same time from two streams
+        self.status_accept = torch.zeros((1,), **i32)
+        self.side = torch.cuda.Stream(device=dev) if concurrent else None
+        self._fork = torch.cuda.Event() if concurrent else None
+        self._join = torch.cuda.Event() if concurrent else None
+
+    def device_status(self) -> int:
+        return int(self.status.item()) | int(self.status_accept.item())
+
+    def clear_status(self):
+        self.status.zero_()
+        self.status_accept.zero_()
 
     def run(self, q, k_new, v_new, k_cache, v_cache, cache_len, parent, cand, logits, scale=0.0,
-            stream=None):
-        clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
-                           workspace=self.ws_attn, status=self.status, stream=stream)
-        clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
-                             self.ws_accept, status=self.status, stream=stream)
+            stream=None, events=None):
+        """One step.  ``events`` (optional, four CUDA events) brackets the
+        attention (0-1) and the compaction (2-3) on ``stream``; the accept call
+        is bracketed by ``events[4:6]`` on the side stream when given."""
+        stream = stream if stream is not None else torch.cuda.current_stream()
+        if self.side is None:
+            if events:
+                events[0].record(stream)
+            clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
+                               workspace=self.ws_attn, status=self.status, stream=stream)
+            if events:
+                events[1].record(stream)
+                if len(events) > 5:
+                    events[4].record(stream)
+            clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
+                                 self.ws_accept, status=self.status_accept, stream=stream)
+            if events and len(events) > 5:
+                events[5].record(stream)
+        else:
+            self._fork.record(stream)
+            self.side.wait_event(self._fork)
+            if events:
+                events[0].record(stream)
+            clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
+                               workspace=self.ws_attn, status=self.status, stream=stream)
+            if events:
+                events[1].record(stream)
+                if len(events) > 5:
+                    events[4].record(self.side)
+            clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
+                                 self.ws_accept, status=self.status_accept, stream=self.side)
+            if events and len(events) > 5:
+                events[5].record(self.side)
+            self._join.record(self.side)
+            stream.wait_event(self._join)
+        if events:
+            events[2].record(stream)
         clover_kv_compact(k_cache, v_cache, cache_len, self.path, self.accept_len, self.new_cache_len,
                           self.src_index, status=self.status, stream=stream)
+        if events:
+            events[3].record(stream)

@@ -20,7 +20,6 @@ namespace clover {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kTargetCtas = 2 * 152 * 2;   // about four resident CTAs per SM on a 152-SM GPU
 
 // Order-preserving map of a float to 32 unsigned bits; -0 is first turned into +0.
 __device__ __forceinline__ uint32_t order_bits(float x) {
@@ -40,53 +39,73 @@ __device__ __forceinline__ void scan_scalar(const T *row, int64_t lo, int64_t hi
     for (int64_t v = lo + threadIdx.x; v < hi; v += kThreads) best = umax64(best, make_key(to_float(row[v]), (uint32_t)v));
 }
 
-// Vector body: 16-byte units [u_lo, u_hi) of the row starting at element `first`.
+constexpr int kUnits = 8;   // 16-byte loads each thread issues at once
+
+// Largest value of a 16-byte unit (8 bf16 or 4 fp32), as fp32.
+__device__ __forceinline__ float unit_max(const uint4 &w, __nv_bfloat16) {
+    const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&w);
+    const __nv_bfloat162 m = __hmax2(__hmax2(h[0], h[1]), __hmax2(h[2], h[3]));
+    return fmaxf(__low2float(m), __high2float(m));
+}
+__device__ __forceinline__ float unit_max(const uint4 &w, float) {
+    return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)), fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
+}
+
+// Position of the first element of a unit equal to v (which the unit holds).
+__device__ __forceinline__ int unit_first(const uint4 &w, float v, __nv_bfloat16) {
+    const uint32_t x[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const float f = __uint_as_float((e & 1) ? (x[e >> 1] & 0xFFFF0000u) : (x[e >> 1] << 16));
+        if (f == v) return e;
+    }
+    return 7;
+}
+__device__ __forceinline__ int unit_first(const uint4 &w, float v, float) {
+    const uint32_t x[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+        if (__uint_as_float(x[e]) == v) return e;
+    return 3;
+}
+
+// Vector body: 16-byte units [0, n_units) of the row from element `first`.
+// Each round a thread issues kUnits independent loads (units tid + k*kThreads),
+// takes the maximum over them, and only then looks for its first position.
 template <typename T>
 __device__ __forceinline__ void scan_vector(const T *row, int64_t first, int64_t n_units, uint64_t &best) {
     constexpr int E = 16 / sizeof(T);
     const uint4 *p = reinterpret_cast<const uint4 *>(row + first);
-    int64_t u = threadIdx.x;
-    // four independent 16-byte loads in flight per thread
-    for (; u + 3 * kThreads < n_units; u += 4 * kThreads) {
-        uint4 w[4];
+    for (int64_t base = 0; base < n_units; base += (int64_t)kThreads * kUnits) {
+        uint4 w[kUnits];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) w[k] = __ldcs(p + u + k * kThreads);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            float f[E];
-            if constexpr (E == 8) {
-                const uint32_t x[4] = {w[k].x, w[k].y, w[k].z, w[k].w};
-#pragma unroll
-                for (int h = 0; h < 4; ++h) {
-                    f[2 * h] = __uint_as_float(x[h] << 16);
-                    f[2 * h + 1] = __uint_as_float(x[h] & 0xFFFF0000u);
-                }
-            } else {
-                f[0] = __uint_as_float(w[k].x); f[1] = __uint_as_float(w[k].y);
-                f[2] = __uint_as_float(w[k].z); f[3] = __uint_as_float(w[k].w);
-            }
-            const int64_t base = first + (u + k * kThreads) * E;
-#pragma unroll
-            for (int e = 0; e < E; ++e) best = umax64(best, make_key(f[e], (uint32_t)(base + e)));
+        for (int k = 0; k < kUnits; ++k) {
+            const int64_t u = base + threadIdx.x + (int64_t)k * kThreads;
+            w[k] = (u < n_units) ? __ldcs(p + u) : make_uint4(0, 0, 0, 0);
         }
-    }
-    for (; u < n_units; u += kThreads) {
-        const uint4 w = __ldcs(p + u);
-        float f[E];
-        if constexpr (E == 8) {
-            const uint32_t x[4] = {w.x, w.y, w.z, w.w};
+        float um[kUnits];
+        float m = -INFINITY;
 #pragma unroll
-            for (int h = 0; h < 4; ++h) {
-                f[2 * h] = __uint_as_float(x[h] << 16);
-                f[2 * h + 1] = __uint_as_float(x[h] & 0xFFFF0000u);
-            }
-        } else {
-            f[0] = __uint_as_float(w.x); f[1] = __uint_as_float(w.y);
-            f[2] = __uint_as_float(w.z); f[3] = __uint_as_float(w.w);
+        for (int k = 0; k < kUnits; ++k) {
+            const int64_t u = base + threadIdx.x + (int64_t)k * kThreads;
+            um[k] = (u < n_units) ? unit_max(w[k], T()) : -INFINITY;
+            m = fmaxf(m, um[k]);
         }
-        const int64_t base = first + u * E;
+        // units are visited in increasing element order, so the first unit
+        // reaching m holds this round's first maximum of the thread
+        int kf = -1;
 #pragma unroll
-        for (int e = 0; e < E; ++e) best = umax64(best, make_key(f[e], (uint32_t)(base + e)));
+        for (int k = kUnits - 1; k >= 0; --k)
+            if (um[k] == m && base + threadIdx.x + (int64_t)k * kThreads < n_units) kf = k;
+        if (kf >= 0) {
+            uint4 wf = w[0];
+#pragma unroll
+            for (int k = 1; k < kUnits; ++k)
+                if (k == kf) wf = w[k];
+            const int64_t u = base + threadIdx.x + (int64_t)kf * kThreads;
+            const int e = unit_first(wf, m, T());
+            best = umax64(best, make_key(m, (uint32_t)(first + u * E + e)));
+        }
     }
 }
 
@@ -218,18 +237,15 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
 
 }  // namespace
 
+// Vocabulary chunk per CTA: one round of kUnits 16-byte loads per thread
+// (32 KB of bf16 or fp32 logits).
 void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk) {
-    const int rows = B * T;
-    int n = (kTargetCtas + rows - 1) / rows;
+    (void)B;
+    (void)T;
     const int elems = 16 / (dtype == CLOVER_F32 ? 4 : 2);
-    const int max_by_size = (V + 4096 - 1) / 4096;          // at least 4096 elements per chunk
-    if (n > max_by_size) n = max_by_size;
-    if (n < 1) n = 1;
-    int c = (V + n - 1) / n;
-    c = (c + elems - 1) / elems * elems;
-    n = (V + c - 1) / c;
-    *n_chunks = n;
+    const int c = kThreads * kUnits * elems;
     *chunk = c;
+    *n_chunks = (V + c - 1) / c;
 }
 
 size_t accept_workspace_bytes(int B, int T, int V, int dtype) {

@@ -21,7 +21,7 @@ def run_gpu(t: dict, scale: float = 0.0, step: pkg.VerifyStep | None = None) -> 
     V = t["logits"].shape[-1]
     if step is None:
         step = pkg.VerifyStep(B, T, Hq, Hkv, D, t["Lcap"], V, t["q"].dtype, device=t["q"].device)
-    step.status.zero_()
+    step.clear_status()
     step.run(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
              t["cand"], t["logits"], scale=scale)
     torch.cuda.synchronize()
@@ -32,7 +32,7 @@ def compare_full(host: dict, step: pkg.VerifyStep, t: dict, scale: float = 0.0):
     """Every output against oracle.verify_step (small shapes)."""
     ref = oracle.verify_step(host, scale=scale)
     dt = host["q"].dtype
-    assert int(step.status.item()) == 0
+    assert step.device_status() == 0
     err = (step.out.double().cpu() - ref["out"]).abs().max().item()
     assert err <= ATOL[dt], f"attention max-abs {err} > {ATOL[dt]}"
     assert torch.equal(step.argmax.cpu(), ref["argmax"])

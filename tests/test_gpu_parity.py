@@ -78,7 +78,7 @@ def test_full_size_workloads(name, cuda):
     host = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in t.items()}
     kc0, vc0 = t["k_cache"].clone(), t["v_cache"].clone()
     step = run_gpu(t)
-    assert int(step.status.item()) == 0
+    assert step.device_status() == 0
 
     B, T, Hq, D = w.B, w.T, w.Hq, w.D
     n_rows = B * T * Hq
@@ -194,7 +194,7 @@ def test_bad_tree_reports_status(cuda):
     host["parent"][0, 5] = 6                             # a node whose parent comes after it
     t = to_dev(host, cuda)
     step = run_gpu(t)
-    assert int(step.status.item()) & pkg.api.ERR_BAD_TREE
+    assert step.device_status() & pkg.api.ERR_BAD_TREE
 
 
 def test_capacity_reports_status(cuda):
@@ -203,7 +203,7 @@ def test_capacity_reports_status(cuda):
     host["cache_len"][0] = host["Lcap"] - w.T + 1
     t = to_dev(host, cuda)
     step = run_gpu(t)
-    assert int(step.status.item()) & pkg.api.ERR_CAPACITY
+    assert step.device_status() & pkg.api.ERR_CAPACITY
 
 
 def test_host_errors_raise(cuda):
