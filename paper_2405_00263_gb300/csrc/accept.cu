@@ -11,9 +11,9 @@
 // with 16-byte loads to a packed 64-bit key (order-preserving value bits in the
 // high word, bit-inverted index in the low word) so that one unsigned max
 // gives "largest value, then smallest index", and folds it into the row's key
-// with a 64-bit atomic max.  The CTA that finishes the last chunk of a
-// sequence (per-sequence arrival counter) decodes the argmax of every node and
-// runs the walk in one warp; it also resets the keys and the counter.
+// with a 64-bit atomic max.  Per-row and per-sequence arrival counters find
+// the CTA that finishes a sequence's last chunk; it decodes the argmax of
+// every node and runs the walk in one warp, and resets the keys and counters.
 #include "common.cuh"
 
 namespace clover {
@@ -129,7 +129,8 @@ struct AcceptArgs {
     int B, T, V, n_chunks, chunk;
     int32_t *argmax_out, *path_out, *accept_len, *bonus;
     unsigned long long *row_key;   // [B*T] running packed maximum of each logit row
-    unsigned *seq_count;           // [B] chunks of the sequence's rows finished
+    unsigned *row_count;           // [B*T] chunks of the row finished
+    unsigned *seq_count;           // [B] rows of the sequence finished
     int32_t *status;
 };
 
@@ -219,13 +220,20 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
     }
     best = block_max(best, s_red);
 
-    // fold this chunk into the row's key, then count the chunk as done for the
-    // sequence; the CTA finishing the sequence's last chunk runs the walk
+    // fold this chunk into the row's key and count it; the CTA finishing a
+    // row's last chunk counts the row for its sequence, and the one finishing
+    // the sequence's last row runs the walk (two levels keep each counter to a
+    // few arrivals)
     if (threadIdx.x == 0) {
         atomicMax(a.row_key + row, static_cast<unsigned long long>(best));
         __threadfence();
-        const unsigned prev = atomicAdd(a.seq_count + b, 1u);
-        s_seq_last = (prev == (unsigned)(a.T * a.n_chunks) - 1u);
+        bool last = false;
+        if (atomicAdd(a.row_count + row, 1u) == (unsigned)a.n_chunks - 1u) {
+            a.row_count[row] = 0u;                              // ready for the next call
+            __threadfence();
+            last = (atomicAdd(a.seq_count + b, 1u) == (unsigned)a.T - 1u);
+        }
+        s_seq_last = last;
     }
     __syncthreads();
     if (!s_seq_last) return;
@@ -251,7 +259,7 @@ void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk) {
 size_t accept_workspace_bytes(int B, int T, int V, int dtype) {
     (void)V;
     (void)dtype;
-    return sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * (size_t)B;
+    return sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * ((size_t)B * T + B);
 }
 
 cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
@@ -270,7 +278,8 @@ cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t
     a.accept_len = accept_len;
     a.bonus = bonus;
     a.row_key = static_cast<unsigned long long *>(workspace);
-    a.seq_count = reinterpret_cast<unsigned *>(a.row_key + (size_t)B * T);
+    a.row_count = reinterpret_cast<unsigned *>(a.row_key + (size_t)B * T);
+    a.seq_count = a.row_count + (size_t)B * T;
     a.status = status;
     dim3 grid(B * T, a.n_chunks);
     if (dtype == CLOVER_F32) accept_kernel<float><<<grid, kThreads, 0, stream>>>(a);

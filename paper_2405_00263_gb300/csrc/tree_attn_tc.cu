@@ -8,17 +8,19 @@
 // One CTA per (row tile of up to 128 query rows, cache-key split, sequence x
 // KV head).  The T*G query rows of a KV head (row i*G + hh = node i, query head
 // g*G + hh) share every K/V tile, so per 64-key tile:
-//   S  = Q K^T        tcgen05.mma M=128 N=64 K=D  (Q, K K-major in smem, S in TMEM)
-//   P  = 2^(S*c - m)  online softmax in registers, bf16 P to smem
-//   O += P V          tcgen05.mma M=128 N=D K=64  (V MN-major in smem, O in TMEM)
+//   S  = Q K^T        tcgen05.mma M=128 N=64 K=D  (Q, K K-major in smem; S in TMEM)
+//   P  = 2^(S*c - m)  online softmax in registers; bf16 P written back to TMEM
+//                     over the S tile it came from
+//   O += P V          tcgen05.mma M=128 N=D K=64  (P from TMEM, V MN-major in smem)
 // O stays in TMEM for the whole key range.  Each row keeps a reference max m;
 // P is taken relative to it, and m (with O and the row sum) is only moved when
 // a tile's max exceeds it by more than 2^8, so O is rarely rescaled.
-// Warp roles (192 threads): warp q in 0-3 runs the softmax, rescales and the
+// Warp roles (224 threads): warp q in 0-3 runs the softmax, rescales and the
 // epilogue of TMEM lanes 32q.. (the lanes warp q may access); warp 4 issues the
-// TMA loads of Q and of the K/V tiles (4-stage ring, 128-byte swizzle) and
-// appends the tree K/V to the cache; warp 5 allocates TMEM and issues the MMAs
-// from one thread.
+// TMA loads of Q and of the K tiles (its own ring) and appends the tree K/V to
+// the cache; warp 6 issues the TMA loads of the V tiles (a deeper ring: a V
+// tile is held until its P.V product, a K tile only until its S); warp 5
+// allocates TMEM and issues the MMAs from one thread.
 // The split that owns the last cache range also takes the tile of T tree keys
 // (read from k_new/v_new) under the ancestor bitmask.  The n_split CTAs of a
 // (sequence, head, row tile) form one thread-block cluster: each leaves its
@@ -39,12 +41,14 @@ using namespace tc;
 
 constexpr int BM = 128;                 // query rows per CTA (MMA M)
 constexpr int BN = 64;                  // keys per tile
-constexpr int NS = 4;                   // K/V pipeline stages
-constexpr int kProducerWarp = 4;
+constexpr int NSK = 5;                  // K ring stages
+constexpr int NSV = 6;                  // V ring stages
+constexpr int kKProducerWarp = 4;
 constexpr int kMmaWarp = 5;
-constexpr int kThreads = 192;
+constexpr int kVProducerWarp = 6;
+constexpr int kThreads = 224;
 constexpr int kMaxCluster = 8;          // portable cluster size: splits per head
-constexpr uint32_t kTmemCols = 256;     // S: 2 x 64 columns, O: D columns
+constexpr uint32_t kTmemCols = 256;     // S/P: 2 x 64 columns, O: D columns
 constexpr float kRescale = 8.0f;        // move the reference max only past 2^8 growth
 constexpr uint64_t kWaitNs = 500ull * 1000 * 1000;   // 0.5 s per wait
 
@@ -52,24 +56,22 @@ template <int D>
 struct TcSmem {
     static constexpr int DH = D / 64;                // 128-byte column blocks per row
     static constexpr int q_bytes = BM * D * 2;       // [DH][BM][128 B]
-    static constexpr int kv_bytes = BN * D * 2;      // one stage of K or V: [DH][BN][128 B]
-    static constexpr int p_bytes = BM * BN * 2;      // [BM][128 B]
+    static constexpr int kv_bytes = BN * D * 2;      // one K or V tile: [DH][BN][128 B]
     static constexpr int q_off = 0;
     static constexpr int k_off = q_off + q_bytes;
-    static constexpr int v_off = k_off + NS * kv_bytes;
-    static constexpr int p_off = v_off + NS * kv_bytes;
-    static constexpr int bar_off = p_off + 2 * p_bytes;
-    static constexpr int n_bars = 2 * NS + 12;
+    static constexpr int v_off = k_off + NSK * kv_bytes;
+    static constexpr int ml_off = v_off + NSV * kv_bytes;          // merge: (m, l) per row [BM]
+    static constexpr int bar_off = ml_off + BM * 8;
+    static constexpr int n_bars = 2 * NSK + 2 * NSV + 11;
     static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad flags
     static constexpr int anc_off = misc_off + 16;                  // ancestor masks [64]
-    static constexpr int mw_off = anc_off + kMaxTreeNodes * 8;     // merge weights [BM][kMaxCluster + 1]
-    static constexpr int total = mw_off + BM * (kMaxCluster + 1) * 4;
+    static constexpr int total = anc_off + kMaxTreeNodes * 8;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
-    // after the key loop the K/V ring holds this CTA's partial O (fp32, rows padded
-    // to D + 4 floats) and the P area its (m, l) pairs
+    // after the key loop the K/V rings hold this CTA's partial O (fp32, rows
+    // padded to D + 4 floats)
     static constexpr int po_stride = D + 4;
-    static_assert(BM * po_stride * 4 <= 2 * NS * kv_bytes, "partial O must fit in the K/V ring");
-    static_assert(BM * 8 <= 2 * p_bytes, "partial (m, l) must fit in the P area");
+    static_assert(BM * po_stride * 4 <= (NSK + NSV) * kv_bytes, "partial O must fit in the K/V rings");
+    static_assert(alloc <= 227 * 1024, "shared memory budget");
 };
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -88,14 +90,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *sQ = sm + S::q_off;
     uint8_t *sK = sm + S::k_off;
     uint8_t *sV = sm + S::v_off;
-    uint8_t *sP = sm + S::p_off;
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + S::bar_off);
-    uint64_t *kv_full = bars;
-    uint64_t *kv_empty = bars + NS;
-    uint64_t *s_full = bars + 2 * NS;
-    uint64_t *s_empty = s_full + 2;
-    uint64_t *p_full = s_empty + 2;
-    uint64_t *o_full = p_full + 2;
+    uint64_t *k_full = bars;
+    uint64_t *k_empty = k_full + NSK;
+    uint64_t *v_full = k_empty + NSK;
+    uint64_t *v_empty = v_full + NSV;
+    uint64_t *s_full = v_empty + NSV;         // [2] S of a tile is in TMEM
+    uint64_t *p_full = s_full + 2;            // [2] P of a tile is in TMEM
+    uint64_t *o_full = p_full + 2;            // [2] the tile's P.V product is done
     uint64_t *mma_done = o_full + 2;
     uint64_t *q_full = mma_done + 1;
     uint64_t *m_ready = q_full + 1;           // partials of all cluster CTAs are in place
@@ -104,7 +106,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     volatile int *s_abort = reinterpret_cast<volatile int *>(sm + S::misc_off + 4);
     bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 8);
     uint64_t *s_anc = reinterpret_cast<uint64_t *>(sm + S::anc_off);
-    float *merge_w = reinterpret_cast<float *>(sm + S::mw_off);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -130,40 +131,37 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
     const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
 
-    // ---------------------------------------------------------------- setup
-    // The producer warp initialises the barriers and issues the Q load and the
-    // first NS tile loads at once (the stages start empty), so they overlap the
-    // TMEM allocation.
-    auto issue_tile = [&](int j) {
-        const int s = j % NS;
-        mbar_arrive_expect_tx(&kv_full[s], 2 * S::kv_bytes);
-        uint8_t *kdst = sK + s * S::kv_bytes;
-        uint8_t *vdst = sV + s * S::kv_bytes;
+    // tile j of K (is_v == false) or V into ring stage `dst`
+    auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar) {
+        mbar_arrive_expect_tx(bar, S::kv_bytes);
+        const CUtensorMap *cache_map = is_v ? &tm_vc : &tm_kc;
+        const CUtensorMap *new_map = is_v ? &tm_vn : &tm_kn;
         if (j < n_cache_tiles) {
-            const int key0 = kbeg + j * BN;
 #pragma unroll
-            for (int dh = 0; dh < S::DH; ++dh) {
-                tma_load_3d(kdst + dh * BN * 128, &tm_kc, &kv_full[s], dh * 64, key0, bg);
-                tma_load_3d(vdst + dh * BN * 128, &tm_vc, &kv_full[s], dh * 64, key0, bg);
-            }
+            for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + j * BN, bg);
         } else {
 #pragma unroll
-            for (int dh = 0; dh < S::DH; ++dh) {
-                tma_load_3d(kdst + dh * BN * 128, &tm_kn, &kv_full[s], dh * 64, g, b * a.T);
-                tma_load_3d(vdst + dh * BN * 128, &tm_vn, &kv_full[s], dh * 64, g, b * a.T);
-            }
+            for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, new_map, bar, dh * 64, g, b * a.T);
         }
     };
-    int producer_issued = 0;
-    if (warp == kProducerWarp) {
+
+    // ---------------------------------------------------------------- setup
+    // The K producer initialises every barrier; the producers issue the Q load
+    // and their first ring loads at once (the stages start empty), so they
+    // overlap the TMEM allocation and the cluster barrier.
+    int k_issued = 0, v_issued = 0;
+    if (warp == kKProducerWarp) {
         if (lane == 0) {
-            for (int i = 0; i < NS; ++i) {
-                mbar_init(&kv_full[i], 1);
-                mbar_init(&kv_empty[i], 1);
+            for (int i = 0; i < NSK; ++i) {
+                mbar_init(&k_full[i], 1);
+                mbar_init(&k_empty[i], 1);
+            }
+            for (int i = 0; i < NSV; ++i) {
+                mbar_init(&v_full[i], 1);
+                mbar_init(&v_empty[i], 1);
             }
             for (int i = 0; i < 2; ++i) {
                 mbar_init(&s_full[i], 1);
-                mbar_init(&s_empty[i], q_act);
                 mbar_init(&p_full[i], q_act);
                 mbar_init(&o_full[i], 1);
             }
@@ -175,11 +173,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             *s_bad = false;
             fence_barrier_init();
             prefetch_tensormap(&tm_kc);
-            prefetch_tensormap(&tm_vc);
             prefetch_tensormap(&tm_kn);
-            prefetch_tensormap(&tm_vn);
             if (a.q_box_nodes > 0) {
                 // Q rows (node, head in group) of this tile: box (64 d, G heads, q_box_nodes nodes)
+                prefetch_tensormap(&tm_q);
                 mbar_arrive_expect_tx(q_full, S::DH * a.G * a.q_box_nodes * 128);
 #pragma unroll
                 for (int dh = 0; dh < S::DH; ++dh)
@@ -187,7 +184,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else {
                 mbar_arrive(q_full);
             }
-            for (; producer_issued < min(NS, n_tiles); ++producer_issued) issue_tile(producer_issued);
+            for (; k_issued < min(NSK, n_tiles); ++k_issued)
+                issue_tile(k_issued, false, sK + k_issued * S::kv_bytes, &k_full[k_issued]);
         }
         __syncwarp();
         if (tree_cta) tree_masks_warp(a.parent + (size_t)b * a.T, a.T, s_anc, s_bad);
@@ -231,21 +229,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     else __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *s_tmem;
-    const uint32_t tS = tmem;                 // S tiles: columns [0, 2*BN)
+    const uint32_t tS = tmem;                 // S tiles (and their P): columns [0, 2*BN)
     const uint32_t tO = tmem + 2 * BN;        // O: columns [2*BN, 2*BN + D)
 
-    // ------------------------------------------------------ TMA producer warp
-    if (warp == kProducerWarp) {
+    // ----------------------------------------------------- TMA producer warps
+    if (warp == kVProducerWarp && lane == 0) {
+        prefetch_tensormap(&tm_vc);
+        prefetch_tensormap(&tm_vn);
+        for (int j = 0; j < n_tiles; ++j) {
+            const int s = j % NSV;
+            if (j >= NSV && !mbar_wait(&v_empty[s], ((j / NSV) - 1) & 1, kWaitNs)) {
+                *s_abort = 1;
+                break;
+            }
+            if (*s_abort) break;
+            issue_tile(j, true, sV + s * S::kv_bytes, &v_full[s]);
+            v_issued = j + 1;
+        }
+    }
+    if (warp == kKProducerWarp) {
         if (lane == 0) {
-            for (int j = producer_issued; j < n_tiles; ++j) {
-                const int s = j % NS;
-                if (!mbar_wait(&kv_empty[s], ((j / NS) - 1) & 1, kWaitNs)) {
+            for (int j = k_issued; j < n_tiles; ++j) {
+                const int s = j % NSK;
+                if (!mbar_wait(&k_empty[s], ((j / NSK) - 1) & 1, kWaitNs)) {
                     *s_abort = 1;
                     break;
                 }
                 if (*s_abort) break;
-                issue_tile(j);
-                producer_issued = j + 1;
+                issue_tile(j, false, sK + s * S::kv_bytes, &k_full[s]);
+                k_issued = j + 1;
             }
         }
         __syncwarp();
@@ -268,16 +280,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // --------------------------------------------------------- MMA issuer warp
+    // Per tile j: S_j (needs K_j) is issued one tile ahead, then P_j.V_j (needs
+    // P_j and V_j).  MMAs from this thread execute in issue order, so S_{j+2}
+    // overwriting the TMEM of P_j comes after the P.V product reading it.
     if (warp == kMmaWarp && lane == 0) {
         const uint32_t idS = idesc_bf16(BM, BN, false, false);
         const uint32_t idO = idesc_bf16(BM, D, false, true);
         const uint32_t q_base = smem_u32(sQ);
         bool ok = mbar_wait(q_full, 0, kWaitNs);
         auto issue_s = [&](int j) -> bool {
-            const int s = j % NS;
+            const int s = j % NSK;
             const int sb = j & 1;
-            if (!mbar_wait(&kv_full[s], (j / NS) & 1, kWaitNs)) return false;
-            if (j >= 2 && !mbar_wait(&s_empty[sb], ((j >> 1) - 1) & 1, kWaitNs)) return false;
+            if (!mbar_wait(&k_full[s], (j / NSK) & 1, kWaitNs)) return false;
             tc_fence_after();
             const uint32_t k_base = smem_u32(sK + s * S::kv_bytes);
 #pragma unroll
@@ -287,6 +301,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mma_bf16(tS + sb * BN, ad, bd, idS, k > 0 ? 1u : 0u);
             }
             mma_commit(&s_full[sb]);
+            mma_commit(&k_empty[s]);
             return true;
         };
         if (ok && n_tiles > 0) ok = issue_s(0);
@@ -296,32 +311,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             if (j + 1 < n_tiles && !(ok = issue_s(j + 1))) break;
-            const int s = j % NS;
+            const int s = j % NSV;
             const int sb = j & 1;
-            if (!mbar_wait(&p_full[sb], (j >> 1) & 1, kWaitNs)) {
+            if (!mbar_wait(&p_full[sb], (j >> 1) & 1, kWaitNs) || !mbar_wait(&v_full[s], (j / NSV) & 1, kWaitNs)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            const uint32_t p_base = smem_u32(sP + sb * S::p_bytes);
             const uint32_t v_base = smem_u32(sV + s * S::kv_bytes);
 #pragma unroll
             for (int k = 0; k < BN / 16; ++k) {
-                const uint64_t ad = sdesc_sw128(p_base + k * 32, 16, 1024);
                 const uint64_t bd = sdesc_sw128(v_base + k * 16 * 128, BN * 128, 1024);
-                mma_bf16(tO, ad, bd, idO, (j > 0 || k > 0) ? 1u : 0u);
+                mma_bf16_tmem_a(tO, tS + sb * BN + k * 8, bd, idO, (j > 0 || k > 0) ? 1u : 0u);
             }
             mma_commit(&o_full[sb]);
-            mma_commit(&kv_empty[s]);
+            mma_commit(&v_empty[s]);
         }
         if (!ok) *s_abort = 1;
         mma_commit(mma_done);
     }
 
     // ------------------------------------------------------------ softmax warps
-    // Warp q owns TMEM lanes 32q.. = tile rows; it reads S, writes P, keeps the
-    // row's reference max m_ref and sum l, and rescales its O row in TMEM when
-    // m_ref has to move.
+    // Warp q owns TMEM lanes 32q.. = tile rows; it reads S, writes P back over
+    // it, keeps the row's reference max m_ref and sum l, and rescales its O row
+    // in TMEM when m_ref has to move.
     const int quad = warp & 3;
     const bool softmax_warp = warp < 4 && quad < q_act;
     const int r = quad * 32 + lane;
@@ -346,9 +359,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_ld32(tS + lane_base + sb * BN, *reinterpret_cast<float(*)[32]>(sv));
             tmem_ld32(tS + lane_base + sb * BN + 32, *reinterpret_cast<float(*)[32]>(sv + 32));
             tmem_wait_ld();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s_empty[sb]);
 
             const bool tree_tile = (j == n_cache_tiles);
             const int key0 = kbeg + j * BN;
@@ -390,47 +400,40 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int c = 0; c < 32; ++c) x[c] *= f;
                     tmem_st32(tO + lane_base + cc * 32, x);
                 }
-                tmem_wait_st();
-                tc_fence_before();
             }
             const float ref = (m_ref == -INFINITY) ? 0.f : m_ref;
             float sum4[4] = {0.f, 0.f, 0.f, 0.f};
+            float pk[32];
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
-                sv[c] = ex2_approx(fmaf(sv[c], sc, -ref));
-                sum4[c & 3] += sv[c];
+            for (int c = 0; c < 64; c += 2) {
+                const float p0 = ex2_approx(fmaf(sv[c], sc, -ref));
+                const float p1 = ex2_approx(fmaf(sv[c + 1], sc, -ref));
+                sum4[c & 3] += p0;
+                sum4[(c + 1) & 3] += p1;
+                pk[c >> 1] = __uint_as_float(pack_bf16x2(p0, p1));
             }
             l_run += (sum4[0] + sum4[1]) + (sum4[2] + sum4[3]);
+            // P over the first 32 columns of this tile's S (two keys per column)
+            tmem_st32(tS + lane_base + sb * BN, pk);
             // value rows of keys past the valid ones may hold anything (even NaN): zero them
             if (n_valid < BN) {
-                uint4 *vrows = reinterpret_cast<uint4 *>(sV + (j % NS) * S::kv_bytes);
+                const int s = j % NSV;
+                const bool got_v = __all_sync(0xffffffffu, mbar_wait(&v_full[s], (j / NSV) & 1, kWaitNs));
+                if (!got_v) {
+                    *s_abort = 1;
+                    break;
+                }
+                uint4 *vrows = reinterpret_cast<uint4 *>(sV + s * S::kv_bytes);
                 const int n_zero = (BN - n_valid) * S::DH * 8;
                 for (int e = r; e < n_zero; e += q_act * 32) {
                     const int row = n_valid + e / (S::DH * 8);
                     const int rest = e % (S::DH * 8);
                     vrows[(rest >> 3) * (BN * 8) + row * 8 + (rest & 7)] = make_uint4(0, 0, 0, 0);
                 }
+                fence_proxy_async_smem();
             }
-            // the P buffer of tile j was read by the P.V product of tile j-2
-            if (j >= 2) {
-                const bool free_p = __all_sync(0xffffffffu, mbar_wait(&o_full[sb], ((j >> 1) - 1) & 1, kWaitNs));
-                if (!free_p) {
-                    *s_abort = 1;
-                    break;
-                }
-            }
-            // P row r (64 keys = 128 bytes, eight swizzled 16-byte chunks)
-            uint8_t *prow = sP + sb * S::p_bytes + r * 128;
-#pragma unroll
-            for (int qd = 0; qd < 8; ++qd) {
-                uint4 w;
-                w.x = pack_bf16x2(sv[qd * 8 + 0], sv[qd * 8 + 1]);
-                w.y = pack_bf16x2(sv[qd * 8 + 2], sv[qd * 8 + 3]);
-                w.z = pack_bf16x2(sv[qd * 8 + 4], sv[qd * 8 + 5]);
-                w.w = pack_bf16x2(sv[qd * 8 + 6], sv[qd * 8 + 7]);
-                *reinterpret_cast<uint4 *>(prow + ((qd ^ (r & 7)) << 4)) = w;
-            }
-            fence_proxy_async_smem();
+            tmem_wait_st();
+            tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&p_full[sb]);
         }
@@ -446,18 +449,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------- epilogue
     tc_fence_before();
     __syncthreads();                          // every role is out of its key loop
-    if (*s_abort && warp == kProducerWarp && lane == 0) {
+    if (*s_abort && lane == 0) {
         // wind down: wait (bounded) for the loads still in flight before the
-        // K/V ring is reused below
-        for (int j = max(0, producer_issued - NS); j < producer_issued; ++j)
-            mbar_wait(&kv_full[j % NS], (j / NS) & 1, kWaitNs);
+        // rings are reused below
+        if (warp == kKProducerWarp)
+            for (int j = max(0, k_issued - NSK); j < k_issued; ++j) mbar_wait(&k_full[j % NSK], (j / NSK) & 1, kWaitNs);
+        if (warp == kVProducerWarp)
+            for (int j = max(0, v_issued - NSV); j < v_issued; ++j) mbar_wait(&v_full[j % NSV], (j / NSV) & 1, kWaitNs);
     }
     __syncthreads();
     tc_fence_after();
     __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(a.out);
     const bool row_ok = softmax_warp && r < rows_here;
-    float *part_o = reinterpret_cast<float *>(sK);   // [BM][D + 4] fp32, this CTA's partial
-    float2 *part_ml = reinterpret_cast<float2 *>(sP); // [BM] (m, l)
+    float *part_o = reinterpret_cast<float *>(sK);            // [BM][D + 4] fp32, this CTA's partial
+    float2 *part_ml = reinterpret_cast<float2 *>(sm + S::ml_off);
     if (softmax_warp) {
         const int R = rt * BM + r;
         const int i = row_ok ? R / a.G : 0;
@@ -511,50 +516,65 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (threadIdx.x < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_ready), threadIdx.x));
         const bool ready = __syncthreads_and(mbar_wait_cluster(m_ready, 0, kWaitNs));
         if (ready) {
-            // this CTA merges rows [r0, r1) of the tile
+            // this CTA merges rows [r0, r1) of the tile.  A thread takes items
+            // (row, 4 columns) in batches of kBatch and issues every split's
+            // (m, l) and columns of the whole batch before using any of them,
+            // so a batch costs one distributed-shared-memory round trip.
+            constexpr int kBatch = 3;
             const int per = (rows_here + n_split - 1) / n_split;
             const int r0 = split * per;
             const int r1 = min(rows_here, r0 + per);
+            const int n_items = (r1 - r0) * (D / 4);
             const uint32_t ml_base = smem_u32(part_ml);
             const uint32_t o_base = smem_u32(part_o);
-            for (int rr = r0 + threadIdx.x; rr < r1; rr += kThreads) {
-                float m[kMaxCluster], l[kMaxCluster];
-                float M = -INFINITY;
-                for (int k = 0; k < n_split; ++k) {
-                    const float2 v = ld_dsmem_f2(mapa_shared(ml_base + rr * 8, k));
-                    m[k] = v.x;
-                    l[k] = v.y;
-                    M = fmaxf(M, v.x);
+            for (int e0 = threadIdx.x; e0 < n_items; e0 += kThreads * kBatch) {
+                float2 ml[kBatch][kMaxCluster];
+                float4 x[kBatch][kMaxCluster];
+#pragma unroll
+                for (int t = 0; t < kBatch; ++t) {
+                    const int e = e0 + t * kThreads;
+                    const int rr = r0 + e / (D / 4);
+                    const int c4 = (e % (D / 4)) * 4;
+#pragma unroll
+                    for (int k = 0; k < kMaxCluster; ++k) {
+                        if (e < n_items && k < n_split) {
+                            ml[t][k] = ld_dsmem_f2(mapa_shared(ml_base + rr * 8, k));
+                            x[t][k] = ld_dsmem_f4(mapa_shared(o_base + (rr * S::po_stride + c4) * 4, k));
+                        }
+                    }
                 }
-                float lsum = 0.f;
-                for (int k = 0; k < n_split; ++k) {
-                    const float w = (m[k] == -INFINITY) ? 0.f : exp2f(m[k] - M);
-                    merge_w[rr * (kMaxCluster + 1) + k] = w;
-                    lsum += w * l[k];
+#pragma unroll
+                for (int t = 0; t < kBatch; ++t) {
+                    const int e = e0 + t * kThreads;
+                    if (e >= n_items) continue;
+                    const int rr = r0 + e / (D / 4);
+                    const int c4 = (e % (D / 4)) * 4;
+                    float M = -INFINITY;
+#pragma unroll
+                    for (int k = 0; k < kMaxCluster; ++k)
+                        if (k < n_split) M = fmaxf(M, ml[t][k].x);
+                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                    float lsum = 0.f;
+#pragma unroll
+                    for (int k = 0; k < kMaxCluster; ++k) {
+                        if (k < n_split) {
+                            const float w = (ml[t][k].x == -INFINITY) ? 0.f : exp2f(ml[t][k].x - M);
+                            lsum = fmaf(w, ml[t][k].y, lsum);
+                            acc.x = fmaf(w, x[t][k].x, acc.x);
+                            acc.y = fmaf(w, x[t][k].y, acc.y);
+                            acc.z = fmaf(w, x[t][k].z, acc.z);
+                            acc.w = fmaf(w, x[t][k].w, acc.w);
+                        }
+                    }
+                    const float inv = 1.f / lsum;
+                    const int R = rt * BM + rr;
+                    const int i = R / a.G;
+                    const int h = g * a.G + (R % a.G);
+                    uint2 w2;
+                    w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+                    w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+                    *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c4) = w2;
                 }
-                merge_w[rr * (kMaxCluster + 1) + kMaxCluster] = 1.f / lsum;
-            }
-            __syncthreads();
-            for (int e = threadIdx.x; e < (r1 - r0) * (D / 4); e += kThreads) {
-                const int rr = r0 + e / (D / 4);
-                const int c4 = (e % (D / 4)) * 4;
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                for (int k = 0; k < n_split; ++k) {
-                    const float w = merge_w[rr * (kMaxCluster + 1) + k];
-                    const float4 x = ld_dsmem_f4(mapa_shared(o_base + (rr * S::po_stride + c4) * 4, k));
-                    acc.x = fmaf(w, x.x, acc.x);
-                    acc.y = fmaf(w, x.y, acc.y);
-                    acc.z = fmaf(w, x.z, acc.z);
-                    acc.w = fmaf(w, x.w, acc.w);
-                }
-                const float inv = merge_w[rr * (kMaxCluster + 1) + kMaxCluster];
-                const int R = rt * BM + rr;
-                const int i = R / a.G;
-                const int h = g * a.G + (R % a.G);
-                uint2 w2;
-                w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-                w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-                *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c4) = w2;
             }
         } else {
             *s_abort = 1;
@@ -574,7 +594,7 @@ struct TcLaunchCache {
 };
 
 template <int D>
-int max_active_clusters(int n, int dev, TcLaunchCache &cache) {
+int max_active_clusters(int n, TcLaunchCache &cache) {
     if (cache.max_clusters[n] == 0) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(1, n, n);
@@ -594,7 +614,6 @@ int max_active_clusters(int n, int dev, TcLaunchCache &cache) {
         }
         cache.max_clusters[n] = num > 0 ? num : -1;
     }
-    (void)dev;
     return cache.max_clusters[n];
 }
 
@@ -617,7 +636,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     int n = 1;
     for (int c = kMaxCluster; c >= 2; --c) {
         if (c > by_len || base * c > cache.sms) continue;
-        if (max_active_clusters<D>(c, dev, cache) >= base) {
+        if (max_active_clusters<D>(c, cache) >= base) {
             n = c;
             break;
         }

@@ -53,7 +53,7 @@ def test_workspace_sizes(lib):
     assert ws(1, 16, 8, 8, 96, 192, 0) == 0              # D = 96 unsupported
     assert ws(1, 16, 6, 4, 64, 192, 0) == 0              # Hq not a multiple of Hkv
     acc = lib.clover_verify_accept_workspace_size
-    assert acc(1, 64, 125696, 1) == 8 * 64 + 4 * 1     # one 64-bit key per row, one counter per sequence
+    assert acc(1, 64, 125696, 1) == 8 * 64 + 4 * (64 + 1)   # a 64-bit key and a counter per row, a counter per sequence
     assert acc(1, 0, 10, 1) == 0 and acc(1, 4, 0, 1) == 0
 
 
