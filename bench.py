@@ -46,7 +46,7 @@ DEFAULT_WORKLOAD = "7b_l4096"
 L2_BYTES = 129 * 1000 * 1000
 FALLBACK_HBM_GBS = 6800.0
 KERNEL_SOURCES = {
-    "tree_attn": ["tree_attn_fma.cu", "common.cuh", "abi.cu"],
+    "tree_attn": ["tree_attn_tc.cu", "tc_ptx.cuh", "tmap_host.cuh", "common.cuh", "abi.cu"],
     "accept": ["accept.cu", "common.cuh"],
     "kv_compact": ["kv_compact.cu", "common.cuh"],
 }
