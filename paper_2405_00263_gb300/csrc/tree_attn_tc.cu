@@ -17,10 +17,11 @@
 // a tile's max exceeds it by more than 2^8, so O is rarely rescaled.
 // Warp roles (224 threads): warp q in 0-3 runs the softmax, rescales and the
 // epilogue of TMEM lanes 32q.. (the lanes warp q may access); warp 4 issues the
-// TMA loads of Q and of the K tiles (its own ring) and appends the tree K/V to
-// the cache; warp 6 issues the TMA loads of the V tiles (a deeper ring: a V
-// tile is held until its P.V product, a K tile only until its S); warp 5
-// allocates TMEM and issues the MMAs from one thread.
+// TMA loads of Q and of the K tiles (its own ring); warp 6 issues the TMA loads
+// of the V tiles (a deeper ring: a V tile is held until its P.V product, a K
+// tile only until its S); warp 5 allocates TMEM and issues the MMAs from one
+// thread.  The tree CTA's producers also append the tree keys and values to
+// the cache, by TMA stores of the tree tile they loaded.
 // The split that owns the last cache range also takes the tile of T tree keys
 // (read from k_new/v_new) under the ancestor bitmask.  The n_split CTAs of a
 // (sequence, head, row tile) form one thread-block cluster: each leaves its
@@ -41,8 +42,6 @@ using namespace tc;
 
 constexpr int BM = 128;                 // query rows per CTA (MMA M)
 constexpr int BN = 64;                  // keys per tile
-constexpr int NSK = 5;                  // K ring stages
-constexpr int NSV = 6;                  // V ring stages
 constexpr int kKProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kVProducerWarp = 6;
@@ -52,10 +51,16 @@ constexpr uint32_t kTmemCols = 256;     // S/P: 2 x 64 columns, O: D columns
 constexpr float kRescale = 8.0f;        // move the reference max only past 2^8 growth
 constexpr uint64_t kWaitNs = 500ull * 1000 * 1000;   // 0.5 s per wait
 
-template <int D>
+// Shared-memory plan.  QR = query rows stored per tile (128, or 64 when no tile
+// has more than 64 real rows: the MMA still reads 128 A rows, and rows 64-127
+// then come from whatever follows in shared memory; they only produce TMEM
+// lanes 64-127, which nothing reads).  The room saved goes to a deeper K ring.
+template <int D, int QR>
 struct TcSmem {
+    static constexpr int NSK = (QR == 64) ? 6 : 5;   // K ring stages
+    static constexpr int NSV = 6;                    // V ring stages
     static constexpr int DH = D / 64;                // 128-byte column blocks per row
-    static constexpr int q_bytes = BM * D * 2;       // [DH][BM][128 B]
+    static constexpr int q_bytes = QR * D * 2;       // [DH][QR][128 B]
     static constexpr int kv_bytes = BN * D * 2;      // one K or V tile: [DH][BN][128 B]
     static constexpr int q_off = 0;
     static constexpr int k_off = q_off + q_bytes;
@@ -70,7 +75,7 @@ struct TcSmem {
     // after the key loop the K/V rings hold this CTA's partial O (fp32, rows
     // padded to D + 4 floats)
     static constexpr int po_stride = D + 4;
-    static_assert(BM * po_stride * 4 <= (NSK + NSV) * kv_bytes, "partial O must fit in the K/V rings");
+    static_assert(QR * po_stride * 4 <= (NSK + NSV) * kv_bytes, "partial O must fit in the K/V rings");
     static_assert(alloc <= 227 * 1024, "shared memory budget");
 };
 
@@ -79,12 +84,15 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<const uint32_t *>(&v);
 }
 
-template <int D>
+template <int D, int QR>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                         const __grid_constant__ CUtensorMap tm_kn, const __grid_constant__ CUtensorMap tm_vn,
-                        const __grid_constant__ CUtensorMap tm_q, const AttnArgs a) {
-    using S = TcSmem<D>;
+                        const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ks,
+                        const __grid_constant__ CUtensorMap tm_vs, const AttnArgs a) {
+    using S = TcSmem<D, QR>;
+    constexpr int NSK = S::NSK;
+    constexpr int NSV = S::NSV;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sQ = sm + S::q_off;
@@ -130,6 +138,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int kend = min(L, kbeg + chunk);
     const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
     const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
+    // this CTA appends the tree K/V to cache slots [L, L+T)
+    const bool appender = tree_cta && rt == 0 && !cap_bad;
 
     // tile j of K (is_v == false) or V into ring stage `dst`
     auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar) {
@@ -145,20 +155,48 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     };
 
+    // The tree tile (the last tile of the tree CTA) holds the T new keys or
+    // values in its first T rows once it has landed; TMA stores those rows
+    // straight from the ring to cache slots [L, L+T), then waits until the
+    // store has read them (the rings are reused after the key loop).
+    auto append_tile = [&](bool is_v) {
+        const int nst = is_v ? NSV : NSK;
+        const int s = n_cache_tiles % nst;
+        uint64_t *full = is_v ? &v_full[s] : &k_full[s];
+        const uint8_t *src = (is_v ? sV : sK) + s * S::kv_bytes;
+        if (*s_abort || !mbar_wait(full, (n_cache_tiles / nst) & 1, kWaitNs)) {
+            *s_abort = 1;
+            return;
+        }
+        fence_proxy_async_smem();
+#pragma unroll
+        for (int dh = 0; dh < S::DH; ++dh) tma_store_3d(is_v ? &tm_vs : &tm_ks, src + dh * BN * 128, dh * 64, L, bg);
+        bulk_commit_group();
+        bulk_wait_group_read0();
+    };
+
     // ---------------------------------------------------------------- setup
-    // The K producer initialises every barrier; the producers issue the Q load
-    // and their first ring loads at once (the stages start empty), so they
-    // overlap the TMEM allocation and the cluster barrier.
+    // Each producer initialises the barriers of its ring (the K producer also
+    // every other one) and issues its first ring loads at once (the stages
+    // start empty), the K producer also the Q load, so that they overlap the
+    // TMEM allocation.
     int k_issued = 0, v_issued = 0;
+    if (warp == kVProducerWarp && lane == 0) {
+        for (int i = 0; i < NSV; ++i) {
+            mbar_init(&v_full[i], 1);
+            mbar_init(&v_empty[i], 1);
+        }
+        fence_barrier_init();
+        prefetch_tensormap(&tm_vc);
+        prefetch_tensormap(&tm_vn);
+        for (; v_issued < min(NSV, n_tiles); ++v_issued)
+            issue_tile(v_issued, true, sV + v_issued * S::kv_bytes, &v_full[v_issued]);
+    }
     if (warp == kKProducerWarp) {
         if (lane == 0) {
             for (int i = 0; i < NSK; ++i) {
                 mbar_init(&k_full[i], 1);
                 mbar_init(&k_empty[i], 1);
-            }
-            for (int i = 0; i < NSV; ++i) {
-                mbar_init(&v_full[i], 1);
-                mbar_init(&v_empty[i], 1);
             }
             for (int i = 0; i < 2; ++i) {
                 mbar_init(&s_full[i], 1);
@@ -180,15 +218,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive_expect_tx(q_full, S::DH * a.G * a.q_box_nodes * 128);
 #pragma unroll
                 for (int dh = 0; dh < S::DH; ++dh)
-                    tma_load_3d(sQ + dh * (BM * 128), &tm_q, q_full, dh * 64, g * a.G, b * a.T + rt * a.q_box_nodes);
+                    tma_load_3d(sQ + dh * (QR * 128), &tm_q, q_full, dh * 64, g * a.G, b * a.T + rt * a.q_box_nodes);
             } else {
                 mbar_arrive(q_full);
             }
             for (; k_issued < min(NSK, n_tiles); ++k_issued)
                 issue_tile(k_issued, false, sK + k_issued * S::kv_bytes, &k_full[k_issued]);
         }
-        __syncwarp();
-        if (tree_cta) tree_masks_warp(a.parent + (size_t)b * a.T, a.T, s_anc, s_bad);
     }
     if (warp == kMmaWarp) {
         tmem_alloc(s_tmem, kTmemCols);
@@ -199,7 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // swizzled K-major layout, rows past this tile's real rows zero
         const __nv_bfloat16 *q = static_cast<const __nv_bfloat16 *>(a.q);
         constexpr int chunks_per_row = S::DH * 8;
-        constexpr int per_thread = BM * chunks_per_row / 128;
+        constexpr int per_thread = QR * chunks_per_row / 128;
         uint4 v[per_thread];
 #pragma unroll
         for (int k = 0; k < per_thread; ++k) {
@@ -220,31 +256,38 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int c = threadIdx.x + 128 * k;
             const int r = c / chunks_per_row;
             const int j = c % chunks_per_row;
-            *reinterpret_cast<uint4 *>(sQ + (j >> 3) * (BM * 128) + r * 128 + (((j & 7) ^ (r & 7)) << 4)) = v[k];
+            *reinterpret_cast<uint4 *>(sQ + (j >> 3) * (QR * 128) + r * 128 + (((j & 7) ^ (r & 7)) << 4)) = v[k];
         }
         fence_proxy_async_smem();
     }
+    // the tree CTA's ancestor masks (warp 3 is otherwise idle here)
+    if (warp == 3 && tree_cta) tree_masks_warp(a.parent + (size_t)b * a.T, a.T, s_anc, s_bad);
+    // The cluster barrier is split: its arrive here publishes this CTA's
+    // barriers, its wait (before the first remote arrive, in the merge) lets
+    // the key loop start without waiting for the other CTAs' setup.
     tc_fence_before();
-    if (n_split > 1) cluster_sync_all();      // every CTA's barriers exist before any remote arrive
-    else __syncthreads();
+    __syncwarp();
+    if (n_split > 1) cluster_arrive_release();
+    __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *s_tmem;
     const uint32_t tS = tmem;                 // S tiles (and their P): columns [0, 2*BN)
     const uint32_t tO = tmem + 2 * BN;        // O: columns [2*BN, 2*BN + D)
 
     // ----------------------------------------------------- TMA producer warps
-    if (warp == kVProducerWarp && lane == 0) {
-        prefetch_tensormap(&tm_vc);
-        prefetch_tensormap(&tm_vn);
-        for (int j = 0; j < n_tiles; ++j) {
-            const int s = j % NSV;
-            if (j >= NSV && !mbar_wait(&v_empty[s], ((j / NSV) - 1) & 1, kWaitNs)) {
-                *s_abort = 1;
-                break;
+    if (warp == kVProducerWarp) {
+        if (lane == 0) {
+            for (int j = v_issued; j < n_tiles; ++j) {
+                const int s = j % NSV;
+                if (!mbar_wait(&v_empty[s], ((j / NSV) - 1) & 1, kWaitNs)) {
+                    *s_abort = 1;
+                    break;
+                }
+                if (*s_abort) break;
+                issue_tile(j, true, sV + s * S::kv_bytes, &v_full[s]);
+                v_issued = j + 1;
             }
-            if (*s_abort) break;
-            issue_tile(j, true, sV + s * S::kv_bytes, &v_full[s]);
-            v_issued = j + 1;
+            if (appender && v_issued == n_tiles) append_tile(true);
         }
     }
     if (warp == kKProducerWarp) {
@@ -259,23 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 issue_tile(j, false, sK + s * S::kv_bytes, &k_full[s]);
                 k_issued = j + 1;
             }
-        }
-        __syncwarp();
-        // append the tree K/V to cache slots [L, L+T) (one CTA per sequence and head)
-        if (tree_cta && rt == 0 && !cap_bad) {
-            const __nv_bfloat16 *kn = static_cast<const __nv_bfloat16 *>(a.k_new);
-            const __nv_bfloat16 *vn = static_cast<const __nv_bfloat16 *>(a.v_new);
-            __nv_bfloat16 *kc = static_cast<__nv_bfloat16 *>(a.k_cache);
-            __nv_bfloat16 *vc = static_cast<__nv_bfloat16 *>(a.v_cache);
-            constexpr int per_row = D / 8;
-            for (int e = lane; e < a.T * per_row; e += 32) {
-                const int m = e / per_row;
-                const int c = (e % per_row) * 8;
-                const size_t src = ((size_t)(b * a.T + m) * a.Hkv + g) * D + c;
-                const size_t dst = ((size_t)(b * a.Hkv + g) * a.Lcap + L + m) * D + c;
-                *reinterpret_cast<uint4 *>(kc + dst) = __ldg(reinterpret_cast<const uint4 *>(kn + src));
-                *reinterpret_cast<uint4 *>(vc + dst) = __ldg(reinterpret_cast<const uint4 *>(vn + src));
-            }
+            if (appender && k_issued == n_tiles) append_tile(false);
         }
     }
 
@@ -296,7 +323,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t k_base = smem_u32(sK + s * S::kv_bytes);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k) {
-                const uint64_t ad = sdesc_sw128(q_base + (k >> 2) * (BM * 128) + (k & 3) * 32, 16, 1024);
+                const uint64_t ad = sdesc_sw128(q_base + (k >> 2) * (QR * 128) + (k & 3) * 32, 16, 1024);
                 const uint64_t bd = sdesc_sw128(k_base + (k >> 2) * (BN * 128) + (k & 3) * 32, 16, 1024);
                 mma_bf16(tS + sb * BN, ad, bd, idS, k > 0 ? 1u : 0u);
             }
@@ -344,7 +371,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (softmax_warp) {
         const int R = rt * BM + r;
         const int node = (r < rows_here) ? R / a.G : 0;
-        const uint64_t anc = tree_cta ? s_anc[node] : 0ull;
         const float sc = a.scale_log2;
         for (int j = 0; j < n_tiles; ++j) {
             const int sb = j & 1;
@@ -363,13 +389,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool tree_tile = (j == n_cache_tiles);
             const int key0 = kbeg + j * BN;
             const int n_valid = tree_tile ? a.T : min(BN, kend - key0);
-            if (tree_tile || n_valid < BN) {
+            // Keys of the tile this row sees: a prefix of the cache keys, or the
+            // row's ancestors among the tree keys.  Every tile runs the same
+            // instructions, so the one tree tile, late in the loop, brings no
+            // code into the instruction cache (a miss then waits on a
+            // saturated memory system).
+            const uint64_t prefix = (n_valid >= BN) ? ~0ull : ((1ull << n_valid) - 1ull);
+            const uint64_t vis = tree_tile ? s_anc[node] : prefix;
 #pragma unroll
-                for (int c = 0; c < 64; ++c) {
-                    const bool ok = tree_tile ? ((anc >> c) & 1ull) != 0 : (c < n_valid);
-                    sv[c] = ok ? sv[c] : -INFINITY;
-                }
-            }
+            for (int c = 0; c < 64; ++c) sv[c] = ((vis >> c) & 1ull) ? sv[c] : -INFINITY;
             float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
             for (int c = 0; c < 64; ++c) mx4[c & 3] = fmaxf(mx4[c & 3], sv[c]);
@@ -512,6 +540,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (tree_cta && rt == 0 && threadIdx.x == 0 && *s_bad) report(a.status, CLOVER_ERR_BAD_TREE);
     if (n_split > 1) {
         // -------------------------------------------- split merge over DSMEM
+        __syncwarp();
+        cluster_wait_acquire();               // every CTA's barriers exist
         // announce this CTA's partial to every CTA of the cluster
         if (threadIdx.x < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_ready), threadIdx.x));
         const bool ready = __syncthreads_and(mbar_wait_cluster(m_ready, 0, kWaitNs));
@@ -585,6 +615,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (threadIdx.x < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_done), threadIdx.x));
         if (!__syncthreads_and(mbar_wait_cluster(m_done, 0, kWaitNs))) *s_abort = 1;
     }
+    // the appended tree K/V is in global memory before the CTA exits
+    if (appender && (warp == kKProducerWarp || warp == kVProducerWarp) && lane == 0) bulk_wait_group0();
     if (*s_abort && threadIdx.x == 0) report(a.status, CLOVER_ERR_TIMEOUT);
 }
 
@@ -593,13 +625,13 @@ struct TcLaunchCache {
     int max_clusters[kMaxCluster + 1] = {0};   // co-resident clusters per cluster size (0: not queried)
 };
 
-template <int D>
+template <int D, int QR>
 int max_active_clusters(int n, TcLaunchCache &cache) {
     if (cache.max_clusters[n] == 0) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(1, n, n);
         cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = TcSmem<D>::alloc;
+        cfg.dynamicSmemBytes = TcSmem<D, QR>::alloc;
         cudaLaunchAttribute attr;
         attr.id = cudaLaunchAttributeClusterDimension;
         attr.val.clusterDim.x = 1;
@@ -608,7 +640,7 @@ int max_active_clusters(int n, TcLaunchCache &cache) {
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
         int num = 0;
-        if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D>, &cfg) != cudaSuccess) {
+        if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D, QR>, &cfg) != cudaSuccess) {
             cudaGetLastError();
             num = -1;
         }
@@ -617,12 +649,12 @@ int max_active_clusters(int n, TcLaunchCache &cache) {
     return cache.max_clusters[n];
 }
 
-template <int D>
+template <int D, int QR>
 cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     static unsigned char done[64];
     static TcLaunchCache caches[64];
-    auto kernel = tree_attn_tc_kernel<D>;
-    cudaError_t err = ensure_smem_attr(kernel, TcSmem<D>::alloc, done);
+    auto kernel = tree_attn_tc_kernel<D, QR>;
+    cudaError_t err = ensure_smem_attr(kernel, TcSmem<D, QR>::alloc, done);
     if (err != cudaSuccess) return err;
     int dev = 0;
     if ((err = cudaGetDevice(&dev)) != cudaSuccess) return err;
@@ -636,7 +668,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     int n = 1;
     for (int c = kMaxCluster; c >= 2; --c) {
         if (c > by_len || base * c > cache.sms) continue;
-        if (max_active_clusters<D>(c, cache) >= base) {
+        if (max_active_clusters<D, QR>(c, cache) >= base) {
             n = c;
             break;
         }
@@ -651,12 +683,15 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     if (G > 256 || box_nodes > 256) box_nodes = 0;
     a.q_box_nodes = box_nodes;
 
-    CUtensorMap kc, vc, kn, vn, qm;
+    CUtensorMap kc, vc, kn, vn, qm, ks, vs;
     const uint64_t e = 2;
     if (!make_tmap_bf16_3d(&kc, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
         !make_tmap_bf16_3d(&vc, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
         !make_tmap_bf16_3d(&kn, a.k_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) ||
-        !make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN))
+        !make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) ||
+        // the append: T rows of one (sequence, head) plane of the cache
+        !make_tmap_bf16_3d(&ks, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, a.T, 1) ||
+        !make_tmap_bf16_3d(&vs, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, a.T, 1))
         return cudaErrorInvalidValue;
     if (box_nodes > 0) {
         if (!make_tmap_bf16_3d(&qm, a.q, D, a.Hq, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hq * D * e, 64, G, box_nodes))
@@ -668,7 +703,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.row_tiles, n, a.B * a.Hkv);
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = TcSmem<D>::alloc;
+    cfg.dynamicSmemBytes = TcSmem<D, QR>::alloc;
     cfg.stream = stream;
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeClusterDimension;
@@ -677,7 +712,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     attr.val.clusterDim.z = 1;
     cfg.attrs = &attr;
     cfg.numAttrs = n > 1 ? 1 : 0;
-    err = cudaLaunchKernelEx(&cfg, kernel, kc, vc, kn, vn, qm, a);
+    err = cudaLaunchKernelEx(&cfg, kernel, kc, vc, kn, vn, qm, ks, vs, a);
     if (err != cudaSuccess) return err;
     return cudaGetLastError();
 }
@@ -687,7 +722,8 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
 int tc_row_tile() { return BM; }
 
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream) {
-    return a.D == 64 ? launch<64>(a, stream) : launch<128>(a, stream);
+    if (a.rows <= 64) return a.D == 64 ? launch<64, 64>(a, stream) : launch<128, 64>(a, stream);
+    return a.D == 64 ? launch<64, 128>(a, stream) : launch<128, 128>(a, stream);
 }
 
 }  // namespace clover
