@@ -102,6 +102,8 @@ __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_saddr) {
 }
 
 // Bounded wait that acquires at cluster scope (sees the arriving CTAs' writes).
+// The waiting thread spins (the suspend hint does not park it here), so one
+// thread of a CTA waits and the others block on a CTA barrier.
 __device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, uint64_t limit_ns) {
     auto try_once = [&]() {
         uint32_t ok;
@@ -121,19 +123,29 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity
     return false;
 }
 
-__device__ __forceinline__ float4 ld_dsmem_f4(uint32_t cluster_saddr) {
-    float4 v;
-    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(cluster_saddr)
-                 : "memory");
-    return v;
+// Non-blocking test of a phase, acquiring at cluster scope when it is complete
+// (for threads that learn of the completion from another thread of the CTA).
+__device__ __forceinline__ bool mbar_test_cluster(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
 }
 
-__device__ __forceinline__ float2 ld_dsmem_f2(uint32_t cluster_saddr) {
-    float2 v;
-    asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(cluster_saddr) : "memory");
-    return v;
+// Bulk copy (the TMA engine) of `bytes` from this CTA's shared memory to the
+// shared memory of a CTA of the cluster; completes as transaction bytes on that
+// CTA's mbarrier.  Addresses 16-byte aligned, size a multiple of 16.
+__device__ __forceinline__ void bulk_copy_to_cluster(uint32_t dst_cluster_saddr, const void *src, uint32_t bytes,
+                                                     uint32_t bar_cluster_saddr) {
+    asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     dst_cluster_saddr),
+                 "r"(smem_u32(src)), "r"(bytes), "r"(bar_cluster_saddr)
+                 : "memory");
 }
 
 // --------------------------------------------------------------------- TMA

@@ -65,23 +65,88 @@ struct TcSmem {
     static constexpr int q_off = 0;
     static constexpr int k_off = q_off + q_bytes;
     static constexpr int v_off = k_off + NSK * kv_bytes;
-    static constexpr int ml_off = v_off + NSV * kv_bytes;          // merge: (m, l) per row [BM]
-    static constexpr int bar_off = ml_off + BM * 8;
+    static constexpr int bar_off = v_off + NSV * kv_bytes;
     static constexpr int n_bars = 2 * NSK + 2 * NSV + 11;
     static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad flags
     static constexpr int anc_off = misc_off + 16;                  // ancestor masks [64]
     static constexpr int total = anc_off + kMaxTreeNodes * 8;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
-    // after the key loop the K/V rings hold this CTA's partial O (fp32, rows
-    // padded to D + 4 floats)
+    // After the key loop the K ring holds this CTA's partial result, one fp32
+    // row of D + 4 floats per query row (O, then m and l in the padding), and
+    // the V ring receives the other splits' partials of the rows this CTA
+    // merges: [n_split][rows per split][D + 4].
     static constexpr int po_stride = D + 4;
-    static_assert(QR * po_stride * 4 <= (NSK + NSV) * kv_bytes, "partial O must fit in the K/V rings");
+    static_assert(QR * po_stride * 4 <= NSK * kv_bytes, "partial result must fit in the K ring");
+    static_assert((QR + kMaxCluster - 1) * po_stride * 4 <= NSV * kv_bytes, "received partials must fit in the V ring");
     static_assert(alloc <= 227 * 1024, "shared memory budget");
 };
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+__device__ __forceinline__ float rcp_approx(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// Merge of the NS split partials of rows [r0, r1) of a tile (Section 2.2's
+// attention over the whole key range, from per-range partial softmax results):
+//   O = sum_k 2^(m_k - M) O_k / sum_k 2^(m_k - M) l_k,  M = max_k m_k.
+// Row rr of split k is `own` (this CTA's) or row (k * per + rr - r0) of `recv`;
+// each row holds O (D floats), then m and l.  A thread takes one (row, 4
+// columns) item at a time.  NS is a template argument so the whole item is
+// one short chain of independent loads and arithmetic (with few warps per
+// SM, the latency of a long chain is not hidden).
+template <int D, int NS>
+__device__ __forceinline__ void merge_rows(const float *own, const float *recv, int po_stride, int split, int per,
+                                           int r0, int r1, int row0, const AttnArgs &a, int b, int g,
+                                           __nv_bfloat16 *out) {
+    const int n_items = (r1 - r0) * (D / 4);
+    const float inv_g = 1.f / (float)a.G;
+    for (int e = threadIdx.x; e < n_items; e += blockDim.x) {
+        const int rr = r0 + e / (D / 4);
+        const int c4 = (e % (D / 4)) * 4;
+        float2 ml[NS];
+        float4 x[NS];
+#pragma unroll
+        for (int k = 0; k < NS; ++k) {
+            const float *row = (k == split) ? own + rr * po_stride : recv + (k * per + rr - r0) * po_stride;
+            ml[k] = *reinterpret_cast<const float2 *>(row + D);
+            x[k] = *reinterpret_cast<const float4 *>(row + c4);
+        }
+        float M = ml[0].x;
+#pragma unroll
+        for (int k = 1; k < NS; ++k) M = fmaxf(M, ml[k].x);
+        float w[NS];
+        float lsum = 0.f;
+#pragma unroll
+        for (int k = 0; k < NS; ++k) {
+            w[k] = (ml[k].x == -INFINITY) ? 0.f : ex2_approx(ml[k].x - M);
+            lsum = fmaf(w[k], ml[k].y, lsum);
+        }
+        const float inv = rcp_approx(lsum);
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int k = 0; k < NS; ++k) {
+            const float wk = w[k] * inv;
+            acc.x = fmaf(wk, x[k].x, acc.x);
+            acc.y = fmaf(wk, x[k].y, acc.y);
+            acc.z = fmaf(wk, x[k].z, acc.z);
+            acc.w = fmaf(wk, x[k].w, acc.w);
+        }
+        // row R = node * G + head-in-group; (R + 1/2) / G is never within
+        // float rounding of an integer, so the truncation is exact
+        const int R = row0 + rr;
+        const int i = __float2int_rz(((float)R + 0.5f) * inv_g);
+        const int h = g * a.G + (R - i * a.G);
+        uint2 w2;
+        w2.x = pack_bf16x2(acc.x, acc.y);
+        w2.y = pack_bf16x2(acc.z, acc.w);
+        *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c4) = w2;
+    }
 }
 
 template <int D, int QR>
@@ -94,7 +159,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr int NSK = S::NSK;
     constexpr int NSV = S::NSV;
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    // base rounded up to 1024 bytes by pointer arithmetic on the shared array,
+    // so that every access below stays a shared-memory access
+    uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     uint8_t *sQ = sm + S::q_off;
     uint8_t *sK = sm + S::k_off;
     uint8_t *sV = sm + S::v_off;
@@ -108,8 +175,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t *o_full = p_full + 2;            // [2] the tile's P.V product is done
     uint64_t *mma_done = o_full + 2;
     uint64_t *q_full = mma_done + 1;
-    uint64_t *m_ready = q_full + 1;           // partials of all cluster CTAs are in place
-    uint64_t *m_done = m_ready + 1;           // all cluster CTAs have read this CTA's partial
+    uint64_t *m_free = q_full + 1;            // every CTA of the cluster is out of its key loop
+    uint64_t *m_done = m_free + 1;            // every CTA has received this CTA's partial rows
+    uint64_t *m_data = m_done + 1;            // the other splits' partials of this CTA's rows are here
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(sm + S::misc_off);
     volatile int *s_abort = reinterpret_cast<volatile int *>(sm + S::misc_off + 4);
     bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 8);
@@ -205,8 +273,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             mbar_init(mma_done, 1);
             mbar_init(q_full, 1);
-            mbar_init(m_ready, n_split);
+            mbar_init(m_free, n_split);
             mbar_init(m_done, n_split);
+            mbar_init(m_data, 1);
+            if (n_split > 1) {
+                // every other split sends this CTA its rows [r0, r1) of the tile
+                const int per = (rows_here + n_split - 1) / n_split;
+                const int mine = max(0, min(rows_here, (split + 1) * per) - split * per);
+                mbar_arrive_expect_tx(m_data, (uint32_t)((n_split - 1) * mine * S::po_stride * 4));
+            }
             *s_abort = 0;
             *s_bad = false;
             fence_barrier_init();
@@ -487,26 +562,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncthreads();
     tc_fence_after();
+    if (n_split > 1) {
+        // this CTA's rings are free: the other splits may send their partials
+        cluster_wait_acquire();               // every CTA's barriers exist
+        if (warp == 1 && lane < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_free), lane));
+    }
     __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(a.out);
     const bool row_ok = softmax_warp && r < rows_here;
-    float *part_o = reinterpret_cast<float *>(sK);            // [BM][D + 4] fp32, this CTA's partial
-    float2 *part_ml = reinterpret_cast<float2 *>(sm + S::ml_off);
+    float *part_o = reinterpret_cast<float *>(sK);            // [QR][D + 4] fp32, this CTA's partial
+    float *recv = reinterpret_cast<float *>(sV);              // [n_split][per][D + 4]
     if (softmax_warp) {
         const int R = rt * BM + r;
         const int i = row_ok ? R / a.G : 0;
         const int h = row_ok ? g * a.G + (R % a.G) : 0;
         const float inv = (n_split == 1 && o_ready) ? 1.f / l_run : 1.f;
-#pragma unroll 1
-        for (int cc = 0; cc < D / 32; ++cc) {
-            float x[32];
-            if (o_ready) {
-                tmem_ld32(tO + lane_base + cc * 32, x);
-                tmem_wait_ld();
-            } else {
-#pragma unroll
-                for (int c = 0; c < 32; ++c) x[c] = 0.f;
-            }
-            if (!row_ok) continue;
+        // 32 columns of the row: the output (one split) or the partial row
+        auto emit = [&](int cc, const float (&x)[32]) {
             if (n_split == 1) {
                 __nv_bfloat16 *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D + cc * 32;
 #pragma unroll
@@ -524,8 +595,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int c = 0; c < 32; c += 4)
                     *reinterpret_cast<float4 *>(po + c) = make_float4(x[c], x[c + 1], x[c + 2], x[c + 3]);
             }
+        };
+        // two TMEM loads in flight per wait
+#pragma unroll 1
+        for (int cc = 0; cc < D / 32; cc += 2) {
+            float x0[32], x1[32];
+            if (o_ready) {
+                tmem_ld32(tO + lane_base + cc * 32, x0);
+                tmem_ld32(tO + lane_base + cc * 32 + 32, x1);
+                tmem_wait_ld();
+            } else {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) x0[c] = x1[c] = 0.f;
+            }
+            if (row_ok) {
+                emit(cc, x0);
+                emit(cc + 1, x1);
+            }
         }
-        if (row_ok) part_ml[r] = make_float2(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f);
+        if (row_ok && n_split > 1)
+            *reinterpret_cast<float2 *>(part_o + r * S::po_stride + D) =
+                make_float2(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f);
+        fence_proxy_async_smem();             // the bulk copies below read these rows
     }
 
     // every TMEM access and MMA is finished before TMEM is released
@@ -539,81 +630,55 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (tree_cta && rt == 0 && threadIdx.x == 0 && *s_bad) report(a.status, CLOVER_ERR_BAD_TREE);
     if (n_split > 1) {
-        // -------------------------------------------- split merge over DSMEM
-        __syncwarp();
-        cluster_wait_acquire();               // every CTA's barriers exist
-        // announce this CTA's partial to every CTA of the cluster
-        if (threadIdx.x < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_ready), threadIdx.x));
-        const bool ready = __syncthreads_and(mbar_wait_cluster(m_ready, 0, kWaitNs));
-        if (ready) {
-            // this CTA merges rows [r0, r1) of the tile.  A thread takes items
-            // (row, 4 columns) in batches of kBatch and issues every split's
-            // (m, l) and columns of the whole batch before using any of them,
-            // so a batch costs one distributed-shared-memory round trip.
-            constexpr int kBatch = 3;
-            const int per = (rows_here + n_split - 1) / n_split;
-            const int r0 = split * per;
-            const int r1 = min(rows_here, r0 + per);
-            const int n_items = (r1 - r0) * (D / 4);
-            const uint32_t ml_base = smem_u32(part_ml);
-            const uint32_t o_base = smem_u32(part_o);
-            for (int e0 = threadIdx.x; e0 < n_items; e0 += kThreads * kBatch) {
-                float2 ml[kBatch][kMaxCluster];
-                float4 x[kBatch][kMaxCluster];
-#pragma unroll
-                for (int t = 0; t < kBatch; ++t) {
-                    const int e = e0 + t * kThreads;
-                    const int rr = r0 + e / (D / 4);
-                    const int c4 = (e % (D / 4)) * 4;
-#pragma unroll
-                    for (int k = 0; k < kMaxCluster; ++k) {
-                        if (e < n_items && k < n_split) {
-                            ml[t][k] = ld_dsmem_f2(mapa_shared(ml_base + rr * 8, k));
-                            x[t][k] = ld_dsmem_f4(mapa_shared(o_base + (rr * S::po_stride + c4) * 4, k));
-                        }
-                    }
+        // ------------------------------------------ split merge in the cluster
+        // CTA `split` merges rows [r0, r1) of the tile.  Once every CTA is out
+        // of its key loop, each sends every other CTA that CTA's rows of its
+        // partial with one bulk copy into the receiver's V ring (completing on
+        // the receiver's m_data), then merges its own rows from shared memory.
+        const int per = (rows_here + n_split - 1) / n_split;
+        const int r0 = split * per;
+        const int r1 = min(rows_here, r0 + per);
+        constexpr uint32_t row_bytes = S::po_stride * 4;
+        bool ok = true;
+        if (threadIdx.x == 0) {
+            if ((ok = mbar_wait_cluster(m_free, 0, kWaitNs))) {
+                for (int k = 0; k < n_split; ++k) {
+                    const int k0 = k * per;
+                    const int k1 = min(rows_here, k0 + per);
+                    if (k == split || k1 <= k0) continue;
+                    bulk_copy_to_cluster(mapa_shared(smem_u32(recv) + split * per * row_bytes, k),
+                                         part_o + k0 * S::po_stride, (k1 - k0) * row_bytes,
+                                         mapa_shared(smem_u32(m_data), k));
                 }
-#pragma unroll
-                for (int t = 0; t < kBatch; ++t) {
-                    const int e = e0 + t * kThreads;
-                    if (e >= n_items) continue;
-                    const int rr = r0 + e / (D / 4);
-                    const int c4 = (e % (D / 4)) * 4;
-                    float M = -INFINITY;
-#pragma unroll
-                    for (int k = 0; k < kMaxCluster; ++k)
-                        if (k < n_split) M = fmaxf(M, ml[t][k].x);
-                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                    float lsum = 0.f;
-#pragma unroll
-                    for (int k = 0; k < kMaxCluster; ++k) {
-                        if (k < n_split) {
-                            const float w = (ml[t][k].x == -INFINITY) ? 0.f : exp2f(ml[t][k].x - M);
-                            lsum = fmaf(w, ml[t][k].y, lsum);
-                            acc.x = fmaf(w, x[t][k].x, acc.x);
-                            acc.y = fmaf(w, x[t][k].y, acc.y);
-                            acc.z = fmaf(w, x[t][k].z, acc.z);
-                            acc.w = fmaf(w, x[t][k].w, acc.w);
-                        }
-                    }
-                    const float inv = 1.f / lsum;
-                    const int R = rt * BM + rr;
-                    const int i = R / a.G;
-                    const int h = g * a.G + (R % a.G);
-                    uint2 w2;
-                    w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-                    w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-                    *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c4) = w2;
-                }
+            }
+            if (ok) ok = mbar_wait_cluster(m_data, 0, kWaitNs);
+        }
+        // one thread waited; every thread acquires the received rows itself
+        const bool got = __syncthreads_and(ok) && mbar_test_cluster(m_data, 0);
+        // every partial row this CTA needs is here: its senders may exit
+        if (warp == 1 && lane < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_done), lane));
+        if (got) {
+            switch (n_split) {
+#define CLOVER_MERGE_CASE(NS) \
+    case NS: merge_rows<D, NS>(part_o, recv, S::po_stride, split, per, r0, r1, rt * BM, a, b, g, out); break;
+                CLOVER_MERGE_CASE(2)
+                CLOVER_MERGE_CASE(3)
+                CLOVER_MERGE_CASE(4)
+                CLOVER_MERGE_CASE(5)
+                CLOVER_MERGE_CASE(6)
+                CLOVER_MERGE_CASE(7)
+                CLOVER_MERGE_CASE(8)
+#undef CLOVER_MERGE_CASE
+                default: break;
             }
         } else {
             *s_abort = 1;
         }
-        // this CTA has finished reading every partial; wait until every CTA
-        // has finished reading this one's before its shared memory goes away
-        __syncthreads();
-        if (threadIdx.x < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_done), threadIdx.x));
-        if (!__syncthreads_and(mbar_wait_cluster(m_done, 0, kWaitNs))) *s_abort = 1;
+        // the copies reading this CTA's partial are complete before its
+        // shared memory goes away
+        ok = true;
+        if (threadIdx.x == 0) ok = mbar_wait_cluster(m_done, 0, kWaitNs);
+        if (!__syncthreads_and(ok)) *s_abort = 1;
     }
     // the appended tree K/V is in global memory before the CTA exits
     if (appender && (warp == kKProducerWarp || warp == kVProducerWarp) && lane == 0) bulk_wait_group0();
