@@ -15,6 +15,13 @@
  *   clover_kv_compact     moves the accepted nodes' K/V to the front of the
  *                         tree slots (an engine step the paper leaves implicit).
  *
+ * A second schedule of the same step: clover_verify_attn_ex with
+ * CLOVER_ATTN_NO_APPEND leaves the caches untouched, and clover_kv_commit then
+ * writes the accepted nodes' K/V straight from k_new/v_new.  The commit needs
+ * only the accept result, so it can run while the attention still runs (its
+ * writes, slots >= cache_len, are outside what the attention reads); the
+ * final cache equals that of the append + compact schedule.
+ *
  * Conventions shared by every entry point
  *   - All tensor pointers are DEVICE pointers owned by the caller; the library
  *     never allocates, frees or retains them.  Tensors are dense row-major.
@@ -116,6 +123,22 @@ CLOVER_API clover_status clover_verify_attn(const void *q, const void *k_new, co
                                  void *workspace, size_t ws_bytes,
                                  int32_t *status, void *stream);
 
+/* Flag of clover_verify_attn_ex: the call only reads k_cache/v_cache (no append). */
+#define CLOVER_ATTN_NO_APPEND 1u
+
+/*
+ * clover_verify_attn with flags: 0 is clover_verify_attn itself;
+ * CLOVER_ATTN_NO_APPEND skips the append, so slots >= cache_len[b] are neither
+ * read for the result nor written.  Other flag bits: CLOVER_ERR_INVALID_ARG.
+ */
+CLOVER_API clover_status clover_verify_attn_ex(const void *q, const void *k_new, const void *v_new,
+                                    void *k_cache, void *v_cache, const int32_t *cache_len,
+                                    const int32_t *parent, void *out,
+                                    int B, int T, int Hq, int Hkv, int D, int Lcap,
+                                    clover_dtype dtype, float scale,
+                                    void *workspace, size_t ws_bytes,
+                                    int32_t *status, void *stream, uint32_t flags);
+
 /* Bytes of device workspace clover_verify_accept needs (0 outside the limits). */
 CLOVER_API size_t clover_verify_accept_workspace_size(int B, int T, int V, clover_dtype dtype);
 
@@ -165,6 +188,27 @@ CLOVER_API clover_status clover_kv_compact(void *k_cache, void *v_cache, const i
                                 int32_t *new_cache_len, int32_t *src_index_out,
                                 int B, int T, int Hkv, int D, int Lcap, clover_dtype dtype,
                                 int32_t *status, void *stream);
+
+/*
+ * Commit of the accepted path straight from the tree's K/V (the engine step of
+ * clover_kv_compact without the append before it).  For every sequence b with
+ * L = cache_len[b] and a = accept_len[b]:
+ *   cache[b,g,L+j,:] <- new[b,path[b][j],g,:]  for j < a, every KV head g, K and V;
+ * slots < L are not touched.
+ *   k_cache, v_cache [B,Hkv,Lcap,D] dtype  out, 16-byte aligned
+ *   k_new, v_new     [B,T,Hkv,D]    dtype  in, 16-byte aligned
+ *   cache_len [B]        int32   length before the step (read only)
+ *   path, accept_len             as produced by clover_verify_accept
+ *   new_cache_len [B]    int32   out: L + a.  Must not overlap cache_len.
+ *   src_index_out [B,T]  int32   out: path[b][j] (a tree node) for j < a, else -1 (may be NULL)
+ * Errors: cache_len[b] + T > Lcap -> CLOVER_ERR_CAPACITY; a path entry outside
+ * [0, T) or an accept_len outside [1, T] -> CLOVER_ERR_INVALID_ARG (device bits).
+ */
+CLOVER_API clover_status clover_kv_commit(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
+                               const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
+                               int32_t *new_cache_len, int32_t *src_index_out,
+                               int B, int T, int Hkv, int D, int Lcap, clover_dtype dtype,
+                               int32_t *status, void *stream);
 
 /*
  * Bytes of the static device scratch buffer behind clover_verify_attn_noalloc.

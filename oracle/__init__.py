@@ -59,8 +59,10 @@ def _load():
             lib.oracle_accept_walk.argtypes = [P, P, P, I, I, P, P, P]
             lib.oracle_append_tree_kv.argtypes = [P, P, P, P, P, I, I, I, I, I, I]
             lib.oracle_kv_compact.argtypes = [P, P, P, P, P, I, I, I, I, I, I, P]
+            lib.oracle_kv_commit.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P]
             for f in (lib.oracle_tree_mask, lib.oracle_tree_attention, lib.oracle_argmax,
-                      lib.oracle_accept_walk, lib.oracle_append_tree_kv, lib.oracle_kv_compact):
+                      lib.oracle_accept_walk, lib.oracle_append_tree_kv, lib.oracle_kv_compact,
+                      lib.oracle_kv_commit):
                 f.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -188,6 +190,21 @@ def kv_compact(k_cache, v_cache, cache_len, path, accept_len):
     src = torch.empty((B, T), dtype=torch.int32)
     _check(_load().oracle_kv_compact(_p(k_cache), _p(v_cache), _p(cache_len), _p(pa), _p(al), B, T,
                                      Hkv, D, Lcap, k_cache.element_size(), _p(src)))
+    return src
+
+
+def kv_commit(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len):
+    """In place on k_cache/v_cache/cache_len (int32): slot L+j <- node path[j]
+    of k_new/v_new; returns src_index [B,T] (the nodes, -1 past a)."""
+    assert k_cache.is_contiguous() and v_cache.is_contiguous() and cache_len.dtype == torch.int32
+    B, Hkv, Lcap, D = k_cache.shape
+    kn, vn = _cpu(k_new), _cpu(v_new)
+    pa = _cpu(path.to(torch.int32))
+    al = _cpu(accept_len.to(torch.int32))
+    T = pa.shape[1]
+    src = torch.empty((B, T), dtype=torch.int32)
+    _check(_load().oracle_kv_commit(_p(k_cache), _p(v_cache), _p(kn), _p(vn), _p(cache_len), _p(pa), _p(al), B, T,
+                                    Hkv, D, Lcap, k_cache.element_size(), _p(src)))
     return src
 
 

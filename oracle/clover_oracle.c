@@ -319,3 +319,39 @@ int oracle_kv_compact(void *k_cache, void *v_cache, int32_t *cache_len, const in
     }
     return ORACLE_OK;
 }
+
+/*
+ * Commit from the tree's K/V (the same end state as append + compaction):
+ * for j = 0..a-1, slot L+j of every KV head receives k_new/v_new of node
+ * path[j]; src_index[b][j] = path[j] (-1 past a); cache_len[b] += a.
+ */
+int oracle_kv_commit(void *k_cache, void *v_cache, const void *k_new, const void *v_new, int32_t *cache_len,
+                     const int32_t *path, const int32_t *accept_len, int B, int T, int Hkv, int D, int Lcap,
+                     int elem_bytes, int32_t *src_index)
+{
+    const size_t row = (size_t)D * elem_bytes;
+    for (int b = 0; b < B; ++b) {
+        const int L = cache_len[b];
+        const int a = accept_len[b];
+        if (a < 1 || a > T || L < 0 || L + T > Lcap) return ORACLE_BAD_ARG;
+        for (int j = 0; j < a; ++j)
+            if (path[(int64_t)b * T + j] < 0 || path[(int64_t)b * T + j] >= T) return ORACLE_BAD_ARG;
+    }
+    for (int b = 0; b < B; ++b) {
+        const int L = cache_len[b];
+        const int a = accept_len[b];
+        for (int j = 0; j < T; ++j) src_index[(int64_t)b * T + j] = -1;
+        for (int j = 0; j < a; ++j) {
+            const int node = path[(int64_t)b * T + j];
+            src_index[(int64_t)b * T + j] = node;
+            for (int g = 0; g < Hkv; ++g) {
+                const int64_t src = ((int64_t)b * T + node) * Hkv + g;
+                const int64_t dst = ((int64_t)b * Hkv + g) * Lcap + L + j;
+                memcpy((char *)k_cache + dst * row, (const char *)k_new + src * row, row);
+                memcpy((char *)v_cache + dst * row, (const char *)v_new + src * row, row);
+            }
+        }
+        cache_len[b] = L + a;
+    }
+    return ORACLE_OK;
+}

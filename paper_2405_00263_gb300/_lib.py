@@ -22,11 +22,16 @@ EXPORTS = (
     "clover_status_string",
     "clover_verify_attn_workspace_size",
     "clover_verify_attn",
+    "clover_verify_attn_ex",
     "clover_verify_accept_workspace_size",
     "clover_verify_accept",
     "clover_kv_compact",
+    "clover_kv_commit",
     "clover_verify_attn_noalloc",
 )
+
+# Flag of clover_verify_attn_ex (CLOVER_ATTN_NO_APPEND in include/clover_verify.h).
+ATTN_NO_APPEND = 1
 
 # Bytes of the static scratch buffer behind clover_verify_attn_noalloc
 # (CLOVER_NOALLOC_SCRATCH_BYTES in include/clover_verify.h).
@@ -60,12 +65,17 @@ def load(build_if_missing: bool = False):
         lib.clover_verify_attn_workspace_size.restype = Z
         lib.clover_verify_attn.argtypes = [P, P, P, P, P, P, P, P, I, I, I, I, I, I, I, F, P, Z, P, P]
         lib.clover_verify_attn.restype = I
+        lib.clover_verify_attn_ex.argtypes = [P, P, P, P, P, P, P, P, I, I, I, I, I, I, I, F, P, Z, P, P,
+                                              ctypes.c_uint32]
+        lib.clover_verify_attn_ex.restype = I
         lib.clover_verify_accept_workspace_size.argtypes = [I, I, I, I]
         lib.clover_verify_accept_workspace_size.restype = Z
         lib.clover_verify_accept.argtypes = [P, P, P, I, I, I, I, P, P, P, P, P, Z, P, P]
         lib.clover_verify_accept.restype = I
         lib.clover_kv_compact.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P, P]
         lib.clover_kv_compact.restype = I
+        lib.clover_kv_commit.argtypes = [P, P, P, P, P, P, P, P, P, I, I, I, I, I, I, P, P]
+        lib.clover_kv_commit.restype = I
         lib.clover_verify_attn_noalloc.argtypes = [P, P, P, P, P, P, P, P, I, I, I, I, I, I, I, F, P, P]
         lib.clover_verify_attn_noalloc.restype = I
         _lib = lib

@@ -90,8 +90,10 @@ def clover_verify_accept_workspace_size(B, T, V, dtype) -> int:
 
 
 def clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, scale=0.0,
-                       workspace=None, status=None, stream=None):
-    """Tree-masked attention; appends k_new/v_new at cache slots [L, L+T)."""
+                       workspace=None, status=None, stream=None, append=True):
+    """Tree-masked attention; with ``append`` (clover_verify_attn) it also
+    writes k_new/v_new at cache slots [L, L+T), without it
+    (clover_verify_attn_ex with CLOVER_ATTN_NO_APPEND) the caches are only read."""
     B, T, Hq, D = q.shape
     Hkv, Lcap = k_cache.shape[1], k_cache.shape[2]
     dt = q.dtype
@@ -106,12 +108,15 @@ def clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out
         _check(status, (1,), torch.int32, "status")
     _dev(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, workspace, status)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    code = _lib.load().clover_verify_attn(
-        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(cache_len), _ptr(parent),
-        _ptr(out), B, T, Hq, Hkv, D, Lcap, dtype_code(dt), float(scale), _ptr(workspace), ws_bytes,
-        _ptr(status), _stream(stream))
+    args = (_ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(cache_len), _ptr(parent),
+            _ptr(out), B, T, Hq, Hkv, D, Lcap, dtype_code(dt), float(scale), _ptr(workspace), ws_bytes,
+            _ptr(status), _stream(stream))
+    if append:
+        code = _lib.load().clover_verify_attn(*args)
+    else:
+        code = _lib.load().clover_verify_attn_ex(*args, _lib.ATTN_NO_APPEND)
     if code != OK:
-        raise CloverError(code, "clover_verify_attn")
+        raise CloverError(code, "clover_verify_attn" if append else "clover_verify_attn_ex")
 
 
 def clover_verify_attn_noalloc(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, scale=0.0,
@@ -183,19 +188,56 @@ def clover_kv_compact(k_cache, v_cache, cache_len, path, accept_len, new_cache_l
         raise CloverError(code, "clover_kv_compact")
 
 
+def clover_kv_commit(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len, new_cache_len,
+                     src_index_out=None, status=None, stream=None):
+    """Writes the accepted nodes' K/V from k_new/v_new to slots [L, L+a);
+    new_cache_len = L + a."""
+    B, Hkv, Lcap, D = k_cache.shape
+    T = path.shape[1]
+    _check(v_cache, (B, Hkv, Lcap, D), k_cache.dtype, "v_cache")
+    _check(k_new, (B, T, Hkv, D), k_cache.dtype, "k_new")
+    _check(v_new, (B, T, Hkv, D), k_cache.dtype, "v_new")
+    _check(cache_len, (B,), torch.int32, "cache_len")
+    _check(path, (B, T), torch.int32, "path")
+    _check(accept_len, (B,), torch.int32, "accept_len")
+    _check(new_cache_len, (B,), torch.int32, "new_cache_len")
+    if src_index_out is not None:
+        _check(src_index_out, (B, T), torch.int32, "src_index_out")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len, new_cache_len, src_index_out, status)
+    code = _lib.load().clover_kv_commit(
+        _ptr(k_cache), _ptr(v_cache), _ptr(k_new), _ptr(v_new), _ptr(cache_len), _ptr(path), _ptr(accept_len),
+        _ptr(new_cache_len), _ptr(src_index_out), B, T, Hkv, D, Lcap, dtype_code(k_cache.dtype), _ptr(status),
+        _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_kv_commit")
+
+
 class VerifyStep:
     """Device buffers for repeated verification steps of one shape.
 
     Owns the two zero-initialised workspaces and the output tensors.  ``run``
-    issues the three library calls: the attention on ``stream`` and, at the
-    same time, the argmax/acceptance walk on a side stream (the two read
-    disjoint inputs); the compaction follows on ``stream`` once both are done.
-    With ``concurrent=False`` all three run in order on ``stream``.
+    issues the three library calls of one step.  Schedules:
+
+    ``"commit"`` (default): the attention (caches only read) on ``stream`` and,
+    at the same time on a side stream, the argmax/acceptance walk followed by
+    clover_kv_commit, which writes the accepted K/V from k_new/v_new to slots
+    [L, L+a) -- outside what the attention reads -- so no call waits for the
+    attention but the end of the step.
+    ``"compact"``: the attention appends the tree K/V while the accept call
+    runs on the side stream; clover_kv_compact follows on ``stream`` once both
+    are done.
+    With ``concurrent=False`` the calls run in order on ``stream``.
+    ``src_index`` holds tree nodes (commit) or cache slots (compact).
     """
 
-    def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda", concurrent=True):
+    def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda", concurrent=True, schedule="commit"):
+        if schedule not in ("commit", "compact"):
+            raise ValueError(f"unknown schedule {schedule!r}")
         self.shape = dict(B=B, T=T, Hq=Hq, Hkv=Hkv, D=D, Lcap=Lcap, V=V)
         self.dtype = dtype
+        self.schedule = schedule
         dev = torch.device(device)
         ws_a = clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, Lcap, dtype)
         ws_b = clover_verify_accept_workspace_size(B, T, V, dtype)
@@ -210,7 +252,7 @@ class VerifyStep:
         self.new_cache_len = torch.empty((B,), **i32)
         self.src_index = torch.empty((B, T), **i32)
         self.status = torch.zeros((1,), **i32)
-        # the accept call gets its own status word so that the two concurrent
+        # the side stream's calls get their own status word so that concurrent
         # calls never update one word at the same time from two streams
         self.status_accept = torch.zeros((1,), **i32)
         self.side = torch.cuda.Stream(device=dev) if concurrent else None
@@ -226,43 +268,37 @@ class VerifyStep:
 
     def run(self, q, k_new, v_new, k_cache, v_cache, cache_len, parent, cand, logits, scale=0.0,
             stream=None, events=None):
-        """One step.  ``events`` (optional, four CUDA events) brackets the
-        attention (0-1) and the compaction (2-3) on ``stream``; the accept call
-        is bracketed by ``events[4:6]`` on the side stream when given."""
+        """One step.  ``events`` (optional, six CUDA events) brackets the
+        attention (0-1), the commit or compaction (2-3) and the accept call
+        (4-5), each on the stream it runs on."""
         stream = stream if stream is not None else torch.cuda.current_stream()
-        if self.side is None:
-            if events:
-                events[0].record(stream)
-            clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
-                               workspace=self.ws_attn, status=self.status, stream=stream)
-            if events:
-                events[1].record(stream)
-                if len(events) > 5:
-                    events[4].record(stream)
-            clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
-                                 self.ws_accept, status=self.status_accept, stream=stream)
-            if events and len(events) > 5:
-                events[5].record(stream)
-        else:
+        commit = self.schedule == "commit"
+        side = self.side if self.side is not None else stream
+        ev = (lambda i, st: events[i].record(st)) if events else (lambda i, st: None)
+        if self.side is not None:
             self._fork.record(stream)
             self.side.wait_event(self._fork)
-            if events:
-                events[0].record(stream)
-            clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
-                               workspace=self.ws_attn, status=self.status, stream=stream)
-            if events:
-                events[1].record(stream)
-                if len(events) > 5:
-                    events[4].record(self.side)
-            clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
-                                 self.ws_accept, status=self.status_accept, stream=self.side)
-            if events and len(events) > 5:
-                events[5].record(self.side)
-            self._join.record(self.side)
-            stream.wait_event(self._join)
-        if events:
-            events[2].record(stream)
-        clover_kv_compact(k_cache, v_cache, cache_len, self.path, self.accept_len, self.new_cache_len,
-                          self.src_index, status=self.status, stream=stream)
-        if events:
-            events[3].record(stream)
+        ev(0, stream)
+        clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
+                           workspace=self.ws_attn, status=self.status, stream=stream, append=not commit)
+        ev(1, stream)
+        ev(4, side)
+        clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
+                             self.ws_accept, status=self.status_accept, stream=side)
+        ev(5, side)
+        if commit:
+            ev(2, side)
+            clover_kv_commit(k_cache, v_cache, k_new, v_new, cache_len, self.path, self.accept_len,
+                             self.new_cache_len, self.src_index, status=self.status_accept, stream=side)
+            ev(3, side)
+            if self.side is not None:
+                self._join.record(self.side)
+                stream.wait_event(self._join)
+        else:
+            if self.side is not None:
+                self._join.record(self.side)
+                stream.wait_event(self._join)
+            ev(2, stream)
+            clover_kv_compact(k_cache, v_cache, cache_len, self.path, self.accept_len, self.new_cache_len,
+                              self.src_index, status=self.status, stream=stream)
+            ev(3, stream)

@@ -17,9 +17,10 @@ size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T, int V,
                           int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len, int32_t *bonus,
                           void *workspace, int32_t *status, cudaStream_t stream);
-cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const int32_t *cache_len, const int32_t *path,
-                              const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index, int B, int T,
-                              int Hkv, int D, int Lcap, int dtype, int32_t *status, cudaStream_t stream);
+cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
+                              const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
+                              int32_t *new_cache_len, int32_t *src_index, int B, int T, int Hkv, int D, int Lcap,
+                              int dtype, int32_t *status, cudaStream_t stream);
 
 namespace {
 
@@ -101,6 +102,31 @@ clover_status from_cuda(cudaError_t e) { return e == cudaSuccess ? CLOVER_OK : C
 
 using namespace clover;
 
+namespace {
+
+// Checks shared by clover_kv_compact and clover_kv_commit (k_new == v_new ==
+// nullptr for the compaction).
+clover_status check_commit(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
+                           const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
+                           int32_t *new_cache_len, int B, int T, int Hkv, int D, int Lcap, clover_dtype dtype,
+                           bool from_new) {
+    if (B < 0 || T < 1 || Hkv < 1 || Lcap < 1) return CLOVER_ERR_INVALID_ARG;
+    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
+    if (T > kMaxTreeNodes || (D != 64 && D != 128)) return CLOVER_ERR_UNSUPPORTED;
+    if (Lcap < T) return CLOVER_ERR_INVALID_ARG;
+    if (B > 65535 || Hkv > 65535) return CLOVER_ERR_UNSUPPORTED;
+    if (B == 0) return CLOVER_OK;
+    if (!k_cache || !v_cache || !cache_len || !path || !accept_len || !new_cache_len) return CLOVER_ERR_INVALID_ARG;
+    if (!aligned16(k_cache) || !aligned16(v_cache)) return CLOVER_ERR_INVALID_ARG;
+    if (from_new && (!k_new || !v_new || !aligned16(k_new) || !aligned16(v_new))) return CLOVER_ERR_INVALID_ARG;
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(cache_len), a1 = a0 + sizeof(int32_t) * (size_t)B;
+    const uintptr_t b0 = reinterpret_cast<uintptr_t>(new_cache_len), b1 = b0 + sizeof(int32_t) * (size_t)B;
+    if (a0 < b1 && b0 < a1) return CLOVER_ERR_INVALID_ARG;      // lengths are read by every CTA: no aliasing
+    return CLOVER_OK;
+}
+
+}  // namespace
+
 extern "C" {
 
 int clover_abi_version(void) { return kAbiVersion; }
@@ -129,6 +155,16 @@ clover_status clover_verify_attn(const void *q, const void *k_new, const void *v
                                  int B, int T, int Hq, int Hkv, int D, int Lcap, clover_dtype dtype,
                                  float scale, void *workspace, size_t ws_bytes, int32_t *status,
                                  void *stream) {
+    return clover_verify_attn_ex(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, B, T, Hq, Hkv, D,
+                                 Lcap, dtype, scale, workspace, ws_bytes, status, stream, 0u);
+}
+
+clover_status clover_verify_attn_ex(const void *q, const void *k_new, const void *v_new, void *k_cache,
+                                    void *v_cache, const int32_t *cache_len, const int32_t *parent, void *out,
+                                    int B, int T, int Hq, int Hkv, int D, int Lcap, clover_dtype dtype,
+                                    float scale, void *workspace, size_t ws_bytes, int32_t *status,
+                                    void *stream, uint32_t flags) {
+    if (flags & ~CLOVER_ATTN_NO_APPEND) return CLOVER_ERR_INVALID_ARG;
     const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype);
     if (s != CLOVER_OK) return s;
     if (B == 0) return CLOVER_OK;
@@ -160,6 +196,7 @@ clover_status clover_verify_attn(const void *q, const void *k_new, const void *v
     a.dtype = dtype;
     const float sc = scale > 0.f ? scale : 1.f / sqrtf((float)D);
     a.scale_log2 = sc * 1.4426950408889634f;
+    a.append = (flags & CLOVER_ATTN_NO_APPEND) ? 0 : 1;
     a.rows = T * a.G;
     a.row_tile = p.row_tile;
     a.row_tiles = p.row_tiles;
@@ -198,23 +235,28 @@ clover_status clover_verify_accept(const void *logits, const int32_t *cand, cons
                                    bonus_token, workspace, status, static_cast<cudaStream_t>(stream)));
 }
 
+clover_status clover_kv_commit(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
+                               const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
+                               int32_t *new_cache_len, int32_t *src_index_out, int B, int T, int Hkv, int D,
+                               int Lcap, clover_dtype dtype, int32_t *status, void *stream) {
+    const clover_status s = check_commit(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len, new_cache_len,
+                                         B, T, Hkv, D, Lcap, dtype, true);
+    if (s != CLOVER_OK || B == 0) return s;
+    return from_cuda(launch_kv_compact(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len, new_cache_len,
+                                       src_index_out, B, T, Hkv, D, Lcap, dtype, status,
+                                       static_cast<cudaStream_t>(stream)));
+}
+
 clover_status clover_kv_compact(void *k_cache, void *v_cache, const int32_t *cache_len, const int32_t *path,
                                 const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index_out, int B,
                                 int T, int Hkv, int D, int Lcap, clover_dtype dtype, int32_t *status,
                                 void *stream) {
-    if (B < 0 || T < 1 || Hkv < 1 || Lcap < 1) return CLOVER_ERR_INVALID_ARG;
-    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
-    if (T > kMaxTreeNodes || (D != 64 && D != 128)) return CLOVER_ERR_UNSUPPORTED;
-    if (Lcap < T) return CLOVER_ERR_INVALID_ARG;
-    if (B > 65535 || Hkv > 65535) return CLOVER_ERR_UNSUPPORTED;
-    if (B == 0) return CLOVER_OK;
-    if (!k_cache || !v_cache || !cache_len || !path || !accept_len || !new_cache_len) return CLOVER_ERR_INVALID_ARG;
-    if (!aligned16(k_cache) || !aligned16(v_cache)) return CLOVER_ERR_INVALID_ARG;
-    const uintptr_t a0 = reinterpret_cast<uintptr_t>(cache_len), a1 = a0 + sizeof(int32_t) * (size_t)B;
-    const uintptr_t b0 = reinterpret_cast<uintptr_t>(new_cache_len), b1 = b0 + sizeof(int32_t) * (size_t)B;
-    if (a0 < b1 && b0 < a1) return CLOVER_ERR_INVALID_ARG;      // lengths are read by every CTA: no aliasing
-    return from_cuda(launch_kv_compact(k_cache, v_cache, cache_len, path, accept_len, new_cache_len, src_index_out,
-                                       B, T, Hkv, D, Lcap, dtype, status, static_cast<cudaStream_t>(stream)));
+    const clover_status s = check_commit(k_cache, v_cache, nullptr, nullptr, cache_len, path, accept_len,
+                                         new_cache_len, B, T, Hkv, D, Lcap, dtype, false);
+    if (s != CLOVER_OK || B == 0) return s;
+    return from_cuda(launch_kv_compact(k_cache, v_cache, nullptr, nullptr, cache_len, path, accept_len,
+                                       new_cache_len, src_index_out, B, T, Hkv, D, Lcap, dtype, status,
+                                       static_cast<cudaStream_t>(stream)));
 }
 
 }  // extern "C"

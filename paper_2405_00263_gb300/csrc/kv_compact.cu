@@ -1,13 +1,17 @@
 // Commit of the accepted path to the KV cache: for sequence b with committed
-// length L and accepted nodes path[0..a-1], the K/V rows at slots L + path[j]
-// (where the attention kernel appended the tree's K/V) move to slots L + j.
-// The paper leaves this engine step implicit; the result is that of copying in
-// increasing j, which equals a gather because path[j] >= j.
+// length L and accepted nodes path[0..a-1], slot L + j receives the K/V of
+// node path[j].  The paper leaves this engine step implicit.  Two sources:
+//   compaction  the rows at slots L + path[j] (where the attention kernel
+//               appended the tree's K/V) move to slots L + j; the result is
+//               that of copying in increasing j, which equals a gather
+//               because path[j] >= j;
+//   commit      the rows come straight from k_new/v_new [B, T, Hkv, D] (no
+//               append before it).
 //
 // One CTA per (KV head, sequence) stages the a accepted rows of K and V in
 // shared memory and only then writes them, so a row that is both a source and
 // a destination is read before it is overwritten.  The CTA of head 0 also
-// writes the source slot indices and the new length.
+// writes the source indices and the new length.
 #include "common.cuh"
 
 namespace clover {
@@ -16,7 +20,8 @@ namespace {
 constexpr int kThreads = 128;
 
 __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
-    uint8_t *k_cache, uint8_t *v_cache, const int32_t *cache_len, const int32_t *path,
+    uint8_t *k_cache, uint8_t *v_cache, const uint8_t *k_new, const uint8_t *v_new, const int32_t *cache_len,
+    const int32_t *path,
     const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index, int T, int Hkv,
     int row_bytes, int Lcap, int32_t *status) {
     extern __shared__ uint4 stage[];          // [2][T][row_bytes / 16]
@@ -46,8 +51,9 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
         }
         if (g == 0 && len_ok && cap_ok) {
             if (src_index) {
-                if (j0 < T) src_index[(size_t)b * T + j0] = (j0 < a) ? L + s_src[j0] : -1;
-                if (j1 < T) src_index[(size_t)b * T + j1] = (j1 < a) ? L + s_src[j1] : -1;
+                const int base = k_new ? 0 : L;     // a tree node (commit) or a cache slot
+                if (j0 < T) src_index[(size_t)b * T + j0] = (j0 < a) ? base + s_src[j0] : -1;
+                if (j1 < T) src_index[(size_t)b * T + j1] = (j1 < a) ? base + s_src[j1] : -1;
             }
             if (threadIdx.x == 0) new_cache_len[b] = L + a;
         }
@@ -57,12 +63,12 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
 
     const int units = row_bytes / 16;
     const size_t head_base = ((size_t)b * Hkv + g) * Lcap;
-    const uint4 *ks = reinterpret_cast<const uint4 *>(k_cache);
-    const uint4 *vs = reinterpret_cast<const uint4 *>(v_cache);
+    const uint4 *ks = reinterpret_cast<const uint4 *>(k_new ? k_new : k_cache);
+    const uint4 *vs = reinterpret_cast<const uint4 *>(v_new ? v_new : v_cache);
     for (int e = threadIdx.x; e < a * units; e += kThreads) {
         const int j = e / units;
         const int u = e % units;
-        const size_t src = (head_base + L + s_src[j]) * units + u;
+        const size_t src = (k_new ? ((size_t)b * T + s_src[j]) * Hkv + g : head_base + L + s_src[j]) * units + u;
         stage[e] = ks[src];
         stage[T * units + e] = vs[src];
     }
@@ -80,10 +86,10 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
 
 }  // namespace
 
-cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const int32_t *cache_len, const int32_t *path,
-                              const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index, int B,
-                              int T, int Hkv, int D, int Lcap, int dtype, int32_t *status,
-                              cudaStream_t stream) {
+cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
+                              const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
+                              int32_t *new_cache_len, int32_t *src_index, int B, int T, int Hkv, int D, int Lcap,
+                              int dtype, int32_t *status, cudaStream_t stream) {
     const int row_bytes = D * (dtype == CLOVER_F32 ? 4 : 2);
     const size_t smem = (size_t)2 * T * row_bytes;
     static unsigned char done[64];
@@ -91,7 +97,9 @@ cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const int32_t *cache
     if (e != cudaSuccess) return e;
     dim3 grid(Hkv, B);
     kv_compact_kernel<<<grid, kThreads, smem, stream>>>(static_cast<uint8_t *>(k_cache),
-                                                        static_cast<uint8_t *>(v_cache), cache_len, path,
+                                                        static_cast<uint8_t *>(v_cache),
+                                                        static_cast<const uint8_t *>(k_new),
+                                                        static_cast<const uint8_t *>(v_new), cache_len, path,
                                                         accept_len, new_cache_len, src_index, T, Hkv,
                                                         row_bytes, Lcap, status);
     return cudaGetLastError();

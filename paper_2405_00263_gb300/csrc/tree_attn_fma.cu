@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
             constexpr int per = TileRegs<T, D>::kPerChunk;
             unpack<T>(regs.k[j], sK + key * S::DQ + col);
             unpack<T>(regs.v[j], sV + key * D + col);
-            if (tree_tile && rt == 0 && !cap_bad && key < a.T) {
+            if (tree_tile && a.append && rt == 0 && !cap_bad && key < a.T) {
                 const size_t off = ((size_t)(b * a.Hkv + g) * a.Lcap + L + key) * D + col;
                 *reinterpret_cast<uint4 *>(static_cast<T *>(a.k_cache) + off) = regs.k[j];
                 *reinterpret_cast<uint4 *>(static_cast<T *>(a.v_cache) + off) = regs.v[j];

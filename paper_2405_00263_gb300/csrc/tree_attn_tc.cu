@@ -207,7 +207,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
     const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
     // this CTA appends the tree K/V to cache slots [L, L+T)
-    const bool appender = tree_cta && rt == 0 && !cap_bad;
+    const bool appender = a.append && tree_cta && rt == 0 && !cap_bad;
 
     // tile j of K (is_v == false) or V into ring stage `dst`
     auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar) {

@@ -15,12 +15,12 @@ def to_dev(host: dict, dev) -> dict:
     return {k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in host.items()}
 
 
-def run_gpu(t: dict, scale: float = 0.0, step: pkg.VerifyStep | None = None) -> pkg.VerifyStep:
+def run_gpu(t: dict, scale: float = 0.0, step: pkg.VerifyStep | None = None, **step_kw) -> pkg.VerifyStep:
     B, T, Hq, D = t["q"].shape
     Hkv = t["k_new"].shape[2]
     V = t["logits"].shape[-1]
     if step is None:
-        step = pkg.VerifyStep(B, T, Hq, Hkv, D, t["Lcap"], V, t["q"].dtype, device=t["q"].device)
+        step = pkg.VerifyStep(B, T, Hq, Hkv, D, t["Lcap"], V, t["q"].dtype, device=t["q"].device, **step_kw)
     step.clear_status()
     step.run(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
              t["cand"], t["logits"], scale=scale)
@@ -39,7 +39,9 @@ def compare_full(host: dict, step: pkg.VerifyStep, t: dict, scale: float = 0.0):
     assert torch.equal(step.path.cpu(), ref["path"])
     assert torch.equal(step.accept_len.cpu(), ref["accept_len"])
     assert torch.equal(step.bonus.cpu(), ref["bonus"])
-    assert torch.equal(step.src_index.cpu(), ref["src_index"])
+    # the commit schedule records tree nodes, the compaction schedule cache slots
+    exp_src = ref["path"] if step.schedule == "commit" else ref["src_index"]
+    assert torch.equal(step.src_index.cpu(), exp_src)
     assert torch.equal(step.new_cache_len.cpu(), ref["cache_len"])
     kc, vc = t["k_cache"].cpu(), t["v_cache"].cpu()
     for b in range(kc.shape[0]):

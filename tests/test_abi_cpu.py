@@ -101,6 +101,23 @@ def test_accept_and_compact_host_validation(lib):
     assert cmp(1024, 2048, B=0) == 0
 
 
+def test_attn_ex_and_commit_host_validation(lib):
+    P = ctypes.c_void_p
+    ex = lambda flags, T=4: lib.clover_verify_attn_ex(
+        P(16), P(16), P(16), P(16), P(16), P(16), P(16), P(16), 1, T, 2, 2, 64, 64, 1, 0.0, None, 0, None, None,
+        flags)
+    assert ex(2) == 1 and ex(0xFFFFFFFE) == 1             # unknown flag bits
+    assert ex(1, T=65) == 2 and ex(0, T=65) == 2           # the limits of clover_verify_attn
+    com = lambda cl, ncl, kn=16, vn=16, B=2, T=4, D=64: lib.clover_kv_commit(
+        P(16), P(16), P(kn), P(vn), P(cl), P(16), P(16), P(ncl), None, B, T, 2, D, 64, 1, None, None)
+    assert com(1024, 1024) == 1                            # new length aliases the old one
+    assert com(1024, 2048, kn=None) == 1                   # k_new missing
+    assert com(1024, 2048, vn=24) == 1                     # v_new misaligned
+    assert com(1024, 2048, D=32) == 2
+    assert com(1024, 2048, T=65) == 2
+    assert com(1024, 2048, B=0) == 0
+
+
 def test_python_binding_rejects_cpu_tensors(lib):
     import paper_2405_00263_gb300 as pkg
     x = torch.zeros(1, 4, 2, 64, dtype=torch.bfloat16)

@@ -105,13 +105,105 @@ def test_full_size_workloads(name, cuda):
     zl = torch.zeros(B, dtype=torch.int32)
     oracle.append_tree_kv(host["k_new"], host["v_new"], zk, zv, zl)
     src = oracle.kv_compact(zk, zv, zl, path, alen)
-    assert torch.equal(step.src_index.cpu(), torch.where(src >= 0, src + L.unsqueeze(1), src))
+    exp_src = path if step.schedule == "commit" else torch.where(src >= 0, src + L.unsqueeze(1), src)
+    assert torch.equal(step.src_index.cpu(), exp_src)
     for b in range(B):
         l0, a = int(L[b]), int(alen[b])
         assert torch.equal(t["k_cache"][b, :, l0:l0 + a].cpu().view(torch.int16), zk[b, :, :a].view(torch.int16))
         assert torch.equal(t["v_cache"][b, :, l0:l0 + a].cpu().view(torch.int16), zv[b, :, :a].view(torch.int16))
         assert torch.equal(t["k_cache"][b, :, :l0].view(torch.int16), kc0[b, :, :l0].view(torch.int16))
         assert torch.equal(t["v_cache"][b, :, :l0].view(torch.int16), vc0[b, :, :l0].view(torch.int16))
+
+
+# ---------------------------------------------------------------------------
+# the two schedules of a step
+# ---------------------------------------------------------------------------
+
+SCHEDULE_CASES = {
+    "f32_splits": ("tiny_f32", dict(D=128, L=1000, Hq=4, Hkv=4, V=5003)),
+    "bf16_ragged_batch": ("7b_batched", dict(B=5, Hq=8, Hkv=8, L_range=(0, 700), V=3001)),
+    "bf16_gqa8": ("100b_gqa", dict(B=2, Hq=16, Hkv=2, L=900, V=2048)),
+}
+
+
+@pytest.mark.parametrize("concurrent", [True, False])
+@pytest.mark.parametrize("case", sorted(SCHEDULE_CASES))
+def test_commit_and_compact_schedules_agree(case, concurrent, cuda):
+    """Attention without the append plus clover_kv_commit, and attention with the
+    append plus clover_kv_compact, leave the same bytes in slots [0, L + a)
+    and give the same outputs; both match the oracle."""
+    name, over = SCHEDULE_CASES[case]
+    host = workloads.make(workloads.get(name, **over))
+    t1, t2 = to_dev(host, cuda), to_dev(host, cuda)
+    s1 = run_gpu(t1, schedule="commit", concurrent=concurrent)
+    s2 = run_gpu(t2, schedule="compact", concurrent=concurrent)
+    compare_full(host, s1, t1)
+    compare_full(host, s2, t2)
+    assert torch.equal(s1.out, s2.out)
+    L = host["cache_len"].to(cuda)
+    assert torch.equal(torch.where(s1.src_index >= 0, s1.src_index + L.unsqueeze(1), s1.src_index), s2.src_index)
+    bits = torch.int16 if host["q"].dtype == torch.bfloat16 else torch.int32
+    for b in range(host["q"].shape[0]):
+        n = int(s1.new_cache_len[b])
+        assert torch.equal(t1["k_cache"][b, :, :n].view(bits), t2["k_cache"][b, :, :n].view(bits))
+        assert torch.equal(t1["v_cache"][b, :, :n].view(bits), t2["v_cache"][b, :, :n].view(bits))
+
+
+@pytest.mark.parametrize("name", ["tiny_f32", "7b_l2048"])
+def test_attention_without_append_only_reads_the_cache(name, cuda):
+    """CLOVER_ATTN_NO_APPEND: every byte of both caches (the NaN tail included)
+    is unchanged, and the output is the appending call's, bit for bit."""
+    w = workloads.get(name, **({} if name == "tiny_f32" else dict(T=64, Hq=8, Hkv=8, L=1500, V=1000)))
+    host = workloads.make(w, logits=False)
+    t = to_dev(host, cuda)
+    bits = torch.int16 if host["q"].dtype == torch.bfloat16 else torch.int32
+    kc0, vc0 = t["k_cache"].clone(), t["v_cache"].clone()
+    B, T, Hq, D = t["q"].shape
+    Hkv = t["k_new"].shape[2]
+    nbytes = pkg.clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, t["Lcap"], t["q"].dtype)
+    ws = torch.zeros(max(nbytes, 16), dtype=torch.uint8, device=cuda) if nbytes else None
+    st = torch.zeros(1, dtype=torch.int32, device=cuda)
+    out_ro, out_ap = torch.empty_like(t["q"]), torch.empty_like(t["q"])
+    pkg.clover_verify_attn(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
+                           out_ro, workspace=ws, status=st, append=False)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert torch.equal(t["k_cache"].view(bits), kc0.view(bits)) and torch.equal(t["v_cache"].view(bits), vc0.view(bits))
+    pkg.clover_verify_attn(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
+                           out_ap, workspace=ws, status=st)
+    torch.cuda.synchronize()
+    assert torch.equal(out_ro.view(bits), out_ap.view(bits))
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_kv_commit_matches_oracle(dtype, cuda):
+    """clover_kv_commit on chosen paths (root only, a chain through every node,
+    branches) against the oracle's commit: cache bytes, source nodes, lengths."""
+    B, T, Hkv, D = 4, 16, 3, 128
+    g = torch.Generator().manual_seed(5)
+    Lcap = 320
+    kc = torch.randn(B, Hkv, Lcap, D, generator=g).to(dtype)
+    vc = torch.randn(B, Hkv, Lcap, D, generator=g).to(dtype)
+    kn = torch.randn(B, T, Hkv, D, generator=g).to(dtype)
+    vn = torch.randn(B, T, Hkv, D, generator=g).to(dtype)
+    L = torch.tensor([0, 17, 150, Lcap - T], dtype=torch.int32)
+    paths = [[0], list(range(T)), [0, 2, 9, 15], [0, 1, 5]]
+    path = torch.full((B, T), -1, dtype=torch.int32)
+    for b, p in enumerate(paths):
+        path[b, :len(p)] = torch.tensor(p)
+    alen = torch.tensor([len(p) for p in paths], dtype=torch.int32)
+    ko, vo, lo = kc.clone(), vc.clone(), L.clone()
+    src_ref = oracle.kv_commit(ko, vo, kn, vn, lo, path, alen)
+    d = lambda x: x.to(cuda)
+    kd, vd = d(kc), d(vc)
+    i32 = dict(dtype=torch.int32, device=cuda)
+    new_len, src, st = torch.empty(B, **i32), torch.empty((B, T), **i32), torch.zeros(1, **i32)
+    pkg.clover_kv_commit(kd, vd, d(kn), d(vn), d(L), d(path), d(alen), new_len, src, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert torch.equal(new_len.cpu(), lo) and torch.equal(src.cpu(), src_ref)
+    bits = torch.int16 if dtype == torch.bfloat16 else torch.int32
+    assert torch.equal(kd.cpu().view(bits), ko.view(bits)) and torch.equal(vd.cpu().view(bits), vo.view(bits))
 
 
 # ---------------------------------------------------------------------------

@@ -502,6 +502,43 @@ def test_compact_equals_out_of_place_gather():
             assert int(L2[b]) == l0 + len(p)
 
 
+def test_commit_equals_append_then_compact():
+    """The commit from k_new/v_new reaches the end state of append + compaction
+    (slots < L + a; the tree slots past L + a are unspecified afterwards)."""
+    B, T, Hkv, D = 3, 8, 2, 4
+    for dtype in (torch.float32, torch.bfloat16):
+        inp = rand_inputs(B, T, Hkv, Hkv, D, [0, 5, 19], seed=22, dtype=dtype)
+        paths = [[0, 3, 6], [0], [0, 1, 2, 3, 4, 5, 6, 7]]
+        path = torch.full((B, T), -1, dtype=torch.int32)
+        for b, q in enumerate(paths):
+            path[b, :len(q)] = torch.tensor(q)
+        alen = torch.tensor([len(q) for q in paths], dtype=torch.int32)
+        k1, v1, L1 = inp["k_cache"].clone(), inp["v_cache"].clone(), inp["cache_len"].clone().to(torch.int32)
+        oracle.append_tree_kv(inp["k_new"], inp["v_new"], k1, v1, L1)
+        src1 = oracle.kv_compact(k1, v1, L1, path, alen)
+        k2, v2, L2 = inp["k_cache"].clone(), inp["v_cache"].clone(), inp["cache_len"].clone().to(torch.int32)
+        src2 = oracle.kv_commit(k2, v2, inp["k_new"], inp["v_new"], L2, path, alen)
+        assert torch.equal(L1, L2)
+        for b, q in enumerate(paths):
+            n = int(L2[b])
+            assert torch.equal(k1[b, :, :n], k2[b, :, :n]) and torch.equal(v1[b, :, :n], v2[b, :, :n])
+            l0 = int(inp["cache_len"][b])
+            assert src2[b].tolist() == q + [-1] * (T - len(q))
+            assert src1[b].tolist() == [l0 + j for j in q] + [-1] * (T - len(q))
+            # slots past the new length are not written by the commit
+            assert torch.equal(k2[b, :, n:], inp["k_cache"][b, :, n:])
+
+
+def test_commit_rejects_bad_paths():
+    B, T, Hkv, D = 1, 4, 1, 4
+    inp = rand_inputs(B, T, Hkv, Hkv, D, [3], seed=23, dtype=torch.float32)
+    for path, alen in (([0, 4, -1, -1], 2), ([0, -1, -1, -1], 0), ([0, 1, 2, 3], 5)):
+        k, v, L = inp["k_cache"].clone(), inp["v_cache"].clone(), inp["cache_len"].clone().to(torch.int32)
+        with pytest.raises(Exception):
+            oracle.kv_commit(k, v, inp["k_new"], inp["v_new"], L, torch.tensor([path], dtype=torch.int32),
+                             torch.tensor([alen], dtype=torch.int32))
+
+
 def test_verify_step_tiny_invariants():
     w = workloads.get("tiny_f32")
     t = workloads.make(w)
