@@ -268,13 +268,19 @@ class VerifyStep:
 
     def run(self, q, k_new, v_new, k_cache, v_cache, cache_len, parent, cand, logits, scale=0.0,
             stream=None, events=None):
-        """One step.  ``events`` (optional, six CUDA events) brackets the
+        """One step.  ``events`` (optional, up to six CUDA events) brackets the
         attention (0-1), the commit or compaction (2-3) and the accept call
-        (4-5), each on the stream it runs on."""
+        (4-5), each on the stream it runs on; a shorter list brackets only the
+        calls it has events for."""
         stream = stream if stream is not None else torch.cuda.current_stream()
         commit = self.schedule == "commit"
         side = self.side if self.side is not None else stream
-        ev = (lambda i, st: events[i].record(st)) if events else (lambda i, st: None)
+        n_ev = len(events) if events else 0
+
+        def ev(i, st):
+            if i < n_ev:
+                events[i].record(st)
+
         if self.side is not None:
             self._fork.record(stream)
             self.side.wait_event(self._fork)
