@@ -51,16 +51,16 @@ constexpr uint32_t kTmemCols = 256;     // S/P: 2 x 64 columns, O: D columns
 constexpr float kRescale = 8.0f;        // move the reference max only past 2^8 growth
 constexpr uint64_t kWaitNs = 500ull * 1000 * 1000;   // 0.5 s per wait
 
-// Shared-memory plan.  QR = query rows stored per tile (128, or 64 when no tile
-// has more than 64 real rows: the MMA still reads 128 A rows, and rows 64-127
-// then come from whatever follows in shared memory; they only produce TMEM
-// lanes 64-127, which nothing reads).  The room saved goes to a deeper K ring.
-template <int D, int QR>
+// Shared-memory plan.  Q always fills the 128 A rows of the MMA.  KS = key
+// groups per tile row: with KS = 2 (a tile of at most 64 real query rows) Q
+// rows 64-127 repeat rows 0-63, so every real row's scores sit in two TMEM
+// lane quadrants and the four softmax warps each take half of a tile's keys.
+template <int D, int KS>
 struct TcSmem {
-    static constexpr int NSK = (QR == 64) ? 6 : 5;   // K ring stages
+    static constexpr int NSK = 5;                    // K ring stages
     static constexpr int NSV = 6;                    // V ring stages
     static constexpr int DH = D / 64;                // 128-byte column blocks per row
-    static constexpr int q_bytes = QR * D * 2;       // [DH][QR][128 B]
+    static constexpr int q_bytes = BM * D * 2;       // [DH][BM][128 B]
     static constexpr int kv_bytes = BN * D * 2;      // one K or V tile: [DH][BN][128 B]
     static constexpr int q_off = 0;
     static constexpr int k_off = q_off + q_bytes;
@@ -72,12 +72,15 @@ struct TcSmem {
     static constexpr int total = anc_off + kMaxTreeNodes * 8;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
     // After the key loop the K ring holds this CTA's partial result, one fp32
-    // row of D + 4 floats per query row (O, then m and l in the padding), and
-    // the V ring receives the other splits' partials of the rows this CTA
-    // merges: [n_split][rows per split][D + 4].
+    // row of D + 4 floats per query row (O, then m and l in the padding; with
+    // KS = 2 rows 64-127 first carry the second key half's rows), and the V
+    // ring receives the other splits' partials of the rows this CTA merges:
+    // [n_split][rows per split][D + 4].
     static constexpr int po_stride = D + 4;
-    static_assert(QR * po_stride * 4 <= NSK * kv_bytes, "partial result must fit in the K ring");
-    static_assert((QR + kMaxCluster - 1) * po_stride * 4 <= NSV * kv_bytes, "received partials must fit in the V ring");
+    static constexpr int rows_max = (KS == 2) ? 64 : BM;         // real rows of a tile
+    static_assert(BM * po_stride * 4 <= NSK * kv_bytes, "partial result must fit in the K ring");
+    static_assert((rows_max + kMaxCluster - 1) * po_stride * 4 <= NSV * kv_bytes,
+                  "received partials must fit in the V ring");
     static_assert(alloc <= 227 * 1024, "shared memory budget");
 };
 
@@ -149,13 +152,13 @@ __device__ __forceinline__ void merge_rows(const float *own, const float *recv, 
     }
 }
 
-template <int D, int QR>
+template <int D, int KS>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                         const __grid_constant__ CUtensorMap tm_kn, const __grid_constant__ CUtensorMap tm_vn,
                         const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ks,
                         const __grid_constant__ CUtensorMap tm_vs, const AttnArgs a) {
-    using S = TcSmem<D, QR>;
+    using S = TcSmem<D, KS>;
     constexpr int NSK = S::NSK;
     constexpr int NSV = S::NSV;
     extern __shared__ uint8_t smem_raw[];
@@ -193,7 +196,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n_split = a.n_split;
     const bool tree_cta = (split == n_split - 1);
     const int rows_here = min(BM, a.rows - rt * BM);
-    const int q_act = (rows_here + 31) >> 5;        // TMEM lane quadrants holding real rows
+    const int q_act = (rows_here + 31) >> 5;        // 32-row quadrants holding real rows
+    const int n_soft_warps = KS * q_act;             // softmax warps of this tile
 
     int L = __ldg(a.cache_len + b);
     const bool cap_bad = (L < 0 || L + a.T > a.Lcap);
@@ -268,7 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             for (int i = 0; i < 2; ++i) {
                 mbar_init(&s_full[i], 1);
-                mbar_init(&p_full[i], q_act);
+                mbar_init(&p_full[i], n_soft_warps);
                 mbar_init(&o_full[i], 1);
             }
             mbar_init(mma_done, 1);
@@ -290,10 +294,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (a.q_box_nodes > 0) {
                 // Q rows (node, head in group) of this tile: box (64 d, G heads, q_box_nodes nodes)
                 prefetch_tensormap(&tm_q);
-                mbar_arrive_expect_tx(q_full, S::DH * a.G * a.q_box_nodes * 128);
+                mbar_arrive_expect_tx(q_full, KS * S::DH * a.G * a.q_box_nodes * 128);
 #pragma unroll
                 for (int dh = 0; dh < S::DH; ++dh)
-                    tma_load_3d(sQ + dh * (QR * 128), &tm_q, q_full, dh * 64, g * a.G, b * a.T + rt * a.q_box_nodes);
+#pragma unroll
+                    for (int rep = 0; rep < KS; ++rep)
+                        tma_load_3d(sQ + dh * (BM * 128) + rep * (64 * 128), &tm_q, q_full, dh * 64, g * a.G,
+                                    b * a.T + rt * a.q_box_nodes);
             } else {
                 mbar_arrive(q_full);
             }
@@ -310,7 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // swizzled K-major layout, rows past this tile's real rows zero
         const __nv_bfloat16 *q = static_cast<const __nv_bfloat16 *>(a.q);
         constexpr int chunks_per_row = S::DH * 8;
-        constexpr int per_thread = QR * chunks_per_row / 128;
+        constexpr int per_thread = S::rows_max * chunks_per_row / 128;
         uint4 v[per_thread];
 #pragma unroll
         for (int k = 0; k < per_thread; ++k) {
@@ -331,7 +338,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int c = threadIdx.x + 128 * k;
             const int r = c / chunks_per_row;
             const int j = c % chunks_per_row;
-            *reinterpret_cast<uint4 *>(sQ + (j >> 3) * (QR * 128) + r * 128 + (((j & 7) ^ (r & 7)) << 4)) = v[k];
+#pragma unroll
+            for (int rep = 0; rep < KS; ++rep) {
+                const int rr = r + rep * 64;
+                *reinterpret_cast<uint4 *>(sQ + (j >> 3) * (BM * 128) + rr * 128 + (((j & 7) ^ (rr & 7)) << 4)) = v[k];
+            }
         }
         fence_proxy_async_smem();
     }
@@ -398,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t k_base = smem_u32(sK + s * S::kv_bytes);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k) {
-                const uint64_t ad = sdesc_sw128(q_base + (k >> 2) * (QR * 128) + (k & 3) * 32, 16, 1024);
+                const uint64_t ad = sdesc_sw128(q_base + (k >> 2) * (BM * 128) + (k & 3) * 32, 16, 1024);
                 const uint64_t bd = sdesc_sw128(k_base + (k >> 2) * (BN * 128) + (k & 3) * 32, 16, 1024);
                 mma_bf16(tS + sb * BN, ad, bd, idS, k > 0 ? 1u : 0u);
             }
@@ -434,12 +445,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // ------------------------------------------------------------ softmax warps
-    // Warp q owns TMEM lanes 32q.. = tile rows; it reads S, writes P back over
-    // it, keeps the row's reference max m_ref and sum l, and rescales its O row
-    // in TMEM when m_ref has to move.
+    // Warp w owns TMEM lanes 32w.. (the lanes it may access); it reads S there,
+    // writes P back over it, keeps the reference max m_ref and sum l, and
+    // rescales its O rows in TMEM when m_ref has to move.  KS = 1: lanes 32w..
+    // are tile rows 32w.. and the warp takes every key of a tile.  KS = 2:
+    // lanes 32w.. are rows 32(w & 1).. and the warp takes keys
+    // [32 (w >> 1), +32) of every tile; the two key halves of a row are two
+    // separate online softmaxes (own m, l and O rows), merged after the loop.
+    constexpr int NK = BN / KS;               // keys of a tile per thread
     const int quad = warp & 3;
-    const bool softmax_warp = warp < 4 && quad < q_act;
-    const int r = quad * 32 + lane;
+    const int rquad = (KS == 2) ? (quad & 1) : quad;
+    const int half = (KS == 2) ? (quad >> 1) : 0;
+    const bool softmax_warp = warp < 4 && rquad < q_act;
+    const int r = rquad * 32 + lane;          // tile row
+    const int soft_rank = ((KS == 2) ? half * q_act + rquad : quad) * 32 + lane;
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
     float m_ref = -INFINITY, l_run = 0.f;
     bool o_ready = false;
@@ -456,9 +475,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after();
-            float sv[64];
-            tmem_ld32(tS + lane_base + sb * BN, *reinterpret_cast<float(*)[32]>(sv));
-            tmem_ld32(tS + lane_base + sb * BN + 32, *reinterpret_cast<float(*)[32]>(sv + 32));
+            float sv[NK];
+#pragma unroll
+            for (int c = 0; c < NK; c += 32)
+                tmem_ld32(tS + lane_base + sb * BN + half * NK + c, *reinterpret_cast<float(*)[32]>(sv + c));
             tmem_wait_ld();
 
             const bool tree_tile = (j == n_cache_tiles);
@@ -470,12 +490,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             // code into the instruction cache (a miss then waits on a
             // saturated memory system).
             const uint64_t prefix = (n_valid >= BN) ? ~0ull : ((1ull << n_valid) - 1ull);
-            const uint64_t vis = tree_tile ? s_anc[node] : prefix;
+            const uint64_t vis = (tree_tile ? s_anc[node] : prefix) >> (half * NK);
 #pragma unroll
-            for (int c = 0; c < 64; ++c) sv[c] = ((vis >> c) & 1ull) ? sv[c] : -INFINITY;
+            for (int c = 0; c < NK; ++c) sv[c] = ((vis >> c) & 1ull) ? sv[c] : -INFINITY;
             float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-            for (int c = 0; c < 64; ++c) mx4[c & 3] = fmaxf(mx4[c & 3], sv[c]);
+            for (int c = 0; c < NK; ++c) mx4[c & 3] = fmaxf(mx4[c & 3], sv[c]);
             const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * sc;   // sc > 0
 
             // move the reference max when this tile exceeds it by more than 2^8
@@ -506,9 +526,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const float ref = (m_ref == -INFINITY) ? 0.f : m_ref;
             float sum4[4] = {0.f, 0.f, 0.f, 0.f};
-            float pk[32];
+            float pk[NK / 2];
 #pragma unroll
-            for (int c = 0; c < 64; c += 2) {
+            for (int c = 0; c < NK; c += 2) {
                 const float p0 = ex2_approx(fmaf(sv[c], sc, -ref));
                 const float p1 = ex2_approx(fmaf(sv[c + 1], sc, -ref));
                 sum4[c & 3] += p0;
@@ -516,8 +536,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 pk[c >> 1] = __uint_as_float(pack_bf16x2(p0, p1));
             }
             l_run += (sum4[0] + sum4[1]) + (sum4[2] + sum4[3]);
-            // P over the first 32 columns of this tile's S (two keys per column)
-            tmem_st32(tS + lane_base + sb * BN, pk);
+            // P over the first 32 columns of this tile's S (two keys per column);
+            // with KS = 2 the other half's keys of the row read as zero here
+            float prow[32];
+#pragma unroll
+            for (int c = 0; c < 32; ++c) prow[c] = (c / (NK / 2) == half) ? pk[c % (NK / 2)] : 0.f;
+            tmem_st32(tS + lane_base + sb * BN, prow);
             // value rows of keys past the valid ones may hold anything (even NaN): zero them
             if (n_valid < BN) {
                 const int s = j % NSV;
@@ -528,7 +552,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 uint4 *vrows = reinterpret_cast<uint4 *>(sV + s * S::kv_bytes);
                 const int n_zero = (BN - n_valid) * S::DH * 8;
-                for (int e = r; e < n_zero; e += q_act * 32) {
+                for (int e = soft_rank; e < n_zero; e += n_soft_warps * 32) {
                     const int row = n_valid + e / (S::DH * 8);
                     const int rest = e % (S::DH * 8);
                     vrows[(rest >> 3) * (BN * 8) + row * 8 + (rest & 7)] = make_uint4(0, 0, 0, 0);
@@ -569,15 +593,72 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(a.out);
     const bool row_ok = softmax_warp && r < rows_here;
-    float *part_o = reinterpret_cast<float *>(sK);            // [QR][D + 4] fp32, this CTA's partial
+    float *part_o = reinterpret_cast<float *>(sK);            // [BM][D + 4] fp32, this CTA's partial
     float *recv = reinterpret_cast<float *>(sV);              // [n_split][per][D + 4]
-    if (softmax_warp) {
+    // KS = 2: the second key half's rows (O, m, l) go to rows 64.. of part_o,
+    // where the warps of the first half merge them into their own
+    if (KS == 2) {
+        // the TMEM loads are warp-collective: every lane runs them, rows past
+        // the tile's real rows only skip the stores
+        if (softmax_warp && half == 1) {
+            float *dst = part_o + (64 + r) * S::po_stride;
+#pragma unroll 1
+            for (int cc = 0; cc < D / 32; cc += 2) {
+                float x0[32], x1[32];
+                if (o_ready) {
+                    tmem_ld32(tO + lane_base + cc * 32, x0);
+                    tmem_ld32(tO + lane_base + cc * 32 + 32, x1);
+                    tmem_wait_ld();
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) x0[c] = x1[c] = 0.f;
+                }
+                if (row_ok) {
+#pragma unroll
+                    for (int c = 0; c < 32; c += 4) {
+                        *reinterpret_cast<float4 *>(dst + cc * 32 + c) =
+                            make_float4(x0[c], x0[c + 1], x0[c + 2], x0[c + 3]);
+                        *reinterpret_cast<float4 *>(dst + cc * 32 + 32 + c) =
+                            make_float4(x1[c], x1[c + 1], x1[c + 2], x1[c + 3]);
+                    }
+                }
+            }
+            if (row_ok)
+                *reinterpret_cast<float2 *>(dst + D) =
+                    make_float2(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f);
+        }
+        __syncthreads();
+    }
+    if (softmax_warp && half == 0) {
         const int R = rt * BM + r;
         const int i = row_ok ? R / a.G : 0;
         const int h = row_ok ? g * a.G + (R % a.G) : 0;
-        const float inv = (n_split == 1 && o_ready) ? 1.f / l_run : 1.f;
+        // this row's (m, l) and the weights of its key halves
+        float m_row = o_ready ? m_ref : -INFINITY;
+        float l_row = o_ready ? l_run : 0.f;
+        float wa = 1.f, wb = 0.f;
+        const float *ob = part_o + (64 + r) * S::po_stride;
+        if (KS == 2 && row_ok) {
+            const float2 mlb = *reinterpret_cast<const float2 *>(ob + D);
+            const float M = fmaxf(m_row, mlb.x);
+            wa = (m_row == -INFINITY) ? 0.f : ex2_approx(m_row - M);
+            wb = (mlb.x == -INFINITY) ? 0.f : ex2_approx(mlb.x - M);
+            m_row = M;
+            l_row = wa * l_row + wb * mlb.y;
+        }
+        const float inv = (n_split == 1 && l_row > 0.f) ? 1.f / l_row : 1.f;
         // 32 columns of the row: the output (one split) or the partial row
-        auto emit = [&](int cc, const float (&x)[32]) {
+        auto emit = [&](int cc, float (&x)[32]) {
+            if (KS == 2) {
+#pragma unroll
+                for (int c = 0; c < 32; c += 4) {
+                    const float4 y = *reinterpret_cast<const float4 *>(ob + cc * 32 + c);
+                    x[c] = fmaf(wb, y.x, wa * x[c]);
+                    x[c + 1] = fmaf(wb, y.y, wa * x[c + 1]);
+                    x[c + 2] = fmaf(wb, y.z, wa * x[c + 2]);
+                    x[c + 3] = fmaf(wb, y.w, wa * x[c + 3]);
+                }
+            }
             if (n_split == 1) {
                 __nv_bfloat16 *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D + cc * 32;
 #pragma unroll
@@ -614,8 +695,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         if (row_ok && n_split > 1)
-            *reinterpret_cast<float2 *>(part_o + r * S::po_stride + D) =
-                make_float2(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f);
+            *reinterpret_cast<float2 *>(part_o + r * S::po_stride + D) = make_float2(m_row, l_row);
         fence_proxy_async_smem();             // the bulk copies below read these rows
     }
 
@@ -690,13 +770,13 @@ struct TcLaunchCache {
     int max_clusters[kMaxCluster + 1] = {0};   // co-resident clusters per cluster size (0: not queried)
 };
 
-template <int D, int QR>
+template <int D, int KS>
 int max_active_clusters(int n, TcLaunchCache &cache) {
     if (cache.max_clusters[n] == 0) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(1, n, n);
         cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = TcSmem<D, QR>::alloc;
+        cfg.dynamicSmemBytes = TcSmem<D, KS>::alloc;
         cudaLaunchAttribute attr;
         attr.id = cudaLaunchAttributeClusterDimension;
         attr.val.clusterDim.x = 1;
@@ -705,7 +785,7 @@ int max_active_clusters(int n, TcLaunchCache &cache) {
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
         int num = 0;
-        if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D, QR>, &cfg) != cudaSuccess) {
+        if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D, KS>, &cfg) != cudaSuccess) {
             cudaGetLastError();
             num = -1;
         }
@@ -714,12 +794,12 @@ int max_active_clusters(int n, TcLaunchCache &cache) {
     return cache.max_clusters[n];
 }
 
-template <int D, int QR>
+template <int D, int KS>
 cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     static unsigned char done[64];
     static TcLaunchCache caches[64];
-    auto kernel = tree_attn_tc_kernel<D, QR>;
-    cudaError_t err = ensure_smem_attr(kernel, TcSmem<D, QR>::alloc, done);
+    auto kernel = tree_attn_tc_kernel<D, KS>;
+    cudaError_t err = ensure_smem_attr(kernel, TcSmem<D, KS>::alloc, done);
     if (err != cudaSuccess) return err;
     int dev = 0;
     if ((err = cudaGetDevice(&dev)) != cudaSuccess) return err;
@@ -733,7 +813,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     int n = 1;
     for (int c = kMaxCluster; c >= 2; --c) {
         if (c > by_len || base * c > cache.sms) continue;
-        if (max_active_clusters<D, QR>(c, cache) >= base) {
+        if (max_active_clusters<D, KS>(c, cache) >= base) {
             n = c;
             break;
         }
@@ -768,7 +848,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.row_tiles, n, a.B * a.Hkv);
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = TcSmem<D, QR>::alloc;
+    cfg.dynamicSmemBytes = TcSmem<D, KS>::alloc;
     cfg.stream = stream;
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeClusterDimension;
@@ -787,8 +867,9 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
 int tc_row_tile() { return BM; }
 
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream) {
-    if (a.rows <= 64) return a.D == 64 ? launch<64, 64>(a, stream) : launch<128, 64>(a, stream);
-    return a.D == 64 ? launch<64, 128>(a, stream) : launch<128, 128>(a, stream);
+    // a tile of at most 64 real rows: two key groups per row (KS = 2)
+    if (a.rows <= 64) return a.D == 64 ? launch<64, 2>(a, stream) : launch<128, 2>(a, stream);
+    return a.D == 64 ? launch<64, 1>(a, stream) : launch<128, 1>(a, stream);
 }
 
 }  // namespace clover
