@@ -25,7 +25,6 @@ struct AttnArgs {
     int row_tiles;         // ceil(rows / row_tile)
     int n_split;           // cache key ranges per (sequence, KV head, row tile)
     int slot_rows;         // rows of one partial-result slot (<= row_tile)
-    int q_box_nodes;       // tensor-core path: tree nodes per Q tile loaded by TMA (0: loaded by threads)
     int append;            // write k_new/v_new to cache slots [L, L+T) (0: the caches are only read)
     float *part_o;         // [B, Hkv, row_tiles, n_split, slot_rows, D]
     float *part_ml;        // [B, Hkv, row_tiles, n_split, slot_rows, 2]  (max, sum)

@@ -8,26 +8,30 @@
 // One CTA per (row tile of up to 128 query rows, cache-key split, sequence x
 // KV head).  The T*G query rows of a KV head (row i*G + hh = node i, query head
 // g*G + hh) share every K/V tile, so per 64-key tile:
-//   S  = Q K^T        tcgen05.mma M=128 N=64 K=D  (Q, K K-major in smem; S in TMEM)
+//   S  = Q K^T        tcgen05.mma M=128 N=64 K=D  (Q in TMEM, K K-major in smem; S in TMEM)
 //   P  = 2^(S*c - m)  online softmax in registers; bf16 P written back to TMEM
 //                     over the S tile it came from
-//   O += P V          tcgen05.mma M=128 N=D K=64  (P from TMEM, V MN-major in smem)
-// O stays in TMEM for the whole key range.  Each row keeps a reference max m;
-// P is taken relative to it, and m (with O and the row sum) is only moved when
-// a tile's max exceeds it by more than 2^8, so O is rarely rescaled.
-// Warp roles (224 threads): warp q in 0-3 runs the softmax, rescales and the
-// epilogue of TMEM lanes 32q.. (the lanes warp q may access); warp 4 issues the
-// TMA loads of Q and of the K tiles (its own ring); warp 6 issues the TMA loads
-// of the V tiles (a deeper ring: a V tile is held until its P.V product, a K
-// tile only until its S); warp 5 allocates TMEM and issues the MMAs from one
-// thread.  The tree CTA's producers also append the tree keys and values to
-// the cache, by TMA stores of the tree tile they loaded.
+//   O += P V          tcgen05.mma M=128 N=D K=64  (P in TMEM, V MN-major in smem)
+// Q and O stay in TMEM for the whole key range, so the tensor core reads only
+// K and V from shared memory (which the TMA writes fill at the same time).
+// Each row keeps a reference max m; P is taken relative to it, and m (with O
+// and the row sum) is only moved when a tile's max exceeds it by more than
+// 2^8, so O is rarely rescaled.  A tile of at most 64 real rows repeats its Q
+// rows in TMEM lanes 64-127, and the rows' keys split into two halves, each a
+// separate online softmax merged after the loop, so all four softmax warps work.
+// Warp roles (224 threads): warp w in 0-3 writes the Q rows of TMEM lanes
+// 32w.. and runs the softmax, rescales and the epilogue of those lanes (the
+// lanes warp w may access); warp 4 issues the TMA loads of the K tiles (its
+// own ring); warp 6 those of the V tiles (a deeper ring: a V tile is held
+// until its P.V product, a K tile only until its S); warp 5 allocates TMEM and
+// issues the MMAs from one thread.  The tree CTA's producers also append the
+// tree keys and values to the cache when asked, by TMA stores of the tree
+// tile they loaded.
 // The split that owns the last cache range also takes the tile of T tree keys
 // (read from k_new/v_new) under the ancestor bitmask.  The n_split CTAs of a
-// (sequence, head, row tile) form one thread-block cluster: each leaves its
-// partial (m, l, O) in its own shared memory and each merges a share of the
-// rows by reading all partials over distributed shared memory, so no partial
-// result touches global memory.
+// (sequence, head, row tile) form one thread-block cluster: each sends every
+// other CTA its rows of the partial result (O, m, l) by shared-to-shared bulk
+// copy, and merges its own rows, so no partial result touches global memory.
 // Every mbarrier wait is bounded; on a timeout the CTA reports
 // CLOVER_ERR_TIMEOUT, winds down, waits (bounded) for its copies in flight and
 // frees its TMEM.
@@ -41,29 +45,27 @@ namespace {
 using namespace tc;
 
 constexpr int BM = 128;                 // query rows per CTA (MMA M)
-constexpr int BN = 64;                  // keys per tile
+constexpr int BN = 128;                 // keys per tile (the N of the S MMA)
 constexpr int kKProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kVProducerWarp = 6;
 constexpr int kThreads = 224;
 constexpr int kMaxCluster = 8;          // portable cluster size: splits per head
-constexpr uint32_t kTmemCols = 256;     // S/P: 2 x 64 columns, O: D columns
 constexpr float kRescale = 8.0f;        // move the reference max only past 2^8 growth
 constexpr uint64_t kWaitNs = 500ull * 1000 * 1000;   // 0.5 s per wait
 
-// Shared-memory plan.  Q always fills the 128 A rows of the MMA.  KS = key
-// groups per tile row: with KS = 2 (a tile of at most 64 real query rows) Q
-// rows 64-127 repeat rows 0-63, so every real row's scores sit in two TMEM
-// lane quadrants and the four softmax warps each take half of a tile's keys.
+// Shared-memory plan: the K and V rings only (Q lives in TMEM).  KS = key
+// groups per tile row: with KS = 2 (a tile of at most 64 real query rows) the
+// Q rows of TMEM lanes 64-127 repeat those of lanes 0-63, so every real row's
+// scores sit in two lane quadrants and the four softmax warps each take half
+// of a tile's keys.
 template <int D, int KS>
 struct TcSmem {
-    static constexpr int NSK = 5;                    // K ring stages
-    static constexpr int NSV = 6;                    // V ring stages
+    static constexpr int NSK = (D == 128) ? 3 : 4;   // K ring stages
+    static constexpr int NSV = (D == 128) ? 3 : 4;   // V ring stages
     static constexpr int DH = D / 64;                // 128-byte column blocks per row
-    static constexpr int q_bytes = BM * D * 2;       // [DH][BM][128 B]
     static constexpr int kv_bytes = BN * D * 2;      // one K or V tile: [DH][BN][128 B]
-    static constexpr int q_off = 0;
-    static constexpr int k_off = q_off + q_bytes;
+    static constexpr int k_off = 0;
     static constexpr int v_off = k_off + NSK * kv_bytes;
     static constexpr int bar_off = v_off + NSV * kv_bytes;
     static constexpr int n_bars = 2 * NSK + 2 * NSV + 11;
@@ -71,6 +73,12 @@ struct TcSmem {
     static constexpr int anc_off = misc_off + 16;                  // ancestor masks [64]
     static constexpr int total = anc_off + kMaxTreeNodes * 8;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
+    // TMEM columns: S/P 2 x BN, O D, Q D / 2 (two bf16 per column), rounded up
+    // to a power of two.  All 512 columns of an SM go to one CTA only when
+    // the shared memory already keeps a second CTA off the SM (a CTA waiting
+    // in tcgen05.alloc would stall its cluster).
+    static constexpr uint32_t tmem_cols = (2 * BN + D + D / 2 <= 256) ? 256 : 512;
+    static_assert(tmem_cols < 512 || 2 * alloc > 228 * 1024, "512 TMEM columns need one CTA per SM");
     // After the key loop the K ring holds this CTA's partial result, one fp32
     // row of D + 4 floats per query row (O, then m and l in the padding; with
     // KS = 2 rows 64-127 first carry the second key half's rows), and the V
@@ -156,7 +164,7 @@ template <int D, int KS>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                         const __grid_constant__ CUtensorMap tm_kn, const __grid_constant__ CUtensorMap tm_vn,
-                        const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ks,
+                        const __grid_constant__ CUtensorMap tm_ks,
                         const __grid_constant__ CUtensorMap tm_vs, const AttnArgs a) {
     using S = TcSmem<D, KS>;
     constexpr int NSK = S::NSK;
@@ -165,7 +173,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     // base rounded up to 1024 bytes by pointer arithmetic on the shared array,
     // so that every access below stays a shared-memory access
     uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-    uint8_t *sQ = sm + S::q_off;
     uint8_t *sK = sm + S::k_off;
     uint8_t *sV = sm + S::v_off;
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + S::bar_off);
@@ -177,7 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t *p_full = s_full + 2;            // [2] P of a tile is in TMEM
     uint64_t *o_full = p_full + 2;            // [2] the tile's P.V product is done
     uint64_t *mma_done = o_full + 2;
-    uint64_t *q_full = mma_done + 1;
+    uint64_t *q_full = mma_done + 1;          // the four lane quadrants hold their Q rows in TMEM
     uint64_t *m_free = q_full + 1;            // every CTA of the cluster is out of its key loop
     uint64_t *m_done = m_free + 1;            // every CTA has received this CTA's partial rows
     uint64_t *m_data = m_done + 1;            // the other splits' partials of this CTA's rows are here
@@ -276,7 +283,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_init(&o_full[i], 1);
             }
             mbar_init(mma_done, 1);
-            mbar_init(q_full, 1);
+            mbar_init(q_full, 4);
             mbar_init(m_free, n_split);
             mbar_init(m_done, n_split);
             mbar_init(m_data, 1);
@@ -291,60 +298,35 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_barrier_init();
             prefetch_tensormap(&tm_kc);
             prefetch_tensormap(&tm_kn);
-            if (a.q_box_nodes > 0) {
-                // Q rows (node, head in group) of this tile: box (64 d, G heads, q_box_nodes nodes)
-                prefetch_tensormap(&tm_q);
-                mbar_arrive_expect_tx(q_full, KS * S::DH * a.G * a.q_box_nodes * 128);
-#pragma unroll
-                for (int dh = 0; dh < S::DH; ++dh)
-#pragma unroll
-                    for (int rep = 0; rep < KS; ++rep)
-                        tma_load_3d(sQ + dh * (BM * 128) + rep * (64 * 128), &tm_q, q_full, dh * 64, g * a.G,
-                                    b * a.T + rt * a.q_box_nodes);
-            } else {
-                mbar_arrive(q_full);
-            }
             for (; k_issued < min(NSK, n_tiles); ++k_issued)
                 issue_tile(k_issued, false, sK + k_issued * S::kv_bytes, &k_full[k_issued]);
         }
     }
     if (warp == kMmaWarp) {
-        tmem_alloc(s_tmem, kTmemCols);
+        tmem_alloc(s_tmem, S::tmem_cols);
         tmem_relinquish();
     }
-    if (warp < 4 && a.q_box_nodes == 0) {
-        // Q tile by threads (group sizes that do not divide the tile): 128-byte
-        // swizzled K-major layout, rows past this tile's real rows zero
-        const __nv_bfloat16 *q = static_cast<const __nv_bfloat16 *>(a.q);
-        constexpr int chunks_per_row = S::DH * 8;
-        constexpr int per_thread = S::rows_max * chunks_per_row / 128;
-        uint4 v[per_thread];
+    // Q rows of this warp's TMEM lane quadrant (row (node, head in group) =
+    // lane-quadrant row; with KS = 2 lanes 64-127 take rows 0-63 again): loaded
+    // now, written to TMEM once its address is known.  Rows past the tile's
+    // real rows are zero.
+    constexpr int QW = D / 2;                 // 32-bit TMEM columns of a Q row (two bf16 each)
+    uint32_t qrow[QW];
+    if (warp < 4) {
+        const int rq = ((KS == 2) ? (warp & 1) : warp) * 32 + lane;
+        const int R = rt * BM + rq;
+        const bool real = rq < rows_here;
+        const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(a.q) +
+                                                           ((size_t)(b * a.T + (real ? R / a.G : 0)) * a.Hq +
+                                                            g * a.G + (real ? R % a.G : 0)) * D);
 #pragma unroll
-        for (int k = 0; k < per_thread; ++k) {
-            const int c = threadIdx.x + 128 * k;
-            const int r = c / chunks_per_row;
-            const int j = c % chunks_per_row;
-            const int R = rt * BM + r;
-            v[k] = make_uint4(0, 0, 0, 0);
-            if (r < rows_here) {
-                const int i = R / a.G;
-                const int h = g * a.G + (R % a.G);
-                v[k] = __ldg(reinterpret_cast<const uint4 *>(q + ((size_t)(b * a.T + i) * a.Hq + h) * D + (j >> 3) * 64 +
-                                                             (j & 7) * 8));
-            }
+        for (int k = 0; k < QW / 4; ++k) {
+            const uint4 v = real ? __ldg(src + k) : make_uint4(0, 0, 0, 0);
+            qrow[4 * k] = v.x;
+            qrow[4 * k + 1] = v.y;
+            qrow[4 * k + 2] = v.z;
+            qrow[4 * k + 3] = v.w;
         }
-#pragma unroll
-        for (int k = 0; k < per_thread; ++k) {
-            const int c = threadIdx.x + 128 * k;
-            const int r = c / chunks_per_row;
-            const int j = c % chunks_per_row;
-#pragma unroll
-            for (int rep = 0; rep < KS; ++rep) {
-                const int rr = r + rep * 64;
-                *reinterpret_cast<uint4 *>(sQ + (j >> 3) * (BM * 128) + rr * 128 + (((j & 7) ^ (rr & 7)) << 4)) = v[k];
-            }
-        }
-        fence_proxy_async_smem();
     }
     // the tree CTA's ancestor masks (warp 3 is otherwise idle here)
     if (warp == 3 && tree_cta) tree_masks_warp(a.parent + (size_t)b * a.T, a.T, s_anc, s_bad);
@@ -359,6 +341,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = *s_tmem;
     const uint32_t tS = tmem;                 // S tiles (and their P): columns [0, 2*BN)
     const uint32_t tO = tmem + 2 * BN;        // O: columns [2*BN, 2*BN + D)
+    const uint32_t tQ = tmem + 2 * BN + D;    // Q (the A operand of S): D / 2 columns after O
+    if (warp < 4) {
+        const uint32_t lanes = static_cast<uint32_t>(warp * 32) << 16;
+#pragma unroll
+        for (int c = 0; c < QW; c += 32)
+            tmem_st32(tQ + lanes + c, *reinterpret_cast<const float(*)[32]>(qrow + c));
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(q_full);
+    }
 
     // ----------------------------------------------------- TMA producer warps
     if (warp == kVProducerWarp) {
@@ -399,8 +392,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kMmaWarp && lane == 0) {
         const uint32_t idS = idesc_bf16(BM, BN, false, false);
         const uint32_t idO = idesc_bf16(BM, D, false, true);
-        const uint32_t q_base = smem_u32(sQ);
         bool ok = mbar_wait(q_full, 0, kWaitNs);
+        tc_fence_after();
         auto issue_s = [&](int j) -> bool {
             const int s = j % NSK;
             const int sb = j & 1;
@@ -409,9 +402,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t k_base = smem_u32(sK + s * S::kv_bytes);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k) {
-                const uint64_t ad = sdesc_sw128(q_base + (k >> 2) * (BM * 128) + (k & 3) * 32, 16, 1024);
                 const uint64_t bd = sdesc_sw128(k_base + (k >> 2) * (BN * 128) + (k & 3) * 32, 16, 1024);
-                mma_bf16(tS + sb * BN, ad, bd, idS, k > 0 ? 1u : 0u);
+                mma_bf16_tmem_a(tS + sb * BN, tQ + k * 8, bd, idS, k > 0 ? 1u : 0u);
             }
             mma_commit(&s_full[sb]);
             mma_commit(&k_empty[s]);
@@ -475,27 +467,40 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after();
-            float sv[NK];
-#pragma unroll
-            for (int c = 0; c < NK; c += 32)
-                tmem_ld32(tS + lane_base + sb * BN + half * NK + c, *reinterpret_cast<float(*)[32]>(sv + c));
-            tmem_wait_ld();
-
             const bool tree_tile = (j == n_cache_tiles);
             const int key0 = kbeg + j * BN;
             const int n_valid = tree_tile ? a.T : min(BN, kend - key0);
-            // Keys of the tile this row sees: a prefix of the cache keys, or the
-            // row's ancestors among the tree keys.  Every tile runs the same
-            // instructions, so the one tree tile, late in the loop, brings no
-            // code into the instruction cache (a miss then waits on a
-            // saturated memory system).
-            const uint64_t prefix = (n_valid >= BN) ? ~0ull : ((1ull << n_valid) - 1ull);
-            const uint64_t vis = (tree_tile ? s_anc[node] : prefix) >> (half * NK);
+            // Keys of a 64-key block of the tile that this row sees: a prefix
+            // of the cache keys, or the row's ancestors among the (at most 64)
+            // tree keys.  Every tile runs the same instructions, so the one
+            // tree tile, late in the loop, brings no code into the instruction
+            // cache (a miss then waits on a saturated memory system).
+            auto block_vis = [&](int blk) -> uint64_t {
+                const int nv = n_valid - 64 * blk;
+                const uint64_t prefix = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
+                return tree_tile ? (blk == 0 ? s_anc[node] : 0ull) : prefix;
+            };
+            // this thread's NB blocks of 64 keys start at block blk0 (KS = 2:
+            // the key half; KS = 1: both halves, S re-read from TMEM per pass)
+            constexpr int NB = NK / 64;
+            const int blk0 = half * NB;
+            float sv[64];
+            auto load_block = [&](int blk) {
+                const uint32_t col = tS + lane_base + sb * BN + blk * 64;
+                tmem_ld32(col, *reinterpret_cast<float(*)[32]>(sv));
+                tmem_ld32(col + 32, *reinterpret_cast<float(*)[32]>(sv + 32));
+                tmem_wait_ld();
+                const uint64_t vis = block_vis(blk);
 #pragma unroll
-            for (int c = 0; c < NK; ++c) sv[c] = ((vis >> c) & 1ull) ? sv[c] : -INFINITY;
+                for (int c = 0; c < 64; ++c) sv[c] = ((vis >> c) & 1ull) ? sv[c] : -INFINITY;
+            };
             float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll 1
+            for (int bi = 0; bi < NB; ++bi) {
+                load_block(blk0 + bi);
 #pragma unroll
-            for (int c = 0; c < NK; ++c) mx4[c & 3] = fmaxf(mx4[c & 3], sv[c]);
+                for (int c = 0; c < 64; ++c) mx4[c & 3] = fmaxf(mx4[c & 3], sv[c]);
+            }
             const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * sc;   // sc > 0
 
             // move the reference max when this tile exceeds it by more than 2^8
@@ -525,23 +530,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             const float ref = (m_ref == -INFINITY) ? 0.f : m_ref;
+            // P of block blk (two keys per column) goes to packed columns
+            // [32 blk, 32 blk + 32) of the tile's TMEM: over S values this
+            // thread has already read (blocks in increasing order)
             float sum4[4] = {0.f, 0.f, 0.f, 0.f};
-            float pk[NK / 2];
+#pragma unroll 1
+            for (int bi = 0; bi < NB; ++bi) {
+                if (NB > 1) load_block(blk0 + bi);
+                float pk[32];
 #pragma unroll
-            for (int c = 0; c < NK; c += 2) {
-                const float p0 = ex2_approx(fmaf(sv[c], sc, -ref));
-                const float p1 = ex2_approx(fmaf(sv[c + 1], sc, -ref));
-                sum4[c & 3] += p0;
-                sum4[(c + 1) & 3] += p1;
-                pk[c >> 1] = __uint_as_float(pack_bf16x2(p0, p1));
+                for (int c = 0; c < 64; c += 2) {
+                    const float p0 = ex2_approx(fmaf(sv[c], sc, -ref));
+                    const float p1 = ex2_approx(fmaf(sv[c + 1], sc, -ref));
+                    sum4[c & 3] += p0;
+                    sum4[(c + 1) & 3] += p1;
+                    pk[c >> 1] = __uint_as_float(pack_bf16x2(p0, p1));
+                }
+                tmem_st32(tS + lane_base + sb * BN + (blk0 + bi) * 32, pk);
             }
             l_run += (sum4[0] + sum4[1]) + (sum4[2] + sum4[3]);
-            // P over the first 32 columns of this tile's S (two keys per column);
-            // with KS = 2 the other half's keys of the row read as zero here
-            float prow[32];
+            if (KS == 2) {
+                // the other half's keys of this row read as zero
+                float z[32];
 #pragma unroll
-            for (int c = 0; c < 32; ++c) prow[c] = (c / (NK / 2) == half) ? pk[c % (NK / 2)] : 0.f;
-            tmem_st32(tS + lane_base + sb * BN, prow);
+                for (int c = 0; c < 32; ++c) z[c] = 0.f;
+                tmem_st32(tS + lane_base + sb * BN + (1 - half) * 32, z);
+            }
             // value rows of keys past the valid ones may hold anything (even NaN): zero them
             if (n_valid < BN) {
                 const int s = j % NSV;
@@ -706,7 +720,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_wait(mma_done, 0, kWaitNs);
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem, kTmemCols);
+        tmem_dealloc(tmem, S::tmem_cols);
     }
     if (tree_cta && rt == 0 && threadIdx.x == 0 && *s_bad) report(a.status, CLOVER_ERR_BAD_TREE);
     if (n_split > 1) {
@@ -820,15 +834,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     }
     a.n_split = n;
 
-    // Q tile by TMA when a tile holds whole nodes: box (64 d, G heads, nodes)
-    const int G = a.G;
-    int box_nodes = 0;
-    if (a.rows <= BM) box_nodes = a.T;
-    else if (BM % G == 0) box_nodes = BM / G;
-    if (G > 256 || box_nodes > 256) box_nodes = 0;
-    a.q_box_nodes = box_nodes;
-
-    CUtensorMap kc, vc, kn, vn, qm, ks, vs;
+    CUtensorMap kc, vc, kn, vn, ks, vs;
     const uint64_t e = 2;
     if (!make_tmap_bf16_3d(&kc, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
         !make_tmap_bf16_3d(&vc, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
@@ -838,12 +844,6 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
         !make_tmap_bf16_3d(&ks, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, a.T, 1) ||
         !make_tmap_bf16_3d(&vs, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, a.T, 1))
         return cudaErrorInvalidValue;
-    if (box_nodes > 0) {
-        if (!make_tmap_bf16_3d(&qm, a.q, D, a.Hq, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hq * D * e, 64, G, box_nodes))
-            return cudaErrorInvalidValue;
-    } else {
-        qm = kn;   // unused
-    }
 
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.row_tiles, n, a.B * a.Hkv);
@@ -857,7 +857,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     attr.val.clusterDim.z = 1;
     cfg.attrs = &attr;
     cfg.numAttrs = n > 1 ? 1 : 0;
-    err = cudaLaunchKernelEx(&cfg, kernel, kc, vc, kn, vn, qm, ks, vs, a);
+    err = cudaLaunchKernelEx(&cfg, kernel, kc, vc, kn, vn, ks, vs, a);
     if (err != cudaSuccess) return err;
     return cudaGetLastError();
 }
