@@ -217,6 +217,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int kend = min(L, kbeg + chunk);
     const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
     const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
+    // the tree CTA takes its tree tile first (tile 0), so the one CTA with an
+    // extra tile does not finish on a load whose latency nothing hides
+    const int first_cache = tree_cta ? 1 : 0;
     // this CTA appends the tree K/V to cache slots [L, L+T)
     const bool appender = a.append && tree_cta && rt == 0 && !cap_bad;
 
@@ -225,25 +228,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive_expect_tx(bar, S::kv_bytes);
         const CUtensorMap *cache_map = is_v ? &tm_vc : &tm_kc;
         const CUtensorMap *new_map = is_v ? &tm_vn : &tm_kn;
-        if (j < n_cache_tiles) {
+        if (j >= first_cache) {
 #pragma unroll
-            for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + j * BN, bg);
+            for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + (j - first_cache) * BN, bg);
         } else {
 #pragma unroll
             for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, new_map, bar, dh * 64, g, b * a.T);
         }
     };
 
-    // The tree tile (the last tile of the tree CTA) holds the T new keys or
-    // values in its first T rows once it has landed; TMA stores those rows
-    // straight from the ring to cache slots [L, L+T), then waits until the
-    // store has read them (the rings are reused after the key loop).
+    // The tree tile (tile 0 of the tree CTA, ring stage 0) holds the T new
+    // keys or values in its first T rows once it has landed; TMA stores those
+    // rows straight from the ring to cache slots [L, L+T), then waits until the
+    // store has read them.  The producer does this before stage 0 takes its
+    // next tile (or after its loop when there is none).
     auto append_tile = [&](bool is_v) {
-        const int nst = is_v ? NSV : NSK;
-        const int s = n_cache_tiles % nst;
-        uint64_t *full = is_v ? &v_full[s] : &k_full[s];
-        const uint8_t *src = (is_v ? sV : sK) + s * S::kv_bytes;
-        if (*s_abort || !mbar_wait(full, (n_cache_tiles / nst) & 1, kWaitNs)) {
+        uint64_t *full = is_v ? &v_full[0] : &k_full[0];
+        const uint8_t *src = is_v ? sV : sK;
+        if (*s_abort || !mbar_wait(full, 0, kWaitNs)) {
             *s_abort = 1;
             return;
         }
@@ -356,8 +358,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ----------------------------------------------------- TMA producer warps
     if (warp == kVProducerWarp) {
         if (lane == 0) {
+            bool appended = false;
             for (int j = v_issued; j < n_tiles; ++j) {
                 const int s = j % NSV;
+                if (appender && j == NSV) {
+                    append_tile(true);
+                    appended = true;
+                }
                 if (!mbar_wait(&v_empty[s], ((j / NSV) - 1) & 1, kWaitNs)) {
                     *s_abort = 1;
                     break;
@@ -366,13 +373,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 issue_tile(j, true, sV + s * S::kv_bytes, &v_full[s]);
                 v_issued = j + 1;
             }
-            if (appender && v_issued == n_tiles) append_tile(true);
+            if (appender && !appended && v_issued == n_tiles) append_tile(true);
         }
     }
     if (warp == kKProducerWarp) {
         if (lane == 0) {
+            bool appended = false;
             for (int j = k_issued; j < n_tiles; ++j) {
                 const int s = j % NSK;
+                if (appender && j == NSK) {
+                    append_tile(false);
+                    appended = true;
+                }
                 if (!mbar_wait(&k_empty[s], ((j / NSK) - 1) & 1, kWaitNs)) {
                     *s_abort = 1;
                     break;
@@ -381,7 +393,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 issue_tile(j, false, sK + s * S::kv_bytes, &k_full[s]);
                 k_issued = j + 1;
             }
-            if (appender && k_issued == n_tiles) append_tile(false);
+            if (appender && !appended && k_issued == n_tiles) append_tile(false);
         }
     }
 
@@ -467,8 +479,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after();
-            const bool tree_tile = (j == n_cache_tiles);
-            const int key0 = kbeg + j * BN;
+            const bool tree_tile = tree_cta && j == 0;
+            const int key0 = kbeg + (j - first_cache) * BN;
             const int n_valid = tree_tile ? a.T : min(BN, kend - key0);
             // Keys of a 64-key block of the tile that this row sees: a prefix
             // of the cache keys, or the row's ancestors among the (at most 64)
