@@ -116,6 +116,28 @@ def test_full_size_workloads(name, cuda):
 
 
 # ---------------------------------------------------------------------------
+# every split count of the tensor-core path's cluster merge
+# ---------------------------------------------------------------------------
+
+# One KV head, so the launcher's split count is min(8, Lcap / 256 rounded up):
+# these cache lengths give 2, 3, 4, 5, 6, 7 and 8 splits.
+SPLIT_LENGTHS = [300, 700, 1000, 1200, 1500, 1700, 3000]
+
+
+@pytest.mark.parametrize("L", SPLIT_LENGTHS)
+@pytest.mark.parametrize("Hq,D", [(4, 128), (8, 128), (8, 64)])
+def test_split_counts_and_row_groups(L, Hq, D, cuda):
+    """T=16 with 4 query heads per KV head is a 64-row tile (two key groups per
+    row); 8 heads make a 128-row tile (one key group); D=64 takes the smaller
+    shared-memory plan."""
+    w = workloads.get("7b_l2048", B=1, T=16, Hq=Hq, Hkv=1, D=D, L=L, V=1000, branching=(4, 2, 1, 1))
+    host = workloads.make(w)
+    t = to_dev(host, cuda)
+    step = run_gpu(t)
+    compare_full(host, step, t)
+
+
+# ---------------------------------------------------------------------------
 # the two schedules of a step
 # ---------------------------------------------------------------------------
 
