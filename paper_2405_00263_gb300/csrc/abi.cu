@@ -29,7 +29,6 @@ constexpr int kSms = 152;                  // SMs of a GB300 (planning constant;
 constexpr int kTargetAttnCtas = 2 * kSms;  // FMA path: two resident CTAs per SM
 constexpr int kMinKeysPerSplit = 256;
 constexpr int kMaxSplits = 64;
-constexpr int kTcMinRows = 16;             // query rows per KV head from which the tensor-core path is used
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -50,10 +49,12 @@ clover_status check_attn_sizes(int B, int T, int Hq, int Hkv, int D, int Lcap, i
     return CLOVER_OK;
 }
 
-// Kernel choice, split count and workspace layout for one shape.  bf16 with at
-// least kTcMinRows query rows per KV head runs on the tensor cores (one CTA per
-// SM, splits merged on chip, no workspace); everything else runs on the FMA
-// kernel with two CTAs per SM and merges splits through the workspace.
+// Kernel choice, split count and workspace layout for one shape.  bf16 runs on
+// the tensor cores (one CTA per SM, splits merged on chip, no workspace) for
+// any number of query rows: even a 4-row tile is bound by HBM there, as the
+// MMA cost of a 128-key tile (about 0.8 us) stays below its HBM time.  fp32
+// runs on the FMA kernel with two CTAs per SM and merges splits through the
+// workspace.
 AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
     AttnPlan p;
     const int G = Hq / Hkv;
@@ -61,7 +62,7 @@ AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
     const long Bp = B > 0 ? B : 1;
     const int by_len = (Lcap + kMinKeysPerSplit - 1) / kMinKeysPerSplit;
     int n;
-    p.tc = (dtype == CLOVER_BF16) && rows >= kTcMinRows;
+    p.tc = (dtype == CLOVER_BF16);
     if (p.tc) {
         // the tensor-core kernel picks its split count at launch (one wave of
         // thread-block clusters) and merges splits in distributed shared memory:

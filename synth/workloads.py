@@ -88,6 +88,19 @@ WORKLOADS = {
         L_range=(512, 8192),
         description="7B-class batched: B16, L_b ~ U[512,8192], 32 heads MHA, D128, "
                     "32-node tree depth 4, V125696, bf16"),
+    # the paper's own serving regime (tree size 4, batch 4-48, 7B MHA shapes, L around 2k)
+    "paper_t4_b4": Workload(
+        "paper_t4_b4", B=4, T=4, Hq=32, Hkv=32, D=128, L=2560, V=125696, dtype="bf16",
+        branching=(2, 1), plant_p=0.5, qkv_std=1 / math.sqrt(128), seed=5, L_range=(1536, 2560),
+        description="paper regime: B4, L_b ~ U[1536,2560], 32 heads MHA, D128, 4-node tree, V125696, bf16"),
+    "paper_t4_b16": Workload(
+        "paper_t4_b16", B=16, T=4, Hq=32, Hkv=32, D=128, L=2560, V=125696, dtype="bf16",
+        branching=(2, 1), plant_p=0.5, qkv_std=1 / math.sqrt(128), seed=6, L_range=(1536, 2560),
+        description="paper regime: B16, L_b ~ U[1536,2560], 32 heads MHA, D128, 4-node tree, V125696, bf16"),
+    "paper_t4_b48": Workload(
+        "paper_t4_b48", B=48, T=4, Hq=32, Hkv=32, D=128, L=2560, V=125696, dtype="bf16",
+        branching=(2, 1), plant_p=0.5, qkv_std=1 / math.sqrt(128), seed=7, L_range=(1536, 2560),
+        description="paper regime: B48, L_b ~ U[1536,2560], 32 heads MHA, D128, 4-node tree, V125696, bf16"),
     "100b_gqa": Workload(
         "100b_gqa", B=4, T=64, Hq=64, Hkv=8, D=128, L=8192, V=125696, dtype="bf16",
         branching=(8, 4, 2, 2, 1), plant_p=0.5, qkv_std=1 / math.sqrt(128), seed=4,

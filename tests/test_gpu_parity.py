@@ -65,7 +65,7 @@ def test_repeated_calls_reuse_workspace(cuda):
     compare_full(host, step, t2)
 
 
-FULL = ["7b_l2048", "7b_l4096", "7b_l16384", "7b_batched", "100b_gqa"]
+FULL = ["7b_l2048", "7b_l4096", "7b_l16384", "7b_batched", "100b_gqa", "paper_t4_b4", "paper_t4_b16", "paper_t4_b48"]
 
 
 @pytest.mark.parametrize("name", FULL)
