@@ -60,6 +60,7 @@ def _load():
             lib.oracle_append_tree_kv.argtypes = [P, P, P, P, P, I, I, I, I, I, I]
             lib.oracle_kv_compact.argtypes = [P, P, P, P, P, I, I, I, I, I, I, P]
             lib.oracle_kv_commit.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P]
+            lib.oracle_accept_typical.argtypes = [P, P, P, I, I, I64, I, D, D, D, P, P, P, P, P, I]
             for f in (lib.oracle_tree_mask, lib.oracle_tree_attention, lib.oracle_argmax,
                       lib.oracle_accept_walk, lib.oracle_append_tree_kv, lib.oracle_kv_compact,
                       lib.oracle_kv_commit):
@@ -167,6 +168,28 @@ def accept_walk(parent, cand, amax):
     _check(_load().oracle_accept_walk(_p(par), _p(cd), _p(am), B, T, _p(path), _p(alen),
                                       _p(bonus)))
     return path, alen, bonus
+
+
+def accept_typical(logits, parent, cand, temperature: float, epsilon: float, delta: float,
+                   n_threads: int | None = None) -> dict:
+    """Typical acceptance of every sequence.  logits [B, T, V] (or [B*T, V]),
+    parent/cand [B, T].  Returns argmax [B,T], path [B,T], accept_len [B],
+    bonus [B] (int32) and margin [B,T] (fp64, ln p - ln theta per edge)."""
+    par = _cpu(parent.to(torch.int32))
+    cd = _cpu(cand.to(torch.int32))
+    B, T = par.shape
+    lg = _cpu(logits)
+    V = lg.shape[-1]
+    assert lg.numel() == B * T * V
+    amax = torch.empty((B, T), dtype=torch.int32)
+    path = torch.empty((B, T), dtype=torch.int32)
+    alen = torch.empty(B, dtype=torch.int32)
+    bonus = torch.empty(B, dtype=torch.int32)
+    margin = torch.empty((B, T), dtype=torch.float64)
+    _check(_load().oracle_accept_typical(_p(lg), _p(par), _p(cd), B, T, V, _dtype_code(lg), float(temperature),
+                                         float(epsilon), float(delta), _p(amax), _p(path), _p(alen), _p(bonus),
+                                         _p(margin), n_threads or default_threads()))
+    return {"argmax": amax, "path": path, "accept_len": alen, "bonus": bonus, "margin": margin}
 
 
 def append_tree_kv(k_new, v_new, k_cache, v_cache, cache_len):

@@ -23,6 +23,11 @@
  *             repeatedly accept the smallest-index child whose candidate token
  *             equals the current node's argmax; the accepted length is the
  *             number of nodes on the path, the bonus token the argmax at its end.
+ *   typical   Section 4 (experiment setup): the tree sampling algorithm taken
+ *             over from Medusa; the edge into a child is accepted when its
+ *             token's probability under the tempered softmax of the parent's
+ *             logits exceeds min(epsilon, delta * exp(-entropy)); the longest
+ *             accepted path wins (ties: lexicographically smallest).
  *   append /  (engine step; the paper is silent) the T tree keys/values occupy
  *   compact   cache slots [L, L+T); the accepted nodes' K/V are then moved, in
  *             path order, to slots [L, L+a) and the length becomes L + a.
@@ -354,4 +359,144 @@ int oracle_kv_commit(void *k_cache, void *v_cache, const void *k_new, const void
         cache_len[b] = L + a;
     }
     return ORACLE_OK;
+}
+
+/*
+ * Typical acceptance: the sampling-side acceptance rule of the tree sampling
+ * algorithm the paper evaluates with (Section 4, experiment setup; the rule is
+ * Medusa's).  All in fp64 on exactly widened logits x of each node i:
+ *   p_i    = softmax(x_i / temperature)
+ *   H_i    = -sum_v p_i(v) ln p_i(v)            (terms with p = 0 add nothing)
+ *   theta_i = min(epsilon, delta * exp(-H_i))
+ * The edge into child c (parent i) is accepted iff p_i(cand[c]) > theta_i,
+ * decided as ln p > ln theta (ln 0 = -inf, so theta = 0 accepts every token of
+ * positive probability); a candidate outside [0, V) is rejected.  A node is
+ * accepted when every edge on its path from the root is; the root always is.
+ * The chosen path ends at the deepest accepted node; among equally deep ones
+ * it is the lexicographically smallest sequence of node indices.  accept_len
+ * is its node count, bonus the argmax of the last node's logits.
+ * argmax_out [B,T] (first index of the maximum), path [B,T] (-1 padded),
+ * margin [B,T]: ln p - ln theta of the edge into each node (root: +inf;
+ * p = 0 or an invalid candidate: -inf).
+ */
+int oracle_accept_typical(const void *logits, const int32_t *parent, const int32_t *cand, int B, int T,
+                          int64_t V, int dtype, double temperature, double epsilon, double delta,
+                          int32_t *argmax_out, int32_t *path, int32_t *accept_len, int32_t *bonus,
+                          double *margin, int n_threads)
+{
+    if (V < 1 || T < 1 || !(temperature > 0.0) || !isfinite(temperature) || !(epsilon >= 0.0) ||
+        !isfinite(epsilon) || !(delta >= 0.0) || !isfinite(delta))
+        return ORACLE_BAD_ARG;
+    for (int b = 0; b < B; ++b)
+        if (!tree_is_valid(parent + (int64_t)b * T, T)) return ORACLE_BAD_TREE;
+    const int64_t rows = (int64_t)B * T;
+    double *row_max = malloc(sizeof(double) * (size_t)rows);     /* max of x / temperature */
+    double *row_lse = malloc(sizeof(double) * (size_t)rows);     /* ln sum exp(z - max) */
+    double *row_log_theta = malloc(sizeof(double) * (size_t)rows);
+    int32_t *row_amax = malloc(sizeof(int32_t) * (size_t)rows);
+    if (!row_max || !row_lse || !row_log_theta || !row_amax) {
+        free(row_max);
+        free(row_lse);
+        free(row_log_theta);
+        free(row_amax);
+        return ORACLE_NO_MEMORY;
+    }
+#pragma omp parallel for schedule(static) num_threads(n_threads > 0 ? n_threads : 1)
+    for (int64_t r = 0; r < rows; ++r) {
+        double best = load_elem(logits, r * V, dtype);
+        int64_t best_v = 0;
+        double m = -INFINITY;
+        for (int64_t v = 0; v < V; ++v) {
+            const double x = load_elem(logits, r * V + v, dtype);
+            if (x > best) {
+                best = x;
+                best_v = v;
+            }
+            const double z = x / temperature;
+            if (z > m) m = z;
+        }
+        double s = 0.0;
+        for (int64_t v = 0; v < V; ++v) s += exp(load_elem(logits, r * V + v, dtype) / temperature - m);
+        const double lse = log(s);
+        double h = 0.0;
+        for (int64_t v = 0; v < V; ++v) {
+            const double log_p = load_elem(logits, r * V + v, dtype) / temperature - m - lse;
+            const double p = exp(log_p);
+            if (p > 0.0) h -= p * log_p;
+        }
+        row_amax[r] = (int32_t)best_v;
+        row_max[r] = m;
+        row_lse[r] = lse;
+        const double log_eps = log(epsilon);           /* -inf for 0 */
+        const double log_dh = log(delta) - h;          /* ln(delta e^-H) */
+        row_log_theta[r] = log_eps < log_dh ? log_eps : log_dh;
+    }
+    int32_t *acc = malloc(sizeof(int32_t) * (size_t)T);
+    int32_t *reach = malloc(sizeof(int32_t) * (size_t)T);
+    int32_t *depth = malloc(sizeof(int32_t) * (size_t)T);
+    int32_t *best_path = malloc(sizeof(int32_t) * (size_t)T);
+    int32_t *this_path = malloc(sizeof(int32_t) * (size_t)T);
+    int status = ORACLE_OK;
+    if (!acc || !reach || !depth || !best_path || !this_path) status = ORACLE_NO_MEMORY;
+    for (int b = 0; b < B && status == ORACLE_OK; ++b) {
+        const int32_t *par = parent + (int64_t)b * T;
+        const int32_t *cd = cand + (int64_t)b * T;
+        double *mg = margin + (int64_t)b * T;
+        for (int c = 0; c < T; ++c) argmax_out[(int64_t)b * T + c] = row_amax[(int64_t)b * T + c];
+        /* each edge on its own */
+        acc[0] = 1;
+        mg[0] = INFINITY;
+        for (int c = 1; c < T; ++c) {
+            const int64_t r = (int64_t)b * T + par[c];
+            if (cd[c] < 0 || (int64_t)cd[c] >= V) {
+                acc[c] = 0;
+                mg[c] = -INFINITY;
+                continue;
+            }
+            const double log_p = load_elem(logits, r * V + cd[c], dtype) / temperature - row_max[r] - row_lse[r];
+            acc[c] = log_p > row_log_theta[r];
+            mg[c] = log_p == -INFINITY ? -INFINITY : log_p - row_log_theta[r];
+        }
+        /* accepted nodes and their depths (parents come before children) */
+        reach[0] = 1;
+        depth[0] = 0;
+        for (int c = 1; c < T; ++c) {
+            reach[c] = reach[par[c]] && acc[c];
+            depth[c] = depth[par[c]] + 1;
+        }
+        /* deepest accepted node; ties by the lexicographically smallest path */
+        int best_len = 0;
+        for (int c = 0; c < T; ++c) {
+            if (!reach[c]) continue;
+            const int len = depth[c] + 1;
+            for (int n = c, k = len - 1; n >= 0; n = par[n], --k) this_path[k] = n;
+            int better = len > best_len;
+            if (len == best_len) {
+                for (int k = 0; k < len; ++k) {
+                    if (this_path[k] != best_path[k]) {
+                        better = this_path[k] < best_path[k];
+                        break;
+                    }
+                }
+            }
+            if (better) {
+                best_len = len;
+                memcpy(best_path, this_path, sizeof(int32_t) * (size_t)len);
+            }
+        }
+        int32_t *pb = path + (int64_t)b * T;
+        for (int k = 0; k < T; ++k) pb[k] = k < best_len ? best_path[k] : -1;
+        accept_len[b] = best_len;
+        bonus[b] = row_amax[(int64_t)b * T + best_path[best_len - 1]];
+    }
+    free(acc);
+    free(reach);
+    free(depth);
+    free(best_path);
+    free(this_path);
+    free(row_max);
+    free(row_lse);
+    free(row_log_theta);
+    free(row_amax);
+    return status;
 }

@@ -550,3 +550,173 @@ def test_verify_step_tiny_invariants():
     p = r["path"][0, :a].tolist()
     assert torch.equal(r["k_cache"][0, :, L:L + a], t["k_new"][0, p].permute(1, 0, 2))
     assert torch.equal(r["v_cache"][0, :, L:L + a], t["v_new"][0, p].permute(1, 0, 2))
+
+
+# ---------------------------------------------------------------------------
+# A6: typical acceptance (the sampling-side acceptance rule)
+# ---------------------------------------------------------------------------
+
+def typical_by_library(logits, parent, cand, tau, eps, delta):
+    """Independent statement with library routines: scipy's softmax and
+    entropy in fp64, the threshold compared in the probability domain, and
+    the path chosen among every fully accepted root path by sort order."""
+    special = pytest.importorskip("scipy.special")
+    stats = pytest.importorskip("scipy.stats")
+    x = logits.double().numpy()
+    T, V = x.shape
+    p = special.softmax(x / tau, axis=-1)
+    theta = np.minimum(eps, delta * np.exp(-stats.entropy(p, axis=-1)))
+    ok = [True] + [0 <= cand[c] < V and bool(p[parent[c], cand[c]] > theta[parent[c]]) for c in range(1, T)]
+    good = [root_path(parent, i) for i in range(T) if all(ok[n] for n in root_path(parent, i))]
+    best = sorted(good, key=lambda q: (-len(q), q))[0]
+    log_margin = [math.inf] + [
+        (math.log(p[parent[c], cand[c]]) - math.log(theta[parent[c]]) if theta[parent[c]] > 0 else math.inf)
+        if 0 <= cand[c] < V else -math.inf for c in range(1, T)]
+    return best, int(np.argmax(x[best[-1]])), np.argmax(x, axis=-1), log_margin
+
+
+def run_typical(logits, parent, cand, tau, eps, delta):
+    T, V = logits.shape
+    r = oracle.accept_typical(logits.reshape(1, T, V), torch.tensor([parent]), torch.tensor([cand]), tau, eps, delta)
+    a = int(r["accept_len"][0])
+    return r["path"][0, :a].tolist(), int(r["bonus"][0]), r["argmax"][0], r["margin"][0], r["path"][0, a:]
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_typical_brute_force_vs_library(dtype):
+    g = torch.Generator().manual_seed(11)
+    n = 0
+    for T in (1, 2, 4, 6, 9):
+        for V in (1, 2, 7, 33):
+            for tau, eps, delta in ((1.0, 0.09, 0.3), (0.3, 0.3, 0.55), (2.5, 0.0, 0.3), (0.7, 0.2, 0.0),
+                                    (1.0, 0.05, 0.9)):
+                for rep in range(3):
+                    parent = trees.random_tree(T, seed=100 * T + rep, tag=V)
+                    logits = (torch.randn(T, V, generator=g, dtype=torch.float64) * 2.0).to(dtype)
+                    cand = torch.randint(-1, V + 1, (T,), generator=g).tolist()
+                    path, bonus, amax, margin, tail = run_typical(logits, parent, cand, tau, eps, delta)
+                    bp, bb, ba, bm = typical_by_library(logits, parent, cand, tau, eps, delta)
+                    assert amax.tolist() == ba.tolist()
+                    for c in range(T):
+                        if math.isinf(bm[c]):
+                            assert float(margin[c]) == bm[c]
+                        else:
+                            assert float(margin[c]) == pytest.approx(bm[c], rel=1e-9, abs=1e-9)
+                    assert min(abs(float(m)) for m in margin) > 1e-9       # no edge on the boundary
+                    assert path == bp and bonus == bb and (tail == -1).all()
+                    n += 1
+    assert n == 2 * 0 + 5 * 4 * 5 * 3
+
+
+def test_typical_two_token_worked_example():
+    """V = 2, logits (ln 4, 0) at temperature 1: p = (0.8, 0.2), entropy
+    0.5004024 nats, e^-H = 0.6062866.  Child token 1 has p = 0.2.
+    (eps, delta) = (0.09, 0.3): theta = min(0.09, 0.1818860) = 0.09, accepted,
+    margin ln(0.2 / 0.09) = 0.7985077.  (0.25, 0.4): theta = 0.2425147,
+    rejected, margin ln(0.2 / 0.2425147) = -0.1927447.  Doubling both the
+    logits and the temperature changes nothing."""
+    for scale in (1.0, 2.0):
+        logits = torch.tensor([[math.log(4.0) * scale, 0.0], [0.0, 0.0]], dtype=torch.float64).float()
+        path, bonus, amax, margin, _ = run_typical(logits, [-1, 0], [7, 1], scale, 0.09, 0.3)
+        assert path == [0, 1] and bonus == 0 and amax.tolist() == [0, 0]
+        assert float(margin[1]) == pytest.approx(0.7985077, abs=2e-6)
+        path, bonus, _, margin, _ = run_typical(logits, [-1, 0], [7, 1], scale, 0.25, 0.4)
+        assert path == [0] and bonus == 0
+        assert float(margin[1]) == pytest.approx(-0.1927447, abs=2e-6)
+        # token 0 (p = 0.8) passes either threshold
+        path, _, _, margin, _ = run_typical(logits, [-1, 0], [7, 0], scale, 0.25, 0.4)
+        assert path == [0, 1] and float(margin[1]) == pytest.approx(math.log(0.8 / 0.2425147), abs=2e-6)
+
+
+def test_typical_uniform_logits_accept_every_edge():
+    """Uniform logits: p = 1/V and H = ln V, so theta = min(eps, delta / V);
+    with delta < 1 < eps * V every edge passes with margin -ln(delta)."""
+    V, delta = 1000, 0.5
+    for branching, T in (([3, 2, 2], 10), ([1, 1, 1, 1], 5), ([4], 5)):
+        parent = trees.topk_tree(T, branching)
+        logits = torch.zeros(T, V, dtype=torch.bfloat16)
+        cand = [0] + [(7 * c) % V for c in range(1, T)]
+        path, bonus, _, margin, _ = run_typical(logits, parent, cand, 0.8, 0.09, delta)
+        _, depth = oracle.tree_mask(parent)
+        deepest = [i for i in range(T) if int(depth[i]) == int(depth.max())]
+        assert path == min(root_path(parent, i) for i in deepest)
+        assert bonus == 0
+        assert np.allclose(margin[1:].numpy(), -math.log(delta), atol=1e-12)
+
+
+def test_typical_zero_epsilon_and_degenerate_candidates():
+    """eps = 0: theta = 0 and every finite candidate passes, however unlikely
+    (here p ~ e^-2000); a -inf logit (p = 0) and a token outside [0, V) do not."""
+    V = 16
+    parent = [-1, 0, 0, 1, 2, 4]
+    logits = torch.zeros(6, V, dtype=torch.float32)
+    logits[:, 3] = 2000.0
+    cand = [0, 5, 9, 1, 2, 8]
+    path, bonus, _, margin, _ = run_typical(logits, parent, cand, 1.0, 0.0, 0.3)
+    assert path == [0, 2, 4, 5] and bonus == 3
+    assert all(math.isinf(float(m)) and float(m) > 0 for m in margin)
+    logits[4, 8] = -math.inf                   # node 5's token under its parent 4
+    path, _, _, margin, _ = run_typical(logits, parent, cand, 1.0, 0.0, 0.3)
+    assert path == [0, 1, 3] and float(margin[5]) == -math.inf
+    cand[3] = V                                 # out of range: rejected
+    path, _, _, margin, _ = run_typical(logits, parent, cand, 1.0, 0.0, 0.3)
+    assert path == [0, 2, 4] and float(margin[3]) == -math.inf
+
+
+def test_typical_small_temperature_is_greedy_on_distinct_siblings():
+    """As the temperature goes to 0 the tempered softmax puts all mass on the
+    argmax: with logit gaps >= 0.01 and temperature 1e-3 the runner-up has
+    p < e^-10, the argmax p > 1 - V e^-10 and H ~ 0, so the accepted edges
+    are exactly those whose token is the parent's argmax.  With distinct
+    siblings that is a single chain: the greedy walk."""
+    g = torch.Generator().manual_seed(5)
+    V = 40
+    for seed in range(40):
+        T = 2 + seed % 20
+        parent = trees.random_tree(T, seed=seed, tag=3)
+        logits = torch.stack([torch.randperm(V, generator=g).double() * 0.01 for _ in range(T)]).float()
+        amax = logits.argmax(-1).tolist()
+        cand = [0] * T
+        for n in range(T):
+            kids = [c for c in range(T) if parent[c] == n]
+            toks = torch.randperm(V, generator=g)[:len(kids)].tolist()
+            if kids and torch.rand(1, generator=g).item() < 0.7:
+                j = int(torch.randint(len(kids), (1,), generator=g))
+                if amax[n] in toks:
+                    toks[toks.index(amax[n])] = toks[j]
+                toks[j] = amax[n]
+            for c, tok in zip(kids, toks):
+                cand[c] = tok
+        path, bonus, _, _, _ = run_typical(logits, parent, cand, 1e-3, 0.09, 0.3)
+        gp, ga, gb = oracle.accept_walk(torch.tensor([parent]), torch.tensor([cand]), torch.tensor([amax]))
+        assert path == gp[0, :int(ga[0])].tolist() and bonus == int(gb[0])
+
+
+def test_typical_epsilon_monotone_and_rejects_bad_arguments():
+    g = torch.Generator().manual_seed(9)
+    T, V = 12, 64
+    parent = trees.topk_tree(T, [3, 2, 2])
+    logits = (torch.randn(T, V, generator=g) * 1.5).to(torch.bfloat16)
+    top = logits.float().topk(3, -1).indices
+    cand = [0] * T
+    for n in range(T):                       # children take the parent's top tokens in sibling order
+        for k, c in enumerate(c for c in range(T) if parent[c] == n):
+            cand[c] = int(top[n, k])
+    # delta = 10 keeps delta e^-H above eps, so theta = eps
+    for delta in (10.0, 0.3):
+        lens = [len(run_typical(logits, parent, cand, 1.0, eps, delta)[0])
+                for eps in (0.0, 0.02, 0.05, 0.1, 0.2, 0.5)]
+        assert lens == sorted(lens, reverse=True)
+        assert delta != 10.0 or lens[0] == 4 > lens[-1]
+    lg = logits.reshape(1, T, V)
+    par, cd = torch.tensor([parent]), torch.tensor([cand])
+    for tau, eps, delta in ((0.0, 0.1, 0.3), (-1.0, 0.1, 0.3), (math.nan, 0.1, 0.3), (math.inf, 0.1, 0.3),
+                            (1.0, -0.1, 0.3), (1.0, math.nan, 0.3), (1.0, 0.1, -1.0), (1.0, 0.1, math.inf)):
+        with pytest.raises(oracle.OracleError) as e:
+            oracle.accept_typical(lg, par, cd, tau, eps, delta)
+        assert e.value.code == oracle.BAD_ARG
+    bad = torch.tensor([parent])
+    bad[0, 3] = 5
+    with pytest.raises(oracle.OracleError) as e:
+        oracle.accept_typical(lg, bad, cd, 1.0, 0.1, 0.3)
+    assert e.value.code == oracle.BAD_TREE
