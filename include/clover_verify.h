@@ -12,6 +12,9 @@
  *   clover_verify_accept  per-node argmax of the logits and the greedy walk
  *                         that selects the accepted path (Section 2.1; the
  *                         tokens/step metric of Section 4.1);
+ *   clover_verify_accept_typical
+ *                         the same with the sampling-side (typical) acceptance
+ *                         rule of the paper's tree sampling algorithm (Section 4);
  *   clover_kv_compact     moves the accepted nodes' K/V to the front of the
  *                         tree slots (an engine step the paper leaves implicit).
  *
@@ -165,6 +168,48 @@ CLOVER_API size_t clover_verify_accept_workspace_size(int B, int T, int V, clove
  */
 CLOVER_API clover_status clover_verify_accept(const void *logits, const int32_t *cand, const int32_t *parent,
                                    int B, int T, int V, clover_dtype dtype,
+                                   int32_t *argmax_out, int32_t *path_out,
+                                   int32_t *accept_len, int32_t *bonus_token,
+                                   void *workspace, size_t ws_bytes,
+                                   int32_t *status, void *stream);
+
+/* Bytes of device workspace clover_verify_accept_typical needs (0 outside the limits). */
+CLOVER_API size_t clover_verify_accept_typical_workspace_size(int B, int T, int V, clover_dtype dtype);
+
+/*
+ * Typical acceptance: the sampling-side acceptance rule of the tree sampling
+ * algorithm the paper evaluates with (Section 4, experiment setup; the rule
+ * is Medusa's), beside the greedy rule of clover_verify_accept.  For node i
+ * with logit row x_i:
+ *     p_i = softmax(x_i / temperature),  H_i = -sum_v p_i(v) ln p_i(v),
+ *     theta_i = min(epsilon, delta * exp(-H_i)).
+ * The edge into child c (parent i) is accepted iff p_i(cand[c]) > theta_i; a
+ * candidate outside [0, V) is rejected.  The accepted path ends at the deepest
+ * node whose every edge from the root is accepted; among equally deep ones it
+ * is the one that takes the smallest-index child at every step (the
+ * lexicographically smallest node sequence).  No random numbers are drawn.
+ *
+ *   logits, cand, parent     as for clover_verify_accept; logits must be finite
+ *                            or -inf (p = 0), with a finite maximum in every row
+ *                            (+inf or NaN: outputs unspecified)
+ *   temperature              > 0 and finite, with log2(e)/temperature a normal
+ *                            fp32 number (else CLOVER_ERR_UNSUPPORTED)
+ *   epsilon, delta           >= 0 and finite (0 makes theta 0: every candidate
+ *                            of positive probability passes)
+ *   argmax_out, path_out, accept_len, bonus_token
+ *                            as for clover_verify_accept (the bonus token is the
+ *                            argmax at the last accepted node)
+ *   workspace, ws_bytes      >= clover_verify_accept_typical_workspace_size(...)
+ *                            bytes, 16-byte aligned, zero-filled before first
+ *                            use; left ready for the next call.  Calls sharing
+ *                            it must not overlap on the device.
+ * Precision: the softmax sums, the entropy and the comparison are fp32
+ * (base-2 exponent and logarithm instructions); an edge whose ln p - ln theta
+ * is within about 1e-4 of zero may be decided either way.
+ */
+CLOVER_API clover_status clover_verify_accept_typical(const void *logits, const int32_t *cand,
+                                   const int32_t *parent, int B, int T, int V, clover_dtype dtype,
+                                   double temperature, double epsilon, double delta,
                                    int32_t *argmax_out, int32_t *path_out,
                                    int32_t *accept_len, int32_t *bonus_token,
                                    void *workspace, size_t ws_bytes,

@@ -25,6 +25,8 @@ EXPORTS = (
     "clover_verify_attn_ex",
     "clover_verify_accept_workspace_size",
     "clover_verify_accept",
+    "clover_verify_accept_typical_workspace_size",
+    "clover_verify_accept_typical",
     "clover_kv_compact",
     "clover_kv_commit",
     "clover_verify_attn_noalloc",
@@ -72,6 +74,11 @@ def load(build_if_missing: bool = False):
         lib.clover_verify_accept_workspace_size.restype = Z
         lib.clover_verify_accept.argtypes = [P, P, P, I, I, I, I, P, P, P, P, P, Z, P, P]
         lib.clover_verify_accept.restype = I
+        lib.clover_verify_accept_typical_workspace_size.argtypes = [I, I, I, I]
+        lib.clover_verify_accept_typical_workspace_size.restype = Z
+        lib.clover_verify_accept_typical.argtypes = [P, P, P, I, I, I, I, ctypes.c_double, ctypes.c_double,
+                                                     ctypes.c_double, P, P, P, P, P, Z, P, P]
+        lib.clover_verify_accept_typical.restype = I
         lib.clover_kv_compact.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P, P]
         lib.clover_kv_compact.restype = I
         lib.clover_kv_commit.argtypes = [P, P, P, P, P, P, P, P, P, I, I, I, I, I, I, P, P]

@@ -89,6 +89,11 @@ def clover_verify_accept_workspace_size(B, T, V, dtype) -> int:
     return int(_lib.load().clover_verify_accept_workspace_size(B, T, V, code))
 
 
+def clover_verify_accept_typical_workspace_size(B, T, V, dtype) -> int:
+    code = dtype if isinstance(dtype, int) else dtype_code(dtype)
+    return int(_lib.load().clover_verify_accept_typical_workspace_size(B, T, V, code))
+
+
 def clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, scale=0.0,
                        workspace=None, status=None, stream=None, append=True):
     """Tree-masked attention; with ``append`` (clover_verify_attn) it also
@@ -164,6 +169,29 @@ def clover_verify_accept(logits, cand, parent, argmax_out, path_out, accept_len,
         _stream(stream))
     if code != OK:
         raise CloverError(code, "clover_verify_accept")
+
+
+def clover_verify_accept_typical(logits, cand, parent, temperature, epsilon, delta, argmax_out, path_out,
+                                 accept_len, bonus_token, workspace, status=None, stream=None):
+    """Per-node argmax and the typical (tempered-softmax, entropy-threshold)
+    acceptance of the longest accepted path."""
+    B, T, V = logits.shape
+    _check(cand, (B, T), torch.int32, "cand")
+    _check(parent, (B, T), torch.int32, "parent")
+    _check(argmax_out, (B, T), torch.int32, "argmax_out")
+    _check(path_out, (B, T), torch.int32, "path_out")
+    _check(accept_len, (B,), torch.int32, "accept_len")
+    _check(bonus_token, (B,), torch.int32, "bonus_token")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(logits, cand, parent, argmax_out, path_out, accept_len, bonus_token, workspace, status)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    code = _lib.load().clover_verify_accept_typical(
+        _ptr(logits), _ptr(cand), _ptr(parent), B, T, V, dtype_code(logits.dtype), float(temperature),
+        float(epsilon), float(delta), _ptr(argmax_out), _ptr(path_out), _ptr(accept_len), _ptr(bonus_token),
+        _ptr(workspace), ws_bytes, _ptr(status), _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_verify_accept_typical")
 
 
 def clover_kv_compact(k_cache, v_cache, cache_len, path, accept_len, new_cache_len, src_index_out=None,

@@ -17,6 +17,11 @@ size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T, int V,
                           int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len, int32_t *bonus,
                           void *workspace, int32_t *status, cudaStream_t stream);
+size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype);
+cudaError_t launch_accept_typical(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
+                                  int V, int dtype, float y_scale, float log2_eps, float log2_delta,
+                                  int32_t *argmax_out, int32_t *path_out, int32_t *accept_len, int32_t *bonus,
+                                  void *workspace, int32_t *status, cudaStream_t stream);
 cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
                               const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
                               int32_t *new_cache_len, int32_t *src_index, int B, int T, int Hkv, int D, int Lcap,
@@ -234,6 +239,40 @@ clover_status clover_verify_accept(const void *logits, const int32_t *cand, cons
     if (reinterpret_cast<uintptr_t>(logits) % (dtype == CLOVER_F32 ? 4 : 2)) return CLOVER_ERR_INVALID_ARG;
     return from_cuda(launch_accept(logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
                                    bonus_token, workspace, status, static_cast<cudaStream_t>(stream)));
+}
+
+size_t clover_verify_accept_typical_workspace_size(int B, int T, int V, clover_dtype dtype) {
+    if (B < 0 || T < 1 || T > kMaxTreeNodes || V < 1) return 0;
+    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return 0;
+    return accept_typical_workspace_bytes(B > 0 ? B : 1, T, V, dtype);
+}
+
+clover_status clover_verify_accept_typical(const void *logits, const int32_t *cand, const int32_t *parent, int B,
+                                           int T, int V, clover_dtype dtype, double temperature, double epsilon,
+                                           double delta, int32_t *argmax_out, int32_t *path_out,
+                                           int32_t *accept_len, int32_t *bonus_token, void *workspace,
+                                           size_t ws_bytes, int32_t *status, void *stream) {
+    if (B < 0 || T < 1 || V < 1) return CLOVER_ERR_INVALID_ARG;
+    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
+    if (!(temperature > 0.0) || !isfinite(temperature) || !(epsilon >= 0.0) || !isfinite(epsilon) ||
+        !(delta >= 0.0) || !isfinite(delta))
+        return CLOVER_ERR_INVALID_ARG;
+    // exponents are kept in base 2: y = x log2(e) / temperature, in fp32
+    const float y_scale = (float)(1.4426950408889634 / temperature);
+    if (!isfinite(y_scale) || !(y_scale >= 1.17549435e-38f)) return CLOVER_ERR_UNSUPPORTED;
+    if (T > kMaxTreeNodes) return CLOVER_ERR_UNSUPPORTED;
+    if (B == 0) return CLOVER_OK;
+    if ((long)B * T > 0x7FFFFFFFL) return CLOVER_ERR_UNSUPPORTED;
+    if (!logits || !cand || !parent || !argmax_out || !path_out || !accept_len || !bonus_token)
+        return CLOVER_ERR_INVALID_ARG;
+    const size_t need = accept_typical_workspace_bytes(B, T, V, dtype);
+    if (ws_bytes < need || !workspace || !aligned16(workspace)) return CLOVER_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(logits) % (dtype == CLOVER_F32 ? 4 : 2)) return CLOVER_ERR_INVALID_ARG;
+    const float log2_eps = epsilon > 0.0 ? (float)log2(epsilon) : -INFINITY;
+    const float log2_delta = delta > 0.0 ? (float)log2(delta) : -INFINITY;
+    return from_cuda(launch_accept_typical(logits, cand, parent, B, T, V, dtype, y_scale, log2_eps, log2_delta,
+                                           argmax_out, path_out, accept_len, bonus_token, workspace, status,
+                                           static_cast<cudaStream_t>(stream)));
 }
 
 clover_status clover_kv_commit(void *k_cache, void *v_cache, const void *k_new, const void *v_new,

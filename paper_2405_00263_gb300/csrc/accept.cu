@@ -14,6 +14,16 @@
 // with a 64-bit atomic max.  Per-row and per-sequence arrival counters find
 // the CTA that finishes a sequence's last chunk; it decodes the argmax of
 // every node and runs the walk in one warp, and resets the keys and counters.
+//
+// Typical acceptance (the tree sampling rule the paper evaluates with, Section
+// 4 setup, after Medusa) is a compile-time mode of the same kernel.  Each chunk
+// CTA keeps its loads in registers and, besides the packed maximum, sums over
+// its chunk s = sum 2^t and u = sum 2^t t with t = (x - max) log2(e) / tau,
+// the base-2 exponent relative to the chunk maximum.  The last CTA merges the
+// chunk sums of every row into the tempered softmax's normaliser and entropy
+// (H = ln 2 (log2 S - U / S) over the merged sums), decides every edge
+// p(cand) > min(eps, delta e^-H) in the log2 domain, and walks the longest
+// accepted path (ties: the smallest-index child at every step).
 #include "common.cuh"
 
 namespace clover {
@@ -69,44 +79,99 @@ __device__ __forceinline__ int unit_first(const uint4 &w, float v, float) {
     return 3;
 }
 
-// Vector body: 16-byte units [0, n_units) of the row from element `first`.
-// Each round a thread issues kUnits independent loads (units tid + k*kThreads),
-// takes the maximum over them, and only then looks for its first position.
+// Vector body: 16-byte units [0, n_units) of the row from element `first`,
+// n_units <= kThreads * kUnits (a chunk is one round).  A thread issues its
+// kUnits independent loads (units tid + k*kThreads) into w, takes the maximum
+// over them, and only then looks for its first position.
 template <typename T>
-__device__ __forceinline__ void scan_vector(const T *row, int64_t first, int64_t n_units, uint64_t &best) {
+__device__ __forceinline__ void scan_vector(const T *row, int64_t first, int64_t n_units, uint64_t &best,
+                                            uint4 (&w)[kUnits]) {
     constexpr int E = 16 / sizeof(T);
     const uint4 *p = reinterpret_cast<const uint4 *>(row + first);
-    for (int64_t base = 0; base < n_units; base += (int64_t)kThreads * kUnits) {
-        uint4 w[kUnits];
 #pragma unroll
-        for (int k = 0; k < kUnits; ++k) {
-            const int64_t u = base + threadIdx.x + (int64_t)k * kThreads;
-            w[k] = (u < n_units) ? __ldcs(p + u) : make_uint4(0, 0, 0, 0);
-        }
-        float um[kUnits];
-        float m = -INFINITY;
-#pragma unroll
-        for (int k = 0; k < kUnits; ++k) {
-            const int64_t u = base + threadIdx.x + (int64_t)k * kThreads;
-            um[k] = (u < n_units) ? unit_max(w[k], T()) : -INFINITY;
-            m = fmaxf(m, um[k]);
-        }
-        // units are visited in increasing element order, so the first unit
-        // reaching m holds this round's first maximum of the thread
-        int kf = -1;
-#pragma unroll
-        for (int k = kUnits - 1; k >= 0; --k)
-            if (um[k] == m && base + threadIdx.x + (int64_t)k * kThreads < n_units) kf = k;
-        if (kf >= 0) {
-            uint4 wf = w[0];
-#pragma unroll
-            for (int k = 1; k < kUnits; ++k)
-                if (k == kf) wf = w[k];
-            const int64_t u = base + threadIdx.x + (int64_t)kf * kThreads;
-            const int e = unit_first(wf, m, T());
-            best = umax64(best, make_key(m, (uint32_t)(first + u * E + e)));
-        }
+    for (int k = 0; k < kUnits; ++k) {
+        const int64_t u = threadIdx.x + (int64_t)k * kThreads;
+        w[k] = (u < n_units) ? __ldcs(p + u) : make_uint4(0, 0, 0, 0);
     }
+    float um[kUnits];
+    float m = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < kUnits; ++k) {
+        const int64_t u = threadIdx.x + (int64_t)k * kThreads;
+        um[k] = (u < n_units) ? unit_max(w[k], T()) : -INFINITY;
+        m = fmaxf(m, um[k]);
+    }
+    // units are visited in increasing element order, so the first unit
+    // reaching m holds the thread's first maximum
+    int kf = -1;
+#pragma unroll
+    for (int k = kUnits - 1; k >= 0; --k)
+        if (um[k] == m && threadIdx.x + (int64_t)k * kThreads < n_units) kf = k;
+    if (kf >= 0) {
+        uint4 wf = w[0];
+#pragma unroll
+        for (int k = 1; k < kUnits; ++k)
+            if (k == kf) wf = w[k];
+        const int64_t u = threadIdx.x + (int64_t)kf * kThreads;
+        const int e = unit_first(wf, m, T());
+        best = umax64(best, make_key(m, (uint32_t)(first + u * E + e)));
+    }
+}
+
+// Inverse of order_bits (the value of a packed key's high word).
+__device__ __forceinline__ float key_value(uint64_t key) {
+    const uint32_t ob = static_cast<uint32_t>(key >> 32);
+    return __uint_as_float((ob & 0x80000000u) ? (ob & 0x7FFFFFFFu) : ~ob);
+}
+
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float lg2_approx(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// Softmax sums of a chunk relative to its scaled maximum my: s += 2^t and
+// u += 2^t t with t = x * ys - my.  t is clamped at -256 (2^t is then 0 in
+// fp32), which also turns the -inf logits (p = 0) into zero terms.
+struct ExpSums {
+    float s = 0.f, u = 0.f;
+    __device__ __forceinline__ void add(float x, float ys, float my) {
+        const float t = fmaxf(fmaf(x, ys, -my), -256.f);
+        const float e = ex2_approx(t);
+        s += e;
+        u = fmaf(e, t, u);
+    }
+};
+
+__device__ __forceinline__ void unit_sums(const uint4 &w, __nv_bfloat16, float ys, float my, ExpSums &acc) {
+    const uint32_t x[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        acc.add(__uint_as_float(x[k] << 16), ys, my);
+        acc.add(__uint_as_float(x[k] & 0xFFFF0000u), ys, my);
+    }
+}
+__device__ __forceinline__ void unit_sums(const uint4 &w, float, float ys, float my, ExpSums &acc) {
+    acc.add(__uint_as_float(w.x), ys, my);
+    acc.add(__uint_as_float(w.y), ys, my);
+    acc.add(__uint_as_float(w.z), ys, my);
+    acc.add(__uint_as_float(w.w), ys, my);
+}
+
+// (m, s, u) of two disjoint parts -> the sums of their union, relative to the
+// larger maximum.  Parts with s = 0 (all -inf) contribute nothing.
+__device__ __forceinline__ float3 merge_sums(float3 a, float3 b) {
+    if (b.y == 0.f) return a;
+    if (a.y == 0.f) return b;
+    const float M = fmaxf(a.x, b.x);
+    const float da = a.x - M, db = b.x - M;
+    const float wa = ex2_approx(da), wb = ex2_approx(db);
+    return make_float3(M, wa * a.y + wb * b.y, wa * fmaf(a.y, da, a.z) + wb * fmaf(b.y, db, b.z));
 }
 
 __device__ __forceinline__ uint64_t block_max(uint64_t v, uint64_t *s_red) {
@@ -131,38 +196,93 @@ struct AcceptArgs {
     unsigned long long *row_key;   // [B*T] running packed maximum of each logit row
     unsigned *row_count;           // [B*T] chunks of the row finished
     unsigned *seq_count;           // [B] rows of the sequence finished
+    // typical acceptance only
+    float4 *chunk_sums;            // [B*T, n_chunks] (scaled chunk maximum, s, u)
+    float y_scale;                 // log2(e) / temperature
+    float log2_eps, log2_delta;    // log2 of the threshold parameters (-inf for 0)
     int32_t *status;
 };
 
-// Argmax of every node of sequence b from the merged row keys, then the greedy
-// walk, by one warp: lane l owns nodes l and l + 32.  The walk reads the argmax
-// of the current node from registers (warp shuffles), so each step costs no
-// memory round trip.  The row keys and the counter are reset for the next call.
-__device__ void accept_walk_warp(const AcceptArgs &a, int b) {
+// The CTA that finished sequence b's last chunk: argmax of every node from the
+// merged row keys, then the walk, by warp 0 (lane l owns nodes l and l + 32;
+// the walk reads the current node's argmax from registers by warp shuffles, so
+// a step costs no memory round trip).  The row keys and the counter are reset
+// for the next call.
+//
+// Greedy: from the root, the smallest-index child whose candidate equals the
+// current node's argmax, until there is none.
+// Typical: first every thread of the CTA merges a quarter of one row's chunk
+// sums (64 rows x 4 threads) into the row's (max, log2 S, log2 theta), warp 1
+// builds the ancestor masks, and warp 0 fetches each child's candidate logit
+// under its parent.  Then warp 0 decides every edge, marks the nodes whose
+// whole root path is accepted, takes the greatest depth among them and the
+// union G of the root paths of the accepted nodes at that depth, and walks
+// from the root through G, the smallest-index child at every step.
+template <typename T, bool TYPICAL>
+__device__ void finish_sequence(const AcceptArgs &a, int b) {
+    __shared__ float4 s_row[kMaxTreeNodes];
+    __shared__ uint64_t s_anc[kMaxTreeNodes];
+    __shared__ bool s_bad;
     const int lane = threadIdx.x & 31;
-    const int T = a.T;
-    const int32_t *par = a.parent + (size_t)b * T;
-    const int32_t *cd = a.cand + (size_t)b * T;
+    const int warp = threadIdx.x >> 5;
+    const int Tn = a.T;
+    __threadfence();
     int p[2], c[2], am[2];
+    float xc[2] = {-INFINITY, -INFINITY};
     bool invalid = false;
+    if (warp == 0) {
+        const int32_t *par = a.parent + (size_t)b * Tn;
+        const int32_t *cd = a.cand + (size_t)b * Tn;
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
-        const int i = lane + 32 * k;
-        p[k] = -2;
-        c[k] = 0;
-        am[k] = 0;
-        if (i < T) {
-            const unsigned long long key = __ldcg(a.row_key + (size_t)b * T + i);
-            am[k] = (int)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
-            a.argmax_out[(size_t)b * T + i] = am[k];
-            a.row_key[(size_t)b * T + i] = 0ull;                      // ready for the next call
-            p[k] = __ldg(par + i);
-            c[k] = __ldg(cd + i);
-            if (i == 0 ? (p[k] != -1) : (p[k] < 0 || p[k] >= i)) invalid = true;
+        for (int k = 0; k < 2; ++k) {
+            const int i = lane + 32 * k;
+            p[k] = -2;
+            c[k] = 0;
+            am[k] = 0;
+            if (i < Tn) {
+                const unsigned long long key = __ldcg(a.row_key + (size_t)b * Tn + i);
+                am[k] = (int)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+                a.argmax_out[(size_t)b * Tn + i] = am[k];
+                a.row_key[(size_t)b * Tn + i] = 0ull;                      // ready for the next call
+                p[k] = __ldg(par + i);
+                c[k] = __ldg(cd + i);
+                if (i == 0 ? (p[k] != -1) : (p[k] < 0 || p[k] >= i)) invalid = true;
+                // the candidate's logit under the parent (the root has no edge)
+                if (TYPICAL && i > 0 && p[k] >= 0 && p[k] < i && c[k] >= 0 && c[k] < a.V)
+                    xc[k] = to_float(static_cast<const T *>(a.logits)[((size_t)b * Tn + p[k]) * a.V + c[k]]);
+            }
         }
     }
-    int32_t *path = a.path_out + (size_t)b * T;
-    for (int i = lane; i < T; i += 32) path[i] = -1;
+    if (TYPICAL) {
+        const int row = threadIdx.x >> 2;
+        const int q = threadIdx.x & 3;
+        float3 st = make_float3(-INFINITY, 0.f, 0.f);
+        if (row < Tn) {
+            const float4 *cs = a.chunk_sums + ((size_t)b * Tn + row) * a.n_chunks;
+            for (int k = q; k < a.n_chunks; k += 4) {
+                const float4 v = __ldcg(cs + k);
+                st = merge_sums(st, make_float3(v.x, v.y, v.z));
+            }
+        }
+#pragma unroll
+        for (int off = 1; off < 4; off <<= 1) {
+            const float3 o = make_float3(__shfl_xor_sync(0xffffffffu, st.x, off), __shfl_xor_sync(0xffffffffu, st.y, off),
+                                         __shfl_xor_sync(0xffffffffu, st.z, off));
+            st = merge_sums(st, o);
+        }
+        if (q == 0 && row < Tn) {
+            // S >= 1 (the maximum's own term); entropy in bits H2 = log2 S - U / S
+            const float log2s = lg2_approx(st.y);
+            const float h2 = log2s - st.z / st.y;
+            s_row[row] = make_float4(st.x, log2s, fminf(a.log2_eps, a.log2_delta - h2), 0.f);
+        }
+        if (warp == 1) tree_masks_warp(a.parent + (size_t)b * Tn, Tn, s_anc, &s_bad);
+        __syncthreads();
+    }
+    if (warp != 0) return;
+
+    int32_t *path = a.path_out + (size_t)b * Tn;
+    for (int i = lane; i < Tn; i += 32) path[i] = -1;
     __syncwarp();
     int cur = 0, len = 1;
     if (lane == 0) path[0] = 0;
@@ -173,12 +293,51 @@ __device__ void accept_walk_warp(const AcceptArgs &a, int b) {
     };
     if (__any_sync(0xffffffffu, invalid)) {
         if (lane == 0) report(a.status, CLOVER_ERR_BAD_TREE);
-    } else {
+    } else if (!TYPICAL) {
         // at most T - 1 steps: every step moves to a larger node index
-        for (int step = 1; step < T; ++step) {
+        for (int step = 1; step < Tn; ++step) {
             const int want = argmax_of(cur);
             const unsigned lo = __ballot_sync(0xffffffffu, p[0] == cur && c[0] == want);
             const unsigned hi = __ballot_sync(0xffffffffu, p[1] == cur && c[1] == want);
+            const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
+            if (hits == 0ull) break;
+            cur = __ffsll(static_cast<long long>(hits)) - 1;
+            if (lane == 0) path[len] = cur;
+            ++len;
+        }
+    } else {
+        uint64_t anc[2];
+        bool ok[2];
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int i = lane + 32 * k;
+            anc[k] = i < Tn ? s_anc[i] : 0ull;
+            ok[k] = false;
+            if (i >= 1 && i < Tn) {
+                const float4 r = s_row[p[k]];
+                ok[k] = fmaf(xc[k], a.y_scale, -r.x) - r.y > r.z;   // log2 p > log2 theta
+            }
+        }
+        const uint64_t acc = (static_cast<uint64_t>(__ballot_sync(0xffffffffu, ok[1])) << 32) |
+                             __ballot_sync(0xffffffffu, ok[0]) | 1ull;
+        int depth[2];
+        unsigned dmax = 0;
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const bool reach = lane + 32 * k < Tn && (anc[k] & ~acc) == 0ull;
+            depth[k] = reach ? __popcll(anc[k]) - 1 : -1;
+            dmax = max(dmax, (unsigned)max(depth[k], 0));
+        }
+        dmax = __reduce_max_sync(0xffffffffu, dmax);
+        uint64_t g = 0ull;
+#pragma unroll
+        for (int k = 0; k < 2; ++k)
+            if (depth[k] == (int)dmax) g |= anc[k];
+        g = (static_cast<uint64_t>(__reduce_or_sync(0xffffffffu, (unsigned)(g >> 32))) << 32) |
+            __reduce_or_sync(0xffffffffu, (unsigned)g);
+        for (unsigned step = 0; step < dmax; ++step) {
+            const unsigned lo = __ballot_sync(0xffffffffu, p[0] == cur && ((g >> lane) & 1ull));
+            const unsigned hi = __ballot_sync(0xffffffffu, p[1] == cur && ((g >> (lane + 32)) & 1ull));
             const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
             if (hits == 0ull) break;
             cur = __ffsll(static_cast<long long>(hits)) - 1;
@@ -194,9 +353,11 @@ __device__ void accept_walk_warp(const AcceptArgs &a, int b) {
     }
 }
 
-template <typename T>
+template <typename T, bool TYPICAL>
 __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
     __shared__ uint64_t s_red[kThreads / 32];
+    __shared__ float2 s_sum[kThreads / 32];
+    __shared__ float s_my;
     __shared__ int s_seq_last;
     const int row = blockIdx.x;               // b * T + i
     const int chunk_id = blockIdx.y;
@@ -205,20 +366,53 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
 
     const int64_t lo = (int64_t)chunk_id * a.chunk;
     const int64_t hi = min((int64_t)a.V, lo + a.chunk);
+    constexpr int E = 16 / sizeof(T);
     uint64_t best = 0ull;
+    uint4 w[kUnits];
+    int64_t head = 0, n_units = 0;
     if (lo < hi) {
         // scalar head up to a 16-byte boundary, vector body, scalar tail
-        constexpr int E = 16 / sizeof(T);
         const uintptr_t addr = reinterpret_cast<uintptr_t>(rowp + lo);
-        int64_t head = (int64_t)(((16 - (addr & 15)) & 15) / sizeof(T));
+        head = (int64_t)(((16 - (addr & 15)) & 15) / sizeof(T));
         if ((addr % sizeof(T)) != 0) head = hi - lo;       // cannot happen for valid tensors
         head = min(head, hi - lo);
-        const int64_t n_units = (hi - lo - head) / E;
+        n_units = (hi - lo - head) / E;
         scan_scalar<T>(rowp, lo, lo + head, best);
-        scan_vector<T>(rowp, lo + head, n_units, best);
+        scan_vector<T>(rowp, lo + head, n_units, best, w);
         scan_scalar<T>(rowp, lo + head + n_units * E, hi, best);
     }
     best = block_max(best, s_red);
+
+    if (TYPICAL) {
+        // the chunk's softmax sums relative to its scaled maximum, from the
+        // registers of the scan (head and tail elements are read again)
+        if (threadIdx.x == 0) s_my = key_value(best) * a.y_scale;
+        __syncthreads();
+        const float my = s_my;
+        ExpSums acc;
+#pragma unroll
+        for (int k = 0; k < kUnits; ++k)
+            if (threadIdx.x + (int64_t)k * kThreads < n_units) unit_sums(w[k], T(), a.y_scale, my, acc);
+        for (int64_t v = lo + threadIdx.x; v < lo + head; v += kThreads) acc.add(to_float(rowp[v]), a.y_scale, my);
+        for (int64_t v = lo + head + n_units * E + threadIdx.x; v < hi; v += kThreads)
+            acc.add(to_float(rowp[v]), a.y_scale, my);
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            acc.s += __shfl_xor_sync(0xffffffffu, acc.s, off);
+            acc.u += __shfl_xor_sync(0xffffffffu, acc.u, off);
+        }
+        if ((threadIdx.x & 31) == 0) s_sum[threadIdx.x >> 5] = make_float2(acc.s, acc.u);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float2 t = s_sum[0];
+#pragma unroll
+            for (int k = 1; k < kThreads / 32; ++k) {
+                t.x += s_sum[k].x;
+                t.y += s_sum[k].y;
+            }
+            __stcg(a.chunk_sums + (size_t)row * a.n_chunks + chunk_id, make_float4(my, t.x, t.y, 0.f));
+        }
+    }
 
     // fold this chunk into the row's key and count it; the CTA finishing a
     // row's last chunk counts the row for its sequence, and the one finishing
@@ -237,10 +431,7 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
     }
     __syncthreads();
     if (!s_seq_last) return;
-    if (threadIdx.x < 32) {
-        __threadfence();
-        accept_walk_warp(a, b);
-    }
+    finish_sequence<T, TYPICAL>(a, b);
 }
 
 }  // namespace
@@ -256,16 +447,28 @@ void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk) {
     *n_chunks = (V + c - 1) / c;
 }
 
+// Keys and counters, then (typical acceptance) the 16-byte aligned chunk sums.
+static size_t accept_sums_offset(int B, int T) {
+    const size_t base = sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * ((size_t)B * T + B);
+    return (base + 15) & ~(size_t)15;
+}
+
 size_t accept_workspace_bytes(int B, int T, int V, int dtype) {
     (void)V;
     (void)dtype;
     return sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * ((size_t)B * T + B);
 }
 
-cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
-                          int V, int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len,
-                          int32_t *bonus, void *workspace, int32_t *status, cudaStream_t stream) {
-    AcceptArgs a;
+size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype) {
+    int n_chunks, chunk;
+    accept_plan(B, T, V, dtype, &n_chunks, &chunk);
+    return accept_sums_offset(B, T) + sizeof(float4) * (size_t)B * T * n_chunks;
+}
+
+static AcceptArgs accept_args(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T, int V,
+                              int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len,
+                              int32_t *bonus, void *workspace, int32_t *status) {
+    AcceptArgs a{};
     a.logits = logits;
     a.cand = cand;
     a.parent = parent;
@@ -281,9 +484,33 @@ cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t
     a.row_count = reinterpret_cast<unsigned *>(a.row_key + (size_t)B * T);
     a.seq_count = a.row_count + (size_t)B * T;
     a.status = status;
+    return a;
+}
+
+cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
+                          int V, int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len,
+                          int32_t *bonus, void *workspace, int32_t *status, cudaStream_t stream) {
+    const AcceptArgs a = accept_args(logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len, bonus,
+                                     workspace, status);
     dim3 grid(B * T, a.n_chunks);
-    if (dtype == CLOVER_F32) accept_kernel<float><<<grid, kThreads, 0, stream>>>(a);
-    else accept_kernel<__nv_bfloat16><<<grid, kThreads, 0, stream>>>(a);
+    if (dtype == CLOVER_F32) accept_kernel<float, false><<<grid, kThreads, 0, stream>>>(a);
+    else accept_kernel<__nv_bfloat16, false><<<grid, kThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_accept_typical(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
+                                  int V, int dtype, float y_scale, float log2_eps, float log2_delta,
+                                  int32_t *argmax_out, int32_t *path_out, int32_t *accept_len, int32_t *bonus,
+                                  void *workspace, int32_t *status, cudaStream_t stream) {
+    AcceptArgs a = accept_args(logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len, bonus,
+                               workspace, status);
+    a.chunk_sums = reinterpret_cast<float4 *>(static_cast<uint8_t *>(workspace) + accept_sums_offset(B, T));
+    a.y_scale = y_scale;
+    a.log2_eps = log2_eps;
+    a.log2_delta = log2_delta;
+    dim3 grid(B * T, a.n_chunks);
+    if (dtype == CLOVER_F32) accept_kernel<float, true><<<grid, kThreads, 0, stream>>>(a);
+    else accept_kernel<__nv_bfloat16, true><<<grid, kThreads, 0, stream>>>(a);
     return cudaGetLastError();
 }
 

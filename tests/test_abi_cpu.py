@@ -3,6 +3,7 @@ header declares, and its host-side validation rejects bad arguments before
 anything is launched."""
 
 import ctypes
+import math
 import os
 import re
 
@@ -116,6 +117,27 @@ def test_attn_ex_and_commit_host_validation(lib):
     assert com(1024, 2048, D=32) == 2
     assert com(1024, 2048, T=65) == 2
     assert com(1024, 2048, B=0) == 0
+
+
+def test_accept_typical_workspace_and_host_validation(lib):
+    P = ctypes.c_void_p
+    # keys + counters (2*4*8 + (2*4 + 2)*4 = 104 bytes, padded to 112), then one
+    # 16-byte (max, s, u) record per row and 16384-element chunk (8 for V = 125696 bf16)
+    need = lib.clover_verify_accept_typical_workspace_size(2, 4, 125696, 1)
+    assert lib.clover_verify_accept_workspace_size(2, 4, 125696, 1) == 104
+    assert need == 112 + 16 * 2 * 4 * 8
+    assert lib.clover_verify_accept_typical_workspace_size(2, 4, 125696, 0) == 112 + 16 * 2 * 4 * 16
+    assert lib.clover_verify_accept_typical_workspace_size(2, 65, 100, 1) == 0
+    call = lambda tau=1.0, eps=0.09, delta=0.3, ws=4096, wsb=need, B=2, T=4, V=125696: \
+        lib.clover_verify_accept_typical(P(64), P(64), P(64), B, T, V, 1, tau, eps, delta, P(64), P(64), P(64),
+                                         P(64), P(ws), wsb, None, None)
+    for bad in (dict(tau=0.0), dict(tau=-1.0), dict(tau=math.nan), dict(tau=math.inf), dict(eps=-0.1),
+                dict(eps=math.nan), dict(delta=-1.0), dict(delta=math.inf), dict(ws=4104), dict(wsb=need - 1),
+                dict(ws=0)):
+        assert call(**bad) == 1, bad
+    assert call(tau=1e-300) == 2 and call(tau=1e39) == 2     # log2(e)/tau not a normal fp32 number
+    assert call(T=65) == 2
+    assert call(B=0) == 0
 
 
 def test_python_binding_rejects_cpu_tensors(lib):
