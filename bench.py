@@ -255,7 +255,9 @@ def run_gpu_arm(args, world, rank, local, dist):
     del base, sets
     base, sets = make_sets(w, device, n_sets)
     Lcap = base["Lcap"]
-    step = pkg.VerifyStep(w.B, w.T, w.Hq, w.Hkv, w.D, Lcap, w.V, w.torch_dtype, device=device)
+    step = pkg.VerifyStep(w.B, w.T, w.Hq, w.Hkv, w.D, Lcap, w.V, w.torch_dtype, device=device,
+                          accept=args.accept, temperature=args.temperature, epsilon=args.epsilon,
+                          delta=args.delta)
     stream = torch.cuda.Stream(device)
 
     ext_ok = True
@@ -324,26 +326,39 @@ def run_gpu_arm(args, world, rank, local, dist):
 
     # per-kernel durations.  The attention: the in-graph events of the last
     # replay of every event-carrying graph inside the timed region.  The accept
-    # and commit calls (on the side stream): eager steps after the timed region.
-    durations = {"tree_attn": [], "accept": [], "kv_commit": []}
+    # and commit calls: each launched alone after an L2 flush by a large read
+    # (which keeps the GPU busy while the call is queued, so the events bracket
+    # the kernel and not the host's launch latency), after the timed region.
+    durations = {"tree_attn": []}
     timing_source = {"tree_attn": "events inside the replayed graphs of the timed region",
-                     "accept": "eager steps with events after the timed region",
-                     "kv_commit": "eager steps with events after the timed region"}
+                     "accept": "launched alone after an L2 flush, events on the launching stream",
+                     "kv_commit": "launched alone after an L2 flush, events on the launching stream"}
     timed_graphs = [evs for i, evs in enumerate(graph_events) if evs and i < args.steps]
     for evs in timed_graphs:
         durations["tree_attn"].append(evs[0].elapsed_time(evs[1]) * 1e3)
-    for i in range(3 * len(sets)):
-        evs = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
-        with torch.cuda.stream(stream):
-            launch(sets[i % n_sets], evs)
-        torch.cuda.synchronize(device)
-        if not timed_graphs:
-            durations["tree_attn"].append(evs[0].elapsed_time(evs[1]) * 1e3)
-        durations["accept"].append(evs[4].elapsed_time(evs[5]) * 1e3)
-        durations["kv_commit"].append(evs[2].elapsed_time(evs[3]) * 1e3)
     if not timed_graphs:
+        for i in range(3 * len(sets)):
+            evs = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+            with torch.cuda.stream(stream):
+                launch(sets[i % n_sets], evs)
+            torch.cuda.synchronize(device)
+            durations["tree_attn"].append(evs[0].elapsed_time(evs[1]) * 1e3)
         timing_source["tree_attn"] = "eager steps with events after the timed region (no external graph events)"
     us = {k: statistics.mean(v) for k, v in durations.items()}
+    flush = torch.zeros(2 * L2_BYTES, dtype=torch.uint8, device=device)
+    us["accept"] = accept_kernel_us(pkg, w, sets, stream, device, args.accept, args, flush)
+    other = "greedy" if args.accept == "typical" else "typical"
+    us_other = accept_kernel_us(pkg, w, sets, stream, device, other, args, flush)
+    us["kv_commit"] = isolated_us(
+        lambda i: pkg.clover_kv_commit(sets[i % n_sets]["k_cache"], sets[i % n_sets]["v_cache"],
+                                       sets[i % n_sets]["k_new"], sets[i % n_sets]["v_new"],
+                                       sets[i % n_sets]["cache_len"], step.path, step.accept_len,
+                                       step.new_cache_len, step.src_index, status=step.status_accept,
+                                       stream=stream),
+        3 * len(sets), stream, flush)
+    del flush
+    if step.device_status() != 0:
+        raise RuntimeError(f"device status {step.device_status()} in the per-kernel timing")
 
     peaks, peak_kind = measured_peaks()
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
@@ -365,7 +380,8 @@ def run_gpu_arm(args, world, rank, local, dist):
                    "l2": f"{n_sets} rotating input sets of {per_set / 1e6:.1f} MB "
                          f"({n_sets * per_set / 1e6:.0f} MB > 3x the 129 MB L2)",
                    "launch": "one CUDA graph replay per step: the attention (cache read only) on one stream, "
-                             "argmax/accept then the commit of the accepted K/V on a second stream"},
+                             "argmax/accept then the commit of the accepted K/V on a second stream",
+                   "accept": accept_desc(args)},
         "roofline": {"bound": "hbm", "kernel": "tree_attn", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm, "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)"
                      if peak_kind == "measured" else "fallback 6.8 TB/s",
@@ -374,14 +390,69 @@ def run_gpu_arm(args, world, rank, local, dist):
                      "flops_per_launch": attn_flops_per_launch(w, lengths),
                      "timing": timing_source["tree_attn"]},
         "kernels": {"tree_attn_us": us["tree_attn"], "accept_us": us["accept"], "kv_commit_us": us["kv_commit"],
+                    "accept_rule": args.accept,
                     "accept_bytes_per_launch": am_bytes,
-                    "accept_gbs": am_bytes / (us["accept"] * 1e-6) / 1e9},
+                    "accept_gbs": am_bytes / (us["accept"] * 1e-6) / 1e9,
+                    "accept_frac": am_bytes / (us["accept"] * 1e-6) / 1e9 / hbm,
+                    f"accept_{other}": {"us": us_other, "gbs": am_bytes / (us_other * 1e-6) / 1e9,
+                                        "frac": am_bytes / (us_other * 1e-6) / 1e9 / hbm,
+                                        "timing": timing_source["accept"]}},
         "gpu_launches": 3 * args.steps,
         "timing": timing_source,
         "clocks": clocks,
         "e2e": e2e,
     }
     return line, w, base
+
+
+def accept_desc(args) -> str:
+    if args.accept == "typical":
+        return (f"typical acceptance (temperature {args.temperature}, epsilon {args.epsilon}, "
+                f"delta {args.delta})")
+    return "greedy"
+
+
+def isolated_us(call, n, stream, flush) -> float:
+    """Mean event-timed duration of call(i), i < n, each launched alone on
+    ``stream`` right after a read of ``flush`` (twice the L2: the L2 then holds
+    only clean lines of it, so the call pays no write-back of a flush)."""
+    times = []
+    with torch.cuda.stream(stream):
+        for i in range(n + 2):
+            torch.amax(flush)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            call(i)
+            b.record(stream)
+            b.synchronize()
+            if i >= 2:
+                times.append(a.elapsed_time(b) * 1e3)
+    return statistics.mean(times)
+
+
+def accept_kernel_us(pkg, w, sets, stream, device, rule, args, flush) -> float:
+    """Mean duration of one acceptance call of ``rule`` (own outputs and
+    workspace) over the rotating input sets."""
+    i32 = dict(dtype=torch.int32, device=device)
+    outs = [torch.empty((w.B, w.T), **i32), torch.empty((w.B, w.T), **i32), torch.empty(w.B, **i32),
+            torch.empty(w.B, **i32)]
+    size = (pkg.clover_verify_accept_typical_workspace_size if rule == "typical"
+            else pkg.clover_verify_accept_workspace_size)(w.B, w.T, w.V, w.torch_dtype)
+    ws = torch.zeros(size, dtype=torch.uint8, device=device)
+    status = torch.zeros(1, **i32)
+
+    def call(i):
+        s = sets[i % len(sets)]
+        if rule == "typical":
+            pkg.clover_verify_accept_typical(s["logits"], s["cand"], s["parent"], args.temperature, args.epsilon,
+                                             args.delta, *outs, ws, status=status, stream=stream)
+        else:
+            pkg.clover_verify_accept(s["logits"], s["cand"], s["parent"], *outs, ws, status=status, stream=stream)
+
+    t = isolated_us(call, 3 * len(sets), stream, flush)
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())} in the {rule} acceptance timing")
+    return t
 
 
 def run_e2e(args, w, step, sets, stream, device, dist, world):
@@ -434,26 +505,31 @@ def run_e2e(args, w, step, sets, stream, device, dist, world):
 # the oracle on the host cores
 # ---------------------------------------------------------------------------
 
-def oracle_step_seconds(host: dict, threads: int) -> float:
+def typical_params(args):
+    return (args.temperature, args.epsilon, args.delta) if args.accept == "typical" else None
+
+
+def oracle_step_seconds(host: dict, threads: int, typical=None) -> float:
     import oracle
     t0 = time.perf_counter()
-    oracle.verify_step(host, n_threads=threads)
+    oracle.verify_step(host, n_threads=threads, typical=typical)
     return time.perf_counter() - t0
 
 
-def cpu_baseline(w, host: dict, budget_s: float = 8.0) -> dict:
+def cpu_baseline(w, host: dict, args, budget_s: float = 8.0) -> dict:
     """Whole oracle verify steps (fp64 attention over every row, argmax over
     every logit row, walk, append, compaction) repeated within a time budget."""
     import oracle
     oracle.build()
     threads = os.cpu_count() or 1
-    times = [oracle_step_seconds(host, threads)]
+    typ = typical_params(args)
+    times = [oracle_step_seconds(host, threads, typ)]
     while sum(times) < budget_s and len(times) < 50:
-        times.append(oracle_step_seconds(host, threads))
+        times.append(oracle_step_seconds(host, threads, typ))
     per = statistics.median(times)
     return {"value": 1.0 / per, "unit": UNIT, "cores": threads, "kind": "oracle",
             "sample": f"{len(times)} whole verify steps of {w.name} (fp64 oracle, OpenMP over attention rows "
-                      f"and logit rows), median {per * 1e3:.1f} ms per step"}
+                      f"and logit rows, {accept_desc(args)}), median {per * 1e3:.1f} ms per step"}
 
 
 def run_reference_arm(args, world, rank):
@@ -465,16 +541,18 @@ def run_reference_arm(args, world, rank):
     import oracle
     oracle.build()
     threads = os.cpu_count() or 1
+    typ = typical_params(args)
     for _ in range(args.warmup):
-        oracle_step_seconds(host, threads)
-    t = [oracle_step_seconds(host, threads) for _ in range(args.steps)]
+        oracle_step_seconds(host, threads, typ)
+    t = [oracle_step_seconds(host, threads, typ) for _ in range(args.steps)]
     total = sum(t)
     value = args.steps / total
     return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f64", "data": "synthetic",
-            "config": {"workload": f"{w.name}: {w.description}", "parallelism": "host cores (rank 0 only)"},
+            "config": {"workload": f"{w.name}: {w.description}", "parallelism": "host cores (rank 0 only)",
+                       "accept": accept_desc(args)},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
                              "sample": f"{args.steps} whole verify steps of {w.name} on the host (fp64 oracle)"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -489,6 +567,11 @@ def main(argv=None):
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],
+                    help="acceptance rule of the step (typical: tempered softmax with an entropy threshold)")
+    ap.add_argument("--temperature", type=float, default=1.0)
+    ap.add_argument("--epsilon", type=float, default=0.09)
+    ap.add_argument("--delta", type=float, default=0.3)
     args = ap.parse_args(argv)
     if args.warmup < 3:
         args.warmup = 3
@@ -505,7 +588,7 @@ def main(argv=None):
     if rank == 0:
         if world == 1 and not args.no_cpu_baseline:
             host = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
-            line["cpu_baseline"] = cpu_baseline(w, host)
+            line["cpu_baseline"] = cpu_baseline(w, host, args)
         else:
             line["cpu_baseline"] = None
         print(json.dumps(line), flush=True)

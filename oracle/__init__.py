@@ -231,16 +231,22 @@ def kv_commit(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len):
     return src
 
 
-def verify_step(inp: dict, scale: float = 0.0, n_threads: int | None = None) -> dict:
-    """The whole step on copies of the inputs: attention, append, argmax, walk, compact."""
+def verify_step(inp: dict, scale: float = 0.0, n_threads: int | None = None, typical=None) -> dict:
+    """The whole step on copies of the inputs: attention, append, argmax, walk
+    (greedy, or typical acceptance with ``typical`` = (temperature, epsilon,
+    delta)), compact."""
     k_cache = inp["k_cache"].clone()
     v_cache = inp["v_cache"].clone()
     cache_len = inp["cache_len"].clone().to(torch.int32)
     out = tree_attention(inp["q"], inp["k_new"], inp["v_new"], k_cache, v_cache, cache_len,
                          inp["parent"], scale=scale, n_threads=n_threads)
     append_tree_kv(inp["k_new"], inp["v_new"], k_cache, v_cache, cache_len)
-    amax = argmax(inp["logits"], n_threads=n_threads)
-    path, alen, bonus = accept_walk(inp["parent"], inp["cand"], amax)
+    if typical is None:
+        amax = argmax(inp["logits"], n_threads=n_threads)
+        path, alen, bonus = accept_walk(inp["parent"], inp["cand"], amax)
+    else:
+        r = accept_typical(inp["logits"], inp["parent"], inp["cand"], *typical, n_threads=n_threads)
+        amax, path, alen, bonus = r["argmax"], r["path"], r["accept_len"], r["bonus"]
     src = kv_compact(k_cache, v_cache, cache_len, path, alen)
     return {"out": out, "argmax": amax, "path": path, "accept_len": alen, "bonus": bonus,
             "src_index": src, "k_cache": k_cache, "v_cache": v_cache, "cache_len": cache_len}

@@ -258,17 +258,25 @@ class VerifyStep:
     are done.
     With ``concurrent=False`` the calls run in order on ``stream``.
     ``src_index`` holds tree nodes (commit) or cache slots (compact).
+    ``accept``: ``"greedy"`` (clover_verify_accept) or ``"typical"``
+    (clover_verify_accept_typical with ``temperature``, ``epsilon``, ``delta``).
     """
 
-    def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda", concurrent=True, schedule="commit"):
+    def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda", concurrent=True, schedule="commit",
+                 accept="greedy", temperature=1.0, epsilon=0.09, delta=0.3):
         if schedule not in ("commit", "compact"):
             raise ValueError(f"unknown schedule {schedule!r}")
+        if accept not in ("greedy", "typical"):
+            raise ValueError(f"unknown acceptance rule {accept!r}")
         self.shape = dict(B=B, T=T, Hq=Hq, Hkv=Hkv, D=D, Lcap=Lcap, V=V)
         self.dtype = dtype
         self.schedule = schedule
+        self.accept = accept
+        self.typical = (float(temperature), float(epsilon), float(delta))
         dev = torch.device(device)
         ws_a = clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, Lcap, dtype)
-        ws_b = clover_verify_accept_workspace_size(B, T, V, dtype)
+        ws_b = (clover_verify_accept_typical_workspace_size if accept == "typical"
+                else clover_verify_accept_workspace_size)(B, T, V, dtype)
         self.ws_attn = torch.zeros(max(ws_a, 16), dtype=torch.uint8, device=dev) if ws_a else None
         self.ws_accept = torch.zeros(max(ws_b, 16), dtype=torch.uint8, device=dev)
         self.out = torch.empty((B, T, Hq, D), dtype=dtype, device=dev)
@@ -317,8 +325,13 @@ class VerifyStep:
                            workspace=self.ws_attn, status=self.status, stream=stream, append=not commit)
         ev(1, stream)
         ev(4, side)
-        clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
-                             self.ws_accept, status=self.status_accept, stream=side)
+        if self.accept == "typical":
+            clover_verify_accept_typical(logits, cand, parent, *self.typical, self.argmax, self.path,
+                                         self.accept_len, self.bonus, self.ws_accept, status=self.status_accept,
+                                         stream=side)
+        else:
+            clover_verify_accept(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
+                                 self.ws_accept, status=self.status_accept, stream=side)
         ev(5, side)
         if commit:
             ev(2, side)

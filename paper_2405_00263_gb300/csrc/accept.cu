@@ -7,23 +7,26 @@
 // token equals its parent's greedy token; the accepted path is walked from the
 // root and its length is the paper's tokens/step (Section 4.1).
 //
-// Grid: one CTA per (logit row, vocabulary chunk).  Each CTA reduces its chunk
-// with 16-byte loads to a packed 64-bit key (order-preserving value bits in the
-// high word, bit-inverted index in the low word) so that one unsigned max
-// gives "largest value, then smallest index", and folds it into the row's key
-// with a 64-bit atomic max.  Per-row and per-sequence arrival counters find
-// the CTA that finishes a sequence's last chunk; it decodes the argmax of
-// every node and runs the walk in one warp, and resets the keys and counters.
+// Grid: one CTA per (logit row, 32 KB vocabulary chunk).  Each CTA reduces its
+// chunk with 16-byte loads (eight in flight per thread) to a packed 64-bit key
+// (order-preserving value bits in the high word, bit-inverted index in the low
+// word) so that one unsigned max gives "largest value, then smallest index",
+// and folds it into the row's key with a 64-bit atomic max.  A per-sequence
+// arrival counter finds the CTA that finishes a sequence's last chunk; it
+// decodes the argmax of every node and runs the walk in one warp, and resets
+// the keys and the counter.
 //
 // Typical acceptance (the tree sampling rule the paper evaluates with, Section
 // 4 setup, after Medusa) is a compile-time mode of the same kernel.  Each chunk
 // CTA keeps its loads in registers and, besides the packed maximum, sums over
-// its chunk s = sum 2^t and u = sum 2^t t with t = (x - max) log2(e) / tau,
-// the base-2 exponent relative to the chunk maximum.  The last CTA merges the
-// chunk sums of every row into the tempered softmax's normaliser and entropy
-// (H = ln 2 (log2 S - U / S) over the merged sums), decides every edge
-// p(cand) > min(eps, delta e^-H) in the log2 domain, and walks the longest
-// accepted path (ties: the smallest-index child at every step).
+// its chunk s = sum 2^t and u = sum 2^t t with t = (x - m) log2(e) / tau, the
+// base-2 exponent relative to a maximum m (each thread's own, then merged
+// across the CTA), and gathers the logits of the candidates that fall in its
+// chunk.  The last CTA merges the chunk sums of every row into the tempered
+// softmax's normaliser and entropy (H = ln 2 (log2 S - U / S) over the merged
+// sums), decides every edge p(cand) > min(eps, delta e^-H) in the log2
+// domain, and walks the longest accepted path (ties: the smallest-index child
+// at every step).
 #include "common.cuh"
 
 namespace clover {
@@ -118,12 +121,6 @@ __device__ __forceinline__ void scan_vector(const T *row, int64_t first, int64_t
     }
 }
 
-// Inverse of order_bits (the value of a packed key's high word).
-__device__ __forceinline__ float key_value(uint64_t key) {
-    const uint32_t ob = static_cast<uint32_t>(key >> 32);
-    return __uint_as_float((ob & 0x80000000u) ? (ob & 0x7FFFFFFFu) : ~ob);
-}
-
 __device__ __forceinline__ float ex2_approx(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -194,62 +191,108 @@ struct AcceptArgs {
     int B, T, V, n_chunks, chunk;
     int32_t *argmax_out, *path_out, *accept_len, *bonus;
     unsigned long long *row_key;   // [B*T] running packed maximum of each logit row
-    unsigned *row_count;           // [B*T] chunks of the row finished
-    unsigned *seq_count;           // [B] rows of the sequence finished
+    unsigned *seq_count;           // [B] chunks of the sequence finished
     // typical acceptance only
-    float4 *chunk_sums;            // [B*T, n_chunks] (scaled chunk maximum, s, u)
+    float4 *chunk_sums;            // [B*T, n_chunks] (scaled maximum, s, u) of every chunk
+    float *cand_x;                 // [B*T] logit of each node's candidate under its parent
     float y_scale;                 // log2(e) / temperature
     float log2_eps, log2_delta;    // log2 of the threshold parameters (-inf for 0)
     int32_t *status;
 };
 
+// Ancestor-or-self bitmasks of a valid tree by pointer jumping in one warp's
+// registers: lane l owns nodes l and l + 32 with parents parent[0..1].  After
+// round k each mask covers the node's 2^k nearest ancestors; six rounds cover
+// depth 63.
+__device__ __forceinline__ void tree_masks_regs(const int (&parent)[2], int T, uint64_t (&m)[2]) {
+    const int lane = threadIdx.x & 31;
+    int up[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int i = lane + 32 * k;
+        m[k] = (i < T) ? (1ull << i) : 0ull;
+        up[k] = (i < T && i > 0) ? parent[k] : -1;
+    }
+#pragma unroll
+    for (int round = 0; round < 6; ++round) {
+        uint64_t nm[2];
+        int nu[2];
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int u = up[k] < 0 ? 0 : up[k];
+            const uint64_t m0 = __shfl_sync(0xffffffffu, m[0], u & 31);
+            const uint64_t m1 = __shfl_sync(0xffffffffu, m[1], u & 31);
+            const int u0 = __shfl_sync(0xffffffffu, up[0], u & 31);
+            const int u1 = __shfl_sync(0xffffffffu, up[1], u & 31);
+            nm[k] = up[k] < 0 ? m[k] : (m[k] | ((u >> 5) ? m1 : m0));
+            nu[k] = up[k] < 0 ? -1 : ((u >> 5) ? u1 : u0);
+        }
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            m[k] = nm[k];
+            up[k] = nu[k];
+        }
+    }
+}
+
+// Sequence b's tree in warp 0's registers: lane l holds nodes l and l + 32.
+struct TreeRegs {
+    int p[2], c[2];
+    bool invalid;
+};
+
+__device__ __forceinline__ TreeRegs load_tree(const AcceptArgs &a, int b) {
+    const int lane = threadIdx.x & 31;
+    const int32_t *par = a.parent + (size_t)b * a.T;
+    const int32_t *cd = a.cand + (size_t)b * a.T;
+    TreeRegs t;
+    t.invalid = false;
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int i = lane + 32 * k;
+        t.p[k] = -2;
+        t.c[k] = 0;
+        if (i < a.T) {
+            t.p[k] = __ldg(par + i);
+            t.c[k] = __ldg(cd + i);
+            if (i == 0 ? (t.p[k] != -1) : (t.p[k] < 0 || t.p[k] >= i)) t.invalid = true;
+        }
+    }
+    return t;
+}
+
 // The CTA that finished sequence b's last chunk: argmax of every node from the
-// merged row keys, then the walk, by warp 0 (lane l owns nodes l and l + 32;
-// the walk reads the current node's argmax from registers by warp shuffles, so
-// a step costs no memory round trip).  The row keys and the counter are reset
-// for the next call.
+// merged row keys, then the walk, by warp 0 (the walk reads the current
+// node's argmax from registers by warp shuffles, so a step costs no memory
+// round trip).  The row keys and the counter are reset for the next call.
 //
 // Greedy: from the root, the smallest-index child whose candidate equals the
 // current node's argmax, until there is none.
 // Typical: first every thread of the CTA merges a quarter of one row's chunk
-// sums (64 rows x 4 threads) into the row's (max, log2 S, log2 theta), warp 1
-// builds the ancestor masks, and warp 0 fetches each child's candidate logit
-// under its parent.  Then warp 0 decides every edge, marks the nodes whose
-// whole root path is accepted, takes the greatest depth among them and the
-// union G of the root paths of the accepted nodes at that depth, and walks
-// from the root through G, the smallest-index child at every step.
+// sums (64 rows x 4 threads) into the row's (max, log2 S, log2 theta), while
+// warp 0 also reads each child's candidate logit (gathered by the chunk CTAs)
+// and builds the ancestor masks in registers.  Then warp 0 decides every edge, marks the
+// nodes whose whole root path is accepted, takes the greatest depth among
+// them and the union G of the root paths of the accepted nodes at that depth,
+// and walks from the root through G, the smallest-index child at every step.
 template <typename T, bool TYPICAL>
-__device__ void finish_sequence(const AcceptArgs &a, int b) {
+__device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) {
     __shared__ float4 s_row[kMaxTreeNodes];
-    __shared__ uint64_t s_anc[kMaxTreeNodes];
-    __shared__ bool s_bad;
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int Tn = a.T;
-    __threadfence();
-    int p[2], c[2], am[2];
+    int am[2] = {0, 0};
     float xc[2] = {-INFINITY, -INFINITY};
-    bool invalid = false;
     if (warp == 0) {
-        const int32_t *par = a.parent + (size_t)b * Tn;
-        const int32_t *cd = a.cand + (size_t)b * Tn;
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
             const int i = lane + 32 * k;
-            p[k] = -2;
-            c[k] = 0;
-            am[k] = 0;
             if (i < Tn) {
                 const unsigned long long key = __ldcg(a.row_key + (size_t)b * Tn + i);
+                if (TYPICAL && i > 0 && tr.c[k] >= 0 && tr.c[k] < a.V) xc[k] = __ldcg(a.cand_x + (size_t)b * Tn + i);
                 am[k] = (int)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
                 a.argmax_out[(size_t)b * Tn + i] = am[k];
                 a.row_key[(size_t)b * Tn + i] = 0ull;                      // ready for the next call
-                p[k] = __ldg(par + i);
-                c[k] = __ldg(cd + i);
-                if (i == 0 ? (p[k] != -1) : (p[k] < 0 || p[k] >= i)) invalid = true;
-                // the candidate's logit under the parent (the root has no edge)
-                if (TYPICAL && i > 0 && p[k] >= 0 && p[k] < i && c[k] >= 0 && c[k] < a.V)
-                    xc[k] = to_float(static_cast<const T *>(a.logits)[((size_t)b * Tn + p[k]) * a.V + c[k]]);
             }
         }
     }
@@ -276,7 +319,6 @@ __device__ void finish_sequence(const AcceptArgs &a, int b) {
             const float h2 = log2s - st.z / st.y;
             s_row[row] = make_float4(st.x, log2s, fminf(a.log2_eps, a.log2_delta - h2), 0.f);
         }
-        if (warp == 1) tree_masks_warp(a.parent + (size_t)b * Tn, Tn, s_anc, &s_bad);
         __syncthreads();
     }
     if (warp != 0) return;
@@ -291,14 +333,14 @@ __device__ void finish_sequence(const AcceptArgs &a, int b) {
         const int hi = __shfl_sync(0xffffffffu, am[1], node & 31);
         return (node >> 5) ? hi : lo;
     };
-    if (__any_sync(0xffffffffu, invalid)) {
+    if (__any_sync(0xffffffffu, tr.invalid)) {
         if (lane == 0) report(a.status, CLOVER_ERR_BAD_TREE);
     } else if (!TYPICAL) {
         // at most T - 1 steps: every step moves to a larger node index
         for (int step = 1; step < Tn; ++step) {
             const int want = argmax_of(cur);
-            const unsigned lo = __ballot_sync(0xffffffffu, p[0] == cur && c[0] == want);
-            const unsigned hi = __ballot_sync(0xffffffffu, p[1] == cur && c[1] == want);
+            const unsigned lo = __ballot_sync(0xffffffffu, tr.p[0] == cur && tr.c[0] == want);
+            const unsigned hi = __ballot_sync(0xffffffffu, tr.p[1] == cur && tr.c[1] == want);
             const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
             if (hits == 0ull) break;
             cur = __ffsll(static_cast<long long>(hits)) - 1;
@@ -307,14 +349,14 @@ __device__ void finish_sequence(const AcceptArgs &a, int b) {
         }
     } else {
         uint64_t anc[2];
+        tree_masks_regs(tr.p, Tn, anc);
         bool ok[2];
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
             const int i = lane + 32 * k;
-            anc[k] = i < Tn ? s_anc[i] : 0ull;
             ok[k] = false;
             if (i >= 1 && i < Tn) {
-                const float4 r = s_row[p[k]];
+                const float4 r = s_row[tr.p[k]];
                 ok[k] = fmaf(xc[k], a.y_scale, -r.x) - r.y > r.z;   // log2 p > log2 theta
             }
         }
@@ -336,8 +378,8 @@ __device__ void finish_sequence(const AcceptArgs &a, int b) {
         g = (static_cast<uint64_t>(__reduce_or_sync(0xffffffffu, (unsigned)(g >> 32))) << 32) |
             __reduce_or_sync(0xffffffffu, (unsigned)g);
         for (unsigned step = 0; step < dmax; ++step) {
-            const unsigned lo = __ballot_sync(0xffffffffu, p[0] == cur && ((g >> lane) & 1ull));
-            const unsigned hi = __ballot_sync(0xffffffffu, p[1] == cur && ((g >> (lane + 32)) & 1ull));
+            const unsigned lo = __ballot_sync(0xffffffffu, tr.p[0] == cur && ((g >> lane) & 1ull));
+            const unsigned hi = __ballot_sync(0xffffffffu, tr.p[1] == cur && ((g >> (lane + 32)) & 1ull));
             const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
             if (hits == 0ull) break;
             cur = __ffsll(static_cast<long long>(hits)) - 1;
@@ -356,13 +398,19 @@ __device__ void finish_sequence(const AcceptArgs &a, int b) {
 template <typename T, bool TYPICAL>
 __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
     __shared__ uint64_t s_red[kThreads / 32];
-    __shared__ float2 s_sum[kThreads / 32];
-    __shared__ float s_my;
+    __shared__ float4 s_sum[kThreads / 32];
     __shared__ int s_seq_last;
-    const int row = blockIdx.x;               // b * T + i
+    const int warp = threadIdx.x >> 5;
+    const int row = blockIdx.x;            // b * T + i
     const int chunk_id = blockIdx.y;
     const int b = row / a.T;
+    const int node = row - b * a.T;
     const T *rowp = static_cast<const T *>(a.logits) + (size_t)row * a.V;
+
+    // the tree, for the walk if this CTA turns out to finish the sequence
+    // (and the candidate gather below); its loads overlap the scan
+    TreeRegs tr;
+    if (warp == 0) tr = load_tree(a, b);
 
     const int64_t lo = (int64_t)chunk_id * a.chunk;
     const int64_t hi = min((int64_t)a.V, lo + a.chunk);
@@ -381,57 +429,66 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
         scan_vector<T>(rowp, lo + head, n_units, best, w);
         scan_scalar<T>(rowp, lo + head + n_units * E, hi, best);
     }
-    best = block_max(best, s_red);
 
     if (TYPICAL) {
-        // the chunk's softmax sums relative to its scaled maximum, from the
-        // registers of the scan (head and tail elements are read again)
-        if (threadIdx.x == 0) s_my = key_value(best) * a.y_scale;
-        __syncthreads();
-        const float my = s_my;
+        // the thread's softmax sums relative to its own scaled maximum, from
+        // the registers of the scan (head and tail elements are read again),
+        // merged across the CTA with the chunk's key
+        const int64_t t0 = lo + head + n_units * E;
+        float mt = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kUnits; ++k)
+            if (threadIdx.x + (int64_t)k * kThreads < n_units) mt = fmaxf(mt, unit_max(w[k], T()));
+        for (int64_t v = lo + threadIdx.x; v < lo + head; v += kThreads) mt = fmaxf(mt, to_float(rowp[v]));
+        for (int64_t v = t0 + threadIdx.x; v < hi; v += kThreads) mt = fmaxf(mt, to_float(rowp[v]));
+        const float my = mt * a.y_scale;
         ExpSums acc;
 #pragma unroll
         for (int k = 0; k < kUnits; ++k)
             if (threadIdx.x + (int64_t)k * kThreads < n_units) unit_sums(w[k], T(), a.y_scale, my, acc);
         for (int64_t v = lo + threadIdx.x; v < lo + head; v += kThreads) acc.add(to_float(rowp[v]), a.y_scale, my);
-        for (int64_t v = lo + head + n_units * E + threadIdx.x; v < hi; v += kThreads)
-            acc.add(to_float(rowp[v]), a.y_scale, my);
+        for (int64_t v = t0 + threadIdx.x; v < hi; v += kThreads) acc.add(to_float(rowp[v]), a.y_scale, my);
+        float3 st = make_float3(my, acc.s, acc.u);
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) {
-            acc.s += __shfl_xor_sync(0xffffffffu, acc.s, off);
-            acc.u += __shfl_xor_sync(0xffffffffu, acc.u, off);
+            const float3 o = make_float3(__shfl_xor_sync(0xffffffffu, st.x, off), __shfl_xor_sync(0xffffffffu, st.y, off),
+                                         __shfl_xor_sync(0xffffffffu, st.z, off));
+            st = merge_sums(st, o);
         }
-        if ((threadIdx.x & 31) == 0) s_sum[threadIdx.x >> 5] = make_float2(acc.s, acc.u);
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            float2 t = s_sum[0];
+        if ((threadIdx.x & 31) == 0) s_sum[warp] = make_float4(st.x, st.y, st.z, 0.f);
+        // candidates of this node's children that fall in this chunk: their
+        // logits for the walk
+        if (warp == 0) {
 #pragma unroll
-            for (int k = 1; k < kThreads / 32; ++k) {
-                t.x += s_sum[k].x;
-                t.y += s_sum[k].y;
+            for (int k = 0; k < 2; ++k) {
+                const int i = threadIdx.x + 32 * k;
+                if (i >= 1 && i < a.T && tr.p[k] == node && tr.c[k] >= lo && tr.c[k] < hi) {
+                    a.cand_x[(size_t)b * a.T + i] = to_float(rowp[tr.c[k]]);
+                    __threadfence();
+                }
             }
-            __stcg(a.chunk_sums + (size_t)row * a.n_chunks + chunk_id, make_float4(my, t.x, t.y, 0.f));
         }
     }
+    best = block_max(best, s_red);            // its barrier also publishes s_sum
+    if (TYPICAL && threadIdx.x == 0) {
+        float3 st = make_float3(s_sum[0].x, s_sum[0].y, s_sum[0].z);
+#pragma unroll
+        for (int k = 1; k < kThreads / 32; ++k) st = merge_sums(st, make_float3(s_sum[k].x, s_sum[k].y, s_sum[k].z));
+        __stcg(a.chunk_sums + (size_t)row * a.n_chunks + chunk_id, make_float4(st.x, st.y, st.z, 0.f));
+    }
 
-    // fold this chunk into the row's key and count it; the CTA finishing a
-    // row's last chunk counts the row for its sequence, and the one finishing
-    // the sequence's last row runs the walk (two levels keep each counter to a
-    // few arrivals)
+    // fold this chunk into the row's key and count it for its sequence; the
+    // CTA that counts the sequence's last chunk runs the walk
     if (threadIdx.x == 0) {
         atomicMax(a.row_key + row, static_cast<unsigned long long>(best));
-        __threadfence();
-        bool last = false;
-        if (atomicAdd(a.row_count + row, 1u) == (unsigned)a.n_chunks - 1u) {
-            a.row_count[row] = 0u;                              // ready for the next call
-            __threadfence();
-            last = (atomicAdd(a.seq_count + b, 1u) == (unsigned)a.T - 1u);
-        }
-        s_seq_last = last;
+        __threadfence();                      // release: the key, sums and candidate logits
+        const bool last = atomicAdd(a.seq_count + b, 1u) == (unsigned)(a.T * a.n_chunks) - 1u;
+        if (last) __threadfence();            // acquire: every other CTA's; the barrier below
+        s_seq_last = last;                    // passes it on, and they are read through L2
     }
     __syncthreads();
     if (!s_seq_last) return;
-    finish_sequence<T, TYPICAL>(a, b);
+    finish_sequence<T, TYPICAL>(a, b, tr);
 }
 
 }  // namespace
@@ -447,22 +504,23 @@ void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk) {
     *n_chunks = (V + c - 1) / c;
 }
 
-// Keys and counters, then (typical acceptance) the 16-byte aligned chunk sums.
+// Keys and counters, then (typical acceptance) the 16-byte aligned chunk sums
+// and the candidates' logits.
 static size_t accept_sums_offset(int B, int T) {
-    const size_t base = sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * ((size_t)B * T + B);
+    const size_t base = sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * (size_t)B;
     return (base + 15) & ~(size_t)15;
 }
 
 size_t accept_workspace_bytes(int B, int T, int V, int dtype) {
     (void)V;
     (void)dtype;
-    return sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * ((size_t)B * T + B);
+    return sizeof(unsigned long long) * (size_t)B * T + sizeof(unsigned) * (size_t)B;
 }
 
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype) {
     int n_chunks, chunk;
     accept_plan(B, T, V, dtype, &n_chunks, &chunk);
-    return accept_sums_offset(B, T) + sizeof(float4) * (size_t)B * T * n_chunks;
+    return accept_sums_offset(B, T) + sizeof(float4) * (size_t)B * T * n_chunks + sizeof(float) * (size_t)B * T;
 }
 
 static AcceptArgs accept_args(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T, int V,
@@ -481,8 +539,7 @@ static AcceptArgs accept_args(const void *logits, const int32_t *cand, const int
     a.accept_len = accept_len;
     a.bonus = bonus;
     a.row_key = static_cast<unsigned long long *>(workspace);
-    a.row_count = reinterpret_cast<unsigned *>(a.row_key + (size_t)B * T);
-    a.seq_count = a.row_count + (size_t)B * T;
+    a.seq_count = reinterpret_cast<unsigned *>(a.row_key + (size_t)B * T);
     a.status = status;
     return a;
 }
@@ -505,6 +562,7 @@ cudaError_t launch_accept_typical(const void *logits, const int32_t *cand, const
     AcceptArgs a = accept_args(logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len, bonus,
                                workspace, status);
     a.chunk_sums = reinterpret_cast<float4 *>(static_cast<uint8_t *>(workspace) + accept_sums_offset(B, T));
+    a.cand_x = reinterpret_cast<float *>(a.chunk_sums + (size_t)B * T * a.n_chunks);
     a.y_scale = y_scale;
     a.log2_eps = log2_eps;
     a.log2_delta = log2_delta;

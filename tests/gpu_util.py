@@ -30,7 +30,7 @@ def run_gpu(t: dict, scale: float = 0.0, step: pkg.VerifyStep | None = None, **s
 
 def compare_full(host: dict, step: pkg.VerifyStep, t: dict, scale: float = 0.0):
     """Every output against oracle.verify_step (small shapes)."""
-    ref = oracle.verify_step(host, scale=scale)
+    ref = oracle.verify_step(host, scale=scale, typical=step.typical if step.accept == "typical" else None)
     dt = host["q"].dtype
     assert step.device_status() == 0
     err = (step.out.double().cpu() - ref["out"]).abs().max().item()

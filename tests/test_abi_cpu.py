@@ -54,7 +54,7 @@ def test_workspace_sizes(lib):
     assert ws(1, 16, 8, 8, 96, 192, 0) == 0              # D = 96 unsupported
     assert ws(1, 16, 6, 4, 64, 192, 0) == 0              # Hq not a multiple of Hkv
     acc = lib.clover_verify_accept_workspace_size
-    assert acc(1, 64, 125696, 1) == 8 * 64 + 4 * (64 + 1)   # a 64-bit key and a counter per row, a counter per sequence
+    assert acc(1, 64, 125696, 1) == 8 * 64 + 4               # a 64-bit key per row, a counter per sequence
     assert acc(1, 0, 10, 1) == 0 and acc(1, 4, 0, 1) == 0
 
 
@@ -121,12 +121,13 @@ def test_attn_ex_and_commit_host_validation(lib):
 
 def test_accept_typical_workspace_and_host_validation(lib):
     P = ctypes.c_void_p
-    # keys + counters (2*4*8 + (2*4 + 2)*4 = 104 bytes, padded to 112), then one
-    # 16-byte (max, s, u) record per row and 16384-element chunk (8 for V = 125696 bf16)
+    # keys + counters (2*4*8 + 2*4 = 72 bytes, padded to 80), one 16-byte
+    # (max, s, u) record per row and 16384-element chunk (8 for V = 125696
+    # bf16), one fp32 candidate logit per node
     need = lib.clover_verify_accept_typical_workspace_size(2, 4, 125696, 1)
-    assert lib.clover_verify_accept_workspace_size(2, 4, 125696, 1) == 104
-    assert need == 112 + 16 * 2 * 4 * 8
-    assert lib.clover_verify_accept_typical_workspace_size(2, 4, 125696, 0) == 112 + 16 * 2 * 4 * 16
+    assert lib.clover_verify_accept_workspace_size(2, 4, 125696, 1) == 72
+    assert need == 80 + 16 * 2 * 4 * 8 + 4 * 2 * 4
+    assert lib.clover_verify_accept_typical_workspace_size(2, 4, 125696, 0) == 80 + 16 * 2 * 4 * 16 + 4 * 2 * 4
     assert lib.clover_verify_accept_typical_workspace_size(2, 65, 100, 1) == 0
     call = lambda tau=1.0, eps=0.09, delta=0.3, ws=4096, wsb=need, B=2, T=4, V=125696: \
         lib.clover_verify_accept_typical(P(64), P(64), P(64), B, T, V, 1, tau, eps, delta, P(64), P(64), P(64),

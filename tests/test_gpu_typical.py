@@ -185,3 +185,21 @@ def test_typical_bad_tree_sets_status():
     got = run_typical(logits, parent, cand, 1.0, 0.09, 0.3)
     assert got["status"] & 4                   # CLOVER_ERR_BAD_TREE
     assert int(got["accept_len"][1]) == 1 and int(got["path"][1, 0]) == 0
+
+
+@pytest.mark.parametrize("schedule", ["commit", "compact"])
+@pytest.mark.parametrize("name,over,params", [
+    ("tiny_f32", {}, (1.0, 0.09, 0.3)),
+    ("7b_l2048", dict(B=2, T=64, Hq=8, Hkv=2, L=700, V=5003), (0.8, 0.09, 0.3)),
+    ("paper_t4_b4", dict(Hq=8, Hkv=8, L_range=(100, 900), V=32000), (1.0, 0.3, 0.55)),
+])
+def test_typical_verify_step_matches_oracle(name, over, params, schedule):
+    """The whole step (attention, typical acceptance, commit or compaction)
+    through VerifyStep against the oracle's step with the same rule."""
+    from tests.gpu_util import compare_full, run_gpu, to_dev
+    host = workloads.make(workloads.get(name, **over))
+    host["cand"], _ = clear_margins(host["logits"], host["parent"], host["cand"], *params)
+    t = to_dev(host, torch.device("cuda"))
+    tau, eps, delta = params
+    step = run_gpu(t, schedule=schedule, accept="typical", temperature=tau, epsilon=eps, delta=delta)
+    compare_full(host, step, t)
