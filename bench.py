@@ -257,7 +257,7 @@ def run_gpu_arm(args, world, rank, local, dist):
     Lcap = base["Lcap"]
     step = pkg.VerifyStep(w.B, w.T, w.Hq, w.Hkv, w.D, Lcap, w.V, w.torch_dtype, device=device,
                           accept=args.accept, temperature=args.temperature, epsilon=args.epsilon,
-                          delta=args.delta)
+                          delta=args.delta, schedule=args.schedule)
     stream = torch.cuda.Stream(device)
 
     ext_ok = True
@@ -379,8 +379,7 @@ def run_gpu_arm(args, world, rank, local, dist):
                    "V": w.V, "Lcap": Lcap, "parallelism": f"replicas x{world} (one per GPU)",
                    "l2": f"{n_sets} rotating input sets of {per_set / 1e6:.1f} MB "
                          f"({n_sets * per_set / 1e6:.0f} MB > 3x the 129 MB L2)",
-                   "launch": "one CUDA graph replay per step: the attention (cache read only) on one stream, "
-                             "argmax/accept then the commit of the accepted K/V on a second stream",
+                   "launch": LAUNCH_DESC[args.schedule],
                    "accept": accept_desc(args)},
         "roofline": {"bound": "hbm", "kernel": "tree_attn", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm, "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)"
@@ -397,12 +396,23 @@ def run_gpu_arm(args, world, rank, local, dist):
                     f"accept_{other}": {"us": us_other, "gbs": am_bytes / (us_other * 1e-6) / 1e9,
                                         "frac": am_bytes / (us_other * 1e-6) / 1e9 / hbm,
                                         "timing": timing_source["accept"]}},
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": (2 if args.schedule == "fused" else 3) * args.steps,
         "timing": timing_source,
         "clocks": clocks,
         "e2e": e2e,
     }
     return line, w, base
+
+
+LAUNCH_DESC = {
+    "commit": "one CUDA graph replay per step: the attention (cache read only) on one stream, argmax/accept "
+              "then the commit of the accepted K/V on a second stream",
+    "compact": "one CUDA graph replay per step: the attention (appending the tree K/V) on one stream and "
+               "argmax/accept on a second, then the compaction of the accepted K/V",
+    "fused": "one CUDA graph replay per step, two launches on one stream: the attention (cache read only), then "
+             "argmax/accept with the commit of the accepted K/V fused in, launched as a programmatic dependent "
+             "of the attention so that it runs beside it",
+}
 
 
 def accept_desc(args) -> str:
@@ -569,6 +579,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],
                     help="acceptance rule of the step (typical: tempered softmax with an entropy threshold)")
+    ap.add_argument("--schedule", default="commit", choices=["commit", "compact", "fused"],
+                    help="call schedule of the step (VerifyStep)")
     ap.add_argument("--temperature", type=float, default=1.0)
     ap.add_argument("--epsilon", type=float, default=0.09)
     ap.add_argument("--delta", type=float, default=0.3)

@@ -15,6 +15,9 @@
  *   clover_verify_accept_typical
  *                         the same with the sampling-side (typical) acceptance
  *                         rule of the paper's tree sampling algorithm (Section 4);
+ *   clover_verify_accept_ex
+ *                         either rule, optionally fused with the commit of the
+ *                         accepted K/V and launched to overlap the attention;
  *   clover_kv_compact     moves the accepted nodes' K/V to the front of the
  *                         tree slots (an engine step the paper leaves implicit).
  *
@@ -213,6 +216,52 @@ CLOVER_API clover_status clover_verify_accept_typical(const void *logits, const 
                                    int32_t *argmax_out, int32_t *path_out,
                                    int32_t *accept_len, int32_t *bonus_token,
                                    void *workspace, size_t ws_bytes,
+                                   int32_t *status, void *stream);
+
+/* Flags of clover_verify_accept_ex. */
+#define CLOVER_ACCEPT_TYPICAL 1u   /* typical rule (temperature, epsilon, delta) instead of greedy */
+#define CLOVER_ACCEPT_COMMIT 2u    /* also commit the accepted K/V, as clover_kv_commit would */
+#define CLOVER_ACCEPT_OVERLAP 4u   /* may start while the kernel queued before it still runs */
+
+/* Bytes of device workspace clover_verify_accept_ex needs with these flags. */
+CLOVER_API size_t clover_verify_accept_ex_workspace_size(int B, int T, int V, clover_dtype dtype, uint32_t flags);
+
+/*
+ * The acceptance step with options, in one launch:
+ *   - the greedy rule (clover_verify_accept) or, with CLOVER_ACCEPT_TYPICAL,
+ *     the typical rule (clover_verify_accept_typical; temperature, epsilon
+ *     and delta are read only then);
+ *   - with CLOVER_ACCEPT_COMMIT, the commit of the accepted path from the
+ *     tree's K/V, with the effect of clover_kv_commit on the path and length
+ *     this call produces: for every sequence b with L = cache_len[b] and a =
+ *     accept_len[b], slot L+j of every KV head receives k_new/v_new of node
+ *     path[j] (j < a), src_index_out[b][j] = path[j] (-1 past a; may be NULL),
+ *     new_cache_len[b] = L + a.  k_cache, v_cache [B,Hkv,Lcap,D], k_new, v_new
+ *     [B,T,Hkv,D] (16-byte aligned), cache_len, new_cache_len [B] (not
+ *     overlapping), D in {64, 128}, Lcap >= T.  cache_len[b] < 0 or
+ *     cache_len[b] + T > Lcap -> CLOVER_ERR_CAPACITY (device bit; that sequence
+ *     is not committed).  Without the flag these arguments are not read.
+ *   - with CLOVER_ACCEPT_OVERLAP, the launch is a programmatic dependent of
+ *     the kernel queued just before it on `stream`: it may start once that
+ *     kernel's CTAs have all started (this library's attention kernels allow
+ *     that at their start) and run beside it.  The caller guarantees that the
+ *     two touch disjoint memory apart from reads of the same inputs and the
+ *     status word, as clover_verify_attn_ex with CLOVER_ATTN_NO_APPEND does
+ *     with a commit into slots >= cache_len.  This call still completes only
+ *     after that kernel has, so stream order is kept for everything queued
+ *     later.  Where the overlap is unavailable the launch simply runs after it.
+ * Other flag bits: CLOVER_ERR_INVALID_ARG.  Workspace: as for the chosen rule
+ * (clover_verify_accept_ex_workspace_size).
+ */
+CLOVER_API clover_status clover_verify_accept_ex(const void *logits, const int32_t *cand, const int32_t *parent,
+                                   int B, int T, int V, clover_dtype dtype,
+                                   double temperature, double epsilon, double delta,
+                                   void *k_cache, void *v_cache, const void *k_new, const void *v_new,
+                                   const int32_t *cache_len, int Hkv, int D, int Lcap,
+                                   int32_t *argmax_out, int32_t *path_out,
+                                   int32_t *accept_len, int32_t *bonus_token,
+                                   int32_t *new_cache_len, int32_t *src_index_out,
+                                   void *workspace, size_t ws_bytes, uint32_t flags,
                                    int32_t *status, void *stream);
 
 /*

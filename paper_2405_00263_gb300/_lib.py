@@ -27,6 +27,8 @@ EXPORTS = (
     "clover_verify_accept",
     "clover_verify_accept_typical_workspace_size",
     "clover_verify_accept_typical",
+    "clover_verify_accept_ex_workspace_size",
+    "clover_verify_accept_ex",
     "clover_kv_compact",
     "clover_kv_commit",
     "clover_verify_attn_noalloc",
@@ -34,6 +36,11 @@ EXPORTS = (
 
 # Flag of clover_verify_attn_ex (CLOVER_ATTN_NO_APPEND in include/clover_verify.h).
 ATTN_NO_APPEND = 1
+
+# Flags of clover_verify_accept_ex (CLOVER_ACCEPT_* in include/clover_verify.h).
+ACCEPT_TYPICAL = 1
+ACCEPT_COMMIT = 2
+ACCEPT_OVERLAP = 4
 
 # Bytes of the static scratch buffer behind clover_verify_attn_noalloc
 # (CLOVER_NOALLOC_SCRATCH_BYTES in include/clover_verify.h).
@@ -79,6 +86,12 @@ def load(build_if_missing: bool = False):
         lib.clover_verify_accept_typical.argtypes = [P, P, P, I, I, I, I, ctypes.c_double, ctypes.c_double,
                                                      ctypes.c_double, P, P, P, P, P, Z, P, P]
         lib.clover_verify_accept_typical.restype = I
+        lib.clover_verify_accept_ex_workspace_size.argtypes = [I, I, I, I, ctypes.c_uint32]
+        lib.clover_verify_accept_ex_workspace_size.restype = Z
+        Dd = ctypes.c_double
+        lib.clover_verify_accept_ex.argtypes = [P, P, P, I, I, I, I, Dd, Dd, Dd, P, P, P, P, P, I, I, I,
+                                                P, P, P, P, P, P, P, Z, ctypes.c_uint32, P, P]
+        lib.clover_verify_accept_ex.restype = I
         lib.clover_kv_compact.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P, P]
         lib.clover_kv_compact.restype = I
         lib.clover_kv_commit.argtypes = [P, P, P, P, P, P, P, P, P, I, I, I, I, I, I, P, P]

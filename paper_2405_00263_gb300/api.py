@@ -242,6 +242,59 @@ def clover_kv_commit(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len
         raise CloverError(code, "clover_kv_commit")
 
 
+def clover_verify_accept_ex_workspace_size(B, T, V, dtype, flags=0) -> int:
+    code = dtype if isinstance(dtype, int) else dtype_code(dtype)
+    return int(_lib.load().clover_verify_accept_ex_workspace_size(B, T, V, code, flags))
+
+
+def clover_verify_accept_ex(logits, cand, parent, argmax_out, path_out, accept_len, bonus_token, workspace,
+                            typical=None, commit=None, overlap=False, status=None, stream=None):
+    """One launch: the greedy rule, or the typical rule with ``typical`` =
+    (temperature, epsilon, delta); with ``commit`` = (k_cache, v_cache, k_new,
+    v_new, cache_len, new_cache_len, src_index_out or None) also the commit of
+    the accepted K/V; with ``overlap`` as a programmatic dependent of the
+    kernel queued before it (see CLOVER_ACCEPT_OVERLAP)."""
+    B, T, V = logits.shape
+    _check(cand, (B, T), torch.int32, "cand")
+    _check(parent, (B, T), torch.int32, "parent")
+    _check(argmax_out, (B, T), torch.int32, "argmax_out")
+    _check(path_out, (B, T), torch.int32, "path_out")
+    _check(accept_len, (B,), torch.int32, "accept_len")
+    _check(bonus_token, (B,), torch.int32, "bonus_token")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    flags = 0
+    tau = eps = delta = 0.0
+    if typical is not None:
+        flags |= _lib.ACCEPT_TYPICAL
+        tau, eps, delta = (float(x) for x in typical)
+    kc = vc = kn = vn = cl = ncl = src = None
+    Hkv = D = Lcap = 0
+    if commit is not None:
+        flags |= _lib.ACCEPT_COMMIT
+        kc, vc, kn, vn, cl, ncl, src = commit
+        _, Hkv, Lcap, D = kc.shape
+        _check(kc, (B, Hkv, Lcap, D), logits.dtype, "k_cache")
+        _check(vc, (B, Hkv, Lcap, D), logits.dtype, "v_cache")
+        _check(kn, (B, T, Hkv, D), logits.dtype, "k_new")
+        _check(vn, (B, T, Hkv, D), logits.dtype, "v_new")
+        _check(cl, (B,), torch.int32, "cache_len")
+        _check(ncl, (B,), torch.int32, "new_cache_len")
+        if src is not None:
+            _check(src, (B, T), torch.int32, "src_index_out")
+    if overlap:
+        flags |= _lib.ACCEPT_OVERLAP
+    _dev(logits, cand, parent, argmax_out, path_out, accept_len, bonus_token, workspace, status, kc, vc, kn, vn,
+         cl, ncl, src)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    code = _lib.load().clover_verify_accept_ex(
+        _ptr(logits), _ptr(cand), _ptr(parent), B, T, V, dtype_code(logits.dtype), tau, eps, delta, _ptr(kc),
+        _ptr(vc), _ptr(kn), _ptr(vn), _ptr(cl), Hkv, D, Lcap, _ptr(argmax_out), _ptr(path_out), _ptr(accept_len),
+        _ptr(bonus_token), _ptr(ncl), _ptr(src), _ptr(workspace), ws_bytes, flags, _ptr(status), _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_verify_accept_ex")
+
+
 class VerifyStep:
     """Device buffers for repeated verification steps of one shape.
 
@@ -256,6 +309,10 @@ class VerifyStep:
     ``"compact"``: the attention appends the tree K/V while the accept call
     runs on the side stream; clover_kv_compact follows on ``stream`` once both
     are done.
+    ``"fused"``: two launches on ``stream``: the attention (caches only read),
+    then clover_verify_accept_ex with the commit fused in, launched as a
+    programmatic dependent of the attention so that it runs beside it on the
+    SM space the attention leaves (and completes after it).
     With ``concurrent=False`` the calls run in order on ``stream``.
     ``src_index`` holds tree nodes (commit) or cache slots (compact).
     ``accept``: ``"greedy"`` (clover_verify_accept) or ``"typical"``
@@ -264,7 +321,7 @@ class VerifyStep:
 
     def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda", concurrent=True, schedule="commit",
                  accept="greedy", temperature=1.0, epsilon=0.09, delta=0.3):
-        if schedule not in ("commit", "compact"):
+        if schedule not in ("commit", "compact", "fused"):
             raise ValueError(f"unknown schedule {schedule!r}")
         if accept not in ("greedy", "typical"):
             raise ValueError(f"unknown acceptance rule {accept!r}")
@@ -316,6 +373,29 @@ class VerifyStep:
         def ev(i, st):
             if i < n_ev:
                 events[i].record(st)
+
+        if self.schedule == "fused":
+            ev(0, stream)
+            clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
+                               workspace=self.ws_attn, status=self.status, stream=stream, append=False)
+            timed_end = n_ev > 1 and self.side is not None
+            if timed_end:
+                # the attention's end, recorded on the side stream: nothing is
+                # queued on `stream` between the attention and the accept call
+                self._fork.record(stream)
+                self.side.wait_event(self._fork)
+                events[1].record(self.side)
+                self._join.record(self.side)
+            elif n_ev > 1:
+                events[1].record(stream)
+            clover_verify_accept_ex(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
+                                    self.ws_accept, typical=self.typical if self.accept == "typical" else None,
+                                    commit=(k_cache, v_cache, k_new, v_new, cache_len, self.new_cache_len,
+                                            self.src_index),
+                                    overlap=self.side is not None, status=self.status_accept, stream=stream)
+            if timed_end:
+                stream.wait_event(self._join)
+            return
 
         if self.side is not None:
             self._fork.record(stream)

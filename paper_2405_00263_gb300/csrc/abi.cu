@@ -14,14 +14,8 @@ cudaError_t launch_tree_attn_fma(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream);
 void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk);
 size_t accept_workspace_bytes(int B, int T, int V, int dtype);
-cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T, int V,
-                          int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len, int32_t *bonus,
-                          void *workspace, int32_t *status, cudaStream_t stream);
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype);
-cudaError_t launch_accept_typical(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
-                                  int V, int dtype, float y_scale, float log2_eps, float log2_delta,
-                                  int32_t *argmax_out, int32_t *path_out, int32_t *accept_len, int32_t *bonus,
-                                  void *workspace, int32_t *status, cudaStream_t stream);
+cudaError_t launch_accept_call(const AcceptCall &c, cudaStream_t stream);
 cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
                               const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
                               int32_t *new_cache_len, int32_t *src_index, int B, int T, int Hkv, int D, int Lcap,
@@ -131,6 +125,54 @@ clover_status check_commit(void *k_cache, void *v_cache, const void *k_new, cons
     return CLOVER_OK;
 }
 
+// Host checks shared by the acceptance entry points; fills c (nothing is
+// launched when the result is not CLOVER_OK).
+clover_status check_accept(AcceptCall &c, const void *logits, const int32_t *cand, const int32_t *parent, int B,
+                           int T, int V, clover_dtype dtype, int32_t *argmax_out, int32_t *path_out,
+                           int32_t *accept_len, int32_t *bonus_token, void *workspace, size_t ws_bytes,
+                           int32_t *status, bool typical, double temperature, double epsilon, double delta) {
+    if (B < 0 || T < 1 || V < 1) return CLOVER_ERR_INVALID_ARG;
+    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
+    c = AcceptCall{};
+    if (typical) {
+        if (!(temperature > 0.0) || !isfinite(temperature) || !(epsilon >= 0.0) || !isfinite(epsilon) ||
+            !(delta >= 0.0) || !isfinite(delta))
+            return CLOVER_ERR_INVALID_ARG;
+        // exponents are kept in base 2: y = x log2(e) / temperature, in fp32
+        c.y_scale = (float)(1.4426950408889634 / temperature);
+        if (!isfinite(c.y_scale) || !(c.y_scale >= 1.17549435e-38f)) return CLOVER_ERR_UNSUPPORTED;
+        c.log2_eps = epsilon > 0.0 ? (float)log2(epsilon) : -INFINITY;
+        c.log2_delta = delta > 0.0 ? (float)log2(delta) : -INFINITY;
+    }
+    if (T > kMaxTreeNodes) return CLOVER_ERR_UNSUPPORTED;
+    if ((long)B * T > 0x7FFFFFFFL) return CLOVER_ERR_UNSUPPORTED;
+    if (B > 0) {
+        if (!logits || !cand || !parent || !argmax_out || !path_out || !accept_len || !bonus_token)
+            return CLOVER_ERR_INVALID_ARG;
+        const size_t need = typical ? accept_typical_workspace_bytes(B, T, V, dtype)
+                                    : accept_workspace_bytes(B, T, V, dtype);
+        if (ws_bytes < need || !workspace || !(typical ? aligned16(workspace)
+                                                       : (reinterpret_cast<uintptr_t>(workspace) & 7u) == 0))
+            return CLOVER_ERR_INVALID_ARG;
+        if (reinterpret_cast<uintptr_t>(logits) % (dtype == CLOVER_F32 ? 4 : 2)) return CLOVER_ERR_INVALID_ARG;
+    }
+    c.logits = logits;
+    c.cand = cand;
+    c.parent = parent;
+    c.B = B;
+    c.T = T;
+    c.V = V;
+    c.dtype = dtype;
+    c.argmax_out = argmax_out;
+    c.path_out = path_out;
+    c.accept_len = accept_len;
+    c.bonus = bonus_token;
+    c.workspace = workspace;
+    c.status = status;
+    c.typical = typical;
+    return CLOVER_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -227,18 +269,11 @@ clover_status clover_verify_accept(const void *logits, const int32_t *cand, cons
                                    int V, clover_dtype dtype, int32_t *argmax_out, int32_t *path_out,
                                    int32_t *accept_len, int32_t *bonus_token, void *workspace, size_t ws_bytes,
                                    int32_t *status, void *stream) {
-    if (B < 0 || T < 1 || V < 1) return CLOVER_ERR_INVALID_ARG;
-    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
-    if (T > kMaxTreeNodes) return CLOVER_ERR_UNSUPPORTED;
-    if (B == 0) return CLOVER_OK;
-    if ((long)B * T > 0x7FFFFFFFL) return CLOVER_ERR_UNSUPPORTED;
-    if (!logits || !cand || !parent || !argmax_out || !path_out || !accept_len || !bonus_token)
-        return CLOVER_ERR_INVALID_ARG;
-    const size_t need = accept_workspace_bytes(B, T, V, dtype);
-    if (ws_bytes < need || !workspace || (reinterpret_cast<uintptr_t>(workspace) & 7u)) return CLOVER_ERR_INVALID_ARG;
-    if (reinterpret_cast<uintptr_t>(logits) % (dtype == CLOVER_F32 ? 4 : 2)) return CLOVER_ERR_INVALID_ARG;
-    return from_cuda(launch_accept(logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
-                                   bonus_token, workspace, status, static_cast<cudaStream_t>(stream)));
+    AcceptCall c;
+    const clover_status s = check_accept(c, logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
+                                         bonus_token, workspace, ws_bytes, status, false, 0.0, 0.0, 0.0);
+    if (s != CLOVER_OK || B == 0) return s;
+    return from_cuda(launch_accept_call(c, static_cast<cudaStream_t>(stream)));
 }
 
 size_t clover_verify_accept_typical_workspace_size(int B, int T, int V, clover_dtype dtype) {
@@ -252,27 +287,54 @@ clover_status clover_verify_accept_typical(const void *logits, const int32_t *ca
                                            double delta, int32_t *argmax_out, int32_t *path_out,
                                            int32_t *accept_len, int32_t *bonus_token, void *workspace,
                                            size_t ws_bytes, int32_t *status, void *stream) {
-    if (B < 0 || T < 1 || V < 1) return CLOVER_ERR_INVALID_ARG;
-    if (dtype != CLOVER_F32 && dtype != CLOVER_BF16) return CLOVER_ERR_INVALID_ARG;
-    if (!(temperature > 0.0) || !isfinite(temperature) || !(epsilon >= 0.0) || !isfinite(epsilon) ||
-        !(delta >= 0.0) || !isfinite(delta))
-        return CLOVER_ERR_INVALID_ARG;
-    // exponents are kept in base 2: y = x log2(e) / temperature, in fp32
-    const float y_scale = (float)(1.4426950408889634 / temperature);
-    if (!isfinite(y_scale) || !(y_scale >= 1.17549435e-38f)) return CLOVER_ERR_UNSUPPORTED;
-    if (T > kMaxTreeNodes) return CLOVER_ERR_UNSUPPORTED;
+    AcceptCall c;
+    const clover_status s = check_accept(c, logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
+                                         bonus_token, workspace, ws_bytes, status, true, temperature, epsilon,
+                                         delta);
+    if (s != CLOVER_OK || B == 0) return s;
+    return from_cuda(launch_accept_call(c, static_cast<cudaStream_t>(stream)));
+}
+
+size_t clover_verify_accept_ex_workspace_size(int B, int T, int V, clover_dtype dtype, uint32_t flags) {
+    return (flags & CLOVER_ACCEPT_TYPICAL) ? clover_verify_accept_typical_workspace_size(B, T, V, dtype)
+                                           : clover_verify_accept_workspace_size(B, T, V, dtype);
+}
+
+clover_status clover_verify_accept_ex(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
+                                      int V, clover_dtype dtype, double temperature, double epsilon, double delta,
+                                      void *k_cache, void *v_cache, const void *k_new, const void *v_new,
+                                      const int32_t *cache_len, int Hkv, int D, int Lcap, int32_t *argmax_out,
+                                      int32_t *path_out, int32_t *accept_len, int32_t *bonus_token,
+                                      int32_t *new_cache_len, int32_t *src_index_out, void *workspace,
+                                      size_t ws_bytes, uint32_t flags, int32_t *status, void *stream) {
+    constexpr uint32_t known = CLOVER_ACCEPT_TYPICAL | CLOVER_ACCEPT_COMMIT | CLOVER_ACCEPT_OVERLAP;
+    if (flags & ~known) return CLOVER_ERR_INVALID_ARG;
+    AcceptCall c;
+    clover_status s = check_accept(c, logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
+                                   bonus_token, workspace, ws_bytes, status, (flags & CLOVER_ACCEPT_TYPICAL) != 0,
+                                   temperature, epsilon, delta);
+    if (s != CLOVER_OK) return s;
+    if (flags & CLOVER_ACCEPT_COMMIT) {
+        // the path and accepted length are this call's own outputs: any
+        // non-NULL pointers pass the commit checks on them
+        s = check_commit(k_cache, v_cache, k_new, v_new, cache_len, path_out, accept_len, new_cache_len, B, T, Hkv,
+                         D, Lcap, dtype, true);
+        if (s != CLOVER_OK) return s;
+        c.commit = true;
+        c.k_cache = k_cache;
+        c.v_cache = v_cache;
+        c.k_new = k_new;
+        c.v_new = v_new;
+        c.cache_len = cache_len;
+        c.new_cache_len = new_cache_len;
+        c.src_index = src_index_out;
+        c.Hkv = Hkv;
+        c.D = D;
+        c.Lcap = Lcap;
+    }
+    c.after_prior = (flags & CLOVER_ACCEPT_OVERLAP) != 0;
     if (B == 0) return CLOVER_OK;
-    if ((long)B * T > 0x7FFFFFFFL) return CLOVER_ERR_UNSUPPORTED;
-    if (!logits || !cand || !parent || !argmax_out || !path_out || !accept_len || !bonus_token)
-        return CLOVER_ERR_INVALID_ARG;
-    const size_t need = accept_typical_workspace_bytes(B, T, V, dtype);
-    if (ws_bytes < need || !workspace || !aligned16(workspace)) return CLOVER_ERR_INVALID_ARG;
-    if (reinterpret_cast<uintptr_t>(logits) % (dtype == CLOVER_F32 ? 4 : 2)) return CLOVER_ERR_INVALID_ARG;
-    const float log2_eps = epsilon > 0.0 ? (float)log2(epsilon) : -INFINITY;
-    const float log2_delta = delta > 0.0 ? (float)log2(delta) : -INFINITY;
-    return from_cuda(launch_accept_typical(logits, cand, parent, B, T, V, dtype, y_scale, log2_eps, log2_delta,
-                                           argmax_out, path_out, accept_len, bonus_token, workspace, status,
-                                           static_cast<cudaStream_t>(stream)));
+    return from_cuda(launch_accept_call(c, static_cast<cudaStream_t>(stream)));
 }
 
 clover_status clover_kv_commit(void *k_cache, void *v_cache, const void *k_new, const void *v_new,

@@ -197,6 +197,14 @@ struct AcceptArgs {
     float *cand_x;                 // [B*T] logit of each node's candidate under its parent
     float y_scale;                 // log2(e) / temperature
     float log2_eps, log2_delta;    // log2 of the threshold parameters (-inf for 0)
+    // commit of the accepted K/V by the sequence's last CTA (commit != 0)
+    uint4 *k_cache, *v_cache;      // [B, Hkv, Lcap, D] as 16-byte units
+    const uint4 *k_new, *v_new;    // [B, T, Hkv, D]
+    const int32_t *cache_len;
+    int32_t *new_cache_len, *src_index;
+    int Hkv, Lcap, row_units;      // row_units = D * element size / 16
+    int commit;
+    int wait_prior;                // the last CTAs end with a wait for the preceding grid
     int32_t *status;
 };
 
@@ -275,9 +283,115 @@ __device__ __forceinline__ TreeRegs load_tree(const AcceptArgs &a, int b) {
 // nodes whose whole root path is accepted, takes the greatest depth among
 // them and the union G of the root paths of the accepted nodes at that depth,
 // and walks from the root through G, the smallest-index child at every step.
+// The walk of finish_sequence, by warp 0; the path also goes to s_path/s_len.
+template <bool TYPICAL>
+__device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, const int (&am)[2],
+                              const float (&xc)[2], const float4 *s_row, int *s_path, int *s_len) {
+    const int lane = threadIdx.x & 31;
+    const int Tn = a.T;
+    int32_t *path = a.path_out + (size_t)b * Tn;
+    for (int i = lane; i < Tn; i += 32) path[i] = -1;
+    __syncwarp();
+    int cur = 0, len = 1;
+    if (lane == 0) path[0] = s_path[0] = 0;
+    auto argmax_of = [&](int node) {
+        const int lo = __shfl_sync(0xffffffffu, am[0], node & 31);
+        const int hi = __shfl_sync(0xffffffffu, am[1], node & 31);
+        return (node >> 5) ? hi : lo;
+    };
+    if (__any_sync(0xffffffffu, tr.invalid)) {
+        if (lane == 0) report(a.status, CLOVER_ERR_BAD_TREE);
+    } else if (!TYPICAL) {
+        // at most T - 1 steps: every step moves to a larger node index
+        for (int step = 1; step < Tn; ++step) {
+            const int want = argmax_of(cur);
+            const unsigned lo = __ballot_sync(0xffffffffu, tr.p[0] == cur && tr.c[0] == want);
+            const unsigned hi = __ballot_sync(0xffffffffu, tr.p[1] == cur && tr.c[1] == want);
+            const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
+            if (hits == 0ull) break;
+            cur = __ffsll(static_cast<long long>(hits)) - 1;
+            if (lane == 0) path[len] = s_path[len] = cur;
+            ++len;
+        }
+    } else {
+        uint64_t anc[2];
+        tree_masks_regs(tr.p, Tn, anc);
+        bool ok[2];
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int i = lane + 32 * k;
+            ok[k] = false;
+            if (i >= 1 && i < Tn) {
+                const float4 r = s_row[tr.p[k]];
+                ok[k] = fmaf(xc[k], a.y_scale, -r.x) - r.y > r.z;   // log2 p > log2 theta
+            }
+        }
+        const uint64_t acc = (static_cast<uint64_t>(__ballot_sync(0xffffffffu, ok[1])) << 32) |
+                             __ballot_sync(0xffffffffu, ok[0]) | 1ull;
+        int depth[2];
+        unsigned dmax = 0;
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const bool reach = lane + 32 * k < Tn && (anc[k] & ~acc) == 0ull;
+            depth[k] = reach ? __popcll(anc[k]) - 1 : -1;
+            dmax = max(dmax, (unsigned)max(depth[k], 0));
+        }
+        dmax = __reduce_max_sync(0xffffffffu, dmax);
+        uint64_t g = 0ull;
+#pragma unroll
+        for (int k = 0; k < 2; ++k)
+            if (depth[k] == (int)dmax) g |= anc[k];
+        g = (static_cast<uint64_t>(__reduce_or_sync(0xffffffffu, (unsigned)(g >> 32))) << 32) |
+            __reduce_or_sync(0xffffffffu, (unsigned)g);
+        for (unsigned step = 0; step < dmax; ++step) {
+            const unsigned lo = __ballot_sync(0xffffffffu, tr.p[0] == cur && ((g >> lane) & 1ull));
+            const unsigned hi = __ballot_sync(0xffffffffu, tr.p[1] == cur && ((g >> (lane + 32)) & 1ull));
+            const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
+            if (hits == 0ull) break;
+            cur = __ffsll(static_cast<long long>(hits)) - 1;
+            if (lane == 0) path[len] = s_path[len] = cur;
+            ++len;
+        }
+    }
+    const int bonus = argmax_of(cur);
+    if (lane == 0) {
+        a.accept_len[b] = len;
+        a.bonus[b] = bonus;
+        a.seq_count[b] = 0u;                                       // ready for the next call
+        *s_len = len;
+    }
+}
+
+// Commit of sequence b's accepted path (len nodes in s_path) by the whole CTA:
+// slot L + j of every KV head receives node s_path[j]'s K/V from k_new/v_new.
+__device__ void commit_sequence(const AcceptArgs &a, int b, const int *s_path, int len) {
+    const int Tn = a.T;
+    const int L = __ldg(a.cache_len + b);
+    if (L < 0 || L + Tn > a.Lcap) {
+        if (threadIdx.x == 0) report(a.status, CLOVER_ERR_CAPACITY);
+        return;
+    }
+    if (a.src_index && threadIdx.x < Tn) a.src_index[(size_t)b * Tn + threadIdx.x] = threadIdx.x < len ? s_path[threadIdx.x] : -1;
+    if (threadIdx.x == 0) a.new_cache_len[b] = L + len;
+    const int per_node = a.Hkv * a.row_units;
+    for (int j = 0; j < len; ++j) {
+        const uint4 *ks = a.k_new + ((size_t)b * Tn + s_path[j]) * per_node;
+        const uint4 *vs = a.v_new + ((size_t)b * Tn + s_path[j]) * per_node;
+        for (int e = threadIdx.x; e < per_node; e += kThreads) {
+            const int g = e / a.row_units;
+            const int u = e - g * a.row_units;
+            const size_t dst = (((size_t)b * a.Hkv + g) * a.Lcap + L + j) * a.row_units + u;
+            a.k_cache[dst] = __ldg(ks + e);
+            a.v_cache[dst] = __ldg(vs + e);
+        }
+    }
+}
+
 template <typename T, bool TYPICAL>
 __device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) {
     __shared__ float4 s_row[kMaxTreeNodes];
+    __shared__ int s_path[kMaxTreeNodes];
+    __shared__ int s_len;
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int Tn = a.T;
@@ -321,77 +435,12 @@ __device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) 
         }
         __syncthreads();
     }
-    if (warp != 0) return;
-
-    int32_t *path = a.path_out + (size_t)b * Tn;
-    for (int i = lane; i < Tn; i += 32) path[i] = -1;
-    __syncwarp();
-    int cur = 0, len = 1;
-    if (lane == 0) path[0] = 0;
-    auto argmax_of = [&](int node) {
-        const int lo = __shfl_sync(0xffffffffu, am[0], node & 31);
-        const int hi = __shfl_sync(0xffffffffu, am[1], node & 31);
-        return (node >> 5) ? hi : lo;
-    };
-    if (__any_sync(0xffffffffu, tr.invalid)) {
-        if (lane == 0) report(a.status, CLOVER_ERR_BAD_TREE);
-    } else if (!TYPICAL) {
-        // at most T - 1 steps: every step moves to a larger node index
-        for (int step = 1; step < Tn; ++step) {
-            const int want = argmax_of(cur);
-            const unsigned lo = __ballot_sync(0xffffffffu, tr.p[0] == cur && tr.c[0] == want);
-            const unsigned hi = __ballot_sync(0xffffffffu, tr.p[1] == cur && tr.c[1] == want);
-            const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
-            if (hits == 0ull) break;
-            cur = __ffsll(static_cast<long long>(hits)) - 1;
-            if (lane == 0) path[len] = cur;
-            ++len;
-        }
-    } else {
-        uint64_t anc[2];
-        tree_masks_regs(tr.p, Tn, anc);
-        bool ok[2];
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            const int i = lane + 32 * k;
-            ok[k] = false;
-            if (i >= 1 && i < Tn) {
-                const float4 r = s_row[tr.p[k]];
-                ok[k] = fmaf(xc[k], a.y_scale, -r.x) - r.y > r.z;   // log2 p > log2 theta
-            }
-        }
-        const uint64_t acc = (static_cast<uint64_t>(__ballot_sync(0xffffffffu, ok[1])) << 32) |
-                             __ballot_sync(0xffffffffu, ok[0]) | 1ull;
-        int depth[2];
-        unsigned dmax = 0;
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            const bool reach = lane + 32 * k < Tn && (anc[k] & ~acc) == 0ull;
-            depth[k] = reach ? __popcll(anc[k]) - 1 : -1;
-            dmax = max(dmax, (unsigned)max(depth[k], 0));
-        }
-        dmax = __reduce_max_sync(0xffffffffu, dmax);
-        uint64_t g = 0ull;
-#pragma unroll
-        for (int k = 0; k < 2; ++k)
-            if (depth[k] == (int)dmax) g |= anc[k];
-        g = (static_cast<uint64_t>(__reduce_or_sync(0xffffffffu, (unsigned)(g >> 32))) << 32) |
-            __reduce_or_sync(0xffffffffu, (unsigned)g);
-        for (unsigned step = 0; step < dmax; ++step) {
-            const unsigned lo = __ballot_sync(0xffffffffu, tr.p[0] == cur && ((g >> lane) & 1ull));
-            const unsigned hi = __ballot_sync(0xffffffffu, tr.p[1] == cur && ((g >> (lane + 32)) & 1ull));
-            const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
-            if (hits == 0ull) break;
-            cur = __ffsll(static_cast<long long>(hits)) - 1;
-            if (lane == 0) path[len] = cur;
-            ++len;
-        }
-    }
-    const int bonus = argmax_of(cur);
-    if (lane == 0) {
-        a.accept_len[b] = len;
-        a.bonus[b] = bonus;
-        a.seq_count[b] = 0u;                                       // ready for the next call
+    if (warp == 0) walk_sequence<TYPICAL>(a, b, tr, am, xc, s_row, s_path, &s_len);
+    if (a.commit || a.wait_prior) {
+        __syncthreads();
+        if (a.commit) commit_sequence(a, b, s_path, s_len);
+        // this grid completes only after the grid it may have overlapped
+        if (a.wait_prior) wait_prerequisite_grids();
     }
 }
 
@@ -523,53 +572,65 @@ size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype) {
     return accept_sums_offset(B, T) + sizeof(float4) * (size_t)B * T * n_chunks + sizeof(float) * (size_t)B * T;
 }
 
-static AcceptArgs accept_args(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T, int V,
-                              int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len,
-                              int32_t *bonus, void *workspace, int32_t *status) {
+// A launch with after_prior is a programmatic dependent of the preceding
+// kernel in the stream (which may let it start early).
+template <typename T, bool TYPICAL>
+static cudaError_t launch_kernel(const AcceptArgs &a, bool after_prior, cudaStream_t stream) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.B * a.T, a.n_chunks);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = after_prior ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, accept_kernel<T, TYPICAL>, a);
+}
+
+cudaError_t launch_accept_call(const AcceptCall &c, cudaStream_t stream) {
     AcceptArgs a{};
-    a.logits = logits;
-    a.cand = cand;
-    a.parent = parent;
-    a.B = B;
-    a.T = T;
-    a.V = V;
-    accept_plan(B, T, V, dtype, &a.n_chunks, &a.chunk);
-    a.argmax_out = argmax_out;
-    a.path_out = path_out;
-    a.accept_len = accept_len;
-    a.bonus = bonus;
-    a.row_key = static_cast<unsigned long long *>(workspace);
-    a.seq_count = reinterpret_cast<unsigned *>(a.row_key + (size_t)B * T);
-    a.status = status;
-    return a;
-}
-
-cudaError_t launch_accept(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
-                          int V, int dtype, int32_t *argmax_out, int32_t *path_out, int32_t *accept_len,
-                          int32_t *bonus, void *workspace, int32_t *status, cudaStream_t stream) {
-    const AcceptArgs a = accept_args(logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len, bonus,
-                                     workspace, status);
-    dim3 grid(B * T, a.n_chunks);
-    if (dtype == CLOVER_F32) accept_kernel<float, false><<<grid, kThreads, 0, stream>>>(a);
-    else accept_kernel<__nv_bfloat16, false><<<grid, kThreads, 0, stream>>>(a);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_accept_typical(const void *logits, const int32_t *cand, const int32_t *parent, int B, int T,
-                                  int V, int dtype, float y_scale, float log2_eps, float log2_delta,
-                                  int32_t *argmax_out, int32_t *path_out, int32_t *accept_len, int32_t *bonus,
-                                  void *workspace, int32_t *status, cudaStream_t stream) {
-    AcceptArgs a = accept_args(logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len, bonus,
-                               workspace, status);
-    a.chunk_sums = reinterpret_cast<float4 *>(static_cast<uint8_t *>(workspace) + accept_sums_offset(B, T));
-    a.cand_x = reinterpret_cast<float *>(a.chunk_sums + (size_t)B * T * a.n_chunks);
-    a.y_scale = y_scale;
-    a.log2_eps = log2_eps;
-    a.log2_delta = log2_delta;
-    dim3 grid(B * T, a.n_chunks);
-    if (dtype == CLOVER_F32) accept_kernel<float, true><<<grid, kThreads, 0, stream>>>(a);
-    else accept_kernel<__nv_bfloat16, true><<<grid, kThreads, 0, stream>>>(a);
-    return cudaGetLastError();
+    a.logits = c.logits;
+    a.cand = c.cand;
+    a.parent = c.parent;
+    a.B = c.B;
+    a.T = c.T;
+    a.V = c.V;
+    accept_plan(c.B, c.T, c.V, c.dtype, &a.n_chunks, &a.chunk);
+    a.argmax_out = c.argmax_out;
+    a.path_out = c.path_out;
+    a.accept_len = c.accept_len;
+    a.bonus = c.bonus;
+    a.row_key = static_cast<unsigned long long *>(c.workspace);
+    a.seq_count = reinterpret_cast<unsigned *>(a.row_key + (size_t)c.B * c.T);
+    if (c.typical) {
+        a.chunk_sums = reinterpret_cast<float4 *>(static_cast<uint8_t *>(c.workspace) + accept_sums_offset(c.B, c.T));
+        a.cand_x = reinterpret_cast<float *>(a.chunk_sums + (size_t)c.B * c.T * a.n_chunks);
+        a.y_scale = c.y_scale;
+        a.log2_eps = c.log2_eps;
+        a.log2_delta = c.log2_delta;
+    }
+    if (c.commit) {
+        a.commit = 1;
+        a.k_cache = static_cast<uint4 *>(c.k_cache);
+        a.v_cache = static_cast<uint4 *>(c.v_cache);
+        a.k_new = static_cast<const uint4 *>(c.k_new);
+        a.v_new = static_cast<const uint4 *>(c.v_new);
+        a.cache_len = c.cache_len;
+        a.new_cache_len = c.new_cache_len;
+        a.src_index = c.src_index;
+        a.Hkv = c.Hkv;
+        a.Lcap = c.Lcap;
+        a.row_units = c.D * (c.dtype == CLOVER_F32 ? 4 : 2) / 16;
+    }
+    a.wait_prior = c.after_prior ? 1 : 0;
+    a.status = c.status;
+    if (c.dtype == CLOVER_F32)
+        return c.typical ? launch_kernel<float, true>(a, c.after_prior, stream)
+                         : launch_kernel<float, false>(a, c.after_prior, stream);
+    return c.typical ? launch_kernel<__nv_bfloat16, true>(a, c.after_prior, stream)
+                     : launch_kernel<__nv_bfloat16, false>(a, c.after_prior, stream);
 }
 
 }  // namespace clover

@@ -32,6 +32,41 @@ struct AttnArgs {
     int32_t *status;
 };
 
+// One acceptance call (clover_verify_accept, _typical or _ex), validated on
+// the host.
+struct AcceptCall {
+    const void *logits;
+    const int32_t *cand, *parent;
+    int B, T, V, dtype;
+    int32_t *argmax_out, *path_out, *accept_len, *bonus;
+    void *workspace;
+    int32_t *status;
+    bool typical;                   // typical rule with the three values below
+    float y_scale, log2_eps, log2_delta;
+    bool commit;                    // also commit the accepted K/V (from k_new/v_new)
+    void *k_cache, *v_cache;
+    const void *k_new, *v_new;
+    const int32_t *cache_len;
+    int32_t *new_cache_len, *src_index;
+    int Hkv, D, Lcap;
+    bool after_prior;               // launch as a programmatic dependent of the preceding kernel
+};
+
+// Programmatic dependent launch: lets the next kernel in the stream, if it
+// was launched as a programmatic dependent, start as soon as every CTA of this
+// grid has issued this (the dependent then waits for this grid's completion
+// itself where it has to).  Without such a dependent it has no effect.
+__device__ __forceinline__ void allow_dependent_launch() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Waits until the grids this one was launched as a programmatic dependent of
+// have completed and their memory operations are visible; returns at once in a
+// grid launched the ordinary way.
+__device__ __forceinline__ void wait_prerequisite_grids() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 __device__ __forceinline__ void report(int32_t *status, int bits) {
     if (status) atomicOr(status, bits);
 }

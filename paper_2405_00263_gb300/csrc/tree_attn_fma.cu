@@ -102,6 +102,7 @@ __device__ __forceinline__ void unpack<__nv_bfloat16>(const uint4 &u, float *dst
 
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnArgs a) {
+    allow_dependent_launch();
     using S = FmaSmem<D>;
     extern __shared__ float4 smem4[];
     float *smem = reinterpret_cast<float *>(smem4);

@@ -169,6 +169,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     using S = TcSmem<D, KS>;
     constexpr int NSK = S::NSK;
     constexpr int NSV = S::NSV;
+    // an accept call queued behind this one as a programmatic dependent may
+    // take the SM space this grid leaves free
+    allow_dependent_launch();
     extern __shared__ uint8_t smem_raw[];
     // base rounded up to 1024 bytes by pointer arithmetic on the shared array,
     // so that every access below stays a shared-memory access

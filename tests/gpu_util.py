@@ -39,8 +39,8 @@ def compare_full(host: dict, step: pkg.VerifyStep, t: dict, scale: float = 0.0):
     assert torch.equal(step.path.cpu(), ref["path"])
     assert torch.equal(step.accept_len.cpu(), ref["accept_len"])
     assert torch.equal(step.bonus.cpu(), ref["bonus"])
-    # the commit schedule records tree nodes, the compaction schedule cache slots
-    exp_src = ref["path"] if step.schedule == "commit" else ref["src_index"]
+    # the commit and fused schedules record tree nodes, the compaction schedule cache slots
+    exp_src = ref["path"] if step.schedule in ("commit", "fused") else ref["src_index"]
     assert torch.equal(step.src_index.cpu(), exp_src)
     assert torch.equal(step.new_cache_len.cpu(), ref["cache_len"])
     kc, vc = t["k_cache"].cpu(), t["v_cache"].cpu()

@@ -141,6 +141,28 @@ def test_accept_typical_workspace_and_host_validation(lib):
     assert call(B=0) == 0
 
 
+def test_accept_ex_host_validation(lib):
+    P = ctypes.c_void_p
+    assert lib.clover_verify_accept_ex_workspace_size(2, 4, 125696, 1, 0) == \
+        lib.clover_verify_accept_workspace_size(2, 4, 125696, 1)
+    assert lib.clover_verify_accept_ex_workspace_size(2, 4, 125696, 1, 1) == \
+        lib.clover_verify_accept_typical_workspace_size(2, 4, 125696, 1)
+
+    def call(flags, tau=1.0, kn=64, D=128, B=2, T=4, ncl=4096, cl=2048, ws=4096):
+        return lib.clover_verify_accept_ex(P(64), P(64), P(64), B, T, 1000, 1, tau, 0.09, 0.3, P(64), P(64), P(kn),
+                                           P(64), P(cl), 2, D, 64, P(64), P(64), P(64), P(64), P(ncl), None, P(ws),
+                                           1 << 20, flags, None, None)
+    assert call(8) == 1 and call(0xFFFFFFF0) == 1             # unknown flag bits
+    assert call(1, tau=0.0) == 1                             # typical: temperature must be > 0
+    assert call(2, kn=0) == 1                                # commit: k_new missing
+    assert call(2, kn=72) == 1                               # commit: k_new misaligned
+    assert call(2, D=96) == 2                                # commit: D not 64/128
+    assert call(2, ncl=2048) == 1                            # commit: new length aliases the old one
+    assert call(1, ws=4104) == 1                             # typical: workspace 16-byte aligned
+    assert call(7, T=65) == 2
+    assert call(7, B=0) == 0
+
+
 def test_python_binding_rejects_cpu_tensors(lib):
     import paper_2405_00263_gb300 as pkg
     x = torch.zeros(1, 4, 2, 64, dtype=torch.bfloat16)

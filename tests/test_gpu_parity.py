@@ -68,8 +68,9 @@ def test_repeated_calls_reuse_workspace(cuda):
 FULL = ["7b_l2048", "7b_l4096", "7b_l16384", "7b_batched", "100b_gqa", "paper_t4_b4", "paper_t4_b16", "paper_t4_b48"]
 
 
+@pytest.mark.parametrize("schedule", ["commit", "fused"])
 @pytest.mark.parametrize("name", FULL)
-def test_full_size_workloads(name, cuda):
+def test_full_size_workloads(name, schedule, cuda):
     """The workloads at their full sizes: attention on sampled rows (the
     oracle computes them one by one), argmax / walk / indices everywhere, the
     tree slots of the cache everywhere, and the committed prefix untouched."""
@@ -77,7 +78,7 @@ def test_full_size_workloads(name, cuda):
     t = workloads.make(w, device=cuda)
     host = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in t.items()}
     kc0, vc0 = t["k_cache"].clone(), t["v_cache"].clone()
-    step = run_gpu(t)
+    step = run_gpu(t, schedule=schedule)
     assert step.device_status() == 0
 
     B, T, Hq, D = w.B, w.T, w.Hq, w.D
@@ -105,7 +106,7 @@ def test_full_size_workloads(name, cuda):
     zl = torch.zeros(B, dtype=torch.int32)
     oracle.append_tree_kv(host["k_new"], host["v_new"], zk, zv, zl)
     src = oracle.kv_compact(zk, zv, zl, path, alen)
-    exp_src = path if step.schedule == "commit" else torch.where(src >= 0, src + L.unsqueeze(1), src)
+    exp_src = path if step.schedule in ("commit", "fused") else torch.where(src >= 0, src + L.unsqueeze(1), src)
     assert torch.equal(step.src_index.cpu(), exp_src)
     for b in range(B):
         l0, a = int(L[b]), int(alen[b])
@@ -156,19 +157,23 @@ def test_commit_and_compact_schedules_agree(case, concurrent, cuda):
     and give the same outputs; both match the oracle."""
     name, over = SCHEDULE_CASES[case]
     host = workloads.make(workloads.get(name, **over))
-    t1, t2 = to_dev(host, cuda), to_dev(host, cuda)
+    t1, t2, t3 = to_dev(host, cuda), to_dev(host, cuda), to_dev(host, cuda)
     s1 = run_gpu(t1, schedule="commit", concurrent=concurrent)
     s2 = run_gpu(t2, schedule="compact", concurrent=concurrent)
+    s3 = run_gpu(t3, schedule="fused", concurrent=concurrent)
     compare_full(host, s1, t1)
     compare_full(host, s2, t2)
-    assert torch.equal(s1.out, s2.out)
+    compare_full(host, s3, t3)
+    assert torch.equal(s1.out, s2.out) and torch.equal(s1.out, s3.out)
+    assert torch.equal(s1.src_index, s3.src_index) and torch.equal(s1.new_cache_len, s3.new_cache_len)
     L = host["cache_len"].to(cuda)
     assert torch.equal(torch.where(s1.src_index >= 0, s1.src_index + L.unsqueeze(1), s1.src_index), s2.src_index)
     bits = torch.int16 if host["q"].dtype == torch.bfloat16 else torch.int32
     for b in range(host["q"].shape[0]):
         n = int(s1.new_cache_len[b])
-        assert torch.equal(t1["k_cache"][b, :, :n].view(bits), t2["k_cache"][b, :, :n].view(bits))
-        assert torch.equal(t1["v_cache"][b, :, :n].view(bits), t2["v_cache"][b, :, :n].view(bits))
+        for t in (t2, t3):
+            assert torch.equal(t1["k_cache"][b, :, :n].view(bits), t["k_cache"][b, :, :n].view(bits))
+            assert torch.equal(t1["v_cache"][b, :, :n].view(bits), t["v_cache"][b, :, :n].view(bits))
 
 
 @pytest.mark.parametrize("name", ["tiny_f32", "7b_l2048"])
@@ -331,3 +336,45 @@ def test_host_errors_raise(cuda):
     with pytest.raises(pkg.CloverError):   # new length may not alias the old one
         pkg.clover_kv_compact(t["k_cache"], t["v_cache"], t["cache_len"], torch.zeros_like(t["parent"]),
                               torch.ones_like(t["cache_len"]), new_len)
+
+
+def test_accept_ex_commit_capacity_and_overlap_flag(cuda):
+    """clover_verify_accept_ex with the commit fused in: a sequence whose cache
+    has no room for T more slots raises CLOVER_ERR_CAPACITY and is left
+    untouched, the others match clover_kv_commit; the overlap flag changes
+    nothing in the results (here the preceding kernel is unrelated work)."""
+    w = workloads.get("7b_l2048", B=3, T=16, Hq=4, Hkv=2, D=64, L=200, V=3000, branching=(4, 2, 1, 1))
+    host = workloads.make(w)
+    Lcap = host["Lcap"]
+    host["cache_len"][1] = Lcap - w.T + 1                   # one slot short
+    for overlap in (False, True):
+        t = to_dev(host, cuda)
+        i32 = dict(dtype=torch.int32, device=cuda)
+        am, path = torch.empty((w.B, w.T), **i32), torch.empty((w.B, w.T), **i32)
+        alen, bonus, ncl = torch.empty(w.B, **i32), torch.empty(w.B, **i32), torch.full((w.B,), -7, **i32)
+        src = torch.empty((w.B, w.T), **i32)
+        st = torch.zeros(1, **i32)
+        ws = torch.zeros(pkg.clover_verify_accept_ex_workspace_size(w.B, w.T, w.V, w.torch_dtype, 2),
+                         dtype=torch.uint8, device=cuda)
+        scratch = torch.zeros(1 << 20, device=cuda)
+        scratch.mul_(2.0)                                      # some unrelated kernel before the call
+        pkg.clover_verify_accept_ex(t["logits"], t["cand"], t["parent"], am, path, alen, bonus, ws,
+                                    commit=(t["k_cache"], t["v_cache"], t["k_new"], t["v_new"], t["cache_len"],
+                                            ncl, src), overlap=overlap, status=st)
+        torch.cuda.synchronize()
+        assert int(st.item()) == 8                             # CLOVER_ERR_CAPACITY
+        amax = oracle.argmax(host["logits"])
+        rpath, ralen, rbonus = oracle.accept_walk(host["parent"], host["cand"], amax)
+        assert torch.equal(path.cpu(), rpath) and torch.equal(alen.cpu(), ralen) and torch.equal(bonus.cpu(), rbonus)
+        ok = torch.tensor([0, 2])
+        kc_ok, vc_ok = host["k_cache"][ok].contiguous(), host["v_cache"][ok].contiguous()
+        rsrc = oracle.kv_commit(kc_ok, vc_ok, host["k_new"][ok].contiguous(), host["v_new"][ok].contiguous(),
+                                host["cache_len"][ok].contiguous(), rpath[ok], ralen[ok])
+        for n, b in enumerate(ok.tolist()):
+            m = int(host["cache_len"][b]) + int(ralen[b])
+            assert int(ncl[b]) == m
+            assert torch.equal(src[b].cpu(), rsrc[n])
+            assert torch.equal(t["k_cache"][b, :, :m].cpu().view(torch.int16), kc_ok[n, :, :m].view(torch.int16))
+            assert torch.equal(t["v_cache"][b, :, :m].cpu().view(torch.int16), vc_ok[n, :, :m].view(torch.int16))
+        assert int(ncl[1]) == -7                              # not committed
+        assert torch.equal(t["k_cache"][1].cpu().view(torch.int16), host["k_cache"][1].view(torch.int16))

@@ -187,7 +187,7 @@ def test_typical_bad_tree_sets_status():
     assert int(got["accept_len"][1]) == 1 and int(got["path"][1, 0]) == 0
 
 
-@pytest.mark.parametrize("schedule", ["commit", "compact"])
+@pytest.mark.parametrize("schedule", ["commit", "compact", "fused"])
 @pytest.mark.parametrize("name,over,params", [
     ("tiny_f32", {}, (1.0, 0.09, 0.3)),
     ("7b_l2048", dict(B=2, T=64, Hq=8, Hkv=2, L=700, V=5003), (0.8, 0.09, 0.3)),
