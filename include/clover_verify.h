@@ -43,7 +43,7 @@
  *     0 <= parent[b][i] < i for i >= 1, so nodes are topologically numbered.
  *     Node i attends to node j iff j is i or an ancestor of i (the tree's
  *     topology as the attention mask, Section 2.2).
- *   - Limits: 1 <= T <= 64, D in {64, 128}, Hq a multiple of Hkv (query head h
+ *   - Limits: 1 <= T <= 128, D in {64, 128}, Hq a multiple of Hkv (query head h
  *     reads KV head h / (Hq/Hkv)), cache_len[b] + T <= Lcap.
  */
 #ifndef CLOVER_VERIFY_H
@@ -65,7 +65,7 @@ extern "C" {
 typedef enum {
     CLOVER_OK = 0,
     CLOVER_ERR_INVALID_ARG = 1,  /* bad size, NULL or misaligned pointer, short workspace */
-    CLOVER_ERR_UNSUPPORTED = 2,  /* outside the limits above (T > 64, D not 64/128, ...) */
+    CLOVER_ERR_UNSUPPORTED = 2,  /* outside the limits above (T > 128, D not 64/128, ...) */
     CLOVER_ERR_BAD_TREE = 4,     /* device: parent array is not a topologically numbered tree */
     CLOVER_ERR_CAPACITY = 8,     /* device: cache_len[b] < 0 or cache_len[b] + T > Lcap */
     CLOVER_ERR_CUDA = 16,        /* a CUDA launch or query failed */

@@ -208,44 +208,11 @@ struct AcceptArgs {
     int32_t *status;
 };
 
-// Ancestor-or-self bitmasks of a valid tree by pointer jumping in one warp's
-// registers: lane l owns nodes l and l + 32 with parents parent[0..1].  After
-// round k each mask covers the node's 2^k nearest ancestors; six rounds cover
-// depth 63.
-__device__ __forceinline__ void tree_masks_regs(const int (&parent)[2], int T, uint64_t (&m)[2]) {
-    const int lane = threadIdx.x & 31;
-    int up[2];
-#pragma unroll
-    for (int k = 0; k < 2; ++k) {
-        const int i = lane + 32 * k;
-        m[k] = (i < T) ? (1ull << i) : 0ull;
-        up[k] = (i < T && i > 0) ? parent[k] : -1;
-    }
-#pragma unroll
-    for (int round = 0; round < 6; ++round) {
-        uint64_t nm[2];
-        int nu[2];
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            const int u = up[k] < 0 ? 0 : up[k];
-            const uint64_t m0 = __shfl_sync(0xffffffffu, m[0], u & 31);
-            const uint64_t m1 = __shfl_sync(0xffffffffu, m[1], u & 31);
-            const int u0 = __shfl_sync(0xffffffffu, up[0], u & 31);
-            const int u1 = __shfl_sync(0xffffffffu, up[1], u & 31);
-            nm[k] = up[k] < 0 ? m[k] : (m[k] | ((u >> 5) ? m1 : m0));
-            nu[k] = up[k] < 0 ? -1 : ((u >> 5) ? u1 : u0);
-        }
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            m[k] = nm[k];
-            up[k] = nu[k];
-        }
-    }
-}
+constexpr int kNodesPerLane = kMaxTreeNodes / 32;
 
-// Sequence b's tree in warp 0's registers: lane l holds nodes l and l + 32.
+// Sequence b's tree in warp 0's registers: lane l holds nodes l + 32 k.
 struct TreeRegs {
-    int p[2], c[2];
+    int p[kNodesPerLane], c[kNodesPerLane];
     bool invalid;
 };
 
@@ -256,7 +223,7 @@ __device__ __forceinline__ TreeRegs load_tree(const AcceptArgs &a, int b) {
     TreeRegs t;
     t.invalid = false;
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < kNodesPerLane; ++k) {
         const int i = lane + 32 * k;
         t.p[k] = -2;
         t.c[k] = 0;
@@ -269,24 +236,21 @@ __device__ __forceinline__ TreeRegs load_tree(const AcceptArgs &a, int b) {
     return t;
 }
 
-// The CTA that finished sequence b's last chunk: argmax of every node from the
-// merged row keys, then the walk, by warp 0 (the walk reads the current
-// node's argmax from registers by warp shuffles, so a step costs no memory
-// round trip).  The row keys and the counter are reset for the next call.
-//
-// Greedy: from the root, the smallest-index child whose candidate equals the
-// current node's argmax, until there is none.
-// Typical: first every thread of the CTA merges a quarter of one row's chunk
-// sums (64 rows x 4 threads) into the row's (max, log2 S, log2 theta), while
-// warp 0 also reads each child's candidate logit (gathered by the chunk CTAs)
-// and builds the ancestor masks in registers.  Then warp 0 decides every edge, marks the
-// nodes whose whole root path is accepted, takes the greatest depth among
-// them and the union G of the root paths of the accepted nodes at that depth,
-// and walks from the root through G, the smallest-index child at every step.
+// First set bit of a warp's per-node predicate (node lane + 32 k for pred[k]);
+// -1 if none.
+__device__ __forceinline__ int first_node(const bool (&pred)[kNodesPerLane]) {
+#pragma unroll
+    for (int k = 0; k < kNodesPerLane; ++k) {
+        const unsigned bits = __ballot_sync(0xffffffffu, pred[k]);
+        if (bits) return 32 * k + __ffs(bits) - 1;
+    }
+    return -1;
+}
+
 // The walk of finish_sequence, by warp 0; the path also goes to s_path/s_len.
 template <bool TYPICAL>
-__device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, const int (&am)[2],
-                              const float (&xc)[2], const float4 *s_row, int *s_path, int *s_len) {
+__device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, const int (&am)[kNodesPerLane],
+                              const float (&xc)[kNodesPerLane], const float4 *s_row, int *s_path, int *s_len) {
     const int lane = threadIdx.x & 31;
     const int Tn = a.T;
     int32_t *path = a.path_out + (size_t)b * Tn;
@@ -295,9 +259,13 @@ __device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, co
     int cur = 0, len = 1;
     if (lane == 0) path[0] = s_path[0] = 0;
     auto argmax_of = [&](int node) {
-        const int lo = __shfl_sync(0xffffffffu, am[0], node & 31);
-        const int hi = __shfl_sync(0xffffffffu, am[1], node & 31);
-        return (node >> 5) ? hi : lo;
+        int v = 0;
+#pragma unroll
+        for (int k = 0; k < kNodesPerLane; ++k) {
+            const int x = __shfl_sync(0xffffffffu, am[k], node & 31);
+            if ((node >> 5) == k) v = x;
+        }
+        return v;
     };
     if (__any_sync(0xffffffffu, tr.invalid)) {
         if (lane == 0) report(a.status, CLOVER_ERR_BAD_TREE);
@@ -305,50 +273,69 @@ __device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, co
         // at most T - 1 steps: every step moves to a larger node index
         for (int step = 1; step < Tn; ++step) {
             const int want = argmax_of(cur);
-            const unsigned lo = __ballot_sync(0xffffffffu, tr.p[0] == cur && tr.c[0] == want);
-            const unsigned hi = __ballot_sync(0xffffffffu, tr.p[1] == cur && tr.c[1] == want);
-            const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
-            if (hits == 0ull) break;
-            cur = __ffsll(static_cast<long long>(hits)) - 1;
+            bool hit[kNodesPerLane];
+#pragma unroll
+            for (int k = 0; k < kNodesPerLane; ++k) hit[k] = tr.p[k] == cur && tr.c[k] == want;
+            const int next = first_node(hit);
+            if (next < 0) break;
+            cur = next;
             if (lane == 0) path[len] = s_path[len] = cur;
             ++len;
         }
     } else {
-        uint64_t anc[2];
-        tree_masks_regs(tr.p, Tn, anc);
-        bool ok[2];
+        uint64_t anc[kNodesPerLane][kMaskWords];
+        tree_masks_jump<kNodesPerLane>(tr.p, Tn, anc);
+        uint64_t acc[kMaskWords];                 // accepted edges (node bits), the root included
 #pragma unroll
-        for (int k = 0; k < 2; ++k) {
+        for (int k = 0; k < kNodesPerLane; ++k) {
             const int i = lane + 32 * k;
-            ok[k] = false;
+            bool ok = false;
             if (i >= 1 && i < Tn) {
                 const float4 r = s_row[tr.p[k]];
-                ok[k] = fmaf(xc[k], a.y_scale, -r.x) - r.y > r.z;   // log2 p > log2 theta
+                ok = fmaf(xc[k], a.y_scale, -r.x) - r.y > r.z;   // log2 p > log2 theta
             }
+            const uint64_t bits = __ballot_sync(0xffffffffu, ok);
+            if ((k & 1) == 0) acc[k >> 1] = bits;
+            else acc[k >> 1] |= bits << 32;
         }
-        const uint64_t acc = (static_cast<uint64_t>(__ballot_sync(0xffffffffu, ok[1])) << 32) |
-                             __ballot_sync(0xffffffffu, ok[0]) | 1ull;
-        int depth[2];
+        acc[0] |= 1ull;
+        int depth[kNodesPerLane];
         unsigned dmax = 0;
 #pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            const bool reach = lane + 32 * k < Tn && (anc[k] & ~acc) == 0ull;
-            depth[k] = reach ? __popcll(anc[k]) - 1 : -1;
+        for (int k = 0; k < kNodesPerLane; ++k) {
+            bool reach = lane + 32 * k < Tn;
+            int pc = -1;
+#pragma unroll
+            for (int w = 0; w < kMaskWords; ++w) {
+                reach = reach && (anc[k][w] & ~acc[w]) == 0ull;
+                pc += __popcll(anc[k][w]);
+            }
+            depth[k] = reach ? pc : -1;
             dmax = max(dmax, (unsigned)max(depth[k], 0));
         }
         dmax = __reduce_max_sync(0xffffffffu, dmax);
-        uint64_t g = 0ull;
+        // G: the nodes on the root paths of the deepest accepted nodes
+        uint64_t g[kMaskWords] = {0ull, 0ull};
 #pragma unroll
-        for (int k = 0; k < 2; ++k)
-            if (depth[k] == (int)dmax) g |= anc[k];
-        g = (static_cast<uint64_t>(__reduce_or_sync(0xffffffffu, (unsigned)(g >> 32))) << 32) |
-            __reduce_or_sync(0xffffffffu, (unsigned)g);
+        for (int k = 0; k < kNodesPerLane; ++k)
+            if (depth[k] == (int)dmax) {
+#pragma unroll
+                for (int w = 0; w < kMaskWords; ++w) g[w] |= anc[k][w];
+            }
+#pragma unroll
+        for (int w = 0; w < kMaskWords; ++w)
+            g[w] = (static_cast<uint64_t>(__reduce_or_sync(0xffffffffu, (unsigned)(g[w] >> 32))) << 32) |
+                   __reduce_or_sync(0xffffffffu, (unsigned)g[w]);
         for (unsigned step = 0; step < dmax; ++step) {
-            const unsigned lo = __ballot_sync(0xffffffffu, tr.p[0] == cur && ((g >> lane) & 1ull));
-            const unsigned hi = __ballot_sync(0xffffffffu, tr.p[1] == cur && ((g >> (lane + 32)) & 1ull));
-            const uint64_t hits = (static_cast<uint64_t>(hi) << 32) | lo;
-            if (hits == 0ull) break;
-            cur = __ffsll(static_cast<long long>(hits)) - 1;
+            bool hit[kNodesPerLane];
+#pragma unroll
+            for (int k = 0; k < kNodesPerLane; ++k) {
+                const int i = lane + 32 * k;
+                hit[k] = tr.p[k] == cur && ((g[i >> 6] >> (i & 63)) & 1ull);
+            }
+            const int next = first_node(hit);
+            if (next < 0) break;
+            cur = next;
             if (lane == 0) path[len] = s_path[len] = cur;
             ++len;
         }
@@ -387,6 +374,21 @@ __device__ void commit_sequence(const AcceptArgs &a, int b, const int *s_path, i
     }
 }
 
+// The CTA that finished sequence b's last chunk: argmax of every node from the
+// merged row keys, then the walk, by warp 0 (the walk reads the current
+// node's argmax from registers by warp shuffles, so a step costs no memory
+// round trip).  The row keys and the counter are reset for the next call.
+//
+// Greedy: from the root, the smallest-index child whose candidate equals the
+// current node's argmax, until there is none.
+// Typical: first every thread of the CTA merges its share of one row's chunk
+// sums (4 or 2 threads a row) into the row's (max, log2 S, log2 theta), while
+// warp 0 also reads each child's candidate logit (gathered by the chunk CTAs).
+// Then warp 0 builds the ancestor masks in registers, decides every edge,
+// marks the nodes whose whole root path is accepted, takes the greatest depth
+// among them and the union G of the root paths of the accepted nodes at that
+// depth, and walks from the root through G, the smallest-index child at every
+// step.  With a commit, the whole CTA then writes the accepted K/V.
 template <typename T, bool TYPICAL>
 __device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) {
     __shared__ float4 s_row[kMaxTreeNodes];
@@ -395,11 +397,16 @@ __device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) 
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int Tn = a.T;
-    int am[2] = {0, 0};
-    float xc[2] = {-INFINITY, -INFINITY};
+    int am[kNodesPerLane];
+    float xc[kNodesPerLane];
+#pragma unroll
+    for (int k = 0; k < kNodesPerLane; ++k) {
+        am[k] = 0;
+        xc[k] = -INFINITY;
+    }
     if (warp == 0) {
 #pragma unroll
-        for (int k = 0; k < 2; ++k) {
+        for (int k = 0; k < kNodesPerLane; ++k) {
             const int i = lane + 32 * k;
             if (i < Tn) {
                 const unsigned long long key = __ldcg(a.row_key + (size_t)b * Tn + i);
@@ -411,18 +418,19 @@ __device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) 
         }
     }
     if (TYPICAL) {
-        const int row = threadIdx.x >> 2;
-        const int q = threadIdx.x & 3;
+        // tpr threads a row, neighbours in one warp
+        const int tpr = Tn <= 64 ? 4 : 2;
+        const int row = threadIdx.x / tpr;
+        const int q = threadIdx.x % tpr;
         float3 st = make_float3(-INFINITY, 0.f, 0.f);
         if (row < Tn) {
             const float4 *cs = a.chunk_sums + ((size_t)b * Tn + row) * a.n_chunks;
-            for (int k = q; k < a.n_chunks; k += 4) {
+            for (int k = q; k < a.n_chunks; k += tpr) {
                 const float4 v = __ldcg(cs + k);
                 st = merge_sums(st, make_float3(v.x, v.y, v.z));
             }
         }
-#pragma unroll
-        for (int off = 1; off < 4; off <<= 1) {
+        for (int off = 1; off < tpr; off <<= 1) {
             const float3 o = make_float3(__shfl_xor_sync(0xffffffffu, st.x, off), __shfl_xor_sync(0xffffffffu, st.y, off),
                                          __shfl_xor_sync(0xffffffffu, st.z, off));
             st = merge_sums(st, o);
@@ -509,7 +517,7 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
         // logits for the walk
         if (warp == 0) {
 #pragma unroll
-            for (int k = 0; k < 2; ++k) {
+            for (int k = 0; k < kNodesPerLane; ++k) {
                 const int i = threadIdx.x + 32 * k;
                 if (i >= 1 && i < a.T && tr.p[k] == node && tr.c[k] >= lo && tr.c[k] < hi) {
                     a.cand_x[(size_t)b * a.T + i] = to_float(rowp[tr.c[k]]);

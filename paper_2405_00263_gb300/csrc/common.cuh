@@ -9,7 +9,8 @@
 
 namespace clover {
 
-constexpr int kMaxTreeNodes = 64;   // one 64-bit ancestor mask per node
+constexpr int kMaxTreeNodes = 128;  // ancestor masks of two 64-bit words per node
+constexpr int kMaskWords = 2;
 
 // Everything clover_verify_attn's kernels need, already validated on the host.
 struct AttnArgs {
@@ -112,57 +113,99 @@ __device__ __forceinline__ float from_float<float>(float x) { return x; }
 template <>
 __device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(float x) { return __float2bfloat16_rn(x); }
 
-// Ancestor-or-self bitmask of every tree node, by pointer jumping, computed by
-// one warp: lane l owns nodes l and l + 32.  After round k each node's mask
-// covers its 2^k nearest ancestors; six rounds cover depth 63.  Invalid parent
-// arrays set *bad (masks are then only self bits and must not be trusted).
-__device__ __forceinline__ void tree_masks_warp(const int32_t *parent, int T, uint64_t *anc,
-                                                bool *bad) {
+// Ancestor-or-self bitmasks by pointer jumping in one warp's registers: lane l
+// owns nodes l + 32 k (k < NS, T <= 32 NS) with parents parent[k]; node n is
+// bit n & 63 of word n >> 6.  After round r a node's mask covers its 2^r
+// nearest ancestors, so log2(32 NS) rounds cover every depth.  The parents must
+// form a valid tree.
+template <int NS>
+__device__ __forceinline__ void tree_masks_jump(const int (&parent)[NS], int T, uint64_t (&m)[NS][kMaskWords]) {
     const int lane = threadIdx.x & 31;
-    uint64_t m[2];
-    int up[2];
+    int up[NS];
+#pragma unroll
+    for (int k = 0; k < NS; ++k) {
+        const int i = lane + 32 * k;
+#pragma unroll
+        for (int w = 0; w < kMaskWords; ++w) m[k][w] = (i < T && (i >> 6) == w) ? (1ull << (i & 63)) : 0ull;
+        up[k] = (i < T && i > 0) ? parent[k] : -1;
+    }
+    constexpr int kRounds = NS <= 2 ? 6 : 7;
+#pragma unroll 1
+    for (int round = 0; round < kRounds; ++round) {
+        uint64_t nm[NS][kMaskWords];
+        int nu[NS];
+#pragma unroll
+        for (int k = 0; k < NS; ++k) {
+            const int u = up[k] < 0 ? 0 : up[k];
+            // mask and pointer of node u: lane u & 31, slot u >> 5
+            uint64_t mu[kMaskWords] = {0ull, 0ull};
+            int uu = -1;
+#pragma unroll
+            for (int sl = 0; sl < NS; ++sl) {
+                const int us = __shfl_sync(0xffffffffu, up[sl], u & 31);
+#pragma unroll
+                for (int w = 0; w < kMaskWords; ++w) {
+                    const uint64_t ms = __shfl_sync(0xffffffffu, m[sl][w], u & 31);
+                    if ((u >> 5) == sl) mu[w] = ms;
+                }
+                if ((u >> 5) == sl) uu = us;
+            }
+#pragma unroll
+            for (int w = 0; w < kMaskWords; ++w) nm[k][w] = up[k] < 0 ? m[k][w] : (m[k][w] | mu[w]);
+            nu[k] = up[k] < 0 ? -1 : uu;
+        }
+#pragma unroll
+        for (int k = 0; k < NS; ++k) {
+#pragma unroll
+            for (int w = 0; w < kMaskWords; ++w) m[k][w] = nm[k][w];
+            up[k] = nu[k];
+        }
+    }
+}
+
+// Ancestor-or-self bitmask of every tree node into anc[node * kMaskWords + w],
+// computed by one warp from the parent array in global memory.  Invalid parent
+// arrays set *bad (masks are then only self bits and must not be trusted).
+template <int NS>
+__device__ __forceinline__ void tree_masks_warp_n(const int32_t *parent, int T, uint64_t *anc, bool *bad) {
+    const int lane = threadIdx.x & 31;
+    int p[NS];
     bool invalid = false;
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < NS; ++k) {
         const int i = lane + 32 * k;
-        int p = -1;
+        p[k] = -1;
         if (i < T) {
-            p = __ldg(parent + i);
-            if (i == 0 ? (p != -1) : (p < 0 || p >= i)) invalid = true;
+            p[k] = __ldg(parent + i);
+            if (i == 0 ? (p[k] != -1) : (p[k] < 0 || p[k] >= i)) invalid = true;
         }
-        if (i >= T || invalid) p = -1;
-        m[k] = (i < T) ? (1ull << i) : 0ull;
-        up[k] = p;
     }
     const bool any_bad = __any_sync(0xffffffffu, invalid);
-    if (!any_bad) {
+    uint64_t m[NS][kMaskWords];
+    if (any_bad) {
 #pragma unroll
-        for (int round = 0; round < 6; ++round) {
-            uint64_t nm[2];
-            int nu[2];
+        for (int k = 0; k < NS; ++k) {
+            const int i = lane + 32 * k;
 #pragma unroll
-            for (int k = 0; k < 2; ++k) {
-                const int u = up[k] < 0 ? 0 : up[k];
-                // fetch mask and pointer of node u (held by lane u & 31, slot u >> 5)
-                const uint64_t m0 = __shfl_sync(0xffffffffu, m[0], u & 31);
-                const uint64_t m1 = __shfl_sync(0xffffffffu, m[1], u & 31);
-                const int u0 = __shfl_sync(0xffffffffu, up[0], u & 31);
-                const int u1 = __shfl_sync(0xffffffffu, up[1], u & 31);
-                const uint64_t mu = (u >> 5) ? m1 : m0;
-                const int uu = (u >> 5) ? u1 : u0;
-                nm[k] = up[k] < 0 ? m[k] : (m[k] | mu);
-                nu[k] = up[k] < 0 ? -1 : uu;
-            }
+            for (int w = 0; w < kMaskWords; ++w) m[k][w] = (i < T && (i >> 6) == w) ? (1ull << (i & 63)) : 0ull;
+        }
+    } else {
+        tree_masks_jump<NS>(p, T, m);
+    }
 #pragma unroll
-            for (int k = 0; k < 2; ++k) {
-                m[k] = nm[k];
-                up[k] = nu[k];
-            }
+    for (int k = 0; k < NS; ++k) {
+        const int i = lane + 32 * k;
+        if (i < T) {
+#pragma unroll
+            for (int w = 0; w < kMaskWords; ++w) anc[i * kMaskWords + w] = m[k][w];
         }
     }
-    if (lane < T) anc[lane] = m[0];
-    if (lane + 32 < T) anc[lane + 32] = m[1];
     if (lane == 0) *bad = any_bad;
+}
+
+__device__ __forceinline__ void tree_masks_warp(const int32_t *parent, int T, uint64_t *anc, bool *bad) {
+    if (T <= 64) tree_masks_warp_n<2>(parent, T, anc, bad);
+    else tree_masks_warp_n<4>(parent, T, anc, bad);
 }
 
 // Raises a kernel's dynamic shared memory limit once per device.  Launchers

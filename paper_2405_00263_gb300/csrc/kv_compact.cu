@@ -25,38 +25,33 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
     const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index, int T, int Hkv,
     int row_bytes, int Lcap, int32_t *status) {
     extern __shared__ uint4 stage[];          // [2][T][row_bytes / 16]
-    __shared__ int s_src[kMaxTreeNodes];
+    __shared__ int s_src[kThreads];
     __shared__ int s_ok;
     const int g = blockIdx.x;
     const int b = blockIdx.y;
-    // the length, the accepted count and the whole path row are loaded at once
+    // the length, the accepted count and the whole path row are loaded at
+    // once, one path entry per thread (T <= kThreads)
+    static_assert(kMaxTreeNodes <= kThreads, "one path entry per thread");
     const int L = __ldg(cache_len + b);
     const int a = __ldg(accept_len + b);
-    if (threadIdx.x < 32) {
-        int p0 = -1, p1 = -1;
-        if (threadIdx.x < T) p0 = __ldg(path + (size_t)b * T + threadIdx.x);
-        if (threadIdx.x + 32 < T) p1 = __ldg(path + (size_t)b * T + threadIdx.x + 32);
-        const bool len_ok = (a >= 1 && a <= T);
-        const bool cap_ok = (L >= 0 && L + T <= Lcap);
-        const int j0 = threadIdx.x, j1 = threadIdx.x + 32;
-        const bool bad0 = j0 < a && (p0 < 0 || p0 >= T);
-        const bool bad1 = j1 < a && (p1 < 0 || p1 >= T);
-        const bool bad_path = __any_sync(0xffffffffu, bad0 || bad1);
-        s_src[j0] = bad0 ? j0 : p0;
-        s_src[j1] = bad1 ? j1 : p1;
-        if (threadIdx.x == 0) {
-            s_ok = len_ok && cap_ok;
-            if (g == 0 && !cap_ok) report(status, CLOVER_ERR_CAPACITY);
-            if (g == 0 && (!len_ok || bad_path)) report(status, CLOVER_ERR_INVALID_ARG);
+    const int jt = threadIdx.x;
+    const int p = jt < T ? __ldg(path + (size_t)b * T + jt) : -1;
+    const bool len_ok = (a >= 1 && a <= T);
+    const bool cap_ok = (L >= 0 && L + T <= Lcap);
+    const bool bad = jt < a && (p < 0 || p >= T);
+    s_src[jt] = bad ? jt : p;
+    const bool bad_path = __syncthreads_or(bad);
+    if (threadIdx.x == 0) {
+        s_ok = len_ok && cap_ok;
+        if (g == 0 && !cap_ok) report(status, CLOVER_ERR_CAPACITY);
+        if (g == 0 && (!len_ok || bad_path)) report(status, CLOVER_ERR_INVALID_ARG);
+    }
+    if (g == 0 && len_ok && cap_ok) {
+        if (src_index && jt < T) {
+            const int base = k_new ? 0 : L;         // a tree node (commit) or a cache slot
+            src_index[(size_t)b * T + jt] = (jt < a) ? base + s_src[jt] : -1;
         }
-        if (g == 0 && len_ok && cap_ok) {
-            if (src_index) {
-                const int base = k_new ? 0 : L;     // a tree node (commit) or a cache slot
-                if (j0 < T) src_index[(size_t)b * T + j0] = (j0 < a) ? base + s_src[j0] : -1;
-                if (j1 < T) src_index[(size_t)b * T + j1] = (j1 < a) ? base + s_src[j1] : -1;
-            }
-            if (threadIdx.x == 0) new_cache_len[b] = L + a;
-        }
+        if (threadIdx.x == 0) new_cache_len[b] = L + a;
     }
     __syncthreads();
     if (!s_ok) return;

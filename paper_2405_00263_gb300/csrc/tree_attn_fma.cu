@@ -54,7 +54,7 @@ __device__ __forceinline__ void chunk_coords(int j, int &key, int &col) {
 }
 
 // Global -> registers for one tile.  Cache tile: keys [base, base+kKT) of head g,
-// valid below `end`.  Tree tile (tree == true): nodes 0..T-1.
+// valid below `end`.  Tree tile (tree == true): nodes [base, base+kKT) below T.
 template <typename T, int D>
 __device__ __forceinline__ void load_tile(const AttnArgs &a, int b, int g, bool tree, int base,
                                           int end, TileRegs<T, D> &r) {
@@ -75,8 +75,8 @@ __device__ __forceinline__ void load_tile(const AttnArgs &a, int b, int g, bool 
                 r.k[j] = __ldg(reinterpret_cast<const uint4 *>(kc + off));
                 r.v[j] = __ldg(reinterpret_cast<const uint4 *>(vc + off));
             }
-        } else if (key < a.T) {
-            const size_t off = ((size_t)(b * a.T + key) * a.Hkv + g) * D + col;
+        } else if (base + key < a.T) {
+            const size_t off = ((size_t)(b * a.T + base + key) * a.Hkv + g) * D + col;
             r.k[j] = __ldg(reinterpret_cast<const uint4 *>(kn + off));
             r.v[j] = __ldg(reinterpret_cast<const uint4 *>(vn + off));
         }
@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
     float *sK = smem + S::k_off;
     float *sV = smem + S::v_off;
     float *sP = smem + S::p_off;
-    __shared__ uint64_t s_anc[kMaxTreeNodes];
+    __shared__ uint64_t s_anc[kMaxTreeNodes * kMaskWords];
     __shared__ bool s_bad;
     __shared__ int s_is_last;
 
@@ -139,7 +139,10 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
     const int kbeg = min(L, split * chunk);
     const int kend = min(L, kbeg + chunk);
     const int n_cache_tiles = (kend - kbeg + kKT - 1) / kKT;
-    const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
+    // the tree CTA ends with the tree keys, in tiles of kKT nodes
+    const int n_tiles = n_cache_tiles + (tree_cta ? (a.T + kKT - 1) / kKT : 0);
+    // first key (cache tile) or first node (tree tile) of tile t
+    auto tile_base = [&](int t) { return t < n_cache_tiles ? kbeg + t * kKT : (t - n_cache_tiles) * kKT; };
 
     // Q tile, pre-multiplied by scale*log2(e)
     {
@@ -184,11 +187,11 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
     }
 
     TileRegs<T, D> regs;
-    if (n_tiles > 0) load_tile<T, D>(a, b, g, n_cache_tiles == 0, kbeg, kend, regs);
+    if (n_tiles > 0) load_tile<T, D>(a, b, g, n_cache_tiles == 0, tile_base(0), kend, regs);
 
     for (int t = 0; t < n_tiles; ++t) {
-        const bool tree_tile = (t == n_cache_tiles);
-        const int base = kbeg + t * kKT;
+        const bool tree_tile = (t >= n_cache_tiles);
+        const int base = tile_base(t);
         // registers -> shared memory (and, for the tree tile, the cache append)
 #pragma unroll
         for (int j = 0; j < TileRegs<T, D>::kChunks; ++j) {
@@ -197,15 +200,15 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
             constexpr int per = TileRegs<T, D>::kPerChunk;
             unpack<T>(regs.k[j], sK + key * S::DQ + col);
             unpack<T>(regs.v[j], sV + key * D + col);
-            if (tree_tile && a.append && rt == 0 && !cap_bad && key < a.T) {
-                const size_t off = ((size_t)(b * a.Hkv + g) * a.Lcap + L + key) * D + col;
+            if (tree_tile && a.append && rt == 0 && !cap_bad && base + key < a.T) {
+                const size_t off = ((size_t)(b * a.Hkv + g) * a.Lcap + L + base + key) * D + col;
                 *reinterpret_cast<uint4 *>(static_cast<T *>(a.k_cache) + off) = regs.k[j];
                 *reinterpret_cast<uint4 *>(static_cast<T *>(a.v_cache) + off) = regs.v[j];
             }
             (void)per;
         }
         __syncthreads();
-        if (t + 1 < n_tiles) load_tile<T, D>(a, b, g, t + 1 == n_cache_tiles, base + kKT, kend, regs);
+        if (t + 1 < n_tiles) load_tile<T, D>(a, b, g, t + 1 >= n_cache_tiles, tile_base(t + 1), kend, regs);
 
         // scores s[r][j] for rows r0+r and keys kg + 16 j
         float s[2][4];
@@ -231,7 +234,10 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
             for (int j = 0; j < 4; ++j) {
                 const int kk = kg + 16 * j;
                 bool ok;
-                if (tree_tile) ok = (kk < a.T) && ((s_anc[node[r]] >> kk) & 1ull);
+                if (tree_tile) {
+                    const int n = base + kk;
+                    ok = (n < a.T) && ((s_anc[node[r] * kMaskWords + (n >> 6)] >> (n & 63)) & 1ull);
+                }
                 else ok = (base + kk < kend);
                 if (!ok) s[r][j] = -INFINITY;
             }

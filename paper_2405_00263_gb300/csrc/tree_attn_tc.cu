@@ -70,8 +70,8 @@ struct TcSmem {
     static constexpr int bar_off = v_off + NSV * kv_bytes;
     static constexpr int n_bars = 2 * NSK + 2 * NSV + 11;
     static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad flags
-    static constexpr int anc_off = misc_off + 16;                  // ancestor masks [64]
-    static constexpr int total = anc_off + kMaxTreeNodes * 8;
+    static constexpr int anc_off = misc_off + 16;                  // ancestor masks [128][2]
+    static constexpr int total = anc_off + kMaxTreeNodes * kMaskWords * 8;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
     // TMEM columns: S/P 2 x BN, O D, Q D / 2 (two bf16 per column), rounded up
     // to a power of two.  All 512 columns of an SM go to one CTA only when
@@ -486,14 +486,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int key0 = kbeg + (j - first_cache) * BN;
             const int n_valid = tree_tile ? a.T : min(BN, kend - key0);
             // Keys of a 64-key block of the tile that this row sees: a prefix
-            // of the cache keys, or the row's ancestors among the (at most 64)
-            // tree keys.  Every tile runs the same instructions, so the one
-            // tree tile, late in the loop, brings no code into the instruction
-            // cache (a miss then waits on a saturated memory system).
+            // of the cache keys, or the row's ancestors among the (at most
+            // 128) tree keys, word blk of its mask.  Every tile runs the same
+            // instructions, so the one tree tile, late in the loop, brings no
+            // code into the instruction cache (a miss then waits on a
+            // saturated memory system).
             auto block_vis = [&](int blk) -> uint64_t {
                 const int nv = n_valid - 64 * blk;
                 const uint64_t prefix = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
-                return tree_tile ? (blk == 0 ? s_anc[node] : 0ull) : prefix;
+                return tree_tile ? s_anc[node * kMaskWords + blk] : prefix;
             };
             // this thread's NB blocks of 64 keys start at block blk0 (KS = 2:
             // the key half; KS = 1: both halves, S re-read from TMEM per pass)

@@ -101,6 +101,11 @@ WORKLOADS = {
         "paper_t4_b48", B=48, T=4, Hq=32, Hkv=32, D=128, L=2560, V=125696, dtype="bf16",
         branching=(2, 1), plant_p=0.5, qkv_std=1 / math.sqrt(128), seed=7, L_range=(1536, 2560),
         description="paper regime: B48, L_b ~ U[1536,2560], 32 heads MHA, D128, 4-node tree, V125696, bf16"),
+    # a larger tree (the tree-size sweep of the paper's appendix), 7B MHA shapes
+    "7b_t128": Workload(
+        "7b_t128", B=1, T=128, Hq=32, Hkv=32, D=128, L=4096, V=125696, dtype="bf16",
+        branching=(8, 4, 2, 2, 2, 1), plant_p=0.5, qkv_std=1 / math.sqrt(128), seed=8,
+        description="7B-class, larger tree: B1, 32 heads MHA, D128, L4096, 128-node tree depth 6, V125696, bf16"),
     "100b_gqa": Workload(
         "100b_gqa", B=4, T=64, Hq=64, Hkv=8, D=128, L=8192, V=125696, dtype="bf16",
         branching=(8, 4, 2, 2, 1), plant_p=0.5, qkv_std=1 / math.sqrt(128), seed=4,

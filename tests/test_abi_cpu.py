@@ -50,7 +50,7 @@ def test_workspace_sizes(lib):
     big = ws(1, 64, 32, 32, 128, 4160, 0)                # fp32: CUDA-core split-KV merge
     assert big > 0 and big % 256 == 0
     assert ws(1, 64, 32, 32, 128, 4160, 1) == 0          # bf16: tensor-core path merges on chip
-    assert ws(1, 65, 8, 8, 64, 192, 0) == 0              # T > 64 unsupported
+    assert ws(1, 129, 8, 8, 64, 192, 0) == 0             # T > 128 unsupported
     assert ws(1, 16, 8, 8, 96, 192, 0) == 0              # D = 96 unsupported
     assert ws(1, 16, 6, 4, 64, 192, 0) == 0              # Hq not a multiple of Hkv
     acc = lib.clover_verify_accept_workspace_size
@@ -70,7 +70,7 @@ def _attn(lib, **kw):
 
 def test_attn_host_validation(lib):
     # every case below returns before any CUDA call
-    assert _attn(lib, T=65) == 2
+    assert _attn(lib, T=129) == 2
     assert _attn(lib, D=80) == 2
     assert _attn(lib, Hq=3, Hkv=2) == 2
     assert _attn(lib, T=0) == 1
@@ -88,7 +88,7 @@ def test_accept_and_compact_host_validation(lib):
     P = ctypes.c_void_p
     acc = lambda B, T, V, ws, wsb, lg=16: lib.clover_verify_accept(
         P(lg), P(16), P(16), B, T, V, 1, P(16), P(16), P(16), P(16), P(ws), wsb, None, None)
-    assert acc(1, 65, 10, 16, 1 << 20) == 2
+    assert acc(1, 129, 10, 16, 1 << 20) == 2
     assert acc(1, 4, 0, 16, 1 << 20) == 1
     assert acc(1, 4, 10, 16, 0) == 1                       # workspace too small
     assert acc(1, 4, 10, 16, 1 << 20, lg=17) == 1          # logits misaligned for bf16
@@ -98,7 +98,7 @@ def test_accept_and_compact_host_validation(lib):
     assert cmp(1024, 1024) == 1                            # new length aliases the old one
     assert cmp(1024, 1028) == 1                            # partial overlap
     assert cmp(1024, 2048, D=32) == 2
-    assert cmp(1024, 2048, T=65) == 2
+    assert cmp(1024, 2048, T=129) == 2
     assert cmp(1024, 2048, B=0) == 0
 
 
@@ -108,14 +108,14 @@ def test_attn_ex_and_commit_host_validation(lib):
         P(16), P(16), P(16), P(16), P(16), P(16), P(16), P(16), 1, T, 2, 2, 64, 64, 1, 0.0, None, 0, None, None,
         flags)
     assert ex(2) == 1 and ex(0xFFFFFFFE) == 1             # unknown flag bits
-    assert ex(1, T=65) == 2 and ex(0, T=65) == 2           # the limits of clover_verify_attn
+    assert ex(1, T=129) == 2 and ex(0, T=129) == 2           # the limits of clover_verify_attn
     com = lambda cl, ncl, kn=16, vn=16, B=2, T=4, D=64: lib.clover_kv_commit(
         P(16), P(16), P(kn), P(vn), P(cl), P(16), P(16), P(ncl), None, B, T, 2, D, 64, 1, None, None)
     assert com(1024, 1024) == 1                            # new length aliases the old one
     assert com(1024, 2048, kn=None) == 1                   # k_new missing
     assert com(1024, 2048, vn=24) == 1                     # v_new misaligned
     assert com(1024, 2048, D=32) == 2
-    assert com(1024, 2048, T=65) == 2
+    assert com(1024, 2048, T=129) == 2
     assert com(1024, 2048, B=0) == 0
 
 
@@ -128,7 +128,7 @@ def test_accept_typical_workspace_and_host_validation(lib):
     assert lib.clover_verify_accept_workspace_size(2, 4, 125696, 1) == 72
     assert need == 80 + 16 * 2 * 4 * 8 + 4 * 2 * 4
     assert lib.clover_verify_accept_typical_workspace_size(2, 4, 125696, 0) == 80 + 16 * 2 * 4 * 16 + 4 * 2 * 4
-    assert lib.clover_verify_accept_typical_workspace_size(2, 65, 100, 1) == 0
+    assert lib.clover_verify_accept_typical_workspace_size(2, 129, 100, 1) == 0
     call = lambda tau=1.0, eps=0.09, delta=0.3, ws=4096, wsb=need, B=2, T=4, V=125696: \
         lib.clover_verify_accept_typical(P(64), P(64), P(64), B, T, V, 1, tau, eps, delta, P(64), P(64), P(64),
                                          P(64), P(ws), wsb, None, None)
@@ -137,7 +137,7 @@ def test_accept_typical_workspace_and_host_validation(lib):
                 dict(ws=0)):
         assert call(**bad) == 1, bad
     assert call(tau=1e-300) == 2 and call(tau=1e39) == 2     # log2(e)/tau not a normal fp32 number
-    assert call(T=65) == 2
+    assert call(T=129) == 2
     assert call(B=0) == 0
 
 
@@ -159,7 +159,7 @@ def test_accept_ex_host_validation(lib):
     assert call(2, D=96) == 2                                # commit: D not 64/128
     assert call(2, ncl=2048) == 1                            # commit: new length aliases the old one
     assert call(1, ws=4104) == 1                             # typical: workspace 16-byte aligned
-    assert call(7, T=65) == 2
+    assert call(7, T=129) == 2
     assert call(7, B=0) == 0
 
 

@@ -27,6 +27,13 @@ SMALL = {
     "bf16_ragged_batch": ("7b_batched", dict(B=5, Hq=8, Hkv=8, L_range=(0, 700), V=3001)),
     "bf16_sharp_scores": ("7b_l2048", dict(T=64, Hq=4, Hkv=2, L=900, V=2048, qkv_std=1.5)),
     "bf16_gqa8_T64": ("100b_gqa", dict(B=1, Hq=16, Hkv=2, L=640, V=2048)),
+    # trees past 64 nodes: two mask words, two FMA tree tiles, four nodes per lane in the walk
+    "bf16_T128_topk": ("7b_l2048", dict(T=128, Hq=4, Hkv=4, L=700, V=3000, branching=(8, 4, 2, 2, 2, 1))),
+    "bf16_T128_chain": ("7b_l2048", dict(T=128, Hq=2, Hkv=2, L=300, V=2048, tree="chain", plant_p=1.0)),
+    "bf16_T100_random_gqa": ("100b_gqa", dict(B=2, T=100, Hq=16, Hkv=2, L=450, V=4099, tree="random")),
+    "bf16_T65_d64": ("7b_l2048", dict(B=2, T=65, Hq=8, Hkv=8, D=64, L=333, V=2048, tree="random")),
+    "f32_T100_random": ("tiny_f32", dict(B=2, T=100, Hq=4, Hkv=2, L=260, V=5003, tree="random")),
+    "f32_T128_d128": ("tiny_f32", dict(T=128, D=128, Hq=2, Hkv=2, L=500, V=1024, branching=(8, 4, 2, 2, 2, 1))),
 }
 
 
@@ -65,7 +72,8 @@ def test_repeated_calls_reuse_workspace(cuda):
     compare_full(host, step, t2)
 
 
-FULL = ["7b_l2048", "7b_l4096", "7b_l16384", "7b_batched", "100b_gqa", "paper_t4_b4", "paper_t4_b16", "paper_t4_b48"]
+FULL = ["7b_l2048", "7b_l4096", "7b_l16384", "7b_batched", "100b_gqa", "paper_t4_b4", "paper_t4_b16", "paper_t4_b48",
+        "7b_t128"]
 
 
 @pytest.mark.parametrize("schedule", ["commit", "fused"])

@@ -110,6 +110,8 @@ CASES = [
     (1, 64, 1, torch.float32, "topk", (1.0, 0.09, 0.3)),           # V = 1: p = 1, H = 0
     (2, 24, 4099, torch.float32, "random", (1.0, 0.0, 0.3)),       # eps = 0: theta = 0
     (2, 24, 4099, torch.bfloat16, "random", (1.0, 0.3, 0.0)),      # delta = 0: theta = 0
+    (2, 128, 20000, torch.bfloat16, "random", (1.0, 0.09, 0.3)),   # two mask words, two threads a row
+    (1, 100, 9000, torch.float32, "topk", (0.8, 0.2, 0.5)),
 ]
 
 
@@ -143,7 +145,7 @@ def test_typical_neg_inf_logits_and_out_of_range_candidates():
         assert_same(run_typical(logits, parent, cd, tau, eps, delta), ref)
 
 
-@pytest.mark.parametrize("name", ["paper_t4_b16", "7b_l4096", "100b_gqa"])
+@pytest.mark.parametrize("name", ["paper_t4_b16", "7b_l4096", "100b_gqa", "7b_t128"])
 def test_typical_full_size_workloads(name):
     w = workloads.get(name)
     t = workloads.make(w)
