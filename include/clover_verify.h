@@ -19,7 +19,9 @@
  *                         either rule, optionally fused with the commit of the
  *                         accepted K/V and launched to overlap the attention;
  *   clover_kv_compact     moves the accepted nodes' K/V to the front of the
- *                         tree slots (an engine step the paper leaves implicit).
+ *                         tree slots (an engine step the paper leaves implicit);
+ *   clover_verify_attn_paged, clover_kv_commit_paged
+ *                         the attention and the commit on a paged KV cache.
  *
  * A second schedule of the same step: clover_verify_attn_ex with
  * CLOVER_ATTN_NO_APPEND leaves the caches untouched, and clover_kv_commit then
@@ -144,6 +146,52 @@ CLOVER_API clover_status clover_verify_attn_ex(const void *q, const void *k_new,
                                     clover_dtype dtype, float scale,
                                     void *workspace, size_t ws_bytes,
                                     int32_t *status, void *stream, uint32_t flags);
+
+/*
+ * Paged KV cache (an engine's block-table layout; the paper leaves the cache
+ * layout implicit).  The pools k_pages, v_pages are [n_pages, Hkv, page_size, D]
+ * (dtype, 16-byte aligned); block_table [B, max_pages] int32 maps cache slot s
+ * of sequence b to row s % page_size of page block_table[b][s / page_size].
+ * page_size is a power of two in [16, 1024]; the cache capacity is
+ * Lcap = page_size * max_pages slots.  Entries for slots < cache_len[b] (and,
+ * for the commit, < cache_len[b] + accept_len[b]) must be page ids in
+ * [0, n_pages); another id found on the device raises CLOVER_ERR_INVALID_ARG
+ * (device bit) and the access goes to page 0 (results unspecified).  Entries
+ * past those are not read.
+ */
+
+/* Bytes of device workspace clover_verify_attn_paged needs (0 outside the limits). */
+CLOVER_API size_t clover_verify_attn_paged_workspace_size(int B, int T, int Hq, int Hkv, int D, int page_size,
+                                                          int max_pages, clover_dtype dtype);
+
+/*
+ * Tree-masked attention over a paged cache: clover_verify_attn_ex with
+ * CLOVER_ATTN_NO_APPEND on the cache the block table describes (the pools are
+ * only read; commit the accepted K/V with clover_kv_commit_paged).  Same
+ * arguments, limits and results, with Lcap = page_size * max_pages; bf16 runs
+ * on the tensor-core kernel (a 128-key tile is read as 128 / page_size boxes
+ * when pages are smaller), fp32 on the FMA kernel.
+ */
+CLOVER_API clover_status clover_verify_attn_paged(const void *q, const void *k_new, const void *v_new,
+                                   const void *k_pages, const void *v_pages, const int32_t *block_table,
+                                   int n_pages, int page_size, int max_pages,
+                                   const int32_t *cache_len, const int32_t *parent, void *out,
+                                   int B, int T, int Hq, int Hkv, int D, clover_dtype dtype, float scale,
+                                   void *workspace, size_t ws_bytes, int32_t *status, void *stream);
+
+/*
+ * clover_kv_commit into a paged cache: for every sequence b with L = cache_len[b]
+ * and a = accept_len[b], slot L+j (its page from block_table) of every KV head
+ * receives k_new/v_new of node path[j]; src_index_out[b][j] = path[j] (-1 past
+ * a; may be NULL); new_cache_len[b] = L + a.  Errors as for clover_kv_commit,
+ * with Lcap = page_size * max_pages.
+ */
+CLOVER_API clover_status clover_kv_commit_paged(void *k_pages, void *v_pages, const int32_t *block_table,
+                                   int n_pages, int page_size, int max_pages,
+                                   const void *k_new, const void *v_new, const int32_t *cache_len,
+                                   const int32_t *path, const int32_t *accept_len, int32_t *new_cache_len,
+                                   int32_t *src_index_out, int B, int T, int Hkv, int D, clover_dtype dtype,
+                                   int32_t *status, void *stream);
 
 /* Bytes of device workspace clover_verify_accept needs (0 outside the limits). */
 CLOVER_API size_t clover_verify_accept_workspace_size(int B, int T, int V, clover_dtype dtype);

@@ -32,6 +32,9 @@ EXPORTS = (
     "clover_kv_compact",
     "clover_kv_commit",
     "clover_verify_attn_noalloc",
+    "clover_verify_attn_paged_workspace_size",
+    "clover_verify_attn_paged",
+    "clover_kv_commit_paged",
 )
 
 # Flag of clover_verify_attn_ex (CLOVER_ATTN_NO_APPEND in include/clover_verify.h).
@@ -98,5 +101,12 @@ def load(build_if_missing: bool = False):
         lib.clover_kv_commit.restype = I
         lib.clover_verify_attn_noalloc.argtypes = [P, P, P, P, P, P, P, P, I, I, I, I, I, I, I, F, P, P]
         lib.clover_verify_attn_noalloc.restype = I
+        lib.clover_verify_attn_paged_workspace_size.argtypes = [I, I, I, I, I, I, I, I]
+        lib.clover_verify_attn_paged_workspace_size.restype = Z
+        lib.clover_verify_attn_paged.argtypes = [P, P, P, P, P, P, I, I, I, P, P, P, I, I, I, I, I, I, F, P, Z,
+                                                 P, P]
+        lib.clover_verify_attn_paged.restype = I
+        lib.clover_kv_commit_paged.argtypes = [P, P, P, I, I, I, P, P, P, P, P, P, P, I, I, I, I, I, P, P]
+        lib.clover_kv_commit_paged.restype = I
         _lib = lib
         return lib

@@ -216,6 +216,69 @@ def clover_kv_compact(k_cache, v_cache, cache_len, path, accept_len, new_cache_l
         raise CloverError(code, "clover_kv_compact")
 
 
+def clover_verify_attn_paged_workspace_size(B, T, Hq, Hkv, D, page_size, max_pages, dtype) -> int:
+    code = dtype if isinstance(dtype, int) else dtype_code(dtype)
+    return int(_lib.load().clover_verify_attn_paged_workspace_size(B, T, Hq, Hkv, D, page_size, max_pages, code))
+
+
+def clover_verify_attn_paged(q, k_new, v_new, k_pages, v_pages, block_table, cache_len, parent, out, scale=0.0,
+                             workspace=None, status=None, stream=None):
+    """Tree-masked attention over a paged cache: pools [n_pages, Hkv, page_size, D],
+    block_table [B, max_pages] (the pools are only read)."""
+    B, T, Hq, D = q.shape
+    n_pages, Hkv, page_size = k_pages.shape[0], k_pages.shape[1], k_pages.shape[2]
+    max_pages = block_table.shape[1]
+    dt = q.dtype
+    _check(k_new, (B, T, Hkv, D), dt, "k_new")
+    _check(v_new, (B, T, Hkv, D), dt, "v_new")
+    _check(k_pages, (n_pages, Hkv, page_size, D), dt, "k_pages")
+    _check(v_pages, (n_pages, Hkv, page_size, D), dt, "v_pages")
+    _check(block_table, (B, max_pages), torch.int32, "block_table")
+    _check(cache_len, (B,), torch.int32, "cache_len")
+    _check(parent, (B, T), torch.int32, "parent")
+    _check(out, (B, T, Hq, D), dt, "out")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(q, k_new, v_new, k_pages, v_pages, block_table, cache_len, parent, out, workspace, status)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    code = _lib.load().clover_verify_attn_paged(
+        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_pages), _ptr(v_pages), _ptr(block_table), n_pages, page_size,
+        max_pages, _ptr(cache_len), _ptr(parent), _ptr(out), B, T, Hq, Hkv, D, dtype_code(dt), float(scale),
+        _ptr(workspace), ws_bytes, _ptr(status), _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_verify_attn_paged")
+
+
+def clover_kv_commit_paged(k_pages, v_pages, block_table, k_new, v_new, cache_len, path, accept_len, new_cache_len,
+                           src_index_out=None, status=None, stream=None):
+    """clover_kv_commit into a paged cache (slot L+j of sequence b: page
+    block_table[b][(L+j) // page_size], row (L+j) % page_size)."""
+    n_pages, Hkv, page_size, D = k_pages.shape
+    B, max_pages = block_table.shape
+    T = path.shape[1]
+    dt = k_pages.dtype
+    _check(v_pages, (n_pages, Hkv, page_size, D), dt, "v_pages")
+    _check(k_new, (B, T, Hkv, D), dt, "k_new")
+    _check(v_new, (B, T, Hkv, D), dt, "v_new")
+    _check(block_table, (B, max_pages), torch.int32, "block_table")
+    _check(cache_len, (B,), torch.int32, "cache_len")
+    _check(path, (B, T), torch.int32, "path")
+    _check(accept_len, (B,), torch.int32, "accept_len")
+    _check(new_cache_len, (B,), torch.int32, "new_cache_len")
+    if src_index_out is not None:
+        _check(src_index_out, (B, T), torch.int32, "src_index_out")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(k_pages, v_pages, block_table, k_new, v_new, cache_len, path, accept_len, new_cache_len, src_index_out,
+         status)
+    code = _lib.load().clover_kv_commit_paged(
+        _ptr(k_pages), _ptr(v_pages), _ptr(block_table), n_pages, page_size, max_pages, _ptr(k_new), _ptr(v_new),
+        _ptr(cache_len), _ptr(path), _ptr(accept_len), _ptr(new_cache_len), _ptr(src_index_out), B, T, Hkv, D,
+        dtype_code(dt), _ptr(status), _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_kv_commit_paged")
+
+
 def clover_kv_commit(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len, new_cache_len,
                      src_index_out=None, status=None, stream=None):
     """Writes the accepted nodes' K/V from k_new/v_new to slots [L, L+a);

@@ -19,7 +19,8 @@ cudaError_t launch_accept_call(const AcceptCall &c, cudaStream_t stream);
 cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
                               const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
                               int32_t *new_cache_len, int32_t *src_index, int B, int T, int Hkv, int D, int Lcap,
-                              int dtype, int32_t *status, cudaStream_t stream);
+                              int dtype, int32_t *status, cudaStream_t stream, const int32_t *block_table = nullptr,
+                              int page_size = 0, int max_pages = 0, int n_pages = 0);
 
 namespace {
 
@@ -173,6 +174,71 @@ clover_status check_accept(AcceptCall &c, const void *logits, const int32_t *can
     return CLOVER_OK;
 }
 
+// Logical capacity of a paged cache (page_size * max_pages slots), or -1 when
+// the page size is not a power of two in [16, 1024] or the product overflows.
+long paged_capacity(int page_size, int max_pages) {
+    if (page_size < 16 || page_size > 1024 || (page_size & (page_size - 1)) || max_pages < 1) return -1;
+    const long c = (long)page_size * max_pages;
+    return c > 0x3FFFFFFFL ? -1 : c;
+}
+
+// The attention call after the size checks (B > 0): pointer checks, the
+// launch plan and the kernel.  block_table != nullptr: paged cache.
+clover_status run_attn(const void *q, const void *k_new, const void *v_new, void *k_cache, void *v_cache,
+                       const int32_t *cache_len, const int32_t *parent, void *out, int B, int T, int Hq, int Hkv,
+                       int D, int Lcap, clover_dtype dtype, float scale, void *workspace, size_t ws_bytes,
+                       int32_t *status, void *stream, bool append, const int32_t *block_table, int page_size,
+                       int max_pages, int n_pages) {
+    if (!q || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !parent || !out)
+        return CLOVER_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache) ||
+        !aligned16(out))
+        return CLOVER_ERR_INVALID_ARG;
+    if (!(scale == scale) || isinf(scale)) return CLOVER_ERR_INVALID_ARG;
+    const AttnPlan p = plan_attn(B, T, Hq, Hkv, D, Lcap, dtype);
+    if (ws_bytes < p.total || (p.total > 0 && (!workspace || !aligned16(workspace)))) return CLOVER_ERR_INVALID_ARG;
+
+    AttnArgs a{};
+    a.q = q;
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_len = cache_len;
+    a.parent = parent;
+    a.out = out;
+    a.B = B;
+    a.T = T;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.D = D;
+    a.Lcap = Lcap;
+    a.G = Hq / Hkv;
+    a.dtype = dtype;
+    const float sc = scale > 0.f ? scale : 1.f / sqrtf((float)D);
+    a.scale_log2 = sc * 1.4426950408889634f;
+    a.append = append ? 1 : 0;
+    a.block_table = block_table;
+    if (block_table) {
+        a.page_size = page_size;
+        while ((1 << a.page_shift) < page_size) ++a.page_shift;
+        a.max_pages = max_pages;
+        a.n_pages = n_pages;
+    }
+    a.rows = T * a.G;
+    a.row_tile = p.row_tile;
+    a.row_tiles = p.row_tiles;
+    a.n_split = p.n_split;
+    a.slot_rows = p.slot_rows;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    a.part_o = p.total ? reinterpret_cast<float *>(ws) : nullptr;
+    a.part_ml = p.total ? reinterpret_cast<float *>(ws + p.o_bytes) : nullptr;
+    a.counters = p.total ? reinterpret_cast<unsigned *>(ws + p.o_bytes + p.ml_bytes) : nullptr;
+    a.status = status;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    return from_cuda(p.tc ? launch_tree_attn_tc(a, st) : launch_tree_attn_fma(a, st));
+}
+
 }  // namespace
 
 extern "C" {
@@ -216,47 +282,32 @@ clover_status clover_verify_attn_ex(const void *q, const void *k_new, const void
     const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype);
     if (s != CLOVER_OK) return s;
     if (B == 0) return CLOVER_OK;
-    if (!q || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !parent || !out)
-        return CLOVER_ERR_INVALID_ARG;
-    if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache) ||
-        !aligned16(out))
-        return CLOVER_ERR_INVALID_ARG;
-    if (!(scale == scale) || isinf(scale)) return CLOVER_ERR_INVALID_ARG;
-    const AttnPlan p = plan_attn(B, T, Hq, Hkv, D, Lcap, dtype);
-    if (ws_bytes < p.total || (p.total > 0 && (!workspace || !aligned16(workspace)))) return CLOVER_ERR_INVALID_ARG;
+    return run_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, B, T, Hq, Hkv, D, Lcap, dtype, scale,
+                    workspace, ws_bytes, status, stream, (flags & CLOVER_ATTN_NO_APPEND) == 0, nullptr, 0, 0, 0);
+}
 
-    AttnArgs a;
-    a.q = q;
-    a.k_new = k_new;
-    a.v_new = v_new;
-    a.k_cache = k_cache;
-    a.v_cache = v_cache;
-    a.cache_len = cache_len;
-    a.parent = parent;
-    a.out = out;
-    a.B = B;
-    a.T = T;
-    a.Hq = Hq;
-    a.Hkv = Hkv;
-    a.D = D;
-    a.Lcap = Lcap;
-    a.G = Hq / Hkv;
-    a.dtype = dtype;
-    const float sc = scale > 0.f ? scale : 1.f / sqrtf((float)D);
-    a.scale_log2 = sc * 1.4426950408889634f;
-    a.append = (flags & CLOVER_ATTN_NO_APPEND) ? 0 : 1;
-    a.rows = T * a.G;
-    a.row_tile = p.row_tile;
-    a.row_tiles = p.row_tiles;
-    a.n_split = p.n_split;
-    a.slot_rows = p.slot_rows;
-    uint8_t *ws = static_cast<uint8_t *>(workspace);
-    a.part_o = p.total ? reinterpret_cast<float *>(ws) : nullptr;
-    a.part_ml = p.total ? reinterpret_cast<float *>(ws + p.o_bytes) : nullptr;
-    a.counters = p.total ? reinterpret_cast<unsigned *>(ws + p.o_bytes + p.ml_bytes) : nullptr;
-    a.status = status;
-    const cudaStream_t st = static_cast<cudaStream_t>(stream);
-    return from_cuda(p.tc ? launch_tree_attn_tc(a, st) : launch_tree_attn_fma(a, st));
+size_t clover_verify_attn_paged_workspace_size(int B, int T, int Hq, int Hkv, int D, int page_size, int max_pages,
+                                               clover_dtype dtype) {
+    const long lcap = paged_capacity(page_size, max_pages);
+    if (lcap < 0) return 0;
+    return clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, (int)lcap, dtype);
+}
+
+clover_status clover_verify_attn_paged(const void *q, const void *k_new, const void *v_new, const void *k_pages,
+                                       const void *v_pages, const int32_t *block_table, int n_pages, int page_size,
+                                       int max_pages, const int32_t *cache_len, const int32_t *parent, void *out,
+                                       int B, int T, int Hq, int Hkv, int D, clover_dtype dtype, float scale,
+                                       void *workspace, size_t ws_bytes, int32_t *status, void *stream) {
+    const long lcap = paged_capacity(page_size, max_pages);
+    if (lcap < 0 || n_pages < 1) return CLOVER_ERR_INVALID_ARG;
+    const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, (int)lcap, dtype);
+    if (s != CLOVER_OK) return s;
+    if ((long)n_pages * Hkv * page_size > 0x7FFFFFFFL) return CLOVER_ERR_UNSUPPORTED;
+    if (B == 0) return CLOVER_OK;
+    if (!block_table) return CLOVER_ERR_INVALID_ARG;
+    return run_attn(q, k_new, v_new, const_cast<void *>(k_pages), const_cast<void *>(v_pages), cache_len, parent, out,
+                    B, T, Hq, Hkv, D, (int)lcap, dtype, scale, workspace, ws_bytes, status, stream, false, block_table,
+                    page_size, max_pages, n_pages);
 }
 
 size_t clover_verify_accept_workspace_size(int B, int T, int V, clover_dtype dtype) {
@@ -347,6 +398,23 @@ clover_status clover_kv_commit(void *k_cache, void *v_cache, const void *k_new, 
     return from_cuda(launch_kv_compact(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len, new_cache_len,
                                        src_index_out, B, T, Hkv, D, Lcap, dtype, status,
                                        static_cast<cudaStream_t>(stream)));
+}
+
+clover_status clover_kv_commit_paged(void *k_pages, void *v_pages, const int32_t *block_table, int n_pages,
+                                     int page_size, int max_pages, const void *k_new, const void *v_new,
+                                     const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
+                                     int32_t *new_cache_len, int32_t *src_index_out, int B, int T, int Hkv, int D,
+                                     clover_dtype dtype, int32_t *status, void *stream) {
+    const long lcap = paged_capacity(page_size, max_pages);
+    if (lcap < 0 || n_pages < 1) return CLOVER_ERR_INVALID_ARG;
+    const clover_status s = check_commit(k_pages, v_pages, k_new, v_new, cache_len, path, accept_len, new_cache_len,
+                                         B, T, Hkv, D, (int)lcap, dtype, true);
+    if (s != CLOVER_OK || B == 0) return s;
+    if ((long)n_pages * Hkv * page_size > 0x7FFFFFFFL) return CLOVER_ERR_UNSUPPORTED;
+    if (!block_table) return CLOVER_ERR_INVALID_ARG;
+    return from_cuda(launch_kv_compact(k_pages, v_pages, k_new, v_new, cache_len, path, accept_len, new_cache_len,
+                                       src_index_out, B, T, Hkv, D, (int)lcap, dtype, status,
+                                       static_cast<cudaStream_t>(stream), block_table, page_size, max_pages, n_pages));
 }
 
 clover_status clover_kv_compact(void *k_cache, void *v_cache, const int32_t *cache_len, const int32_t *path,

@@ -27,6 +27,11 @@ struct AttnArgs {
     int n_split;           // cache key ranges per (sequence, KV head, row tile)
     int slot_rows;         // rows of one partial-result slot (<= row_tile)
     int append;            // write k_new/v_new to cache slots [L, L+T) (0: the caches are only read)
+    // paged cache (block_table != nullptr): k_cache/v_cache are page pools
+    // [n_pages, Hkv, page_size, D]; slot s of sequence b is row s % page_size
+    // of page block_table[b * max_pages + s / page_size]; Lcap = page_size * max_pages
+    const int32_t *block_table;
+    int page_size, page_shift, max_pages, n_pages;
     float *part_o;         // [B, Hkv, row_tiles, n_split, slot_rows, D]
     float *part_ml;        // [B, Hkv, row_tiles, n_split, slot_rows, 2]  (max, sum)
     unsigned *counters;    // [B, Hkv, row_tiles]
@@ -70,6 +75,18 @@ __device__ __forceinline__ void wait_prerequisite_grids() {
 
 __device__ __forceinline__ void report(int32_t *status, int bits) {
     if (status) atomicOr(status, bits);
+}
+
+// Page of cache slot `slot` (< cache_len) of sequence b in a paged cache; an
+// id outside [0, n_pages) is reported and replaced by page 0, so that every
+// access stays inside the pool (the result is then unspecified).
+__device__ __forceinline__ int cache_page(const AttnArgs &a, int b, int slot) {
+    const int p = __ldg(a.block_table + (size_t)b * a.max_pages + (slot >> a.page_shift));
+    if (p < 0 || p >= a.n_pages) {
+        report(a.status, CLOVER_ERR_INVALID_ARG);
+        return 0;
+    }
+    return p;
 }
 
 __device__ __forceinline__ float bf16_bits_to_float(uint16_t h) {

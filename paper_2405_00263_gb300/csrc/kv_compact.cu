@@ -6,7 +6,8 @@
 //               that of copying in increasing j, which equals a gather
 //               because path[j] >= j;
 //   commit      the rows come straight from k_new/v_new [B, T, Hkv, D] (no
-//               append before it).
+//               append before it), into a dense cache or a paged one (slot
+//               L + j is row (L + j) % page of page block_table[b][(L + j) / page]).
 //
 // One CTA per (KV head, sequence) stages the a accepted rows of K and V in
 // shared memory and only then writes them, so a row that is both a source and
@@ -23,9 +24,11 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
     uint8_t *k_cache, uint8_t *v_cache, const uint8_t *k_new, const uint8_t *v_new, const int32_t *cache_len,
     const int32_t *path,
     const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index, int T, int Hkv,
-    int row_bytes, int Lcap, int32_t *status) {
+    int row_bytes, int Lcap, const int32_t *block_table, int page_size, int page_shift, int max_pages,
+    int n_pages, int32_t *status) {
     extern __shared__ uint4 stage[];          // [2][T][row_bytes / 16]
     __shared__ int s_src[kThreads];
+    __shared__ int s_dst_page[kThreads];      // paged cache: page of slot L + j (-1: invalid id, skipped)
     __shared__ int s_ok;
     const int g = blockIdx.x;
     const int b = blockIdx.y;
@@ -40,7 +43,13 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
     const bool cap_ok = (L >= 0 && L + T <= Lcap);
     const bool bad = jt < a && (p < 0 || p >= T);
     s_src[jt] = bad ? jt : p;
-    const bool bad_path = __syncthreads_or(bad);
+    bool bad_page = false;
+    if (block_table && jt < a && a <= T && L >= 0 && L + T <= Lcap) {
+        const int pg = __ldg(block_table + (size_t)b * max_pages + ((L + jt) >> page_shift));
+        bad_page = pg < 0 || pg >= n_pages;
+        s_dst_page[jt] = bad_page ? -1 : pg;
+    }
+    const bool bad_path = __syncthreads_or(bad || bad_page);
     if (threadIdx.x == 0) {
         s_ok = len_ok && cap_ok;
         if (g == 0 && !cap_ok) report(status, CLOVER_ERR_CAPACITY);
@@ -73,7 +82,11 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
     for (int e = threadIdx.x; e < a * units; e += kThreads) {
         const int j = e / units;
         const int u = e % units;
-        const size_t dst = (head_base + L + j) * units + u;
+        size_t dst = (head_base + L + j) * units + u;
+        if (block_table) {
+            if (s_dst_page[j] < 0) continue;
+            dst = (((size_t)s_dst_page[j] * Hkv + g) * page_size + ((L + j) & (page_size - 1))) * units + u;
+        }
         kd[dst] = stage[e];
         vd[dst] = stage[T * units + e];
     }
@@ -84,7 +97,10 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
 cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
                               const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
                               int32_t *new_cache_len, int32_t *src_index, int B, int T, int Hkv, int D, int Lcap,
-                              int dtype, int32_t *status, cudaStream_t stream) {
+                              int dtype, int32_t *status, cudaStream_t stream, const int32_t *block_table,
+                              int page_size, int max_pages, int n_pages) {
+    int page_shift = 0;
+    while (block_table && (1 << page_shift) < page_size) ++page_shift;
     const int row_bytes = D * (dtype == CLOVER_F32 ? 4 : 2);
     const size_t smem = (size_t)2 * T * row_bytes;
     static unsigned char done[64];
@@ -96,7 +112,8 @@ cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, c
                                                         static_cast<const uint8_t *>(k_new),
                                                         static_cast<const uint8_t *>(v_new), cache_len, path,
                                                         accept_len, new_cache_len, src_index, T, Hkv,
-                                                        row_bytes, Lcap, status);
+                                                        row_bytes, Lcap, block_table, page_size, page_shift,
+                                                        max_pages, n_pages, status);
     return cudaGetLastError();
 }
 

@@ -71,7 +71,13 @@ __device__ __forceinline__ void load_tile(const AttnArgs &a, int b, int g, bool 
         if (!tree) {
             const int slot = base + key;
             if (slot < end) {
-                const size_t off = ((size_t)(b * a.Hkv + g) * a.Lcap + slot) * D + col;
+                // dense: plane (b, g) of the cache; paged: row slot % page of
+                // plane (page, g) of the pool
+                const size_t row = a.block_table
+                                       ? ((size_t)cache_page(a, b, slot) * a.Hkv + g) * a.page_size +
+                                             (slot & (a.page_size - 1))
+                                       : (size_t)(b * a.Hkv + g) * a.Lcap + slot;
+                const size_t off = row * D + col;
                 r.k[j] = __ldg(reinterpret_cast<const uint4 *>(kc + off));
                 r.v[j] = __ldg(reinterpret_cast<const uint4 *>(vc + off));
             }

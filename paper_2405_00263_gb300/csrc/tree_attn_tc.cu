@@ -46,6 +46,8 @@ using namespace tc;
 
 constexpr int BM = 128;                 // query rows per CTA (MMA M)
 constexpr int BN = 128;                 // keys per tile (the N of the S MMA)
+constexpr int kMinPage = 16;             // smallest page of a paged cache (rows)
+constexpr int kMaxBoxes = BN / kMinPage; // TMA boxes of one paged cache tile
 constexpr int kKProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kVProducerWarp = 6;
@@ -226,12 +228,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     // this CTA appends the tree K/V to cache slots [L, L+T)
     const bool appender = a.append && tree_cta && rt == 0 && !cap_bad;
 
+    // Paged cache: a cache tile is read as boxes of `box` rows, each inside one
+    // page (box = min(page size, BN); tiles start at multiples of BN).  The
+    // page ids of tile j, looked up before the producer waits for the stage.
+    const bool paged = a.block_table != nullptr;
+    const int box = paged ? min(a.page_size, BN) : BN;
+    auto tile_pages = [&](int j, int (&pg)[kMaxBoxes]) {
+        if (!paged || j < first_cache) return;
+        const int key0 = kbeg + (j - first_cache) * BN;
+        for (int r = 0, x = 0; r < BN; r += box, ++x) pg[x] = (key0 + r < kend) ? cache_page(a, b, key0 + r) : 0;
+    };
     // tile j of K (is_v == false) or V into ring stage `dst`
-    auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar) {
+    auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar, const int (&pg)[kMaxBoxes]) {
         mbar_arrive_expect_tx(bar, S::kv_bytes);
         const CUtensorMap *cache_map = is_v ? &tm_vc : &tm_kc;
         const CUtensorMap *new_map = is_v ? &tm_vn : &tm_kn;
-        if (j >= first_cache) {
+        if (j >= first_cache && paged) {
+            const int key0 = kbeg + (j - first_cache) * BN;
+            for (int r = 0, x = 0; r < BN; r += box, ++x) {
+                const int row = (key0 + r) & (a.page_size - 1);
+#pragma unroll
+                for (int dh = 0; dh < S::DH; ++dh)
+                    tma_load_3d(dst + dh * BN * 128 + r * 128, cache_map, bar, dh * 64, row, pg[x] * a.Hkv + g);
+            }
+        } else if (j >= first_cache) {
 #pragma unroll
             for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + (j - first_cache) * BN, bg);
         } else {
@@ -273,8 +293,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_barrier_init();
         prefetch_tensormap(&tm_vc);
         prefetch_tensormap(&tm_vn);
+        int pg[NSV][kMaxBoxes];
+        for (int j = 0; j < min(NSV, n_tiles); ++j) tile_pages(j, pg[j]);
         for (; v_issued < min(NSV, n_tiles); ++v_issued)
-            issue_tile(v_issued, true, sV + v_issued * S::kv_bytes, &v_full[v_issued]);
+            issue_tile(v_issued, true, sV + v_issued * S::kv_bytes, &v_full[v_issued], pg[v_issued]);
     }
     if (warp == kKProducerWarp) {
         if (lane == 0) {
@@ -303,8 +325,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_barrier_init();
             prefetch_tensormap(&tm_kc);
             prefetch_tensormap(&tm_kn);
+            int pg[NSK][kMaxBoxes];
+            for (int j = 0; j < min(NSK, n_tiles); ++j) tile_pages(j, pg[j]);
             for (; k_issued < min(NSK, n_tiles); ++k_issued)
-                issue_tile(k_issued, false, sK + k_issued * S::kv_bytes, &k_full[k_issued]);
+                issue_tile(k_issued, false, sK + k_issued * S::kv_bytes, &k_full[k_issued], pg[k_issued]);
         }
     }
     if (warp == kMmaWarp) {
@@ -368,12 +392,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     append_tile(true);
                     appended = true;
                 }
+                int pg[kMaxBoxes];
+                tile_pages(j, pg);
                 if (!mbar_wait(&v_empty[s], ((j / NSV) - 1) & 1, kWaitNs)) {
                     *s_abort = 1;
                     break;
                 }
                 if (*s_abort) break;
-                issue_tile(j, true, sV + s * S::kv_bytes, &v_full[s]);
+                issue_tile(j, true, sV + s * S::kv_bytes, &v_full[s], pg);
                 v_issued = j + 1;
             }
             if (appender && !appended && v_issued == n_tiles) append_tile(true);
@@ -388,12 +414,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     append_tile(false);
                     appended = true;
                 }
+                int pg[kMaxBoxes];
+                tile_pages(j, pg);
                 if (!mbar_wait(&k_empty[s], ((j / NSK) - 1) & 1, kWaitNs)) {
                     *s_abort = 1;
                     break;
                 }
                 if (*s_abort) break;
-                issue_tile(j, false, sK + s * S::kv_bytes, &k_full[s]);
+                issue_tile(j, false, sK + s * S::kv_bytes, &k_full[s], pg);
                 k_issued = j + 1;
             }
             if (appender && !appended && k_issued == n_tiles) append_tile(false);
@@ -852,14 +880,28 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
 
     CUtensorMap kc, vc, kn, vn, ks, vs;
     const uint64_t e = 2;
-    if (!make_tmap_bf16_3d(&kc, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
-        !make_tmap_bf16_3d(&vc, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, BN, 1) ||
-        !make_tmap_bf16_3d(&kn, a.k_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) ||
-        !make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) ||
-        // the append: T rows of one (sequence, head) plane of the cache
-        !make_tmap_bf16_3d(&ks, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, a.T, 1) ||
-        !make_tmap_bf16_3d(&vs, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, (uint64_t)a.Lcap * D * e, 64, a.T, 1))
-        return cudaErrorInvalidValue;
+    bool ok = make_tmap_bf16_3d(&kn, a.k_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) &&
+              make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN);
+    if (a.block_table) {
+        // page pools [n_pages * Hkv planes][page_size rows][D]; a paged call
+        // never appends, so the append maps are not used
+        const uint32_t box = (uint32_t)(a.page_size < BN ? a.page_size : BN);
+        const uint64_t plane = (uint64_t)a.page_size * D * e;
+        ok = ok &&
+             make_tmap_bf16_3d(&kc, a.k_cache, D, a.page_size, (uint64_t)a.n_pages * a.Hkv, D * e, plane, 64, box, 1) &&
+             make_tmap_bf16_3d(&vc, a.v_cache, D, a.page_size, (uint64_t)a.n_pages * a.Hkv, D * e, plane, 64, box, 1);
+        ks = kc;
+        vs = vc;
+    } else {
+        const uint64_t plane = (uint64_t)a.Lcap * D * e;
+        ok = ok &&
+             make_tmap_bf16_3d(&kc, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, BN, 1) &&
+             make_tmap_bf16_3d(&vc, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, BN, 1) &&
+             // the append: T rows of one (sequence, head) plane of the cache
+             make_tmap_bf16_3d(&ks, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, a.T, 1) &&
+             make_tmap_bf16_3d(&vs, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, a.T, 1);
+    }
+    if (!ok) return cudaErrorInvalidValue;
 
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.row_tiles, n, a.B * a.Hkv);

@@ -163,6 +163,28 @@ def test_accept_ex_host_validation(lib):
     assert call(7, B=0) == 0
 
 
+def test_paged_host_validation(lib):
+    P = ctypes.c_void_p
+    pw = lib.clover_verify_attn_paged_workspace_size
+    assert pw(1, 64, 32, 32, 128, 64, 65, 0) == lib.clover_verify_attn_workspace_size(1, 64, 32, 32, 128, 64 * 65, 0)
+    assert pw(1, 16, 8, 8, 64, 24, 10, 0) == 0 and pw(1, 16, 8, 8, 64, 8, 10, 0) == 0   # page 24, page 8
+    assert pw(1, 16, 8, 8, 64, 2048, 10, 0) == 0 and pw(1, 16, 8, 8, 64, 64, 0, 0) == 0
+
+    def attn(ps=64, n_pages=10, bt=64, T=4, B=1, D=64):
+        return lib.clover_verify_attn_paged(P(64), P(64), P(64), P(64), P(64), P(bt), n_pages, ps, 8, P(64), P(64),
+                                            P(64), B, T, 2, 2, D, 1, 0.0, None, 0, None, None)
+    assert attn(ps=24) == 1 and attn(ps=8) == 1 and attn(n_pages=0) == 1 and attn(bt=0) == 1
+    assert attn(T=129) == 2 and attn(D=96) == 2
+    assert attn(B=0) == 0
+
+    def commit(ps=64, bt=64, D=64, B=2, kn=64):
+        return lib.clover_kv_commit_paged(P(64), P(64), P(bt), 10, ps, 8, P(kn), P(64), P(1024), P(64), P(64),
+                                          P(2048), None, B, 4, 2, D, 1, None, None)
+    assert commit(ps=100) == 1 and commit(bt=0) == 1 and commit(kn=0) == 1
+    assert commit(D=96) == 2
+    assert commit(B=0) == 0
+
+
 def test_python_binding_rejects_cpu_tensors(lib):
     import paper_2405_00263_gb300 as pkg
     x = torch.zeros(1, 4, 2, 64, dtype=torch.bfloat16)

@@ -73,3 +73,26 @@ def test_bf16_scaled_distribution():
     q = t["q"].float()
     assert abs(float(q.std()) - 1 / math.sqrt(128)) < 2e-3
     assert t["q"].dtype == torch.bfloat16 and t["logits"].dtype == torch.bfloat16
+
+
+def test_paging_round_trip_and_scatter():
+    """A dense cache put into pages by a seeded table and read back is unchanged
+    where a page exists; the table scatters neighbouring slots; spare pages are
+    NaN and entries past each sequence's need are -1."""
+    from synth import paging
+    need = [100, 0, 257, 64]
+    table, n_pages = paging.page_table(need, 64, 6, seed=3)
+    assert n_pages == 2 + 0 + 5 + 1 + 3
+    owned = sorted(int(x) for x in table.flatten() if x >= 0)
+    assert owned == sorted(set(owned)) and len(owned) == n_pages - 3       # each page owned once
+    assert (table[1] == -1).all() and int(table[0, 2]) == -1
+    cache = torch.randn(4, 2, 384, 8)
+    pool = paging.to_pages(cache, table, 64, n_pages)
+    spare = sorted(set(range(n_pages)) - set(owned))
+    assert torch.isnan(pool[spare]).all()
+    back = paging.from_pages(pool, table, 64, 384)
+    for b, n in enumerate(need):
+        m = -(-n // 64) * 64
+        assert torch.equal(back[b, :, :m], cache[b, :, :m])
+        assert torch.isnan(back[b, :, m:]).all()
+    assert table[2, :5].tolist() != sorted(table[2, :5].tolist()) or table[2, :5].tolist() != list(range(5))
