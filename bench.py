@@ -237,6 +237,22 @@ def make_sets(w, device, n_sets):
     return base, sets
 
 
+def page_sets(w, sets, page_size, Lcap):
+    """Replace every set's dense caches by page pools under a seeded block
+    table (synth.paging), giving each sequence pages for L + T slots.  Returns
+    the capacity page_size * max_pages."""
+    from synth import paging, workloads
+    max_pages = -(-Lcap // page_size)
+    need = [L + w.T for L in workloads.cache_lengths(w)]
+    for i, s in enumerate(sets):
+        table, n_pages = paging.page_table(need, page_size, max_pages, seed=w.seed * 131 + i)
+        dev = s["k_cache"].device
+        s["k_cache"] = paging.to_pages(s["k_cache"].cpu(), table, page_size, n_pages).to(dev)
+        s["v_cache"] = paging.to_pages(s["v_cache"].cpu(), table, page_size, n_pages).to(dev)
+        s["block_table"] = table.to(dev)
+    return max_pages * page_size
+
+
 def set_bytes(s) -> int:
     return sum(t.numel() * t.element_size() for t in s.values())
 
@@ -255,9 +271,11 @@ def run_gpu_arm(args, world, rank, local, dist):
     del base, sets
     base, sets = make_sets(w, device, n_sets)
     Lcap = base["Lcap"]
+    if args.page_size:
+        Lcap = page_sets(w, sets, args.page_size, Lcap)
     step = pkg.VerifyStep(w.B, w.T, w.Hq, w.Hkv, w.D, Lcap, w.V, w.torch_dtype, device=device,
                           accept=args.accept, temperature=args.temperature, epsilon=args.epsilon,
-                          delta=args.delta, schedule=args.schedule)
+                          delta=args.delta, schedule=args.schedule, page_size=args.page_size or None)
     stream = torch.cuda.Stream(device)
 
     ext_ok = True
@@ -268,7 +286,7 @@ def run_gpu_arm(args, world, rank, local, dist):
 
     def launch(s, evs=None):
         step.run(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"], s["parent"],
-                 s["cand"], s["logits"], stream=stream, events=evs)
+                 s["cand"], s["logits"], stream=stream, events=evs, block_table=s.get("block_table"))
 
     # eager warm-up (also initialises per-kernel attributes before capture)
     with torch.cuda.stream(stream):
@@ -349,13 +367,18 @@ def run_gpu_arm(args, world, rank, local, dist):
     us["accept"] = accept_kernel_us(pkg, w, sets, stream, device, args.accept, args, flush)
     other = "greedy" if args.accept == "typical" else "typical"
     us_other = accept_kernel_us(pkg, w, sets, stream, device, other, args, flush)
-    us["kv_commit"] = isolated_us(
-        lambda i: pkg.clover_kv_commit(sets[i % n_sets]["k_cache"], sets[i % n_sets]["v_cache"],
-                                       sets[i % n_sets]["k_new"], sets[i % n_sets]["v_new"],
-                                       sets[i % n_sets]["cache_len"], step.path, step.accept_len,
-                                       step.new_cache_len, step.src_index, status=step.status_accept,
-                                       stream=stream),
-        3 * len(sets), stream, flush)
+    def commit_call(i):
+        c = sets[i % n_sets]
+        if args.page_size:
+            pkg.clover_kv_commit_paged(c["k_cache"], c["v_cache"], c["block_table"], c["k_new"], c["v_new"],
+                                       c["cache_len"], step.path, step.accept_len, step.new_cache_len,
+                                       step.src_index, status=step.status_accept, stream=stream)
+        else:
+            pkg.clover_kv_commit(c["k_cache"], c["v_cache"], c["k_new"], c["v_new"], c["cache_len"], step.path,
+                                 step.accept_len, step.new_cache_len, step.src_index, status=step.status_accept,
+                                 stream=stream)
+
+    us["kv_commit"] = isolated_us(commit_call, 3 * len(sets), stream, flush)
     del flush
     if step.device_status() != 0:
         raise RuntimeError(f"device status {step.device_status()} in the per-kernel timing")
@@ -364,7 +387,7 @@ def run_gpu_arm(args, world, rank, local, dist):
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     a_bytes = attn_bytes_per_launch(w, lengths)
     achieved = a_bytes / (us["tree_attn"] * 1e-6) / 1e9
-    traffic = recorded_traffic("tree_attn", w.name)
+    traffic = recorded_traffic("tree_attn", w.name + (f"_paged{args.page_size}" if args.page_size else ""))
     am_bytes = argmax_bytes_per_launch(w)
 
     # end to end through the public API from pinned host buffers
@@ -377,6 +400,8 @@ def run_gpu_arm(args, world, rank, local, dist):
         "config": {"workload": f"{w.name}: {w.description}", "B": w.B, "T": w.T, "Hq": w.Hq, "Hkv": w.Hkv,
                    "D": w.D, "L": lengths if len(lengths) <= 4 else f"{len(lengths)} lengths, sum {sum(lengths)}",
                    "V": w.V, "Lcap": Lcap, "parallelism": f"replicas x{world} (one per GPU)",
+                   "kv_cache": (f"paged, {args.page_size}-slot pages scattered over the pool by a seeded table"
+                                if args.page_size else "dense [B, Hkv, Lcap, D]"),
                    "l2": f"{n_sets} rotating input sets of {per_set / 1e6:.1f} MB "
                          f"({n_sets * per_set / 1e6:.0f} MB > 3x the 129 MB L2)",
                    "launch": LAUNCH_DESC[args.schedule],
@@ -487,7 +512,7 @@ def run_e2e(args, w, step, sets, stream, device, dist, world):
         for k in inputs:
             d[k].copy_(host_in[k], non_blocking=True)
         step.run(d["q"], d["k_new"], d["v_new"], s["k_cache"], s["v_cache"], d["cache_len"], d["parent"],
-                 d["cand"], d["logits"], stream=stream)
+                 d["cand"], d["logits"], stream=stream, block_table=s.get("block_table"))
         for h, o in zip(host_out, outs):
             h.copy_(o, non_blocking=True)
 
@@ -579,6 +604,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],
                     help="acceptance rule of the step (typical: tempered softmax with an entropy threshold)")
+    ap.add_argument("--page-size", type=int, default=0,
+                    help="run on a paged KV cache with pages of this many slots (0: dense cache)")
     ap.add_argument("--schedule", default="commit", choices=["commit", "compact", "fused"],
                     help="call schedule of the step (VerifyStep)")
     ap.add_argument("--temperature", type=float, default=1.0)

@@ -380,12 +380,19 @@ class VerifyStep:
     ``src_index`` holds tree nodes (commit) or cache slots (compact).
     ``accept``: ``"greedy"`` (clover_verify_accept) or ``"typical"``
     (clover_verify_accept_typical with ``temperature``, ``epsilon``, ``delta``).
+    ``page_size``: a paged cache (commit schedule only): ``run`` then takes the
+    page pools as k_cache/v_cache and the ``block_table``, and calls
+    clover_verify_attn_paged and clover_kv_commit_paged; ``Lcap`` is the
+    capacity page_size * max_pages.
     """
 
     def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda", concurrent=True, schedule="commit",
-                 accept="greedy", temperature=1.0, epsilon=0.09, delta=0.3):
+                 accept="greedy", temperature=1.0, epsilon=0.09, delta=0.3, page_size=None):
         if schedule not in ("commit", "compact", "fused"):
             raise ValueError(f"unknown schedule {schedule!r}")
+        if page_size is not None and (schedule != "commit" or Lcap % page_size):
+            raise ValueError("a paged cache takes the commit schedule and a capacity of whole pages")
+        self.page_size = page_size
         if accept not in ("greedy", "typical"):
             raise ValueError(f"unknown acceptance rule {accept!r}")
         self.shape = dict(B=B, T=T, Hq=Hq, Hkv=Hkv, D=D, Lcap=Lcap, V=V)
@@ -423,7 +430,7 @@ class VerifyStep:
         self.status_accept.zero_()
 
     def run(self, q, k_new, v_new, k_cache, v_cache, cache_len, parent, cand, logits, scale=0.0,
-            stream=None, events=None):
+            stream=None, events=None, block_table=None):
         """One step.  ``events`` (optional, up to six CUDA events) brackets the
         attention (0-1), the commit or compaction (2-3) and the accept call
         (4-5), each on the stream it runs on; a shorter list brackets only the
@@ -464,8 +471,12 @@ class VerifyStep:
             self._fork.record(stream)
             self.side.wait_event(self._fork)
         ev(0, stream)
-        clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
-                           workspace=self.ws_attn, status=self.status, stream=stream, append=not commit)
+        if self.page_size is not None:
+            clover_verify_attn_paged(q, k_new, v_new, k_cache, v_cache, block_table, cache_len, parent, self.out,
+                                     scale=scale, workspace=self.ws_attn, status=self.status, stream=stream)
+        else:
+            clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
+                               workspace=self.ws_attn, status=self.status, stream=stream, append=not commit)
         ev(1, stream)
         ev(4, side)
         if self.accept == "typical":
@@ -478,8 +489,13 @@ class VerifyStep:
         ev(5, side)
         if commit:
             ev(2, side)
-            clover_kv_commit(k_cache, v_cache, k_new, v_new, cache_len, self.path, self.accept_len,
-                             self.new_cache_len, self.src_index, status=self.status_accept, stream=side)
+            if self.page_size is not None:
+                clover_kv_commit_paged(k_cache, v_cache, block_table, k_new, v_new, cache_len, self.path,
+                                       self.accept_len, self.new_cache_len, self.src_index, status=self.status_accept,
+                                       stream=side)
+            else:
+                clover_kv_commit(k_cache, v_cache, k_new, v_new, cache_len, self.path, self.accept_len,
+                                 self.new_cache_len, self.src_index, status=self.status_accept, stream=side)
             ev(3, side)
             if self.side is not None:
                 self._join.record(self.side)

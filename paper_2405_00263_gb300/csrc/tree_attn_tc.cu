@@ -48,6 +48,7 @@ constexpr int BM = 128;                 // query rows per CTA (MMA M)
 constexpr int BN = 128;                 // keys per tile (the N of the S MMA)
 constexpr int kMinPage = 16;             // smallest page of a paged cache (rows)
 constexpr int kMaxBoxes = BN / kMinPage; // TMA boxes of one paged cache tile
+constexpr int kPageSmem = 512;           // page ids of a split staged in shared memory
 constexpr int kKProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kVProducerWarp = 6;
@@ -73,7 +74,8 @@ struct TcSmem {
     static constexpr int n_bars = 2 * NSK + 2 * NSV + 11;
     static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad flags
     static constexpr int anc_off = misc_off + 16;                  // ancestor masks [128][2]
-    static constexpr int total = anc_off + kMaxTreeNodes * kMaskWords * 8;
+    static constexpr int pages_off = anc_off + kMaxTreeNodes * kMaskWords * 8;   // paged: page ids of the split
+    static constexpr int total = pages_off + kPageSmem * 4;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
     // TMEM columns: S/P 2 x BN, O D, Q D / 2 (two bf16 per column), rounded up
     // to a power of two.  All 512 columns of an SM go to one CTA only when
@@ -197,6 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     volatile int *s_abort = reinterpret_cast<volatile int *>(sm + S::misc_off + 4);
     bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 8);
     uint64_t *s_anc = reinterpret_cast<uint64_t *>(sm + S::anc_off);
+    int *s_pages = reinterpret_cast<int *>(sm + S::pages_off);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -233,10 +236,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     // page ids of tile j, looked up before the producer waits for the stage.
     const bool paged = a.block_table != nullptr;
     const int box = paged ? min(a.page_size, BN) : BN;
-    auto tile_pages = [&](int j, int (&pg)[kMaxBoxes]) {
+    const int first_page = kbeg >> a.page_shift;     // the split's first page (paged)
+    // staged: the split's first kPageSmem page ids are in s_pages (after the
+    // setup barrier); later ones, and all of them before it, come from the table
+    auto tile_pages = [&](int j, int (&pg)[kMaxBoxes], bool staged) {
         if (!paged || j < first_cache) return;
         const int key0 = kbeg + (j - first_cache) * BN;
-        for (int r = 0, x = 0; r < BN; r += box, ++x) pg[x] = (key0 + r < kend) ? cache_page(a, b, key0 + r) : 0;
+        for (int r = 0, x = 0; r < BN; r += box, ++x) {
+            const int slot = key0 + r;
+            const int pi = (slot >> a.page_shift) - first_page;
+            pg[x] = slot >= kend ? 0 : (staged && pi < kPageSmem) ? s_pages[pi] : cache_page(a, b, slot);
+        }
     };
     // tile j of K (is_v == false) or V into ring stage `dst`
     auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar, const int (&pg)[kMaxBoxes]) {
@@ -294,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         prefetch_tensormap(&tm_vc);
         prefetch_tensormap(&tm_vn);
         int pg[NSV][kMaxBoxes];
-        for (int j = 0; j < min(NSV, n_tiles); ++j) tile_pages(j, pg[j]);
+        for (int j = 0; j < min(NSV, n_tiles); ++j) tile_pages(j, pg[j], false);
         for (; v_issued < min(NSV, n_tiles); ++v_issued)
             issue_tile(v_issued, true, sV + v_issued * S::kv_bytes, &v_full[v_issued], pg[v_issued]);
     }
@@ -326,7 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             prefetch_tensormap(&tm_kc);
             prefetch_tensormap(&tm_kn);
             int pg[NSK][kMaxBoxes];
-            for (int j = 0; j < min(NSK, n_tiles); ++j) tile_pages(j, pg[j]);
+            for (int j = 0; j < min(NSK, n_tiles); ++j) tile_pages(j, pg[j], false);
             for (; k_issued < min(NSK, n_tiles); ++k_issued)
                 issue_tile(k_issued, false, sK + k_issued * S::kv_bytes, &k_full[k_issued], pg[k_issued]);
         }
@@ -334,6 +344,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kMmaWarp) {
         tmem_alloc(s_tmem, S::tmem_cols);
         tmem_relinquish();
+        // paged: the split's page ids, for the producers' loops
+        if (paged && kend > kbeg) {
+            const int n_pg = min(kPageSmem, ((kend - 1) >> a.page_shift) - first_page + 1);
+            for (int i = lane; i < n_pg; i += 32) s_pages[i] = cache_page(a, b, (first_page + i) << a.page_shift);
+        }
     }
     // Q rows of this warp's TMEM lane quadrant (row (node, head in group) =
     // lane-quadrant row; with KS = 2 lanes 64-127 take rows 0-63 again): loaded
@@ -393,7 +408,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     appended = true;
                 }
                 int pg[kMaxBoxes];
-                tile_pages(j, pg);
+                tile_pages(j, pg, true);
                 if (!mbar_wait(&v_empty[s], ((j / NSV) - 1) & 1, kWaitNs)) {
                     *s_abort = 1;
                     break;
@@ -415,7 +430,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     appended = true;
                 }
                 int pg[kMaxBoxes];
-                tile_pages(j, pg);
+                tile_pages(j, pg, true);
                 if (!mbar_wait(&k_empty[s], ((j / NSK) - 1) & 1, kWaitNs)) {
                     *s_abort = 1;
                     break;
