@@ -164,7 +164,7 @@ __device__ __forceinline__ void merge_rows(const float *own, const float *recv, 
     }
 }
 
-template <int D, int KS>
+template <int D, int KS, bool PAGED>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                         const __grid_constant__ CUtensorMap tm_kn, const __grid_constant__ CUtensorMap tm_vn,
@@ -234,7 +234,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Paged cache: a cache tile is read as boxes of `box` rows, each inside one
     // page (box = min(page size, BN); tiles start at multiples of BN).  The
     // page ids of tile j, looked up before the producer waits for the stage.
-    const bool paged = a.block_table != nullptr;
+    // PAGED is a template flag: the dense kernel carries none of this code
+    constexpr bool paged = PAGED;
     const int box = paged ? min(a.page_size, BN) : BN;
     const int first_page = kbeg >> a.page_shift;     // the split's first page (paged)
     // staged: the split's first kPageSmem page ids are in s_pages (after the
@@ -843,7 +844,7 @@ struct TcLaunchCache {
     int max_clusters[kMaxCluster + 1] = {0};   // co-resident clusters per cluster size (0: not queried)
 };
 
-template <int D, int KS>
+template <int D, int KS, bool PAGED>
 int max_active_clusters(int n, TcLaunchCache &cache) {
     if (cache.max_clusters[n] == 0) {
         cudaLaunchConfig_t cfg = {};
@@ -858,7 +859,7 @@ int max_active_clusters(int n, TcLaunchCache &cache) {
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
         int num = 0;
-        if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D, KS>, &cfg) != cudaSuccess) {
+        if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D, KS, PAGED>, &cfg) != cudaSuccess) {
             cudaGetLastError();
             num = -1;
         }
@@ -867,11 +868,11 @@ int max_active_clusters(int n, TcLaunchCache &cache) {
     return cache.max_clusters[n];
 }
 
-template <int D, int KS>
+template <int D, int KS, bool PAGED>
 cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     static unsigned char done[64];
     static TcLaunchCache caches[64];
-    auto kernel = tree_attn_tc_kernel<D, KS>;
+    auto kernel = tree_attn_tc_kernel<D, KS, PAGED>;
     cudaError_t err = ensure_smem_attr(kernel, TcSmem<D, KS>::alloc, done);
     if (err != cudaSuccess) return err;
     int dev = 0;
@@ -886,7 +887,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     int n = 1;
     for (int c = kMaxCluster; c >= 2; --c) {
         if (c > by_len || base * c > cache.sms) continue;
-        if (max_active_clusters<D, KS>(c, cache) >= base) {
+        if (max_active_clusters<D, KS, PAGED>(c, cache) >= base) {
             n = c;
             break;
         }
@@ -897,7 +898,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     const uint64_t e = 2;
     bool ok = make_tmap_bf16_3d(&kn, a.k_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) &&
               make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN);
-    if (a.block_table) {
+    if (PAGED) {
         // page pools [n_pages * Hkv planes][page_size rows][D]; a paged call
         // never appends, so the append maps are not used
         const uint32_t box = (uint32_t)(a.page_size < BN ? a.page_size : BN);
@@ -941,8 +942,12 @@ int tc_row_tile() { return BM; }
 
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream) {
     // a tile of at most 64 real rows: two key groups per row (KS = 2)
-    if (a.rows <= 64) return a.D == 64 ? launch<64, 2>(a, stream) : launch<128, 2>(a, stream);
-    return a.D == 64 ? launch<64, 1>(a, stream) : launch<128, 1>(a, stream);
+    if (a.block_table) {
+        if (a.rows <= 64) return a.D == 64 ? launch<64, 2, true>(a, stream) : launch<128, 2, true>(a, stream);
+        return a.D == 64 ? launch<64, 1, true>(a, stream) : launch<128, 1, true>(a, stream);
+    }
+    if (a.rows <= 64) return a.D == 64 ? launch<64, 2, false>(a, stream) : launch<128, 2, false>(a, stream);
+    return a.D == 64 ? launch<64, 1, false>(a, stream) : launch<128, 1, false>(a, stream);
 }
 
 }  // namespace clover
