@@ -61,6 +61,9 @@ def _load():
             lib.oracle_kv_compact.argtypes = [P, P, P, P, P, I, I, I, I, I, I, P]
             lib.oracle_kv_commit.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P]
             lib.oracle_accept_typical.argtypes = [P, P, P, I, I, I64, I, D, D, D, P, P, P, P, P, I]
+            lib.oracle_linear.argtypes = [P, P, P, I, I, I, I, I, P, I]
+            lib.oracle_embed_rows.argtypes = [P, P, I, I, I, I, P]
+            lib.oracle_topk.argtypes = [P, I, I, I, P, P]
             for f in (lib.oracle_tree_mask, lib.oracle_tree_attention, lib.oracle_argmax,
                       lib.oracle_accept_walk, lib.oracle_append_tree_kv, lib.oracle_kv_compact,
                       lib.oracle_kv_commit):
@@ -250,3 +253,63 @@ def verify_step(inp: dict, scale: float = 0.0, n_threads: int | None = None, typ
     src = kv_compact(k_cache, v_cache, cache_len, path, alen)
     return {"out": out, "argmax": amax, "path": path, "accept_len": alen, "bonus": bonus,
             "src_index": src, "k_cache": k_cache, "v_cache": v_cache, "cache_len": cache_len}
+
+
+def linear(x, w, res=None, act=0, n_threads: int | None = None) -> torch.Tensor:
+    """fp64 y [R,N] = x [R,K] . w [N,K]^T (act 0), or res + silu(x . w^T) (act 1);
+    x, w, res share one dtype."""
+    xc, wc = _cpu(x), _cpu(w)
+    R, K = xc.shape
+    N = wc.shape[0]
+    assert wc.shape[1] == K and wc.dtype == xc.dtype
+    rc = _cpu(res) if res is not None else None
+    if rc is not None:
+        assert rc.shape == (R, N) and rc.dtype == xc.dtype
+    y = torch.empty((R, N), dtype=torch.float64)
+    _check(_load().oracle_linear(_p(xc), _p(wc), _p(rc), R, N, K, _dtype_code(xc), act, _p(y),
+                                 n_threads or default_threads()))
+    return y
+
+
+def embed_rows(w, tokens) -> torch.Tensor:
+    """fp64 e [R,H]: row tokens[r] of w [V,H] divided by its L2 norm."""
+    wc = _cpu(w)
+    V, H = wc.shape
+    t = _cpu(torch.as_tensor(tokens, dtype=torch.int32))
+    e = torch.empty((t.numel(), H), dtype=torch.float64)
+    _check(_load().oracle_embed_rows(_p(wc), _p(t), t.numel(), V, H, _dtype_code(wc), _p(e)))
+    return e
+
+
+def topk(x, k: int):
+    """(values fp64 [R,k], indices int32 [R,k]) of each row of x (widened to fp64):
+    decreasing value, equal values by increasing index."""
+    xc = _cpu(x.to(torch.float64))
+    R, V = xc.shape
+    vals = torch.empty((R, k), dtype=torch.float64)
+    idx = torch.empty((R, k), dtype=torch.int32)
+    _check(_load().oracle_topk(_p(xc), R, V, k, _p(vals), _p(idx)))
+    return vals, idx
+
+
+def clover_head_step(h, tokens, w_lm, w_v, w_o, w_1, k: int):
+    """One speculative head (Section 3.2 Eq. 1-2, the MLP block, the shared LM
+    head), from bf16 inputs h [R,H] (the previous hidden state) and tokens [R]
+    (the previous token).  The cross attention has a single key and value (the
+    previous token's embedding), so its softmax weight is 1 and its output is
+    W_o . W_v . e whatever the query; W_Q and W_K do not enter.  Every layer's
+    input is a bf16 tensor (rounded to nearest even), as the layers take them:
+      e  = embed_rows(w_lm, tokens)
+      h' = h + W_o (W_v e)
+      z  = h' + silu(W_1 h')
+      logits = W_lm z, and their top-k.
+    Returns a dict of the fp64 intermediates, the logits and the top-k."""
+    bf = torch.bfloat16
+    e = embed_rows(w_lm, tokens)
+    a = linear(e.to(bf), w_v)
+    d = linear(a.to(bf), w_o)
+    h1 = h.double() + d
+    z = linear(h1.to(bf), w_1, res=h1.to(bf), act=1)
+    logits = linear(z.to(bf), w_lm)
+    vals, idx = topk(logits, k)
+    return {"e": e, "v": a, "attn": d, "h": h1, "z": z, "logits": logits, "top_values": vals, "top_indices": idx}

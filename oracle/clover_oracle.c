@@ -28,6 +28,10 @@
  *             token's probability under the tempered softmax of the parent's
  *             logits exceeds min(epsilon, delta * exp(-entropy)); the longest
  *             accepted path wins (ties: lexicographically smallest).
+ *   draft     Section 3 (the Clover heads): a linear layer with an optional
+ *             residual SiLU (the heads' MLP block), the LM-head row embedding
+ *             of the regressive connection (Section 3.4), and the top-k of the
+ *             shared LM head's logits.
  *   append /  (engine step; the paper is silent) the T tree keys/values occupy
  *   compact   cache slots [L, L+T); the accepted nodes' K/V are then moved, in
  *             path order, to slots [L, L+a) and the length becomes L + a.
@@ -499,4 +503,76 @@ int oracle_accept_typical(const void *logits, const int32_t *parent, const int32
     free(row_log_theta);
     free(row_amax);
     return status;
+}
+
+/*
+ * Draft side (Section 3: the Clover heads), the dense pieces of one head step.
+ *
+ * Linear layer, fp64 on exactly widened inputs:
+ *   y[r][n] = sum_k x[r][k] * w[n][k]                       (act 0)
+ *   y[r][n] = res[r][n] + silu(sum_k x[r][k] * w[n][k])      (act 1: the
+ *            residual SiLU block of the speculative heads' MLP)
+ * with silu(v) = v / (1 + exp(-v)).  x [R,K], w [N,K] (output features by
+ * input features), res [R,N] (act 1 only), y [R,N].
+ */
+int oracle_linear(const void *x, const void *w, const void *res, int R, int N, int K, int dtype, int act,
+                  double *y, int n_threads)
+{
+    if (R < 0 || N < 1 || K < 1 || (act != 0 && act != 1) || (act == 1 && !res)) return ORACLE_BAD_ARG;
+#pragma omp parallel for schedule(static) num_threads(n_threads > 0 ? n_threads : 1)
+    for (int64_t rn = 0; rn < (int64_t)R * N; ++rn) {
+        const int64_t r = rn / N, n = rn % N;
+        double s = 0.0;
+        for (int k = 0; k < K; ++k) s += load_elem(x, r * K + k, dtype) * load_elem(w, n * K + k, dtype);
+        if (act == 1) s = load_elem(res, r * N + n, dtype) + s / (1.0 + exp(-s));
+        y[rn] = s;
+    }
+    return ORACLE_OK;
+}
+
+/*
+ * The regressive connection's embedding (Section 3.4): the token's row of the
+ * LM-head weight after normalisation, e = w[t] / ||w[t]||_2.  w [V,H], tokens
+ * [R] in [0, V), e [R,H].
+ */
+int oracle_embed_rows(const void *w, const int32_t *tokens, int R, int V, int H, int dtype, double *e)
+{
+    for (int r = 0; r < R; ++r)
+        if (tokens[r] < 0 || tokens[r] >= V) return ORACLE_BAD_ARG;
+    for (int r = 0; r < R; ++r) {
+        double s = 0.0;
+        for (int h = 0; h < H; ++h) {
+            const double v = load_elem(w, (int64_t)tokens[r] * H + h, dtype);
+            s += v * v;
+        }
+        const double inv = s > 0.0 ? 1.0 / sqrt(s) : 0.0;
+        for (int h = 0; h < H; ++h) e[(int64_t)r * H + h] = load_elem(w, (int64_t)tokens[r] * H + h, dtype) * inv;
+    }
+    return ORACLE_OK;
+}
+
+/*
+ * Top-k of each row of fp64 values x [R,V]: the k largest, in decreasing
+ * order, equal values by increasing index.  values, indices [R,k].
+ */
+int oracle_topk(const double *x, int R, int V, int k, double *values, int32_t *indices)
+{
+    if (k < 1 || k > V) return ORACLE_BAD_ARG;
+    for (int r = 0; r < R; ++r) {
+        const double *row = x + (int64_t)r * V;
+        for (int j = 0; j < k; ++j) {
+            /* the best element not yet taken: larger value, then smaller index */
+            int best = -1;
+            for (int v = 0; v < V; ++v) {
+                int taken = 0;
+                for (int q = 0; q < j; ++q)
+                    if (indices[(int64_t)r * k + q] == v) taken = 1;
+                if (taken) continue;
+                if (best < 0 || row[v] > row[best]) best = v;
+            }
+            indices[(int64_t)r * k + j] = best;
+            values[(int64_t)r * k + j] = row[best];
+        }
+    }
+    return ORACLE_OK;
 }

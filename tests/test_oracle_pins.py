@@ -720,3 +720,90 @@ def test_typical_epsilon_monotone_and_rejects_bad_arguments():
     with pytest.raises(oracle.OracleError) as e:
         oracle.accept_typical(lg, bad, cd, 1.0, 0.1, 0.3)
     assert e.value.code == oracle.BAD_TREE
+
+
+# ---------------------------------------------------------------------------
+# A8: draft side (the Clover head's linear layers, embedding, top-k)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_linear_vs_library_matmul_and_silu(dtype):
+    special = pytest.importorskip("scipy.special")
+    g = torch.Generator().manual_seed(21)
+    for R, N, K in ((1, 1, 1), (3, 7, 5), (8, 33, 64), (17, 9, 130)):
+        x = torch.randn(R, K, generator=g).to(dtype)
+        w = torch.randn(N, K, generator=g).to(dtype)
+        res = torch.randn(R, N, generator=g).to(dtype)
+        ref = (x.double().numpy() @ w.double().numpy().T)
+        assert np.allclose(oracle.linear(x, w).numpy(), ref, rtol=1e-12, atol=1e-12)
+        got = oracle.linear(x, w, res=res, act=1).numpy()
+        assert np.allclose(got, res.double().numpy() + ref * special.expit(ref), rtol=1e-12, atol=1e-12)
+
+
+def test_linear_identity_and_zero_weight():
+    x = torch.randn(5, 16).bfloat16()
+    res = torch.randn(5, 16).bfloat16()
+    eye = torch.eye(16).bfloat16()
+    assert torch.equal(oracle.linear(x, eye), x.double())
+    assert torch.equal(oracle.linear(x, torch.zeros(16, 16).bfloat16(), res=res, act=1), res.double())
+    with pytest.raises(oracle.OracleError):
+        oracle.linear(x, eye, act=1)                  # the residual block needs its residual
+
+
+def test_embed_rows_unit_norm_and_direction():
+    g = torch.Generator().manual_seed(4)
+    w = torch.randn(50, 24, generator=g).bfloat16()
+    w[7] = 0
+    toks = [3, 7, 49, 3, 0]
+    e = oracle.embed_rows(w, toks)
+    for r, t in enumerate(toks):
+        row = w[t].double()
+        if t == 7:
+            assert (e[r] == 0).all()
+            continue
+        assert abs(e[r].norm().item() - 1.0) < 1e-12
+        assert torch.allclose(e[r] * row.norm(), row, rtol=1e-12, atol=1e-12)
+    # scaling a row does not change its embedding
+    w2 = w.clone()
+    w2[3] = (w[3].float() * 4).bfloat16()
+    assert torch.allclose(oracle.embed_rows(w2, [3]), e[:1], rtol=1e-12, atol=1e-12)
+    with pytest.raises(oracle.OracleError):
+        oracle.embed_rows(w, [50])
+
+
+def test_topk_vs_stable_sort_with_ties():
+    g = torch.Generator().manual_seed(8)
+    for R, V, k in ((1, 1, 1), (4, 10, 3), (3, 200, 8), (2, 64, 64)):
+        x = torch.randint(-5, 6, (R, V), generator=g).double()     # many ties
+        vals, idx = oracle.topk(x, k)
+        for r in range(R):
+            order = np.lexsort((np.arange(V), -x[r].numpy()))[:k]
+            assert idx[r].tolist() == order.tolist()
+            assert vals[r].tolist() == x[r, order].tolist()
+    with pytest.raises(oracle.OracleError):
+        oracle.topk(torch.zeros(1, 4), 5)
+
+
+def test_head_step_special_cases():
+    """W_v = 0: the decoder adds nothing; W_1 = 0 as well: the MLP block is the
+    identity (silu(0) = 0), so the logits are the LM head of bf16(h).  The
+    embedding ignores the scale of the LM-head rows."""
+    g = torch.Generator().manual_seed(12)
+    R, H, V, k = 3, 32, 300, 4
+    bf = torch.bfloat16
+    h = torch.randn(R, H, generator=g).to(bf)
+    toks = torch.tensor([5, 77, 299], dtype=torch.int32)
+    w_lm = torch.randn(V, H, generator=g).to(bf)
+    z0 = torch.zeros(H, H, dtype=bf)
+    w_o = torch.randn(H, H, generator=g).to(bf)
+    out = oracle.clover_head_step(h, toks, w_lm, z0, w_o, z0, k)
+    assert torch.equal(out["h"], h.double())
+    assert torch.equal(out["z"], h.double())
+    assert torch.equal(out["logits"], oracle.linear(h, w_lm))
+    ref_v, ref_i = oracle.topk(out["logits"], k)
+    assert torch.equal(out["top_indices"], ref_i)
+    w_v = torch.randn(H, H, generator=g).to(bf)
+    full = oracle.clover_head_step(h, toks, w_lm, w_v, w_o, z0, k)
+    e = oracle.embed_rows(w_lm, toks)
+    assert torch.allclose(full["attn"], oracle.linear(oracle.linear(e.to(bf), w_v).to(bf), w_o))
+    assert torch.allclose(full["h"], h.double() + full["attn"])
