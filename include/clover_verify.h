@@ -21,7 +21,11 @@
  *   clover_kv_compact     moves the accepted nodes' K/V to the front of the
  *                         tree slots (an engine step the paper leaves implicit);
  *   clover_verify_attn_paged, clover_kv_commit_paged
- *                         the attention and the commit on a paged KV cache.
+ *                         the attention and the commit on a paged KV cache;
+ *   clover_linear, clover_embed_rows, clover_topk
+ *                         the draft side: the dense layers of a Clover head,
+ *                         the LM-head row embedding and the top-k of its
+ *                         logits (Section 3).
  *
  * A second schedule of the same step: clover_verify_attn_ex with
  * CLOVER_ATTN_NO_APPEND leaves the caches untouched, and clover_kv_commit then
@@ -192,6 +196,52 @@ CLOVER_API clover_status clover_kv_commit_paged(void *k_pages, void *v_pages, co
                                    const int32_t *path, const int32_t *accept_len, int32_t *new_cache_len,
                                    int32_t *src_index_out, int B, int T, int Hkv, int D, clover_dtype dtype,
                                    int32_t *status, void *stream);
+
+/*
+ * Draft side: the dense pieces of one Clover head step (Section 3).  All
+ * tensors are device pointers, row-major, bf16 unless stated; no workspace
+ * unless stated.
+ */
+
+/* Epilogues of clover_linear (y = x . w^T accumulated in fp32). */
+#define CLOVER_LINEAR_F32 0       /* out fp32 = y (the LM head's logits) */
+#define CLOVER_LINEAR_BF16 1      /* out bf16 = y */
+#define CLOVER_LINEAR_RES_SILU 2  /* out bf16 = res + silu(y): the residual SiLU block of a head's MLP */
+#define CLOVER_LINEAR_RES 3       /* out bf16 = res + y: a residual add (the attention decoder's Eq. 2) */
+
+/*
+ * Linear layer on the tensor cores: x [R,K], w [N,K] (output features by input
+ * features), res [R,N] (modes 2-3; else may be NULL), out [R,N] (fp32 for
+ * CLOVER_LINEAR_F32, else bf16).  Rounding: one fp32 accumulation, then one
+ * rounding to bf16 (after the residual and SiLU) for the bf16 modes.
+ * K a multiple of 64 (16 <= K); R >= 0, N >= 1; x, w, res, out 16-byte
+ * aligned; out must not overlap x, w or res.  A bounded device wait that gives
+ * up raises CLOVER_ERR_TIMEOUT (device bit).
+ */
+CLOVER_API clover_status clover_linear(const void *x, const void *w, const void *res, void *out,
+                                   int R, int N, int K, int mode, int32_t *status, void *stream);
+
+/*
+ * The regressive connection's embedding (Section 3.4): e[r] = w[t[r]] / ||w[t[r]]||_2
+ * (the token's row of the LM-head weight, normalised), w [V,H], tokens [R]
+ * int32, e [R,H] bf16.  A token outside [0, V) -> CLOVER_ERR_INVALID_ARG
+ * (device bit; that row of e is zero).  A zero row gives a zero embedding.
+ */
+CLOVER_API clover_status clover_embed_rows(const void *w, const int32_t *tokens, void *e,
+                                   int R, int V, int H, int32_t *status, void *stream);
+
+/* Bytes of device workspace clover_topk needs (0 outside the limits). */
+CLOVER_API size_t clover_topk_workspace_size(int R, int V, int k);
+
+/*
+ * Top-k of each row of fp32 x [R,V] (the LM head's logits): values [R,k] fp32
+ * and indices [R,k] int32, in decreasing value, equal values by increasing
+ * index (-0 == +0).  1 <= k <= 32, k <= V.  The workspace (zero-filled before
+ * first use) is left ready for the next call; calls sharing it must not
+ * overlap on the device.  NaN in x: unspecified.
+ */
+CLOVER_API clover_status clover_topk(const float *x, int R, int V, int k, float *values, int32_t *indices,
+                                   void *workspace, size_t ws_bytes, int32_t *status, void *stream);
 
 /* Bytes of device workspace clover_verify_accept needs (0 outside the limits). */
 CLOVER_API size_t clover_verify_accept_workspace_size(int B, int T, int V, clover_dtype dtype);

@@ -35,6 +35,10 @@ EXPORTS = (
     "clover_verify_attn_paged_workspace_size",
     "clover_verify_attn_paged",
     "clover_kv_commit_paged",
+    "clover_linear",
+    "clover_embed_rows",
+    "clover_topk_workspace_size",
+    "clover_topk",
 )
 
 # Flag of clover_verify_attn_ex (CLOVER_ATTN_NO_APPEND in include/clover_verify.h).
@@ -44,6 +48,12 @@ ATTN_NO_APPEND = 1
 ACCEPT_TYPICAL = 1
 ACCEPT_COMMIT = 2
 ACCEPT_OVERLAP = 4
+
+# Epilogues of clover_linear (CLOVER_LINEAR_* in include/clover_verify.h).
+LINEAR_F32 = 0
+LINEAR_BF16 = 1
+LINEAR_RES_SILU = 2
+LINEAR_RES = 3
 
 # Bytes of the static scratch buffer behind clover_verify_attn_noalloc
 # (CLOVER_NOALLOC_SCRATCH_BYTES in include/clover_verify.h).
@@ -108,5 +118,13 @@ def load(build_if_missing: bool = False):
         lib.clover_verify_attn_paged.restype = I
         lib.clover_kv_commit_paged.argtypes = [P, P, P, I, I, I, P, P, P, P, P, P, P, I, I, I, I, I, P, P]
         lib.clover_kv_commit_paged.restype = I
+        lib.clover_linear.argtypes = [P, P, P, P, I, I, I, I, P, P]
+        lib.clover_linear.restype = I
+        lib.clover_embed_rows.argtypes = [P, P, P, I, I, I, P, P]
+        lib.clover_embed_rows.restype = I
+        lib.clover_topk_workspace_size.argtypes = [I, I, I]
+        lib.clover_topk_workspace_size.restype = Z
+        lib.clover_topk.argtypes = [P, I, I, I, P, P, P, Z, P, P]
+        lib.clover_topk.restype = I
         _lib = lib
         return lib

@@ -358,6 +358,98 @@ def clover_verify_accept_ex(logits, cand, parent, argmax_out, path_out, accept_l
         raise CloverError(code, "clover_verify_accept_ex")
 
 
+_LINEAR_MODES = {"f32": 0, "bf16": 1, "res_silu": 2, "res": 3}
+
+
+def clover_linear(x, w, out, res=None, mode="bf16", status=None, stream=None):
+    """out = x . w^T (fp32 accumulation) with the epilogue `mode`: "f32" (fp32
+    out), "bf16", "res_silu" (res + silu(.)), "res" (res + .); x [R,K], w [N,K],
+    res/out [R,N]."""
+    code = _LINEAR_MODES[mode]
+    R, K = x.shape
+    N = w.shape[0]
+    _check(x, (R, K), torch.bfloat16, "x")
+    _check(w, (N, K), torch.bfloat16, "w")
+    _check(out, (R, N), torch.float32 if code == 0 else torch.bfloat16, "out")
+    if code >= 2:
+        _check(res, (R, N), torch.bfloat16, "res")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(x, w, out, res if code >= 2 else None, status)
+    rc = _lib.load().clover_linear(_ptr(x), _ptr(w), _ptr(res if code >= 2 else None), _ptr(out), R, N, K, code,
+                                   _ptr(status), _stream(stream))
+    if rc != OK:
+        raise CloverError(rc, "clover_linear")
+
+
+def clover_embed_rows(w, tokens, out, status=None, stream=None):
+    """out[r] = w[tokens[r]] / ||w[tokens[r]]||_2 (bf16), w [V,H], tokens [R]."""
+    V, H = w.shape
+    R = tokens.shape[0]
+    _check(w, (V, H), torch.bfloat16, "w")
+    _check(tokens, (R,), torch.int32, "tokens")
+    _check(out, (R, H), torch.bfloat16, "out")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(w, tokens, out, status)
+    rc = _lib.load().clover_embed_rows(_ptr(w), _ptr(tokens), _ptr(out), R, V, H, _ptr(status), _stream(stream))
+    if rc != OK:
+        raise CloverError(rc, "clover_embed_rows")
+
+
+def clover_topk_workspace_size(R, V, k) -> int:
+    return int(_lib.load().clover_topk_workspace_size(R, V, k))
+
+
+def clover_topk(x, k, values, indices, workspace, status=None, stream=None):
+    """Top-k of each row of fp32 x [R,V]: values [R,k] fp32, indices [R,k] int32."""
+    R, V = x.shape
+    _check(x, (R, V), torch.float32, "x")
+    _check(values, (R, k), torch.float32, "values")
+    _check(indices, (R, k), torch.int32, "indices")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    _dev(x, values, indices, workspace, status)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    rc = _lib.load().clover_topk(_ptr(x), R, V, k, _ptr(values), _ptr(indices), _ptr(workspace), ws_bytes,
+                                 _ptr(status), _stream(stream))
+    if rc != OK:
+        raise CloverError(rc, "clover_topk")
+
+
+class DraftHead:
+    """One speculative head step of a Clover draft (Section 3), on R rows:
+    the previous token's embedding e (its row of the LM-head weight,
+    normalised), the attention decoder's h' = h + W_o W_v e (one key and value
+    per row, so the softmax weight is 1 and the query projections do not
+    enter), the MLP block z = h' + silu(W_1 h'), the shared LM head's fp32
+    logits and their top-k.  Weights are bf16 [out, in]; every layer's input
+    is bf16.  Owns the activations, the logits and the top-k workspace."""
+
+    def __init__(self, R, H, V, k, device="cuda"):
+        dev = torch.device(device)
+        bf = dict(dtype=torch.bfloat16, device=dev)
+        self.e = torch.empty((R, H), **bf)
+        self.v = torch.empty((R, H), **bf)
+        self.h = torch.empty((R, H), **bf)
+        self.z = torch.empty((R, H), **bf)
+        self.logits = torch.empty((R, V), dtype=torch.float32, device=dev)
+        self.values = torch.empty((R, k), dtype=torch.float32, device=dev)
+        self.indices = torch.empty((R, k), dtype=torch.int32, device=dev)
+        self.ws = torch.zeros(max(16, clover_topk_workspace_size(R, V, k)), dtype=torch.uint8, device=dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.k = k
+
+    def run(self, h, tokens, w_lm, w_v, w_o, w_1, stream=None):
+        st = dict(status=self.status, stream=stream)
+        clover_embed_rows(w_lm, tokens, self.e, **st)
+        clover_linear(self.e, w_v, self.v, mode="bf16", **st)
+        clover_linear(self.v, w_o, self.h, res=h, mode="res", **st)
+        clover_linear(self.h, w_1, self.z, res=self.h, mode="res_silu", **st)
+        clover_linear(self.z, w_lm, self.logits, mode="f32", **st)
+        clover_topk(self.logits, self.k, self.values, self.indices, self.ws, **st)
+
+
 class VerifyStep:
     """Device buffers for repeated verification steps of one shape.
 

@@ -15,6 +15,14 @@ cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream);
 void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk);
 size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype);
+cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
+                             int32_t *status, cudaStream_t stream);
+size_t topk_workspace_bytes(int R, int V, int k);
+int topk_max_k();
+cudaError_t launch_topk(const float *x, int R, int V, int k, float *values, int32_t *indices, void *workspace,
+                        int32_t *status, cudaStream_t stream);
+cudaError_t launch_embed_rows(const void *w, const int32_t *tokens, void *e, int R, int V, int H, int32_t *status,
+                              cudaStream_t stream);
 cudaError_t launch_accept_call(const AcceptCall &c, cudaStream_t stream);
 cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, const void *v_new,
                               const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
@@ -398,6 +406,46 @@ clover_status clover_kv_commit(void *k_cache, void *v_cache, const void *k_new, 
     return from_cuda(launch_kv_compact(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len, new_cache_len,
                                        src_index_out, B, T, Hkv, D, Lcap, dtype, status,
                                        static_cast<cudaStream_t>(stream)));
+}
+
+clover_status clover_linear(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
+                            int32_t *status, void *stream) {
+    if (R < 0 || N < 1 || K < 64 || K % 64 != 0) return CLOVER_ERR_INVALID_ARG;
+    if (mode < CLOVER_LINEAR_F32 || mode > CLOVER_LINEAR_RES) return CLOVER_ERR_INVALID_ARG;
+    const bool with_res = mode == CLOVER_LINEAR_RES_SILU || mode == CLOVER_LINEAR_RES;
+    if ((long)R * N > 0x7FFFFFFFL * 4L) return CLOVER_ERR_UNSUPPORTED;
+    if (R == 0) return CLOVER_OK;
+    if (!x || !w || !out || (with_res && !res)) return CLOVER_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(w) || !aligned16(out) || (with_res && !aligned16(res)))
+        return CLOVER_ERR_INVALID_ARG;
+    return from_cuda(launch_linear_tc(x, w, with_res ? res : nullptr, out, R, N, K, mode, status,
+                                      static_cast<cudaStream_t>(stream)));
+}
+
+clover_status clover_embed_rows(const void *w, const int32_t *tokens, void *e, int R, int V, int H, int32_t *status,
+                                void *stream) {
+    if (R < 0 || V < 1 || H < 1) return CLOVER_ERR_INVALID_ARG;
+    if (R == 0) return CLOVER_OK;
+    if (!w || !tokens || !e) return CLOVER_ERR_INVALID_ARG;
+    return from_cuda(launch_embed_rows(w, tokens, e, R, V, H, status, static_cast<cudaStream_t>(stream)));
+}
+
+size_t clover_topk_workspace_size(int R, int V, int k) {
+    if (R < 0 || V < 1 || k < 1 || k > topk_max_k() || k > V) return 0;
+    return topk_workspace_bytes(R > 0 ? R : 1, V, k);
+}
+
+clover_status clover_topk(const float *x, int R, int V, int k, float *values, int32_t *indices, void *workspace,
+                          size_t ws_bytes, int32_t *status, void *stream) {
+    if (R < 0 || V < 1 || k < 1 || k > V) return CLOVER_ERR_INVALID_ARG;
+    if (k > topk_max_k()) return CLOVER_ERR_UNSUPPORTED;
+    // the final merge holds two candidates a thread: chunks x k <= 512
+    if ((long)((V + 8191) / 8192) * k > 512) return CLOVER_ERR_UNSUPPORTED;
+    if (R == 0) return CLOVER_OK;
+    if (!x || !values || !indices) return CLOVER_ERR_INVALID_ARG;
+    if (ws_bytes < topk_workspace_bytes(R, V, k) || !workspace || (reinterpret_cast<uintptr_t>(workspace) & 7u))
+        return CLOVER_ERR_INVALID_ARG;
+    return from_cuda(launch_topk(x, R, V, k, values, indices, workspace, status, static_cast<cudaStream_t>(stream)));
 }
 
 clover_status clover_kv_commit_paged(void *k_pages, void *v_pages, const int32_t *block_table, int n_pages,

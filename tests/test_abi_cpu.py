@@ -185,6 +185,27 @@ def test_paged_host_validation(lib):
     assert commit(B=0) == 0
 
 
+def test_draft_host_validation(lib):
+    P = ctypes.c_void_p
+    lin = lambda R=4, N=128, K=64, mode=1, x=64, res=None, out=128: lib.clover_linear(
+        P(x), P(64), P(res) if res else None, P(out), R, N, K, mode, None, None)
+    assert lin(K=96) == 1 and lin(K=0) == 1 and lin(N=0) == 1 and lin(mode=4) == 1 and lin(mode=-1) == 1
+    assert lin(mode=2) == 1 and lin(mode=3) == 1             # residual modes need res
+    assert lin(x=72) == 1 and lin(out=136) == 1              # 16-byte alignment
+    assert lin(R=0) == 0
+    assert lib.clover_topk_workspace_size(3, 1000, 8) == 8 * 3 * 1 * 8 + 4 * 3
+    assert lib.clover_topk_workspace_size(3, 125696, 8) == 8 * 3 * 16 * 8 + 4 * 3
+    assert lib.clover_topk_workspace_size(1, 100, 33) == 0 and lib.clover_topk_workspace_size(1, 4, 5) == 0
+    tk = lambda R=2, V=1000, k=4, ws=64, wsb=1 << 20: lib.clover_topk(P(64), R, V, k, P(64), P(64), P(ws), wsb,
+                                                                     None, None)
+    assert tk(k=0) == 1 and tk(k=1001) == 1 and tk(k=33) == 2
+    assert tk(V=200000, k=32) == 2                          # 25 chunks x 32 candidates > 512
+    assert tk(ws=68) == 1 and tk(wsb=8) == 1
+    assert tk(R=0) == 0
+    emb = lambda R=2, V=10, H=8: lib.clover_embed_rows(P(64), P(64), P(64), R, V, H, None, None)
+    assert emb(V=0) == 1 and emb(H=0) == 1 and emb(R=-1) == 1 and emb(R=0) == 0
+
+
 def test_python_binding_rejects_cpu_tensors(lib):
     import paper_2405_00263_gb300 as pkg
     x = torch.zeros(1, 4, 2, 64, dtype=torch.bfloat16)

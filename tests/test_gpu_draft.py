@@ -1,0 +1,159 @@
+"""GPU parity of the draft side (Clover head step): clover_linear,
+clover_embed_rows, clover_topk and DraftHead against the oracle.
+
+Linear layer: the kernel multiplies bf16 exactly and sums in fp32, the oracle
+in fp64; the difference is bounded by a small multiple of the absolute sum
+A = sum_k |x_k w_k| (oracle.linear of |x| and |w|), and the bf16 epilogues add
+one rounding (half a bf16 unit, 2^-9 relative, here taken as 2^-8).  Top-k is
+bit-exact (it compares stored fp32 values).  The embedding is one bf16
+rounding of an fp32 normalisation.
+"""
+
+from __future__ import annotations
+
+import pytest
+import torch
+
+import oracle
+import paper_2405_00263_gb300 as pkg
+
+pytestmark = pytest.mark.gpu
+
+DEV = torch.device("cuda")
+BF = torch.bfloat16
+
+
+def rand(shape, g, std=1.0, dtype=BF):
+    return (torch.randn(*shape, generator=g, dtype=torch.float64) * std).to(dtype)
+
+
+def linear_tol(x, w, ref, bf16_out):
+    A = oracle.linear(x.abs(), w.abs())
+    return 1e-3 * A + (2.0 ** -8) * ref.abs() * (1 if bf16_out else 0) + 1e-6
+
+
+SHAPES = [
+    # R, N, K
+    (1, 128, 64),
+    (5, 127, 64),                 # N below one tile
+    (7, 300, 128),                # a tail tile
+    (16, 1000, 256),
+    (40, 257, 4096),
+    (200, 640, 512),
+    (256, 128, 64),               # the most rows of one launch
+    (300, 200, 128),              # two launches (256 + 44 rows)
+]
+
+
+@pytest.mark.parametrize("R,N,K", SHAPES)
+@pytest.mark.parametrize("mode", ["f32", "bf16", "res_silu", "res"])
+def test_linear_matches_oracle(R, N, K, mode):
+    g = torch.Generator().manual_seed(R * 7 + N + K)
+    x = rand((R, K), g)
+    w = rand((N, K), g, std=K ** -0.5)
+    res = rand((R, N), g) if mode in ("res_silu", "res") else None
+    act = 1 if mode == "res_silu" else 0
+    if mode == "res":
+        ref = oracle.linear(x, w) + res.double()
+    else:
+        ref = oracle.linear(x, w, res=res, act=act)
+    out = torch.empty((R, N), dtype=torch.float32 if mode == "f32" else BF, device=DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    pkg.clover_linear(x.to(DEV), w.to(DEV), out, res=None if res is None else res.to(DEV), mode=mode, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    err = (out.cpu().double() - ref).abs()
+    tol = linear_tol(x, w, ref, mode != "f32")
+    assert (err <= tol).all(), (err - tol).max().item()
+
+
+def test_linear_lm_head_full_size():
+    """The shared LM head of a 7B model: 16 rows against 125696 x 4096
+    weights, checked on sampled output columns (every tile's neighbourhood
+    and the tail)."""
+    g = torch.Generator().manual_seed(3)
+    R, N, K = 16, 125696, 4096
+    x = rand((R, K), g)
+    w = rand((N, K), g, std=K ** -0.5)
+    out = torch.empty((R, N), dtype=torch.float32, device=DEV)
+    pkg.clover_linear(x.to(DEV), w.to(DEV), out, mode="f32")
+    torch.cuda.synchronize()
+    cols = sorted(set([0, 127, 128, N - 1, N - 128] + torch.randint(0, N, (250,), generator=g).tolist()))
+    ref = oracle.linear(x, w[cols])
+    err = (out[:, cols].cpu().double() - ref).abs()
+    assert (err <= linear_tol(x, w[cols], ref, False)).all()
+
+
+@pytest.mark.parametrize("R,V,k", [(1, 1, 1), (3, 1000, 8), (4, 125696, 10), (2, 8193, 32), (5, 20000, 1),
+                                   (64, 32000, 16)])
+def test_topk_matches_oracle(R, V, k):
+    g = torch.Generator().manual_seed(V + k)
+    x = torch.randn(R, V, generator=g)
+    # planted ties (equal values at several indices), signed zeros, infinities
+    for r in range(R):
+        idx = torch.randperm(V, generator=g)[: min(V, 6)]
+        x[r, idx] = x[r].max() + 1.0
+        if V > 10:
+            x[r, 3] = -0.0
+            x[r, 7] = 0.0
+            x[r, 9] = -float("inf")
+    vals, ind = oracle.topk(x, k)
+    ws = torch.zeros(pkg.clover_topk_workspace_size(R, V, k), dtype=torch.uint8, device=DEV)
+    xd = x.to(DEV)
+    for _ in range(2):                                       # the workspace resets itself
+        v = torch.empty((R, k), dtype=torch.float32, device=DEV)
+        i = torch.empty((R, k), dtype=torch.int32, device=DEV)
+        pkg.clover_topk(xd, k, v, i, ws)
+        torch.cuda.synchronize()
+        assert torch.equal(i.cpu(), ind)
+        assert torch.equal(v.cpu().double(), vals)
+
+
+def test_embed_rows_and_invalid_token():
+    g = torch.Generator().manual_seed(9)
+    V, H = 5000, 4096
+    w = rand((V, H), g)
+    w[11] = 0
+    toks = torch.tensor([4, 4999, 0, 11, 4, 2500], dtype=torch.int32)
+    ref = oracle.embed_rows(w, toks)
+    e = torch.empty((len(toks), H), dtype=BF, device=DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    pkg.clover_embed_rows(w.to(DEV), toks.to(DEV), e, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert ((e.cpu().double() - ref).abs() <= (2.0 ** -8) * ref.abs() + 1e-6).all()
+    bad = toks.clone()
+    bad[2] = V
+    pkg.clover_embed_rows(w.to(DEV), bad.to(DEV), e, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & 1 and (e[2] == 0).all()
+
+
+@pytest.mark.parametrize("R,H,V,k", [(8, 512, 3000, 8), (48, 1024, 20000, 4)])
+def test_draft_head_step_matches_oracle(R, H, V, k):
+    g = torch.Generator().manual_seed(R + H)
+    h = rand((R, H), g)
+    toks = torch.randint(0, V, (R,), generator=g, dtype=torch.int32)
+    w_lm = rand((V, H), g, std=H ** -0.5)
+    w_v, w_o, w_1 = (rand((H, H), g, std=H ** -0.5) for _ in range(3))
+    ref = oracle.clover_head_step(h, toks, w_lm, w_v, w_o, w_1, k)
+    head = pkg.DraftHead(R, H, V, k, device=DEV)
+    head.run(h.to(DEV), toks.to(DEV), w_lm.to(DEV), w_v.to(DEV), w_o.to(DEV), w_1.to(DEV))
+    torch.cuda.synchronize()
+    assert int(head.status.item()) == 0
+    logits = head.logits.cpu().double()
+    # intermediate bf16 roundings may differ by one unit where the fp32 and
+    # fp64 sums straddle a rounding boundary; each such unit moves a logit by
+    # at most 2^-8 |z_j| |w_lm[v, j]|
+    tol = 1e-3 * oracle.linear(ref["z"].abs().to(BF), w_lm.abs()) + 1e-2 * ref["logits"].abs().mean()
+    err = (logits - ref["logits"]).abs()
+    assert (err <= tol).all(), (err - tol).max().item()
+    # top-k: the same indices wherever the oracle's ranking has clear gaps
+    srt = ref["logits"].sort(dim=-1, descending=True).values
+    for r in range(R):
+        gaps = (srt[r, :k] - srt[r, 1: k + 1]).abs()
+        if (gaps > 4 * tol[r].max()).all():
+            assert head.indices[r].cpu().tolist() == ref["top_indices"][r].tolist()
+        else:
+            got = head.indices[r].cpu().long()
+            assert ((ref["logits"][r, got] - ref["top_values"][r]).abs() <= 4 * tol[r].max()).all()
