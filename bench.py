@@ -490,6 +490,148 @@ def accept_kernel_us(pkg, w, sets, stream, device, rule, args, flush) -> float:
     return t
 
 
+DRAFT_METRIC = "Clover draft head steps/s (one speculative head: embedding, attention decoder, MLP block, " \
+               "shared LM head, top-k) and LM-head achieved HBM GB/s at 1 GPU"
+DRAFT_UNIT = "head steps/s"
+
+
+def run_draft_arm(args, world, rank, local, dist):
+    """One speculative head step of a 7B-class Clover draft on R rows: the
+    weights are synthetic (seeded normal, std 1/sqrt(H)); the LM head alone
+    is 1.03 GB of bf16, so every step streams its weights from HBM."""
+    import paper_2405_00263_gb300 as pkg
+
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    R, H, V, k = args.draft, 4096, 125696, 8
+    gen = torch.Generator(device=device).manual_seed(1234 + rank)
+
+    def rnd(*shape, std=1.0):
+        return (torch.randn(*shape, generator=gen, device=device, dtype=torch.float32) * std).to(torch.bfloat16)
+
+    w_lm = rnd(V, H, std=H ** -0.5)
+    w_v, w_o, w_1 = (rnd(H, H, std=H ** -0.5) for _ in range(3))
+    h = rnd(R, H)
+    toks = torch.randint(0, V, (R,), generator=gen, device=device, dtype=torch.int32)
+    head = pkg.DraftHead(R, H, V, k, device=device)
+    stream = torch.cuda.Stream(device)
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            head.run(h, toks, w_lm, w_v, w_o, w_1, stream=stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        head.run(h, toks, w_lm, w_v, w_o, w_1, stream=stream)
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            g.replay()
+    torch.cuda.synchronize(device)
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(dist, device)
+    torch.cuda.synchronize(device)
+    if sampler:
+        sampler.mark("t0")
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for _ in range(args.steps):
+            g.replay()
+        end.record(stream)
+    end.synchronize()
+    if sampler:
+        sampler.mark("t1")
+    barrier(dist, device)
+    clocks = sampler.stop() if sampler else None
+    seconds_max = max_over_ranks(dist, start.elapsed_time(end) / 1e3, device)
+    value, ms = aggregate(seconds_max, args.steps, world)
+    if int(head.status.item()) != 0:
+        raise RuntimeError(f"device status {int(head.status.item())} in the draft timing")
+
+    # the LM head alone: events around one launch (its 1 GB read keeps the L2 cold)
+    flush = torch.zeros(2 * L2_BYTES, dtype=torch.uint8, device=device)
+    lm_us = isolated_us(lambda i: pkg.clover_linear(head.z, w_lm, head.logits, mode="f32", stream=stream),
+                        10, stream, flush)
+    topk_us = isolated_us(lambda i: pkg.clover_topk(head.logits, k, head.values, head.indices, head.ws,
+                                                    stream=stream), 10, stream, flush)
+    del flush
+    peaks, peak_kind = measured_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    lm_bytes = V * H * 2 + R * H * 2 + R * V * 4
+    achieved = lm_bytes / (lm_us * 1e-6) / 1e9
+
+    # end to end: h and the tokens from pinned host memory, the top-k back
+    h_host = h.cpu().pin_memory()
+    t_host = toks.cpu().pin_memory()
+    out_host = torch.empty((R, k), dtype=torch.int32).pin_memory()
+    h_dev, t_dev = torch.empty_like(h), torch.empty_like(toks)
+
+    def e2e_step():
+        h_dev.copy_(h_host, non_blocking=True)
+        t_dev.copy_(t_host, non_blocking=True)
+        head.run(h_dev, t_dev, w_lm, w_v, w_o, w_1, stream=stream)
+        out_host.copy_(head.indices, non_blocking=True)
+
+    n = max(10, min(args.steps, 200))
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            e2e_step()
+    stream.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(n):
+            e2e_step()
+        e1.record(stream)
+    e1.synchronize()
+    e_val, e_ms = aggregate(max_over_ranks(dist, e0.elapsed_time(e1) / 1e3, device), n, world)
+
+    line = {
+        "metric": DRAFT_METRIC, "value": value, "unit": DRAFT_UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded normal weights, std 1/sqrt(H))",
+        "config": {"workload": f"Clover head step, 7B shapes: R{R} rows, H{H}, V{V}, top-{k}",
+                   "R": R, "H": H, "V": V, "k": k, "parallelism": f"replicas x{world} (one per GPU)",
+                   "l2": "the 1.03 GB LM head is read every step (more than 7x the 129 MB L2)",
+                   "launch": "one CUDA graph replay per step: embedding, 4 tcgen05 linear layers "
+                             "(W_v, W_o + residual, W_1 residual SiLU, LM head), top-k"},
+        "roofline": {"bound": "hbm", "kernel": "linear_tc (LM head)", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": achieved / hbm,
+                     "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)" if peak_kind == "measured"
+                     else "fallback 6.8 TB/s", "traffic": None, "bytes_per_launch": lm_bytes,
+                     "launch_us": lm_us, "flops_per_launch": 2 * R * V * H,
+                     "timing": "launched alone after an L2 flush by a large read, events on the launching stream"},
+        "kernels": {"lm_head_us": lm_us, "topk_us": topk_us,
+                    "topk_gbs": R * V * 4 / (topk_us * 1e-6) / 1e9},
+        "gpu_launches": 6 * args.steps,
+        "clocks": clocks,
+        "e2e": {"value": e_val, "unit": DRAFT_UNIT, "h2d_bytes_per_step": R * H * 2 + R * 4,
+                "d2h_bytes_per_step": R * k * 4, "steps": n, "ms_per_step": e_ms,
+                "api": "paper_2405_00263_gb300.DraftHead.run (C ABI)"},
+    }
+    return line, (R, H, V, k, w_lm, w_v, w_o, w_1, h, toks)
+
+
+def draft_cpu_baseline(inputs, budget_s: float = 8.0) -> dict:
+    """The oracle's head step for one row of the same weights (host cores),
+    its layers on a tenth of their outputs, scaled to whole layers and to R
+    rows (every row costs the same)."""
+    import oracle
+    oracle.build()
+    sampler = DraftOracleSampler([t.cpu() if isinstance(t, torch.Tensor) else t for t in inputs])
+    times = []
+    while not times or (sum(times) < budget_s and len(times) < 20):
+        t0 = time.perf_counter()
+        times.append(sampler.seconds(0.1))
+        if time.perf_counter() - t0 > budget_s:
+            break
+    per = statistics.median(times)
+    return {"value": 1.0 / per, "unit": DRAFT_UNIT, "cores": os.cpu_count() or 1, "kind": "oracle",
+            "sample": f"{len(times)} oracle head steps of 1 row, layers on a 0.1 fraction of their outputs, "
+                      f"scaled to whole layers and to {inputs[0]} rows; median {per:.2f} s a step"}
+
+
 def run_e2e(args, w, step, sets, stream, device, dist, world):
     """Same steps through the public API: inputs copied from pinned host memory,
     the step's results (attention output, path, accepted length, bonus token,
@@ -551,6 +693,65 @@ def oracle_step_seconds(host: dict, threads: int, typical=None) -> float:
     return time.perf_counter() - t0
 
 
+class OracleSampler:
+    """Times the oracle's verify step on a bounded sample of the workload and
+    scales it to the whole step: the attention on a fraction f of the query
+    rows, the argmax on a fraction of the logit rows (typical acceptance: the
+    first fraction of the vocabulary, its cost being linear in V), the walk,
+    the append and the compaction in full (they are small).  f = 1 times the
+    whole oracle step (oracle.verify_step)."""
+
+    def __init__(self, host: dict, threads: int, typical=None):
+        import oracle
+        self.oracle = oracle
+        self.host, self.threads, self.typ = host, threads, typical
+        B, T, Hq, _ = host["q"].shape
+        self.n_rows = B * T * Hq
+        self.n_logit_rows = B * T
+        self.V = host["logits"].shape[-1]
+        self.amax = oracle.argmax(host["logits"], n_threads=threads)
+        self.sub_logits = {}
+        # caches the sampled append and compaction write into (their contents
+        # do not matter for the time; the lengths are reset every step)
+        self.kc, self.vc = host["k_cache"].clone(), host["v_cache"].clone()
+
+    def step_seconds(self, f: float) -> float:
+        if f >= 1.0:
+            return oracle_step_seconds(self.host, self.threads, self.typ)
+        o, h, th = self.oracle, self.host, self.threads
+        # at least one row a thread, so that a sample runs as parallel as the whole
+        ra = min(self.n_rows, max(th, round(f * self.n_rows)))
+        t0 = time.perf_counter()
+        o.tree_attention(h["q"], h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["cache_len"], h["parent"],
+                         rows=list(range(ra)), n_threads=th)
+        t_attn = (time.perf_counter() - t0) * self.n_rows / ra
+        if self.typ is None:
+            rl = min(self.n_logit_rows, max(th, round(f * self.n_logit_rows)))
+            t0 = time.perf_counter()
+            o.argmax(h["logits"], rows=list(range(rl)), n_threads=th)
+            t_acc = (time.perf_counter() - t0) * self.n_logit_rows / rl
+            t0 = time.perf_counter()
+            path, alen, _ = o.accept_walk(h["parent"], h["cand"], self.amax)
+            t_acc += time.perf_counter() - t0
+        else:
+            vs = max(1, round(f * self.V))
+            if vs not in self.sub_logits:
+                self.sub_logits[vs] = h["logits"][..., :vs].contiguous()
+            t0 = time.perf_counter()
+            r = o.accept_typical(self.sub_logits[vs], h["parent"], h["cand"], *self.typ, n_threads=th)
+            t_acc = (time.perf_counter() - t0) * self.V / vs
+            path, alen = r["path"], r["accept_len"]
+        cl = h["cache_len"].clone().to(torch.int32)
+        t0 = time.perf_counter()
+        o.append_tree_kv(h["k_new"], h["v_new"], self.kc, self.vc, cl)
+        o.kv_compact(self.kc, self.vc, cl, path, alen)
+        return t_attn + t_acc + time.perf_counter() - t0
+
+
+def sample_fraction(t_full: float, n_steps: int, budget_s: float) -> float:
+    return min(1.0, budget_s / max(1e-9, n_steps * t_full))
+
+
 def cpu_baseline(w, host: dict, args, budget_s: float = 8.0) -> dict:
     """Whole oracle verify steps (fp64 attention over every row, argmax over
     every logit row, walk, append, compaction) repeated within a time budget."""
@@ -567,30 +768,108 @@ def cpu_baseline(w, host: dict, args, budget_s: float = 8.0) -> dict:
                       f"and logit rows, {accept_desc(args)}), median {per * 1e3:.1f} ms per step"}
 
 
-def run_reference_arm(args, world, rank):
+def run_reference_arm(args, world, rank, budget_s: float = 120.0):
+    """The oracle on the host cores: `--steps` timed steps after `--warmup`,
+    each one a bounded sample of the workload (OracleSampler, or one row of a
+    draft head step) scaled to the whole step, so that the run stays within
+    about `budget_s` seconds whatever the step count."""
     from synth import workloads
     if rank != 0:
         return None
-    w = workloads.get(args.workload)
-    host = workloads.make(w)
     import oracle
     oracle.build()
     threads = os.cpu_count() or 1
+    if args.draft:
+        return run_reference_draft(args, world, threads, budget_s)
+    w = workloads.get(args.workload)
+    host = workloads.make(w)
     typ = typical_params(args)
+    sampler = OracleSampler(host, threads, typ)
+    t_full = sampler.step_seconds(1.0)
+    f = sample_fraction(t_full, args.steps + args.warmup, budget_s)
     for _ in range(args.warmup):
-        oracle_step_seconds(host, threads, typ)
-    t = [oracle_step_seconds(host, threads, typ) for _ in range(args.steps)]
+        sampler.step_seconds(f)
+    t = [sampler.step_seconds(f) for _ in range(args.steps)]
     total = sum(t)
     value = args.steps / total
+    sample = (f"{args.steps} verify steps of {w.name} (fp64 oracle, OpenMP), each timed on "
+              + ("the whole step" if f >= 1.0 else f"a {f:.2e} fraction of the attention rows and of the logit "
+                 "rows (vocabulary for typical acceptance), scaled to the whole step; walk, append and "
+                 "compaction in full"))
     return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f64", "data": "synthetic",
             "config": {"workload": f"{w.name}: {w.description}", "parallelism": "host cores (rank 0 only)",
                        "accept": accept_desc(args)},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
-                             "sample": f"{args.steps} whole verify steps of {w.name} on the host (fp64 oracle)"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+
+
+class DraftOracleSampler:
+    """Times the oracle's head step on a bounded sample: one row, every layer on
+    a fraction f of its output features (the LM head and the top-k on that
+    fraction of the vocabulary), each scaled to the whole layer, the total to
+    R rows.  Each layer's input is the full one, computed once."""
+
+    def __init__(self, inputs):
+        import oracle
+        self.o = oracle
+        self.R, self.H, self.V, self.k, self.w_lm, self.w_v, self.w_o, self.w_1, h, toks = inputs
+        bf = torch.bfloat16
+        self.toks = toks[:1]
+        self.e = oracle.embed_rows(self.w_lm, self.toks).to(bf)
+        self.a = oracle.linear(self.e, self.w_v).to(bf)
+        self.h1 = (h[:1].double() + oracle.linear(self.a, self.w_o)).to(bf)
+        self.z = oracle.linear(self.h1, self.w_1, res=self.h1, act=1).to(bf)
+
+    def seconds(self, f: float) -> float:
+        o, H, V = self.o, self.H, self.V
+        th = os.cpu_count() or 1
+        # at least a few outputs a thread, so that a sample runs as parallel as the whole
+        ns = min(H, max(4 * th, round(f * H)))
+        vs = min(V, max(self.k, 4 * th, round(f * V)))
+        t0 = time.perf_counter()
+        o.embed_rows(self.w_lm, self.toks)
+        t = time.perf_counter() - t0
+        t0 = time.perf_counter()
+        o.linear(self.e, self.w_v[:ns])
+        o.linear(self.a, self.w_o[:ns])
+        o.linear(self.h1, self.w_1[:ns], res=self.h1[:, :ns].contiguous(), act=1)
+        t += (time.perf_counter() - t0) * H / ns
+        t0 = time.perf_counter()
+        logits = o.linear(self.z, self.w_lm[:vs])
+        o.topk(logits, self.k)
+        t += (time.perf_counter() - t0) * V / vs
+        return t * self.R
+
+
+def run_reference_draft(args, world, threads, budget_s):
+    R, H, V, k = args.draft, 4096, 125696, 8
+    g = torch.Generator().manual_seed(1234)
+    rnd = lambda *sh, std=1.0: (torch.randn(*sh, generator=g) * std).to(torch.bfloat16)
+    w_lm = rnd(V, H, std=H ** -0.5)
+    w_v, w_o, w_1 = (rnd(H, H, std=H ** -0.5) for _ in range(3))
+    inputs = (R, H, V, k, w_lm, w_v, w_o, w_1, rnd(R, H), torch.randint(0, V, (R,), generator=g, dtype=torch.int32))
+    sampler = DraftOracleSampler(inputs)
+    t_row = sampler.seconds(0.01) / R                  # one row of a whole step, estimated
+    f = sample_fraction(t_row, args.steps + args.warmup, budget_s)
+    for _ in range(args.warmup):
+        sampler.seconds(f)
+    t = [sampler.seconds(f) for _ in range(args.steps)]
+    total = sum(t)
+    value = args.steps / total
+    sample = (f"{args.steps} head steps, each timed on 1 row with every layer (the LM head and top-k included) "
+              f"on a {f:.2e} fraction of its outputs, scaled to whole layers and to {R} rows (fp64 oracle, OpenMP)")
+    return {"impl": "reference", "metric": DRAFT_METRIC, "value": value, "unit": DRAFT_UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"Clover head step, 7B shapes: R{R} rows, H{H}, V{V}, top-{k}",
+                       "parallelism": "host cores (rank 0 only)"},
+            "cpu_baseline": {"value": value, "unit": DRAFT_UNIT, "cores": threads, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": DRAFT_UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}
 
 
@@ -604,6 +883,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],
                     help="acceptance rule of the step (typical: tempered softmax with an entropy threshold)")
+    ap.add_argument("--draft", type=int, default=0,
+                    help="time one Clover draft head step on this many rows (7B shapes) instead of verification")
     ap.add_argument("--page-size", type=int, default=0,
                     help="run on a paged KV cache with pages of this many slots (0: dense cache)")
     ap.add_argument("--schedule", default="commit", choices=["commit", "compact", "fused"],
@@ -623,6 +904,14 @@ def main(argv=None):
         return 0
 
     dist = dist_init(world, "nccl" if torch.cuda.is_available() else "gloo")
+    if args.draft:
+        line, inputs = run_draft_arm(args, world, rank, local, dist)
+        if rank == 0:
+            line["cpu_baseline"] = draft_cpu_baseline(inputs) if world == 1 and not args.no_cpu_baseline else None
+            print(json.dumps(line), flush=True)
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
     line, w, base = run_gpu_arm(args, world, rank, local, dist)
     if rank == 0:
         if world == 1 and not args.no_cpu_baseline:
