@@ -214,12 +214,21 @@ CLOVER_API clover_status clover_kv_commit_paged(void *k_pages, void *v_pages, co
  * features), res [R,N] (modes 2-3; else may be NULL), out [R,N] (fp32 for
  * CLOVER_LINEAR_F32, else bf16).  Rounding: one fp32 accumulation, then one
  * rounding to bf16 (after the residual and SiLU) for the bf16 modes.
- * K a multiple of 64 (16 <= K); R >= 0, N >= 1; x, w, res, out 16-byte
+ * K a multiple of 64 (64 <= K); R >= 0, N >= 1; x, w, res, out 16-byte
  * aligned; out must not overlap x, w or res.  A bounded device wait that gives
  * up raises CLOVER_ERR_TIMEOUT (device bit).
+ * workspace, ws_bytes: with at least clover_linear_workspace_size(R, N, K)
+ * bytes (16-byte aligned, zero-filled before first use, left ready for the
+ * next call; calls sharing it must not overlap on the device), a layer of at
+ * most 32 rows with fewer 128-row weight tiles than a GB300 has SMs splits K
+ * over more CTAs and sums the parts in a fixed order; with NULL (or a smaller
+ * one), or more rows, it does not (the size is then 0).
+ * The result is the same function either way (the fp32 summation order differs).
  */
+CLOVER_API size_t clover_linear_workspace_size(int R, int N, int K);
 CLOVER_API clover_status clover_linear(const void *x, const void *w, const void *res, void *out,
-                                   int R, int N, int K, int mode, int32_t *status, void *stream);
+                                   int R, int N, int K, int mode, void *workspace, size_t ws_bytes,
+                                   int32_t *status, void *stream);
 
 /*
  * The regressive connection's embedding (Section 3.4): e[r] = w[t[r]] / ||w[t[r]]||_2

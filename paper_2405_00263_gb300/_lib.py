@@ -35,6 +35,7 @@ EXPORTS = (
     "clover_verify_attn_paged_workspace_size",
     "clover_verify_attn_paged",
     "clover_kv_commit_paged",
+    "clover_linear_workspace_size",
     "clover_linear",
     "clover_embed_rows",
     "clover_topk_workspace_size",
@@ -118,7 +119,9 @@ def load(build_if_missing: bool = False):
         lib.clover_verify_attn_paged.restype = I
         lib.clover_kv_commit_paged.argtypes = [P, P, P, I, I, I, P, P, P, P, P, P, P, I, I, I, I, I, P, P]
         lib.clover_kv_commit_paged.restype = I
-        lib.clover_linear.argtypes = [P, P, P, P, I, I, I, I, P, P]
+        lib.clover_linear_workspace_size.argtypes = [I, I, I]
+        lib.clover_linear_workspace_size.restype = Z
+        lib.clover_linear.argtypes = [P, P, P, P, I, I, I, I, P, Z, P, P]
         lib.clover_linear.restype = I
         lib.clover_embed_rows.argtypes = [P, P, P, I, I, I, P, P]
         lib.clover_embed_rows.restype = I

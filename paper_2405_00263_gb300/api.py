@@ -361,10 +361,15 @@ def clover_verify_accept_ex(logits, cand, parent, argmax_out, path_out, accept_l
 _LINEAR_MODES = {"f32": 0, "bf16": 1, "res_silu": 2, "res": 3}
 
 
-def clover_linear(x, w, out, res=None, mode="bf16", status=None, stream=None):
+def clover_linear_workspace_size(R, N, K) -> int:
+    return int(_lib.load().clover_linear_workspace_size(R, N, K))
+
+
+def clover_linear(x, w, out, res=None, mode="bf16", workspace=None, status=None, stream=None):
     """out = x . w^T (fp32 accumulation) with the epilogue `mode`: "f32" (fp32
     out), "bf16", "res_silu" (res + silu(.)), "res" (res + .); x [R,K], w [N,K],
-    res/out [R,N]."""
+    res/out [R,N].  With a workspace of clover_linear_workspace_size bytes a
+    layer with few weight tiles splits K over more CTAs."""
     code = _LINEAR_MODES[mode]
     R, K = x.shape
     N = w.shape[0]
@@ -375,9 +380,10 @@ def clover_linear(x, w, out, res=None, mode="bf16", status=None, stream=None):
         _check(res, (R, N), torch.bfloat16, "res")
     if status is not None:
         _check(status, (1,), torch.int32, "status")
-    _dev(x, w, out, res if code >= 2 else None, status)
+    _dev(x, w, out, res if code >= 2 else None, workspace, status)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     rc = _lib.load().clover_linear(_ptr(x), _ptr(w), _ptr(res if code >= 2 else None), _ptr(out), R, N, K, code,
-                                   _ptr(status), _stream(stream))
+                                   _ptr(workspace), ws_bytes, _ptr(status), _stream(stream))
     if rc != OK:
         raise CloverError(rc, "clover_linear")
 
@@ -437,15 +443,17 @@ class DraftHead:
         self.values = torch.empty((R, k), dtype=torch.float32, device=dev)
         self.indices = torch.empty((R, k), dtype=torch.int32, device=dev)
         self.ws = torch.zeros(max(16, clover_topk_workspace_size(R, V, k)), dtype=torch.uint8, device=dev)
+        # the three H x H layers (run one after another) share one split workspace
+        self.ws_lin = torch.zeros(max(16, clover_linear_workspace_size(R, H, H)), dtype=torch.uint8, device=dev)
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.k = k
 
     def run(self, h, tokens, w_lm, w_v, w_o, w_1, stream=None):
         st = dict(status=self.status, stream=stream)
         clover_embed_rows(w_lm, tokens, self.e, **st)
-        clover_linear(self.e, w_v, self.v, mode="bf16", **st)
-        clover_linear(self.v, w_o, self.h, res=h, mode="res", **st)
-        clover_linear(self.h, w_1, self.z, res=self.h, mode="res_silu", **st)
+        clover_linear(self.e, w_v, self.v, mode="bf16", workspace=self.ws_lin, **st)
+        clover_linear(self.v, w_o, self.h, res=h, mode="res", workspace=self.ws_lin, **st)
+        clover_linear(self.h, w_1, self.z, res=self.h, mode="res_silu", workspace=self.ws_lin, **st)
         clover_linear(self.z, w_lm, self.logits, mode="f32", **st)
         clover_topk(self.logits, self.k, self.values, self.indices, self.ws, **st)
 

@@ -16,7 +16,8 @@ void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk);
 size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype);
 cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
-                             int32_t *status, cudaStream_t stream);
+                             void *workspace, size_t ws_bytes, int32_t *status, cudaStream_t stream);
+size_t linear_workspace_bytes(int R, int N, int K);
 size_t topk_workspace_bytes(int R, int V, int k);
 int topk_max_k();
 cudaError_t launch_topk(const float *x, int R, int V, int k, float *values, int32_t *indices, void *workspace,
@@ -408,8 +409,13 @@ clover_status clover_kv_commit(void *k_cache, void *v_cache, const void *k_new, 
                                        static_cast<cudaStream_t>(stream)));
 }
 
+size_t clover_linear_workspace_size(int R, int N, int K) {
+    if (R < 0 || N < 1 || K < 64 || K % 64 != 0) return 0;
+    return linear_workspace_bytes(R > 0 ? R : 1, N, K);
+}
+
 clover_status clover_linear(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
-                            int32_t *status, void *stream) {
+                            void *workspace, size_t ws_bytes, int32_t *status, void *stream) {
     if (R < 0 || N < 1 || K < 64 || K % 64 != 0) return CLOVER_ERR_INVALID_ARG;
     if (mode < CLOVER_LINEAR_F32 || mode > CLOVER_LINEAR_RES) return CLOVER_ERR_INVALID_ARG;
     const bool with_res = mode == CLOVER_LINEAR_RES_SILU || mode == CLOVER_LINEAR_RES;
@@ -418,7 +424,8 @@ clover_status clover_linear(const void *x, const void *w, const void *res, void 
     if (!x || !w || !out || (with_res && !res)) return CLOVER_ERR_INVALID_ARG;
     if (!aligned16(x) || !aligned16(w) || !aligned16(out) || (with_res && !aligned16(res)))
         return CLOVER_ERR_INVALID_ARG;
-    return from_cuda(launch_linear_tc(x, w, with_res ? res : nullptr, out, R, N, K, mode, status,
+    if (workspace && !aligned16(workspace)) return CLOVER_ERR_INVALID_ARG;
+    return from_cuda(launch_linear_tc(x, w, with_res ? res : nullptr, out, R, N, K, mode, workspace, ws_bytes, status,
                                       static_cast<cudaStream_t>(stream)));
 }
 

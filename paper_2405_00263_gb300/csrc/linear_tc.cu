@@ -32,6 +32,7 @@ constexpr int kThreadsL = 192;             // producer, MMA, 4 epilogue warps
 constexpr int kProducer = 0;
 constexpr int kMma = 1;
 constexpr uint64_t kWaitL = 500000000ull;  // 0.5 s
+constexpr int kMaxSplit = 8;               // K ranges per tile pair at most
 
 struct LinSmem {
     static constexpr int w_bytes = LM * LK * 2;                      // one weight tile's stage: 16 KB
@@ -50,10 +51,28 @@ struct LinArgs {
     void *out;                             // [R, N]: fp32 (mode 0) or bf16
     int R, Rp, N, K, mode;
     int n_tiles;                           // ceil(N / LM)
+    // split K (n_split > 1): CTA = (tile pair, K range); fp32 partials in
+    // part [n_split, R, N], one arrival counter per tile pair
+    int n_split;
+    float *part;
+    unsigned *counters;
     int32_t *status;
 };
 
+// The epilogue of one output element from its fp32 sum.
+__device__ __forceinline__ void store_out(const LinArgs &a, size_t o, float y);
+
 __device__ __forceinline__ float silu(float v) { return v / (1.f + ex2_approx(-v * 1.4426950408889634f)); }
+
+__device__ __forceinline__ void store_out(const LinArgs &a, size_t o, float y) {
+    if (a.mode == CLOVER_LINEAR_F32) {
+        static_cast<float *>(a.out)[o] = y;
+        return;
+    }
+    if (a.mode == CLOVER_LINEAR_RES_SILU) y = __bfloat162float(a.res[o]) + silu(y);
+    else if (a.mode == CLOVER_LINEAR_RES) y = __bfloat162float(a.res[o]) + y;
+    static_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(y);
+}
 
 __global__ void __launch_bounds__(kThreadsL, 1)
     linear_tc_kernel(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_x,
@@ -71,10 +90,15 @@ __global__ void __launch_bounds__(kThreadsL, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    // this CTA's tiles [t0, t1), walked in pairs
-    const int t0 = (int)((long)blockIdx.x * a.n_tiles / gridDim.x);
-    const int t1 = (int)((long)(blockIdx.x + 1) * a.n_tiles / gridDim.x);
+    // this CTA's tiles [t0, t1), walked in pairs, and its K chunks [c_lo, c_hi)
     const int n_chunks = a.K / LK;
+    const bool split = a.n_split > 1;
+    const int pair = blockIdx.x / a.n_split;
+    const int ks = blockIdx.x % a.n_split;
+    const int t0 = split ? 2 * pair : (int)((long)blockIdx.x * a.n_tiles / gridDim.x);
+    const int t1 = split ? min(a.n_tiles, 2 * pair + 2) : (int)((long)(blockIdx.x + 1) * a.n_tiles / gridDim.x);
+    const int c_lo = split ? ks * n_chunks / a.n_split : 0;
+    const int c_hi = split ? (ks + 1) * n_chunks / a.n_split : n_chunks;
     // accumulator of tile h at TMEM columns [h * RS, h * RS + Rp); the
     // epilogue reads 32 columns at a time, so RS and the allocation are whole
     // multiples of 32 covering both
@@ -110,7 +134,7 @@ __global__ void __launch_bounds__(kThreadsL, 1)
         for (int t = t0; t < t1 && !*s_abort; t += 2) {
             const bool two = t + 1 < t1;
             const uint32_t bytes = (uint32_t)((two ? 2 : 1) * S::w_bytes + a.Rp * LK * 2);
-            for (int c = 0; c < n_chunks; ++c, ++it) {
+            for (int c = c_lo; c < c_hi; ++c, ++it) {
                 const int s = it % kStages;
                 if (!mbar_wait(&empty[s], ((it / kStages) - 1) & 1, kWaitL)) {
                     *s_abort = 1;
@@ -138,7 +162,7 @@ __global__ void __launch_bounds__(kThreadsL, 1)
             }
             tc_fence_after();
             bool ok = true;
-            for (int c = 0; c < n_chunks; ++c, ++it) {
+            for (int c = c_lo; c < c_hi; ++c, ++it) {
                 const int s = it % kStages;
                 if (!mbar_wait(&full[s], (it / kStages) & 1, kWaitL)) {
                     ok = false;
@@ -149,9 +173,9 @@ __global__ void __launch_bounds__(kThreadsL, 1)
 #pragma unroll
                 for (int k = 0; k < LK / 16; ++k) {
                     const uint64_t bd = sdesc_sw128(st + 2 * S::w_bytes + k * 32, 16, 1024);
-                    mma_bf16(tmem, sdesc_sw128(st + k * 32, 16, 1024), bd, idesc, (c | k) != 0);
+                    mma_bf16(tmem, sdesc_sw128(st + k * 32, 16, 1024), bd, idesc, (c - c_lo) + k != 0);
                     if (two) mma_bf16(tmem + RS, sdesc_sw128(st + S::w_bytes + k * 32, 16, 1024), bd, idesc,
-                                      (c | k) != 0);
+                                      (c - c_lo) + k != 0);
                 }
                 mma_commit(&empty[s]);         // the stage is free once these MMAs have read it
             }
@@ -193,14 +217,8 @@ __global__ void __launch_bounds__(kThreadsL, 1)
                             const int r = c0 + c;
                             if (r >= a.R) break;
                             const size_t o = (size_t)r * a.N + n;
-                            float y = v[c];
-                            if (a.mode == CLOVER_LINEAR_F32) {
-                                static_cast<float *>(a.out)[o] = y;
-                                continue;
-                            }
-                            if (a.mode == CLOVER_LINEAR_RES_SILU) y = __bfloat162float(a.res[o]) + silu(y);
-                            else if (a.mode == CLOVER_LINEAR_RES) y = __bfloat162float(a.res[o]) + y;
-                            static_cast<__nv_bfloat16 *>(a.out)[o] = __float2bfloat16_rn(y);
+                            if (split) a.part[(size_t)ks * a.R * a.N + o] = v[c];    // this K range's partial
+                            else store_out(a, o, v[c]);
                         }
                     }
                 }
@@ -208,6 +226,51 @@ __global__ void __launch_bounds__(kThreadsL, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(acc_empty);
+            if (split) {
+                // this warp's rows (quadrant `quad` of both tiles) are its own:
+                // the last K range to finish them, by a per-(pair, quadrant)
+                // arrival counter, sums the partials in split order (the
+                // result does not depend on the arrival order)
+                __threadfence();
+                __syncwarp();
+                unsigned last = 0;
+                if (lane == 0) {
+                    unsigned *cnt = a.counters + pair * 4 + quad;
+                    last = atomicAdd(cnt, 1u) == (unsigned)a.n_split - 1u;
+                    if (last) {
+                        *cnt = 0u;                                          // ready for the next call
+                        __threadfence();
+                    }
+                }
+                if (__shfl_sync(0xffffffffu, last, 0)) {
+                    __threadfence();
+                    // 8 rows a round: all their partials are loaded at once,
+                    // then summed in split order
+                    constexpr int RB = 8;
+                    const size_t plane = (size_t)a.R * a.N;
+                    for (int half = 0; half < (two ? 2 : 1); ++half) {
+                        const int n = (t + half) * LM + m;
+                        if (n >= a.N) continue;
+                        for (int r0 = 0; r0 < a.R; r0 += RB) {
+                            float p[kMaxSplit][RB];
+#pragma unroll
+                            for (int q = 0; q < kMaxSplit; ++q)
+#pragma unroll
+                                for (int j = 0; j < RB; ++j)
+                                    p[q][j] = (q < a.n_split && r0 + j < a.R)
+                                                  ? __ldcg(a.part + q * plane + (size_t)(r0 + j) * a.N + n) : 0.f;
+#pragma unroll
+                            for (int j = 0; j < RB; ++j) {
+                                if (r0 + j >= a.R) break;
+                                float y = 0.f;
+#pragma unroll
+                                for (int q = 0; q < kMaxSplit; ++q) y += p[q][j];
+                                store_out(a, (size_t)(r0 + j) * a.N + n, y);
+                            }
+                        }
+                    }
+                }
+            }
         }
     }
 
@@ -233,9 +296,41 @@ __global__ void __launch_bounds__(kThreadsL, 1)
 
 int linear_max_rows() { return kMaxRows; }
 
-// One launch per slice of at most kMaxRows rows of x.
+constexpr int kSmsPlan = 152;              // SMs of a GB300 (planning constant; any GPU runs the plan)
+
+// K ranges per tile pair: a layer with fewer weight tiles than SMs splits K so
+// that about one CTA per SM streams it (at least 4 stages of K per range).
+// The ranges' sum costs one L2 round trip per 8 rows at the end; measured at
+// H = 4096 it pays off up to 32 rows (a head step at R = 4: 287 -> 252 us,
+// R = 16: 303 -> 288 us) and not at 48 (355 -> 410 us).
+constexpr int kSplitMaxRows = 32;
+
+int linear_split(int R, int N, int K) {
+    const int n_tiles = (N + LM - 1) / LM;
+    if (n_tiles >= kSmsPlan || R > kSplitMaxRows) return 1;
+    const int n_pairs = (n_tiles + 1) / 2;
+    int s = kSmsPlan / n_pairs;
+    s = min(s, (K / LK) / 4);
+    s = min(s, kMaxSplit);
+    return s < 1 ? 1 : s;
+}
+
+// Partials of one launch (at most kMaxRows rows) and the per-(pair, quadrant)
+// counters, 16-byte aligned.
+size_t linear_workspace_bytes(int R, int N, int K) {
+    const int s = linear_split(R, N, K);
+    if (s <= 1) return 0;
+    const int rows = min(R, kMaxRows);
+    const int n_pairs = ((N + LM - 1) / LM + 1) / 2;
+    const size_t part = ((size_t)s * rows * N * 4 + 15) / 16 * 16;
+    return part + sizeof(unsigned) * 4 * (size_t)n_pairs;
+}
+
+// One launch per slice of at most kMaxRows rows of x.  With a workspace of
+// linear_workspace_bytes(R, N, K) bytes (zero-filled before first use) the
+// plan's K split is used; without one, none.
 cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
-                             int32_t *status, cudaStream_t stream) {
+                             void *workspace, size_t ws_bytes, int32_t *status, cudaStream_t stream) {
     static unsigned char done[64];
     static int sms[64];
     cudaError_t err = ensure_smem_attr(linear_tc_kernel, LinSmem::alloc, done);
@@ -246,6 +341,9 @@ cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void
     if (n_sm == 0 && (err = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return err;
     const int n_tiles = (N + LM - 1) / LM;
+    const int n_pairs = (n_tiles + 1) / 2;
+    const size_t need = linear_workspace_bytes(R, N, K);
+    const int n_split = (need > 0 && workspace && ws_bytes >= need) ? linear_split(R, N, K) : 1;
     const size_t out_elem = mode == CLOVER_LINEAR_F32 ? 4 : 2;
     CUtensorMap tw;
     if (!make_tmap_bf16_3d(&tw, w, K, N, 1, (uint64_t)K * 2, (uint64_t)N * K * 2, LK, LM, 1)) return cudaErrorInvalidValue;
@@ -265,8 +363,13 @@ cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void
         a.K = K;
         a.mode = mode;
         a.n_tiles = n_tiles;
+        a.n_split = n_split;
+        a.part = n_split > 1 ? static_cast<float *>(workspace) : nullptr;
+        a.counters = n_split > 1 ? reinterpret_cast<unsigned *>(static_cast<uint8_t *>(workspace) + need -
+                                                                sizeof(unsigned) * 4 * (size_t)n_pairs)
+                                 : nullptr;
         a.status = status;
-        const int grid = min(n_sm, n_tiles);
+        const int grid = n_split > 1 ? n_pairs * n_split : min(n_sm, n_tiles);
         linear_tc_kernel<<<grid, kThreadsL, LinSmem::alloc, stream>>>(tw, tx, a);
         if ((err = cudaGetLastError()) != cudaSuccess) return err;
     }

@@ -187,8 +187,13 @@ def test_paged_host_validation(lib):
 
 def test_draft_host_validation(lib):
     P = ctypes.c_void_p
-    lin = lambda R=4, N=128, K=64, mode=1, x=64, res=None, out=128: lib.clover_linear(
-        P(x), P(64), P(res) if res else None, P(out), R, N, K, mode, None, None)
+    lin = lambda R=4, N=128, K=64, mode=1, x=64, res=None, out=128, ws=None: lib.clover_linear(
+        P(x), P(64), P(res) if res else None, P(out), R, N, K, mode, P(ws) if ws else None, 1 << 20, None, None)
+    assert lin(ws=72) == 1                                   # workspace 16-byte aligned
+    # 4096 x 4096: 32 tiles, 16 pairs -> 8 K ranges; partials of 16 rows and 4 counters a pair
+    assert lib.clover_linear_workspace_size(16, 4096, 4096) == 8 * 16 * 4096 * 4 + 4 * 4 * 16
+    assert lib.clover_linear_workspace_size(16, 125696, 4096) == 0     # enough tiles: no split
+    assert lib.clover_linear_workspace_size(300, 256, 128) == 0         # under 4 stages of K per range: no split
     assert lin(K=96) == 1 and lin(K=0) == 1 and lin(N=0) == 1 and lin(mode=4) == 1 and lin(mode=-1) == 1
     assert lin(mode=2) == 1 and lin(mode=3) == 1             # residual modes need res
     assert lin(x=72) == 1 and lin(out=136) == 1              # 16-byte alignment

@@ -42,6 +42,9 @@ SHAPES = [
     (200, 640, 512),
     (256, 128, 64),               # the most rows of one launch
     (300, 200, 128),              # two launches (256 + 44 rows)
+    (16, 4096, 4096),             # a head's H x H layer: 32 tiles, K split 8 ways
+    (32, 1000, 1024),             # 8 tiles, K split 4 ways, the most rows that split
+    (3, 384, 2048),               # 3 tiles: one pair and a single tile, split
 ]
 
 
@@ -57,14 +60,19 @@ def test_linear_matches_oracle(R, N, K, mode):
         ref = oracle.linear(x, w) + res.double()
     else:
         ref = oracle.linear(x, w, res=res, act=act)
-    out = torch.empty((R, N), dtype=torch.float32 if mode == "f32" else BF, device=DEV)
-    st = torch.zeros(1, dtype=torch.int32, device=DEV)
-    pkg.clover_linear(x.to(DEV), w.to(DEV), out, res=None if res is None else res.to(DEV), mode=mode, status=st)
-    torch.cuda.synchronize()
-    assert int(st.item()) == 0
-    err = (out.cpu().double() - ref).abs()
     tol = linear_tol(x, w, ref, mode != "f32")
-    assert (err <= tol).all(), (err - tol).max().item()
+    n_ws = pkg.clover_linear_workspace_size(R, N, K)
+    # without a workspace (no K split) and with one (split when the plan splits), twice
+    for ws in (None, torch.zeros(max(16, n_ws), dtype=torch.uint8, device=DEV)):
+        for _ in range(2 if ws is not None else 1):
+            out = torch.empty((R, N), dtype=torch.float32 if mode == "f32" else BF, device=DEV)
+            st = torch.zeros(1, dtype=torch.int32, device=DEV)
+            pkg.clover_linear(x.to(DEV), w.to(DEV), out, res=None if res is None else res.to(DEV), mode=mode,
+                              workspace=ws, status=st)
+            torch.cuda.synchronize()
+            assert int(st.item()) == 0
+            err = (out.cpu().double() - ref).abs()
+            assert (err <= tol).all(), (err - tol).max().item()
 
 
 def test_linear_lm_head_full_size():
