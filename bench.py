@@ -278,15 +278,9 @@ def run_gpu_arm(args, world, rank, local, dist):
                           delta=args.delta, schedule=args.schedule, page_size=args.page_size or None)
     stream = torch.cuda.Stream(device)
 
-    ext_ok = True
-    try:
-        torch.cuda.Event(enable_timing=True, external=True)
-    except TypeError:
-        ext_ok = False
-
-    def launch(s, evs=None):
+    def launch(s):
         step.run(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"], s["parent"],
-                 s["cand"], s["logits"], stream=stream, events=evs, block_table=s.get("block_table"))
+                 s["cand"], s["logits"], stream=stream, block_table=s.get("block_table"))
 
     # eager warm-up (also initialises per-kernel attributes before capture)
     with torch.cuda.stream(stream):
@@ -296,24 +290,23 @@ def run_gpu_arm(args, world, rank, local, dist):
     if step.device_status() != 0:
         raise RuntimeError(f"device status {step.device_status()} during warm-up")
 
-    # one CUDA graph per input set and replica; the graphs of the first replica
-    # carry two timing events around the attention (an event node costs about
-    # a microsecond of the step, so the other calls are timed after the timed
-    # region)
-    reps = 4
-    graphs, graph_events = [], []
-    for r in range(reps):
+    # CUDA graphs of consecutive steps: the full graph runs one step on every
+    # input set in turn, each step's calls queued behind the previous step's
+    # (as in a decoding loop); single-step graphs time the remainder of K.  The
+    # timed graphs carry no timing nodes.
+    full = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(full, stream=stream):
         for s in sets:
-            evs = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)] \
-                if ext_ok and r == 0 else None
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                launch(s, evs)
-            graphs.append(g)
-            graph_events.append(evs)
+            launch(s)
+    singles = []
+    for s in sets[:args.steps % n_sets]:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            launch(s)
+        singles.append(g)
     torch.cuda.synchronize(device)
-    for i in range(max(3, args.warmup)):
-        graphs[i % len(graphs)].replay()
+    for _ in range(max(1, -(-max(3, args.warmup) // n_sets))):
+        full.replay()
     torch.cuda.synchronize(device)
 
     sampler = ClockSampler(local) if rank == 0 else None
@@ -327,8 +320,10 @@ def run_gpu_arm(args, world, rank, local, dist):
         sampler.mark("t0")
     with torch.cuda.stream(stream):
         start.record(stream)
-        for i in range(args.steps):
-            graphs[i % len(graphs)].replay()
+        for _ in range(args.steps // n_sets):
+            full.replay()
+        for g in singles:
+            g.replay()
         end.record(stream)
     end.synchronize()
     torch.cuda.synchronize(device)
@@ -341,28 +336,19 @@ def run_gpu_arm(args, world, rank, local, dist):
     value, ms = aggregate(seconds_max, args.steps, world)
     if step.device_status() != 0:
         raise RuntimeError(f"device status {step.device_status()} in the timed region")
+    del full, singles
 
-    # per-kernel durations.  The attention: the in-graph events of the last
-    # replay of every event-carrying graph inside the timed region.  The accept
-    # and commit calls: each launched alone after an L2 flush by a large read
-    # (which keeps the GPU busy while the call is queued, so the events bracket
-    # the kernel and not the host's launch latency), after the timed region.
-    durations = {"tree_attn": []}
-    timing_source = {"tree_attn": "events inside the replayed graphs of the timed region",
+    # per-kernel durations, after the timed region.  The attention: its
+    # average launch duration over back-to-back launches on the rotating input
+    # sets (inputs larger than the L2), one CUDA graph, events around the
+    # replays.  The accept and commit calls: each launched alone after an L2
+    # flush by a large read (which keeps the GPU busy while the call is queued,
+    # so the events bracket the kernel and not the host's launch latency).
+    timing_source = {"tree_attn": f"back-to-back attention launches over the {n_sets} rotating input sets in one "
+                                  "CUDA graph, events around the replays, after the timed region",
                      "accept": "launched alone after an L2 flush, events on the launching stream",
                      "kv_commit": "launched alone after an L2 flush, events on the launching stream"}
-    timed_graphs = [evs for i, evs in enumerate(graph_events) if evs and i < args.steps]
-    for evs in timed_graphs:
-        durations["tree_attn"].append(evs[0].elapsed_time(evs[1]) * 1e3)
-    if not timed_graphs:
-        for i in range(3 * len(sets)):
-            evs = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-            with torch.cuda.stream(stream):
-                launch(sets[i % n_sets], evs)
-            torch.cuda.synchronize(device)
-            durations["tree_attn"].append(evs[0].elapsed_time(evs[1]) * 1e3)
-        timing_source["tree_attn"] = "eager steps with events after the timed region (no external graph events)"
-    us = {k: statistics.mean(v) for k, v in durations.items()}
+    us = {"tree_attn": attn_launch_us(step, sets, stream, device, args)}
     flush = torch.zeros(2 * L2_BYTES, dtype=torch.uint8, device=device)
     us["accept"] = accept_kernel_us(pkg, w, sets, stream, device, args.accept, args, flush)
     other = "greedy" if args.accept == "typical" else "typical"
@@ -430,13 +416,16 @@ def run_gpu_arm(args, world, rank, local, dist):
 
 
 LAUNCH_DESC = {
-    "commit": "one CUDA graph replay per step: the attention (cache read only) on one stream, argmax/accept "
-              "then the commit of the accepted K/V on a second stream",
-    "compact": "one CUDA graph replay per step: the attention (appending the tree K/V) on one stream and "
-               "argmax/accept on a second, then the compaction of the accepted K/V",
-    "fused": "one CUDA graph replay per step, two launches on one stream: the attention (cache read only), then "
-             "argmax/accept with the commit of the accepted K/V fused in, launched as a programmatic dependent "
-             "of the attention so that it runs beside it",
+    "commit": "CUDA graphs of consecutive steps (one per input set, each queued behind the last); a step: the "
+              "attention (cache read only) on one stream, argmax/accept then the commit of the accepted K/V on a "
+              "second stream",
+    "compact": "CUDA graphs of consecutive steps (one per input set, each queued behind the last); a step: the "
+               "attention (appending the tree K/V) on one stream and argmax/accept on a second, then the "
+               "compaction of the accepted K/V",
+    "fused": "CUDA graphs of consecutive steps (one per input set, each queued behind the last); a step: two "
+             "launches on one stream, the attention (cache read only), then argmax/accept with the commit of the "
+             "accepted K/V fused in, launched as a programmatic dependent of the attention so that it runs "
+             "beside it",
 }
 
 
@@ -445,6 +434,41 @@ def accept_desc(args) -> str:
         return (f"typical acceptance (temperature {args.temperature}, epsilon {args.epsilon}, "
                 f"delta {args.delta})")
     return "greedy"
+
+
+def attn_launch_us(step, sets, stream, device, args, launches: int = 200) -> float:
+    """Mean duration of the step's attention call over back-to-back launches
+    on the rotating input sets: one CUDA graph of one launch per set, replayed
+    until about ``launches`` launches, CUDA events around the replays."""
+    import paper_2405_00263_gb300 as pkg
+
+    def attn(s):
+        if args.page_size:
+            pkg.clover_verify_attn_paged(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"],
+                                         s["block_table"], s["cache_len"], s["parent"], step.out,
+                                         workspace=step.ws_attn, status=step.status, stream=stream)
+        else:
+            pkg.clover_verify_attn(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"],
+                                   s["parent"], step.out, workspace=step.ws_attn, status=step.status,
+                                   stream=stream, append=args.schedule == "compact")
+
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for s in sets:
+            attn(s)
+    reps = max(3, launches // len(sets))
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            g.replay()
+        a.record(stream)
+        for _ in range(reps):
+            g.replay()
+        b.record(stream)
+    b.synchronize()
+    if step.device_status() != 0:
+        raise RuntimeError(f"device status {step.device_status()} in the attention timing")
+    return a.elapsed_time(b) * 1e3 / (reps * len(sets))
 
 
 def isolated_us(call, n, stream, flush) -> float:

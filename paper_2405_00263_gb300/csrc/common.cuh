@@ -180,11 +180,23 @@ __device__ __forceinline__ void tree_masks_jump(const int (&parent)[NS], int T, 
     }
 }
 
+// The parent array of a tree, read by one warp: lane l holds node l + 32k in
+// p[k] (-1 past T).  Split from the mask computation so that a kernel can
+// issue these loads at its start, ahead of its bulk traffic.
+__device__ __forceinline__ void tree_parents_load(const int32_t *parent, int T, int (&p)[4]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int i = lane + 32 * k;
+        p[k] = (i < T && (k < 2 || T > 64)) ? __ldg(parent + i) : -1;
+    }
+}
+
 // Ancestor-or-self bitmask of every tree node into anc[node * kMaskWords + w],
-// computed by one warp from the parent array in global memory.  Invalid parent
-// arrays set *bad (masks are then only self bits and must not be trusted).
+// computed by one warp from the parents loaded by tree_parents_load.  Invalid
+// parent arrays set *bad (masks are then only self bits and must not be trusted).
 template <int NS>
-__device__ __forceinline__ void tree_masks_warp_n(const int32_t *parent, int T, uint64_t *anc, bool *bad) {
+__device__ __forceinline__ void tree_masks_from(const int (&pl)[4], int T, uint64_t *anc, bool *bad) {
     const int lane = threadIdx.x & 31;
     int p[NS];
     bool invalid = false;
@@ -193,7 +205,7 @@ __device__ __forceinline__ void tree_masks_warp_n(const int32_t *parent, int T, 
         const int i = lane + 32 * k;
         p[k] = -1;
         if (i < T) {
-            p[k] = __ldg(parent + i);
+            p[k] = pl[k];
             if (i == 0 ? (p[k] != -1) : (p[k] < 0 || p[k] >= i)) invalid = true;
         }
     }
@@ -220,9 +232,15 @@ __device__ __forceinline__ void tree_masks_warp_n(const int32_t *parent, int T, 
     if (lane == 0) *bad = any_bad;
 }
 
+__device__ __forceinline__ void tree_masks_build(const int (&p)[4], int T, uint64_t *anc, bool *bad) {
+    if (T <= 64) tree_masks_from<2>(p, T, anc, bad);
+    else tree_masks_from<4>(p, T, anc, bad);
+}
+
 __device__ __forceinline__ void tree_masks_warp(const int32_t *parent, int T, uint64_t *anc, bool *bad) {
-    if (T <= 64) tree_masks_warp_n<2>(parent, T, anc, bad);
-    else tree_masks_warp_n<4>(parent, T, anc, bad);
+    int p[4];
+    tree_parents_load(parent, T, p);
+    tree_masks_build(p, T, anc, bad);
 }
 
 // Raises a kernel's dynamic shared memory limit once per device.  Launchers

@@ -89,8 +89,11 @@ __device__ __forceinline__ void cluster_sync_all() {
 
 // The two halves of cluster_sync_all, for work in between: every thread
 // arrives once, then waits once before its next arrive.
-__device__ __forceinline__ void cluster_arrive_release() {
-    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+// Arrive without release semantics: it does not wait for the thread's
+// outstanding memory operations (a producer's ring loads).  Barrier
+// initialisations are published to the cluster by fence_barrier_init instead.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void cluster_wait_acquire() {
     asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");

@@ -214,6 +214,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q_act = (rows_here + 31) >> 5;        // 32-row quadrants holding real rows
     const int n_soft_warps = KS * q_act;             // softmax warps of this tile
 
+    // The loads that do not depend on the cache length go out first, ahead of
+    // the ring's bulk traffic (issued once the length is known), so that they
+    // do not queue behind it.  Q rows of this warp's TMEM lane quadrant (row
+    // (node, head in group) = lane-quadrant row; with KS = 2 lanes 64-127 take
+    // rows 0-63 again) are written to TMEM once its address is known; rows past
+    // the tile's real rows are zero.  The tree CTA's warp 3 loads the parents.
+    constexpr int QW = D / 2;                 // 32-bit TMEM columns of a Q row (two bf16 each)
+    uint32_t qrow[QW];
+    if (warp < 4) {
+        const int rq = ((KS == 2) ? (warp & 1) : warp) * 32 + lane;
+        const int R = rt * BM + rq;
+        const bool real = rq < rows_here;
+        const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(a.q) +
+                                                           ((size_t)(b * a.T + (real ? R / a.G : 0)) * a.Hq +
+                                                            g * a.G + (real ? R % a.G : 0)) * D);
+#pragma unroll
+        for (int k = 0; k < QW / 4; ++k) {
+            const uint4 v = real ? __ldg(src + k) : make_uint4(0, 0, 0, 0);
+            qrow[4 * k] = v.x;
+            qrow[4 * k + 1] = v.y;
+            qrow[4 * k + 2] = v.z;
+            qrow[4 * k + 3] = v.w;
+        }
+    }
+    int parents[4];
+    if (warp == 3 && tree_cta) tree_parents_load(a.parent + (size_t)b * a.T, a.T, parents);
+
     int L = __ldg(a.cache_len + b);
     const bool cap_bad = (L < 0 || L + a.T > a.Lcap);
     if (cap_bad) {
@@ -351,36 +378,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = lane; i < n_pg; i += 32) s_pages[i] = cache_page(a, b, (first_page + i) << a.page_shift);
         }
     }
-    // Q rows of this warp's TMEM lane quadrant (row (node, head in group) =
-    // lane-quadrant row; with KS = 2 lanes 64-127 take rows 0-63 again): loaded
-    // now, written to TMEM once its address is known.  Rows past the tile's
-    // real rows are zero.
-    constexpr int QW = D / 2;                 // 32-bit TMEM columns of a Q row (two bf16 each)
-    uint32_t qrow[QW];
-    if (warp < 4) {
-        const int rq = ((KS == 2) ? (warp & 1) : warp) * 32 + lane;
-        const int R = rt * BM + rq;
-        const bool real = rq < rows_here;
-        const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(a.q) +
-                                                           ((size_t)(b * a.T + (real ? R / a.G : 0)) * a.Hq +
-                                                            g * a.G + (real ? R % a.G : 0)) * D);
-#pragma unroll
-        for (int k = 0; k < QW / 4; ++k) {
-            const uint4 v = real ? __ldg(src + k) : make_uint4(0, 0, 0, 0);
-            qrow[4 * k] = v.x;
-            qrow[4 * k + 1] = v.y;
-            qrow[4 * k + 2] = v.z;
-            qrow[4 * k + 3] = v.w;
-        }
-    }
     // the tree CTA's ancestor masks (warp 3 is otherwise idle here)
-    if (warp == 3 && tree_cta) tree_masks_warp(a.parent + (size_t)b * a.T, a.T, s_anc, s_bad);
-    // The cluster barrier is split: its arrive here publishes this CTA's
-    // barriers, its wait (before the first remote arrive, in the merge) lets
-    // the key loop start without waiting for the other CTAs' setup.
+    if (warp == 3 && tree_cta) tree_masks_build(parents, a.T, s_anc, s_bad);
+    // The cluster barrier is split: its wait (before the first remote arrive,
+    // in the merge) lets the key loop start without waiting for the other
+    // CTAs' setup.  The arrive is relaxed: fence_barrier_init has already
+    // published this CTA's barriers to the cluster, and a releasing arrive
+    // would hold each producer until its ring loads have landed.
     tc_fence_before();
     __syncwarp();
-    if (n_split > 1) cluster_arrive_release();
+    if (n_split > 1) cluster_arrive_relaxed();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *s_tmem;
@@ -669,24 +676,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool row_ok = softmax_warp && r < rows_here;
     float *part_o = reinterpret_cast<float *>(sK);            // [BM][D + 4] fp32, this CTA's partial
     float *recv = reinterpret_cast<float *>(sV);              // [n_split][per][D + 4]
+    // 64 O columns of this warp's lanes.  The TMEM loads are warp-collective:
+    // every lane runs them, rows past the tile's real rows only skip the stores
+    auto load_o = [&](int cc, float (&x0)[32], float (&x1)[32]) {
+        if (o_ready) {
+            tmem_ld32(tO + lane_base + cc * 32, x0);
+            tmem_ld32(tO + lane_base + cc * 32 + 32, x1);
+            tmem_wait_ld();
+        } else {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) x0[c] = x1[c] = 0.f;
+        }
+    };
     // KS = 2: the second key half's rows (O, m, l) go to rows 64.. of part_o,
-    // where the warps of the first half merge them into their own
+    // where the warps of the first half merge them into their own.  Those
+    // warps load their first 64 O columns meanwhile.
+    float x0[32], x1[32];
     if (KS == 2) {
-        // the TMEM loads are warp-collective: every lane runs them, rows past
-        // the tile's real rows only skip the stores
         if (softmax_warp && half == 1) {
             float *dst = part_o + (64 + r) * S::po_stride;
 #pragma unroll 1
             for (int cc = 0; cc < D / 32; cc += 2) {
-                float x0[32], x1[32];
-                if (o_ready) {
-                    tmem_ld32(tO + lane_base + cc * 32, x0);
-                    tmem_ld32(tO + lane_base + cc * 32 + 32, x1);
-                    tmem_wait_ld();
-                } else {
-#pragma unroll
-                    for (int c = 0; c < 32; ++c) x0[c] = x1[c] = 0.f;
-                }
+                load_o(cc, x0, x1);
                 if (row_ok) {
 #pragma unroll
                     for (int c = 0; c < 32; c += 4) {
@@ -701,6 +712,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 *reinterpret_cast<float2 *>(dst + D) =
                     make_float2(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f);
         }
+        if (softmax_warp && half == 0) load_o(0, x0, x1);
         __syncthreads();
     }
     if (softmax_warp && half == 0) {
@@ -720,57 +732,56 @@ __global__ void __launch_bounds__(kThreads, 1)
             m_row = M;
             l_row = wa * l_row + wb * mlb.y;
         }
-        const float inv = (n_split == 1 && l_row > 0.f) ? 1.f / l_row : 1.f;
-        // 32 columns of the row: the output (one split) or the partial row
-        auto emit = [&](int cc, float (&x)[32]) {
+        const float inv = (n_split == 1 && l_row > 0.f) ? rcp_approx(l_row) : 1.f;
+        // 64 columns of the row: the output (one split) or the partial row.
+        // The other half's 64 values are read in one batch before any store.
+        auto emit = [&](int cc, float (&y0)[32], float (&y1)[32]) {
             if (KS == 2) {
+                float4 yb[16];
 #pragma unroll
-                for (int c = 0; c < 32; c += 4) {
-                    const float4 y = *reinterpret_cast<const float4 *>(ob + cc * 32 + c);
-                    x[c] = fmaf(wb, y.x, wa * x[c]);
-                    x[c + 1] = fmaf(wb, y.y, wa * x[c + 1]);
-                    x[c + 2] = fmaf(wb, y.z, wa * x[c + 2]);
-                    x[c + 3] = fmaf(wb, y.w, wa * x[c + 3]);
+                for (int c = 0; c < 16; ++c) yb[c] = *reinterpret_cast<const float4 *>(ob + cc * 32 + 4 * c);
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    y0[4 * c] = fmaf(wb, yb[c].x, wa * y0[4 * c]);
+                    y0[4 * c + 1] = fmaf(wb, yb[c].y, wa * y0[4 * c + 1]);
+                    y0[4 * c + 2] = fmaf(wb, yb[c].z, wa * y0[4 * c + 2]);
+                    y0[4 * c + 3] = fmaf(wb, yb[c].w, wa * y0[4 * c + 3]);
+                    y1[4 * c] = fmaf(wb, yb[8 + c].x, wa * y1[4 * c]);
+                    y1[4 * c + 1] = fmaf(wb, yb[8 + c].y, wa * y1[4 * c + 1]);
+                    y1[4 * c + 2] = fmaf(wb, yb[8 + c].z, wa * y1[4 * c + 2]);
+                    y1[4 * c + 3] = fmaf(wb, yb[8 + c].w, wa * y1[4 * c + 3]);
                 }
             }
             if (n_split == 1) {
                 __nv_bfloat16 *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D + cc * 32;
 #pragma unroll
-                for (int c = 0; c < 32; c += 8) {
+                for (int c = 0; c < 64; c += 8) {
+                    const float *x = c < 32 ? y0 + c : y1 + (c - 32);
                     uint4 w;
-                    w.x = pack_bf16x2(x[c] * inv, x[c + 1] * inv);
-                    w.y = pack_bf16x2(x[c + 2] * inv, x[c + 3] * inv);
-                    w.z = pack_bf16x2(x[c + 4] * inv, x[c + 5] * inv);
-                    w.w = pack_bf16x2(x[c + 6] * inv, x[c + 7] * inv);
+                    w.x = pack_bf16x2(x[0] * inv, x[1] * inv);
+                    w.y = pack_bf16x2(x[2] * inv, x[3] * inv);
+                    w.z = pack_bf16x2(x[4] * inv, x[5] * inv);
+                    w.w = pack_bf16x2(x[6] * inv, x[7] * inv);
                     *reinterpret_cast<uint4 *>(dst + c) = w;
                 }
             } else {
                 float *po = part_o + r * S::po_stride + cc * 32;
 #pragma unroll
-                for (int c = 0; c < 32; c += 4)
-                    *reinterpret_cast<float4 *>(po + c) = make_float4(x[c], x[c + 1], x[c + 2], x[c + 3]);
+                for (int c = 0; c < 32; c += 4) {
+                    *reinterpret_cast<float4 *>(po + c) = make_float4(y0[c], y0[c + 1], y0[c + 2], y0[c + 3]);
+                    *reinterpret_cast<float4 *>(po + 32 + c) = make_float4(y1[c], y1[c + 1], y1[c + 2], y1[c + 3]);
+                }
             }
         };
-        // two TMEM loads in flight per wait
+        // two TMEM loads in flight per wait (the first pair is loaded already with KS = 2)
 #pragma unroll 1
         for (int cc = 0; cc < D / 32; cc += 2) {
-            float x0[32], x1[32];
-            if (o_ready) {
-                tmem_ld32(tO + lane_base + cc * 32, x0);
-                tmem_ld32(tO + lane_base + cc * 32 + 32, x1);
-                tmem_wait_ld();
-            } else {
-#pragma unroll
-                for (int c = 0; c < 32; ++c) x0[c] = x1[c] = 0.f;
-            }
-            if (row_ok) {
-                emit(cc, x0);
-                emit(cc + 1, x1);
-            }
+            if (KS == 1 || cc > 0) load_o(cc, x0, x1);
+            if (row_ok) emit(cc, x0, x1);
         }
         if (row_ok && n_split > 1)
             *reinterpret_cast<float2 *>(part_o + r * S::po_stride + D) = make_float2(m_row, l_row);
-        fence_proxy_async_smem();             // the bulk copies below read these rows
+        if (n_split > 1) fence_proxy_async_smem();   // the bulk copies below read these rows
     }
 
     // every TMEM access and MMA is finished before TMEM is released
@@ -786,26 +797,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (n_split > 1) {
         // ------------------------------------------ split merge in the cluster
         // CTA `split` merges rows [r0, r1) of the tile.  Once every CTA is out
-        // of its key loop, each sends every other CTA that CTA's rows of its
-        // partial with one bulk copy into the receiver's V ring (completing on
-        // the receiver's m_data), then merges its own rows from shared memory.
+        // of its key loop (m_free), lane k of warp 0 sends CTA k (k != split)
+        // that CTA's rows of this CTA's partial with one bulk copy into its V
+        // ring (completing on its m_data); then every CTA merges its own rows
+        // from shared memory.
         const int per = (rows_here + n_split - 1) / n_split;
         const int r0 = split * per;
         const int r1 = min(rows_here, r0 + per);
         constexpr uint32_t row_bytes = S::po_stride * 4;
         bool ok = true;
-        if (threadIdx.x == 0) {
-            if ((ok = mbar_wait_cluster(m_free, 0, kWaitNs))) {
-                for (int k = 0; k < n_split; ++k) {
-                    const int k0 = k * per;
-                    const int k1 = min(rows_here, k0 + per);
-                    if (k == split || k1 <= k0) continue;
-                    bulk_copy_to_cluster(mapa_shared(smem_u32(recv) + split * per * row_bytes, k),
+        if (warp == 0) {
+            if (lane < n_split) {
+                ok = mbar_wait_cluster(m_free, 0, kWaitNs);
+                const int k0 = lane * per;
+                const int k1 = min(rows_here, k0 + per);
+                if (ok && lane != split && k1 > k0)
+                    bulk_copy_to_cluster(mapa_shared(smem_u32(recv) + split * per * row_bytes, lane),
                                          part_o + k0 * S::po_stride, (k1 - k0) * row_bytes,
-                                         mapa_shared(smem_u32(m_data), k));
-                }
+                                         mapa_shared(smem_u32(m_data), lane));
             }
-            if (ok) ok = mbar_wait_cluster(m_data, 0, kWaitNs);
+            ok = __all_sync(0xffffffffu, ok);
+            if (lane == 0 && ok) ok = mbar_wait_cluster(m_data, 0, kWaitNs);
         }
         // one thread waited; every thread acquires the received rows itself
         const bool got = __syncthreads_and(ok) && mbar_test_cluster(m_data, 0);
