@@ -360,16 +360,36 @@ __device__ void commit_sequence(const AcceptArgs &a, int b, const int *s_path, i
     }
     if (a.src_index && threadIdx.x < Tn) a.src_index[(size_t)b * Tn + threadIdx.x] = threadIdx.x < len ? s_path[threadIdx.x] : -1;
     if (threadIdx.x == 0) a.new_cache_len[b] = L + len;
+    // The accepted rows (len nodes x Hkv heads x row_units 16-byte units, K
+    // and V) in batches: every thread loads its kBatch units of K and V, then
+    // stores them, so a batch costs one load round trip.
     const int per_node = a.Hkv * a.row_units;
-    for (int j = 0; j < len; ++j) {
-        const uint4 *ks = a.k_new + ((size_t)b * Tn + s_path[j]) * per_node;
-        const uint4 *vs = a.v_new + ((size_t)b * Tn + s_path[j]) * per_node;
-        for (int e = threadIdx.x; e < per_node; e += kThreads) {
-            const int g = e / a.row_units;
-            const int u = e - g * a.row_units;
-            const size_t dst = (((size_t)b * a.Hkv + g) * a.Lcap + L + j) * a.row_units + u;
-            a.k_cache[dst] = __ldg(ks + e);
-            a.v_cache[dst] = __ldg(vs + e);
+    const int total = len * per_node;
+    constexpr int kBatch = 4;
+    for (int e0 = threadIdx.x; e0 < total; e0 += kBatch * kThreads) {
+        uint4 kb[kBatch], vb[kBatch];
+#pragma unroll
+        for (int t = 0; t < kBatch; ++t) {
+            const int e = e0 + t * kThreads;
+            if (e < total) {
+                const int j = e / per_node;
+                const size_t src = ((size_t)b * Tn + s_path[j]) * per_node + (e - j * per_node);
+                kb[t] = __ldg(a.k_new + src);
+                vb[t] = __ldg(a.v_new + src);
+            }
+        }
+#pragma unroll
+        for (int t = 0; t < kBatch; ++t) {
+            const int e = e0 + t * kThreads;
+            if (e < total) {
+                const int j = e / per_node;
+                const int r = e - j * per_node;
+                const int g = r / a.row_units;
+                const int u = r - g * a.row_units;
+                const size_t dst = (((size_t)b * a.Hkv + g) * a.Lcap + L + j) * a.row_units + u;
+                a.k_cache[dst] = kb[t];
+                a.v_cache[dst] = vb[t];
+            }
         }
     }
 }
@@ -453,10 +473,13 @@ __device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) 
 }
 
 template <typename T, bool TYPICAL>
-__global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
+__device__ __forceinline__ void accept_body(const AcceptArgs &a) {
     __shared__ uint64_t s_red[kThreads / 32];
     __shared__ float4 s_sum[kThreads / 32];
     __shared__ int s_seq_last;
+    // a commit queued behind this call as a programmatic dependent may place
+    // its CTAs now; it waits for this grid's completion before its first access
+    allow_dependent_launch();
     const int warp = threadIdx.x >> 5;
     const int row = blockIdx.x;            // b * T + i
     const int chunk_id = blockIdx.y;
@@ -548,6 +571,19 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptArgs a) {
     finish_sequence<T, TYPICAL>(a, b, tr);
 }
 
+// The greedy kernel is held to 56 registers, so that two of its CTAs fit on an
+// SM beside an attention CTA (160 registers x 224 threads) when the two calls
+// run at the same time; the typical kernel needs more.
+template <typename T>
+__global__ void __maxnreg__(56) accept_kernel(const AcceptArgs a) {
+    accept_body<T, false>(a);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) accept_typical_kernel(const AcceptArgs a) {
+    accept_body<T, true>(a);
+}
+
 }  // namespace
 
 // Vocabulary chunk per CTA: one round of kUnits 16-byte loads per thread
@@ -594,7 +630,8 @@ static cudaError_t launch_kernel(const AcceptArgs &a, bool after_prior, cudaStre
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = after_prior ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, accept_kernel<T, TYPICAL>, a);
+    if (TYPICAL) return cudaLaunchKernelEx(&cfg, accept_typical_kernel<T>, a);
+    return cudaLaunchKernelEx(&cfg, accept_kernel<T>, a);
 }
 
 cudaError_t launch_accept_call(const AcceptCall &c, cudaStream_t stream) {

@@ -32,6 +32,9 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
     __shared__ int s_ok;
     const int g = blockIdx.x;
     const int b = blockIdx.y;
+    // launched as a programmatic dependent of the kernel before it in the
+    // stream: every global access comes after that grid has completed
+    wait_prerequisite_grids();
     // the length, the accepted count and the whole path row are loaded at
     // once, one path entry per thread (T <= kThreads)
     static_assert(kMaxTreeNodes <= kThreads, "one path entry per thread");
@@ -106,14 +109,25 @@ cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, c
     static unsigned char done[64];
     cudaError_t e = ensure_smem_attr(kv_compact_kernel, (size_t)2 * kMaxTreeNodes * 128 * 4, done);
     if (e != cudaSuccess) return e;
-    dim3 grid(Hkv, B);
-    kv_compact_kernel<<<grid, kThreads, smem, stream>>>(static_cast<uint8_t *>(k_cache),
-                                                        static_cast<uint8_t *>(v_cache),
-                                                        static_cast<const uint8_t *>(k_new),
-                                                        static_cast<const uint8_t *>(v_new), cache_len, path,
-                                                        accept_len, new_cache_len, src_index, T, Hkv,
-                                                        row_bytes, Lcap, block_table, page_size, page_shift,
-                                                        max_pages, n_pages, status);
+    // A programmatic dependent of the preceding kernel in the stream: its CTAs
+    // may be placed while that kernel runs (an accept call lets them in at its
+    // start) and wait in the kernel for its completion, so the copy starts
+    // without a launch gap.
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(Hkv, B);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kv_compact_kernel, static_cast<uint8_t *>(k_cache), static_cast<uint8_t *>(v_cache),
+                           static_cast<const uint8_t *>(k_new), static_cast<const uint8_t *>(v_new), cache_len, path,
+                           accept_len, new_cache_len, src_index, T, Hkv, row_bytes, Lcap, block_table, page_size,
+                           page_shift, max_pages, n_pages, status);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
