@@ -716,9 +716,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncthreads();
     }
     if (softmax_warp && half == 0) {
-        const int R = rt * BM + r;
-        const int i = row_ok ? R / a.G : 0;
-        const int h = row_ok ? g * a.G + (R % a.G) : 0;
         // this row's (m, l) and the weights of its key halves
         float m_row = o_ready ? m_ref : -INFINITY;
         float l_row = o_ready ? l_run : 0.f;
@@ -732,7 +729,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             m_row = M;
             l_row = wa * l_row + wb * mlb.y;
         }
-        const float inv = (n_split == 1 && l_row > 0.f) ? rcp_approx(l_row) : 1.f;
         // 64 columns of the row: the output (one split) or the partial row.
         // The other half's 64 values are read in one batch before any store.
         auto emit = [&](int cc, float (&y0)[32], float (&y1)[32]) {
@@ -753,6 +749,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             if (n_split == 1) {
+                // the output row (node, head); only this path needs it
+                const int R = rt * BM + r;
+                const int i = R / a.G;
+                const int h = g * a.G + (R % a.G);
+                const float inv = l_row > 0.f ? rcp_approx(l_row) : 1.f;
                 __nv_bfloat16 *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D + cc * 32;
 #pragma unroll
                 for (int c = 0; c < 64; c += 8) {
