@@ -40,7 +40,11 @@
  *   - Calls are asynchronous on `stream` (a cudaStream_t passed as void*;
  *     NULL = the legacy default stream).  The return value reports errors
  *     found on the host before anything is launched (and launch failures);
- *     nothing is launched when it is not CLOVER_OK.
+ *     nothing is launched when it is not CLOVER_OK.  Stream order holds for
+ *     every call.  clover_kv_commit, clover_kv_commit_paged and
+ *     clover_kv_compact launch as programmatic dependents of the kernel before
+ *     them in the stream: their CTAs may be placed early, but they wait for
+ *     that kernel's completion before their first memory access.
  *   - Errors found on the device (an invalid parent array, a cache that is too
  *     small, an invalid path) are OR-ed into `*status` (a device int32 the
  *     caller zeroes; may be NULL).  Kernels never trap and never wait without
