@@ -820,9 +820,18 @@ def cpu_baseline(w, host: dict, args, budget_s: float = 8.0) -> dict:
     while sum(times) < budget_s and len(times) < 50:
         times.append(oracle_step_seconds(host, threads, typ))
     per = statistics.median(times)
+    # the same oracle on one core: one step on a sample of the rows sized to
+    # about a quarter of the budget (OracleSampler), scaled to the whole step
+    one = OracleSampler(host, 1, typ)
+    f1 = sample_fraction(per * threads, 1, budget_s / 4)
+    t1 = one.step_seconds(f1)
     return {"value": 1.0 / per, "unit": UNIT, "cores": threads, "kind": "oracle",
             "sample": f"{len(times)} whole verify steps of {w.name} (fp64 oracle, OpenMP over attention rows "
-                      f"and logit rows, {accept_desc(args)}), median {per * 1e3:.1f} ms per step"}
+                      f"and logit rows, {accept_desc(args)}), median {per * 1e3:.1f} ms per step",
+            "single_core": {"value": 1.0 / t1, "unit": UNIT, "cores": 1,
+                            "sample": "one verify step" + ("" if f1 >= 1.0 else
+                                      f", {f1:.2e} of the attention rows and of the logit rows, scaled to the "
+                                      "whole step")}}
 
 
 def run_reference_arm(args, world, rank, budget_s: float = 120.0):

@@ -44,3 +44,13 @@ def test_batched_bytes_follow_the_lengths():
     per_key = 2 * w.Hkv * w.D * 2
     assert bench.attn_bytes_per_launch(w, lengths) == \
         per_key * sum(L + w.T for L in lengths) + 2 * w.B * w.T * w.Hq * w.D * 2
+
+
+def test_cpu_baseline_reports_all_cores_and_one():
+    from types import SimpleNamespace
+    w = workloads.get("tiny_f32")
+    host = workloads.make(w)
+    args = SimpleNamespace(accept="greedy", temperature=1.0, epsilon=0.09, delta=0.3)
+    rec = bench.cpu_baseline(w, host, args, budget_s=0.5)
+    assert rec["kind"] == "oracle" and rec["value"] > 0 and rec["cores"] >= 1
+    assert rec["single_core"]["cores"] == 1 and rec["single_core"]["value"] > 0
