@@ -79,9 +79,18 @@ typedef enum {
     CLOVER_ERR_BAD_TREE = 4,     /* device: parent array is not a topologically numbered tree */
     CLOVER_ERR_CAPACITY = 8,     /* device: cache_len[b] < 0 or cache_len[b] + T > Lcap */
     CLOVER_ERR_CUDA = 16,        /* a CUDA launch or query failed */
-    CLOVER_ERR_TIMEOUT = 32,     /* reserved: a bounded device wait gave up */
+    CLOVER_ERR_TIMEOUT = 32,     /* device: a bounded wait gave up (see below) */
     CLOVER_ERR_SCRATCH_LIMIT = 64 /* clover_verify_attn_noalloc: scratch need exceeds its static buffer */
 } clover_status;
+
+/*
+ * CLOVER_ERR_TIMEOUT is raised by the kernels that wait on barriers: the bf16
+ * tensor-core attention (clover_verify_attn, _ex, _paged, _noalloc with bf16)
+ * and clover_linear.  Each of their waits gives up after about 0.5 s; the
+ * kernel then winds down (waits, again bounded, for its copies in flight and
+ * frees its tensor memory) and sets this bit.  The outputs of that call are
+ * unspecified; the context stays usable.  The other kernels never wait.
+ */
 
 typedef enum {
     CLOVER_F32 = 0,   /* float32 storage, fp32 arithmetic (no TF32) */
@@ -436,9 +445,11 @@ CLOVER_API clover_status clover_kv_commit(void *k_cache, void *v_cache, const vo
  * CLOVER_NOALLOC_SCRATCH_BYTES (8 MiB).  Every GPU that loads the library holds
  * that array until the process exits.  This call allocates nothing: it calls no
  * cudaMalloc, cudaFree or allocating library routine.
- *   - The first call on a device looks up the array's device address with that
- *     device current (cudaGetSymbolAddress) and caches it.  Make this first call
- *     before any stream capture that contains later calls.
+ *   - The first call in a CUDA context (normally once per device; again after
+ *     cudaDeviceReset or under another context of the device) looks up the
+ *     array's device address with that context current (cudaGetSymbolAddress)
+ *     and caches it under the context's id.  Make this first call before any
+ *     stream capture that contains later calls.
  *   - Each call clears the part of the array that must start at zero (the
  *     arrival counters) with an asynchronous memset on `stream`, then launches.
  *     The rest of the array keeps the previous call's contents, which are

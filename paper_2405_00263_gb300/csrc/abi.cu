@@ -3,7 +3,7 @@
 // each call are in include/clover_verify.h.
 #include <math.h>
 
-#include <atomic>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -499,20 +499,35 @@ static_assert(CLOVER_NOALLOC_SCRATCH_BYTES % 256 == 0, "scratch size must keep 2
 // Resident on every device that loads this library, until the process exits.
 static __device__ __align__(256) unsigned char g_attn_scratch[CLOVER_NOALLOC_SCRATCH_BYTES];
 
-// Device address of g_attn_scratch per device, looked up once with that device current.
-constexpr int kMaxDevices = 64;
-std::atomic<void *> g_attn_scratch_addr[kMaxDevices];
+// Device address of g_attn_scratch, looked up with cudaGetSymbolAddress once
+// per CUDA context (the context current on the calling thread) and cached
+// under that context's id.  A device ordinal alone would not do: after
+// cudaDeviceReset, or under a non-primary context of the same device, the
+// module (and with it the array) is loaded anew, possibly at another address.
+constexpr int kAddrSlots = 64;
+struct ScratchAddr {
+    unsigned long long ctx;   // current_context_id() of the lookup (0: slot unused)
+    void *addr;
+};
+std::mutex g_attn_scratch_mu;
+ScratchAddr g_attn_scratch_addr[kAddrSlots];
+int g_attn_scratch_next = 0;   // slot to fill (round robin once every slot is used)
 
 cudaError_t attn_scratch_address(void **addr) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    const unsigned long long ctx = current_context_id();
+    std::lock_guard<std::mutex> lock(g_attn_scratch_mu);
+    if (ctx != 0)
+        for (const ScratchAddr &s : g_attn_scratch_addr)
+            if (s.ctx == ctx) {
+                *addr = s.addr;
+                return cudaSuccess;
+            }
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_attn_scratch);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    void *p = g_attn_scratch_addr[dev].load(std::memory_order_acquire);
-    if (p == nullptr) {
-        e = cudaGetSymbolAddress(&p, g_attn_scratch);
-        if (e != cudaSuccess) return e;
-        g_attn_scratch_addr[dev].store(p, std::memory_order_release);
+    if (ctx != 0) {
+        g_attn_scratch_addr[g_attn_scratch_next] = ScratchAddr{ctx, p};
+        g_attn_scratch_next = (g_attn_scratch_next + 1) % kAddrSlots;
     }
     *addr = p;
     return cudaSuccess;

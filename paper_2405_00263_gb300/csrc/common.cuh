@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include "clover_verify.h"
+#include "ctx_host.cuh"
 
 namespace clover {
 
@@ -243,18 +244,21 @@ __device__ __forceinline__ void tree_masks_warp(const int32_t *parent, int T, ui
     tree_masks_build(p, T, anc, bad);
 }
 
-// Raises a kernel's dynamic shared memory limit once per device.  Launchers
-// call it before every launch; only the first call on a device reaches the
-// driver, so launches captured into a CUDA graph after a first eager launch
-// issue no attribute call.
+// Raises a kernel's dynamic shared memory limit once per CUDA context.
+// Launchers call it before every launch; only the first call in a context
+// reaches the driver, so launches captured into a CUDA graph after a first
+// eager launch issue no attribute call.  `done` holds, per device ordinal, the
+// context in which the attribute was last set: a reset device (or another
+// context on it) starts without the attribute and gets it again.
 template <typename Kernel>
-cudaError_t ensure_smem_attr(Kernel kernel, size_t bytes, unsigned char (&done)[64]) {
+cudaError_t ensure_smem_attr(Kernel kernel, size_t bytes, unsigned long long (&done)[64]) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev < 64 && done[dev]) return cudaSuccess;
+    const unsigned long long ctx = current_context_id();
+    if (ctx != 0 && dev >= 0 && dev < 64 && done[dev] == ctx) return cudaSuccess;
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-    if (e == cudaSuccess && dev < 64) done[dev] = 1;
+    if (e == cudaSuccess && dev >= 0 && dev < 64) done[dev] = ctx;
     return e;
 }
 

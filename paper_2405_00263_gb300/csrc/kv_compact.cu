@@ -106,7 +106,7 @@ cudaError_t launch_kv_compact(void *k_cache, void *v_cache, const void *k_new, c
     while (block_table && (1 << page_shift) < page_size) ++page_shift;
     const int row_bytes = D * (dtype == CLOVER_F32 ? 4 : 2);
     const size_t smem = (size_t)2 * T * row_bytes;
-    static unsigned char done[64];
+    static unsigned long long done[64];
     cudaError_t e = ensure_smem_attr(kv_compact_kernel, (size_t)2 * kMaxTreeNodes * 128 * 4, done);
     if (e != cudaSuccess) return e;
     // A programmatic dependent of the preceding kernel in the stream: its CTAs

@@ -331,7 +331,7 @@ size_t linear_workspace_bytes(int R, int N, int K) {
 // plan's K split is used; without one, none.
 cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
                              void *workspace, size_t ws_bytes, int32_t *status, cudaStream_t stream) {
-    static unsigned char done[64];
+    static unsigned long long done[64];
     static int sms[64];
     cudaError_t err = ensure_smem_attr(linear_tc_kernel, LinSmem::alloc, done);
     if (err != cudaSuccess) return err;

@@ -392,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
 
 template <typename T, int D>
 cudaError_t launch(const AttnArgs &a, cudaStream_t stream) {
-    static unsigned char done[64];
+    static unsigned long long done[64];
     auto kernel = tree_attn_fma_kernel<T, D>;
     cudaError_t e = ensure_smem_attr(kernel, FmaSmem<D>::bytes, done);
     if (e != cudaSuccess) return e;

@@ -7,11 +7,13 @@
 //
 // One CTA per (row tile of up to 128 query rows, cache-key split, sequence x
 // KV head).  The T*G query rows of a KV head (row i*G + hh = node i, query head
-// g*G + hh) share every K/V tile, so per 64-key tile:
-//   S  = Q K^T        tcgen05.mma M=128 N=64 K=D  (Q in TMEM, K K-major in smem; S in TMEM)
+// g*G + hh) share every K/V tile, so per 128-key tile:
+//   S  = Q K^T        tcgen05.mma M=128 N=128, D/16 instructions of K=16
+//                     (Q in TMEM, K K-major in smem; S in TMEM)
 //   P  = 2^(S*c - m)  online softmax in registers; bf16 P written back to TMEM
 //                     over the S tile it came from
-//   O += P V          tcgen05.mma M=128 N=D K=64  (P in TMEM, V MN-major in smem)
+//   O += P V          tcgen05.mma M=128 N=D, 8 instructions of K=16 over the
+//                     tile's 128 keys (P in TMEM, V MN-major in smem)
 // Q and O stay in TMEM for the whole key range, so the tensor core reads only
 // K and V from shared memory (which the TMA writes fill at the same time).
 // Each row keeps a reference max m; P is taken relative to it, and m (with O
@@ -883,7 +885,7 @@ int max_active_clusters(int n, TcLaunchCache &cache) {
 
 template <int D, int KS, bool PAGED>
 cudaError_t launch(AttnArgs a, cudaStream_t stream) {
-    static unsigned char done[64];
+    static unsigned long long done[64];
     static TcLaunchCache caches[64];
     auto kernel = tree_attn_tc_kernel<D, KS, PAGED>;
     cudaError_t err = ensure_smem_attr(kernel, TcSmem<D, KS>::alloc, done);

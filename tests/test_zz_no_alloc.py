@@ -5,9 +5,12 @@ process has already reserved the free HBM for its own pool, or code that must
 not make a call that may synchronise the device).  clover_verify_attn_noalloc
 serves them by keeping its split-KV scratch in a static device buffer.  This
 test checks that it gives the same results as clover_verify_attn with a
-caller-provided workspace, on two calls in a row (the second call finds the
-buffer holding the first call's contents), and that a size whose scratch need
-exceeds the buffer is refused before anything runs.
+caller-provided workspace, bit for bit, on two calls in a row (the second call
+finds the buffer holding the first call's contents); both calls run the same
+kernel with the same split plan and merge order, so any difference is a wrong
+or stale partial.  It also checks the output against the fp64 oracle of the
+tree attention (Section 2.2) at the fp32 tolerance, and that a size whose
+scratch need exceeds the buffer is refused before anything runs.
 
 The file is named so that pytest collects it last.
 """
@@ -17,6 +20,7 @@ import ctypes
 import pytest
 import torch
 
+import oracle
 import paper_2405_00263_gb300 as pkg
 from paper_2405_00263_gb300 import _lib
 from synth import workloads
@@ -70,6 +74,9 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(cuda):
                            ref["parent"], out_ref, workspace=ws, status=st_ref)
     torch.cuda.synchronize()
     assert int(st_ref.item()) == 0
+    host = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
+    want = oracle.tree_attention(host["q"], host["k_new"], host["v_new"], host["k_cache"], host["v_cache"],
+                                 host["cache_len"], host["parent"]).reshape(out_ref.shape)
 
     for call in range(2):
         t = {k: (v.clone() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
@@ -79,8 +86,11 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(cuda):
         assert code == 0, lib.clover_status_string(code)
         torch.cuda.synchronize()
         assert int(st.item()) == 0, f"call {call}: device status {int(st.item())}"
-        err = (out.float() - out_ref.float()).abs().max().item()
-        assert err <= ATOL[w.torch_dtype], f"call {call}: max-abs difference {err}"
+        assert torch.equal(out, out_ref), (
+            f"call {call}: differs from clover_verify_attn by up to "
+            f"{(out.float() - out_ref.float()).abs().max().item()}")
+        err = (out.double().cpu() - want).abs().max().item()
+        assert err <= ATOL[w.torch_dtype], f"call {call}: max-abs error {err} against the oracle"
         # the tree K/V append is the same as well
         L = int(base["cache_len"][0])
         assert torch.equal(t["k_cache"][:, :, :L + T], ref["k_cache"][:, :, :L + T])
