@@ -106,8 +106,8 @@ CLOVER_API const char *clover_status_string(int status);
 /*
  * Bytes of device workspace clover_verify_attn needs for these sizes
  * (split-KV partial results and per-head arrival counters).  0 when none is
- * needed (the bf16 tensor-core path merges its splits on chip) and when the
- * sizes are outside the limits.
+ * needed (one key range per head: no split) and when the sizes are outside
+ * the limits.
  */
 CLOVER_API size_t clover_verify_attn_workspace_size(int B, int T, int Hq, int Hkv, int D, int Lcap,
                                          clover_dtype dtype);
@@ -135,8 +135,14 @@ CLOVER_API size_t clover_verify_attn_workspace_size(int B, int T, int Hq, int Hk
  *                                    clover_verify_attn_workspace_size(...) bytes,
  *                                    16-byte aligned.  It must be zero-filled before
  *                                    its first use; every call leaves it ready for the
- *                                    next one.  Calls sharing a workspace must not
- *                                    overlap on the device.
+ *                                    next one.  One workspace serves calls with the
+ *                                    same B, T, Hq, Hkv, D and dtype and any Lcap up to
+ *                                    the one it was sized for; for other sizes zero it
+ *                                    again.  After a call that raised
+ *                                    CLOVER_ERR_TIMEOUT, zero it again.  Calls sharing
+ *                                    a workspace must not overlap on the device, apart
+ *                                    from the overlap of CLOVER_ATTN_PDL launches
+ *                                    (clover_verify_attn_ex), which is safe.
  *   status                           device int32 error bits (may be NULL)
  * q, k_new, v_new, caches and out must be 16-byte aligned.
  */
@@ -148,13 +154,45 @@ CLOVER_API clover_status clover_verify_attn(const void *q, const void *k_new, co
                                  void *workspace, size_t ws_bytes,
                                  int32_t *status, void *stream);
 
-/* Flag of clover_verify_attn_ex: the call only reads k_cache/v_cache (no append). */
-#define CLOVER_ATTN_NO_APPEND 1u
+/* Flags of clover_verify_attn_ex. */
+#define CLOVER_ATTN_NO_APPEND 1u    /* the call only reads k_cache/v_cache (no append) */
+#define CLOVER_ATTN_PDL 2u          /* launch as a programmatic dependent of the kernel queued before it */
+#define CLOVER_ATTN_CACHE_READY 4u  /* with CLOVER_ATTN_PDL: the cache may be read before that kernel ends */
+#define CLOVER_ATTN_INPUTS_READY 8u /* with CLOVER_ATTN_PDL: every input may be read before that kernel ends */
 
 /*
- * clover_verify_attn with flags: 0 is clover_verify_attn itself;
- * CLOVER_ATTN_NO_APPEND skips the append, so slots >= cache_len[b] are neither
- * read for the result nor written.  Other flag bits: CLOVER_ERR_INVALID_ARG.
+ * clover_verify_attn with flags: 0 is clover_verify_attn itself.
+ *   CLOVER_ATTN_NO_APPEND skips the append, so slots >= cache_len[b] are
+ *     neither read for the result nor written.
+ *   CLOVER_ATTN_PDL launches the bf16 (tensor-core) kernel as a programmatic
+ *     dependent of the kernel queued just before it on `stream`: its CTAs may
+ *     be placed once every CTA of that kernel has started (this library's
+ *     attention kernels allow it at their start), and they set up their
+ *     barriers and tensor memory while it runs.  Every read of an input still
+ *     waits for that kernel's completion (griddepcontrol.wait), so the results
+ *     and stream order are those of an ordinary launch.
+ *   CLOVER_ATTN_CACHE_READY (with CLOVER_ATTN_PDL) states that cache_len, the
+ *     cache slots [0, cache_len[b]) and (paged) the block table are not
+ *     written by the kernel queued before this call, nor by any kernel that
+ *     may still run beside it (with programmatic launches, every kernel of the
+ *     chain of programmatic dependents that ends in it).  The kernel then
+ *     reads those before the preceding kernel completes: it loads the lengths
+ *     and streams its first cache tiles while that kernel finishes.  q, k_new,
+ *     v_new and parent are still read only after it completes, and every write
+ *     (out, the append, the workspace) comes after that too.  Example: the
+ *     attention launched right behind the projection that produced q, k_new
+ *     and v_new.
+ *   CLOVER_ATTN_INPUTS_READY (with CLOVER_ATTN_PDL) states the same of every
+ *     input: q, k_new, v_new, parent, cache_len, the cache slots
+ *     [0, cache_len[b]) and the block table.  The kernel then reads all of
+ *     them, and runs its whole key loop, while the preceding kernel finishes;
+ *     only its writes (out, the append, the workspace) wait for that kernel's
+ *     completion.  Example: the attention of one micro-batch launched right
+ *     behind the attention of another micro-batch, whose inputs were produced
+ *     earlier.  Neither statement is checked: a kernel that does write one of
+ *     these inputs while this call reads it gives unspecified results.
+ * The fp32 (CUDA-core) kernel is launched the ordinary way whatever the launch
+ * flags say.  Other flag bits: CLOVER_ERR_INVALID_ARG.
  */
 CLOVER_API clover_status clover_verify_attn_ex(const void *q, const void *k_new, const void *v_new,
                                     void *k_cache, void *v_cache, const int32_t *cache_len,

@@ -42,8 +42,11 @@ EXPORTS = (
     "clover_topk",
 )
 
-# Flag of clover_verify_attn_ex (CLOVER_ATTN_NO_APPEND in include/clover_verify.h).
+# Flags of clover_verify_attn_ex (CLOVER_ATTN_* in include/clover_verify.h).
 ATTN_NO_APPEND = 1
+ATTN_PDL = 2
+ATTN_CACHE_READY = 4
+ATTN_INPUTS_READY = 8
 
 # Flags of clover_verify_accept_ex (CLOVER_ACCEPT_* in include/clover_verify.h).
 ACCEPT_TYPICAL = 1

@@ -95,10 +95,17 @@ def clover_verify_accept_typical_workspace_size(B, T, V, dtype) -> int:
 
 
 def clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, scale=0.0,
-                       workspace=None, status=None, stream=None, append=True):
+                       workspace=None, status=None, stream=None, append=True, pdl=False, cache_ready=False,
+                       inputs_ready=False):
     """Tree-masked attention; with ``append`` (clover_verify_attn) it also
     writes k_new/v_new at cache slots [L, L+T), without it
-    (clover_verify_attn_ex with CLOVER_ATTN_NO_APPEND) the caches are only read."""
+    (clover_verify_attn_ex with CLOVER_ATTN_NO_APPEND) the caches are only read.
+    ``pdl``: CLOVER_ATTN_PDL (launched as a programmatic dependent of the
+    kernel queued before it); ``cache_ready`` (with ``pdl``):
+    CLOVER_ATTN_CACHE_READY, the caller's statement that the caches and
+    cache_len are not being written by the kernels that may still run;
+    ``inputs_ready`` (with ``pdl``): CLOVER_ATTN_INPUTS_READY, the same
+    statement of every input."""
     B, T, Hq, D = q.shape
     Hkv, Lcap = k_cache.shape[1], k_cache.shape[2]
     dt = q.dtype
@@ -116,12 +123,14 @@ def clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out
     args = (_ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(cache_len), _ptr(parent),
             _ptr(out), B, T, Hq, Hkv, D, Lcap, dtype_code(dt), float(scale), _ptr(workspace), ws_bytes,
             _ptr(status), _stream(stream))
-    if append:
+    flags = (0 if append else _lib.ATTN_NO_APPEND) | (_lib.ATTN_PDL if pdl else 0) | \
+        (_lib.ATTN_CACHE_READY if cache_ready else 0) | (_lib.ATTN_INPUTS_READY if inputs_ready else 0)
+    if flags == 0:
         code = _lib.load().clover_verify_attn(*args)
     else:
-        code = _lib.load().clover_verify_attn_ex(*args, _lib.ATTN_NO_APPEND)
+        code = _lib.load().clover_verify_attn_ex(*args, flags)
     if code != OK:
-        raise CloverError(code, "clover_verify_attn" if append else "clover_verify_attn_ex")
+        raise CloverError(code, "clover_verify_attn" if flags == 0 else "clover_verify_attn_ex")
 
 
 def clover_verify_attn_noalloc(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, scale=0.0,

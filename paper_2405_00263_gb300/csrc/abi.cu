@@ -10,6 +10,7 @@
 namespace clover {
 int fma_row_tile();
 int tc_row_tile();
+int tc_max_splits();
 cudaError_t launch_tree_attn_fma(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream);
 void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk);
@@ -43,6 +44,8 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Workspace layout: [arrival counters][split partials (O rows; FMA: then
+// max and sum)], each part rounded up to 256 bytes.
 struct AttnPlan {
     bool tc;                 // tensor-core (tcgen05) kernel, else the FMA kernel
     int row_tile, row_tiles, n_split, slot_rows;
@@ -59,11 +62,13 @@ clover_status check_attn_sizes(int B, int T, int Hq, int Hkv, int D, int Lcap, i
 }
 
 // Kernel choice, split count and workspace layout for one shape.  bf16 runs on
-// the tensor cores (one CTA per SM, splits merged on chip, no workspace) for
-// any number of query rows: even a 4-row tile is bound by HBM there, as the
-// MMA cost of a 128-key tile (about 0.8 us) stays below its HBM time.  fp32
-// runs on the FMA kernel with two CTAs per SM and merges splits through the
-// workspace.
+// the tensor cores for any number of query rows: even a 4-row tile is bound by
+// HBM there, as the MMA cost of a 128-key tile (about 0.8 us) stays below its
+// HBM time.  One CTA per SM: the cache keys of a (sequence, head, row tile)
+// split over as many CTAs as fill the SMs in one wave (at most tc_max_splits,
+// at least kMinKeysPerSplit keys each), partials merged through the workspace
+// (rows of D + 4 floats).  fp32 runs on the FMA kernel with two CTAs per SM
+// and merges splits through the workspace too.
 AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
     AttnPlan p;
     const int G = Hq / Hkv;
@@ -73,14 +78,24 @@ AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
     int n;
     p.tc = (dtype == CLOVER_BF16);
     if (p.tc) {
-        // the tensor-core kernel picks its split count at launch (one wave of
-        // thread-block clusters) and merges splits in distributed shared memory:
-        // it needs no workspace
         p.row_tile = tc_row_tile();
         p.row_tiles = (rows + p.row_tile - 1) / p.row_tile;
         p.slot_rows = rows < p.row_tile ? rows : p.row_tile;
-        p.n_split = 1;
-        p.o_bytes = p.ml_bytes = p.counter_bytes = p.total = 0;
+        const long base = Bp * Hkv * p.row_tiles;
+        n = (int)(kSms / base);
+        if (n > tc_max_splits()) n = tc_max_splits();
+        if (n > by_len) n = by_len;
+        if (n < 1) n = 1;
+        p.n_split = n;
+        const size_t heads = (size_t)Bp * Hkv * p.row_tiles;
+        if (n == 1) {
+            p.o_bytes = p.ml_bytes = p.counter_bytes = p.total = 0;
+        } else {
+            p.o_bytes = round_up(sizeof(float) * heads * n * p.slot_rows * (D + 4), 256);
+            p.ml_bytes = 0;
+            p.counter_bytes = round_up(sizeof(unsigned) * heads, 256);
+            p.total = p.o_bytes + p.counter_bytes;
+        }
         return p;
     } else {
         p.row_tile = fma_row_tile();
@@ -197,7 +212,7 @@ clover_status run_attn(const void *q, const void *k_new, const void *v_new, void
                        const int32_t *cache_len, const int32_t *parent, void *out, int B, int T, int Hq, int Hkv,
                        int D, int Lcap, clover_dtype dtype, float scale, void *workspace, size_t ws_bytes,
                        int32_t *status, void *stream, bool append, const int32_t *block_table, int page_size,
-                       int max_pages, int n_pages) {
+                       int max_pages, int n_pages, uint32_t launch_flags = 0u) {
     if (!q || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !parent || !out)
         return CLOVER_ERR_INVALID_ARG;
     if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache) ||
@@ -240,10 +255,17 @@ clover_status run_attn(const void *q, const void *k_new, const void *v_new, void
     a.n_split = p.n_split;
     a.slot_rows = p.slot_rows;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
-    a.part_o = p.total ? reinterpret_cast<float *>(ws) : nullptr;
-    a.part_ml = p.total ? reinterpret_cast<float *>(ws + p.o_bytes) : nullptr;
-    a.counters = p.total ? reinterpret_cast<unsigned *>(ws + p.o_bytes + p.ml_bytes) : nullptr;
+    // counters first: their place does not depend on the split count, so a
+    // workspace sized for a capacity serves every smaller one
+    a.counters = p.total ? reinterpret_cast<unsigned *>(ws) : nullptr;
+    a.part_o = p.total ? reinterpret_cast<float *>(ws + p.counter_bytes) : nullptr;
+    a.part_ml = p.total && p.ml_bytes ? reinterpret_cast<float *>(ws + p.counter_bytes + p.o_bytes) : nullptr;
     a.status = status;
+    // the launch options apply to the tensor-core kernel; the FMA kernel is
+    // launched the ordinary way (stream order) whatever they say
+    a.pdl = (launch_flags & CLOVER_ATTN_PDL) ? 1 : 0;
+    a.cache_early = (a.pdl && (launch_flags & CLOVER_ATTN_CACHE_READY)) ? 1 : 0;
+    a.inputs_early = (a.pdl && (launch_flags & CLOVER_ATTN_INPUTS_READY)) ? 1 : 0;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     return from_cuda(p.tc ? launch_tree_attn_tc(a, st) : launch_tree_attn_fma(a, st));
 }
@@ -287,12 +309,14 @@ clover_status clover_verify_attn_ex(const void *q, const void *k_new, const void
                                     int B, int T, int Hq, int Hkv, int D, int Lcap, clover_dtype dtype,
                                     float scale, void *workspace, size_t ws_bytes, int32_t *status,
                                     void *stream, uint32_t flags) {
-    if (flags & ~CLOVER_ATTN_NO_APPEND) return CLOVER_ERR_INVALID_ARG;
+    if (flags & ~(CLOVER_ATTN_NO_APPEND | CLOVER_ATTN_PDL | CLOVER_ATTN_CACHE_READY | CLOVER_ATTN_INPUTS_READY))
+        return CLOVER_ERR_INVALID_ARG;
     const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype);
     if (s != CLOVER_OK) return s;
     if (B == 0) return CLOVER_OK;
     return run_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, B, T, Hq, Hkv, D, Lcap, dtype, scale,
-                    workspace, ws_bytes, status, stream, (flags & CLOVER_ATTN_NO_APPEND) == 0, nullptr, 0, 0, 0);
+                    workspace, ws_bytes, status, stream, (flags & CLOVER_ATTN_NO_APPEND) == 0, nullptr, 0, 0, 0,
+                    flags);
 }
 
 size_t clover_verify_attn_paged_workspace_size(int B, int T, int Hq, int Hkv, int D, int page_size, int max_pages,
@@ -560,7 +584,7 @@ extern "C" clover_status clover_verify_attn_noalloc(const void *q, const void *k
     if (attn_scratch_address(&scratch) != cudaSuccess) return CLOVER_ERR_CUDA;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (p.counter_bytes > 0 &&
-        cudaMemsetAsync(static_cast<uint8_t *>(scratch) + p.o_bytes + p.ml_bytes, 0, p.counter_bytes, st) !=
+        cudaMemsetAsync(scratch, 0, p.counter_bytes, st) !=
             cudaSuccess)
         return CLOVER_ERR_CUDA;
     return clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, B, T, Hq, Hkv, D, Lcap,

@@ -33,10 +33,17 @@ struct AttnArgs {
     // of page block_table[b * max_pages + s / page_size]; Lcap = page_size * max_pages
     const int32_t *block_table;
     int page_size, page_shift, max_pages, n_pages;
-    float *part_o;         // [B, Hkv, row_tiles, n_split, slot_rows, D]
-    float *part_ml;        // [B, Hkv, row_tiles, n_split, slot_rows, 2]  (max, sum)
-    unsigned *counters;    // [B, Hkv, row_tiles]
+    // split partials (n_split > 1).  FMA kernel: part_o [B, Hkv, row_tiles,
+    // n_split, slot_rows, D] and part_ml [..., slot_rows, 2] (max, sum);
+    // tensor-core kernel: part_o [B, Hkv, row_tiles, n_split, slot_rows, D + 4]
+    // (O, then max and sum), part_ml unused
+    float *part_o;
+    float *part_ml;
+    unsigned *counters;    // [B, Hkv, row_tiles] arrival counters, zero between calls
     int32_t *status;
+    int pdl;               // launched as a programmatic dependent of the preceding kernel
+    int cache_early;       // caches, lengths and block table may be read before that kernel completes
+    int inputs_early;      // every input may be read before that kernel completes (only writes wait)
 };
 
 // One acceptance call (clover_verify_accept, _typical or _ex), validated on
@@ -242,6 +249,41 @@ __device__ __forceinline__ void tree_masks_warp(const int32_t *parent, int T, ui
     int p[4];
     tree_parents_load(parent, T, p);
     tree_masks_build(p, T, anc, bad);
+}
+
+// Ancestor-or-self bitmasks by walking each node's root path, in one warp:
+// lane l holds the parents of nodes l + 32 k in p[k] (tree_parents_load's
+// layout) and copies them to `par` in shared memory; then node i's mask
+// collects i and every node on the way up to the root (depth(i) + 1 steps,
+// as parent[i] < i).  Node n is bit n & 63 of word n >> 6 of anc[i].  An
+// invalid parent array (parent[0] != -1, or parent[i] outside [0, i)) sets
+// *bad and leaves only the self bits.  Small code, for kernels that run it
+// once per launch; its time grows with the tree's depth.
+static __device__ __noinline__ void tree_masks_walk(const int (&p)[4], int T, int *par, uint64_t *anc, bool *bad) {
+    const int lane = threadIdx.x & 31;
+    bool invalid = false;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int i = lane + 32 * k;
+        if (i < T) {
+            par[i] = p[k];
+            if (i == 0 ? (p[k] != -1) : (p[k] < 0 || p[k] >= i)) invalid = true;
+        }
+    }
+    const bool any_bad = __any_sync(0xffffffffu, invalid);
+    __syncwarp();
+#pragma unroll 1
+    for (int i = lane; i < T; i += 32) {
+        uint64_t m[kMaskWords] = {0ull, 0ull};
+        int j = i;
+        do {
+            m[j >> 6] |= 1ull << (j & 63);
+            j = any_bad ? -1 : par[j];
+        } while (j >= 0);
+        anc[i * kMaskWords] = m[0];
+        anc[i * kMaskWords + 1] = m[1];
+    }
+    if (lane == 0) *bad = any_bad;
 }
 
 // Raises a kernel's dynamic shared memory limit once per CUDA context.

@@ -54,17 +54,24 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity, ui
     return ok != 0;
 }
 
+constexpr uint32_t kTryHintNs = 1000000;    // 1 ms per suspended try
+
+// The bounded part of mbar_wait, out of line: one copy per kernel instead of
+// one per wait, so that the kernels' code stays small.
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parity, uint64_t limit_ns) {
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < limit_ns) {
+        if (mbar_try_wait(bar, parity, kTryHintNs)) return true;
+    }
+    return false;
+}
+
 // Waits for the phase with the given parity to complete.  Gives up after
 // about `limit_ns` nanoseconds and returns false (the caller reports a timeout
 // and winds down); never waits without a bound.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint64_t limit_ns) {
-    constexpr uint32_t kHintNs = 1000000;    // 1 ms per suspended try
-    if (mbar_try_wait(bar, parity, kHintNs)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    while (globaltimer_ns() - t0 < limit_ns) {
-        if (mbar_try_wait(bar, parity, kHintNs)) return true;
-    }
-    return false;
+    if (mbar_try_wait(bar, parity, kTryHintNs)) return true;
+    return mbar_wait_slow(bar, parity, limit_ns);
 }
 
 // ------------------------------------------------------------ thread-block cluster
@@ -162,12 +169,74 @@ __device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m
         : "memory");
 }
 
+// L2 policy for data read once: its lines are the first to be evicted, so a
+// stream of them does not push out what other accesses reuse (code, small
+// inputs, partial results).
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+// tma_load_3d with an L2 cache policy (see l2_policy_evict_first).
+__device__ __forceinline__ void tma_load_3d_hint(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x, int y,
+                                                 int z, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%2, "
+        "%3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(policy)
+        : "memory");
+}
+
+// Bulk copy (TMA engine) of `bytes` contiguous bytes from global memory to this
+// CTA's shared memory, completing as transaction bytes on `bar`.  Both
+// addresses 16-byte aligned, size a multiple of 16.
+__device__ __forceinline__ void bulk_load_g2s(void *smem_dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(smem_dst)),
+                 "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+
+// Orders this thread's generic-proxy global accesses with its async-proxy
+// (bulk copy) global accesses, in both directions.
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// Global-memory load with acquire semantics at GPU scope (sees every write
+// that a releasing writer made before the value it reads).
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(reinterpret_cast<uint64_t>(p)) : "memory");
+    return v;
+}
+
+// Atomic add with release semantics at GPU scope (no return value).
+__device__ __forceinline__ void red_add_release_gpu(unsigned *p, unsigned v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)), "r"(v) : "memory");
+}
+
+// Hint: bring the 128-byte line holding `p` into L2 (no effect on values).
+__device__ __forceinline__ void prefetch_l2(const void *p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<uint64_t>(p)) : "memory");
+}
+
 // shared -> global tile store (bulk async-group completion; x must keep the
 // 16-byte rule and no coordinate may be negative)
 __device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, const void *smem_src, int x, int y, int z) {
     asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
                      reinterpret_cast<uint64_t>(map)),
                  "r"(x), "r"(y), "r"(z), "r"(smem_u32(smem_src))
+                 : "memory");
+}
+
+// Bulk copy (TMA engine) of `bytes` contiguous bytes from this CTA's shared
+// memory to global memory (bulk async-group completion: commit, then wait).
+// Both addresses 16-byte aligned, size a multiple of 16.
+__device__ __forceinline__ void bulk_store_s2g(void *dst, const void *smem_src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(reinterpret_cast<uint64_t>(dst)),
+                 "r"(smem_u32(smem_src)), "r"(bytes)
                  : "memory");
 }
 

@@ -24,16 +24,32 @@
 // Warp roles (224 threads): warp w in 0-3 writes the Q rows of TMEM lanes
 // 32w.. and runs the softmax, rescales and the epilogue of those lanes (the
 // lanes warp w may access); warp 4 issues the TMA loads of the K tiles (its
-// own ring); warp 6 those of the V tiles (a deeper ring: a V tile is held
-// until its P.V product, a K tile only until its S); warp 5 allocates TMEM and
-// issues the MMAs from one thread.  The tree CTA's producers also append the
-// tree keys and values to the cache when asked, by TMA stores of the tree
-// tile they loaded.
+// own ring); warp 6 those of the V tiles; warp 5 allocates TMEM and issues the
+// MMAs from one thread.  The cache tiles are read with an L2 evict-first
+// policy: they are read once, and must not push out of L2 what is reused.
 // The split that owns the last cache range also takes the tile of T tree keys
-// (read from k_new/v_new) under the ancestor bitmask.  The n_split CTAs of a
-// (sequence, head, row tile) form one thread-block cluster: each sends every
-// other CTA its rows of the partial result (O, m, l) by shared-to-shared bulk
-// copy, and merges its own rows, so no partial result touches global memory.
+// (read from k_new/v_new) under the ancestor bitmask, as its first tile; its
+// producers also append the tree keys and values to the cache when asked, by
+// TMA stores of that tile.
+//
+// Split merge: every CTA of a (sequence, head, row tile) group but the last
+// (the one with the tree tile, which ends last) combines its two key halves,
+// copies its partial result (unnormalised O rows with their max m and sum l)
+// from shared memory to its workspace slot by one bulk copy and counts itself
+// in at the group's arrival counter; then it exits, so its SM is free.  The
+// last CTA waits (bounded) for the others' arrival, bulk-loads their rows and
+// merges every source of a row (its own key halves and the other splits' rows)
+// straight into the output.
+//
+// Programmatic dependent launch (AttnArgs::pdl): the grid may start while the
+// kernel before it in the stream still runs.  Barrier setup and the TMEM
+// allocation come first.  Every read of an input comes after
+// griddepcontrol.wait, except when the caller states that they are not being
+// written by the kernels that may still run: with cache_early the cache
+// length, the block table and the cache tiles of the free ring stages are read
+// before it; with inputs_early every input is, and only the writes (the
+// append, the workspace, the output) wait.
+//
 // Every mbarrier wait is bounded; on a timeout the CTA reports
 // CLOVER_ERR_TIMEOUT, winds down, waits (bounded) for its copies in flight and
 // frees its TMEM.
@@ -55,15 +71,16 @@ constexpr int kKProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kVProducerWarp = 6;
 constexpr int kThreads = 224;
-constexpr int kMaxCluster = 8;          // portable cluster size: splits per head
+constexpr int kMaxSplits = 8;           // key ranges per (sequence, head, row tile)
+constexpr int kMaxSrc = kMaxSplits + 2;  // partial rows merged into one output row (own halves + others)
 constexpr float kRescale = 8.0f;        // move the reference max only past 2^8 growth
 constexpr uint64_t kWaitNs = 500ull * 1000 * 1000;   // 0.5 s per wait
 
-// Shared-memory plan: the K and V rings only (Q lives in TMEM).  KS = key
-// groups per tile row: with KS = 2 (a tile of at most 64 real query rows) the
-// Q rows of TMEM lanes 64-127 repeat those of lanes 0-63, so every real row's
-// scores sit in two lane quadrants and the four softmax warps each take half
-// of a tile's keys.
+// Shared-memory plan: the K and V rings (Q lives in TMEM).  KS = key groups
+// per tile row: with KS = 2 (a tile of at most 64 real query rows) the Q rows
+// of TMEM lanes 64-127 repeat those of lanes 0-63, so every real row's scores
+// sit in two lane quadrants and the four softmax warps each take half of a
+// tile's keys.
 template <int D, int KS>
 struct TcSmem {
     static constexpr int NSK = (D == 128) ? 3 : 4;   // K ring stages
@@ -73,28 +90,32 @@ struct TcSmem {
     static constexpr int k_off = 0;
     static constexpr int v_off = k_off + NSK * kv_bytes;
     static constexpr int bar_off = v_off + NSV * kv_bytes;
-    static constexpr int n_bars = 2 * NSK + 2 * NSV + 11;
-    static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad flags
+    static constexpr int n_bars = 2 * NSK + 2 * NSV + 9;
+    static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad
     static constexpr int anc_off = misc_off + 16;                  // ancestor masks [128][2]
     static constexpr int pages_off = anc_off + kMaxTreeNodes * kMaskWords * 8;   // paged: page ids of the split
-    static constexpr int total = pages_off + kPageSmem * 4;
+    static constexpr int wts_off = pages_off + kPageSmem * 4;      // merge weights [BM][kMaxSrc]
+    static constexpr int par_off = wts_off + BM * kMaxSrc * 4;     // the tree's parent array [128]
+    static constexpr int total = par_off + kMaxTreeNodes * 4;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
     // TMEM columns: S/P 2 x BN, O D, Q D / 2 (two bf16 per column), rounded up
     // to a power of two.  All 512 columns of an SM go to one CTA only when
-    // the shared memory already keeps a second CTA off the SM (a CTA waiting
-    // in tcgen05.alloc would stall its cluster).
+    // the shared memory already keeps a second CTA off the SM (a second CTA
+    // would wait in tcgen05.alloc).
     static constexpr uint32_t tmem_cols = (2 * BN + D + D / 2 <= 256) ? 256 : 512;
     static_assert(tmem_cols < 512 || 2 * alloc > 228 * 1024, "512 TMEM columns need one CTA per SM");
-    // After the key loop the K ring holds this CTA's partial result, one fp32
-    // row of D + 4 floats per query row (O, then m and l in the padding; with
-    // KS = 2 rows 64-127 first carry the second key half's rows), and the V
-    // ring receives the other splits' partials of the rows this CTA merges:
-    // [n_split][rows per split][D + 4].
+    // After the key loop the rings hold the partial results: this CTA's at the
+    // start of the K ring, one fp32 row of D + 4 floats per query row (O, then
+    // m and l; with KS = 2 rows 64-127 first carry the second key half's
+    // rows), and, in the merging CTA, the other splits' rows after it, in the
+    // same row format (the workspace's format too).
     static constexpr int po_stride = D + 4;
-    static constexpr int rows_max = (KS == 2) ? 64 : BM;         // real rows of a tile
-    static_assert(BM * po_stride * 4 <= NSK * kv_bytes, "partial result must fit in the K ring");
-    static_assert((rows_max + kMaxCluster - 1) * po_stride * 4 <= NSV * kv_bytes,
-                  "received partials must fit in the V ring");
+    static constexpr int own_bytes = BM * po_stride * 4;
+    static constexpr int recv_bytes = (NSK + NSV) * kv_bytes - own_bytes;
+    static_assert(own_bytes % 16 == 0 && (po_stride * 4) % 16 == 0, "bulk copies move 16-byte units");
+    static_assert(own_bytes <= NSK * kv_bytes, "partial result must fit in the K ring");
+    static_assert(recv_bytes >= (kMaxSplits - 1) * po_stride * 4, "a merge pass must hold one row of each split");
+    static_assert(KS == 1 || BM == 128, "the second key half's rows sit 64 rows below the first's");
     static_assert(alloc <= 227 * 1024, "shared memory budget");
 };
 
@@ -109,60 +130,102 @@ __device__ __forceinline__ float rcp_approx(float x) {
     return y;
 }
 
-// Merge of the NS split partials of rows [r0, r1) of a tile (Section 2.2's
-// attention over the whole key range, from per-range partial softmax results):
-//   O = sum_k 2^(m_k - M) O_k / sum_k 2^(m_k - M) l_k,  M = max_k m_k.
-// Row rr of split k is `own` (this CTA's) or row (k * per + rr - r0) of `recv`;
-// each row holds O (D floats), then m and l.  A thread takes one (row, 4
-// columns) item at a time.  NS is a template argument so the whole item is
-// one short chain of independent loads and arithmetic (with few warps per
-// SM, the latency of a long chain is not hidden).
-template <int D, int NS>
-__device__ __forceinline__ void merge_rows(const float *own, const float *recv, int po_stride, int split, int per,
-                                           int r0, int r1, int row0, const AttnArgs &a, int b, int g,
-                                           __nv_bfloat16 *out) {
-    const int n_items = (r1 - r0) * (D / 4);
-    const float inv_g = 1.f / (float)a.G;
-    for (int e = threadIdx.x; e < n_items; e += blockDim.x) {
-        const int rr = r0 + e / (D / 4);
-        const int c4 = (e % (D / 4)) * 4;
-        float2 ml[NS];
-        float4 x[NS];
+// One pass of the merge of partial softmax results into output rows (Section
+// 2.2's attention over the whole key range, from per-range partial results):
+//   O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
+// over the sources s of a row, with the weights w[row][s] = 2^(m_s - M) /
+// sum_s 2^(m_s - M) l_s already in shared memory.  Source s < KS of row rr is
+// this CTA's row rr + 64 s of `own` (its key halves); source KS + k is the
+// k-th other split's, row rr - p0 of slot k of `recv`.  Rows [p0, p1).  A warp
+// takes 4 rows at a time and lane l their columns [4 l, 4 l + 4) (D = 128;
+// D = 64 uses lanes 0-15): each shared-memory load of the warp reads one row's
+// contiguous 512 bytes, free of bank conflicts.  With `out` == nullptr the
+// result (weights not normalised) goes back to `own` row rr instead.
+template <int D, int KS>
+__device__ __noinline__ void merge_pass(float *own, const float *recv, const float *wts, int n_src, int rpp, int p0,
+                                        int p1, int row0, const AttnArgs &a, int b, int g,
+                                        __nv_bfloat16 *out) {
+    constexpr int PS = D + 4;
+    constexpr int RG = 4;                     // rows per warp step
+    const int lane = threadIdx.x & 31;
+    const int c = lane * 4;
+    if (c >= D) return;
+    const int n_warps = blockDim.x >> 5;
+    const int G = a.G;
+    for (int r0 = p0 + (int)(threadIdx.x >> 5) * RG; r0 < p1; r0 += n_warps * RG) {
+        const int nr = min(RG, p1 - r0);
+        float4 acc[RG];
 #pragma unroll
-        for (int k = 0; k < NS; ++k) {
-            const float *row = (k == split) ? own + rr * po_stride : recv + (k * per + rr - r0) * po_stride;
-            ml[k] = *reinterpret_cast<const float2 *>(row + D);
-            x[k] = *reinterpret_cast<const float4 *>(row + c4);
+        for (int k = 0; k < RG; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 1
+        for (int sidx = 0; sidx < n_src; ++sidx) {
+            const float *base = sidx < KS ? own + (r0 + 64 * sidx) * PS : recv + ((sidx - KS) * rpp + r0 - p0) * PS;
+#pragma unroll
+            for (int k = 0; k < RG; ++k) {
+                if (k < nr) {
+                    const float w = wts[(r0 + k) * kMaxSrc + sidx];
+                    const float4 x = *reinterpret_cast<const float4 *>(base + k * PS + c);
+                    acc[k].x = fmaf(w, x.x, acc[k].x);
+                    acc[k].y = fmaf(w, x.y, acc[k].y);
+                    acc[k].z = fmaf(w, x.z, acc[k].z);
+                    acc[k].w = fmaf(w, x.w, acc[k].w);
+                }
+            }
         }
-        float M = ml[0].x;
 #pragma unroll
-        for (int k = 1; k < NS; ++k) M = fmaxf(M, ml[k].x);
-        float w[NS];
-        float lsum = 0.f;
-#pragma unroll
-        for (int k = 0; k < NS; ++k) {
-            w[k] = (ml[k].x == -INFINITY) ? 0.f : ex2_approx(ml[k].x - M);
-            lsum = fmaf(w[k], ml[k].y, lsum);
+        for (int k = 0; k < RG; ++k) {
+            if (k >= nr) continue;
+            const int rr = r0 + k;
+            if (out == nullptr) {
+                *reinterpret_cast<float4 *>(own + rr * PS + c) = acc[k];
+                continue;
+            }
+            // tile row R = node * G + head-in-group
+            const int R = row0 + rr;
+            const int i = R / G;
+            const int h = g * G + (R - i * G);
+            uint2 w2;
+            w2.x = pack_bf16x2(acc[k].x, acc[k].y);
+            w2.y = pack_bf16x2(acc[k].z, acc[k].w);
+            *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c) = w2;
         }
-        const float inv = rcp_approx(lsum);
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int k = 0; k < NS; ++k) {
-            const float wk = w[k] * inv;
-            acc.x = fmaf(wk, x[k].x, acc.x);
-            acc.y = fmaf(wk, x[k].y, acc.y);
-            acc.z = fmaf(wk, x[k].z, acc.z);
-            acc.w = fmaf(wk, x[k].w, acc.w);
-        }
-        // row R = node * G + head-in-group; (R + 1/2) / G is never within
-        // float rounding of an integer, so the truncation is exact
-        const int R = row0 + rr;
-        const int i = __float2int_rz(((float)R + 0.5f) * inv_g);
-        const int h = g * a.G + (R - i * a.G);
-        uint2 w2;
-        w2.x = pack_bf16x2(acc.x, acc.y);
-        w2.y = pack_bf16x2(acc.z, acc.w);
-        *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c4) = w2;
+    }
+}
+
+// Merge weights of the sources of rows [p0, p1) (one thread a row), from the
+// (m, l) stored after each source row's O: source s < KS is `own` row
+// rr + 64 s, source KS + k row rr - p0 of slot k of `recv` (both in shared
+// memory).  w[rr][s] = 2^(m_s - M) with M the largest m, divided by
+// sum_s 2^(m_s - M) l_s when `normalise`; otherwise the combined row's M and
+// sum go to w[rr][kMaxSrc - 2] and w[rr][kMaxSrc - 1].
+template <int D, int KS>
+__device__ __noinline__ void row_weights(const float *own, const float *recv, int rpp, int p0, int p1, int n_src,
+                                         float *wts, bool normalise) {
+    constexpr int PS = D + 4;
+    const int rr = p0 + (int)threadIdx.x;
+    if (rr >= p1) return;
+    auto ml = [&](int sidx) {
+        const float *row = sidx < KS ? own + (rr + 64 * sidx) * PS : recv + ((sidx - KS) * rpp + rr - p0) * PS;
+        return *reinterpret_cast<const float2 *>(row + D);
+    };
+    float M = -INFINITY;
+#pragma unroll 1
+    for (int sidx = 0; sidx < n_src; ++sidx) M = fmaxf(M, ml(sidx).x);
+    float lsum = 0.f;
+#pragma unroll 1
+    for (int sidx = 0; sidx < n_src; ++sidx) {
+        const float2 v = ml(sidx);
+        const float w = (v.x == -INFINITY) ? 0.f : ex2_approx(v.x - M);
+        wts[rr * kMaxSrc + sidx] = w;
+        lsum = fmaf(w, v.y, lsum);
+    }
+    if (normalise) {
+        const float inv = lsum > 0.f ? rcp_approx(lsum) : 0.f;
+#pragma unroll 1
+        for (int sidx = 0; sidx < n_src; ++sidx) wts[rr * kMaxSrc + sidx] *= inv;
+    } else {
+        wts[rr * kMaxSrc + kMaxSrc - 2] = M;
+        wts[rr * kMaxSrc + kMaxSrc - 1] = lsum;
     }
 }
 
@@ -175,8 +238,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     using S = TcSmem<D, KS>;
     constexpr int NSK = S::NSK;
     constexpr int NSV = S::NSV;
-    // an accept call queued behind this one as a programmatic dependent may
-    // take the SM space this grid leaves free
+    // a kernel queued behind this one as a programmatic dependent may start
+    // on the SM space this grid leaves free
     allow_dependent_launch();
     extern __shared__ uint8_t smem_raw[];
     // base rounded up to 1024 bytes by pointer arithmetic on the shared array,
@@ -194,14 +257,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t *o_full = p_full + 2;            // [2] the tile's P.V product is done
     uint64_t *mma_done = o_full + 2;
     uint64_t *q_full = mma_done + 1;          // the four lane quadrants hold their Q rows in TMEM
-    uint64_t *m_free = q_full + 1;            // every CTA of the cluster is out of its key loop
-    uint64_t *m_done = m_free + 1;            // every CTA has received this CTA's partial rows
-    uint64_t *m_data = m_done + 1;            // the other splits' partials of this CTA's rows are here
+    uint64_t *g_full = q_full + 1;            // the merging CTA: a pass of the other splits' partials is here
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(sm + S::misc_off);
     volatile int *s_abort = reinterpret_cast<volatile int *>(sm + S::misc_off + 4);
     bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 8);
     uint64_t *s_anc = reinterpret_cast<uint64_t *>(sm + S::anc_off);
     int *s_pages = reinterpret_cast<int *>(sm + S::pages_off);
+    float *s_wts = reinterpret_cast<float *>(sm + S::wts_off);
+    int *s_par = reinterpret_cast<int *>(sm + S::par_off);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -216,34 +279,91 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q_act = (rows_here + 31) >> 5;        // 32-row quadrants holding real rows
     const int n_soft_warps = KS * q_act;             // softmax warps of this tile
 
-    // The loads that do not depend on the cache length go out first, ahead of
-    // the ring's bulk traffic (issued once the length is known), so that they
-    // do not queue behind it.  Q rows of this warp's TMEM lane quadrant (row
-    // (node, head in group) = lane-quadrant row; with KS = 2 lanes 64-127 take
-    // rows 0-63 again) are written to TMEM once its address is known; rows past
-    // the tile's real rows are zero.  The tree CTA's warp 3 loads the parents.
-    constexpr int QW = D / 2;                 // 32-bit TMEM columns of a Q row (two bf16 each)
-    uint32_t qrow[QW];
-    if (warp < 4) {
-        const int rq = ((KS == 2) ? (warp & 1) : warp) * 32 + lane;
-        const int R = rt * BM + rq;
-        const bool real = rq < rows_here;
-        const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(a.q) +
-                                                           ((size_t)(b * a.T + (real ? R / a.G : 0)) * a.Hq +
-                                                            g * a.G + (real ? R % a.G : 0)) * D);
-#pragma unroll
-        for (int k = 0; k < QW / 4; ++k) {
-            const uint4 v = real ? __ldg(src + k) : make_uint4(0, 0, 0, 0);
-            qrow[4 * k] = v.x;
-            qrow[4 * k + 1] = v.y;
-            qrow[4 * k + 2] = v.z;
-            qrow[4 * k + 3] = v.w;
+    // ------------------------------------------ setup that reads no input
+    // Each producer initialises the barriers of its ring (the K producer also
+    // every other one); warp 5 allocates TMEM.
+    if (warp == kVProducerWarp && lane == 0) {
+        for (int i = 0; i < NSV; ++i) {
+            mbar_init(&v_full[i], 1);
+            mbar_init(&v_empty[i], 1);
         }
+        fence_barrier_init();
+        prefetch_tensormap(&tm_vc);
+        prefetch_tensormap(&tm_vn);
     }
-    int parents[4];
-    if (warp == 3 && tree_cta) tree_parents_load(a.parent + (size_t)b * a.T, a.T, parents);
+    if (warp == kKProducerWarp && lane == 0) {
+        for (int i = 0; i < NSK; ++i) {
+            mbar_init(&k_full[i], 1);
+            mbar_init(&k_empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&s_full[i], 1);
+            mbar_init(&p_full[i], n_soft_warps);
+            mbar_init(&o_full[i], 1);
+        }
+        mbar_init(mma_done, 1);
+        mbar_init(q_full, 4);
+        mbar_init(g_full, 1);
+        *s_abort = 0;
+        *s_bad = false;
+        fence_barrier_init();
+        prefetch_tensormap(&tm_kc);
+        prefetch_tensormap(&tm_kn);
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(s_tmem, S::tmem_cols);
+        tmem_relinquish();
+    }
 
-    int L = __ldg(a.cache_len + b);
+    // Q rows of this warp's TMEM lane quadrant (row (node, head in group) =
+    // lane-quadrant row; with KS = 2 lanes 64-127 take rows 0-63 again); rows
+    // past the tile's real rows are zero.  The tree CTA's warp 3 reads the
+    // parent array.
+    constexpr int QW = D / 2;                 // 32-bit TMEM columns of a Q row (two bf16 each)
+    const int rq = ((KS == 2) ? (warp & 1) : (warp & 3)) * 32 + lane;
+    const bool q_real = warp < 4 && rq < rows_here;
+    const uint4 *q_src = reinterpret_cast<const uint4 *>(
+        static_cast<const __nv_bfloat16 *>(a.q) +
+        ((size_t)(b * a.T + (q_real ? (rt * BM + rq) / a.G : 0)) * a.Hq + g * a.G +
+         (q_real ? (rt * BM + rq) % a.G : 0)) * D);
+    uint32_t qrow[QW];
+    int parents[4];
+    // Plain loads (L1-cached, so that a row's 16-byte pieces share their
+    // lines; coherent, since in a programmatic launch the preceding kernel may
+    // have written these inputs while this grid already ran).
+    auto load_q_and_parents = [&]() {
+        if (warp < 4) {
+#pragma unroll
+            for (int k = 0; k < QW / 4; ++k) {
+                const uint4 v = q_real ? q_src[k] : make_uint4(0, 0, 0, 0);
+                qrow[4 * k] = v.x;
+                qrow[4 * k + 1] = v.y;
+                qrow[4 * k + 2] = v.z;
+                qrow[4 * k + 3] = v.w;
+            }
+        }
+        if (warp == 3 && tree_cta) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int i = lane + 32 * k;
+                parents[k] = (i < a.T && (k < 2 || a.T > 64)) ? a.parent[(size_t)b * a.T + i] : -1;
+            }
+        }
+    };
+
+    // ------------------------------------ cache length and this CTA's keys
+    // Launch modes: an ordinary launch (or pdl alone) reads every input after
+    // the prerequisite grids complete; with cache_early the cache length, the
+    // block table and the cache tiles of the free ring stages are read before
+    // that; with inputs_early every input is, and only the writes wait.
+    const bool in_early = a.inputs_early != 0;
+    const bool c_early = in_early || a.cache_early != 0;
+    if (!c_early) wait_prerequisite_grids();
+    int L = a.cache_len[b];
+    // the Q and parent loads go out while the length is read, ahead of the
+    // ring's bulk traffic (issued once the length is known), so that they do
+    // not queue behind it
+    if (!c_early || in_early) load_q_and_parents();
     const bool cap_bad = (L < 0 || L + a.T > a.Lcap);
     if (cap_bad) {
         if (threadIdx.x == 0 && split == 0 && rt == 0 && g == 0) report(a.status, CLOVER_ERR_CAPACITY);
@@ -254,9 +374,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int kend = min(L, kbeg + chunk);
     const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
     const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
-    // the tree CTA takes its tree tile first (tile 0), so the one CTA with an
-    // extra tile does not finish on a load whose latency nothing hides
-    const int first_cache = tree_cta ? 1 : 0;
+    // The tree CTA takes its tree tile first, so that the one CTA with an
+    // extra tile does not end on a load whose latency nothing hides.  The
+    // order is the same in every launch mode, and with it the result.
+    const bool split_wait = c_early && !in_early;
+    const int tree_j = tree_cta ? 0 : -1;
+    const int tree_shift = tree_cta ? 1 : 0;   // tile j is cache tile j - tree_shift
     // this CTA appends the tree K/V to cache slots [L, L+T)
     const bool appender = a.append && tree_cta && rt == 0 && !cap_bad;
 
@@ -270,45 +393,68 @@ __global__ void __launch_bounds__(kThreads, 1)
     // staged: the split's first kPageSmem page ids are in s_pages (after the
     // setup barrier); later ones, and all of them before it, come from the table
     auto tile_pages = [&](int j, int (&pg)[kMaxBoxes], bool staged) {
-        if (!paged || j < first_cache) return;
-        const int key0 = kbeg + (j - first_cache) * BN;
+        if (!paged || j == tree_j) return;
+        const int key0 = kbeg + (j - tree_shift) * BN;
         for (int r = 0, x = 0; r < BN; r += box, ++x) {
             const int slot = key0 + r;
             const int pi = (slot >> a.page_shift) - first_page;
             pg[x] = slot >= kend ? 0 : (staged && pi < kPageSmem) ? s_pages[pi] : cache_page(a, b, slot);
         }
     };
-    // tile j of K (is_v == false) or V into ring stage `dst`
+    // tile j of K (is_v == false) or V into ring stage `dst`: a cache tile (an
+    // evict-first read) or, past the cache tiles, the tree tile
+    const uint64_t pol = l2_policy_evict_first();
     auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar, const int (&pg)[kMaxBoxes]) {
         mbar_arrive_expect_tx(bar, S::kv_bytes);
         const CUtensorMap *cache_map = is_v ? &tm_vc : &tm_kc;
         const CUtensorMap *new_map = is_v ? &tm_vn : &tm_kn;
-        if (j >= first_cache && paged) {
-            const int key0 = kbeg + (j - first_cache) * BN;
+        if (j != tree_j && paged) {
+            const int key0 = kbeg + (j - tree_shift) * BN;
             for (int r = 0, x = 0; r < BN; r += box, ++x) {
                 const int row = (key0 + r) & (a.page_size - 1);
 #pragma unroll
                 for (int dh = 0; dh < S::DH; ++dh)
-                    tma_load_3d(dst + dh * BN * 128 + r * 128, cache_map, bar, dh * 64, row, pg[x] * a.Hkv + g);
+                    tma_load_3d_hint(dst + dh * BN * 128 + r * 128, cache_map, bar, dh * 64, row, pg[x] * a.Hkv + g,
+                                     pol);
             }
-        } else if (j >= first_cache) {
+        } else if (j != tree_j) {
 #pragma unroll
-            for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + (j - first_cache) * BN, bg);
+            for (int dh = 0; dh < S::DH; ++dh)
+                tma_load_3d_hint(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + (j - tree_shift) * BN, bg, pol);
         } else {
 #pragma unroll
             for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, new_map, bar, dh * 64, g, b * a.T);
         }
     };
+    // The first ring stages start empty: their tiles are issued without a
+    // wait, in phase 0 (before the prerequisite grids complete, with
+    // cache_early alone: the cache tiles among them) or phase 1 (the rest).
+    auto issue_first = [&](bool is_v, int &issued, int phase) {
+        constexpr int NSmax = NSK > NSV ? NSK : NSV;
+        const int ns = is_v ? NSV : NSK;
+        uint8_t *ring = is_v ? sV : sK;
+        uint64_t *full = is_v ? v_full : k_full;
+        const int upto = min(ns, n_tiles);
+        int pg[NSmax][kMaxBoxes];
+        for (int j = 0; j < upto; ++j)
+            if ((phase == 0) == (split_wait && j != tree_j)) tile_pages(j, pg[j], false);
+        for (int j = 0; j < upto; ++j)
+            if ((phase == 0) == (split_wait && j != tree_j)) issue_tile(j, is_v, ring + j * S::kv_bytes, &full[j], pg[j]);
+        if (phase == 1) issued = upto;
+    };
 
-    // The tree tile (tile 0 of the tree CTA, ring stage 0) holds the T new
-    // keys or values in its first T rows once it has landed; TMA stores those
-    // rows straight from the ring to cache slots [L, L+T), then waits until the
-    // store has read them.  The producer does this before stage 0 takes its
-    // next tile (or after its loop when there is none).
+    // The tree tile (the tree CTA's last tile) holds the T new keys or values in
+    // its first T rows once it has landed; TMA stores those rows straight from
+    // the ring to cache slots [L, L+T), then waits until the store has read
+    // them (the rings hold the partial result after the loop).
     auto append_tile = [&](bool is_v) {
-        uint64_t *full = is_v ? &v_full[0] : &k_full[0];
-        const uint8_t *src = is_v ? sV : sK;
-        if (*s_abort || !mbar_wait(full, 0, kWaitNs)) {
+        const int jt = tree_j;
+        const int ns = is_v ? NSV : NSK;
+        const int s = jt % ns;
+        const uint32_t ph = (jt / ns) & 1;
+        uint64_t *full = is_v ? &v_full[s] : &k_full[s];
+        const uint8_t *src = (is_v ? sV : sK) + s * S::kv_bytes;
+        if (*s_abort || !mbar_wait(full, ph, kWaitNs)) {
             *s_abort = 1;
             return;
         }
@@ -319,77 +465,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         bulk_wait_group_read0();
     };
 
-    // ---------------------------------------------------------------- setup
-    // Each producer initialises the barriers of its ring (the K producer also
-    // every other one) and issues its first ring loads at once (the stages
-    // start empty), the K producer also the Q load, so that they overlap the
-    // TMEM allocation.
+    // The first ring stages, in two phases: with cache_early only, phase 0
+    // issues the cache tiles among them before the prerequisite grids
+    // complete (after an L2 prefetch of the Q rows); phase 1 stages the
+    // split's page ids (paged), waits for those grids and loads Q (with
+    // cache_early), and issues the rest of the first stages.
+    const bool producer = (warp == kVProducerWarp || warp == kKProducerWarp) && lane == 0;
+    const bool prod_v = warp == kVProducerWarp;
     int k_issued = 0, v_issued = 0;
-    if (warp == kVProducerWarp && lane == 0) {
-        for (int i = 0; i < NSV; ++i) {
-            mbar_init(&v_full[i], 1);
-            mbar_init(&v_empty[i], 1);
-        }
-        fence_barrier_init();
-        prefetch_tensormap(&tm_vc);
-        prefetch_tensormap(&tm_vn);
-        int pg[NSV][kMaxBoxes];
-        for (int j = 0; j < min(NSV, n_tiles); ++j) tile_pages(j, pg[j], false);
-        for (; v_issued < min(NSV, n_tiles); ++v_issued)
-            issue_tile(v_issued, true, sV + v_issued * S::kv_bytes, &v_full[v_issued], pg[v_issued]);
-    }
-    if (warp == kKProducerWarp) {
-        if (lane == 0) {
-            for (int i = 0; i < NSK; ++i) {
-                mbar_init(&k_full[i], 1);
-                mbar_init(&k_empty[i], 1);
-            }
-            for (int i = 0; i < 2; ++i) {
-                mbar_init(&s_full[i], 1);
-                mbar_init(&p_full[i], n_soft_warps);
-                mbar_init(&o_full[i], 1);
-            }
-            mbar_init(mma_done, 1);
-            mbar_init(q_full, 4);
-            mbar_init(m_free, n_split);
-            mbar_init(m_done, n_split);
-            mbar_init(m_data, 1);
-            if (n_split > 1) {
-                // every other split sends this CTA its rows [r0, r1) of the tile
-                const int per = (rows_here + n_split - 1) / n_split;
-                const int mine = max(0, min(rows_here, (split + 1) * per) - split * per);
-                mbar_arrive_expect_tx(m_data, (uint32_t)((n_split - 1) * mine * S::po_stride * 4));
-            }
-            *s_abort = 0;
-            *s_bad = false;
-            fence_barrier_init();
-            prefetch_tensormap(&tm_kc);
-            prefetch_tensormap(&tm_kn);
-            int pg[NSK][kMaxBoxes];
-            for (int j = 0; j < min(NSK, n_tiles); ++j) tile_pages(j, pg[j], false);
-            for (; k_issued < min(NSK, n_tiles); ++k_issued)
-                issue_tile(k_issued, false, sK + k_issued * S::kv_bytes, &k_full[k_issued], pg[k_issued]);
-        }
-    }
-    if (warp == kMmaWarp) {
-        tmem_alloc(s_tmem, S::tmem_cols);
-        tmem_relinquish();
-        // paged: the split's page ids, for the producers' loops
-        if (paged && kend > kbeg) {
+#pragma unroll 1
+    for (int phase = split_wait ? 0 : 1; phase < 2; ++phase) {
+        if (phase == 0 && q_real)
+            for (int c = 0; c < D * 2; c += 128) prefetch_l2(reinterpret_cast<const uint8_t *>(q_src) + c);
+        if (phase == 1 && paged && warp == kMmaWarp && kend > kbeg) {
             const int n_pg = min(kPageSmem, ((kend - 1) >> a.page_shift) - first_page + 1);
             for (int i = lane; i < n_pg; i += 32) s_pages[i] = cache_page(a, b, (first_page + i) << a.page_shift);
         }
+        if (phase == 1 && split_wait) {
+            wait_prerequisite_grids();
+            load_q_and_parents();
+        }
+        if (producer) issue_first(prod_v, prod_v ? v_issued : k_issued, phase);
     }
-    // the tree CTA's ancestor masks (warp 3 is otherwise idle here)
-    if (warp == 3 && tree_cta) tree_masks_build(parents, a.T, s_anc, s_bad);
-    // The cluster barrier is split: its wait (before the first remote arrive,
-    // in the merge) lets the key loop start without waiting for the other
-    // CTAs' setup.  The arrive is relaxed: fence_barrier_init has already
-    // published this CTA's barriers to the cluster, and a releasing arrive
-    // would hold each producer until its ring loads have landed.
+    // the tree CTA's ancestor masks (warp 3 has no other setup work)
+    if (warp == 3 && tree_cta) tree_masks_walk(parents, a.T, s_par, s_anc, s_bad);
+
     tc_fence_before();
-    __syncwarp();
-    if (n_split > 1) cluster_arrive_relaxed();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *s_tmem;
@@ -408,49 +509,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // ----------------------------------------------------- TMA producer warps
-    if (warp == kVProducerWarp) {
-        if (lane == 0) {
-            bool appended = false;
-            for (int j = v_issued; j < n_tiles; ++j) {
-                const int s = j % NSV;
-                if (appender && j == NSV) {
-                    append_tile(true);
-                    appended = true;
-                }
-                int pg[kMaxBoxes];
-                tile_pages(j, pg, true);
-                if (!mbar_wait(&v_empty[s], ((j / NSV) - 1) & 1, kWaitNs)) {
-                    *s_abort = 1;
-                    break;
-                }
-                if (*s_abort) break;
-                issue_tile(j, true, sV + s * S::kv_bytes, &v_full[s], pg);
-                v_issued = j + 1;
+    if ((warp == kVProducerWarp || warp == kKProducerWarp) && lane == 0) {
+        const bool is_v = warp == kVProducerWarp;
+        const int ns = is_v ? NSV : NSK;
+        uint8_t *ring = is_v ? sV : sK;
+        uint64_t *full = is_v ? v_full : k_full;
+        uint64_t *empty = is_v ? v_empty : k_empty;
+        int &issued = is_v ? v_issued : k_issued;
+        // the append reads the tree tile's stage: before the stage takes its
+        // next tile, or after the loop (a write: after the prerequisite grids)
+        bool appended = false;
+        auto append = [&]() {
+            if (in_early) wait_prerequisite_grids();
+            append_tile(is_v);
+            appended = true;
+        };
+        for (int j = issued; j < n_tiles; ++j) {
+            const int s = j % ns;
+            if (appender && !appended && j == tree_j + ns) append();
+            int pg[kMaxBoxes];
+            tile_pages(j, pg, true);
+            if (!mbar_wait(&empty[s], ((j / ns) - 1) & 1, kWaitNs)) {
+                *s_abort = 1;
+                break;
             }
-            if (appender && !appended && v_issued == n_tiles) append_tile(true);
+            if (*s_abort) break;
+            issue_tile(j, is_v, ring + s * S::kv_bytes, &full[s], pg);
+            issued = j + 1;
         }
-    }
-    if (warp == kKProducerWarp) {
-        if (lane == 0) {
-            bool appended = false;
-            for (int j = k_issued; j < n_tiles; ++j) {
-                const int s = j % NSK;
-                if (appender && j == NSK) {
-                    append_tile(false);
-                    appended = true;
-                }
-                int pg[kMaxBoxes];
-                tile_pages(j, pg, true);
-                if (!mbar_wait(&k_empty[s], ((j / NSK) - 1) & 1, kWaitNs)) {
-                    *s_abort = 1;
-                    break;
-                }
-                if (*s_abort) break;
-                issue_tile(j, false, sK + s * S::kv_bytes, &k_full[s], pg);
-                k_issued = j + 1;
-            }
-            if (appender && !appended && k_issued == n_tiles) append_tile(false);
-        }
+        if (appender && !appended && issued == n_tiles) append();
     }
 
     // --------------------------------------------------------- MMA issuer warp
@@ -477,13 +564,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_commit(&k_empty[s]);
             return true;
         };
-        if (ok && n_tiles > 0) ok = issue_s(0);
+        int s_issued = 0;
         for (int j = 0; ok && j < n_tiles; ++j) {
             if (*s_abort) {
                 ok = false;
                 break;
             }
-            if (j + 1 < n_tiles && !(ok = issue_s(j + 1))) break;
+            // S of tiles j and j + 1 are issued before the P.V product of tile j
+            while (ok && s_issued < min(j + 2, n_tiles)) ok = issue_s(s_issued++);
+            if (!ok) break;
             const int s = j % NSV;
             const int sb = j & 1;
             if (!mbar_wait(&p_full[sb], (j >> 1) & 1, kWaitNs) || !mbar_wait(&v_full[s], (j / NSV) & 1, kWaitNs)) {
@@ -535,15 +624,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after();
-            const bool tree_tile = tree_cta && j == 0;
-            const int key0 = kbeg + (j - first_cache) * BN;
+            const bool tree_tile = j == tree_j;
+            const int key0 = kbeg + (j - tree_shift) * BN;
             const int n_valid = tree_tile ? a.T : min(BN, kend - key0);
             // Keys of a 64-key block of the tile that this row sees: a prefix
             // of the cache keys, or the row's ancestors among the (at most
             // 128) tree keys, word blk of its mask.  Every tile runs the same
-            // instructions, so the one tree tile, late in the loop, brings no
-            // code into the instruction cache (a miss then waits on a
-            // saturated memory system).
+            // instructions, so the one tree tile brings no code into the
+            // instruction cache (a miss then waits on a saturated memory system).
             auto block_vis = [&](int blk) -> uint64_t {
                 const int nv = n_valid - 64 * blk;
                 const uint64_t prefix = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
@@ -669,124 +757,39 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncthreads();
     tc_fence_after();
-    if (n_split > 1) {
-        // this CTA's rings are free: the other splits may send their partials
-        cluster_wait_acquire();               // every CTA's barriers exist
-        if (warp == 1 && lane < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_free), lane));
-    }
-    __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(a.out);
-    const bool row_ok = softmax_warp && r < rows_here;
-    float *part_o = reinterpret_cast<float *>(sK);            // [BM][D + 4] fp32, this CTA's partial
-    float *recv = reinterpret_cast<float *>(sV);              // [n_split][per][D + 4]
-    // 64 O columns of this warp's lanes.  The TMEM loads are warp-collective:
-    // every lane runs them, rows past the tile's real rows only skip the stores
-    auto load_o = [&](int cc, float (&x0)[32], float (&x1)[32]) {
-        if (o_ready) {
-            tmem_ld32(tO + lane_base + cc * 32, x0);
-            tmem_ld32(tO + lane_base + cc * 32 + 32, x1);
-            tmem_wait_ld();
-        } else {
-#pragma unroll
-            for (int c = 0; c < 32; ++c) x0[c] = x1[c] = 0.f;
-        }
-    };
-    // KS = 2: the second key half's rows (O, m, l) go to rows 64.. of part_o,
-    // where the warps of the first half merge them into their own.  Those
-    // warps load their first 64 O columns meanwhile.
-    float x0[32], x1[32];
-    if (KS == 2) {
-        if (softmax_warp && half == 1) {
-            float *dst = part_o + (64 + r) * S::po_stride;
-#pragma unroll 1
-            for (int cc = 0; cc < D / 32; cc += 2) {
-                load_o(cc, x0, x1);
-                if (row_ok) {
-#pragma unroll
-                    for (int c = 0; c < 32; c += 4) {
-                        *reinterpret_cast<float4 *>(dst + cc * 32 + c) =
-                            make_float4(x0[c], x0[c + 1], x0[c + 2], x0[c + 3]);
-                        *reinterpret_cast<float4 *>(dst + cc * 32 + 32 + c) =
-                            make_float4(x1[c], x1[c + 1], x1[c + 2], x1[c + 3]);
-                    }
-                }
-            }
-            if (row_ok)
-                *reinterpret_cast<float2 *>(dst + D) =
-                    make_float2(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f);
-        }
-        if (softmax_warp && half == 0) load_o(0, x0, x1);
-        __syncthreads();
-    }
-    if (softmax_warp && half == 0) {
-        // this row's (m, l) and the weights of its key halves
-        float m_row = o_ready ? m_ref : -INFINITY;
-        float l_row = o_ready ? l_run : 0.f;
-        float wa = 1.f, wb = 0.f;
-        const float *ob = part_o + (64 + r) * S::po_stride;
-        if (KS == 2 && row_ok) {
-            const float2 mlb = *reinterpret_cast<const float2 *>(ob + D);
-            const float M = fmaxf(m_row, mlb.x);
-            wa = (m_row == -INFINITY) ? 0.f : ex2_approx(m_row - M);
-            wb = (mlb.x == -INFINITY) ? 0.f : ex2_approx(mlb.x - M);
-            m_row = M;
-            l_row = wa * l_row + wb * mlb.y;
-        }
-        // 64 columns of the row: the output (one split) or the partial row.
-        // The other half's 64 values are read in one batch before any store.
-        auto emit = [&](int cc, float (&y0)[32], float (&y1)[32]) {
-            if (KS == 2) {
-                float4 yb[16];
-#pragma unroll
-                for (int c = 0; c < 16; ++c) yb[c] = *reinterpret_cast<const float4 *>(ob + cc * 32 + 4 * c);
-#pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    y0[4 * c] = fmaf(wb, yb[c].x, wa * y0[4 * c]);
-                    y0[4 * c + 1] = fmaf(wb, yb[c].y, wa * y0[4 * c + 1]);
-                    y0[4 * c + 2] = fmaf(wb, yb[c].z, wa * y0[4 * c + 2]);
-                    y0[4 * c + 3] = fmaf(wb, yb[c].w, wa * y0[4 * c + 3]);
-                    y1[4 * c] = fmaf(wb, yb[8 + c].x, wa * y1[4 * c]);
-                    y1[4 * c + 1] = fmaf(wb, yb[8 + c].y, wa * y1[4 * c + 1]);
-                    y1[4 * c + 2] = fmaf(wb, yb[8 + c].z, wa * y1[4 * c + 2]);
-                    y1[4 * c + 3] = fmaf(wb, yb[8 + c].w, wa * y1[4 * c + 3]);
-                }
-            }
-            if (n_split == 1) {
-                // the output row (node, head); only this path needs it
-                const int R = rt * BM + r;
-                const int i = R / a.G;
-                const int h = g * a.G + (R % a.G);
-                const float inv = l_row > 0.f ? rcp_approx(l_row) : 1.f;
-                __nv_bfloat16 *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D + cc * 32;
-#pragma unroll
-                for (int c = 0; c < 64; c += 8) {
-                    const float *x = c < 32 ? y0 + c : y1 + (c - 32);
-                    uint4 w;
-                    w.x = pack_bf16x2(x[0] * inv, x[1] * inv);
-                    w.y = pack_bf16x2(x[2] * inv, x[3] * inv);
-                    w.z = pack_bf16x2(x[4] * inv, x[5] * inv);
-                    w.w = pack_bf16x2(x[6] * inv, x[7] * inv);
-                    *reinterpret_cast<uint4 *>(dst + c) = w;
-                }
-            } else {
-                float *po = part_o + r * S::po_stride + cc * 32;
-#pragma unroll
-                for (int c = 0; c < 32; c += 4) {
-                    *reinterpret_cast<float4 *>(po + c) = make_float4(y0[c], y0[c + 1], y0[c + 2], y0[c + 3]);
-                    *reinterpret_cast<float4 *>(po + 32 + c) = make_float4(y1[c], y1[c + 1], y1[c + 2], y1[c + 3]);
-                }
-            }
-        };
-        // two TMEM loads in flight per wait (the first pair is loaded already with KS = 2)
+    // (1) every softmax warp moves the O rows, m and l of its TMEM lanes to
+    // part_o row 32 quad + lane: KS = 1, tile row r; KS = 2, the first key half
+    // of tile row r in rows 0-63 and the second half in rows 64-127.  The TMEM
+    // loads are warp-collective: every lane runs them, rows past the tile's
+    // real rows only skip the stores.
+    float *part_o = reinterpret_cast<float *>(sK);            // [BM][D + 4] fp32
+    if (softmax_warp) {
+        const bool real = r < rows_here;
+        float *dst = part_o + (quad * 32 + lane) * S::po_stride;
 #pragma unroll 1
         for (int cc = 0; cc < D / 32; cc += 2) {
-            if (KS == 1 || cc > 0) load_o(cc, x0, x1);
-            if (row_ok) emit(cc, x0, x1);
+            float x0[32], x1[32];
+            if (o_ready) {
+                tmem_ld32(tO + lane_base + cc * 32, x0);
+                tmem_ld32(tO + lane_base + cc * 32 + 32, x1);
+                tmem_wait_ld();
+            } else {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) x0[c] = x1[c] = 0.f;
+            }
+            if (real) {
+#pragma unroll
+                for (int c = 0; c < 32; c += 4) {
+                    *reinterpret_cast<float4 *>(dst + cc * 32 + c) = make_float4(x0[c], x0[c + 1], x0[c + 2], x0[c + 3]);
+                    *reinterpret_cast<float4 *>(dst + cc * 32 + 32 + c) =
+                        make_float4(x1[c], x1[c + 1], x1[c + 2], x1[c + 3]);
+                }
+            }
         }
-        if (row_ok && n_split > 1)
-            *reinterpret_cast<float2 *>(part_o + r * S::po_stride + D) = make_float2(m_row, l_row);
-        if (n_split > 1) fence_proxy_async_smem();   // the bulk copies below read these rows
+        if (real)
+            *reinterpret_cast<float4 *>(dst + D) =
+                make_float4(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f, 0.f, 0.f);
     }
-
     // every TMEM access and MMA is finished before TMEM is released
     tc_fence_before();
     __syncthreads();
@@ -797,117 +800,93 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_dealloc(tmem, S::tmem_cols);
     }
     if (tree_cta && rt == 0 && threadIdx.x == 0 && *s_bad) report(a.status, CLOVER_ERR_BAD_TREE);
-    if (n_split > 1) {
-        // ------------------------------------------ split merge in the cluster
-        // CTA `split` merges rows [r0, r1) of the tile.  Once every CTA is out
-        // of its key loop (m_free), lane k of warp 0 sends CTA k (k != split)
-        // that CTA's rows of this CTA's partial with one bulk copy into its V
-        // ring (completing on its m_data); then every CTA merges its own rows
-        // from shared memory.
-        const int per = (rows_here + n_split - 1) / n_split;
-        const int r0 = split * per;
-        const int r1 = min(rows_here, r0 + per);
-        constexpr uint32_t row_bytes = S::po_stride * 4;
-        bool ok = true;
-        if (warp == 0) {
-            if (lane < n_split) {
-                ok = mbar_wait_cluster(m_free, 0, kWaitNs);
-                const int k0 = lane * per;
-                const int k1 = min(rows_here, k0 + per);
-                if (ok && lane != split && k1 > k0)
-                    bulk_copy_to_cluster(mapa_shared(smem_u32(recv) + split * per * row_bytes, lane),
-                                         part_o + k0 * S::po_stride, (k1 - k0) * row_bytes,
-                                         mapa_shared(smem_u32(m_data), lane));
-            }
-            ok = __all_sync(0xffffffffu, ok);
-            if (lane == 0 && ok) ok = mbar_wait_cluster(m_data, 0, kWaitNs);
-        }
-        // one thread waited; every thread acquires the received rows itself
-        const bool got = __syncthreads_and(ok) && mbar_test_cluster(m_data, 0);
-        // every partial row this CTA needs is here: its senders may exit
-        if (warp == 1 && lane < n_split) mbar_arrive_remote(mapa_shared(smem_u32(m_done), lane));
-        if (got) {
-            switch (n_split) {
-#define CLOVER_MERGE_CASE(NS) \
-    case NS: merge_rows<D, NS>(part_o, recv, S::po_stride, split, per, r0, r1, rt * BM, a, b, g, out); break;
-                CLOVER_MERGE_CASE(2)
-                CLOVER_MERGE_CASE(3)
-                CLOVER_MERGE_CASE(4)
-                CLOVER_MERGE_CASE(5)
-                CLOVER_MERGE_CASE(6)
-                CLOVER_MERGE_CASE(7)
-                CLOVER_MERGE_CASE(8)
-#undef CLOVER_MERGE_CASE
-                default: break;
-            }
-        } else {
-            *s_abort = 1;
-        }
-        // the copies reading this CTA's partial are complete before its
-        // shared memory goes away
-        ok = true;
-        if (threadIdx.x == 0) ok = mbar_wait_cluster(m_done, 0, kWaitNs);
-        if (!__syncthreads_and(ok)) *s_abort = 1;
-    }
+    // every global write below comes after the prerequisite grids complete
+    if (in_early) wait_prerequisite_grids();
     // the appended tree K/V is in global memory before the CTA exits
     if (appender && (warp == kKProducerWarp || warp == kVProducerWarp) && lane == 0) bulk_wait_group0();
-    if (*s_abort && threadIdx.x == 0) report(a.status, CLOVER_ERR_TIMEOUT);
-}
 
-struct TcLaunchCache {
-    int sms = 0;
-    int max_clusters[kMaxCluster + 1] = {0};   // co-resident clusters per cluster size (0: not queried)
-};
-
-template <int D, int KS, bool PAGED>
-int max_active_clusters(int n, TcLaunchCache &cache) {
-    if (cache.max_clusters[n] == 0) {
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(1, n, n);
-        cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = TcSmem<D, KS>::alloc;
-        cudaLaunchAttribute attr;
-        attr.id = cudaLaunchAttributeClusterDimension;
-        attr.val.clusterDim.x = 1;
-        attr.val.clusterDim.y = n;
-        attr.val.clusterDim.z = 1;
-        cfg.attrs = &attr;
-        cfg.numAttrs = 1;
-        int num = 0;
-        if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D, KS, PAGED>, &cfg) != cudaSuccess) {
-            cudaGetLastError();
-            num = -1;
+    // (2) The split merge.  Every split but the last (the tree split, which
+    // has the most work and ends last) combines its two key halves, copies its
+    // rows to its workspace slot and counts itself in at the group's counter
+    // (release); then it is done.  The last split waits (bounded) until the
+    // others are in (acquire), loads their rows and merges every source of a
+    // row (its own halves and the other splits' rows) into the output.  With
+    // one split there are no others.
+    const int grp = bg * a.row_tiles + rt;
+    float *slots = n_split > 1 ? a.part_o + (size_t)grp * n_split * a.slot_rows * S::po_stride : nullptr;
+    constexpr uint32_t row_bytes = S::po_stride * 4;
+    const int others = tree_cta ? n_split - 1 : 0;
+    const int n_src = KS + others;
+    __nv_bfloat16 *out = static_cast<__nv_bfloat16 *>(a.out);
+    if (n_split > 1 && !tree_cta) {
+        if (KS == 2) {
+            row_weights<D, KS>(part_o, nullptr, 0, 0, rows_here, KS, s_wts, false);
+            __syncthreads();
+            merge_pass<D, KS>(part_o, nullptr, s_wts, KS, 0, 0, rows_here, rt * BM, a, b, g, nullptr);
+            if (threadIdx.x < rows_here)
+                *reinterpret_cast<float2 *>(part_o + threadIdx.x * S::po_stride + D) =
+                    make_float2(s_wts[threadIdx.x * kMaxSrc + kMaxSrc - 2], s_wts[threadIdx.x * kMaxSrc + kMaxSrc - 1]);
         }
-        cache.max_clusters[n] = num > 0 ? num : -1;
+        fence_proxy_async_smem();             // the bulk copy reads these rows
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            bulk_store_s2g(slots + (size_t)split * a.slot_rows * S::po_stride, part_o, rows_here * row_bytes);
+            bulk_commit_group();
+            bulk_wait_group0();
+            fence_proxy_async_global();
+            red_add_release_gpu(a.counters + grp, 1u);
+        }
+    } else {
+        if (others > 0 && threadIdx.x == 0) {
+            bool in = ld_acquire_gpu(a.counters + grp) >= (unsigned)others;
+            if (!in) {
+                const uint64_t t0 = globaltimer_ns();
+                while (!(in = ld_acquire_gpu(a.counters + grp) >= (unsigned)others) && globaltimer_ns() - t0 < kWaitNs)
+                    __nanosleep(64);
+            }
+            if (in) {
+                a.counters[grp] = 0u;                 // ready for the next call
+                fence_proxy_async_global();
+            } else {
+                *s_abort = 1;
+            }
+        }
+        __syncthreads();
+        if (!*s_abort) {
+            float *recv = reinterpret_cast<float *>(sK + S::own_bytes);
+            const int rpp = others > 0 ? min(rows_here, S::recv_bytes / (others * (int)row_bytes)) : rows_here;
+            int pass = 0;
+            for (int p0 = 0; p0 < rows_here; p0 += rpp, ++pass) {
+                const int p1 = min(rows_here, p0 + rpp);
+                if (others > 0 && threadIdx.x == 0) {
+                    const uint32_t bytes = (uint32_t)(p1 - p0) * row_bytes;
+                    mbar_arrive_expect_tx(g_full, bytes * others);
+                    for (int k = 0; k < others; ++k)
+                        bulk_load_g2s(recv + (size_t)k * rpp * S::po_stride,
+                                      slots + ((size_t)k * a.slot_rows + p0) * S::po_stride, bytes, g_full);
+                }
+                const bool got = others == 0 || mbar_wait(g_full, pass & 1, kWaitNs);
+                if (got) row_weights<D, KS>(part_o, recv, rpp, p0, p1, n_src, s_wts, true);
+                else *s_abort = 1;
+                __syncthreads();   // the weights are in shared memory
+                if (!*s_abort) merge_pass<D, KS>(part_o, recv, s_wts, n_src, rpp, p0, p1, rt * BM, a, b, g, out);
+                // the received rows are read before the next pass overwrites them
+                __syncthreads();
+                if (*s_abort) break;
+            }
+        }
     }
-    return cache.max_clusters[n];
+    if (*s_abort && threadIdx.x == 0) report(a.status, CLOVER_ERR_TIMEOUT);
 }
 
 template <int D, int KS, bool PAGED>
 cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     static unsigned long long done[64];
-    static TcLaunchCache caches[64];
     auto kernel = tree_attn_tc_kernel<D, KS, PAGED>;
     cudaError_t err = ensure_smem_attr(kernel, TcSmem<D, KS>::alloc, done);
     if (err != cudaSuccess) return err;
-    int dev = 0;
-    if ((err = cudaGetDevice(&dev)) != cudaSuccess) return err;
-    TcLaunchCache &cache = caches[dev < 64 ? dev : 63];
-    if (cache.sms == 0 && (err = cudaDeviceGetAttribute(&cache.sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
-        return err;
-
-    // splits per head: as many as fill the SMs in one wave of clusters
-    const long base = (long)a.B * a.Hkv * a.row_tiles;
-    const int by_len = (a.Lcap + 255) / 256;
-    int n = 1;
-    for (int c = kMaxCluster; c >= 2; --c) {
-        if (c > by_len || base * c > cache.sms) continue;
-        if (max_active_clusters<D, KS, PAGED>(c, cache) >= base) {
-            n = c;
-            break;
-        }
-    }
-    a.n_split = n;
+    if (a.n_split < 1 || a.n_split > kMaxSplits) return cudaErrorInvalidValue;
+    if (a.n_split > 1 && (!a.part_o || !a.counters)) return cudaErrorInvalidValue;
 
     CUtensorMap kc, vc, kn, vn, ks, vs;
     const uint64_t e = 2;
@@ -935,17 +914,15 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     if (!ok) return cudaErrorInvalidValue;
 
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(a.row_tiles, n, a.B * a.Hkv);
+    cfg.gridDim = dim3(a.row_tiles, a.n_split, a.B * a.Hkv);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = TcSmem<D, KS>::alloc;
     cfg.stream = stream;
     cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeClusterDimension;
-    attr.val.clusterDim.x = 1;
-    attr.val.clusterDim.y = n;
-    attr.val.clusterDim.z = 1;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = &attr;
-    cfg.numAttrs = n > 1 ? 1 : 0;
+    cfg.numAttrs = a.pdl ? 1 : 0;
     err = cudaLaunchKernelEx(&cfg, kernel, kc, vc, kn, vn, ks, vs, a);
     if (err != cudaSuccess) return err;
     return cudaGetLastError();
@@ -954,6 +931,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
 }  // namespace
 
 int tc_row_tile() { return BM; }
+int tc_max_splits() { return kMaxSplits; }
 
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream) {
     // a tile of at most 64 real rows: two key groups per row (KS = 2)

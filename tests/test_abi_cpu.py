@@ -49,7 +49,11 @@ def test_workspace_sizes(lib):
     assert ws(1, 16, 8, 8, 64, 192, 0) == 0              # short cache: one split, no workspace
     big = ws(1, 64, 32, 32, 128, 4160, 0)                # fp32: CUDA-core split-KV merge
     assert big > 0 and big % 256 == 0
-    assert ws(1, 64, 32, 32, 128, 4160, 1) == 0          # bf16: tensor-core path merges on chip
+    # bf16 (tensor cores): 32 heads x 4 splits (one wave of 152 SMs) of 64 partial rows of
+    # D + 4 floats, plus 32 arrival counters rounded up to 256 bytes
+    assert ws(1, 64, 32, 32, 128, 4160, 1) == 32 * 4 * 64 * (128 + 4) * 4 + 256
+    assert ws(4, 64, 64, 8, 128, 8256, 1) == 0            # 128 (head, row tile) groups: one split each
+    assert ws(16, 32, 32, 32, 128, 8256, 1) == 0          # 512 heads: one split each
     assert ws(1, 129, 8, 8, 64, 192, 0) == 0             # T > 128 unsupported
     assert ws(1, 16, 8, 8, 96, 192, 0) == 0              # D = 96 unsupported
     assert ws(1, 16, 6, 4, 64, 192, 0) == 0              # Hq not a multiple of Hkv
@@ -107,7 +111,8 @@ def test_attn_ex_and_commit_host_validation(lib):
     ex = lambda flags, T=4: lib.clover_verify_attn_ex(
         P(16), P(16), P(16), P(16), P(16), P(16), P(16), P(16), 1, T, 2, 2, 64, 64, 1, 0.0, None, 0, None, None,
         flags)
-    assert ex(2) == 1 and ex(0xFFFFFFFE) == 1             # unknown flag bits
+    assert ex(16) == 1 and ex(0xFFFFFFF0) == 1            # unknown flag bits
+    assert ex(15, T=129) == 2                                # the known bits (append off, PDL, cache/inputs ready)
     assert ex(1, T=129) == 2 and ex(0, T=129) == 2           # the limits of clover_verify_attn
     com = lambda cl, ncl, kn=16, vn=16, B=2, T=4, D=64: lib.clover_kv_commit(
         P(16), P(16), P(kn), P(vn), P(cl), P(16), P(16), P(ncl), None, B, T, 2, D, 64, 1, None, None)

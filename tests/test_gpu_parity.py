@@ -125,7 +125,7 @@ def test_full_size_workloads(name, schedule, cuda):
 
 
 # ---------------------------------------------------------------------------
-# every split count of the tensor-core path's cluster merge
+# every split count of the tensor-core path's split merge
 # ---------------------------------------------------------------------------
 
 # One KV head, so the launcher's split count is min(8, Lcap / 256 rounded up):
@@ -144,6 +144,145 @@ def test_split_counts_and_row_groups(L, Hq, D, cuda):
     t = to_dev(host, cuda)
     step = run_gpu(t)
     compare_full(host, step, t)
+
+
+@pytest.mark.parametrize("dtype_name", ["tiny_f32", "7b_l2048"])
+def test_one_workspace_serves_smaller_capacities(dtype_name, cuda):
+    """A workspace sized for the largest capacity serves calls with smaller
+    ones (fewer splits, a smaller partial area): the arrival counters sit at
+    the start, where every split count finds them.  Calls alternate between
+    capacities; every output equals a call with its own fresh workspace."""
+    over = dict(T=16, Hq=4, Hkv=4, D=128, V=1000, branching=(4, 2, 1, 1))
+    lens = [2900, 700, 1300, 2900, 300, 1700]
+    sets = [to_dev(workloads.make(workloads.get(dtype_name, L=L, seed=90 + i, **over), logits=False), cuda)
+            for i, L in enumerate(lens)]
+    dt = sets[0]["q"].dtype
+    size = lambda s: pkg.clover_verify_attn_workspace_size(1, 16, 4, 4, 128, s["Lcap"], dt)
+    sizes = [size(s) for s in sets]
+    assert len(set(sizes)) > 2                            # several split counts
+    ws = torch.zeros(max(sizes), dtype=torch.uint8, device=cuda)
+    st = torch.zeros(1, dtype=torch.int32, device=cuda)
+    for rep in range(2):
+        for i, s in enumerate(sets):
+            out = torch.empty_like(s["q"])
+            pkg.clover_verify_attn(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"],
+                                   s["parent"], out, workspace=ws, status=st, append=False)
+            own = torch.zeros(max(sizes[i], 16), dtype=torch.uint8, device=cuda)
+            ref = torch.empty_like(s["q"])
+            pkg.clover_verify_attn(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"],
+                                   s["parent"], ref, workspace=own if sizes[i] else None, status=st, append=False)
+            torch.cuda.synchronize()
+            assert int(st.item()) == 0
+            bits = torch.int16 if dt == torch.bfloat16 else torch.int32
+            assert torch.equal(out.view(bits), ref.view(bits)), (rep, i)
+
+
+# ---------------------------------------------------------------------------
+# programmatic dependent launch of the tensor-core attention
+# ---------------------------------------------------------------------------
+
+def _attn_chain(sets, ws, st, pdl, cache_ready, graph=False):
+    """Attention calls back to back on one stream, call i+1 taking call i's
+    output as its q, k_new and v_new (MHA: out has their shape) and its own
+    cache; returns the outputs (optionally captured and replayed as one CUDA
+    graph)."""
+    outs = [torch.full_like(s["q"], float("nan")) for s in sets]
+
+    def run():
+        q = kn = vn = None
+        for i, s in enumerate(sets):
+            q, kn, vn = (s["q"], s["k_new"], s["v_new"]) if i == 0 else (outs[i - 1],) * 3
+            pkg.clover_verify_attn(q, kn, vn, s["k_cache"], s["v_cache"], s["cache_len"], s["parent"], outs[i],
+                                   workspace=ws, status=st, append=False, pdl=pdl, cache_ready=cache_ready)
+
+    if graph:
+        stream = torch.cuda.Stream()
+        with torch.cuda.stream(stream):
+            run()                       # eager first: per-kernel attributes are set outside the capture
+        torch.cuda.synchronize()
+        for o in outs:
+            o.fill_(float("nan"))
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            run()
+        g.replay()
+    else:
+        run()
+    torch.cuda.synchronize()
+    return outs
+
+
+@pytest.mark.parametrize("graph", [False, True])
+@pytest.mark.parametrize("cache_ready", [False, True])
+def test_pdl_chain_reads_inputs_after_the_previous_kernel(cache_ready, graph, cuda):
+    """CLOVER_ATTN_PDL (and CLOVER_ATTN_CACHE_READY, true here: every call has
+    its own cache): a call may start while the previous one runs, but its q,
+    k_new and v_new are that call's output, so it must read them only after it
+    completes.  The outputs equal ordinary launches' bit for bit (same split
+    plan, shared workspace), and the first matches the oracle."""
+    n = 4
+    ws_ = [workloads.get("7b_l2048", T=64, Hq=8, Hkv=8, L=1900 + 97 * i, V=1000, seed=50 + i) for i in range(n)]
+    hosts = [workloads.make(w, logits=False) for w in ws_]
+    sets = [to_dev(h, cuda) for h in hosts]
+    need = max(pkg.clover_verify_attn_workspace_size(1, 64, 8, 8, 128, s["Lcap"], torch.bfloat16) for s in sets)
+    assert need > 0                                       # several splits per head: the L2 merge runs
+    ws = torch.zeros(need, dtype=torch.uint8, device=cuda)
+    st = torch.zeros(1, dtype=torch.int32, device=cuda)
+    ref = _attn_chain(sets, ws, st, pdl=False, cache_ready=False)
+    got = _attn_chain(sets, ws, st, pdl=True, cache_ready=cache_ready, graph=graph)
+    assert int(st.item()) == 0
+    for i in range(n):
+        assert torch.equal(got[i].view(torch.int16), ref[i].view(torch.int16)), f"call {i}"
+    h = hosts[0]
+    want = oracle.tree_attention(h["q"], h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["cache_len"],
+                                 h["parent"])
+    assert (ref[0].double().cpu() - want).abs().max().item() <= ATOL[torch.bfloat16]
+
+
+@pytest.mark.parametrize("graph", [False, True])
+def test_pdl_inputs_ready_independent_calls(graph, cuda):
+    """CLOVER_ATTN_INPUTS_READY: calls on independent inputs (the statement
+    holds) run their key loops while the previous call finishes; their writes
+    (the shared workspace's slots and counters, the output) still wait for
+    it.  Six calls, three of them into one output buffer: every output equals
+    ordinary launches' bit for bit, the shared buffer holds the last call's."""
+    n = 6
+    ws_ = [workloads.get("7b_l2048", T=64, Hq=8, Hkv=8, L=1500 + 211 * i, V=1000, seed=70 + i) for i in range(n)]
+    sets = [to_dev(workloads.make(w, logits=False), cuda) for w in ws_]
+    need = max(pkg.clover_verify_attn_workspace_size(1, 64, 8, 8, 128, s["Lcap"], torch.bfloat16) for s in sets)
+    assert need > 0
+    ws = torch.zeros(need, dtype=torch.uint8, device=cuda)
+    st = torch.zeros(1, dtype=torch.int32, device=cuda)
+
+    def run(pdl, outs):
+        for i, s in enumerate(sets):
+            pkg.clover_verify_attn(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"],
+                                   s["parent"], outs[i], workspace=ws, status=st, append=False, pdl=pdl,
+                                   inputs_ready=pdl)
+
+    ref = [torch.empty_like(s["q"]) for s in sets]
+    run(False, ref)
+    shared = torch.full_like(sets[0]["q"], float("nan"))
+    outs = [torch.full_like(s["q"], float("nan")) for s in sets]
+    outs[1] = outs[3] = outs[5] = shared
+    if graph:
+        stream = torch.cuda.Stream()
+        with torch.cuda.stream(stream):
+            run(True, outs)
+        torch.cuda.synchronize()
+        for o in outs:
+            o.fill_(float("nan"))
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            run(True, outs)
+        g.replay()
+    else:
+        run(True, outs)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    for i in (0, 2, 4):
+        assert torch.equal(outs[i].view(torch.int16), ref[i].view(torch.int16)), f"call {i}"
+    assert torch.equal(shared.view(torch.int16), ref[5].view(torch.int16))
 
 
 # ---------------------------------------------------------------------------
