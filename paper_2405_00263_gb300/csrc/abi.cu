@@ -58,6 +58,7 @@ clover_status check_attn_sizes(int B, int T, int Hq, int Hkv, int D, int Lcap, i
     if (T > kMaxTreeNodes || (D != 64 && D != 128) || Hq % Hkv != 0) return CLOVER_ERR_UNSUPPORTED;
     if (Lcap < T) return CLOVER_ERR_INVALID_ARG;
     if (B > 65535 || Hkv > 65535) return CLOVER_ERR_UNSUPPORTED;
+    if ((unsigned long long)B * T * Hq >= (1ull << 32)) return CLOVER_ERR_UNSUPPORTED;   // output rows: 32-bit ids
     return CLOVER_OK;
 }
 

@@ -90,13 +90,14 @@ struct TcSmem {
     static constexpr int k_off = 0;
     static constexpr int v_off = k_off + NSK * kv_bytes;
     static constexpr int bar_off = v_off + NSV * kv_bytes;
-    static constexpr int n_bars = 2 * NSK + 2 * NSV + 9;
+    static constexpr int n_bars = 2 * NSK + 2 * NSV + 10;
     static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad
     static constexpr int anc_off = misc_off + 16;                  // ancestor masks [128][2]
     static constexpr int pages_off = anc_off + kMaxTreeNodes * kMaskWords * 8;   // paged: page ids of the split
     static constexpr int wts_off = pages_off + kPageSmem * 4;      // merge weights [BM][kMaxSrc]
     static constexpr int par_off = wts_off + BM * kMaxSrc * 4;     // the tree's parent array [128]
-    static constexpr int total = par_off + kMaxTreeNodes * 4;
+    static constexpr int orow_off = par_off + kMaxTreeNodes * 4;   // output row of each tile row [BM]
+    static constexpr int total = orow_off + BM * 4;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
     // TMEM columns: S/P 2 x BN, O D, Q D / 2 (two bf16 per column), rounded up
     // to a power of two.  All 512 columns of an SM go to one CTA only when
@@ -137,21 +138,20 @@ __device__ __forceinline__ float rcp_approx(float x) {
 // sum_s 2^(m_s - M) l_s already in shared memory.  Source s < KS of row rr is
 // this CTA's row rr + 64 s of `own` (its key halves); source KS + k is the
 // k-th other split's, row rr - p0 of slot k of `recv`.  Rows [p0, p1).  A warp
-// takes 4 rows at a time and lane l their columns [4 l, 4 l + 4) (D = 128;
+// takes 8 rows at a time and lane l their columns [4 l, 4 l + 4) (D = 128;
 // D = 64 uses lanes 0-15): each shared-memory load of the warp reads one row's
-// contiguous 512 bytes, free of bank conflicts.  With `out` == nullptr the
+// contiguous 512 bytes, free of bank conflicts, and 8 are in flight per
+// source.  Output row rr goes to out + orow[rr] * D; with `out` == nullptr the
 // result (weights not normalised) goes back to `own` row rr instead.
 template <int D, int KS>
-__device__ __noinline__ void merge_pass(float *own, const float *recv, const float *wts, int n_src, int rpp, int p0,
-                                        int p1, int row0, const AttnArgs &a, int b, int g,
-                                        __nv_bfloat16 *out) {
+__device__ __forceinline__ void merge_pass(float *own, const float *recv, const float *wts, const unsigned *orow,
+                                           int n_src, int rpp, int p0, int p1, __nv_bfloat16 *out) {
     constexpr int PS = D + 4;
-    constexpr int RG = 4;                     // rows per warp step
+    constexpr int RG = 8;                     // rows per warp step
     const int lane = threadIdx.x & 31;
     const int c = lane * 4;
     if (c >= D) return;
     const int n_warps = blockDim.x >> 5;
-    const int G = a.G;
     for (int r0 = p0 + (int)(threadIdx.x >> 5) * RG; r0 < p1; r0 += n_warps * RG) {
         const int nr = min(RG, p1 - r0);
         float4 acc[RG];
@@ -178,16 +178,12 @@ __device__ __noinline__ void merge_pass(float *own, const float *recv, const flo
             const int rr = r0 + k;
             if (out == nullptr) {
                 *reinterpret_cast<float4 *>(own + rr * PS + c) = acc[k];
-                continue;
+            } else {
+                uint2 w2;
+                w2.x = pack_bf16x2(acc[k].x, acc[k].y);
+                w2.y = pack_bf16x2(acc[k].z, acc[k].w);
+                *reinterpret_cast<uint2 *>(out + (size_t)orow[rr] * D + c) = w2;
             }
-            // tile row R = node * G + head-in-group
-            const int R = row0 + rr;
-            const int i = R / G;
-            const int h = g * G + (R - i * G);
-            uint2 w2;
-            w2.x = pack_bf16x2(acc[k].x, acc[k].y);
-            w2.y = pack_bf16x2(acc[k].z, acc[k].w);
-            *reinterpret_cast<uint2 *>(out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c) = w2;
         }
     }
 }
@@ -199,31 +195,32 @@ __device__ __noinline__ void merge_pass(float *own, const float *recv, const flo
 // sum_s 2^(m_s - M) l_s when `normalise`; otherwise the combined row's M and
 // sum go to w[rr][kMaxSrc - 2] and w[rr][kMaxSrc - 1].
 template <int D, int KS>
-__device__ __noinline__ void row_weights(const float *own, const float *recv, int rpp, int p0, int p1, int n_src,
-                                         float *wts, bool normalise) {
+__device__ __forceinline__ void row_weights(const float *own, const float *recv, int rpp, int p0, int p1, int n_src,
+                                            float *wts, bool normalise) {
     constexpr int PS = D + 4;
     const int rr = p0 + (int)threadIdx.x;
     if (rr >= p1) return;
-    auto ml = [&](int sidx) {
+    float2 v[kMaxSrc];
+#pragma unroll
+    for (int sidx = 0; sidx < kMaxSrc; ++sidx) {
         const float *row = sidx < KS ? own + (rr + 64 * sidx) * PS : recv + ((sidx - KS) * rpp + rr - p0) * PS;
-        return *reinterpret_cast<const float2 *>(row + D);
-    };
-    float M = -INFINITY;
-#pragma unroll 1
-    for (int sidx = 0; sidx < n_src; ++sidx) M = fmaxf(M, ml(sidx).x);
-    float lsum = 0.f;
-#pragma unroll 1
-    for (int sidx = 0; sidx < n_src; ++sidx) {
-        const float2 v = ml(sidx);
-        const float w = (v.x == -INFINITY) ? 0.f : ex2_approx(v.x - M);
-        wts[rr * kMaxSrc + sidx] = w;
-        lsum = fmaf(w, v.y, lsum);
+        v[sidx] = sidx < n_src ? *reinterpret_cast<const float2 *>(row + D) : make_float2(-INFINITY, 0.f);
     }
-    if (normalise) {
-        const float inv = lsum > 0.f ? rcp_approx(lsum) : 0.f;
-#pragma unroll 1
-        for (int sidx = 0; sidx < n_src; ++sidx) wts[rr * kMaxSrc + sidx] *= inv;
-    } else {
+    float M = v[0].x;
+#pragma unroll
+    for (int sidx = 1; sidx < kMaxSrc; ++sidx) M = fmaxf(M, v[sidx].x);
+    float w[kMaxSrc];
+    float lsum = 0.f;
+#pragma unroll
+    for (int sidx = 0; sidx < kMaxSrc; ++sidx) {
+        w[sidx] = (v[sidx].x == -INFINITY) ? 0.f : ex2_approx(v[sidx].x - M);
+        lsum = fmaf(w[sidx], v[sidx].y, lsum);
+    }
+    const float inv = normalise ? (lsum > 0.f ? rcp_approx(lsum) : 0.f) : 1.f;
+#pragma unroll
+    for (int sidx = 0; sidx < kMaxSrc; ++sidx)
+        if (sidx < n_src) wts[rr * kMaxSrc + sidx] = w[sidx] * inv;
+    if (!normalise) {
         wts[rr * kMaxSrc + kMaxSrc - 2] = M;
         wts[rr * kMaxSrc + kMaxSrc - 1] = lsum;
     }
@@ -258,6 +255,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t *mma_done = o_full + 2;
     uint64_t *q_full = mma_done + 1;          // the four lane quadrants hold their Q rows in TMEM
     uint64_t *g_full = q_full + 1;            // the merging CTA: a pass of the other splits' partials is here
+    uint64_t *anc_full = g_full + 1;          // the tree CTA: the ancestor masks are in shared memory
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(sm + S::misc_off);
     volatile int *s_abort = reinterpret_cast<volatile int *>(sm + S::misc_off + 4);
     bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 8);
@@ -265,11 +263,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     int *s_pages = reinterpret_cast<int *>(sm + S::pages_off);
     float *s_wts = reinterpret_cast<float *>(sm + S::wts_off);
     int *s_par = reinterpret_cast<int *>(sm + S::par_off);
+    unsigned *s_orow = reinterpret_cast<unsigned *>(sm + S::orow_off);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    // grid (row tiles, split, sequence x KV head) with a group's tree split
+    // (the merging one, which has the most work) at y = 0: CTAs are placed in
+    // block order, so when SMs free up one by one it starts first in its group
     const int rt = blockIdx.x;
-    const int split = blockIdx.y;
+    const int split = a.n_split - 1 - (int)blockIdx.y;
     const int bg = blockIdx.z;
     const int b = bg / a.Hkv;
     const int g = bg % a.Hkv;
@@ -304,6 +306,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(mma_done, 1);
         mbar_init(q_full, 4);
         mbar_init(g_full, 1);
+        mbar_init(anc_full, 1);
         *s_abort = 0;
         *s_bad = false;
         fence_barrier_init();
@@ -374,9 +377,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int kend = min(L, kbeg + chunk);
     const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
     const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
-    // The tree CTA takes its tree tile first, so that the one CTA with an
-    // extra tile does not end on a load whose latency nothing hides.  The
-    // order is the same in every launch mode, and with it the result.
+    // The tree CTA takes its tree tile first, in every launch mode (so that
+    // the result does not depend on the mode): the one CTA with an extra tile
+    // then does not end on a load whose latency nothing hides.  With
+    // cache_early the free ring stages after stage 0 fill with cache tiles
+    // before k_new/v_new may be read.
     const bool split_wait = c_early && !in_early;
     const int tree_j = tree_cta ? 0 : -1;
     const int tree_shift = tree_cta ? 1 : 0;   // tile j is cache tile j - tree_shift
@@ -487,8 +492,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (producer) issue_first(prod_v, prod_v ? v_issued : k_issued, phase);
     }
-    // the tree CTA's ancestor masks (warp 3 has no other setup work)
-    if (warp == 3 && tree_cta) tree_masks_walk(parents, a.T, s_par, s_anc, s_bad);
 
     tc_fence_before();
     __syncthreads();
@@ -506,6 +509,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(q_full);
+    }
+    // The tree CTA's ancestor masks, built by warp 3 while the first tiles
+    // are still on their way (they are needed by the tree tile's step only).
+    if (warp == 3 && tree_cta) {
+        tree_masks_walk(parents, a.T, s_par, s_anc, s_bad);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(anc_full);
     }
 
     // ----------------------------------------------------- TMA producer warps
@@ -625,6 +635,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
             const bool tree_tile = j == tree_j;
+            if (tree_tile) {
+                const bool got_anc = __all_sync(0xffffffffu, mbar_wait(anc_full, 0, kWaitNs));
+                if (!got_anc) {
+                    *s_abort = 1;
+                    break;
+                }
+            }
             const int key0 = kbeg + (j - tree_shift) * BN;
             const int n_valid = tree_tile ? a.T : min(BN, kend - key0);
             // Keys of a 64-key block of the tile that this row sees: a prefix
@@ -822,7 +839,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (KS == 2) {
             row_weights<D, KS>(part_o, nullptr, 0, 0, rows_here, KS, s_wts, false);
             __syncthreads();
-            merge_pass<D, KS>(part_o, nullptr, s_wts, KS, 0, 0, rows_here, rt * BM, a, b, g, nullptr);
+            merge_pass<D, KS>(part_o, nullptr, s_wts, nullptr, KS, 0, 0, rows_here, nullptr);
             if (threadIdx.x < rows_here)
                 *reinterpret_cast<float2 *>(part_o + threadIdx.x * S::po_stride + D) =
                     make_float2(s_wts[threadIdx.x * kMaxSrc + kMaxSrc - 2], s_wts[threadIdx.x * kMaxSrc + kMaxSrc - 1]);
@@ -852,6 +869,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         __syncthreads();
+        // output row (node i, query head h) of tile row rr: (b T + i) Hq + h
+        if ((int)threadIdx.x < rows_here) {
+            const int R = rt * BM + (int)threadIdx.x;
+            const int i = R / a.G;
+            s_orow[threadIdx.x] = (unsigned)(((size_t)b * a.T + i) * a.Hq + g * a.G + (R - i * a.G));
+        }
         if (!*s_abort) {
             float *recv = reinterpret_cast<float *>(sK + S::own_bytes);
             const int rpp = others > 0 ? min(rows_here, S::recv_bytes / (others * (int)row_bytes)) : rows_here;
@@ -869,7 +892,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (got) row_weights<D, KS>(part_o, recv, rpp, p0, p1, n_src, s_wts, true);
                 else *s_abort = 1;
                 __syncthreads();   // the weights are in shared memory
-                if (!*s_abort) merge_pass<D, KS>(part_o, recv, s_wts, n_src, rpp, p0, p1, rt * BM, a, b, g, out);
+                if (!*s_abort) merge_pass<D, KS>(part_o, recv, s_wts, s_orow, n_src, rpp, p0, p1, out);
                 // the received rows are read before the next pass overwrites them
                 __syncthreads();
                 if (*s_abort) break;
