@@ -275,7 +275,8 @@ def run_gpu_arm(args, world, rank, local, dist):
         Lcap = page_sets(w, sets, args.page_size, Lcap)
     step = pkg.VerifyStep(w.B, w.T, w.Hq, w.Hkv, w.D, Lcap, w.V, w.torch_dtype, device=device,
                           accept=args.accept, temperature=args.temperature, epsilon=args.epsilon,
-                          delta=args.delta, schedule=args.schedule, page_size=args.page_size or None)
+                          delta=args.delta, schedule=args.schedule, page_size=args.page_size or None,
+                          attn_launch="ordinary" if args.page_size else args.attn_launch)
     stream = torch.cuda.Stream(device)
 
     def launch(s):
@@ -344,11 +345,14 @@ def run_gpu_arm(args, world, rank, local, dist):
     # replays.  The accept and commit calls: each launched alone after an L2
     # flush by a large read (which keeps the GPU busy while the call is queued,
     # so the events bracket the kernel and not the host's launch latency).
-    timing_source = {"tree_attn": f"back-to-back attention launches over the {n_sets} rotating input sets in one "
-                                  "CUDA graph, events around the replays, after the timed region",
+    timing_source = {"tree_attn": f"back-to-back attention launches ({step.attn_launch} launch) over the {n_sets} "
+                                  "rotating input sets, four passes in one CUDA graph, events around the replays, "
+                                  "after the timed region",
                      "accept": "launched alone after an L2 flush, events on the launching stream",
                      "kv_commit": "launched alone after an L2 flush, events on the launching stream"}
-    us = {"tree_attn": attn_launch_us(step, sets, stream, device, args)}
+    us = {"tree_attn": attn_launch_us(step, sets, stream, device, args, mode=step.attn_launch)}
+    us["tree_attn_ordinary"] = (us["tree_attn"] if step.attn_launch == "ordinary"
+                                else attn_launch_us(step, sets, stream, device, args, mode="ordinary"))
     flush = torch.zeros(2 * L2_BYTES, dtype=torch.uint8, device=device)
     us["accept"] = accept_kernel_us(pkg, w, sets, stream, device, args.accept, args, flush)
     other = "greedy" if args.accept == "typical" else "typical"
@@ -391,11 +395,15 @@ def run_gpu_arm(args, world, rank, local, dist):
                    "l2": f"{n_sets} rotating input sets of {per_set / 1e6:.1f} MB "
                          f"({n_sets * per_set / 1e6:.0f} MB > 3x the 129 MB L2)",
                    "launch": LAUNCH_DESC[args.schedule],
+                   "attn_launch": step.attn_launch,
                    "accept": accept_desc(args)},
         "roofline": {"bound": "hbm", "kernel": "tree_attn", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm, "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)"
                      if peak_kind == "measured" else "fallback 6.8 TB/s",
                      "traffic": traffic, "bytes_per_launch": a_bytes, "launch_us": us["tree_attn"],
+                     "attn_launch": step.attn_launch,
+                     "launch_us_ordinary": us["tree_attn_ordinary"],
+                     "frac_ordinary": a_bytes / (us["tree_attn_ordinary"] * 1e-6) / 1e9 / hbm,
                      "frac_of_8TBs": achieved / 8000.0,
                      "flops_per_launch": attn_flops_per_launch(w, lengths),
                      "timing": timing_source["tree_attn"]},
@@ -436,11 +444,13 @@ def accept_desc(args) -> str:
     return "greedy"
 
 
-def attn_launch_us(step, sets, stream, device, args, launches: int = 200) -> float:
+def attn_launch_us(step, sets, stream, device, args, mode: str, launches: int = 200, passes: int = 4) -> float:
     """Mean duration of the step's attention call over back-to-back launches
-    on the rotating input sets: one CUDA graph of one launch per set, replayed
-    until about ``launches`` launches, CUDA events around the replays."""
+    on the rotating input sets, launched as ``mode`` (VerifyStep.ATTN_LAUNCHES):
+    one CUDA graph of ``passes`` launches per set, replayed until about
+    ``launches`` launches, CUDA events around the replays."""
     import paper_2405_00263_gb300 as pkg
+    kw = pkg.VerifyStep.ATTN_LAUNCHES[mode]
 
     def attn(s):
         if args.page_size:
@@ -450,13 +460,14 @@ def attn_launch_us(step, sets, stream, device, args, launches: int = 200) -> flo
         else:
             pkg.clover_verify_attn(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"],
                                    s["parent"], step.out, workspace=step.ws_attn, status=step.status,
-                                   stream=stream, append=args.schedule == "compact")
+                                   stream=stream, append=args.schedule == "compact", **kw)
 
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=stream):
-        for s in sets:
-            attn(s)
-    reps = max(3, launches // len(sets))
+        for _ in range(passes):
+            for s in sets:
+                attn(s)
+    reps = max(3, launches // (passes * len(sets)))
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         for _ in range(3):
@@ -468,7 +479,7 @@ def attn_launch_us(step, sets, stream, device, args, launches: int = 200) -> flo
     b.synchronize()
     if step.device_status() != 0:
         raise RuntimeError(f"device status {step.device_status()} in the attention timing")
-    return a.elapsed_time(b) * 1e3 / (reps * len(sets))
+    return a.elapsed_time(b) * 1e3 / (reps * passes * len(sets))
 
 
 def isolated_us(call, n, stream, flush) -> float:
@@ -955,6 +966,11 @@ def main(argv=None):
                     help="run on a paged KV cache with pages of this many slots (0: dense cache)")
     ap.add_argument("--schedule", default="commit", choices=["commit", "compact", "fused"],
                     help="call schedule of the step (VerifyStep)")
+    ap.add_argument("--attn-launch", default="inputs_ready", choices=["ordinary", "pdl", "cache_ready", "inputs_ready"],
+                    help="attention launch: ordinary, or a programmatic dependent of the kernel before it, with the "
+                         "statement that the caches (cache_ready) or all inputs (inputs_ready) are not being written "
+                         "by the kernels that may still run -- true here: consecutive steps serve independent input "
+                         "sets, as independent batches do (dense cache; a paged cache launches the ordinary way)")
     ap.add_argument("--temperature", type=float, default=1.0)
     ap.add_argument("--epsilon", type=float, default=0.09)
     ap.add_argument("--delta", type=float, default=0.3)

@@ -489,16 +489,29 @@ class VerifyStep:
     ``src_index`` holds tree nodes (commit) or cache slots (compact).
     ``accept``: ``"greedy"`` (clover_verify_accept) or ``"typical"``
     (clover_verify_accept_typical with ``temperature``, ``epsilon``, ``delta``).
+    ``attn_launch``: how the attention is launched (clover_verify_attn_ex
+    flags): ``"ordinary"``; ``"pdl"`` (CLOVER_ATTN_PDL); ``"cache_ready"``
+    (with CLOVER_ATTN_CACHE_READY) or ``"inputs_ready"`` (with
+    CLOVER_ATTN_INPUTS_READY): the caller's statement that the kernels
+    queued before a step do not write its inputs, as when consecutive steps
+    serve independent batches (dense cache only).
     ``page_size``: a paged cache (commit schedule only): ``run`` then takes the
     page pools as k_cache/v_cache and the ``block_table``, and calls
     clover_verify_attn_paged and clover_kv_commit_paged; ``Lcap`` is the
     capacity page_size * max_pages.
     """
 
+    ATTN_LAUNCHES = {"ordinary": {}, "pdl": dict(pdl=True), "cache_ready": dict(pdl=True, cache_ready=True),
+                     "inputs_ready": dict(pdl=True, inputs_ready=True)}
+
     def __init__(self, B, T, Hq, Hkv, D, Lcap, V, dtype, device="cuda", concurrent=True, schedule="commit",
-                 accept="greedy", temperature=1.0, epsilon=0.09, delta=0.3, page_size=None):
+                 accept="greedy", temperature=1.0, epsilon=0.09, delta=0.3, page_size=None, attn_launch="ordinary"):
         if schedule not in ("commit", "compact", "fused"):
             raise ValueError(f"unknown schedule {schedule!r}")
+        if attn_launch not in self.ATTN_LAUNCHES:
+            raise ValueError(f"unknown attention launch {attn_launch!r}")
+        self.attn_launch = attn_launch
+        self._attn_kw = self.ATTN_LAUNCHES[attn_launch]
         if page_size is not None and (schedule != "commit" or Lcap % page_size):
             raise ValueError("a paged cache takes the commit schedule and a capacity of whole pages")
         self.page_size = page_size
@@ -527,7 +540,10 @@ class VerifyStep:
         # the side stream's calls get their own status word so that concurrent
         # calls never update one word at the same time from two streams
         self.status_accept = torch.zeros((1,), **i32)
-        self.side = torch.cuda.Stream(device=dev) if concurrent else None
+        # the side stream (argmax/accept, commit) at the highest priority: its
+        # CTAs are placed ahead of the attention's when both wait for SM space
+        lo, hi = torch.cuda.Stream.priority_range() if hasattr(torch.cuda.Stream, "priority_range") else (0, -1)
+        self.side = torch.cuda.Stream(device=dev, priority=min(lo, hi)) if concurrent else None
         self._fork = torch.cuda.Event() if concurrent else None
         self._join = torch.cuda.Event() if concurrent else None
 
@@ -556,7 +572,8 @@ class VerifyStep:
         if self.schedule == "fused":
             ev(0, stream)
             clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
-                               workspace=self.ws_attn, status=self.status, stream=stream, append=False)
+                               workspace=self.ws_attn, status=self.status, stream=stream, append=False,
+                               **self._attn_kw)
             timed_end = n_ev > 1 and self.side is not None
             if timed_end:
                 # the attention's end, recorded on the side stream: nothing is
@@ -585,7 +602,8 @@ class VerifyStep:
                                      scale=scale, workspace=self.ws_attn, status=self.status, stream=stream)
         else:
             clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
-                               workspace=self.ws_attn, status=self.status, stream=stream, append=not commit)
+                               workspace=self.ws_attn, status=self.status, stream=stream, append=not commit,
+                               **self._attn_kw)
         ev(1, stream)
         ev(4, side)
         if self.accept == "typical":

@@ -226,8 +226,11 @@ __device__ __forceinline__ void row_weights(const float *own, const float *recv,
     }
 }
 
+// At most 160 registers a thread (35,840 for the CTA): two 56-register CTAs
+// of the accept kernel (28,672) still fit beside it on an SM, so that the
+// argmax running beside the attention is not held back to one CTA an SM.
 template <int D, int KS, bool PAGED>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(160)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                         const __grid_constant__ CUtensorMap tm_kn, const __grid_constant__ CUtensorMap tm_vn,
                         const __grid_constant__ CUtensorMap tm_ks,

@@ -285,6 +285,28 @@ def test_pdl_inputs_ready_independent_calls(graph, cuda):
     assert torch.equal(shared.view(torch.int16), ref[5].view(torch.int16))
 
 
+@pytest.mark.parametrize("mode", ["pdl", "cache_ready", "inputs_ready"])
+@pytest.mark.parametrize("schedule", ["commit", "fused"])
+def test_step_attention_launch_modes(mode, schedule, cuda):
+    """VerifyStep with the attention launched as a programmatic dependent:
+    three steps in a row on independent input sets (the statement holds), each
+    bit-equal to an ordinary step's outputs and matching the oracle."""
+    hosts = [workloads.make(workloads.get("7b_l2048", T=64, Hq=8, Hkv=8, L=1100 + 300 * i, V=3000, seed=40 + i))
+             for i in range(3)]
+    ref = [run_gpu(to_dev(h, cuda), schedule=schedule) for h in hosts]
+    ref_out = [r.out.clone() for r in ref]
+    sets = [to_dev(h, cuda) for h in hosts]
+    B, T, Hq, D = sets[0]["q"].shape
+    step = pkg.VerifyStep(B, T, Hq, 8, D, max(s["Lcap"] for s in sets), 3000, torch.bfloat16, device=cuda,
+                          schedule=schedule, attn_launch=mode)
+    for i, t in enumerate(sets):
+        step.run(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
+                 t["cand"], t["logits"])
+        torch.cuda.synchronize()
+        assert torch.equal(step.out.view(torch.int16), ref_out[i].view(torch.int16)), i
+        compare_full(hosts[i], step, t)
+
+
 # ---------------------------------------------------------------------------
 # the two schedules of a step
 # ---------------------------------------------------------------------------
