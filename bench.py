@@ -45,6 +45,7 @@ UNIT = "verify steps/s"
 DEFAULT_WORKLOAD = "7b_l4096"
 L2_BYTES = 129 * 1000 * 1000
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
 KERNEL_SOURCES = {
     "tree_attn": ["tree_attn_tc.cu", "tc_ptx.cuh", "tmap_host.cuh", "common.cuh", "abi.cu"],
     "accept": ["accept.cu", "common.cuh"],
@@ -375,8 +376,14 @@ def run_gpu_arm(args, world, rank, local, dist):
 
     peaks, peak_kind = measured_peaks()
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    tc_peak = float(peaks.get("bf16_tflops", FALLBACK_BF16_TFLOPS))
     a_bytes = attn_bytes_per_launch(w, lengths)
+    a_flops = attn_flops_per_launch(w, lengths)
     achieved = a_bytes / (us["tree_attn"] * 1e-6) / 1e9
+    tflops = a_flops / (us["tree_attn"] * 1e-6) / 1e12
+    # the bound of this shape: HBM when its bytes take longer at the measured
+    # copy rate than its flops at the measured bf16 rate, else the tensor pipe
+    tensor_bound = a_flops / (tc_peak * 1e12) > a_bytes / (hbm * 1e9)
     traffic = recorded_traffic("tree_attn", w.name + (f"_paged{args.page_size}" if args.page_size else ""))
     am_bytes = argmax_bytes_per_launch(w)
 
@@ -397,9 +404,16 @@ def run_gpu_arm(args, world, rank, local, dist):
                    "launch": LAUNCH_DESC[args.schedule],
                    "attn_launch": step.attn_launch,
                    "accept": accept_desc(args)},
-        "roofline": {"bound": "hbm", "kernel": "tree_attn", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm, "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)"
-                     if peak_kind == "measured" else "fallback 6.8 TB/s",
+        "roofline": {"bound": "tensor" if tensor_bound else "hbm", "kernel": "tree_attn",
+                     "achieved": tflops if tensor_bound else achieved, "peak": tc_peak if tensor_bound else hbm,
+                     "unit": "TFLOP/s" if tensor_bound else "GB/s",
+                     "frac": tflops / tc_peak if tensor_bound else achieved / hbm,
+                     "peak_source": (f"{peak_kind} " + ("bf16_tflops (burst: the kernel is timed alone)"
+                                                        if tensor_bound else "hbm_gbs") + " (MEASURED_PEAKS.json)")
+                     if peak_kind == "measured" else ("fallback 1.9 PFLOP/s bf16" if tensor_bound
+                                                      else "fallback 6.8 TB/s"),
+                     "hbm_gbs": achieved, "frac_hbm": achieved / hbm, "tflops": tflops,
+                     "frac_tensor": tflops / tc_peak,
                      "traffic": traffic, "bytes_per_launch": a_bytes, "launch_us": us["tree_attn"],
                      "attn_launch": step.attn_launch,
                      "launch_us_ordinary": us["tree_attn_ordinary"],
@@ -971,6 +985,9 @@ def main(argv=None):
                          "statement that the caches (cache_ready) or all inputs (inputs_ready) are not being written "
                          "by the kernels that may still run -- true here: consecutive steps serve independent input "
                          "sets, as independent batches do (dense cache; a paged cache launches the ordinary way)")
+    ap.add_argument("--workloads", default="",
+                    help="comma-separated workloads: one JSON line each (stdout, and --record FILE if given)")
+    ap.add_argument("--record", default="", help="file that --workloads appends its JSON lines to")
     ap.add_argument("--temperature", type=float, default=1.0)
     ap.add_argument("--epsilon", type=float, default=0.09)
     ap.add_argument("--delta", type=float, default=0.3)
@@ -994,14 +1011,21 @@ def main(argv=None):
         if dist is not None:
             dist.destroy_process_group()
         return 0
-    line, w, base = run_gpu_arm(args, world, rank, local, dist)
-    if rank == 0:
-        if world == 1 and not args.no_cpu_baseline:
-            host = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
-            line["cpu_baseline"] = cpu_baseline(w, host, args)
-        else:
-            line["cpu_baseline"] = None
-        print(json.dumps(line), flush=True)
+    for name in (args.workloads.split(",") if args.workloads else [args.workload]):
+        args.workload = name
+        line, w, base = run_gpu_arm(args, world, rank, local, dist)
+        if rank == 0:
+            if world == 1 and not args.no_cpu_baseline:
+                host = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
+                line["cpu_baseline"] = cpu_baseline(w, host, args)
+            else:
+                line["cpu_baseline"] = None
+            print(json.dumps(line), flush=True)
+            if args.record:
+                with open(args.record, "a") as f:
+                    f.write(json.dumps(line) + "\n")
+        del base
+        torch.cuda.empty_cache()
     if dist is not None:
         dist.destroy_process_group()
     return 0

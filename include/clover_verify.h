@@ -80,8 +80,21 @@ typedef enum {
     CLOVER_ERR_CAPACITY = 8,     /* device: cache_len[b] < 0 or cache_len[b] + T > Lcap */
     CLOVER_ERR_CUDA = 16,        /* a CUDA launch or query failed */
     CLOVER_ERR_TIMEOUT = 32,     /* device: a bounded wait gave up (see below) */
-    CLOVER_ERR_SCRATCH_LIMIT = 64 /* clover_verify_attn_noalloc: scratch need exceeds its static buffer */
+    CLOVER_ERR_SCRATCH_LIMIT = 64, /* clover_verify_attn_noalloc: scratch need exceeds its static buffer */
+    CLOVER_ERR_CHECK = 128       /* device, CLOVER_CHECKED builds only: an index check failed (see below) */
 } clover_status;
+
+/*
+ * CLOVER_ERR_CHECK: a library built with -DCLOVER_CHECKED checks, on the
+ * device, the indices its kernels compute before the global accesses they
+ * guard: query rows and key ranges of the attention against B*T and the
+ * sequence's key count, output rows against B*T, split-KV workspace slots and
+ * arrival counters against ws_bytes, committed and compacted cache slots
+ * against Lcap, and the source nodes of a commit against T.  A failed check
+ * sets this bit and skips the access; it never traps.  Ordinary builds
+ * compile the checks out and never set it; clover_build_flags() tells the two
+ * apart.
+ */
 
 /*
  * CLOVER_ERR_TIMEOUT is raised by the kernels that wait on barriers: the bf16
@@ -99,6 +112,11 @@ typedef enum {
 
 /* Version of this ABI (incremented on any incompatible change). */
 CLOVER_API int clover_abi_version(void);
+
+/* Build options of the loaded library: CLOVER_BUILD_CHECKED when it was
+ * compiled with -DCLOVER_CHECKED (device index checks, CLOVER_ERR_CHECK). */
+#define CLOVER_BUILD_CHECKED 1
+CLOVER_API int clover_build_flags(void);
 
 /* Short English name of a status code (static storage). */
 CLOVER_API const char *clover_status_string(int status);

@@ -6,7 +6,8 @@ same names.  There is no CPU fallback.
 """
 
 from .api import (  # noqa: F401
-    BF16, F32, OK, CloverError, DraftHead, VerifyStep, clover_abi_version, clover_embed_rows, clover_linear,
+    BF16, F32, OK, CloverError, DraftHead, VerifyStep, clover_abi_version, clover_build_flags, clover_embed_rows,
+    clover_linear,
     clover_linear_workspace_size,
     clover_topk, clover_topk_workspace_size, clover_kv_commit, clover_kv_commit_paged,
     clover_kv_compact, clover_verify_attn_paged, clover_verify_attn_paged_workspace_size,

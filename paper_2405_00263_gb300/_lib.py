@@ -19,6 +19,7 @@ _lib = None
 # Every symbol include/clover_verify.h declares.
 EXPORTS = (
     "clover_abi_version",
+    "clover_build_flags",
     "clover_status_string",
     "clover_verify_attn_workspace_size",
     "clover_verify_attn",
@@ -64,8 +65,15 @@ LINEAR_RES = 3
 NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
+# Bit of clover_build_flags(): the library was built with -DCLOVER_CHECKED.
+BUILD_CHECKED = 1
+
+# Set to 1 to load the checked build (``build(checked=True)``) instead.
+CHECKED_ENV = "CLOVER_VERIFY_CHECKED"
+
+
 def library_path() -> str:
-    return _build.LIB
+    return _build.CHECKED_LIB if os.environ.get(CHECKED_ENV) == "1" else _build.LIB
 
 
 def load(build_if_missing: bool = False):
@@ -80,11 +88,13 @@ def load(build_if_missing: bool = False):
                 raise RuntimeError(
                     f"libclover_verify.so is not built ({path}); run "
                     "`python -c 'import __graft_entry__ as g; g.build()'` first")
-            _build.build()
+            _build.build(checked=path == _build.CHECKED_LIB)
         lib = ctypes.CDLL(path)
         P, I, Z, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
         lib.clover_abi_version.argtypes = []
         lib.clover_abi_version.restype = I
+        lib.clover_build_flags.argtypes = []
+        lib.clover_build_flags.restype = I
         lib.clover_status_string.argtypes = [I]
         lib.clover_status_string.restype = ctypes.c_char_p
         lib.clover_verify_attn_workspace_size.argtypes = [I, I, I, I, I, I, I]

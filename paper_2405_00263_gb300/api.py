@@ -22,6 +22,7 @@ ERR_CAPACITY = 8
 ERR_CUDA = 16
 ERR_TIMEOUT = 32
 ERR_SCRATCH_LIMIT = 64
+ERR_CHECK = 128
 
 F32 = 0
 BF16 = 1
@@ -77,6 +78,11 @@ def _check(t, shape, dtype, name):
 
 def clover_abi_version() -> int:
     return _lib.load().clover_abi_version()
+
+
+def clover_build_flags() -> int:
+    """Build options of the loaded library (bit 1: device index checks)."""
+    return _lib.load().clover_build_flags()
 
 
 def clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, Lcap, dtype) -> int:

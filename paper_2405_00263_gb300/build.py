@@ -2,9 +2,11 @@
 
 Each .cu under csrc/ compiles to an object in parallel; the objects link into
 ``_build/libclover_verify.so``.  Objects are rebuilt when their source, any
-header, or the flags change.
+header, or the flags change.  ``checked=True`` builds the same library with
+``-DCLOVER_CHECKED`` (device-side index checks that raise CLOVER_ERR_CHECK in
+the status word) into ``_build/checked/``.
 
-    python -m paper_2405_00263_gb300.build [--verbose-ptxas]
+    python -m paper_2405_00263_gb300.build [--verbose-ptxas] [--checked]
 """
 
 from __future__ import annotations
@@ -23,6 +25,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT, "libclover_verify.so")
+CHECKED_OUT = os.path.join(OUT, "checked")
+CHECKED_LIB = os.path.join(CHECKED_OUT, "libclover_verify.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
@@ -45,19 +49,20 @@ def _stamp(extra: list[str]) -> str:
     return h.hexdigest()
 
 
-def build(verbose_ptxas: bool = False, force: bool = False) -> str:
-    os.makedirs(OUT, exist_ok=True)
-    extra = ["-Xptxas", "-v"] if verbose_ptxas else []
-    stamp_file = os.path.join(OUT, "stamp")
+def build(verbose_ptxas: bool = False, force: bool = False, checked: bool = False) -> str:
+    out_dir, lib = (CHECKED_OUT, CHECKED_LIB) if checked else (OUT, LIB)
+    os.makedirs(out_dir, exist_ok=True)
+    extra = (["-Xptxas", "-v"] if verbose_ptxas else []) + (["-DCLOVER_CHECKED"] if checked else [])
+    stamp_file = os.path.join(out_dir, "stamp")
     stamp = _stamp(extra)
-    if not force and os.path.exists(LIB) and os.path.exists(stamp_file):
+    if not force and os.path.exists(lib) and os.path.exists(stamp_file):
         if open(stamp_file).read() == stamp:
-            return LIB
+            return lib
     exe = nvcc()
     sources = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
 
     def compile_one(src: str) -> str:
-        obj = os.path.join(OUT, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(out_dir, os.path.basename(src)[:-3] + ".o")
         cmd = [exe, *ARCH, *FLAGS, *extra, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -68,15 +73,16 @@ def build(verbose_ptxas: bool = False, force: bool = False) -> str:
 
     with ThreadPoolExecutor(max_workers=min(8, len(sources))) as pool:
         objs = list(pool.map(compile_one, sources))
-    tmp = LIB + f".tmp{os.getpid()}"
-    r = subprocess.run([exe, *ARCH, "-shared", "-o", tmp, *objs, "-lcudart"], capture_output=True, text=True)
+    tmp = lib + f".tmp{os.getpid()}"
+    r = subprocess.run([exe, *ARCH, "-shared", "-o", tmp, *objs, "-lcudart", "-ldl"], capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
+    os.replace(tmp, lib)
     with open(stamp_file, "w") as f:
         f.write(stamp)
-    return LIB
+    return lib
 
 
 if __name__ == "__main__":
-    print(build(verbose_ptxas="--verbose-ptxas" in sys.argv, force="--force" in sys.argv))
+    print(build(verbose_ptxas="--verbose-ptxas" in sys.argv, force="--force" in sys.argv,
+                checked="--checked" in sys.argv))

@@ -5,6 +5,8 @@
 
 #include <mutex>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "common.cuh"
 
 namespace clover {
@@ -122,6 +124,16 @@ AttnPlan plan_attn(int B, int T, int Hq, int Hkv, int D, int Lcap, int dtype) {
 }
 
 clover_status from_cuda(cudaError_t e) { return e == cudaSuccess ? CLOVER_OK : CLOVER_ERR_CUDA; }
+
+// An NVTX range (named after the entry point) around each call, so that a
+// profiler's timeline shows the library's host-side calls; without a tool
+// attached it costs a few nanoseconds.
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange &) = delete;
+    NvtxRange &operator=(const NvtxRange &) = delete;
+};
 
 }  // namespace
 }  // namespace clover
@@ -262,6 +274,7 @@ clover_status run_attn(const void *q, const void *k_new, const void *v_new, void
     a.part_o = p.total ? reinterpret_cast<float *>(ws + p.counter_bytes) : nullptr;
     a.part_ml = p.total && p.ml_bytes ? reinterpret_cast<float *>(ws + p.counter_bytes + p.o_bytes) : nullptr;
     a.status = status;
+    a.ws_bytes = workspace ? ws_bytes : 0;
     // the launch options apply to the tensor-core kernel; the FMA kernel is
     // launched the ordinary way (stream order) whatever they say
     a.pdl = (launch_flags & CLOVER_ATTN_PDL) ? 1 : 0;
@@ -277,6 +290,14 @@ extern "C" {
 
 int clover_abi_version(void) { return kAbiVersion; }
 
+int clover_build_flags(void) {
+#ifdef CLOVER_CHECKED
+    return CLOVER_BUILD_CHECKED;
+#else
+    return 0;
+#endif
+}
+
 const char *clover_status_string(int status) {
     switch (status) {
         case CLOVER_OK: return "ok";
@@ -287,6 +308,7 @@ const char *clover_status_string(int status) {
         case CLOVER_ERR_CUDA: return "CUDA error";
         case CLOVER_ERR_TIMEOUT: return "device wait timed out";
         case CLOVER_ERR_SCRATCH_LIMIT: return "scratch need exceeds the static buffer of clover_verify_attn_noalloc";
+        case CLOVER_ERR_CHECK: return "a device index check failed (CLOVER_CHECKED build)";
         default: return "several errors (bitwise OR of codes)";
     }
 }
@@ -301,6 +323,7 @@ clover_status clover_verify_attn(const void *q, const void *k_new, const void *v
                                  int B, int T, int Hq, int Hkv, int D, int Lcap, clover_dtype dtype,
                                  float scale, void *workspace, size_t ws_bytes, int32_t *status,
                                  void *stream) {
+    const NvtxRange nvtx_range("clover_verify_attn");
     return clover_verify_attn_ex(q, k_new, v_new, k_cache, v_cache, cache_len, parent, out, B, T, Hq, Hkv, D,
                                  Lcap, dtype, scale, workspace, ws_bytes, status, stream, 0u);
 }
@@ -310,6 +333,7 @@ clover_status clover_verify_attn_ex(const void *q, const void *k_new, const void
                                     int B, int T, int Hq, int Hkv, int D, int Lcap, clover_dtype dtype,
                                     float scale, void *workspace, size_t ws_bytes, int32_t *status,
                                     void *stream, uint32_t flags) {
+    const NvtxRange nvtx_range("clover_verify_attn_ex");
     if (flags & ~(CLOVER_ATTN_NO_APPEND | CLOVER_ATTN_PDL | CLOVER_ATTN_CACHE_READY | CLOVER_ATTN_INPUTS_READY))
         return CLOVER_ERR_INVALID_ARG;
     const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype);
@@ -332,6 +356,7 @@ clover_status clover_verify_attn_paged(const void *q, const void *k_new, const v
                                        int max_pages, const int32_t *cache_len, const int32_t *parent, void *out,
                                        int B, int T, int Hq, int Hkv, int D, clover_dtype dtype, float scale,
                                        void *workspace, size_t ws_bytes, int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_verify_attn_paged");
     const long lcap = paged_capacity(page_size, max_pages);
     if (lcap < 0 || n_pages < 1) return CLOVER_ERR_INVALID_ARG;
     const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, (int)lcap, dtype);
@@ -354,6 +379,7 @@ clover_status clover_verify_accept(const void *logits, const int32_t *cand, cons
                                    int V, clover_dtype dtype, int32_t *argmax_out, int32_t *path_out,
                                    int32_t *accept_len, int32_t *bonus_token, void *workspace, size_t ws_bytes,
                                    int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_verify_accept");
     AcceptCall c;
     const clover_status s = check_accept(c, logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
                                          bonus_token, workspace, ws_bytes, status, false, 0.0, 0.0, 0.0);
@@ -372,6 +398,7 @@ clover_status clover_verify_accept_typical(const void *logits, const int32_t *ca
                                            double delta, int32_t *argmax_out, int32_t *path_out,
                                            int32_t *accept_len, int32_t *bonus_token, void *workspace,
                                            size_t ws_bytes, int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_verify_accept_typical");
     AcceptCall c;
     const clover_status s = check_accept(c, logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
                                          bonus_token, workspace, ws_bytes, status, true, temperature, epsilon,
@@ -392,6 +419,7 @@ clover_status clover_verify_accept_ex(const void *logits, const int32_t *cand, c
                                       int32_t *path_out, int32_t *accept_len, int32_t *bonus_token,
                                       int32_t *new_cache_len, int32_t *src_index_out, void *workspace,
                                       size_t ws_bytes, uint32_t flags, int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_verify_accept_ex");
     constexpr uint32_t known = CLOVER_ACCEPT_TYPICAL | CLOVER_ACCEPT_COMMIT | CLOVER_ACCEPT_OVERLAP;
     if (flags & ~known) return CLOVER_ERR_INVALID_ARG;
     AcceptCall c;
@@ -426,6 +454,7 @@ clover_status clover_kv_commit(void *k_cache, void *v_cache, const void *k_new, 
                                const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
                                int32_t *new_cache_len, int32_t *src_index_out, int B, int T, int Hkv, int D,
                                int Lcap, clover_dtype dtype, int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_kv_commit");
     const clover_status s = check_commit(k_cache, v_cache, k_new, v_new, cache_len, path, accept_len, new_cache_len,
                                          B, T, Hkv, D, Lcap, dtype, true);
     if (s != CLOVER_OK || B == 0) return s;
@@ -441,6 +470,7 @@ size_t clover_linear_workspace_size(int R, int N, int K) {
 
 clover_status clover_linear(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
                             void *workspace, size_t ws_bytes, int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_linear");
     if (R < 0 || N < 1 || K < 64 || K % 64 != 0) return CLOVER_ERR_INVALID_ARG;
     if (mode < CLOVER_LINEAR_F32 || mode > CLOVER_LINEAR_RES) return CLOVER_ERR_INVALID_ARG;
     const bool with_res = mode == CLOVER_LINEAR_RES_SILU || mode == CLOVER_LINEAR_RES;
@@ -456,6 +486,7 @@ clover_status clover_linear(const void *x, const void *w, const void *res, void 
 
 clover_status clover_embed_rows(const void *w, const int32_t *tokens, void *e, int R, int V, int H, int32_t *status,
                                 void *stream) {
+    const NvtxRange nvtx_range("clover_embed_rows");
     if (R < 0 || V < 1 || H < 1) return CLOVER_ERR_INVALID_ARG;
     if (R == 0) return CLOVER_OK;
     if (!w || !tokens || !e) return CLOVER_ERR_INVALID_ARG;
@@ -469,6 +500,7 @@ size_t clover_topk_workspace_size(int R, int V, int k) {
 
 clover_status clover_topk(const float *x, int R, int V, int k, float *values, int32_t *indices, void *workspace,
                           size_t ws_bytes, int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_topk");
     if (R < 0 || V < 1 || k < 1 || k > V) return CLOVER_ERR_INVALID_ARG;
     if (k > topk_max_k()) return CLOVER_ERR_UNSUPPORTED;
     // the final merge holds two candidates a thread: chunks x k <= 512
@@ -485,6 +517,7 @@ clover_status clover_kv_commit_paged(void *k_pages, void *v_pages, const int32_t
                                      const int32_t *cache_len, const int32_t *path, const int32_t *accept_len,
                                      int32_t *new_cache_len, int32_t *src_index_out, int B, int T, int Hkv, int D,
                                      clover_dtype dtype, int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_kv_commit_paged");
     const long lcap = paged_capacity(page_size, max_pages);
     if (lcap < 0 || n_pages < 1) return CLOVER_ERR_INVALID_ARG;
     const clover_status s = check_commit(k_pages, v_pages, k_new, v_new, cache_len, path, accept_len, new_cache_len,
@@ -501,6 +534,7 @@ clover_status clover_kv_compact(void *k_cache, void *v_cache, const int32_t *cac
                                 const int32_t *accept_len, int32_t *new_cache_len, int32_t *src_index_out, int B,
                                 int T, int Hkv, int D, int Lcap, clover_dtype dtype, int32_t *status,
                                 void *stream) {
+    const NvtxRange nvtx_range("clover_kv_compact");
     const clover_status s = check_commit(k_cache, v_cache, nullptr, nullptr, cache_len, path, accept_len,
                                          new_cache_len, B, T, Hkv, D, Lcap, dtype, false);
     if (s != CLOVER_OK || B == 0) return s;
@@ -566,6 +600,7 @@ extern "C" clover_status clover_verify_attn_noalloc(const void *q, const void *k
                                                     const int32_t *parent, void *out, int B, int T, int Hq,
                                                     int Hkv, int D, int Lcap, clover_dtype dtype, float scale,
                                                     int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_verify_attn_noalloc");
     using namespace clover;
     const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, Lcap, dtype);
     if (s != CLOVER_OK) return s;

@@ -373,6 +373,7 @@ __device__ void commit_sequence(const AcceptArgs &a, int b, const int *s_path, i
             const int e = e0 + t * kThreads;
             if (e < total) {
                 const int j = e / per_node;
+                if (!CLOVER_IN(a.status, s_path[j], Tn)) continue;
                 const size_t src = ((size_t)b * Tn + s_path[j]) * per_node + (e - j * per_node);
                 kb[t] = __ldg(a.k_new + src);
                 vb[t] = __ldg(a.v_new + src);
@@ -386,6 +387,7 @@ __device__ void commit_sequence(const AcceptArgs &a, int b, const int *s_path, i
                 const int r = e - j * per_node;
                 const int g = r / a.row_units;
                 const int u = r - g * a.row_units;
+                if (!CLOVER_IN(a.status, s_path[j], Tn) || !CLOVER_IN(a.status, L + j, a.Lcap)) continue;
                 const size_t dst = (((size_t)b * a.Hkv + g) * a.Lcap + L + j) * a.row_units + u;
                 a.k_cache[dst] = kb[t];
                 a.v_cache[dst] = vb[t];

@@ -44,6 +44,7 @@ struct AttnArgs {
     int pdl;               // launched as a programmatic dependent of the preceding kernel
     int cache_early;       // caches, lengths and block table may be read before that kernel completes
     int inputs_early;      // every input may be read before that kernel completes (only writes wait)
+    size_t ws_bytes;       // workspace bytes (index checks of CLOVER_CHECKED builds)
 };
 
 // One acceptance call (clover_verify_accept, _typical or _ex), validated on
@@ -84,6 +85,21 @@ __device__ __forceinline__ void wait_prerequisite_grids() {
 __device__ __forceinline__ void report(int32_t *status, int bits) {
     if (status) atomicOr(status, bits);
 }
+
+// Index checks of a CLOVER_CHECKED build: CLOVER_IN(status, i, n) is true
+// when 0 <= i < n; otherwise it raises CLOVER_ERR_CHECK in the status word
+// (never traps) and is false, and the call site skips the access it guards.
+// Ordinary builds compile it to true.
+#ifdef CLOVER_CHECKED
+__device__ __forceinline__ bool check_in(int32_t *status, long long i, long long n) {
+    if (i >= 0 && i < n) return true;
+    report(status, CLOVER_ERR_CHECK);
+    return false;
+}
+#define CLOVER_IN(status, i, n) ::clover::check_in((status), (long long)(i), (long long)(n))
+#else
+#define CLOVER_IN(status, i, n) true
+#endif
 
 // Page of cache slot `slot` (< cache_len) of sequence b in a paged cache; an
 // id outside [0, n_pages) is reported and replaced by page 0, so that every

@@ -75,6 +75,7 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
     for (int e = threadIdx.x; e < a * units; e += kThreads) {
         const int j = e / units;
         const int u = e % units;
+        if (!CLOVER_IN(status, k_new ? s_src[j] : L + s_src[j], k_new ? T : Lcap)) continue;
         const size_t src = (k_new ? ((size_t)b * T + s_src[j]) * Hkv + g : head_base + L + s_src[j]) * units + u;
         stage[e] = ks[src];
         stage[T * units + e] = vs[src];
@@ -85,6 +86,7 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(
     for (int e = threadIdx.x; e < a * units; e += kThreads) {
         const int j = e / units;
         const int u = e % units;
+        if (!CLOVER_IN(status, L + j, Lcap)) continue;
         size_t dst = (head_base + L + j) * units + u;
         if (block_table) {
             if (s_dst_page[j] < 0) continue;

@@ -314,6 +314,7 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
             if (R >= a.rows) continue;
             const int i = R / a.G;
             const int h = g * a.G + (R % a.G);
+            if (!CLOVER_IN(a.status, ((size_t)b * a.T + i) * a.Hq + h, (size_t)a.B * a.T * a.Hq)) continue;
             const float inv = 1.f / l_run[r];
             T *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D;
 #pragma unroll
@@ -326,9 +327,11 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
 
     // publish this split's partial result
     const size_t head_tile = (size_t)(b * a.Hkv + g) * a.row_tiles + rt;
-    {
-        float *po = a.part_o + (head_tile * a.n_split + split) * kRT * D;
-        float *pml = a.part_ml + (head_tile * a.n_split + split) * kRT * 2;
+    float *po = a.part_o + (head_tile * a.n_split + split) * kRT * D;
+    float *pml = a.part_ml + (head_tile * a.n_split + split) * kRT * 2;
+    // the workspace starts with the counters: slots must end inside it
+    if (CLOVER_IN(a.status, (const char *)(pml + kRT * 2) - (const char *)a.counters - 1, a.ws_bytes) &&
+        CLOVER_IN(a.status, head_tile, (size_t)a.B * a.Hkv * a.row_tiles)) {
 #pragma unroll
         for (int r = 0; r < 2; ++r) {
 #pragma unroll
@@ -384,8 +387,10 @@ __global__ void __launch_bounds__(kThreads, 2) tree_attn_fma_kernel(const AttnAr
         const int i = R / a.G;
         const int h = g * a.G + (R % a.G);
         T *dst = out + ((size_t)(b * a.T + i) * a.Hq + h) * D + c0;
+        if (CLOVER_IN(a.status, ((size_t)b * a.T + i) * a.Hq + h, (size_t)a.B * a.T * a.Hq)) {
 #pragma unroll
-        for (int e = 0; e < kColsPerThread; ++e) dst[e] = from_float<T>(acc[e] * inv);
+            for (int e = 0; e < kColsPerThread; ++e) dst[e] = from_float<T>(acc[e] * inv);
+        }
     }
     if (tid == 0) a.counters[head_tile] = 0u;   // ready for the next call
 }

@@ -182,6 +182,9 @@ __device__ __forceinline__ void merge_pass(float *own, const float *recv, const 
                 uint2 w2;
                 w2.x = pack_bf16x2(acc[k].x, acc[k].y);
                 w2.y = pack_bf16x2(acc[k].z, acc[k].w);
+#ifdef CLOVER_CHECKED
+                if (orow[rr] == ~0u) continue;   // its index check failed (reported)
+#endif
                 *reinterpret_cast<uint2 *>(out + (size_t)orow[rr] * D + c) = w2;
             }
         }
@@ -327,7 +330,9 @@ __global__ void __maxnreg__(160)
     // parent array.
     constexpr int QW = D / 2;                 // 32-bit TMEM columns of a Q row (two bf16 each)
     const int rq = ((KS == 2) ? (warp & 1) : (warp & 3)) * 32 + lane;
-    const bool q_real = warp < 4 && rq < rows_here;
+    const bool q_real = warp < 4 && rq < rows_here &&
+                        CLOVER_IN(a.status, ((size_t)b * a.T + (rt * BM + rq) / a.G) * a.Hq + g * a.G +
+                                                (rt * BM + rq) % a.G, (size_t)a.B * a.T * a.Hq);
     const uint4 *q_src = reinterpret_cast<const uint4 *>(
         static_cast<const __nv_bfloat16 *>(a.q) +
         ((size_t)(b * a.T + (q_real ? (rt * BM + rq) / a.G : 0)) * a.Hq + g * a.G +
@@ -378,7 +383,8 @@ __global__ void __maxnreg__(160)
     const int chunk = (((L + n_split - 1) / n_split) + BN - 1) / BN * BN;
     const int kbeg = min(L, split * chunk);
     const int kend = min(L, kbeg + chunk);
-    const int n_cache_tiles = (kend - kbeg + BN - 1) / BN;
+    const int n_cache_tiles = (CLOVER_IN(a.status, kbeg, a.Lcap + 1) && CLOVER_IN(a.status, kend, a.Lcap + 1))
+                                  ? (kend - kbeg + BN - 1) / BN : 0;
     const int n_tiles = n_cache_tiles + (tree_cta ? 1 : 0);
     // The tree CTA takes its tree tile first, in every launch mode (so that
     // the result does not depend on the mode): the one CTA with an extra tile
@@ -849,7 +855,10 @@ __global__ void __maxnreg__(160)
         }
         fence_proxy_async_smem();             // the bulk copy reads these rows
         __syncthreads();
-        if (threadIdx.x == 0) {
+        if (threadIdx.x == 0 &&
+            CLOVER_IN(a.status, (((size_t)grp * n_split + split) * a.slot_rows + rows_here) * row_bytes - 1,
+                      a.ws_bytes) &&
+            CLOVER_IN(a.status, grp, (size_t)a.B * a.Hkv * a.row_tiles)) {
             bulk_store_s2g(slots + (size_t)split * a.slot_rows * S::po_stride, part_o, rows_here * row_bytes);
             bulk_commit_group();
             bulk_wait_group0();
@@ -857,7 +866,12 @@ __global__ void __maxnreg__(160)
             red_add_release_gpu(a.counters + grp, 1u);
         }
     } else {
-        if (others > 0 && threadIdx.x == 0) {
+        if (others > 0 && threadIdx.x == 0 &&
+            !(CLOVER_IN(a.status, grp, (size_t)a.B * a.Hkv * a.row_tiles) &&
+              CLOVER_IN(a.status, (((size_t)grp * n_split + others - 1) * a.slot_rows + rows_here) * row_bytes - 1,
+                        a.ws_bytes)))
+            *s_abort = 1;
+        if (others > 0 && threadIdx.x == 0 && !*s_abort) {
             bool in = ld_acquire_gpu(a.counters + grp) >= (unsigned)others;
             if (!in) {
                 const uint64_t t0 = globaltimer_ns();
@@ -876,7 +890,8 @@ __global__ void __maxnreg__(160)
         if ((int)threadIdx.x < rows_here) {
             const int R = rt * BM + (int)threadIdx.x;
             const int i = R / a.G;
-            s_orow[threadIdx.x] = (unsigned)(((size_t)b * a.T + i) * a.Hq + g * a.G + (R - i * a.G));
+            const size_t orow = ((size_t)b * a.T + i) * a.Hq + g * a.G + (R - i * a.G);
+            s_orow[threadIdx.x] = CLOVER_IN(a.status, orow, (size_t)a.B * a.T * a.Hq) ? (unsigned)orow : ~0u;
         }
         if (!*s_abort) {
             float *recv = reinterpret_cast<float *>(sK + S::own_bytes);

@@ -42,6 +42,8 @@ def test_version_and_status_strings(lib):
     assert lib.clover_abi_version() == 1
     assert lib.clover_status_string(0) == b"ok"
     assert b"tree" in lib.clover_status_string(4)
+    assert b"check" in lib.clover_status_string(128)
+    assert lib.clover_build_flags() == 0          # the ordinary build compiles the device checks out
 
 
 def test_workspace_sizes(lib):
@@ -235,3 +237,17 @@ def test_oracle_and_library_share_no_code():
         assert "import oracle" not in open(os.path.join(ROOT, "paper_2405_00263_gb300", fn)).read()
     src = open(os.path.join(ROOT, "oracle", "clover_oracle.c")).read()
     assert "#include \"" not in src and "clover_verify.h" not in src
+
+
+def test_checked_build_exports_the_same_symbols():
+    """The -DCLOVER_CHECKED variant builds, exports the declared symbols and
+    reports itself through clover_build_flags (host-only calls)."""
+    import ctypes
+    from paper_2405_00263_gb300 import _lib
+    from paper_2405_00263_gb300 import build as _build
+    path = _build.build(checked=True)
+    assert path == _build.CHECKED_LIB != _build.LIB
+    lib = ctypes.CDLL(path)
+    for n in declared_symbols():
+        assert hasattr(lib, n), n
+    assert lib.clover_build_flags() & _lib.BUILD_CHECKED
