@@ -313,3 +313,21 @@ def clover_head_step(h, tokens, w_lm, w_v, w_o, w_1, k: int):
     logits = linear(z.to(bf), w_lm)
     vals, idx = topk(logits, k)
     return {"e": e, "v": a, "attn": d, "h": h1, "z": z, "logits": logits, "top_values": vals, "top_indices": idx}
+
+
+def clover_head_step_exact(h, tokens, w_lm, w_v, w_o, w_1, k: int):
+    """The same head step (Section 3.2 Eq. 1-2, the MLP block, the shared LM
+    head) in fp64 throughout: the bf16 inputs h and weights are widened once
+    and no intermediate is rounded, so this is the step's plain definition on
+    those inputs.  Each layer is one fp64 matrix product (a library routine),
+    silu(x) = x / (1 + e^-x).  Same keys as clover_head_step."""
+    W_v, W_o, W_1, W_lm = (_cpu(w).double() for w in (w_v, w_o, w_1, w_lm))
+    e = embed_rows(w_lm, tokens)
+    a = e @ W_v.T
+    d = a @ W_o.T
+    h1 = _cpu(h).double() + d
+    u = h1 @ W_1.T
+    z = h1 + u / (1.0 + torch.exp(-u))
+    logits = z @ W_lm.T
+    vals, idx = topk(logits, k)
+    return {"e": e, "v": a, "attn": d, "h": h1, "z": z, "logits": logits, "top_values": vals, "top_indices": idx}

@@ -673,16 +673,25 @@ __global__ void __maxnreg__(160)
                 tmem_ld32(col, *reinterpret_cast<float(*)[32]>(sv));
                 tmem_ld32(col + 32, *reinterpret_cast<float(*)[32]>(sv + 32));
                 tmem_wait_ld();
+                // a full block (every cache block but a tile's last) needs
+                // no mask: warp-uniform there, so the branch costs nothing
                 const uint64_t vis = block_vis(blk);
+                if (vis != ~0ull) {
 #pragma unroll
-                for (int c = 0; c < 64; ++c) sv[c] = ((vis >> c) & 1ull) ? sv[c] : -INFINITY;
+                    for (int c = 0; c < 64; ++c) sv[c] = ((vis >> c) & 1ull) ? sv[c] : -INFINITY;
+                }
             };
             float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll 1
             for (int bi = 0; bi < NB; ++bi) {
                 load_block(blk0 + bi);
 #pragma unroll
-                for (int c = 0; c < 64; ++c) mx4[c & 3] = fmaxf(mx4[c & 3], sv[c]);
+                for (int c = 0; c < 64; c += 8) {
+                    mx4[0] = fmax3(mx4[0], sv[c], sv[c + 1]);
+                    mx4[1] = fmax3(mx4[1], sv[c + 2], sv[c + 3]);
+                    mx4[2] = fmax3(mx4[2], sv[c + 4], sv[c + 5]);
+                    mx4[3] = fmax3(mx4[3], sv[c + 6], sv[c + 7]);
+                }
             }
             const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * sc;   // sc > 0
 
@@ -708,7 +717,11 @@ __global__ void __maxnreg__(160)
                     tmem_ld32(tO + lane_base + cc * 32, x);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) x[c] *= f;
+                    for (int c = 0; c < 32; c += 2) {
+                        const float2 y = __fmul2_rn(make_float2(x[c], x[c + 1]), make_float2(f, f));
+                        x[c] = y.x;
+                        x[c + 1] = y.y;
+                    }
                     tmem_st32(tO + lane_base + cc * 32, x);
                 }
             }
@@ -716,22 +729,29 @@ __global__ void __maxnreg__(160)
             // P of block blk (two keys per column) goes to packed columns
             // [32 blk, 32 blk + 32) of the tile's TMEM: over S values this
             // thread has already read (blocks in increasing order)
-            float sum4[4] = {0.f, 0.f, 0.f, 0.f};
+            // the exponent arguments and the running sums two at a time
+            // (packed f32x2 FMA and add: the same roundings as one at a time)
+            const float2 sc2 = make_float2(sc, sc);
+            const float2 nref2 = make_float2(-ref, -ref);
+            float2 sum01 = make_float2(0.f, 0.f), sum23 = make_float2(0.f, 0.f);
 #pragma unroll 1
             for (int bi = 0; bi < NB; ++bi) {
                 if (NB > 1) load_block(blk0 + bi);
                 float pk[32];
 #pragma unroll
-                for (int c = 0; c < 64; c += 2) {
-                    const float p0 = ex2_approx(fmaf(sv[c], sc, -ref));
-                    const float p1 = ex2_approx(fmaf(sv[c + 1], sc, -ref));
-                    sum4[c & 3] += p0;
-                    sum4[(c + 1) & 3] += p1;
-                    pk[c >> 1] = __uint_as_float(pack_bf16x2(p0, p1));
+                for (int c = 0; c < 64; c += 4) {
+                    const float2 t01 = __ffma2_rn(make_float2(sv[c], sv[c + 1]), sc2, nref2);
+                    const float2 t23 = __ffma2_rn(make_float2(sv[c + 2], sv[c + 3]), sc2, nref2);
+                    const float2 p01 = make_float2(ex2_approx(t01.x), ex2_approx(t01.y));
+                    const float2 p23 = make_float2(ex2_approx(t23.x), ex2_approx(t23.y));
+                    sum01 = __fadd2_rn(sum01, p01);
+                    sum23 = __fadd2_rn(sum23, p23);
+                    pk[c >> 1] = __uint_as_float(pack_bf16x2(p01.x, p01.y));
+                    pk[(c >> 1) + 1] = __uint_as_float(pack_bf16x2(p23.x, p23.y));
                 }
                 tmem_st32(tS + lane_base + sb * BN + (blk0 + bi) * 32, pk);
             }
-            l_run += (sum4[0] + sum4[1]) + (sum4[2] + sum4[3]);
+            l_run += (sum01.x + sum01.y) + (sum23.x + sum23.y);
             if (KS == 2) {
                 // the other half's keys of this row read as zero
                 float z[32];

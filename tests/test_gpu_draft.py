@@ -165,3 +165,31 @@ def test_draft_head_step_matches_oracle(R, H, V, k):
         else:
             got = head.indices[r].cpu().long()
             assert ((ref["logits"][r, got] - ref["top_values"][r]).abs() <= 4 * tol[r].max()).all()
+
+
+@pytest.mark.parametrize("R,H,V,k", [(8, 512, 3000, 8), (48, 1024, 20000, 4)])
+def test_draft_head_step_against_exact_arithmetic(R, H, V, k):
+    """The head step against the oracle in fp64 throughout (no intermediate
+    bf16 rounding: oracle.clover_head_step_exact), within the rigorous bound
+    of tests/draft_bound.py on what bf16 layer inputs and fp32 sums can cost
+    (its derivation is in that module's docstring).  The bf16 rounding of the
+    layer inputs is the library's reading of the step; this bounds it."""
+    from tests.draft_bound import head_step_bound
+    g = torch.Generator().manual_seed(R * 3 + H)
+    h = rand((R, H), g)
+    toks = torch.randint(0, V, (R,), generator=g, dtype=torch.int32)
+    w_lm = rand((V, H), g, std=H ** -0.5)
+    w_v, w_o, w_1 = (rand((H, H), g, std=H ** -0.5) for _ in range(3))
+    ex = oracle.clover_head_step_exact(h, toks, w_lm, w_v, w_o, w_1, k)
+    E = head_step_bound(h, w_lm, w_v, w_o, w_1, ex)
+    head = pkg.DraftHead(R, H, V, k, device=DEV)
+    head.run(h.to(DEV), toks.to(DEV), w_lm.to(DEV), w_v.to(DEV), w_o.to(DEV), w_1.to(DEV))
+    torch.cuda.synchronize()
+    assert int(head.status.item()) == 0
+    err = (head.logits.cpu().double() - ex["logits"]).abs()
+    assert (err <= E).all(), (err - E).max().item()
+    # the top-k: each chosen index's exact logit within 2 E of the exact k-th best
+    for r in range(R):
+        got = head.indices[r].cpu().long()
+        kth = ex["top_values"][r, -1]
+        assert (ex["logits"][r, got] >= kth - 2 * E[r].max()).all()

@@ -807,3 +807,67 @@ def test_head_step_special_cases():
     e = oracle.embed_rows(w_lm, toks)
     assert torch.allclose(full["attn"], oracle.linear(oracle.linear(e.to(bf), w_v).to(bf), w_o))
     assert torch.allclose(full["h"], h.double() + full["attn"])
+
+
+def test_head_step_exact_hand_example():
+    """A head step worked by hand (H = 2, V = 3, token 0).  The LM-head row
+    (3, 4) has norm 5, so e = (0.6, 0.8); W_v = I gives v = e; W_o = [[1, 1],
+    [0, 2]] gives (1.4, 1.6); with h = (0.5, -1), h' = (1.9, 0.6); W_1 =
+    [[1, 0], [0, 0]] gives W_1 h' = (1.9, 0) and silu(1.9) = 1.9 / (1 +
+    e^-1.9) = 1.652793898710304, silu(0) = 0, so z = (3.552793898710304, 0.6);
+    the LM head rows (3, 4), (1, 0), (0, 2) give 3 z0 + 4 z1, z0 and 2 z1."""
+    bf = torch.bfloat16
+    w_lm = torch.tensor([[3.0, 4.0], [1.0, 0.0], [0.0, 2.0]]).to(bf)
+    w_v = torch.eye(2).to(bf)
+    w_o = torch.tensor([[1.0, 1.0], [0.0, 2.0]]).to(bf)
+    w_1 = torch.tensor([[1.0, 0.0], [0.0, 0.0]]).to(bf)
+    h = torch.tensor([[0.5, -1.0]]).to(bf)
+    out = oracle.clover_head_step_exact(h, torch.tensor([0], dtype=torch.int32), w_lm, w_v, w_o, w_1, 2)
+    close = lambda a, b: torch.allclose(a, torch.tensor([b], dtype=torch.float64), rtol=1e-14, atol=1e-14)
+    assert close(out["e"], [0.6, 0.8])
+    assert close(out["v"], [0.6, 0.8])
+    assert close(out["attn"], [1.4, 1.6])
+    assert close(out["h"], [1.9, 0.6])
+    assert close(out["z"], [3.552793898710304, 0.6])
+    assert close(out["logits"], [13.058381696130912, 3.552793898710304, 1.2])
+    assert out["top_indices"].tolist() == [[0, 1]]
+
+
+def test_head_step_exact_special_cases():
+    """W_v = W_1 = 0: the step reduces to the LM head of h (the oracle's C
+    linear layer, an independent fp64 sum)."""
+    g = torch.Generator().manual_seed(21)
+    R, H, V = 3, 48, 200
+    bf = torch.bfloat16
+    h = torch.randn(R, H, generator=g).to(bf)
+    w_lm = torch.randn(V, H, generator=g).to(bf)
+    z0 = torch.zeros(H, H, dtype=bf)
+    w_o = torch.randn(H, H, generator=g).to(bf)
+    out = oracle.clover_head_step_exact(h, torch.tensor([1, 2, 3], dtype=torch.int32), w_lm, z0, w_o, z0, 5)
+    assert torch.equal(out["z"], h.double())
+    assert torch.allclose(out["logits"], oracle.linear(h, w_lm), rtol=1e-13, atol=1e-13)
+
+
+def test_head_step_bf16_reading_within_derived_bound():
+    """The oracle's bf16-input reading of the head step stays within the
+    worst-case rounding bound of tests/draft_bound.py of the exact step, the
+    bound is small against the logits, and plausible mistakes (the residual
+    dropped, W_o's sign flipped) break it."""
+    from tests.draft_bound import head_step_bound
+    g = torch.Generator().manual_seed(22)
+    R, H, V, k = 4, 128, 600, 4
+    bf = torch.bfloat16
+    rnd = lambda *s, std=1.0: (torch.randn(*s, generator=g, dtype=torch.float64) * std).to(bf)
+    h = rnd(R, H)
+    w_lm = rnd(V, H, std=H ** -0.5)
+    w_v, w_o, w_1 = (rnd(H, H, std=H ** -0.5) for _ in range(3))
+    toks = torch.randint(0, V, (R,), generator=g, dtype=torch.int32)
+    ex = oracle.clover_head_step_exact(h, toks, w_lm, w_v, w_o, w_1, k)
+    rd = oracle.clover_head_step(h, toks, w_lm, w_v, w_o, w_1, k)
+    E = head_step_bound(h, w_lm, w_v, w_o, w_1, ex)
+    assert ((rd["logits"] - ex["logits"]).abs() <= E).all()
+    assert E.max() < 0.25 * ex["logits"].abs().max()
+    no_res = oracle.clover_head_step_exact(torch.zeros_like(h), toks, w_lm, w_v, w_o, w_1, k)
+    assert ((no_res["logits"] - ex["logits"]).abs() > E).any()
+    flip = oracle.clover_head_step_exact(h, toks, w_lm, w_v, (-w_o.double()).to(bf), w_1, k)
+    assert ((flip["logits"] - ex["logits"]).abs() > E).any()
