@@ -70,7 +70,11 @@ constexpr int kPageSmem = 512;           // page ids of a split staged in shared
 constexpr int kKProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kVProducerWarp = 6;
-constexpr int kThreads = 224;
+constexpr int kSoft2Warp = 7;           // KS = 1: warps 7-10 are a second softmax group
+// Threads of a CTA: 7 warps; with KS = 1 (full 128-row tiles) 4 more, so that
+// two softmax warps share each TMEM lane quadrant, 64 keys of a tile each.
+template <int KS>
+constexpr int threads_of() { return KS == 1 ? 352 : 224; }
 constexpr int kMaxSplits = 8;           // key ranges per (sequence, head, row tile)
 constexpr int kMaxSrc = kMaxSplits + 2;  // partial rows merged into one output row (own halves + others)
 constexpr float kRescale = 8.0f;        // move the reference max only past 2^8 growth
@@ -90,14 +94,15 @@ struct TcSmem {
     static constexpr int k_off = 0;
     static constexpr int v_off = k_off + NSK * kv_bytes;
     static constexpr int bar_off = v_off + NSV * kv_bytes;
-    static constexpr int n_bars = 2 * NSK + 2 * NSV + 10;
+    static constexpr int n_bars = 2 * NSK + 2 * NSV + 14;
     static constexpr int misc_off = bar_off + 8 * n_bars;          // tmem addr, abort, bad
     static constexpr int anc_off = misc_off + 16;                  // ancestor masks [128][2]
     static constexpr int pages_off = anc_off + kMaxTreeNodes * kMaskWords * 8;   // paged: page ids of the split
     static constexpr int wts_off = pages_off + kPageSmem * 4;      // merge weights [BM][kMaxSrc]
     static constexpr int par_off = wts_off + BM * kMaxSrc * 4;     // the tree's parent array [128]
     static constexpr int orow_off = par_off + kMaxTreeNodes * 4;   // output row of each tile row [BM]
-    static constexpr int total = orow_off + BM * 4;
+    static constexpr int x_off = orow_off + BM * 4;              // KS = 1: pair exchange [2][2][BM] + flags [2][2][4]
+    static constexpr int total = x_off + 2 * 2 * BM * 4 + 2 * 2 * 4 * 4;
     static constexpr size_t alloc = total + 1024;                  // base rounded up to 1024 bytes
     // TMEM columns: S/P 2 x BN, O D, Q D / 2 (two bf16 per column), rounded up
     // to a power of two.  All 512 columns of an SM go to one CTA only when
@@ -262,12 +267,15 @@ __global__ void __maxnreg__(160)
     uint64_t *q_full = mma_done + 1;          // the four lane quadrants hold their Q rows in TMEM
     uint64_t *g_full = q_full + 1;            // the merging CTA: a pass of the other splits' partials is here
     uint64_t *anc_full = g_full + 1;          // the tree CTA: the ancestor masks are in shared memory
+    uint64_t *x_bar = anc_full + 1;           // [4] KS = 1: the two softmax warps of a lane quadrant exchanged a value
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(sm + S::misc_off);
     volatile int *s_abort = reinterpret_cast<volatile int *>(sm + S::misc_off + 4);
     bool *s_bad = reinterpret_cast<bool *>(sm + S::misc_off + 8);
     uint64_t *s_anc = reinterpret_cast<uint64_t *>(sm + S::anc_off);
     int *s_pages = reinterpret_cast<int *>(sm + S::pages_off);
     float *s_wts = reinterpret_cast<float *>(sm + S::wts_off);
+    float *s_xv = reinterpret_cast<float *>(sm + S::x_off);               // [parity][group][row]
+    volatile int *s_xf = reinterpret_cast<volatile int *>(sm + S::x_off + 2 * 2 * BM * 4);   // [parity][group][quad]
     int *s_par = reinterpret_cast<int *>(sm + S::par_off);
     unsigned *s_orow = reinterpret_cast<unsigned *>(sm + S::orow_off);
 
@@ -285,7 +293,8 @@ __global__ void __maxnreg__(160)
     const bool tree_cta = (split == n_split - 1);
     const int rows_here = min(BM, a.rows - rt * BM);
     const int q_act = (rows_here + 31) >> 5;        // 32-row quadrants holding real rows
-    const int n_soft_warps = KS * q_act;             // softmax warps of this tile
+    constexpr int NG = (KS == 1) ? 2 : 1;            // softmax warps per TMEM lane quadrant
+    const int n_soft_warps = 2 * q_act;              // softmax warps of this tile (KS * NG per quadrant)
 
     // ------------------------------------------ setup that reads no input
     // Each producer initialises the barriers of its ring (the K producer also
@@ -313,6 +322,7 @@ __global__ void __maxnreg__(160)
         mbar_init(q_full, 4);
         mbar_init(g_full, 1);
         mbar_init(anc_full, 1);
+        for (int i = 0; i < 4; ++i) mbar_init(&x_bar[i], 2);
         *s_abort = 0;
         *s_bad = false;
         fence_barrier_init();
@@ -613,23 +623,47 @@ __global__ void __maxnreg__(160)
     }
 
     // ------------------------------------------------------------ softmax warps
-    // Warp w owns TMEM lanes 32w.. (the lanes it may access); it reads S there,
-    // writes P back over it, keeps the reference max m_ref and sum l, and
-    // rescales its O rows in TMEM when m_ref has to move.  KS = 1: lanes 32w..
-    // are tile rows 32w.. and the warp takes every key of a tile.  KS = 2:
-    // lanes 32w.. are rows 32(w & 1).. and the warp takes keys
-    // [32 (w >> 1), +32) of every tile; the two key halves of a row are two
-    // separate online softmaxes (own m, l and O rows), merged after the loop.
-    constexpr int NK = BN / KS;               // keys of a tile per thread
+    // A softmax warp reads S in the TMEM lanes of its quadrant (warp % 4, the
+    // lanes it may access), one 64-key block of every tile, writes that
+    // block's P back over S, keeps the reference max m_ref and the sum l, and
+    // rescales its share of the O rows in TMEM when m_ref has to move.
+    //   KS = 2 (a tile of at most 64 real rows): warps 0-3; lanes 32w.. are
+    //   rows 32 (w & 1).. and the warp takes key block w >> 1; the two key
+    //   halves of a row are two separate online softmaxes (own m, l and O
+    //   rows), merged after the loop.
+    //   KS = 1: warps 0-3 (group 0) and 7-10 (group 1); lanes 32 (w % 4).. are
+    //   rows 32 (w % 4).. and group g takes key block g.  The two warps of a
+    //   quadrant exchange their block maxima through shared memory (an
+    //   mbarrier of two arrivals a tile, its wait bounded), so that both use
+    //   one reference max and the P of a row is one softmax; each rescales
+    //   half of the O columns, and their sums add up after the loop.
+    const int sgroup = warp < 4 ? 0 : (NG == 2 && warp >= kSoft2Warp && warp < kSoft2Warp + 4) ? 1 : -1;
     const int quad = warp & 3;
     const int rquad = (KS == 2) ? (quad & 1) : quad;
     const int half = (KS == 2) ? (quad >> 1) : 0;
-    const bool softmax_warp = warp < 4 && rquad < q_act;
+    const bool softmax_warp = sgroup >= 0 && rquad < q_act;
     const int r = rquad * 32 + lane;          // tile row
-    const int soft_rank = ((KS == 2) ? half * q_act + rquad : quad) * 32 + lane;
+    const int blk = (KS == 2) ? half : sgroup;   // this thread's 64-key block of a tile
+    const int soft_rank = (((KS == 2) ? half : sgroup) * q_act + rquad) * 32 + lane;
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
+    constexpr int OC = D / 32 / NG;           // 32-column chunks of O a softmax warp rescales and stores
+    const int oc0 = (sgroup > 0 ? sgroup : 0) * OC;
     float m_ref = -INFINITY, l_run = 0.f;
     bool o_ready = false;
+    int xn = 0;                               // exchanges made with the other warp of the quadrant
+    // KS = 1: swap v (and a stop flag) with the quadrant's other warp; on a
+    // timeout the partner's value reads as -inf and the flag as set
+    auto exchange = [&](float v, bool &stop) -> float {
+        const int par = xn & 1;
+        s_xv[(par * 2 + sgroup) * BM + r] = v;
+        if (lane == 0) s_xf[(par * 2 + sgroup) * 4 + quad] = stop ? 1 : 0;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&x_bar[quad]);
+        const bool got = __all_sync(0xffffffffu, mbar_wait(&x_bar[quad], par, kWaitNs));
+        ++xn;
+        stop = stop || !got || s_xf[(par * 2 + 1 - sgroup) * 4 + quad] != 0;
+        return got ? s_xv[(par * 2 + 1 - sgroup) * BM + r] : -INFINITY;
+    };
     if (softmax_warp) {
         const int R = rt * BM + r;
         const int node = (r < rows_here) ? R / a.G : 0;
@@ -637,54 +671,35 @@ __global__ void __maxnreg__(160)
         for (int j = 0; j < n_tiles; ++j) {
             const int sb = j & 1;
             const uint32_t ph = (j >> 1) & 1;
-            const bool got = __all_sync(0xffffffffu, mbar_wait(&s_full[sb], ph, kWaitNs));
-            if (!got || __any_sync(0xffffffffu, *s_abort != 0)) {
-                *s_abort = 1;
-                break;
-            }
-            tc_fence_after();
             const bool tree_tile = j == tree_j;
-            if (tree_tile) {
-                const bool got_anc = __all_sync(0xffffffffu, mbar_wait(anc_full, 0, kWaitNs));
-                if (!got_anc) {
-                    *s_abort = 1;
-                    break;
-                }
-            }
+            bool stop = !__all_sync(0xffffffffu, mbar_wait(&s_full[sb], ph, kWaitNs)) ||
+                        __any_sync(0xffffffffu, *s_abort != 0);
+            if (!stop && tree_tile) stop = !__all_sync(0xffffffffu, mbar_wait(anc_full, 0, kWaitNs));
             const int key0 = kbeg + (j - tree_shift) * BN;
             const int n_valid = tree_tile ? a.T : min(BN, kend - key0);
-            // Keys of a 64-key block of the tile that this row sees: a prefix
-            // of the cache keys, or the row's ancestors among the (at most
-            // 128) tree keys, word blk of its mask.  Every tile runs the same
+            // Keys of the thread's 64-key block that its row sees: a prefix of
+            // the cache keys, or the row's ancestors among the (at most 128)
+            // tree keys, word blk of its mask.  Every tile runs the same
             // instructions, so the one tree tile brings no code into the
             // instruction cache (a miss then waits on a saturated memory system).
-            auto block_vis = [&](int blk) -> uint64_t {
-                const int nv = n_valid - 64 * blk;
-                const uint64_t prefix = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
-                return tree_tile ? s_anc[node * kMaskWords + blk] : prefix;
-            };
-            // this thread's NB blocks of 64 keys start at block blk0 (KS = 2:
-            // the key half; KS = 1: both halves, S re-read from TMEM per pass)
-            constexpr int NB = NK / 64;
-            const int blk0 = half * NB;
             float sv[64];
-            auto load_block = [&](int blk) {
+            float mxb = -INFINITY;
+            if (!stop) {
+                tc_fence_after();
                 const uint32_t col = tS + lane_base + sb * BN + blk * 64;
                 tmem_ld32(col, *reinterpret_cast<float(*)[32]>(sv));
                 tmem_ld32(col + 32, *reinterpret_cast<float(*)[32]>(sv + 32));
                 tmem_wait_ld();
-                // a full block (every cache block but a tile's last) needs
-                // no mask: warp-uniform there, so the branch costs nothing
-                const uint64_t vis = block_vis(blk);
+                const int nv = n_valid - 64 * blk;
+                const uint64_t prefix = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
+                const uint64_t vis = tree_tile ? s_anc[node * kMaskWords + blk] : prefix;
+                // a full block (every cache block but a tile's last) needs no
+                // mask: warp-uniform there, so the branch costs nothing
                 if (vis != ~0ull) {
 #pragma unroll
                     for (int c = 0; c < 64; ++c) sv[c] = ((vis >> c) & 1ull) ? sv[c] : -INFINITY;
                 }
-            };
-            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll 1
-            for (int bi = 0; bi < NB; ++bi) {
-                load_block(blk0 + bi);
+                float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
                 for (int c = 0; c < 64; c += 8) {
                     mx4[0] = fmax3(mx4[0], sv[c], sv[c + 1]);
@@ -692,8 +707,19 @@ __global__ void __maxnreg__(160)
                     mx4[2] = fmax3(mx4[2], sv[c + 4], sv[c + 5]);
                     mx4[3] = fmax3(mx4[3], sv[c + 6], sv[c + 7]);
                 }
+                mxb = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
             }
-            const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])) * sc;   // sc > 0
+            // the row's max over the tile (KS = 1: over both warps' blocks;
+            // group 0's first, so both warps compute the same value)
+            if (NG == 2) {
+                const float other = exchange(mxb, stop);
+                mxb = sgroup == 0 ? fmaxf(mxb, other) : fmaxf(other, mxb);
+            }
+            if (stop) {
+                *s_abort = 1;
+                break;
+            }
+            const float mx = mxb * sc;            // sc > 0
 
             // move the reference max when this tile exceeds it by more than 2^8
             const bool move = (mx > m_ref + kRescale);
@@ -712,7 +738,7 @@ __global__ void __maxnreg__(160)
                 l_run *= f;
                 if (move) m_ref = mx;
 #pragma unroll 1
-                for (int cc = 0; cc < D / 32; ++cc) {
+                for (int cc = oc0; cc < oc0 + OC; ++cc) {
                     float x[32];
                     tmem_ld32(tO + lane_base + cc * 32, x);
                     tmem_wait_ld();
@@ -726,17 +752,17 @@ __global__ void __maxnreg__(160)
                 }
             }
             const float ref = (m_ref == -INFINITY) ? 0.f : m_ref;
-            // P of block blk (two keys per column) goes to packed columns
-            // [32 blk, 32 blk + 32) of the tile's TMEM: over S values this
-            // thread has already read (blocks in increasing order)
-            // the exponent arguments and the running sums two at a time
-            // (packed f32x2 FMA and add: the same roundings as one at a time)
+            // P of the block (two keys per column) goes to packed columns
+            // [32 blk, 32 blk + 32) of the tile's TMEM, over S values already
+            // read: this thread's own (block 0) or, for block 1, those of
+            // block 0, which its reader had loaded before the exchange
+            // (KS = 1) or which sit in other lanes (KS = 2).  The exponent
+            // arguments and the running sums go two at a time (packed f32x2
+            // FMA and add: the same roundings as one at a time).
             const float2 sc2 = make_float2(sc, sc);
             const float2 nref2 = make_float2(-ref, -ref);
             float2 sum01 = make_float2(0.f, 0.f), sum23 = make_float2(0.f, 0.f);
-#pragma unroll 1
-            for (int bi = 0; bi < NB; ++bi) {
-                if (NB > 1) load_block(blk0 + bi);
+            {
                 float pk[32];
 #pragma unroll
                 for (int c = 0; c < 64; c += 4) {
@@ -749,7 +775,7 @@ __global__ void __maxnreg__(160)
                     pk[c >> 1] = __uint_as_float(pack_bf16x2(p01.x, p01.y));
                     pk[(c >> 1) + 1] = __uint_as_float(pack_bf16x2(p23.x, p23.y));
                 }
-                tmem_st32(tS + lane_base + sb * BN + (blk0 + bi) * 32, pk);
+                tmem_st32(tS + lane_base + sb * BN + blk * 32, pk);
             }
             l_run += (sum01.x + sum01.y) + (sum23.x + sum23.y);
             if (KS == 2) {
@@ -804,37 +830,48 @@ __global__ void __maxnreg__(160)
     __syncthreads();
     tc_fence_after();
     // (1) every softmax warp moves the O rows, m and l of its TMEM lanes to
-    // part_o row 32 quad + lane: KS = 1, tile row r; KS = 2, the first key half
-    // of tile row r in rows 0-63 and the second half in rows 64-127.  The TMEM
-    // loads are warp-collective: every lane runs them, rows past the tile's
-    // real rows only skip the stores.
+    // part_o row 32 quad + lane: KS = 1, tile row r (each warp of the quadrant
+    // its half of the columns, group 0 m and the sum of both warps' l); KS =
+    // 2, the first key half of tile row r in rows 0-63 and the second half in
+    // rows 64-127.  The TMEM loads are warp-collective: every lane runs them,
+    // rows past the tile's real rows only skip the stores.
     float *part_o = reinterpret_cast<float *>(sK);            // [BM][D + 4] fp32
     if (softmax_warp) {
         const bool real = r < rows_here;
         float *dst = part_o + (quad * 32 + lane) * S::po_stride;
+        float l_tot = l_run;
+        if (NG == 2) {
+            bool stop = !o_ready;
+            const float other = exchange(l_run, stop);
+            l_tot = sgroup == 0 ? l_run + other : other + l_run;
+            if (stop) *s_abort = 1;
+        }
+        constexpr int NP = (OC % 2 == 0) ? 2 : 1;             // chunks per TMEM round trip
 #pragma unroll 1
-        for (int cc = 0; cc < D / 32; cc += 2) {
-            float x0[32], x1[32];
+        for (int cc = oc0; cc < oc0 + OC; cc += NP) {
+            float x[NP][32];
             if (o_ready) {
-                tmem_ld32(tO + lane_base + cc * 32, x0);
-                tmem_ld32(tO + lane_base + cc * 32 + 32, x1);
+#pragma unroll
+                for (int p = 0; p < NP; ++p) tmem_ld32(tO + lane_base + (cc + p) * 32, x[p]);
                 tmem_wait_ld();
             } else {
 #pragma unroll
-                for (int c = 0; c < 32; ++c) x0[c] = x1[c] = 0.f;
+                for (int p = 0; p < NP; ++p)
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) x[p][c] = 0.f;
             }
             if (real) {
 #pragma unroll
-                for (int c = 0; c < 32; c += 4) {
-                    *reinterpret_cast<float4 *>(dst + cc * 32 + c) = make_float4(x0[c], x0[c + 1], x0[c + 2], x0[c + 3]);
-                    *reinterpret_cast<float4 *>(dst + cc * 32 + 32 + c) =
-                        make_float4(x1[c], x1[c + 1], x1[c + 2], x1[c + 3]);
-                }
+                for (int p = 0; p < NP; ++p)
+#pragma unroll
+                    for (int c = 0; c < 32; c += 4)
+                        *reinterpret_cast<float4 *>(dst + (cc + p) * 32 + c) =
+                            make_float4(x[p][c], x[p][c + 1], x[p][c + 2], x[p][c + 3]);
             }
         }
-        if (real)
+        if (real && sgroup == 0)
             *reinterpret_cast<float4 *>(dst + D) =
-                make_float4(o_ready ? m_ref : -INFINITY, o_ready ? l_run : 0.f, 0.f, 0.f);
+                make_float4(o_ready ? m_ref : -INFINITY, o_ready ? l_tot : 0.f, 0.f, 0.f);
     }
     // every TMEM access and MMA is finished before TMEM is released
     tc_fence_before();
@@ -976,7 +1013,7 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
 
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.row_tiles, a.n_split, a.B * a.Hkv);
-    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.blockDim = dim3(threads_of<KS>(), 1, 1);
     cfg.dynamicSmemBytes = TcSmem<D, KS>::alloc;
     cfg.stream = stream;
     cudaLaunchAttribute attr;
