@@ -44,6 +44,7 @@ METRIC = "verify steps/sec and tree-attn achieved HBM GB/s (% of GB300 peak) at 
 UNIT = "verify steps/s"
 DEFAULT_WORKLOAD = "7b_l4096"
 L2_BYTES = 129 * 1000 * 1000
+STEP_PASSES = 4          # passes over the input sets in one captured graph of steps
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 KERNEL_SOURCES = {
@@ -292,22 +293,24 @@ def run_gpu_arm(args, world, rank, local, dist):
     if step.device_status() != 0:
         raise RuntimeError(f"device status {step.device_status()} during warm-up")
 
-    # CUDA graphs of consecutive steps: the full graph runs one step on every
-    # input set in turn, each step's calls queued behind the previous step's
-    # (as in a decoding loop); single-step graphs time the remainder of K.  The
-    # timed graphs carry no timing nodes.
+    # CUDA graphs of consecutive steps: the full graph runs STEP_PASSES steps on
+    # every input set in turn, each step's calls queued behind the previous
+    # step's (as in a decoding loop captured as one graph); single-step graphs
+    # time the remainder of K.  The timed graphs carry no timing nodes.
+    per_graph = STEP_PASSES * n_sets
     full = torch.cuda.CUDAGraph()
     with torch.cuda.graph(full, stream=stream):
-        for s in sets:
-            launch(s)
+        for _ in range(STEP_PASSES):
+            for s in sets:
+                launch(s)
     singles = []
-    for s in sets[:args.steps % n_sets]:
+    for i in range(args.steps % per_graph):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            launch(s)
+            launch(sets[i % n_sets])
         singles.append(g)
     torch.cuda.synchronize(device)
-    for _ in range(max(1, -(-max(3, args.warmup) // n_sets))):
+    for _ in range(max(1, -(-max(3, args.warmup) // per_graph))):
         full.replay()
     torch.cuda.synchronize(device)
 
@@ -322,7 +325,7 @@ def run_gpu_arm(args, world, rank, local, dist):
         sampler.mark("t0")
     with torch.cuda.stream(stream):
         start.record(stream)
-        for _ in range(args.steps // n_sets):
+        for _ in range(args.steps // per_graph):
             full.replay()
         for g in singles:
             g.replay()
@@ -438,13 +441,13 @@ def run_gpu_arm(args, world, rank, local, dist):
 
 
 LAUNCH_DESC = {
-    "commit": "CUDA graphs of consecutive steps (one per input set, each queued behind the last); a step: the "
+    "commit": "CUDA graphs of consecutive steps (four passes over the input sets, each step queued behind the last); a step: the "
               "attention (cache read only) on one stream, argmax/accept then the commit of the accepted K/V on a "
               "second stream",
-    "compact": "CUDA graphs of consecutive steps (one per input set, each queued behind the last); a step: the "
+    "compact": "CUDA graphs of consecutive steps (four passes over the input sets, each step queued behind the last); a step: the "
                "attention (appending the tree K/V) on one stream and argmax/accept on a second, then the "
                "compaction of the accepted K/V",
-    "fused": "CUDA graphs of consecutive steps (one per input set, each queued behind the last); a step: two "
+    "fused": "CUDA graphs of consecutive steps (four passes over the input sets, each step queued behind the last); a step: two "
              "launches on one stream, the attention (cache read only), then argmax/accept with the commit of the "
              "accepted K/V fused in, launched as a programmatic dependent of the attention so that it runs "
              "beside it",
@@ -978,7 +981,7 @@ def main(argv=None):
                     help="time one Clover draft head step on this many rows (7B shapes) instead of verification")
     ap.add_argument("--page-size", type=int, default=0,
                     help="run on a paged KV cache with pages of this many slots (0: dense cache)")
-    ap.add_argument("--schedule", default="commit", choices=["commit", "compact", "fused"],
+    ap.add_argument("--schedule", default="fused", choices=["commit", "compact", "fused"],
                     help="call schedule of the step (VerifyStep)")
     ap.add_argument("--attn-launch", default="inputs_ready", choices=["ordinary", "pdl", "cache_ready", "inputs_ready"],
                     help="attention launch: ordinary, or a programmatic dependent of the kernel before it, with the "

@@ -27,6 +27,8 @@ SMALL = {
     "bf16_ragged_batch": ("7b_batched", dict(B=5, Hq=8, Hkv=8, L_range=(0, 700), V=3001)),
     "bf16_sharp_scores": ("7b_l2048", dict(T=64, Hq=4, Hkv=2, L=900, V=2048, qkv_std=1.5)),
     "bf16_gqa8_T64": ("100b_gqa", dict(B=1, Hq=16, Hkv=2, L=640, V=2048)),
+    # two 128-row tiles per key range: a cluster of two sharing K/V tiles by multicast, with split merges
+    "bf16_gqa4_T64_pairs": ("100b_gqa", dict(B=2, Hq=16, Hkv=4, L=900, V=2048)),
     # trees past 64 nodes: two mask words, two FMA tree tiles, four nodes per lane in the walk
     "bf16_T128_topk": ("7b_l2048", dict(T=128, Hq=4, Hkv=4, L=700, V=3000, branching=(8, 4, 2, 2, 2, 1))),
     "bf16_T128_chain": ("7b_l2048", dict(T=128, Hq=2, Hkv=2, L=300, V=2048, tree="chain", plant_p=1.0)),
