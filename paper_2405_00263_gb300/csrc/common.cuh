@@ -45,8 +45,6 @@ struct AttnArgs {
     int cache_early;       // caches, lengths and block table may be read before that kernel completes
     int inputs_early;      // every input may be read before that kernel completes (only writes wait)
     size_t ws_bytes;       // workspace bytes (index checks of CLOVER_CHECKED builds)
-    int mc;                // tensor-core kernel: CTAs of one cluster (the row tiles of a key range)
-                           // that share every K/V tile by TMA multicast; set by its launcher (1: none)
 };
 
 // One acceptance call (clover_verify_accept, _typical or _ex), validated on

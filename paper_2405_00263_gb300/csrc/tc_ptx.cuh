@@ -188,18 +188,6 @@ __device__ __forceinline__ void tma_load_3d_hint(void *smem_dst, const CUtensorM
         : "memory");
 }
 
-// tma_load_3d to the same shared-memory offset in every CTA of the cluster
-// named by `mask` (bit r: rank r), completing as transaction bytes on the
-// mbarrier at `bar`'s offset in each of them; with an L2 cache policy.
-__device__ __forceinline__ void tma_load_3d_mc_hint(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x,
-                                                    int y, int z, uint16_t mask, uint64_t policy) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster.L2::cache_hint"
-        " [%0], [%1, {%2, %3, %4}], [%5], %6, %7;" ::"r"(smem_u32(smem_dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "h"(mask), "l"(policy)
-        : "memory");
-}
-
 // Bulk copy (TMA engine) of `bytes` contiguous bytes from global memory to this
 // CTA's shared memory, completing as transaction bytes on `bar`.  Both
 // addresses 16-byte aligned, size a multiple of 16.
@@ -319,24 +307,6 @@ __device__ __forceinline__ void mma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tmem
 __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                      smem_u32(bar))
-                 : "memory");
-}
-
-// tma_load_3d_mc_hint without a cache policy.
-__device__ __forceinline__ void tma_load_3d_mc(void *smem_dst, const CUtensorMap *map, uint64_t *bar, int x, int y,
-                                               int z, uint16_t mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "h"(mask)
-        : "memory");
-}
-
-// mma_commit on the mbarrier at `bar`'s offset in every CTA of the cluster
-// named by `mask`.
-__device__ __forceinline__ void mma_commit_mc(uint64_t *bar, uint16_t mask) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-                     smem_u32(bar)), "h"(mask)
                  : "memory");
 }
 

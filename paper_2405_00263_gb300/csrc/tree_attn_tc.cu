@@ -290,14 +290,6 @@ __global__ void __maxnreg__(160)
     const int b = bg / a.Hkv;
     const int g = bg % a.Hkv;
     const int n_split = a.n_split;
-    // With mc > 1 the mc row tiles of a key range form a cluster that shares
-    // every K/V tile: each CTA loads rows [crank BN / mc, +BN / mc) of a tile
-    // into all of them (TMA multicast), so L2 sends each tile once to the
-    // cluster instead of once to every row tile.
-    const int mc = PAGED ? 1 : a.mc;
-    const uint32_t crank = mc > 1 ? cluster_ctarank() : 0u;
-    const uint16_t cmask = static_cast<uint16_t>((1u << mc) - 1u);
-    const int rows_mc = BN / mc;
     const bool tree_cta = (split == n_split - 1);
     const int rows_here = min(BM, a.rows - rt * BM);
     const int q_act = (rows_here + 31) >> 5;        // 32-row quadrants holding real rows
@@ -310,7 +302,7 @@ __global__ void __maxnreg__(160)
     if (warp == kVProducerWarp && lane == 0) {
         for (int i = 0; i < NSV; ++i) {
             mbar_init(&v_full[i], 1);
-            mbar_init(&v_empty[i], mc);           // every CTA of the cluster releases the stage
+            mbar_init(&v_empty[i], 1);
         }
         fence_barrier_init();
         prefetch_tensormap(&tm_vc);
@@ -319,7 +311,7 @@ __global__ void __maxnreg__(160)
     if (warp == kKProducerWarp && lane == 0) {
         for (int i = 0; i < NSK; ++i) {
             mbar_init(&k_full[i], 1);
-            mbar_init(&k_empty[i], mc);
+            mbar_init(&k_empty[i], 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&s_full[i], 1);
@@ -341,9 +333,6 @@ __global__ void __maxnreg__(160)
         tmem_alloc(s_tmem, S::tmem_cols);
         tmem_relinquish();
     }
-    // a cluster's barriers are initialised everywhere before any tile is
-    // multicast into it
-    if (mc > 1) cluster_sync_all();
 
     // Q rows of this warp's TMEM lane quadrant (row (node, head in group) =
     // lane-quadrant row; with KS = 2 lanes 64-127 take rows 0-63 again); rows
@@ -452,21 +441,10 @@ __global__ void __maxnreg__(160)
                     tma_load_3d_hint(dst + dh * BN * 128 + r * 128, cache_map, bar, dh * 64, row, pg[x] * a.Hkv + g,
                                      pol);
             }
-        } else if (j != tree_j && mc > 1) {
-            const int r0 = (int)crank * rows_mc;
-#pragma unroll
-            for (int dh = 0; dh < S::DH; ++dh)
-                tma_load_3d_mc_hint(dst + dh * BN * 128 + r0 * 128, cache_map, bar, dh * 64,
-                                    kbeg + (j - tree_shift) * BN + r0, bg, cmask, pol);
         } else if (j != tree_j) {
 #pragma unroll
             for (int dh = 0; dh < S::DH; ++dh)
                 tma_load_3d_hint(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + (j - tree_shift) * BN, bg, pol);
-        } else if (mc > 1) {
-            const int r0 = (int)crank * rows_mc;
-#pragma unroll
-            for (int dh = 0; dh < S::DH; ++dh)
-                tma_load_3d_mc(dst + dh * BN * 128 + r0 * 128, new_map, bar, dh * 64, g, b * a.T + r0, cmask);
         } else {
 #pragma unroll
             for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, new_map, bar, dh * 64, g, b * a.T);
@@ -612,8 +590,7 @@ __global__ void __maxnreg__(160)
                 mma_bf16_tmem_a(tS + sb * BN, tQ + k * 8, bd, idS, k > 0 ? 1u : 0u);
             }
             mma_commit(&s_full[sb]);
-            if (mc > 1) mma_commit_mc(&k_empty[s], cmask);
-            else mma_commit(&k_empty[s]);
+            mma_commit(&k_empty[s]);
             return true;
         };
         int s_issued = 0;
@@ -639,8 +616,7 @@ __global__ void __maxnreg__(160)
                 mma_bf16_tmem_a(tO, tS + sb * BN + k * 8, bd, idO, (j > 0 || k > 0) ? 1u : 0u);
             }
             mma_commit(&o_full[sb]);
-            if (mc > 1) mma_commit_mc(&v_empty[s], cmask);
-            else mma_commit(&v_empty[s]);
+            mma_commit(&v_empty[s]);
         }
         if (!ok) *s_abort = 1;
         mma_commit(mma_done);
@@ -906,10 +882,6 @@ __global__ void __maxnreg__(160)
         tc_fence_after();
         tmem_dealloc(tmem, S::tmem_cols);
     }
-    // no CTA of a cluster exits before the others' MMAs are done (their
-    // completions arrive on its empty barriers); every multicast tile has
-    // landed, since each CTA waited for all of them in its loop
-    if (mc > 1) cluster_sync_all();
     if (tree_cta && rt == 0 && threadIdx.x == 0 && *s_bad) report(a.status, CLOVER_ERR_BAD_TREE);
     // every global write below comes after the prerequisite grids complete
     if (in_early) wait_prerequisite_grids();
@@ -1005,37 +977,6 @@ __global__ void __maxnreg__(160)
     if (*s_abort && threadIdx.x == 0) report(a.status, CLOVER_ERR_TIMEOUT);
 }
 
-// Clusters of mc CTAs of this kernel that can be resident at once (0 when
-// clusters of mc cannot be launched), cached per device and context.
-template <int D, int KS, bool PAGED>
-int max_active_clusters(int mc) {
-    static unsigned long long ctx_of[64][5];
-    static int count[64][5];
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64 || mc < 2 || mc > 4) return 0;
-    const unsigned long long ctx = current_context_id();
-    if (ctx != 0 && ctx_of[dev][mc] == ctx) return count[dev][mc];
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(mc, 1, 1);
-    cfg.blockDim = dim3(threads_of<KS>(), 1, 1);
-    cfg.dynamicSmemBytes = TcSmem<D, KS>::alloc;
-    cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeClusterDimension;
-    attr.val.clusterDim.x = mc;
-    attr.val.clusterDim.y = 1;
-    attr.val.clusterDim.z = 1;
-    cfg.attrs = &attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, tree_attn_tc_kernel<D, KS, PAGED>, &cfg) != cudaSuccess) {
-        (void)cudaGetLastError();
-        n = 0;
-    }
-    ctx_of[dev][mc] = ctx;
-    count[dev][mc] = n;
-    return n;
-}
-
 template <int D, int KS, bool PAGED>
 cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     static unsigned long long done[64];
@@ -1044,21 +985,11 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     if (err != cudaSuccess) return err;
     if (a.n_split < 1 || a.n_split > kMaxSplits) return cudaErrorInvalidValue;
     if (a.n_split > 1 && (!a.part_o || !a.counters)) return cudaErrorInvalidValue;
-    // Row tiles of one key range share their K/V tiles in a cluster (2 or 4
-    // of them: a tile's rows split into slices of whole 8-row swizzle atoms)
-    // when every cluster of the grid can be resident at once.
-    a.mc = 1;
-    if (!PAGED && KS == 1 && (a.row_tiles == 2 || a.row_tiles == 4) &&
-        (long long)a.n_split * a.B * a.Hkv <= max_active_clusters<D, KS, PAGED>(a.row_tiles))
-        a.mc = a.row_tiles;
-    const uint32_t box_rows = (uint32_t)(BN / a.mc);
 
     CUtensorMap kc, vc, kn, vn, ks, vs;
     const uint64_t e = 2;
-    bool ok = make_tmap_bf16_3d(&kn, a.k_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1,
-                                box_rows) &&
-              make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1,
-                                box_rows);
+    bool ok = make_tmap_bf16_3d(&kn, a.k_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN) &&
+              make_tmap_bf16_3d(&vn, a.v_new, D, a.Hkv, (uint64_t)a.B * a.T, D * e, (uint64_t)a.Hkv * D * e, 64, 1, BN);
     if (PAGED) {
         // page pools [n_pages * Hkv planes][page_size rows][D]; a paged call
         // never appends, so the append maps are not used
@@ -1072,8 +1003,8 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     } else {
         const uint64_t plane = (uint64_t)a.Lcap * D * e;
         ok = ok &&
-             make_tmap_bf16_3d(&kc, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, box_rows, 1) &&
-             make_tmap_bf16_3d(&vc, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, box_rows, 1) &&
+             make_tmap_bf16_3d(&kc, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, BN, 1) &&
+             make_tmap_bf16_3d(&vc, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, BN, 1) &&
              // the append: T rows of one (sequence, head) plane of the cache
              make_tmap_bf16_3d(&ks, a.k_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, a.T, 1) &&
              make_tmap_bf16_3d(&vs, a.v_cache, D, a.Lcap, (uint64_t)a.B * a.Hkv, D * e, plane, 64, a.T, 1);
@@ -1085,22 +1016,11 @@ cudaError_t launch(AttnArgs a, cudaStream_t stream) {
     cfg.blockDim = dim3(threads_of<KS>(), 1, 1);
     cfg.dynamicSmemBytes = TcSmem<D, KS>::alloc;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[2];
-    unsigned n_attr = 0;
-    if (a.pdl) {
-        attr[n_attr].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[n_attr].val.programmaticStreamSerializationAllowed = 1;
-        ++n_attr;
-    }
-    if (a.mc > 1) {
-        attr[n_attr].id = cudaLaunchAttributeClusterDimension;
-        attr[n_attr].val.clusterDim.x = (unsigned)a.mc;
-        attr[n_attr].val.clusterDim.y = 1;
-        attr[n_attr].val.clusterDim.z = 1;
-        ++n_attr;
-    }
-    cfg.attrs = attr;
-    cfg.numAttrs = n_attr;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = a.pdl ? 1 : 0;
     err = cudaLaunchKernelEx(&cfg, kernel, kc, vc, kn, vn, ks, vs, a);
     if (err != cudaSuccess) return err;
     return cudaGetLastError();
