@@ -280,6 +280,16 @@ clover_status run_attn(const void *q, const void *k_new, const void *v_new, void
     a.pdl = (launch_flags & CLOVER_ATTN_PDL) ? 1 : 0;
     a.cache_early = (a.pdl && (launch_flags & CLOVER_ATTN_CACHE_READY)) ? 1 : 0;
     a.inputs_early = (a.pdl && (launch_flags & CLOVER_ATTN_INPUTS_READY)) ? 1 : 0;
+    // A launch that runs its whole key loop beside the kernels before it is
+    // one of a chain that shares the GPU: one CTA per (sequence, head, row
+    // tile) takes every key, so that no setup and merge of split ranges is
+    // spent (and the workspace is not used).
+    if (p.tc && a.inputs_early) {
+        a.n_split = 1;
+        a.counters = nullptr;
+        a.part_o = nullptr;
+        a.part_ml = nullptr;
+    }
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     return from_cuda(p.tc ? launch_tree_attn_tc(a, st) : launch_tree_attn_fma(a, st));
 }

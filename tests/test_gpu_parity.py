@@ -244,69 +244,100 @@ def test_pdl_chain_reads_inputs_after_the_previous_kernel(cache_ready, graph, cu
 @pytest.mark.parametrize("graph", [False, True])
 def test_pdl_inputs_ready_independent_calls(graph, cuda):
     """CLOVER_ATTN_INPUTS_READY: calls on independent inputs (the statement
-    holds) run their key loops while the previous call finishes; their writes
-    (the shared workspace's slots and counters, the output) still wait for
-    it.  Six calls, three of them into one output buffer: every output equals
-    ordinary launches' bit for bit, the shared buffer holds the last call's."""
+    holds) run their key loops while the previous calls finish; their writes
+    (the output) still wait for them.  Such calls take every key of a head in
+    one CTA, so they are compared with the same calls made one at a time
+    (synchronised): six calls, three of them into one output buffer, every
+    output equal bit for bit, the shared buffer holding the last call's; and
+    every output within the tolerance of the oracle."""
     n = 6
     ws_ = [workloads.get("7b_l2048", T=64, Hq=8, Hkv=8, L=1500 + 211 * i, V=1000, seed=70 + i) for i in range(n)]
-    sets = [to_dev(workloads.make(w, logits=False), cuda) for w in ws_]
+    hosts = [workloads.make(w, logits=False) for w in ws_]
+    sets = [to_dev(h, cuda) for h in hosts]
     need = max(pkg.clover_verify_attn_workspace_size(1, 64, 8, 8, 128, s["Lcap"], torch.bfloat16) for s in sets)
     assert need > 0
     ws = torch.zeros(need, dtype=torch.uint8, device=cuda)
     st = torch.zeros(1, dtype=torch.int32, device=cuda)
 
-    def run(pdl, outs):
+    def run(outs, sync):
         for i, s in enumerate(sets):
             pkg.clover_verify_attn(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"],
-                                   s["parent"], outs[i], workspace=ws, status=st, append=False, pdl=pdl,
-                                   inputs_ready=pdl)
+                                   s["parent"], outs[i], workspace=ws, status=st, append=False, pdl=True,
+                                   inputs_ready=True)
+            if sync:
+                torch.cuda.synchronize()
 
     ref = [torch.empty_like(s["q"]) for s in sets]
-    run(False, ref)
+    run(ref, True)
     shared = torch.full_like(sets[0]["q"], float("nan"))
     outs = [torch.full_like(s["q"], float("nan")) for s in sets]
     outs[1] = outs[3] = outs[5] = shared
     if graph:
         stream = torch.cuda.Stream()
         with torch.cuda.stream(stream):
-            run(True, outs)
+            run(outs, False)
         torch.cuda.synchronize()
         for o in outs:
             o.fill_(float("nan"))
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            run(True, outs)
+            run(outs, False)
         g.replay()
     else:
-        run(True, outs)
+        run(outs, False)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     for i in (0, 2, 4):
         assert torch.equal(outs[i].view(torch.int16), ref[i].view(torch.int16)), f"call {i}"
     assert torch.equal(shared.view(torch.int16), ref[5].view(torch.int16))
+    for i, h in enumerate(hosts):
+        want = oracle.tree_attention(h["q"], h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["cache_len"],
+                                     h["parent"])
+        assert (ref[i].double().cpu() - want).abs().max().item() <= ATOL[torch.bfloat16], i
 
 
 @pytest.mark.parametrize("mode", ["pdl", "cache_ready", "inputs_ready"])
 @pytest.mark.parametrize("schedule", ["commit", "fused"])
 def test_step_attention_launch_modes(mode, schedule, cuda):
-    """VerifyStep with the attention launched as a programmatic dependent:
-    three steps in a row on independent input sets (the statement holds), each
-    bit-equal to an ordinary step's outputs and matching the oracle."""
+    """VerifyStep with the attention launched as a programmatic dependent, on
+    three independent input sets (the statement holds): steps made one at a
+    time match the oracle and, with pdl and cache_ready (the same split plan),
+    an ordinary step's outputs bit for bit; three steps queued back to back
+    (each its own VerifyStep, so that each keeps its outputs) give the same
+    outputs as the steps made one at a time."""
     hosts = [workloads.make(workloads.get("7b_l2048", T=64, Hq=8, Hkv=8, L=1100 + 300 * i, V=3000, seed=40 + i))
              for i in range(3)]
     ref = [run_gpu(to_dev(h, cuda), schedule=schedule) for h in hosts]
     ref_out = [r.out.clone() for r in ref]
-    sets = [to_dev(h, cuda) for h in hosts]
-    B, T, Hq, D = sets[0]["q"].shape
-    step = pkg.VerifyStep(B, T, Hq, 8, D, max(s["Lcap"] for s in sets), 3000, torch.bfloat16, device=cuda,
-                          schedule=schedule, attn_launch=mode)
-    for i, t in enumerate(sets):
+    B, T, Hq, D = ref_out[0].shape
+    Lcap = max(h["Lcap"] for h in hosts)
+
+    def new_step():
+        return pkg.VerifyStep(B, T, Hq, 8, D, Lcap, 3000, torch.bfloat16, device=cuda, schedule=schedule,
+                              attn_launch=mode)
+
+    def run(step, t):
         step.run(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
                  t["cand"], t["logits"])
+
+    alone = []
+    for i, h in enumerate(hosts):
+        t = to_dev(h, cuda)
+        step = new_step()
+        run(step, t)
         torch.cuda.synchronize()
-        assert torch.equal(step.out.view(torch.int16), ref_out[i].view(torch.int16)), i
-        compare_full(hosts[i], step, t)
+        if mode != "inputs_ready":
+            assert torch.equal(step.out.view(torch.int16), ref_out[i].view(torch.int16)), i
+        compare_full(h, step, t)
+        alone.append(step.out.clone())
+    sets = [to_dev(h, cuda) for h in hosts]
+    steps = [new_step() for _ in hosts]
+    for step, t in zip(steps, sets):
+        run(step, t)
+    torch.cuda.synchronize()
+    for i, (h, step, t) in enumerate(zip(hosts, steps, sets)):
+        assert torch.equal(step.out.view(torch.int16), alone[i].view(torch.int16)), i
+        compare_full(h, step, t)
 
 
 # ---------------------------------------------------------------------------
