@@ -166,7 +166,7 @@ class ClockSampler:
         except Exception:
             pass
         self.cmd = ["nvidia-smi", f"--query-gpu={','.join(self.FIELDS)}", "--format=csv,noheader,nounits",
-                    "-lms", "100", "-i", target]
+                    "-lms", "20", "-i", target]
 
     def start(self):
         try:
@@ -207,7 +207,7 @@ class ClockSampler:
         if not inside and rows:
             # region shorter than the sampling period: nearest samples around it
             inside = sorted(rows, key=lambda r: abs(r[0] - (self.t0 or 0)))[:3]
-            note = "timed region shorter than the 100 ms sampling period: nearest samples"
+            note = "timed region shorter than the 20 ms sampling period: nearest samples"
         def num(x):
             try:
                 return float(x)
@@ -423,7 +423,13 @@ def run_gpu_arm(args, world, rank, local, dist):
                      "frac_ordinary": a_bytes / (us["tree_attn_ordinary"] * 1e-6) / 1e9 / hbm,
                      "frac_of_8TBs": achieved / 8000.0,
                      "flops_per_launch": attn_flops_per_launch(w, lengths),
-                     "timing": timing_source["tree_attn"]},
+                     "timing": timing_source["tree_attn"],
+                     # the whole step against HBM: the attention's bytes and
+                     # the logits read by the argmax (the commit's few rows,
+                     # under 0.3 % here, left out) per ms_per_step
+                     "step": {"bytes": a_bytes + am_bytes,
+                              "gbs": (a_bytes + am_bytes) / (ms * 1e-3) / 1e9,
+                              "frac": (a_bytes + am_bytes) / (ms * 1e-3) / 1e9 / hbm}},
         "kernels": {"tree_attn_us": us["tree_attn"], "accept_us": us["accept"], "kv_commit_us": us["kv_commit"],
                     "accept_rule": args.accept,
                     "accept_bytes_per_launch": am_bytes,
@@ -970,7 +976,7 @@ def run_reference_draft(args, world, threads, budget_s):
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--steps", type=int, default=40000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
@@ -1005,6 +1011,8 @@ def main(argv=None):
             print(json.dumps(line), flush=True)
         return 0
 
+    if args.page_size and args.schedule == "fused":
+        args.schedule = "commit"             # the paged calls take the commit schedule
     dist = dist_init(world, "nccl" if torch.cuda.is_available() else "gloo")
     if args.draft:
         line, inputs = run_draft_arm(args, world, rank, local, dist)
