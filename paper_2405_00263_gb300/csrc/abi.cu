@@ -15,7 +15,7 @@ int tc_row_tile();
 int tc_max_splits();
 cudaError_t launch_tree_attn_fma(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream);
-void accept_plan(int B, int T, int V, int dtype, bool typical, int *n_chunks, int *chunk);
+void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk);
 size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype);
 cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,

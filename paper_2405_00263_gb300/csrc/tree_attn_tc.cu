@@ -66,6 +66,7 @@ constexpr int BM = 128;                 // query rows per CTA (MMA M)
 constexpr int BN = 128;                 // keys per tile (the N of the S MMA)
 constexpr int kMinPage = 16;             // smallest page of a paged cache (rows)
 constexpr int kMaxBoxes = BN / kMinPage; // TMA boxes of one paged cache tile
+static_assert(kMaxBoxes * 2 <= 32, "a paged tile's boxes and column blocks go one to a producer lane");
 constexpr int kPageSmem = 512;           // page ids of a split staged in shared memory
 constexpr int kKProducerWarp = 4;
 constexpr int kMmaWarp = 5;
@@ -414,40 +415,47 @@ __global__ void __maxnreg__(160)
     constexpr bool paged = PAGED;
     const int box = paged ? min(a.page_size, BN) : BN;
     const int first_page = kbeg >> a.page_shift;     // the split's first page (paged)
-    // staged: the split's first kPageSmem page ids are in s_pages (after the
-    // setup barrier); later ones, and all of them before it, come from the table
-    auto tile_pages = [&](int j, int (&pg)[kMaxBoxes], bool staged) {
-        if (!paged || j == tree_j) return;
-        const int key0 = kbeg + (j - tree_shift) * BN;
-        for (int r = 0, x = 0; r < BN; r += box, ++x) {
-            const int slot = key0 + r;
-            const int pi = (slot >> a.page_shift) - first_page;
-            pg[x] = slot >= kend ? 0 : (staged && pi < kPageSmem) ? s_pages[pi] : cache_page(a, b, slot);
-        }
+    // A paged cache tile is read by the whole producer warp at once: lane l
+    // takes box l / DH (rows [box (l / DH), +box) of the tile) in 64-column
+    // block l % DH, with its own page id (at most 8 boxes x 2 blocks).  The
+    // page id of a lane's box of tile j, looked up before the producer waits
+    // for the stage; staged: the split's first kPageSmem page ids are in
+    // s_pages (after the setup barrier); later ones, and all of them before
+    // it, come from the table.
+    const int n_box_issues = paged ? (BN / box) * S::DH : 0;
+    auto lane_page = [&](int j, bool staged) -> int {
+        if (!paged || j == tree_j || lane >= n_box_issues) return 0;
+        const int slot = kbeg + (j - tree_shift) * BN + (lane / S::DH) * box;
+        const int pi = (slot >> a.page_shift) - first_page;
+        return slot >= kend ? 0 : (staged && pi < kPageSmem) ? s_pages[pi] : cache_page(a, b, slot);
     };
     // tile j of K (is_v == false) or V into ring stage `dst`: a cache tile (an
-    // evict-first read) or, past the cache tiles, the tree tile
+    // evict-first read) or the tree tile.  Dense: run by the producer's lane 0;
+    // paged: by all its lanes together (lane 0 alone for the tree tile).
     const uint64_t pol = l2_policy_evict_first();
-    auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar, const int (&pg)[kMaxBoxes]) {
-        mbar_arrive_expect_tx(bar, S::kv_bytes);
+    auto issue_tile = [&](int j, bool is_v, uint8_t *dst, uint64_t *bar, int pg) {
         const CUtensorMap *cache_map = is_v ? &tm_vc : &tm_kc;
         const CUtensorMap *new_map = is_v ? &tm_vn : &tm_kn;
         if (j != tree_j && paged) {
-            const int key0 = kbeg + (j - tree_shift) * BN;
-            for (int r = 0, x = 0; r < BN; r += box, ++x) {
-                const int row = (key0 + r) & (a.page_size - 1);
+            if (lane == 0) mbar_arrive_expect_tx(bar, S::kv_bytes);
+            __syncwarp();
+            if (lane < n_box_issues) {
+                const int r = (lane / S::DH) * box;
+                const int dh = lane % S::DH;
+                const int row = (kbeg + (j - tree_shift) * BN + r) & (a.page_size - 1);
+                tma_load_3d_hint(dst + dh * BN * 128 + r * 128, cache_map, bar, dh * 64, row, pg * a.Hkv + g, pol);
+            }
+        } else if (lane == 0) {
+            mbar_arrive_expect_tx(bar, S::kv_bytes);
+            if (j != tree_j) {
 #pragma unroll
                 for (int dh = 0; dh < S::DH; ++dh)
-                    tma_load_3d_hint(dst + dh * BN * 128 + r * 128, cache_map, bar, dh * 64, row, pg[x] * a.Hkv + g,
+                    tma_load_3d_hint(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + (j - tree_shift) * BN, bg,
                                      pol);
+            } else {
+#pragma unroll
+                for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, new_map, bar, dh * 64, g, b * a.T);
             }
-        } else if (j != tree_j) {
-#pragma unroll
-            for (int dh = 0; dh < S::DH; ++dh)
-                tma_load_3d_hint(dst + dh * BN * 128, cache_map, bar, dh * 64, kbeg + (j - tree_shift) * BN, bg, pol);
-        } else {
-#pragma unroll
-            for (int dh = 0; dh < S::DH; ++dh) tma_load_3d(dst + dh * BN * 128, new_map, bar, dh * 64, g, b * a.T);
         }
     };
     // The first ring stages start empty: their tiles are issued without a
@@ -459,9 +467,9 @@ __global__ void __maxnreg__(160)
         uint8_t *ring = is_v ? sV : sK;
         uint64_t *full = is_v ? v_full : k_full;
         const int upto = min(ns, n_tiles);
-        int pg[NSmax][kMaxBoxes];
+        int pg[NSmax];
         for (int j = 0; j < upto; ++j)
-            if ((phase == 0) == (split_wait && j != tree_j)) tile_pages(j, pg[j], false);
+            if ((phase == 0) == (split_wait && j != tree_j)) pg[j] = lane_page(j, false);
         for (int j = 0; j < upto; ++j)
             if ((phase == 0) == (split_wait && j != tree_j)) issue_tile(j, is_v, ring + j * S::kv_bytes, &full[j], pg[j]);
         if (phase == 1) issued = upto;
@@ -494,7 +502,7 @@ __global__ void __maxnreg__(160)
     // complete (after an L2 prefetch of the Q rows); phase 1 stages the
     // split's page ids (paged), waits for those grids and loads Q (with
     // cache_early), and issues the rest of the first stages.
-    const bool producer = (warp == kVProducerWarp || warp == kKProducerWarp) && lane == 0;
+    const bool producer = (warp == kVProducerWarp || warp == kKProducerWarp) && (paged || lane == 0);
     const bool prod_v = warp == kVProducerWarp;
     int k_issued = 0, v_issued = 0;
 #pragma unroll 1
@@ -538,7 +546,8 @@ __global__ void __maxnreg__(160)
     }
 
     // ----------------------------------------------------- TMA producer warps
-    if ((warp == kVProducerWarp || warp == kKProducerWarp) && lane == 0) {
+    // (lane 0; with a paged cache the whole warp, its waits and exits uniform)
+    if (producer) {
         const bool is_v = warp == kVProducerWarp;
         const int ns = is_v ? NSV : NSK;
         uint8_t *ring = is_v ? sV : sK;
@@ -556,13 +565,14 @@ __global__ void __maxnreg__(160)
         for (int j = issued; j < n_tiles; ++j) {
             const int s = j % ns;
             if (appender && !appended && j == tree_j + ns) append();
-            int pg[kMaxBoxes];
-            tile_pages(j, pg, true);
-            if (!mbar_wait(&empty[s], ((j / ns) - 1) & 1, kWaitNs)) {
+            const int pg = lane_page(j, true);
+            bool ok = mbar_wait(&empty[s], ((j / ns) - 1) & 1, kWaitNs);
+            if (paged) ok = __all_sync(0xffffffffu, ok);
+            if (!ok) {
                 *s_abort = 1;
                 break;
             }
-            if (*s_abort) break;
+            if (paged ? __any_sync(0xffffffffu, *s_abort != 0) : *s_abort != 0) break;
             issue_tile(j, is_v, ring + s * S::kv_bytes, &full[s], pg);
             issued = j + 1;
         }
