@@ -48,9 +48,9 @@ STEP_PASSES = 4          # passes over the input sets in one captured graph of s
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 KERNEL_SOURCES = {
-    "tree_attn": ["tree_attn_tc.cu", "tc_ptx.cuh", "tmap_host.cuh", "common.cuh", "abi.cu"],
-    "accept": ["accept.cu", "common.cuh"],
-    "kv_compact": ["kv_compact.cu", "common.cuh"],
+    "tree_attn": ["tree_attn_tc.cu", "tc_ptx.cuh", "tmap_host.cuh", "common.cuh", "ctx_host.cuh", "abi.cu"],
+    "accept": ["accept.cu", "common.cuh", "ctx_host.cuh"],
+    "kv_compact": ["kv_compact.cu", "common.cuh", "ctx_host.cuh"],
 }
 
 
