@@ -25,8 +25,11 @@
 // 32w.. and runs the softmax, rescales and the epilogue of those lanes (the
 // lanes warp w may access); warp 4 issues the TMA loads of the K tiles (its
 // own ring); warp 6 those of the V tiles; warp 5 allocates TMEM and issues the
-// MMAs from one thread.  The cache tiles are read with an L2 evict-first
-// policy: they are read once, and must not push out of L2 what is reused.
+// MMAs from one thread.  A full 128-row tile (KS = 1) adds warps 7-10 (352
+// threads): a second softmax warp per lane quadrant, the two taking 64 keys
+// of a tile each and sharing one reference max through shared memory.  The
+// cache tiles are read with an L2 evict-first policy: they are read once, and
+// must not push out of L2 what is reused.
 // The split that owns the last cache range also takes the tile of T tree keys
 // (read from k_new/v_new) under the ancestor bitmask, as its first tile; its
 // producers also append the tree keys and values to the cache when asked, by
