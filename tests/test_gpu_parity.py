@@ -49,6 +49,18 @@ def test_small_step_matches_oracle(case, cuda):
     compare_full(host, step, t)
 
 
+@pytest.mark.parametrize("case", sorted(c for c in SMALL if not c.startswith("f32")))
+def test_small_step_inputs_ready_plan(case, cuda):
+    """The inputs-ready launch plan (one CTA takes every key of a head tile, no
+    split) on every bf16 shape, in the bench's fused schedule: the whole step
+    against the oracle."""
+    name, over = SMALL[case]
+    host = workloads.make(workloads.get(name, **over))
+    t = to_dev(host, cuda)
+    step = run_gpu(t, schedule="fused", attn_launch="inputs_ready")
+    compare_full(host, step, t)
+
+
 def test_scale_argument(cuda):
     w = workloads.get("tiny_f32", L=300)
     host = workloads.make(w)
