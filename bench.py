@@ -352,8 +352,8 @@ def run_gpu_arm(args, world, rank, local, dist):
     timing_source = {"tree_attn": f"back-to-back attention launches ({step.attn_launch} launch) over the {n_sets} "
                                   "rotating input sets, four passes in one CUDA graph, events around the replays, "
                                   "after the timed region",
-                     "accept": "launched alone after an L2 flush, events on the launching stream",
-                     "kv_commit": "launched alone after an L2 flush, events on the launching stream"}
+                     "accept": "launched alone after an L2 flush (a read of twice the L2), device time: CUDA graphs of (flush, call) pairs less graphs of the flushes alone",
+                     "kv_commit": "launched alone after an L2 flush (a read of twice the L2), device time: CUDA graphs of (flush, call) pairs less graphs of the flushes alone"}
     us = {"tree_attn": attn_launch_us(step, sets, stream, device, args, mode=step.attn_launch)}
     us["tree_attn_ordinary"] = (us["tree_attn"] if step.attn_launch == "ordinary"
                                 else attn_launch_us(step, sets, stream, device, args, mode="ordinary"))
@@ -505,22 +505,40 @@ def attn_launch_us(step, sets, stream, device, args, mode: str, launches: int = 
     return a.elapsed_time(b) * 1e3 / (reps * passes * len(sets))
 
 
-def isolated_us(call, n, stream, flush) -> float:
-    """Mean event-timed duration of call(i), i < n, each launched alone on
-    ``stream`` right after a read of ``flush`` (twice the L2: the L2 then holds
-    only clean lines of it, so the call pays no write-back of a flush)."""
-    times = []
+def isolated_us(call, n, stream, flush, reps: int = 10) -> float:
+    """Mean duration of call(i), i < n, each launched alone on ``stream`` right
+    after a read of ``flush`` (twice the L2: the L2 then holds only clean lines
+    of it, so the call pays no write-back of a flush).  Device time only: one
+    CUDA graph holds the n (flush, call) pairs and another the n flushes alone;
+    both are replayed ``reps`` times between CUDA events, and the difference is
+    the calls' time (with no host launch latency in it)."""
     with torch.cuda.stream(stream):
-        for i in range(n + 2):
+        for i in range(n):                  # eager first: per-kernel attributes outside the capture
+            call(i)
+    stream.synchronize()
+    g_pairs, g_flush = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_pairs, stream=stream):
+        for i in range(n):
             torch.amax(flush)
+            call(i)
+    with torch.cuda.graph(g_flush, stream=stream):
+        for i in range(n):
+            torch.amax(flush)
+
+    def timed(g):
+        with torch.cuda.stream(stream):
+            g.replay()
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record(stream)
-            call(i)
+            for _ in range(reps):
+                g.replay()
             b.record(stream)
-            b.synchronize()
-            if i >= 2:
-                times.append(a.elapsed_time(b) * 1e3)
-    return statistics.mean(times)
+        b.synchronize()
+        return a.elapsed_time(b) * 1e3
+
+    t_pairs, t_flush = timed(g_pairs), timed(g_flush)
+    del g_pairs, g_flush
+    return (t_pairs - t_flush) / (n * reps)
 
 
 def accept_kernel_us(pkg, w, sets, stream, device, rule, args, flush) -> float:
@@ -659,7 +677,7 @@ def run_draft_arm(args, world, rank, local, dist):
                      "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)" if peak_kind == "measured"
                      else "fallback 6.8 TB/s", "traffic": None, "bytes_per_launch": lm_bytes,
                      "launch_us": lm_us, "flops_per_launch": 2 * R * V * H,
-                     "timing": "launched alone after an L2 flush by a large read, events on the launching stream"},
+                     "timing": "launched alone after an L2 flush by a large read, device time: CUDA graphs of (flush, call) pairs less graphs of the flushes alone"},
         "kernels": {"lm_head_us": lm_us, "topk_us": topk_us,
                     "topk_gbs": R * V * 4 / (topk_us * 1e-6) / 1e9},
         "gpu_launches": 6 * args.steps,

@@ -581,8 +581,12 @@ __global__ void __maxnreg__(56) accept_kernel(const AcceptArgs a) {
     accept_body<T, false>(a);
 }
 
+// The typical kernel is held to 64 registers: four of its 256-thread CTAs an SM
+// (65,536 registers), so that the 512 CTAs of a 7B-vocabulary step (64 rows x
+// 8 chunks) are all resident at once on 152 SMs; at 71 registers three fit,
+// and the grid took two waves.
 template <typename T>
-__global__ void __launch_bounds__(kThreads) accept_typical_kernel(const AcceptArgs a) {
+__global__ void __maxnreg__(64) accept_typical_kernel(const AcceptArgs a) {
     accept_body<T, true>(a);
 }
 
