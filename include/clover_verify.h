@@ -210,12 +210,14 @@ CLOVER_API clover_status clover_verify_attn(const void *q, const void *k_new, co
  *     earlier.  Neither statement is checked: a kernel that does write one of
  *     these inputs while this call reads it gives unspecified results.  Such a
  *     launch is planned for a chain of them, several sharing the GPU at once:
- *     one CTA takes every key of a (sequence, KV head, 128-row tile), with no
- *     split of the keys and no use of the workspace.  Fewer, longer CTAs then
- *     spend less of the GPU on setup and on merging splits, and the chain
- *     keeps the memory busy; a single such call on its own takes longer than
- *     an ordinary one.  Its results may differ from an ordinary launch's in
- *     the last bits (the key ranges are summed in another order); they do not
+ *     it takes about a fifth of the SMs' worth of CTAs, each over as long a
+ *     key range as that allows; with at least that many (sequence, KV head,
+ *     128-row tile) groups, one CTA takes every key of a group, with no split
+ *     of the keys and no use of the workspace.  Fewer, longer CTAs then spend
+ *     less of the GPU on setup and on merging splits, and the chain keeps the
+ *     memory busy; a single such call on its own takes longer than an
+ *     ordinary one.  Its results may differ from an ordinary launch's in the
+ *     last bits (the key ranges are summed in another order); they do not
  *     depend on what runs beside it.
  * The fp32 (CUDA-core) kernel is launched the ordinary way whatever the launch
  * flags say.  Other flag bits: CLOVER_ERR_INVALID_ARG.

@@ -15,7 +15,7 @@ int tc_row_tile();
 int tc_max_splits();
 cudaError_t launch_tree_attn_fma(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream);
-void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk);
+void accept_plan(int B, int T, int V, int dtype, bool typical, int resident, int *n_chunks, int *chunk);
 size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype);
 cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
@@ -41,6 +41,10 @@ constexpr int kSms = 152;                  // SMs of a GB300 (planning constant;
 constexpr int kTargetAttnCtas = 2 * kSms;  // FMA path: two resident CTAs per SM
 constexpr int kMinKeysPerSplit = 256;
 constexpr int kMaxSplits = 64;
+
+// CTAs an inputs-ready attention launch aims for: about a fifth of the SMs
+// (see run_attn).
+constexpr long kChainCtas = kSms / 5;
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -281,14 +285,20 @@ clover_status run_attn(const void *q, const void *k_new, const void *v_new, void
     a.cache_early = (a.pdl && (launch_flags & CLOVER_ATTN_CACHE_READY)) ? 1 : 0;
     a.inputs_early = (a.pdl && (launch_flags & CLOVER_ATTN_INPUTS_READY)) ? 1 : 0;
     // A launch that runs its whole key loop beside the kernels before it is
-    // one of a chain that shares the GPU: one CTA per (sequence, head, row
-    // tile) takes every key, so that no setup and merge of split ranges is
-    // spent (and the workspace is not used).
+    // one of a chain that shares the GPU: it takes about kChainCtas CTAs (a
+    // fifth of the SMs), so that about five launches run at once, each CTA
+    // over as long a key range as that allows: one CTA per (sequence, head,
+    // row tile) when there are that many, which spends no setup and no merge
+    // on split ranges (and does not use the workspace).
     if (p.tc && a.inputs_early) {
-        a.n_split = 1;
-        a.counters = nullptr;
-        a.part_o = nullptr;
-        a.part_ml = nullptr;
+        const long base = (long)B * Hkv * p.row_tiles;
+        const long want = (kChainCtas + base - 1) / base;
+        a.n_split = (int)(want < p.n_split ? want : p.n_split);
+        if (a.n_split == 1) {
+            a.counters = nullptr;
+            a.part_o = nullptr;
+            a.part_ml = nullptr;
+        }
     }
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     return from_cuda(p.tc ? launch_tree_attn_tc(a, st) : launch_tree_attn_fma(a, st));

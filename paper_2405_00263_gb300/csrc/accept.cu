@@ -7,8 +7,9 @@
 // token equals its parent's greedy token; the accepted path is walked from the
 // root and its length is the paper's tokens/step (Section 4.1).
 //
-// Grid: one CTA per (logit row, 32 KB vocabulary chunk).  Each CTA reduces its
-// chunk with 16-byte loads (eight in flight per thread) to a packed 64-bit key
+// Grid: one CTA per (logit row, vocabulary chunk of one to four 32 KB rounds).
+// Each CTA reduces its chunk with 16-byte loads (eight in flight per thread a
+// round) to a packed 64-bit key
 // (order-preserving value bits in the high word, bit-inverted index in the low
 // word) so that one unsigned max gives "largest value, then smallest index",
 // and folds it into the row's key with a 64-bit atomic max.  A per-sequence
@@ -27,6 +28,8 @@
 // sums), decides every edge p(cand) > min(eps, delta e^-H) in the log2
 // domain, and walks the longest accepted path (ties: the smallest-index child
 // at every step).
+#include <algorithm>
+
 #include "common.cuh"
 
 namespace clover {
@@ -83,7 +86,7 @@ __device__ __forceinline__ int unit_first(const uint4 &w, float v, float) {
 }
 
 // Vector body: 16-byte units [0, n_units) of the row from element `first`,
-// n_units <= kThreads * kUnits (a chunk is one round).  A thread issues its
+// n_units <= kThreads * kUnits (one round).  A thread issues its
 // kUnits independent loads (units tid + k*kThreads) into w, takes the maximum
 // over them, and only then looks for its first position.
 template <typename T>
@@ -508,7 +511,12 @@ __device__ __forceinline__ void accept_body(const AcceptArgs &a) {
         head = min(head, hi - lo);
         n_units = (hi - lo - head) / E;
         scan_scalar<T>(rowp, lo, lo + head, best);
-        scan_vector<T>(rowp, lo + head, n_units, best, w);
+        // rounds of the vector body (the typical rule's plan has one, whose
+        // units stay in w for its sums)
+        constexpr int kRound = kThreads * kUnits;
+        const int nu = (int)n_units;           // at most four rounds
+        for (int u0 = 0; u0 < nu; u0 += kRound)
+            scan_vector<T>(rowp, lo + head + (int64_t)u0 * E, min(nu - u0, kRound), best, w);
         scan_scalar<T>(rowp, lo + head + n_units * E, hi, best);
     }
 
@@ -592,15 +600,30 @@ __global__ void __maxnreg__(64) accept_typical_kernel(const AcceptArgs a) {
 
 }  // namespace
 
-// Vocabulary chunk per CTA: one round of kUnits 16-byte loads per thread
-// (32 KB of bf16 or fp32 logits).
-void accept_plan(int B, int T, int V, int dtype, int *n_chunks, int *chunk) {
-    (void)B;
-    (void)T;
+// Vocabulary chunk per CTA: rounds of kUnits 16-byte loads per thread (32 KB
+// of bf16 or fp32 logits a round).  The typical rule keeps its one round in
+// registers for the sums.  The greedy rule takes as many rounds (up to four)
+// as bring the grid within `resident` CTAs, what the GPU holds at once, so
+// that a call with many rows (a 128-node tree, a batch of sequences) runs in
+// one wave instead of two or more; a grid that fits already keeps one round.
+void accept_plan(int B, int T, int V, int dtype, bool typical, int resident, int *n_chunks, int *chunk) {
+    constexpr int kMaxRounds = 4;
     const int elems = 16 / (dtype == CLOVER_F32 ? 4 : 2);
-    const int c = kThreads * kUnits * elems;
-    *chunk = c;
-    *n_chunks = (V + c - 1) / c;
+    const int round = kThreads * kUnits * elems;
+    const long long one_round = (long long)B * T * ((V + round - 1) / round);
+    const long long cap = resident > 0 ? resident : one_round;
+    const int rounds = typical ? 1 : (int)std::min<long long>(kMaxRounds, std::max<long long>(1, (one_round + cap - 1) / cap));
+    *chunk = round * rounds;
+    *n_chunks = (V + *chunk - 1) / *chunk;
+}
+
+// CTAs of the greedy accept kernel the current device holds at once: four a
+// multiprocessor (256 threads at 56 registers).
+static int greedy_resident_ctas() {
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return 0;
+    return 4 * sms;
 }
 
 // Keys and counters, then (typical acceptance) the 16-byte aligned chunk sums
@@ -618,7 +641,7 @@ size_t accept_workspace_bytes(int B, int T, int V, int dtype) {
 
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype) {
     int n_chunks, chunk;
-    accept_plan(B, T, V, dtype, &n_chunks, &chunk);
+    accept_plan(B, T, V, dtype, true, 0, &n_chunks, &chunk);
     return accept_sums_offset(B, T) + sizeof(float4) * (size_t)B * T * n_chunks + sizeof(float) * (size_t)B * T;
 }
 
@@ -648,7 +671,7 @@ cudaError_t launch_accept_call(const AcceptCall &c, cudaStream_t stream) {
     a.B = c.B;
     a.T = c.T;
     a.V = c.V;
-    accept_plan(c.B, c.T, c.V, c.dtype, &a.n_chunks, &a.chunk);
+    accept_plan(c.B, c.T, c.V, c.dtype, c.typical, c.typical ? 0 : greedy_resident_ctas(), &a.n_chunks, &a.chunk);
     a.argmax_out = c.argmax_out;
     a.path_out = c.path_out;
     a.accept_len = c.accept_len;

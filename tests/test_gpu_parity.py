@@ -90,17 +90,22 @@ FULL = ["7b_l2048", "7b_l4096", "7b_l16384", "7b_batched", "100b_gqa", "paper_t4
         "7b_t128"]
 
 
-@pytest.mark.parametrize("schedule", ["commit", "fused"])
+@pytest.mark.parametrize("schedule", ["commit", "fused", "fused_inputs_ready"])
 @pytest.mark.parametrize("name", FULL)
 def test_full_size_workloads(name, schedule, cuda):
     """The workloads at their full sizes: attention on sampled rows (the
     oracle computes them one by one), argmax / walk / indices everywhere, the
-    tree slots of the cache everywhere, and the committed prefix untouched."""
+    tree slots of the cache everywhere, and the committed prefix untouched.
+    "fused_inputs_ready" is the bench's step: the fused schedule with the
+    attention launched inputs-ready (one CTA per head tile)."""
     w = workloads.get(name)
     t = workloads.make(w, device=cuda)
     host = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in t.items()}
     kc0, vc0 = t["k_cache"].clone(), t["v_cache"].clone()
-    step = run_gpu(t, schedule=schedule)
+    if schedule == "fused_inputs_ready":
+        step = run_gpu(t, schedule="fused", attn_launch="inputs_ready")
+    else:
+        step = run_gpu(t, schedule=schedule)
     assert step.device_status() == 0
 
     B, T, Hq, D = w.B, w.T, w.Hq, w.D
