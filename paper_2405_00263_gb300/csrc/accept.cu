@@ -140,21 +140,33 @@ __device__ __forceinline__ float lg2_approx(float x) {
 // fp32), which also turns the -inf logits (p = 0) into zero terms.
 struct ExpSums {
     float s = 0.f, u = 0.f;
+    float2 s2 = make_float2(0.f, 0.f), u2 = make_float2(0.f, 0.f);   // two lanes of sums, folded in at the end
     __device__ __forceinline__ void add(float x, float ys, float my) {
         const float t = fmaxf(fmaf(x, ys, -my), -256.f);
         const float e = ex2_approx(t);
         s += e;
         u = fmaf(e, t, u);
     }
+    // two terms at once: the exponent arguments and both sums as packed f32x2
+    // operations (each lane rounded as the scalar form would be)
+    __device__ __forceinline__ void add2(float x0, float x1, float2 ys2, float2 nmy2) {
+        float2 t = __ffma2_rn(make_float2(x0, x1), ys2, nmy2);
+        t.x = fmaxf(t.x, -256.f);
+        t.y = fmaxf(t.y, -256.f);
+        const float2 e = make_float2(ex2_approx(t.x), ex2_approx(t.y));
+        s2 = __fadd2_rn(s2, e);
+        u2 = __ffma2_rn(e, t, u2);
+    }
+    __device__ __forceinline__ float sum_s() const { return s + (s2.x + s2.y); }
+    __device__ __forceinline__ float sum_u() const { return u + (u2.x + u2.y); }
 };
 
 __device__ __forceinline__ void unit_sums(const uint4 &w, __nv_bfloat16, float ys, float my, ExpSums &acc) {
     const uint32_t x[4] = {w.x, w.y, w.z, w.w};
+    const float2 ys2 = make_float2(ys, ys), nmy2 = make_float2(-my, -my);
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        acc.add(__uint_as_float(x[k] << 16), ys, my);
-        acc.add(__uint_as_float(x[k] & 0xFFFF0000u), ys, my);
-    }
+    for (int k = 0; k < 4; ++k)
+        acc.add2(__uint_as_float(x[k] << 16), __uint_as_float(x[k] & 0xFFFF0000u), ys2, nmy2);
 }
 __device__ __forceinline__ void unit_sums(const uint4 &w, float, float ys, float my, ExpSums &acc) {
     acc.add(__uint_as_float(w.x), ys, my);
@@ -286,8 +298,20 @@ __device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, co
             ++len;
         }
     } else {
+        // ancestor masks by pointer jumping: two nodes a lane and 6 rounds for
+        // trees of up to 64 nodes (a sixth of the shuffles of the general
+        // four-node form)
         uint64_t anc[kNodesPerLane][kMaskWords];
-        tree_masks_jump<kNodesPerLane>(tr.p, Tn, anc);
+        if (Tn <= 64) {
+            tree_masks_jump<2>(*reinterpret_cast<const int(*)[2]>(&tr.p[0]), Tn,
+                               *reinterpret_cast<uint64_t(*)[2][kMaskWords]>(&anc[0]));
+#pragma unroll
+            for (int k = 2; k < kNodesPerLane; ++k)
+#pragma unroll
+                for (int w = 0; w < kMaskWords; ++w) anc[k][w] = 0ull;
+        } else {
+            tree_masks_jump<kNodesPerLane>(tr.p, Tn, anc);
+        }
         uint64_t acc[kMaskWords];                 // accepted edges (node bits), the root included
 #pragma unroll
         for (int k = 0; k < kNodesPerLane; ++k) {
@@ -538,7 +562,7 @@ __device__ __forceinline__ void accept_body(const AcceptArgs &a) {
             if (threadIdx.x + (int64_t)k * kThreads < n_units) unit_sums(w[k], T(), a.y_scale, my, acc);
         for (int64_t v = lo + threadIdx.x; v < lo + head; v += kThreads) acc.add(to_float(rowp[v]), a.y_scale, my);
         for (int64_t v = t0 + threadIdx.x; v < hi; v += kThreads) acc.add(to_float(rowp[v]), a.y_scale, my);
-        float3 st = make_float3(my, acc.s, acc.u);
+        float3 st = make_float3(my, acc.sum_s(), acc.sum_u());
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) {
             const float3 o = make_float3(__shfl_xor_sync(0xffffffffu, st.x, off), __shfl_xor_sync(0xffffffffu, st.y, off),
