@@ -278,7 +278,7 @@ def run_gpu_arm(args, world, rank, local, dist):
     step = pkg.VerifyStep(w.B, w.T, w.Hq, w.Hkv, w.D, Lcap, w.V, w.torch_dtype, device=device,
                           accept=args.accept, temperature=args.temperature, epsilon=args.epsilon,
                           delta=args.delta, schedule=args.schedule, page_size=args.page_size or None,
-                          attn_launch="ordinary" if args.page_size else args.attn_launch)
+                          attn_launch=args.attn_launch)
     stream = torch.cuda.Stream(device)
 
     def launch(s):
@@ -479,7 +479,7 @@ def attn_launch_us(step, sets, stream, device, args, mode: str, launches: int = 
         if args.page_size:
             pkg.clover_verify_attn_paged(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"],
                                          s["block_table"], s["cache_len"], s["parent"], step.out,
-                                         workspace=step.ws_attn, status=step.status, stream=stream)
+                                         workspace=step.ws_attn, status=step.status, stream=stream, **kw)
         else:
             pkg.clover_verify_attn(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"],
                                    s["parent"], step.out, workspace=step.ws_attn, status=step.status,
@@ -1011,7 +1011,7 @@ def main(argv=None):
                     help="attention launch: ordinary, or a programmatic dependent of the kernel before it, with the "
                          "statement that the caches (cache_ready) or all inputs (inputs_ready) are not being written "
                          "by the kernels that may still run -- true here: consecutive steps serve independent input "
-                         "sets, as independent batches do (dense cache; a paged cache launches the ordinary way)")
+                         "sets, as independent batches do")
     ap.add_argument("--workloads", default="",
                     help="comma-separated workloads: one JSON line each (stdout, and --record FILE if given)")
     ap.add_argument("--record", default="", help="file that --workloads appends its JSON lines to")
@@ -1029,8 +1029,8 @@ def main(argv=None):
             print(json.dumps(line), flush=True)
         return 0
 
-    if args.page_size and args.schedule == "fused":
-        args.schedule = "commit"             # the paged calls take the commit schedule
+    if args.page_size and args.schedule == "compact":
+        raise SystemExit("a paged cache takes the commit or the fused schedule")
     dist = dist_init(world, "nccl" if torch.cuda.is_available() else "gloo")
     if args.draft:
         line, inputs = run_draft_arm(args, world, rank, local, dist)

@@ -263,6 +263,21 @@ CLOVER_API clover_status clover_verify_attn_paged(const void *q, const void *k_n
                                    void *workspace, size_t ws_bytes, int32_t *status, void *stream);
 
 /*
+ * clover_verify_attn_paged with the launch flags of clover_verify_attn_ex:
+ * CLOVER_ATTN_PDL, CLOVER_ATTN_CACHE_READY, CLOVER_ATTN_INPUTS_READY (the
+ * statements cover the pools, the block table and the lengths), and
+ * CLOVER_ATTN_NO_APPEND, accepted and implied (a paged call never appends).
+ * Other flag bits: CLOVER_ERR_INVALID_ARG.
+ */
+CLOVER_API clover_status clover_verify_attn_paged_ex(const void *q, const void *k_new, const void *v_new,
+                                   const void *k_pages, const void *v_pages, const int32_t *block_table,
+                                   int n_pages, int page_size, int max_pages,
+                                   const int32_t *cache_len, const int32_t *parent, void *out,
+                                   int B, int T, int Hq, int Hkv, int D, clover_dtype dtype, float scale,
+                                   void *workspace, size_t ws_bytes, int32_t *status, void *stream,
+                                   uint32_t flags);
+
+/*
  * clover_kv_commit into a paged cache: for every sequence b with L = cache_len[b]
  * and a = accept_len[b], slot L+j (its page from block_table) of every KV head
  * receives k_new/v_new of node path[j]; src_index_out[b][j] = path[j] (-1 past
@@ -444,6 +459,27 @@ CLOVER_API clover_status clover_verify_accept_ex(const void *logits, const int32
                                    double temperature, double epsilon, double delta,
                                    void *k_cache, void *v_cache, const void *k_new, const void *v_new,
                                    const int32_t *cache_len, int Hkv, int D, int Lcap,
+                                   int32_t *argmax_out, int32_t *path_out,
+                                   int32_t *accept_len, int32_t *bonus_token,
+                                   int32_t *new_cache_len, int32_t *src_index_out,
+                                   void *workspace, size_t ws_bytes, uint32_t flags,
+                                   int32_t *status, void *stream);
+
+/*
+ * clover_verify_accept_ex with the commit (CLOVER_ACCEPT_COMMIT, implied and
+ * accepted) into a paged cache: slot L+j of every KV head lives in row
+ * (L+j) % page_size of page block_table[b][(L+j) / page_size] of the pools
+ * k_pages, v_pages [n_pages, Hkv, page_size, D]; Lcap = page_size * max_pages;
+ * page ids as for clover_verify_attn_paged (an id outside [0, n_pages) found
+ * on the device raises CLOVER_ERR_INVALID_ARG and that row is not written).
+ * Every other argument, flag and result as for clover_verify_accept_ex.
+ */
+CLOVER_API clover_status clover_verify_accept_paged_ex(const void *logits, const int32_t *cand, const int32_t *parent,
+                                   int B, int T, int V, clover_dtype dtype,
+                                   double temperature, double epsilon, double delta,
+                                   void *k_pages, void *v_pages, const int32_t *block_table,
+                                   int n_pages, int page_size, int max_pages,
+                                   const void *k_new, const void *v_new, const int32_t *cache_len, int Hkv, int D,
                                    int32_t *argmax_out, int32_t *path_out,
                                    int32_t *accept_len, int32_t *bonus_token,
                                    int32_t *new_cache_len, int32_t *src_index_out,

@@ -35,6 +35,8 @@ EXPORTS = (
     "clover_verify_attn_noalloc",
     "clover_verify_attn_paged_workspace_size",
     "clover_verify_attn_paged",
+    "clover_verify_attn_paged_ex",
+    "clover_verify_accept_paged_ex",
     "clover_kv_commit_paged",
     "clover_linear_workspace_size",
     "clover_linear",
@@ -130,6 +132,11 @@ def load(build_if_missing: bool = False):
         lib.clover_verify_attn_paged.argtypes = [P, P, P, P, P, P, I, I, I, P, P, P, I, I, I, I, I, I, F, P, Z,
                                                  P, P]
         lib.clover_verify_attn_paged.restype = I
+        lib.clover_verify_attn_paged_ex.argtypes = lib.clover_verify_attn_paged.argtypes + [ctypes.c_uint32]
+        lib.clover_verify_attn_paged_ex.restype = I
+        lib.clover_verify_accept_paged_ex.argtypes = [P, P, P, I, I, I, I, Dd, Dd, Dd, P, P, P, I, I, I, P, P, P, I,
+                                                      I, P, P, P, P, P, P, P, Z, ctypes.c_uint32, P, P]
+        lib.clover_verify_accept_paged_ex.restype = I
         lib.clover_kv_commit_paged.argtypes = [P, P, P, I, I, I, P, P, P, P, P, P, P, I, I, I, I, I, P, P]
         lib.clover_kv_commit_paged.restype = I
         lib.clover_linear_workspace_size.argtypes = [I, I, I]

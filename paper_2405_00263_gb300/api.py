@@ -237,9 +237,12 @@ def clover_verify_attn_paged_workspace_size(B, T, Hq, Hkv, D, page_size, max_pag
 
 
 def clover_verify_attn_paged(q, k_new, v_new, k_pages, v_pages, block_table, cache_len, parent, out, scale=0.0,
-                             workspace=None, status=None, stream=None):
+                             workspace=None, status=None, stream=None, pdl=False, cache_ready=False,
+                             inputs_ready=False):
     """Tree-masked attention over a paged cache: pools [n_pages, Hkv, page_size, D],
-    block_table [B, max_pages] (the pools are only read)."""
+    block_table [B, max_pages] (the pools are only read).  ``pdl``,
+    ``cache_ready`` and ``inputs_ready`` as for clover_verify_attn (through
+    clover_verify_attn_paged_ex; the statements also cover the block table)."""
     B, T, Hq, D = q.shape
     n_pages, Hkv, page_size = k_pages.shape[0], k_pages.shape[1], k_pages.shape[2]
     max_pages = block_table.shape[1]
@@ -256,12 +259,17 @@ def clover_verify_attn_paged(q, k_new, v_new, k_pages, v_pages, block_table, cac
         _check(status, (1,), torch.int32, "status")
     _dev(q, k_new, v_new, k_pages, v_pages, block_table, cache_len, parent, out, workspace, status)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    code = _lib.load().clover_verify_attn_paged(
-        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_pages), _ptr(v_pages), _ptr(block_table), n_pages, page_size,
-        max_pages, _ptr(cache_len), _ptr(parent), _ptr(out), B, T, Hq, Hkv, D, dtype_code(dt), float(scale),
-        _ptr(workspace), ws_bytes, _ptr(status), _stream(stream))
+    args = (_ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_pages), _ptr(v_pages), _ptr(block_table), n_pages, page_size,
+            max_pages, _ptr(cache_len), _ptr(parent), _ptr(out), B, T, Hq, Hkv, D, dtype_code(dt), float(scale),
+            _ptr(workspace), ws_bytes, _ptr(status), _stream(stream))
+    flags = (_lib.ATTN_PDL if pdl else 0) | (_lib.ATTN_CACHE_READY if cache_ready else 0) | \
+        (_lib.ATTN_INPUTS_READY if inputs_ready else 0)
+    if flags == 0:
+        code = _lib.load().clover_verify_attn_paged(*args)
+    else:
+        code = _lib.load().clover_verify_attn_paged_ex(*args, flags)
     if code != OK:
-        raise CloverError(code, "clover_verify_attn_paged")
+        raise CloverError(code, "clover_verify_attn_paged" if flags == 0 else "clover_verify_attn_paged_ex")
 
 
 def clover_kv_commit_paged(k_pages, v_pages, block_table, k_new, v_new, cache_len, path, accept_len, new_cache_len,
@@ -371,6 +379,54 @@ def clover_verify_accept_ex(logits, cand, parent, argmax_out, path_out, accept_l
         _ptr(bonus_token), _ptr(ncl), _ptr(src), _ptr(workspace), ws_bytes, flags, _ptr(status), _stream(stream))
     if code != OK:
         raise CloverError(code, "clover_verify_accept_ex")
+
+
+def clover_verify_accept_paged_ex(logits, cand, parent, argmax_out, path_out, accept_len, bonus_token, workspace,
+                                  commit, block_table, typical=None, overlap=False, status=None, stream=None):
+    """clover_verify_accept_ex with the commit into a paged cache: ``commit`` =
+    (k_pages, v_pages, k_new, v_new, cache_len, new_cache_len, src_index_out
+    or None) with pools [n_pages, Hkv, page_size, D] and ``block_table``
+    [B, max_pages]; slot L+j of sequence b is row (L+j) % page_size of page
+    block_table[b][(L+j) // page_size]."""
+    B, T, V = logits.shape
+    _check(cand, (B, T), torch.int32, "cand")
+    _check(parent, (B, T), torch.int32, "parent")
+    _check(argmax_out, (B, T), torch.int32, "argmax_out")
+    _check(path_out, (B, T), torch.int32, "path_out")
+    _check(accept_len, (B,), torch.int32, "accept_len")
+    _check(bonus_token, (B,), torch.int32, "bonus_token")
+    if status is not None:
+        _check(status, (1,), torch.int32, "status")
+    flags = _lib.ACCEPT_COMMIT
+    tau = eps = delta = 0.0
+    if typical is not None:
+        flags |= _lib.ACCEPT_TYPICAL
+        tau, eps, delta = (float(x) for x in typical)
+    if overlap:
+        flags |= _lib.ACCEPT_OVERLAP
+    kp, vp, kn, vn, cl, ncl, src = commit
+    n_pages, Hkv, page_size, D = kp.shape
+    max_pages = block_table.shape[1]
+    dt = logits.dtype
+    _check(kp, (n_pages, Hkv, page_size, D), dt, "k_pages")
+    _check(vp, (n_pages, Hkv, page_size, D), dt, "v_pages")
+    _check(block_table, (B, max_pages), torch.int32, "block_table")
+    _check(kn, (B, T, Hkv, D), dt, "k_new")
+    _check(vn, (B, T, Hkv, D), dt, "v_new")
+    _check(cl, (B,), torch.int32, "cache_len")
+    _check(ncl, (B,), torch.int32, "new_cache_len")
+    if src is not None:
+        _check(src, (B, T), torch.int32, "src_index_out")
+    _dev(logits, cand, parent, argmax_out, path_out, accept_len, bonus_token, workspace, status, kp, vp, block_table,
+         kn, vn, cl, ncl, src)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    code = _lib.load().clover_verify_accept_paged_ex(
+        _ptr(logits), _ptr(cand), _ptr(parent), B, T, V, dtype_code(dt), tau, eps, delta, _ptr(kp), _ptr(vp),
+        _ptr(block_table), n_pages, page_size, max_pages, _ptr(kn), _ptr(vn), _ptr(cl), Hkv, D, _ptr(argmax_out),
+        _ptr(path_out), _ptr(accept_len), _ptr(bonus_token), _ptr(ncl), _ptr(src), _ptr(workspace), ws_bytes, flags,
+        _ptr(status), _stream(stream))
+    if code != OK:
+        raise CloverError(code, "clover_verify_accept_paged_ex")
 
 
 _LINEAR_MODES = {"f32": 0, "bf16": 1, "res_silu": 2, "res": 3}
@@ -500,11 +556,12 @@ class VerifyStep:
     (with CLOVER_ATTN_CACHE_READY) or ``"inputs_ready"`` (with
     CLOVER_ATTN_INPUTS_READY): the caller's statement that the kernels
     queued before a step do not write its inputs, as when consecutive steps
-    serve independent batches (dense cache only).
-    ``page_size``: a paged cache (commit schedule only): ``run`` then takes the
-    page pools as k_cache/v_cache and the ``block_table``, and calls
-    clover_verify_attn_paged and clover_kv_commit_paged; ``Lcap`` is the
-    capacity page_size * max_pages.
+    serve independent batches.
+    ``page_size``: a paged cache (the commit or the fused schedule): ``run``
+    then takes the page pools as k_cache/v_cache and the ``block_table``, and
+    calls clover_verify_attn_paged(_ex) with clover_kv_commit_paged (commit)
+    or clover_verify_accept_paged_ex (fused); ``Lcap`` is the capacity
+    page_size * max_pages.
     """
 
     ATTN_LAUNCHES = {"ordinary": {}, "pdl": dict(pdl=True), "cache_ready": dict(pdl=True, cache_ready=True),
@@ -518,8 +575,8 @@ class VerifyStep:
             raise ValueError(f"unknown attention launch {attn_launch!r}")
         self.attn_launch = attn_launch
         self._attn_kw = self.ATTN_LAUNCHES[attn_launch]
-        if page_size is not None and (schedule != "commit" or Lcap % page_size):
-            raise ValueError("a paged cache takes the commit schedule and a capacity of whole pages")
+        if page_size is not None and (schedule == "compact" or Lcap % page_size):
+            raise ValueError("a paged cache takes the commit or the fused schedule and a capacity of whole pages")
         self.page_size = page_size
         if accept not in ("greedy", "typical"):
             raise ValueError(f"unknown acceptance rule {accept!r}")
@@ -577,9 +634,14 @@ class VerifyStep:
 
         if self.schedule == "fused":
             ev(0, stream)
-            clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
-                               workspace=self.ws_attn, status=self.status, stream=stream, append=False,
-                               **self._attn_kw)
+            if self.page_size is not None:
+                clover_verify_attn_paged(q, k_new, v_new, k_cache, v_cache, block_table, cache_len, parent,
+                                         self.out, scale=scale, workspace=self.ws_attn, status=self.status,
+                                         stream=stream, **self._attn_kw)
+            else:
+                clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
+                                   workspace=self.ws_attn, status=self.status, stream=stream, append=False,
+                                   **self._attn_kw)
             timed_end = n_ev > 1 and self.side is not None
             if timed_end:
                 # the attention's end, recorded on the side stream: nothing is
@@ -590,11 +652,17 @@ class VerifyStep:
                 self._join.record(self.side)
             elif n_ev > 1:
                 events[1].record(stream)
-            clover_verify_accept_ex(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
-                                    self.ws_accept, typical=self.typical if self.accept == "typical" else None,
-                                    commit=(k_cache, v_cache, k_new, v_new, cache_len, self.new_cache_len,
-                                            self.src_index),
-                                    overlap=self.side is not None, status=self.status_accept, stream=stream)
+            typical = self.typical if self.accept == "typical" else None
+            commit_args = (k_cache, v_cache, k_new, v_new, cache_len, self.new_cache_len, self.src_index)
+            if self.page_size is not None:
+                clover_verify_accept_paged_ex(logits, cand, parent, self.argmax, self.path, self.accept_len,
+                                              self.bonus, self.ws_accept, commit_args, block_table, typical=typical,
+                                              overlap=self.side is not None, status=self.status_accept,
+                                              stream=stream)
+            else:
+                clover_verify_accept_ex(logits, cand, parent, self.argmax, self.path, self.accept_len, self.bonus,
+                                        self.ws_accept, typical=typical, commit=commit_args,
+                                        overlap=self.side is not None, status=self.status_accept, stream=stream)
             if timed_end:
                 stream.wait_event(self._join)
             return
@@ -605,7 +673,8 @@ class VerifyStep:
         ev(0, stream)
         if self.page_size is not None:
             clover_verify_attn_paged(q, k_new, v_new, k_cache, v_cache, block_table, cache_len, parent, self.out,
-                                     scale=scale, workspace=self.ws_attn, status=self.status, stream=stream)
+                                     scale=scale, workspace=self.ws_attn, status=self.status, stream=stream,
+                                     **self._attn_kw)
         else:
             clover_verify_attn(q, k_new, v_new, k_cache, v_cache, cache_len, parent, self.out, scale=scale,
                                workspace=self.ws_attn, status=self.status, stream=stream, append=not commit,

@@ -371,12 +371,14 @@ size_t clover_verify_attn_paged_workspace_size(int B, int T, int Hq, int Hkv, in
     return clover_verify_attn_workspace_size(B, T, Hq, Hkv, D, (int)lcap, dtype);
 }
 
-clover_status clover_verify_attn_paged(const void *q, const void *k_new, const void *v_new, const void *k_pages,
-                                       const void *v_pages, const int32_t *block_table, int n_pages, int page_size,
-                                       int max_pages, const int32_t *cache_len, const int32_t *parent, void *out,
-                                       int B, int T, int Hq, int Hkv, int D, clover_dtype dtype, float scale,
-                                       void *workspace, size_t ws_bytes, int32_t *status, void *stream) {
-    const NvtxRange nvtx_range("clover_verify_attn_paged");
+static clover_status attn_paged(const void *q, const void *k_new, const void *v_new, const void *k_pages,
+                                const void *v_pages, const int32_t *block_table, int n_pages, int page_size,
+                                int max_pages, const int32_t *cache_len, const int32_t *parent, void *out, int B,
+                                int T, int Hq, int Hkv, int D, clover_dtype dtype, float scale, void *workspace,
+                                size_t ws_bytes, int32_t *status, void *stream, uint32_t flags) {
+    constexpr uint32_t known = CLOVER_ATTN_NO_APPEND | CLOVER_ATTN_PDL | CLOVER_ATTN_CACHE_READY |
+                               CLOVER_ATTN_INPUTS_READY;
+    if (flags & ~known) return CLOVER_ERR_INVALID_ARG;
     const long lcap = paged_capacity(page_size, max_pages);
     if (lcap < 0 || n_pages < 1) return CLOVER_ERR_INVALID_ARG;
     const clover_status s = check_attn_sizes(B, T, Hq, Hkv, D, (int)lcap, dtype);
@@ -386,7 +388,28 @@ clover_status clover_verify_attn_paged(const void *q, const void *k_new, const v
     if (!block_table) return CLOVER_ERR_INVALID_ARG;
     return run_attn(q, k_new, v_new, const_cast<void *>(k_pages), const_cast<void *>(v_pages), cache_len, parent, out,
                     B, T, Hq, Hkv, D, (int)lcap, dtype, scale, workspace, ws_bytes, status, stream, false, block_table,
-                    page_size, max_pages, n_pages);
+                    page_size, max_pages, n_pages, flags & ~CLOVER_ATTN_NO_APPEND);
+}
+
+clover_status clover_verify_attn_paged(const void *q, const void *k_new, const void *v_new, const void *k_pages,
+                                       const void *v_pages, const int32_t *block_table, int n_pages, int page_size,
+                                       int max_pages, const int32_t *cache_len, const int32_t *parent, void *out,
+                                       int B, int T, int Hq, int Hkv, int D, clover_dtype dtype, float scale,
+                                       void *workspace, size_t ws_bytes, int32_t *status, void *stream) {
+    const NvtxRange nvtx_range("clover_verify_attn_paged");
+    return attn_paged(q, k_new, v_new, k_pages, v_pages, block_table, n_pages, page_size, max_pages, cache_len, parent,
+                      out, B, T, Hq, Hkv, D, dtype, scale, workspace, ws_bytes, status, stream, 0u);
+}
+
+clover_status clover_verify_attn_paged_ex(const void *q, const void *k_new, const void *v_new, const void *k_pages,
+                                          const void *v_pages, const int32_t *block_table, int n_pages,
+                                          int page_size, int max_pages, const int32_t *cache_len,
+                                          const int32_t *parent, void *out, int B, int T, int Hq, int Hkv, int D,
+                                          clover_dtype dtype, float scale, void *workspace, size_t ws_bytes,
+                                          int32_t *status, void *stream, uint32_t flags) {
+    const NvtxRange nvtx_range("clover_verify_attn_paged_ex");
+    return attn_paged(q, k_new, v_new, k_pages, v_pages, block_table, n_pages, page_size, max_pages, cache_len, parent,
+                      out, B, T, Hq, Hkv, D, dtype, scale, workspace, ws_bytes, status, stream, flags);
 }
 
 size_t clover_verify_accept_workspace_size(int B, int T, int V, clover_dtype dtype) {
@@ -465,6 +488,50 @@ clover_status clover_verify_accept_ex(const void *logits, const int32_t *cand, c
         c.D = D;
         c.Lcap = Lcap;
     }
+    c.after_prior = (flags & CLOVER_ACCEPT_OVERLAP) != 0;
+    if (B == 0) return CLOVER_OK;
+    return from_cuda(launch_accept_call(c, static_cast<cudaStream_t>(stream)));
+}
+
+clover_status clover_verify_accept_paged_ex(const void *logits, const int32_t *cand, const int32_t *parent, int B,
+                                            int T, int V, clover_dtype dtype, double temperature, double epsilon,
+                                            double delta, void *k_pages, void *v_pages, const int32_t *block_table,
+                                            int n_pages, int page_size, int max_pages, const void *k_new,
+                                            const void *v_new, const int32_t *cache_len, int Hkv, int D,
+                                            int32_t *argmax_out, int32_t *path_out, int32_t *accept_len,
+                                            int32_t *bonus_token, int32_t *new_cache_len, int32_t *src_index_out,
+                                            void *workspace, size_t ws_bytes, uint32_t flags, int32_t *status,
+                                            void *stream) {
+    const NvtxRange nvtx_range("clover_verify_accept_paged_ex");
+    constexpr uint32_t known = CLOVER_ACCEPT_TYPICAL | CLOVER_ACCEPT_COMMIT | CLOVER_ACCEPT_OVERLAP;
+    if (flags & ~known) return CLOVER_ERR_INVALID_ARG;
+    const long lcap = paged_capacity(page_size, max_pages);
+    if (lcap < 0 || n_pages < 1) return CLOVER_ERR_INVALID_ARG;
+    AcceptCall c;
+    clover_status s = check_accept(c, logits, cand, parent, B, T, V, dtype, argmax_out, path_out, accept_len,
+                                   bonus_token, workspace, ws_bytes, status, (flags & CLOVER_ACCEPT_TYPICAL) != 0,
+                                   temperature, epsilon, delta);
+    if (s != CLOVER_OK) return s;
+    s = check_commit(k_pages, v_pages, k_new, v_new, cache_len, path_out, accept_len, new_cache_len, B, T, Hkv, D,
+                     (int)lcap, dtype, true);
+    if (s != CLOVER_OK) return s;
+    if ((long)n_pages * Hkv * page_size > 0x7FFFFFFFL) return CLOVER_ERR_UNSUPPORTED;
+    if (B > 0 && !block_table) return CLOVER_ERR_INVALID_ARG;
+    c.commit = true;
+    c.k_cache = k_pages;
+    c.v_cache = v_pages;
+    c.k_new = k_new;
+    c.v_new = v_new;
+    c.cache_len = cache_len;
+    c.new_cache_len = new_cache_len;
+    c.src_index = src_index_out;
+    c.Hkv = Hkv;
+    c.D = D;
+    c.Lcap = (int)lcap;
+    c.block_table = block_table;
+    c.page_size = page_size;
+    c.max_pages = max_pages;
+    c.n_pages = n_pages;
     c.after_prior = (flags & CLOVER_ACCEPT_OVERLAP) != 0;
     if (B == 0) return CLOVER_OK;
     return from_cuda(launch_accept_call(c, static_cast<cudaStream_t>(stream)));

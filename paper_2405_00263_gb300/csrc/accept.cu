@@ -218,6 +218,8 @@ struct AcceptArgs {
     const int32_t *cache_len;
     int32_t *new_cache_len, *src_index;
     int Hkv, Lcap, row_units;      // row_units = D * element size / 16
+    const int32_t *block_table;    // paged cache: [B, max_pages] page ids, else nullptr
+    int page_size, page_shift, max_pages, n_pages;
     int commit;
     int wait_prior;                // the last CTAs end with a wait for the preceding grid
     int32_t *status;
@@ -377,8 +379,11 @@ __device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, co
 }
 
 // Commit of sequence b's accepted path (len nodes in s_path) by the whole CTA:
-// slot L + j of every KV head receives node s_path[j]'s K/V from k_new/v_new.
+// slot L + j of every KV head receives node s_path[j]'s K/V from k_new/v_new,
+// into a dense cache or, through the block table, a paged one (a page id
+// outside [0, n_pages) raises CLOVER_ERR_INVALID_ARG and its row is skipped).
 __device__ void commit_sequence(const AcceptArgs &a, int b, const int *s_path, int len) {
+    __shared__ int s_page[kMaxTreeNodes];     // paged: the page of slot L + j
     const int Tn = a.T;
     const int L = __ldg(a.cache_len + b);
     if (L < 0 || L + Tn > a.Lcap) {
@@ -387,6 +392,15 @@ __device__ void commit_sequence(const AcceptArgs &a, int b, const int *s_path, i
     }
     if (a.src_index && threadIdx.x < Tn) a.src_index[(size_t)b * Tn + threadIdx.x] = threadIdx.x < len ? s_path[threadIdx.x] : -1;
     if (threadIdx.x == 0) a.new_cache_len[b] = L + len;
+    if (a.block_table) {
+        if ((int)threadIdx.x < len) {
+            const int pg = __ldg(a.block_table + (size_t)b * a.max_pages + ((L + (int)threadIdx.x) >> a.page_shift));
+            const bool bad = pg < 0 || pg >= a.n_pages;
+            if (bad) report(a.status, CLOVER_ERR_INVALID_ARG);
+            s_page[threadIdx.x] = bad ? -1 : pg;
+        }
+        __syncthreads();
+    }
     // The accepted rows (len nodes x Hkv heads x row_units 16-byte units, K
     // and V) in batches: every thread loads its kBatch units of K and V, then
     // stores them, so a batch costs one load round trip.
@@ -415,7 +429,11 @@ __device__ void commit_sequence(const AcceptArgs &a, int b, const int *s_path, i
                 const int g = r / a.row_units;
                 const int u = r - g * a.row_units;
                 if (!CLOVER_IN(a.status, s_path[j], Tn) || !CLOVER_IN(a.status, L + j, a.Lcap)) continue;
-                const size_t dst = (((size_t)b * a.Hkv + g) * a.Lcap + L + j) * a.row_units + u;
+                size_t dst = (((size_t)b * a.Hkv + g) * a.Lcap + L + j) * a.row_units + u;
+                if (a.block_table) {
+                    if (s_page[j] < 0) continue;
+                    dst = (((size_t)s_page[j] * a.Hkv + g) * a.page_size + ((L + j) & (a.page_size - 1))) * a.row_units + u;
+                }
                 a.k_cache[dst] = kb[t];
                 a.v_cache[dst] = vb[t];
             }
@@ -721,6 +739,13 @@ cudaError_t launch_accept_call(const AcceptCall &c, cudaStream_t stream) {
         a.Hkv = c.Hkv;
         a.Lcap = c.Lcap;
         a.row_units = c.D * (c.dtype == CLOVER_F32 ? 4 : 2) / 16;
+        if (c.block_table) {
+            a.block_table = c.block_table;
+            a.page_size = c.page_size;
+            while ((1 << a.page_shift) < c.page_size) ++a.page_shift;
+            a.max_pages = c.max_pages;
+            a.n_pages = c.n_pages;
+        }
     }
     a.wait_prior = c.after_prior ? 1 : 0;
     a.status = c.status;

@@ -64,6 +64,11 @@ struct AcceptCall {
     const int32_t *cache_len;
     int32_t *new_cache_len, *src_index;
     int Hkv, D, Lcap;
+    // paged cache (block_table != nullptr): k_cache/v_cache are page pools
+    // [n_pages, Hkv, page_size, D]; slot s of sequence b is row s % page_size
+    // of page block_table[b * max_pages + s / page_size]
+    const int32_t *block_table;
+    int page_size, max_pages, n_pages;
     bool after_prior;               // launch as a programmatic dependent of the preceding kernel
 };
 

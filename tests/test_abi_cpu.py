@@ -192,6 +192,30 @@ def test_paged_host_validation(lib):
     assert commit(B=0) == 0
 
 
+def test_paged_ex_host_validation(lib):
+    P = ctypes.c_void_p
+
+    def attn(flags, ps=64, bt=64, T=4, B=1):
+        return lib.clover_verify_attn_paged_ex(P(64), P(64), P(64), P(64), P(64), P(bt), 10, ps, 8, P(64), P(64),
+                                               P(64), B, T, 2, 2, 64, 1, 0.0, None, 0, None, None, flags)
+    assert attn(16) == 1 and attn(0xFFFFFFF0) == 1            # unknown flag bits
+    assert attn(2, ps=24) == 1 and attn(8 | 2, bt=0) == 1
+    assert attn(2, T=129) == 2
+    assert attn(1 | 2 | 4 | 8, B=0) == 0                     # every known bit, NO_APPEND included
+
+    def accept(flags, ps=64, bt=64, kn=64, D=64, B=2, T=4, ncl=4096, tau=1.0):
+        return lib.clover_verify_accept_paged_ex(P(64), P(64), P(64), B, T, 1000, 1, tau, 0.09, 0.3, P(64), P(64),
+                                                 P(bt), 10, ps, 8, P(kn), P(64), P(2048), 2, D, P(64), P(64), P(64),
+                                                 P(64), P(ncl), None, P(4096), 1 << 20, flags, None, None)
+    assert accept(8) == 1 and accept(0xFFFFFFF0) == 1        # unknown flag bits
+    assert accept(2, ps=100) == 1 and accept(2, ps=8) == 1   # page size: a power of two >= 16
+    assert accept(2, bt=0) == 1 and accept(0, kn=0) == 1     # block table, k_new (commit implied)
+    assert accept(2, ncl=2048) == 1                          # new length aliases the old one
+    assert accept(1, tau=0.0) == 1
+    assert accept(2, D=96) == 2 and accept(2, T=129) == 2
+    assert accept(7, B=0) == 0
+
+
 def test_draft_host_validation(lib):
     P = ctypes.c_void_p
     lin = lambda R=4, N=128, K=64, mode=1, x=64, res=None, out=128, ws=None: lib.clover_linear(

@@ -161,3 +161,90 @@ def test_paged_invalid_page_ids_report_status():
                                torch.empty(w.B, **i32), status=st)
     torch.cuda.synchronize()
     assert int(st.item()) & 1
+
+
+def fused_pair(host, pc, ps, dev, **step_kw):
+    """The fused step on the dense padded caches and on the pools: (dense
+    step, paged step, dense K/V caches, K/V pools) after one run each."""
+    B, T, Hq, D = host["q"].shape
+    Hkv = host["k_new"].shape[2]
+    V = host["logits"].shape[-1]
+    dt = host["q"].dtype
+    t = {k: host[k].to(dev) for k in ("q", "k_new", "v_new", "cache_len", "parent", "cand", "logits")}
+    args = (t["q"], t["k_new"], t["v_new"])
+    tail = (t["cache_len"], t["parent"], t["cand"], t["logits"])
+    dense = pkg.VerifyStep(B, T, Hq, Hkv, D, pc["cap"], V, dt, device=dev, schedule="fused", **step_kw)
+    paged = pkg.VerifyStep(B, T, Hq, Hkv, D, pc["cap"], V, dt, device=dev, schedule="fused", page_size=ps,
+                           **step_kw)
+    kd, vd = pc["k_dense"].to(dev), pc["v_dense"].to(dev)
+    kp, vp = pc["k_pool"].to(dev), pc["v_pool"].to(dev)
+    dense.run(*args, kd, vd, *tail)
+    paged.run(*args, kp, vp, *tail, block_table=pc["table"].to(dev))
+    torch.cuda.synchronize()
+    return dense, paged, (kd.cpu(), vd.cpu()), (kp.cpu(), vp.cpu())
+
+
+def check_pair(pc, ps, dense, paged, dense_kv, pools):
+    """The paged step equals the dense one bit for bit: outputs, indices and
+    the committed prefix in the dense view of the pools; unowned pages keep
+    their NaN."""
+    assert dense.device_status() == 0 and paged.device_status() == 0
+    iview = torch.int16 if dense.out.dtype == torch.bfloat16 else torch.int32
+    assert torch.equal(paged.out.view(iview), dense.out.view(iview))
+    for name in ("argmax", "path", "accept_len", "bonus", "src_index", "new_cache_len"):
+        assert torch.equal(getattr(paged, name), getattr(dense, name)), name
+    for pool, kd in zip(pools, dense_kv):
+        view = paging.from_pages(pool, pc["table"], ps, pc["cap"])
+        for b in range(kd.shape[0]):
+            m = int(dense.new_cache_len[b])
+            assert torch.equal(view[b, :, :m].view(iview), kd[b, :, :m].view(iview))
+        owned = set(int(x) for x in pc["table"].flatten() if x >= 0)
+        spare = [p for p in range(pc["n_pages"]) if p not in owned]
+        assert torch.isnan(pool[spare].float()).all()
+
+
+@pytest.mark.parametrize("launch", ["ordinary", "pdl", "cache_ready", "inputs_ready"])
+@pytest.mark.parametrize("accept", ["greedy", "typical"])
+def test_paged_fused_step_equals_dense(launch, accept):
+    """The fused schedule on a paged cache (clover_verify_attn_paged_ex, then
+    clover_verify_accept_paged_ex with the commit into the pools) in every
+    attention launch mode: bit-equal to the dense fused step, whose accept
+    outputs are checked against the oracle here too."""
+    w = workloads.get("7b_l2048", B=3, T=32, Hq=8, Hkv=4, L=900, L_range=(1, 900), V=3001, branching=(4, 2, 2, 1))
+    host = workloads.make(w)
+    dev = torch.device("cuda")
+    ps = 16 if launch in ("ordinary", "inputs_ready") else 64
+    pc = paged_case(host, ps, seed=21)
+    dense, paged, dense_kv, pools = fused_pair(host, pc, ps, dev, accept=accept, attn_launch=launch)
+    check_pair(pc, ps, dense, paged, dense_kv, pools)
+    ref = oracle.verify_step(host, typical=paged.typical if accept == "typical" else None)
+    for name in ("argmax", "path", "accept_len", "bonus"):
+        assert torch.equal(getattr(paged, name).cpu(), ref[name]), name
+    assert torch.equal(paged.new_cache_len.cpu(), ref["cache_len"])
+    err = (paged.out.double().cpu() - ref["out"]).abs().max().item()
+    assert err <= ATOL[torch.bfloat16], err
+
+
+@pytest.mark.parametrize("name,ps", [("7b_l4096", 16), ("paper_t4_b16", 64)])
+def test_paged_fused_step_full_size(name, ps):
+    """The bench's paged step at full size (inputs-ready attention, fused
+    accept + commit): bit-equal to the dense step, attention rows sampled
+    against the oracle."""
+    host = workloads.make(workloads.get(name))
+    pc = paged_case(host, ps, seed=4)
+    dense, paged, dense_kv, pools = fused_pair(host, pc, ps, torch.device("cuda"), attn_launch="inputs_ready")
+    check_pair(pc, ps, dense, paged, dense_kv, pools)
+    check_rows_against_oracle(host, paged.out.cpu())
+
+
+def test_paged_fused_invalid_page_id_reports_status():
+    """A bad table entry for a slot the fused commit writes raises
+    CLOVER_ERR_INVALID_ARG in the accept call's status; the row is skipped."""
+    w = workloads.get("7b_l2048", B=2, T=8, Hq=2, Hkv=2, L=256, V=1000, branching=(2, 2, 1))
+    host = workloads.make(w)
+    pc = paged_case(host, 64, seed=5)
+    pc["table"][0, 4] = -5                                # slot 256 = L + 0 of sequence 0 (no slot < L on it)
+    dev = torch.device("cuda")
+    _, paged, _, _ = fused_pair(host, pc, 64, dev)
+    assert int(paged.status.item()) == 0
+    assert int(paged.status_accept.item()) & 1
