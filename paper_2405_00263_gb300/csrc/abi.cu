@@ -15,6 +15,8 @@ int tc_row_tile();
 int tc_max_splits();
 cudaError_t launch_tree_attn_fma(const AttnArgs &a, cudaStream_t stream);
 cudaError_t launch_tree_attn_tc(const AttnArgs &a, cudaStream_t stream);
+bool tc_pair_eligible(const AttnArgs &a);
+cudaError_t launch_tree_attn_tc_pair(const AttnArgs &a, cudaStream_t stream);
 void accept_plan(int B, int T, int V, int dtype, bool typical, int resident, int *n_chunks, int *chunk);
 size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype);
@@ -301,6 +303,10 @@ clover_status run_attn(const void *q, const void *k_new, const void *v_new, void
         }
     }
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // Such a launch with one CTA per head and at least two row tiles a head
+    // (grouped-query shapes) runs two row tiles per CTA: each K/V tile an SM
+    // loads then serves 256 query rows.
+    if (p.tc && a.inputs_early && tc_pair_eligible(a)) return from_cuda(launch_tree_attn_tc_pair(a, st));
     return from_cuda(p.tc ? launch_tree_attn_tc(a, st) : launch_tree_attn_fma(a, st));
 }
 

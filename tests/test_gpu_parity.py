@@ -61,6 +61,54 @@ def test_small_step_inputs_ready_plan(case, cuda):
     compare_full(host, step, t)
 
 
+# Grouped-query shapes whose inputs-ready launch takes one CTA per (sequence,
+# KV head, row tile) -- at least 30 row tiles -- with two or more row tiles a
+# head: that launch runs two row tiles per CTA (tree_attn_tc_pair.cu).
+PAIR = {
+    "pair_gqa8_T64": ("100b_gqa", dict(B=2, Hq=32, Hkv=4, L=900, V=2048)),
+    # three row tiles a head: the second CTA has one (64 rows) and no second tile
+    "pair_odd_tiles_T40": ("100b_gqa", dict(B=2, T=40, Hq=40, Hkv=5, L=700, V=2048, tree="random")),
+    # four row tiles a head, the last of 16 rows
+    "pair_partial_T100_G4": ("7b_l2048", dict(B=1, T=100, Hq=32, Hkv=8, L=1000, V=2048, tree="random")),
+    "pair_empty_cache": ("100b_gqa", dict(B=2, Hq=32, Hkv=4, L=0, V=2048)),
+    "pair_whole_tiles_L1024": ("100b_gqa", dict(B=2, Hq=32, Hkv=4, L=1024, V=2048)),
+    "pair_ragged_lengths": ("100b_gqa", dict(B=3, Hq=24, Hkv=3, L=1500, L_range=(0, 1500), V=2048)),
+    "pair_sharp_scores": ("100b_gqa", dict(B=2, Hq=32, Hkv=4, L=800, V=2048, qkv_std=1.5)),
+}
+
+
+@pytest.mark.parametrize("case", sorted(PAIR))
+def test_pair_kernel_step_matches_oracle(case, cuda):
+    """The bench's step (fused schedule, inputs-ready attention) on
+    grouped-query shapes that take the two-row-tile kernel: every output
+    against the oracle."""
+    name, over = PAIR[case]
+    host = workloads.make(workloads.get(name, **over))
+    t = to_dev(host, cuda)
+    step = run_gpu(t, schedule="fused", attn_launch="inputs_ready")
+    compare_full(host, step, t)
+
+
+def test_pair_kernel_equals_single_tile_kernel(cuda):
+    """100b_gqa at full size: an ordinary launch (one row tile a CTA; its 128
+    CTAs fill the GPU, so one key range each) and an inputs-ready launch (two
+    row tiles a CTA) compute every row the same way: equal bytes."""
+    w = workloads.get("100b_gqa")
+    t = workloads.make(w, device=cuda, logits=False)
+    ws_n = pkg.clover_verify_attn_workspace_size(w.B, w.T, w.Hq, w.Hkv, w.D, t["Lcap"], torch.bfloat16)
+    ws = torch.zeros(max(16, ws_n), dtype=torch.uint8, device=cuda)
+    st = torch.zeros(1, dtype=torch.int32, device=cuda)
+    outs = []
+    for kw in (dict(), dict(pdl=True, inputs_ready=True)):
+        out = torch.full_like(t["q"], float("nan"))
+        pkg.clover_verify_attn(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"],
+                               t["parent"], out, workspace=ws, status=st, append=False, **kw)
+        torch.cuda.synchronize()
+        outs.append(out)
+    assert int(st.item()) == 0
+    assert torch.equal(outs[0].view(torch.int16), outs[1].view(torch.int16))
+
+
 def test_scale_argument(cuda):
     w = workloads.get("tiny_f32", L=300)
     host = workloads.make(w)
