@@ -267,7 +267,8 @@ __device__ __forceinline__ int first_node(const bool (&pred)[kNodesPerLane]) {
 // The walk of finish_sequence, by warp 0; the path also goes to s_path/s_len.
 template <bool TYPICAL>
 __device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, const int (&am)[kNodesPerLane],
-                              const float (&xc)[kNodesPerLane], const float4 *s_row, int *s_path, int *s_len) {
+                              const float (&xc)[kNodesPerLane], const uint64_t (&anc)[kNodesPerLane][kMaskWords],
+                              const float4 *s_row, int *s_path, int *s_len) {
     const int lane = threadIdx.x & 31;
     const int Tn = a.T;
     int32_t *path = a.path_out + (size_t)b * Tn;
@@ -300,20 +301,6 @@ __device__ void walk_sequence(const AcceptArgs &a, int b, const TreeRegs &tr, co
             ++len;
         }
     } else {
-        // ancestor masks by pointer jumping: two nodes a lane and 6 rounds for
-        // trees of up to 64 nodes (a sixth of the shuffles of the general
-        // four-node form)
-        uint64_t anc[kNodesPerLane][kMaskWords];
-        if (Tn <= 64) {
-            tree_masks_jump<2>(*reinterpret_cast<const int(*)[2]>(&tr.p[0]), Tn,
-                               *reinterpret_cast<uint64_t(*)[2][kMaskWords]>(&anc[0]));
-#pragma unroll
-            for (int k = 2; k < kNodesPerLane; ++k)
-#pragma unroll
-                for (int w = 0; w < kMaskWords; ++w) anc[k][w] = 0ull;
-        } else {
-            tree_masks_jump<kNodesPerLane>(tr.p, Tn, anc);
-        }
         uint64_t acc[kMaskWords];                 // accepted edges (node bits), the root included
 #pragma unroll
         for (int k = 0; k < kNodesPerLane; ++k) {
@@ -460,39 +447,105 @@ template <typename T, bool TYPICAL>
 __device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) {
     __shared__ float4 s_row[kMaxTreeNodes];
     __shared__ int s_path[kMaxTreeNodes];
+    __shared__ int s_par[kMaxTreeNodes];      // typical: the parent array, for the root-path walks
     __shared__ int s_len;
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int Tn = a.T;
+    // Typical: tpr threads a row (neighbours in one warp) merge its chunk
+    // records.  Each thread's first two records are loaded before warp 0's
+    // key loads, so that the two round trips overlap.
+    constexpr int kPre = 2;
+    const int tpr = Tn <= 64 ? 4 : 2;
+    const int row = threadIdx.x / tpr;
+    const int q = threadIdx.x % tpr;
+    const float4 *cs = a.chunk_sums + ((size_t)b * Tn + row) * a.n_chunks;
+    float4 pre[kPre];
+    if (TYPICAL) {
+#pragma unroll
+        for (int p = 0; p < kPre; ++p) {
+            const int k = q + p * tpr;
+            pre[p] = (row < Tn && k < a.n_chunks) ? __ldcg(cs + k) : make_float4(-INFINITY, 0.f, 0.f, 0.f);
+        }
+    }
     int am[kNodesPerLane];
     float xc[kNodesPerLane];
+    uint64_t anc[kNodesPerLane][kMaskWords];
 #pragma unroll
     for (int k = 0; k < kNodesPerLane; ++k) {
         am[k] = 0;
         xc[k] = -INFINITY;
     }
     if (warp == 0) {
+        // the row keys and candidate logits are requested first; the typical
+        // rule's ancestor masks are built while they are on their way
+        unsigned long long key[kNodesPerLane];
+#pragma unroll
+        for (int k = 0; k < kNodesPerLane; ++k) {
+            const int i = lane + 32 * k;
+            key[k] = i < Tn ? __ldcg(a.row_key + (size_t)b * Tn + i) : 0ull;
+            if (TYPICAL && i > 0 && i < Tn && tr.c[k] >= 0 && tr.c[k] < a.V)
+                xc[k] = __ldcg(a.cand_x + (size_t)b * Tn + i);
+        }
+        if (TYPICAL) {
+            // Each lane walks its nodes' root paths through the parent array
+            // in shared memory, at most kShortDepth steps a node: the trees
+            // of speculative decoding are shallow.  A deeper tree (or an
+            // invalid one, which is reported and not walked) takes pointer
+            // jumping instead: two nodes a lane and 6 rounds for trees of up
+            // to 64 nodes, four nodes and 7 rounds above that.
+            constexpr int kShortDepth = 8;
+            bool done = !__any_sync(0xffffffffu, tr.invalid);
+            if (done) {
+#pragma unroll
+                for (int k = 0; k < kNodesPerLane; ++k)
+                    if (lane + 32 * k < Tn) s_par[lane + 32 * k] = tr.p[k];
+                __syncwarp();
+#pragma unroll
+                for (int k = 0; k < kNodesPerLane; ++k) {
+                    uint64_t m0 = 0ull, m1 = 0ull;
+                    int j = lane + 32 * k < Tn ? lane + 32 * k : -1;
+                    for (int d = 0; d < kShortDepth && j >= 0; ++d) {
+                        if (j < 64) m0 |= 1ull << j;
+                        else m1 |= 1ull << (j - 64);
+                        j = s_par[j];
+                    }
+                    done = done && j < 0;
+                    anc[k][0] = m0;
+                    anc[k][1] = m1;
+                }
+                done = __all_sync(0xffffffffu, done);
+            }
+            if (!done) {
+                if (Tn <= 64) {
+                    tree_masks_jump<2>(*reinterpret_cast<const int(*)[2]>(&tr.p[0]), Tn,
+                                       *reinterpret_cast<uint64_t(*)[2][kMaskWords]>(&anc[0]));
+#pragma unroll
+                    for (int k = 2; k < kNodesPerLane; ++k)
+#pragma unroll
+                        for (int w = 0; w < kMaskWords; ++w) anc[k][w] = 0ull;
+                } else {
+                    tree_masks_jump<kNodesPerLane>(tr.p, Tn, anc);
+                }
+            }
+        }
 #pragma unroll
         for (int k = 0; k < kNodesPerLane; ++k) {
             const int i = lane + 32 * k;
             if (i < Tn) {
-                const unsigned long long key = __ldcg(a.row_key + (size_t)b * Tn + i);
-                if (TYPICAL && i > 0 && tr.c[k] >= 0 && tr.c[k] < a.V) xc[k] = __ldcg(a.cand_x + (size_t)b * Tn + i);
-                am[k] = (int)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+                am[k] = (int)(0xFFFFFFFFu - (uint32_t)(key[k] & 0xFFFFFFFFull));
                 a.argmax_out[(size_t)b * Tn + i] = am[k];
                 a.row_key[(size_t)b * Tn + i] = 0ull;                      // ready for the next call
             }
         }
     }
     if (TYPICAL) {
-        // tpr threads a row, neighbours in one warp
-        const int tpr = Tn <= 64 ? 4 : 2;
-        const int row = threadIdx.x / tpr;
-        const int q = threadIdx.x % tpr;
+        // the records of a row in the order k = q, q + tpr, ...
         float3 st = make_float3(-INFINITY, 0.f, 0.f);
+#pragma unroll
+        for (int p = 0; p < kPre; ++p) st = merge_sums(st, make_float3(pre[p].x, pre[p].y, pre[p].z));
         if (row < Tn) {
-            const float4 *cs = a.chunk_sums + ((size_t)b * Tn + row) * a.n_chunks;
-            for (int k = q; k < a.n_chunks; k += tpr) {
+            for (int k = q + kPre * tpr; k < a.n_chunks; k += tpr) {
                 const float4 v = __ldcg(cs + k);
                 st = merge_sums(st, make_float3(v.x, v.y, v.z));
             }
@@ -510,7 +563,7 @@ __device__ void finish_sequence(const AcceptArgs &a, int b, const TreeRegs &tr) 
         }
         __syncthreads();
     }
-    if (warp == 0) walk_sequence<TYPICAL>(a, b, tr, am, xc, s_row, s_path, &s_len);
+    if (warp == 0) walk_sequence<TYPICAL>(a, b, tr, am, xc, anc, s_row, s_path, &s_len);
     if (a.commit || a.wait_prior) {
         __syncthreads();
         if (a.commit) commit_sequence(a, b, s_path, s_len);

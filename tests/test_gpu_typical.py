@@ -42,13 +42,15 @@ def peaked_logits(B, T, V, dtype, seed):
 
 
 def tree_and_cand(B, T, V, logits, kind, seed):
-    """Parents (top-k style or random trees) and candidates: each child takes
+    """Parents (top-k style, random or chain trees) and candidates: each child takes
     a uniform token, or with probability 1/2 one of its parent's top-4 tokens."""
     g = torch.Generator().manual_seed(seed + 1)
     par = []
     for b in range(B):
         if kind == "random":
             par.append(trees.random_tree(T, seed=seed, tag=b))
+        elif kind == "chain":
+            par.append(trees.chain_tree(T))
         else:
             par.append(trees.topk_tree(T, [8, 4, 2, 2, 1]))
     top = logits.float().topk(min(4, V), -1).indices
@@ -112,6 +114,9 @@ CASES = [
     (2, 24, 4099, torch.bfloat16, "random", (1.0, 0.3, 0.0)),      # delta = 0: theta = 0
     (2, 128, 20000, torch.bfloat16, "random", (1.0, 0.09, 0.3)),   # two mask words, two threads a row
     (1, 100, 9000, torch.float32, "topk", (0.8, 0.2, 0.5)),
+    # root paths longer than the walk CTA's short walks (8 steps): the masks by pointer jumping
+    (2, 40, 3000, torch.bfloat16, "chain", (1.0, 0.09, 0.3)),
+    (1, 100, 3000, torch.bfloat16, "chain", (1.0, 0.0, 0.3)),    # theta = 0: the whole chain is accepted
 ]
 
 
