@@ -48,7 +48,8 @@ STEP_PASSES = 4          # passes over the input sets in one captured graph of s
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 KERNEL_SOURCES = {
-    "tree_attn": ["tree_attn_tc.cu", "tc_ptx.cuh", "tmap_host.cuh", "common.cuh", "ctx_host.cuh", "abi.cu"],
+    "tree_attn": ["tree_attn_tc.cu", "tree_attn_tc_pair.cu", "tc_ptx.cuh", "tmap_host.cuh", "common.cuh", "ctx_host.cuh",
+                  "abi.cu"],
     "accept": ["accept.cu", "common.cuh", "ctx_host.cuh"],
     "kv_compact": ["kv_compact.cu", "common.cuh", "ctx_host.cuh"],
 }
@@ -420,7 +421,10 @@ def run_gpu_arm(args, world, rank, local, dist):
                      "traffic": traffic, "bytes_per_launch": a_bytes, "launch_us": us["tree_attn"],
                      "attn_launch": step.attn_launch,
                      "launch_us_ordinary": us["tree_attn_ordinary"],
-                     "frac_ordinary": a_bytes / (us["tree_attn_ordinary"] * 1e-6) / 1e9 / hbm,
+                     # an ordinary launch against the same bound's peak, and against HBM
+                     "frac_ordinary": (a_flops / (us["tree_attn_ordinary"] * 1e-6) / 1e12 / tc_peak if tensor_bound
+                                       else a_bytes / (us["tree_attn_ordinary"] * 1e-6) / 1e9 / hbm),
+                     "frac_hbm_ordinary": a_bytes / (us["tree_attn_ordinary"] * 1e-6) / 1e9 / hbm,
                      "frac_of_8TBs": achieved / 8000.0,
                      "flops_per_launch": attn_flops_per_launch(w, lengths),
                      "timing": timing_source["tree_attn"],
