@@ -216,7 +216,10 @@ CLOVER_API clover_status clover_verify_attn(const void *q, const void *k_new, co
  *     of the keys and no use of the workspace.  Fewer, longer CTAs then spend
  *     less of the GPU on setup and on merging splits, and the chain keeps the
  *     memory busy; a single such call on its own takes longer than an
- *     ordinary one.  Its results may differ from an ordinary launch's in the
+ *     ordinary one.  With two or more 128-row tiles per (sequence, KV head)
+ *     (grouped-query shapes, T * Hq / Hkv > 128), D = 128, a dense cache and
+ *     no append, one CTA takes two row tiles, so each K/V tile it loads
+ *     serves both.  Its results may differ from an ordinary launch's in the
  *     last bits (the key ranges are summed in another order); they do not
  *     depend on what runs beside it.
  * The fp32 (CUDA-core) kernel is launched the ordinary way whatever the launch
