@@ -225,6 +225,19 @@ def test_paged_fused_step_equals_dense(launch, accept):
     assert err <= ATOL[torch.bfloat16], err
 
 
+def test_paged_fused_step_grouped_query_rows():
+    """A grouped-query shape with four 128-row tiles a head, inputs-ready: the
+    dense step runs two row tiles per CTA (tree_attn_tc_pair.cu), the paged
+    one a row tile per CTA with one key range (tree_attn_tc.cu); the two
+    kernels compute every row the same way, so the steps agree bit for bit."""
+    w = workloads.get("100b_gqa", B=2, Hq=32, Hkv=4, L=900, L_range=(300, 900), V=2048)
+    host = workloads.make(w)
+    pc = paged_case(host, 16, seed=8)
+    dense, paged, dense_kv, pools = fused_pair(host, pc, 16, torch.device("cuda"), attn_launch="inputs_ready")
+    check_pair(pc, 16, dense, paged, dense_kv, pools)
+    check_rows_against_oracle(host, paged.out.cpu())
+
+
 @pytest.mark.parametrize("name,ps", [("7b_l4096", 16), ("paper_t4_b16", 64)])
 def test_paged_fused_step_full_size(name, ps):
     """The bench's paged step at full size (inputs-ready attention, fused
