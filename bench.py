@@ -742,10 +742,11 @@ def run_e2e(args, w, step, sets, stream, device, dist, world):
         host_in[k].copy_(src[k].cpu())
     dev_bufs = [torch.empty(off, dtype=torch.uint8, device=device) for _ in sets]
     dev_in = [views(buf) for buf in dev_bufs]
-    outs = (step.out, step.path, step.accept_len, step.bonus, step.new_cache_len)
-    host_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
+    # the step's results (out, path, accept_len, bonus, new_cache_len) are one
+    # byte range of the step's output buffer: one read-back copy
+    host_res = torch.empty(step.results.numel(), dtype=torch.uint8).pin_memory()
     h2d = off
-    d2h = sum(t.numel() * t.element_size() for t in host_out)
+    d2h = step.results.numel()
     n = max(10, min(args.steps, 200))
     n_sets = len(sets)
     copy_stream = torch.cuda.Stream(device)
@@ -764,8 +765,7 @@ def run_e2e(args, w, step, sets, stream, device, dist, world):
         step.run(d["q"], d["k_new"], d["v_new"], s["k_cache"], s["v_cache"], d["cache_len"], d["parent"],
                  d["cand"], d["logits"], stream=stream, block_table=s.get("block_table"))
         with torch.cuda.stream(stream):
-            for h, o in zip(host_out, outs):
-                h.copy_(o, non_blocking=True)
+            host_res.copy_(step.results, non_blocking=True)
         join.record(copy_stream)
         stream.wait_event(join)
 
@@ -805,7 +805,7 @@ def run_e2e(args, w, step, sets, stream, device, dist, world):
             "steps": n, "ms_per_step": ms,
             "api": "paper_2405_00263_gb300.VerifyStep.run (C ABI), one CUDA graph per input set: step i, the "
                    "upload of step i+1's inputs (one copy of one pinned buffer holding them all) on a copy stream, "
-                   "the read-back of step i's results"}
+                   "the read-back of step i's results (one copy of VerifyStep.results)"}
 
 
 # ---------------------------------------------------------------------------

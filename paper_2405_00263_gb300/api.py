@@ -9,6 +9,7 @@ defaults to torch's current stream.
 from __future__ import annotations
 
 import ctypes
+import math
 
 import torch
 
@@ -549,6 +550,9 @@ class VerifyStep:
     SM space the attention leaves (and completes after it).
     With ``concurrent=False`` the calls run in order on ``stream``.
     ``src_index`` holds tree nodes (commit) or cache slots (compact).
+    The outputs are views of one device buffer; ``results`` is the byte range
+    holding ``out``, ``path``, ``accept_len``, ``bonus`` and ``new_cache_len``,
+    for a read-back in one copy.
     ``accept``: ``"greedy"`` (clover_verify_accept) or ``"typical"``
     (clover_verify_accept_typical with ``temperature``, ``epsilon``, ``delta``).
     ``attn_launch``: how the attention is launched (clover_verify_attn_ex
@@ -591,14 +595,23 @@ class VerifyStep:
                 else clover_verify_accept_workspace_size)(B, T, V, dtype)
         self.ws_attn = torch.zeros(max(ws_a, 16), dtype=torch.uint8, device=dev) if ws_a else None
         self.ws_accept = torch.zeros(max(ws_b, 16), dtype=torch.uint8, device=dev)
-        self.out = torch.empty((B, T, Hq, D), dtype=dtype, device=dev)
+        # The outputs are views of one device buffer (each region 256-byte
+        # aligned): out, path, accept_len, bonus, new_cache_len, then argmax
+        # and src_index.  `results` is the byte range of the first five, the
+        # step's results, so that a caller reads them back with one copy.
+        fields = [("out", (B, T, Hq, D), dtype), ("path", (B, T), torch.int32), ("accept_len", (B,), torch.int32),
+                  ("bonus", (B,), torch.int32), ("new_cache_len", (B,), torch.int32),
+                  ("argmax", (B, T), torch.int32), ("src_index", (B, T), torch.int32)]
+        offs, off = [], 0
+        for _, shape, dt in fields:
+            n = math.prod(shape) * torch.empty((), dtype=dt).element_size()
+            offs.append((off, n))
+            off = (off + n + 255) // 256 * 256
+        self._outputs = torch.empty(off, dtype=torch.uint8, device=dev)
+        for (name, shape, dt), (o, n) in zip(fields, offs):
+            setattr(self, name, self._outputs[o:o + n].view(dt).view(shape))
+        self.results = self._outputs[:offs[4][0] + offs[4][1]]
         i32 = dict(dtype=torch.int32, device=dev)
-        self.argmax = torch.empty((B, T), **i32)
-        self.path = torch.empty((B, T), **i32)
-        self.accept_len = torch.empty((B,), **i32)
-        self.bonus = torch.empty((B,), **i32)
-        self.new_cache_len = torch.empty((B,), **i32)
-        self.src_index = torch.empty((B, T), **i32)
         self.status = torch.zeros((1,), **i32)
         # the side stream's calls get their own status word so that concurrent
         # calls never update one word at the same time from two streams

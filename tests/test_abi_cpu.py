@@ -275,3 +275,37 @@ def test_checked_build_exports_the_same_symbols():
     for n in declared_symbols():
         assert hasattr(lib, n), n
     assert lib.clover_build_flags() & _lib.BUILD_CHECKED
+
+
+def test_verify_step_outputs_are_views_of_one_buffer(monkeypatch):
+    """VerifyStep's host-side set-up without a GPU (streams, events and the
+    workspace-size calls stubbed): every output is a contiguous, 16-byte
+    aligned view of one buffer, and `results` spans exactly out, path,
+    accept_len, bonus and new_cache_len."""
+    from paper_2405_00263_gb300 import api
+
+    class FakeStream:
+        def __init__(self, *args, **kwargs):
+            pass
+
+        @staticmethod
+        def priority_range():
+            return (0, -1)
+
+    monkeypatch.setattr(api, "clover_verify_attn_workspace_size", lambda *a: 0)
+    monkeypatch.setattr(api, "clover_verify_accept_workspace_size", lambda *a: 64)
+    monkeypatch.setattr(torch.cuda, "Stream", FakeStream)
+    monkeypatch.setattr(torch.cuda, "Event", lambda *a, **k: None)
+    B, T, Hq, D = 3, 37, 8, 128
+    st = api.VerifyStep(B, T, Hq, 8, D, 512, 1000, torch.bfloat16, device="cpu")
+    base = st._outputs.data_ptr()
+    names = ["out", "path", "accept_len", "bonus", "new_cache_len", "argmax", "src_index"]
+    shapes = [(B, T, Hq, D), (B, T), (B,), (B,), (B,), (B, T), (B, T)]
+    spans = []
+    for name, shape in zip(names, shapes):
+        t = getattr(st, name)
+        assert tuple(t.shape) == shape and t.is_contiguous() and t.data_ptr() % 16 == 0, name
+        lo = t.data_ptr() - base
+        spans.append((lo, lo + t.numel() * t.element_size()))
+    assert all(a[1] <= b[0] for a, b in zip(spans, spans[1:]))      # disjoint, in order
+    assert st.results.data_ptr() == base and st.results.numel() == spans[4][1]
