@@ -854,7 +854,9 @@ __global__ void __maxnreg__(160)
         float *dst = part_o + (quad * 32 + lane) * S::po_stride;
         float l_tot = l_run;
         if (NG == 2) {
-            bool stop = !o_ready;
+            // a split with no keys (a short sequence's empty range) has no O
+            // and is not a failure: its rows carry m = -inf and l = 0
+            bool stop = n_tiles > 0 && !o_ready;
             const float other = exchange(l_run, stop);
             l_tot = sgroup == 0 ? l_run + other : other + l_run;
             if (stop) *s_abort = 1;

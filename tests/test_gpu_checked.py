@@ -30,6 +30,7 @@ SELECTION = [
     "tests/test_gpu_parity.py::test_small_step_matches_oracle",
     "tests/test_gpu_parity.py::test_small_step_inputs_ready_plan",
     "tests/test_gpu_parity.py::test_pair_kernel_step_matches_oracle",
+    "tests/test_gpu_parity.py::test_full_row_tiles_with_empty_splits",
     "tests/test_gpu_parity.py::test_split_counts_and_row_groups",
     "tests/test_gpu_parity.py::test_step_attention_launch_modes",
     "tests/test_gpu_parity.py::test_commit_and_compact_schedules_agree",

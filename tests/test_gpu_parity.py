@@ -109,6 +109,27 @@ def test_pair_kernel_equals_single_tile_kernel(cuda):
     assert torch.equal(outs[0].view(torch.int16), outs[1].view(torch.int16))
 
 
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("T,Hq,Hkv,lengths", [(33, 8, 4, [651, 1219]), (33, 8, 4, [0, 1219]),
+                                               (64, 8, 4, [512, 1219]), (33, 16, 4, [700, 1219, 40])],
+                         ids=["T33_G2_651", "T33_G2_empty", "T64_G2_512", "T33_G4_three"])
+def test_full_row_tiles_with_empty_splits(T, Hq, Hkv, lengths, D, cuda):
+    """More than 64 query rows a head (full 128-row tiles: two softmax warps
+    a lane quadrant) with ragged lengths, so that a short sequence leaves some
+    of its non-tree key ranges empty: such a range has no O and reports no
+    error, and the whole step matches the oracle.  (A range with no keys once
+    raised CLOVER_ERR_TIMEOUT in this layout.)"""
+    w = workloads.get("7b_l2048", B=len(lengths), T=T, Hq=Hq, Hkv=Hkv, D=D, L=max(lengths), V=2048,
+                      tree="random", seed=620)
+    host = workloads.make(w)
+    host["cache_len"] = torch.tensor(lengths, dtype=torch.int32)
+    t = to_dev(host, cuda)
+    for schedule in ("commit", "fused"):
+        t = to_dev(host, cuda)
+        step = run_gpu(t, schedule=schedule)
+        compare_full(host, step, t)
+
+
 def test_scale_argument(cuda):
     w = workloads.get("tiny_f32", L=300)
     host = workloads.make(w)

@@ -1,0 +1,108 @@
+"""A seeded sweep over the supported space: random batch sizes, tree sizes and
+shapes, head counts and group sizes, head dimensions, cache lengths (ragged or
+not, empty included), vocabulary sizes, dtypes, step schedules, attention
+launch modes, acceptance rules and cache layouts (dense or paged).  Each case
+runs one whole step through VerifyStep and compares it with the oracle:
+attention within the dtype's tolerance, argmax, path, accepted length, bonus
+token, source indices, new lengths and the committed cache rows bit for bit.
+
+Typical acceptance is drawn with epsilon = 0 (threshold 0: an edge is accepted
+iff its candidate has positive probability), so no decision sits near its
+threshold; tests/test_gpu_typical.py covers thresholds in general."""
+
+from __future__ import annotations
+
+import random
+
+import pytest
+import torch
+
+import oracle
+import paper_2405_00263_gb300 as pkg
+from synth import paging, workloads
+from tests.gpu_util import ATOL, compare_full, to_dev
+
+pytestmark = pytest.mark.gpu
+
+N_CASES = 200
+
+
+def draw(i: int) -> dict:
+    r = random.Random(9000 + i)
+    dtype = r.choice(["bf16", "bf16", "bf16", "f32"])
+    Hkv = r.choice([1, 2, 4])
+    G = r.choice([1, 2, 4, 8])
+    T = r.choice([1, 4, 16, 33, 64, 100, 128])
+    B = r.choice([1, 2, 3])
+    L = r.choice([0, r.randint(1, 300), r.randint(300, 1600)])
+    ragged = L > 0 and r.random() < 0.5
+    schedule = r.choice(["fused", "fused", "commit", "compact"])
+    paged = schedule != "compact" and r.random() < 0.35
+    return dict(
+        w=workloads.Workload(
+            f"sweep{i}", B=B, T=T, Hq=Hkv * G, Hkv=Hkv, D=r.choice([64, 128]), L=L, V=r.choice([1000, 2049, 4099]),
+            dtype=dtype, branching=(8, 4, 2, 2, 2, 1), plant_p=r.choice([0.0, 0.5, 1.0]),
+            qkv_std=r.choice([1.0, 1.0 / 128 ** 0.5]), seed=500 + i, L_range=(0, L) if ragged else None,
+            tree=r.choice(["topk", "random", "chain", "star"])),
+        schedule=schedule,
+        attn_launch=r.choice(["ordinary", "pdl", "cache_ready", "inputs_ready"]),
+        accept=r.choice(["greedy", "greedy", "typical"]),
+        page_size=r.choice([16, 32, 64, 128]) if paged else None,
+    )
+
+
+def describe(i: int) -> str:
+    c = draw(i)
+    w = c["w"]
+    return (f"{i}-{w.dtype}-B{w.B}-T{w.T}-{w.tree}-h{w.Hq}x{w.Hkv}-D{w.D}-L{w.L}{'r' if w.L_range else ''}-"
+            f"{c['schedule']}-{c['attn_launch']}-{c['accept']}" + (f"-p{c['page_size']}" if c["page_size"] else ""))
+
+
+@pytest.mark.parametrize("i", range(N_CASES), ids=[describe(i) for i in range(N_CASES)])
+def test_sweep_step_matches_oracle(i, cuda):
+    c = draw(i)
+    w = c["w"]
+    host = workloads.make(w)
+    B, T, Hq, D = host["q"].shape
+    V = host["logits"].shape[-1]
+    typical = (1.0, 0.0, 0.3) if c["accept"] == "typical" else None
+    kw = dict(schedule=c["schedule"], attn_launch=c["attn_launch"], accept=c["accept"])
+    if typical is not None:
+        kw.update(temperature=typical[0], epsilon=typical[1], delta=typical[2])
+    if c["page_size"] is None:
+        t = to_dev(host, cuda)
+        step = pkg.VerifyStep(B, T, Hq, w.Hkv, D, t["Lcap"], V, w.torch_dtype, device=cuda, **kw)
+        step.run(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
+                 t["cand"], t["logits"])
+        torch.cuda.synchronize()
+        compare_full(host, step, t)
+        return
+
+    # paged: the pools hold the dense cache, padded to whole pages, under a seeded table
+    ps = c["page_size"]
+    cap = -(-host["Lcap"] // max(256, ps)) * max(256, ps)
+    pad = torch.full((B, w.Hkv, cap - host["Lcap"], D), float("nan"), dtype=host["k_cache"].dtype)
+    kc = torch.cat([host["k_cache"], pad], 2)
+    vc = torch.cat([host["v_cache"], pad], 2)
+    table, n_pages = paging.page_table([int(L) + T for L in host["cache_len"]], ps, cap // ps, seed=w.seed)
+    kp = paging.to_pages(kc, table, ps, n_pages).to(cuda)
+    vp = paging.to_pages(vc, table, ps, n_pages).to(cuda)
+    t = to_dev(host, cuda)
+    step = pkg.VerifyStep(B, T, Hq, w.Hkv, D, cap, V, w.torch_dtype, device=cuda, page_size=ps, **kw)
+    step.run(t["q"], t["k_new"], t["v_new"], kp, vp, t["cache_len"], t["parent"], t["cand"], t["logits"],
+             block_table=table.to(cuda))
+    torch.cuda.synchronize()
+    ref = oracle.verify_step(host, typical=typical)
+    assert step.device_status() == 0
+    err = (step.out.double().cpu() - ref["out"]).abs().max().item()
+    assert err <= ATOL[w.torch_dtype], err
+    for name in ("argmax", "path", "accept_len", "bonus"):
+        assert torch.equal(getattr(step, name).cpu(), ref[name]), name
+    assert torch.equal(step.src_index.cpu(), ref["path"])
+    assert torch.equal(step.new_cache_len.cpu(), ref["cache_len"])
+    iview = torch.int16 if w.torch_dtype == torch.bfloat16 else torch.int32
+    for pool, want in ((kp, ref["k_cache"]), (vp, ref["v_cache"])):
+        view = paging.from_pages(pool.cpu(), table, ps, cap)
+        for b in range(B):
+            n = int(ref["cache_len"][b])
+            assert torch.equal(view[b, :, :n].view(iview), want[b, :, :n].view(iview)), b
