@@ -51,6 +51,38 @@ def draw(i: int) -> dict:
     )
 
 
+N_LONG = 40
+
+
+def draw_long(i: int) -> dict:
+    """Long caches (up to 8 key ranges a head) and batches up to 6, the
+    oracle's work bounded to about 4e9 multiply-adds a case."""
+    r = random.Random(77000 + i)
+    Hkv = r.choice([1, 2, 4, 8])
+    G = r.choice([1, 2, 4, 8])
+    T = r.choice([4, 16, 64, 128])
+    B = r.choice([1, 2, 4, 6])
+    L = r.randint(1600, 9000)
+    D = r.choice([64, 128])
+    while B * T * Hkv * G * L * D > 4e9 and B > 1:
+        B -= 1
+    while B * T * Hkv * G * L * D > 4e9 and T > 4:
+        T //= 2
+    schedule = r.choice(["fused", "fused", "commit", "compact"])
+    paged = schedule != "compact" and r.random() < 0.3
+    return dict(
+        w=workloads.Workload(
+            f"long{i}", B=B, T=T, Hq=Hkv * G, Hkv=Hkv, D=D, L=L, V=r.choice([1000, 4099]),
+            dtype=r.choice(["bf16", "bf16", "f32"]), branching=(8, 4, 2, 2, 2, 1), plant_p=r.choice([0.0, 0.5, 1.0]),
+            qkv_std=r.choice([1.0, 1.0 / 128 ** 0.5]), seed=8000 + i, L_range=(0, L) if r.random() < 0.6 else None,
+            tree=r.choice(["topk", "random", "chain", "star"])),
+        schedule=schedule,
+        attn_launch=r.choice(["ordinary", "pdl", "cache_ready", "inputs_ready"]),
+        accept=r.choice(["greedy", "typical"]),
+        page_size=r.choice([16, 64, 256]) if paged else None,
+    )
+
+
 def describe(i: int) -> str:
     c = draw(i)
     w = c["w"]
@@ -60,7 +92,15 @@ def describe(i: int) -> str:
 
 @pytest.mark.parametrize("i", range(N_CASES), ids=[describe(i) for i in range(N_CASES)])
 def test_sweep_step_matches_oracle(i, cuda):
-    c = draw(i)
+    check_case(draw(i), cuda)
+
+
+@pytest.mark.parametrize("i", range(N_LONG))
+def test_sweep_long_caches_match_oracle(i, cuda):
+    check_case(draw_long(i), cuda)
+
+
+def check_case(c: dict, cuda):
     w = c["w"]
     host = workloads.make(w)
     B, T, Hq, D = host["q"].shape
