@@ -13,6 +13,7 @@ The argmax, the path, its length and the bonus token must then be identical.
 from __future__ import annotations
 
 import math
+import random
 
 import pytest
 import torch
@@ -210,3 +211,31 @@ def test_typical_verify_step_matches_oracle(name, over, params, schedule):
     tau, eps, delta = params
     step = run_gpu(t, schedule=schedule, accept="typical", temperature=tau, epsilon=eps, delta=delta)
     compare_full(host, step, t)
+
+
+def draw_typical(i: int):
+    r = random.Random(53000 + i)
+    B = r.choice([1, 2, 3, 5])
+    T = r.choice([1, 2, 9, 16, 33, 64, 65, 100, 128])
+    V = r.choice([1, 2, 100, 1000, 4099, 16384, 16385, 50257, 125696])
+    dtype = r.choice([torch.bfloat16, torch.bfloat16, torch.float32])
+    kind = r.choice(["topk", "random", "chain"])
+    tau = r.choice([0.3, 0.7, 1.0, 1.5, 3.0])
+    eps = r.choice([0.0, 0.01, 0.09, 0.3, 0.9])
+    delta = r.choice([0.0, 0.1, 0.3, 0.6, 1.0])
+    return B, T, V, dtype, kind, (tau, eps, delta)
+
+
+N_SWEEP = 60
+
+
+@pytest.mark.parametrize("i", range(N_SWEEP))
+def test_typical_sweep(i):
+    """Seeded random shapes, trees and (temperature, epsilon, delta), with
+    candidates moved off the threshold's neighbourhood as above."""
+    B, T, V, dtype, kind, (tau, eps, delta) = draw_typical(i)
+    seed = 53000 + i
+    logits = peaked_logits(B, T, V, dtype, seed)
+    parent, cand = tree_and_cand(B, T, V, logits, kind, seed)
+    cand, ref = clear_margins(logits, parent, cand, tau, eps, delta)
+    assert_same(run_typical(logits, parent, cand, tau, eps, delta), ref)
