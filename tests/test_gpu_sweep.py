@@ -146,3 +146,67 @@ def check_case(c: dict, cuda):
         for b in range(B):
             n = int(ref["cache_len"][b])
             assert torch.equal(view[b, :, :n].view(iview), want[b, :, :n].view(iview)), b
+
+
+N_ERRORS = 40
+
+
+def draw_error(i: int) -> dict:
+    """A seeded small case (from draw) with one invalid input: a parent array
+    that is not a topologically numbered tree, a cache length past the
+    capacity, or (paged) a block-table entry outside the pool."""
+    c = draw(1000 + i)
+    r = random.Random(61000 + i)
+    kinds = ["tree", "capacity"] + (["page"] if c["page_size"] else [])
+    c["error"] = r.choice(kinds)
+    c["r"] = r
+    return c
+
+
+@pytest.mark.parametrize("i", range(N_ERRORS))
+def test_sweep_device_errors_are_reported(i, cuda):
+    """The step completes, the status word carries the error's bit
+    (CLOVER_ERR_BAD_TREE 4, CLOVER_ERR_CAPACITY 8, CLOVER_ERR_INVALID_ARG 1)
+    and never CLOVER_ERR_TIMEOUT: every kernel turns the invalid input into a
+    reported error and winds down without a wait running out."""
+    c = draw_error(i)
+    w, r = c["w"], c["r"]
+    host = workloads.make(w)
+    B, T, Hq, D = host["q"].shape
+    V = host["logits"].shape[-1]
+    bit = {"tree": 4, "capacity": 8, "page": 1}[c["error"]]
+    b = r.randrange(B)
+    if c["error"] == "tree":
+        if T == 1 or r.random() < 0.3:
+            host["parent"][b, 0] = r.choice([0, 5, -7])
+        else:
+            j = r.randrange(1, T)
+            host["parent"][b, j] = r.choice([j, j + 1 if j + 1 < T else j, -3, T + 4])
+    elif c["error"] == "capacity":
+        host["cache_len"][b] = host["Lcap"] - T + 1 + r.randrange(40)
+    kw = dict(schedule=c["schedule"], attn_launch=c["attn_launch"], accept=c["accept"])
+    t = to_dev(host, cuda)
+    if c["page_size"] is None:
+        step = pkg.VerifyStep(B, T, Hq, w.Hkv, D, t["Lcap"], V, w.torch_dtype, device=cuda, **kw)
+        step.run(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
+                 t["cand"], t["logits"])
+    else:
+        ps = c["page_size"]
+        cap = -(-host["Lcap"] // max(256, ps)) * max(256, ps)
+        lens = [min(int(L), host["Lcap"] - T) for L in host["cache_len"]]
+        table, n_pages = paging.page_table([L + T for L in lens], ps, cap // ps, seed=w.seed)
+        if c["error"] == "capacity":
+            t["cache_len"][b] = cap - T + 1           # past the paged capacity
+        if c["error"] == "page":
+            # an entry the step always uses: the page of slot 0 (read when L > 0) or of slot L (the commit
+            # writes the accepted root there)
+            k = 0 if lens[b] > 0 and r.random() < 0.5 else lens[b] // ps
+            table[b, k] = r.choice([-2, n_pages, n_pages + 9])
+        pool = torch.zeros((n_pages, w.Hkv, ps, D), dtype=w.torch_dtype, device=cuda)
+        step = pkg.VerifyStep(B, T, Hq, w.Hkv, D, cap, V, w.torch_dtype, device=cuda, page_size=ps, **kw)
+        step.run(t["q"], t["k_new"], t["v_new"], pool, pool.clone(), t["cache_len"], t["parent"], t["cand"],
+                 t["logits"], block_table=table.to(cuda))
+    torch.cuda.synchronize()
+    status = step.device_status()
+    assert status & bit, (c["error"], status)
+    assert not status & 32, status
