@@ -116,3 +116,44 @@ def test_noalloc_rejects_scratch_beyond_its_buffer():
                                           1, 64, Hq, Hkv, 128, Lcap, dt, 0.0, None, None)
     assert code == pkg.api.ERR_SCRATCH_LIMIT
     assert b"static buffer" in lib.clover_status_string(code)
+
+
+def test_noalloc_sweep_matches_workspace_entry_point(cuda):
+    """Seeded random shapes (both dtypes, GQA groups, D = 64 and 128, ragged
+    cache lengths), each within the static buffer: the allocation-free call
+    and clover_verify_attn with a workspace give the same bytes (output and
+    appended tree K/V), one after the other, so each call finds the previous
+    shape's scratch in the buffer."""
+    import random
+    lib = _lib.load(build_if_missing=True)
+    stream = torch.cuda.current_stream()
+    r = random.Random(71000)
+    done = 0
+    for i in range(60):
+        Hkv = r.choice([1, 2, 4, 8])
+        w = workloads.Workload(
+            f"noalloc{i}", B=r.choice([1, 2, 3]), T=r.choice([1, 4, 16, 64, 128]), Hq=Hkv * r.choice([1, 2, 4]),
+            Hkv=Hkv, D=r.choice([64, 128]), L=r.randint(0, 3000), V=1000, dtype=r.choice(["bf16", "f32"]),
+            branching=(8, 4, 2, 2, 2, 1), seed=71000 + i, L_range=(0, 3000) if r.random() < 0.5 else None,
+            tree=r.choice(["topk", "random", "chain"]))
+        need = pkg.clover_verify_attn_workspace_size(w.B, w.T, w.Hq, w.Hkv, w.D, workloads.lcap(w), w.torch_dtype)
+        if need > _lib.NOALLOC_SCRATCH_BYTES:
+            continue
+        base = workloads.make(w, device=cuda, logits=False)
+        ref = {k: (v.clone() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
+        out_ref = torch.empty_like(ref["q"])
+        ws = torch.zeros(max(16, need), dtype=torch.uint8, device=cuda)
+        pkg.clover_verify_attn(ref["q"], ref["k_new"], ref["v_new"], ref["k_cache"], ref["v_cache"],
+                               ref["cache_len"], ref["parent"], out_ref, workspace=ws)
+        t = {k: (v.clone() if isinstance(v, torch.Tensor) else v) for k, v in base.items()}
+        out = torch.full_like(t["q"], float("nan"))
+        st = torch.zeros(1, dtype=torch.int32, device=cuda)
+        assert _call_noalloc(lib, t, out, st, stream) == 0
+        torch.cuda.synchronize()
+        assert int(st.item()) == 0, i
+        iv = torch.int16 if w.dtype == "bf16" else torch.int32       # bytes (slots past L + T hold NaN)
+        assert torch.equal(out.view(iv), out_ref.view(iv)), i
+        assert torch.equal(t["k_cache"].view(iv), ref["k_cache"].view(iv)), i
+        assert torch.equal(t["v_cache"].view(iv), ref["v_cache"].view(iv)), i
+        done += 1
+    assert done >= 30
