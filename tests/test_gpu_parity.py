@@ -666,3 +666,52 @@ def test_accept_ex_commit_capacity_and_overlap_flag(cuda):
             assert torch.equal(t["v_cache"][b, :, :m].cpu().view(torch.int16), vc_ok[n, :, :m].view(torch.int16))
         assert int(ncl[1]) == -7                              # not committed
         assert torch.equal(t["k_cache"][1].cpu().view(torch.int16), host["k_cache"][1].view(torch.int16))
+
+
+@pytest.mark.parametrize("shared_step", [False, True])
+@pytest.mark.parametrize("name,over", [("7b_l2048", dict(T=64, Hq=8, Hkv=8, L=1500, V=3000)),
+                                       ("100b_gqa", dict(B=2, Hq=32, Hkv=4, L=900, V=2048))],
+                         ids=["mha", "gqa_pair"])
+def test_graph_of_overlapping_steps(name, over, shared_step, cuda):
+    """The bench's arrangement: a CUDA graph of 30 fused steps (inputs-ready
+    attention, accept + commit as its programmatic dependent) over three
+    independent input sets, consecutive steps overlapping, replayed three
+    times.  With one VerifyStep a set (or one shared by all, whose outputs
+    then hold the last step's), every set's outputs and committed cache rows
+    match the oracle afterwards (a step repeated on the same set rewrites the
+    same rows), and no status bit is set."""
+    hosts = [workloads.make(workloads.get(name, seed=90 + k, **over)) for k in range(3)]
+    sets = [to_dev(h, cuda) for h in hosts]
+    B, T, Hq, D = sets[0]["q"].shape
+    Hkv = sets[0]["k_new"].shape[2]
+    V = sets[0]["logits"].shape[-1]
+    Lcap = max(s["Lcap"] for s in sets)
+    assert all(s["Lcap"] == Lcap for s in sets)
+
+    def new_step():
+        return pkg.VerifyStep(B, T, Hq, Hkv, D, Lcap, V, torch.bfloat16, device=cuda, schedule="fused",
+                              attn_launch="inputs_ready")
+
+    steps = [new_step()] * 3 if shared_step else [new_step() for _ in range(3)]
+    stream = torch.cuda.Stream()
+
+    def run_all():
+        for _ in range(10):
+            for step, s in zip(steps, sets):
+                step.run(s["q"], s["k_new"], s["v_new"], s["k_cache"], s["v_cache"], s["cache_len"], s["parent"],
+                         s["cand"], s["logits"], stream=stream)
+
+    with torch.cuda.stream(stream):
+        run_all()                                  # eager warm-up (kernel attributes set before capture)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        run_all()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    if shared_step:
+        compare_full(hosts[2], steps[2], sets[2])
+    else:
+        for h, step, s in zip(hosts, steps, sets):
+            compare_full(h, step, s)
