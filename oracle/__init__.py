@@ -46,29 +46,34 @@ def build(force: bool = False) -> str:
     return _LIB
 
 
+def _open(path: str):
+    """Load a compiled copy of clover_oracle.c and declare its signatures."""
+    lib = ctypes.CDLL(path)
+    P, I, I64, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_double
+    lib.oracle_tree_mask.argtypes = [P, I, P, P]
+    lib.oracle_tree_attention.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, I, D,
+                                          P, I64, P, I]
+    lib.oracle_argmax.argtypes = [P, I64, I64, I, P, I64, P, I]
+    lib.oracle_accept_walk.argtypes = [P, P, P, I, I, P, P, P]
+    lib.oracle_append_tree_kv.argtypes = [P, P, P, P, P, I, I, I, I, I, I]
+    lib.oracle_kv_compact.argtypes = [P, P, P, P, P, I, I, I, I, I, I, P]
+    lib.oracle_kv_commit.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P]
+    lib.oracle_accept_typical.argtypes = [P, P, P, I, I, I64, I, D, D, D, P, P, P, P, P, I]
+    lib.oracle_linear.argtypes = [P, P, P, I, I, I, I, I, P, I]
+    lib.oracle_embed_rows.argtypes = [P, P, I, I, I, I, P]
+    lib.oracle_topk.argtypes = [P, I, I, I, P, P]
+    for f in (lib.oracle_tree_mask, lib.oracle_tree_attention, lib.oracle_argmax,
+              lib.oracle_accept_walk, lib.oracle_append_tree_kv, lib.oracle_kv_compact,
+              lib.oracle_kv_commit):
+        f.restype = ctypes.c_int
+    return lib
+
+
 def _load():
     global _lib
     with _lock:
         if _lib is None:
-            lib = ctypes.CDLL(build())
-            P, I, I64, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_double
-            lib.oracle_tree_mask.argtypes = [P, I, P, P]
-            lib.oracle_tree_attention.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, I, D,
-                                                  P, I64, P, I]
-            lib.oracle_argmax.argtypes = [P, I64, I64, I, P, I64, P, I]
-            lib.oracle_accept_walk.argtypes = [P, P, P, I, I, P, P, P]
-            lib.oracle_append_tree_kv.argtypes = [P, P, P, P, P, I, I, I, I, I, I]
-            lib.oracle_kv_compact.argtypes = [P, P, P, P, P, I, I, I, I, I, I, P]
-            lib.oracle_kv_commit.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, P]
-            lib.oracle_accept_typical.argtypes = [P, P, P, I, I, I64, I, D, D, D, P, P, P, P, P, I]
-            lib.oracle_linear.argtypes = [P, P, P, I, I, I, I, I, P, I]
-            lib.oracle_embed_rows.argtypes = [P, P, I, I, I, I, P]
-            lib.oracle_topk.argtypes = [P, I, I, I, P, P]
-            for f in (lib.oracle_tree_mask, lib.oracle_tree_attention, lib.oracle_argmax,
-                      lib.oracle_accept_walk, lib.oracle_append_tree_kv, lib.oracle_kv_compact,
-                      lib.oracle_kv_commit):
-                f.restype = ctypes.c_int
-            _lib = lib
+            _lib = _open(build())
     return _lib
 
 

@@ -279,6 +279,24 @@ def test_attention_scale_closed_form():
         assert float(got[0, 0, 0, 0]) == pytest.approx((vc * w + v0) / (w + 1), abs=1e-15)
 
 
+def test_attention_huge_scores_closed_form():
+    """Scores far past exp's range (s*a up to 1e4): the softmax is taken
+    relative to the row maximum, so the output is the closed form of
+    test_attention_scale_closed_form with e^{-s a} underflowing to 0: v_c
+    when the cache key dominates, v_0 when its score is hugely negative, and
+    the plain mean when both scores are equal and huge."""
+    inp = rand_inputs(1, 1, 1, 1, 1, 1, seed=14)
+    vc, v0 = 2.0, -3.0
+    inp["v_cache"][0, 0, 0, 0] = vc
+    inp["v_new"][:] = v0
+    for qv, a, kr, want in ((1.0, 800.0, 0.0, vc), (1.0, -5000.0, 0.0, v0), (10.0, 1000.0, 1000.0, (vc + v0) / 2)):
+        inp["q"][:] = qv
+        inp["k_cache"][0, 0, 0, 0] = a
+        inp["k_new"][:] = kr
+        got = run_oracle_attn(inp, [[-1]], scale=1.0)
+        assert float(got[0, 0, 0, 0]) == want
+
+
 def test_attention_hand_worked_example():
     ex = json.load(open(os.path.join(GOLDEN, "hand_tree_attention.json")))
     T = len(ex["parent"])
