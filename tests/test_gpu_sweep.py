@@ -101,6 +101,16 @@ def test_sweep_long_caches_match_oracle(i, cuda):
 
 
 def check_case(c: dict, cuda):
+    run, check = prepare_case(c, cuda)
+    run(None)
+    torch.cuda.synchronize()
+    check()
+
+
+def prepare_case(c: dict, cuda):
+    """The case's device inputs and VerifyStep; returns run(stream), which
+    issues one step, and check(), which compares the finished step with the
+    oracle."""
     w = c["w"]
     host = workloads.make(w)
     B, T, Hq, D = host["q"].shape
@@ -112,11 +122,12 @@ def check_case(c: dict, cuda):
     if c["page_size"] is None:
         t = to_dev(host, cuda)
         step = pkg.VerifyStep(B, T, Hq, w.Hkv, D, t["Lcap"], V, w.torch_dtype, device=cuda, **kw)
-        step.run(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
-                 t["cand"], t["logits"])
-        torch.cuda.synchronize()
-        compare_full(host, step, t)
-        return
+
+        def run(stream):
+            step.run(t["q"], t["k_new"], t["v_new"], t["k_cache"], t["v_cache"], t["cache_len"], t["parent"],
+                     t["cand"], t["logits"], stream=stream)
+
+        return run, lambda: compare_full(host, step, t)
 
     # paged: the pools hold the dense cache, padded to whole pages, under a seeded table
     ps = c["page_size"]
@@ -128,24 +139,52 @@ def check_case(c: dict, cuda):
     kp = paging.to_pages(kc, table, ps, n_pages).to(cuda)
     vp = paging.to_pages(vc, table, ps, n_pages).to(cuda)
     t = to_dev(host, cuda)
+    table_dev = table.to(cuda)
     step = pkg.VerifyStep(B, T, Hq, w.Hkv, D, cap, V, w.torch_dtype, device=cuda, page_size=ps, **kw)
-    step.run(t["q"], t["k_new"], t["v_new"], kp, vp, t["cache_len"], t["parent"], t["cand"], t["logits"],
-             block_table=table.to(cuda))
+
+    def run(stream):
+        step.run(t["q"], t["k_new"], t["v_new"], kp, vp, t["cache_len"], t["parent"], t["cand"], t["logits"],
+                 block_table=table_dev, stream=stream)
+
+    def check():
+        ref = oracle.verify_step(host, typical=typical)
+        assert step.device_status() == 0
+        err = (step.out.double().cpu() - ref["out"]).abs().max().item()
+        assert err <= ATOL[w.torch_dtype], err
+        for name in ("argmax", "path", "accept_len", "bonus"):
+            assert torch.equal(getattr(step, name).cpu(), ref[name]), name
+        assert torch.equal(step.src_index.cpu(), ref["path"])
+        assert torch.equal(step.new_cache_len.cpu(), ref["cache_len"])
+        iview = torch.int16 if w.torch_dtype == torch.bfloat16 else torch.int32
+        for pool, want in ((kp, ref["k_cache"]), (vp, ref["v_cache"])):
+            view = paging.from_pages(pool.cpu(), table, ps, cap)
+            for b in range(B):
+                n = int(ref["cache_len"][b])
+                assert torch.equal(view[b, :, :n].view(iview), want[b, :, :n].view(iview)), b
+
+    return run, check
+
+
+N_STREAMS = 6
+
+
+@pytest.mark.parametrize("group", range(4))
+def test_independent_steps_on_separate_streams(group, cuda):
+    """Six seeded cases (dense and paged caches, every schedule, launch mode
+    and acceptance rule that draw() gives), each with its own VerifyStep on its
+    own stream, issued interleaved three times over without any dependency
+    between the streams, so that their kernels run at the same time: every
+    case still matches the oracle, so steps share no device state."""
+    cases = [prepare_case(draw(3000 + N_STREAMS * group + k), cuda) for k in range(N_STREAMS)]
+    streams = [torch.cuda.Stream() for _ in cases]
     torch.cuda.synchronize()
-    ref = oracle.verify_step(host, typical=typical)
-    assert step.device_status() == 0
-    err = (step.out.double().cpu() - ref["out"]).abs().max().item()
-    assert err <= ATOL[w.torch_dtype], err
-    for name in ("argmax", "path", "accept_len", "bonus"):
-        assert torch.equal(getattr(step, name).cpu(), ref[name]), name
-    assert torch.equal(step.src_index.cpu(), ref["path"])
-    assert torch.equal(step.new_cache_len.cpu(), ref["cache_len"])
-    iview = torch.int16 if w.torch_dtype == torch.bfloat16 else torch.int32
-    for pool, want in ((kp, ref["k_cache"]), (vp, ref["v_cache"])):
-        view = paging.from_pages(pool.cpu(), table, ps, cap)
-        for b in range(B):
-            n = int(ref["cache_len"][b])
-            assert torch.equal(view[b, :, :n].view(iview), want[b, :, :n].view(iview)), b
+    for _ in range(3):
+        for (run, _), s in zip(cases, streams):
+            with torch.cuda.stream(s):
+                run(s)
+    torch.cuda.synchronize()
+    for _, check in cases:
+        check()
 
 
 N_ERRORS = 40
