@@ -128,7 +128,29 @@ __global__ void __launch_bounds__(kTkThreads) topk_kernel(const TopkArgs a) {
     }
 }
 
-// e[r] = w[t] / ||w[t]||_2, one CTA per row.
+// 16-byte chunks of a row that each thread of the embedding keeps in registers
+// (rows of up to 8 * 256 * 4 = 8192 bf16 take the one-read path).
+constexpr int kEmbedChunks = 4;
+
+__device__ __forceinline__ float bf16_lo(uint32_t u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t u) { return __uint_as_float(u & 0xFFFF0000u); }
+
+// Sum of squares over a CTA of 256 threads (8 warps).
+__device__ __forceinline__ float block_sum(float s, float *s_sum) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if ((threadIdx.x & 31) == 0) s_sum[threadIdx.x >> 5] = s;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) tot += s_sum[i];
+    return tot;
+}
+
+// e[r] = w[t] / ||w[t]||_2, one CTA per row.  Rows of whole 16-byte chunks
+// (H a multiple of 8, 16-byte aligned w and e) are read once, all of a
+// thread's chunks at the same time, and scaled from registers; others take a
+// plain element loop.
 __global__ void __launch_bounds__(256) embed_rows_kernel(const __nv_bfloat16 *w, const int32_t *tokens,
                                                          __nv_bfloat16 *e, int V, int H, int32_t *status) {
     __shared__ float s_sum[8];
@@ -141,18 +163,49 @@ __global__ void __launch_bounds__(256) embed_rows_kernel(const __nv_bfloat16 *w,
         return;
     }
     const __nv_bfloat16 *src = w + (size_t)t * H;
+    const int n_chunks = H / 8;
+    const bool vec = (H % 8) == 0 && n_chunks <= kEmbedChunks * 256 &&
+                     ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0;
+    if (vec) {
+        uint4 c[kEmbedChunks];
+#pragma unroll
+        for (int k = 0; k < kEmbedChunks; ++k) {
+            const int i = threadIdx.x + 256 * k;
+            c[k] = i < n_chunks ? __ldg(reinterpret_cast<const uint4 *>(src) + i) : make_uint4(0, 0, 0, 0);
+        }
+        float s = 0.f;
+#pragma unroll
+        for (int k = 0; k < kEmbedChunks; ++k) {
+            const uint32_t u[4] = {c[k].x, c[k].y, c[k].z, c[k].w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                s = fmaf(bf16_lo(u[q]), bf16_lo(u[q]), s);
+                s = fmaf(bf16_hi(u[q]), bf16_hi(u[q]), s);
+            }
+        }
+        const float tot = block_sum(s, s_sum);
+        const float inv = tot > 0.f ? 1.f / sqrtf(tot) : 0.f;
+#pragma unroll
+        for (int k = 0; k < kEmbedChunks; ++k) {
+            const int i = threadIdx.x + 256 * k;
+            if (i >= n_chunks) break;
+            const uint32_t u[4] = {c[k].x, c[k].y, c[k].z, c[k].w};
+            uint32_t o[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const __nv_bfloat162 v = __floats2bfloat162_rn(bf16_lo(u[q]) * inv, bf16_hi(u[q]) * inv);
+                o[q] = *reinterpret_cast<const uint32_t *>(&v);
+            }
+            reinterpret_cast<uint4 *>(dst)[i] = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+        return;
+    }
     float s = 0.f;
     for (int h = threadIdx.x; h < H; h += blockDim.x) {
         const float v = __bfloat162float(src[h]);
         s = fmaf(v, v, s);
     }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-    if ((threadIdx.x & 31) == 0) s_sum[threadIdx.x >> 5] = s;
-    __syncthreads();
-    float tot = 0.f;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) tot += s_sum[i];
+    const float tot = block_sum(s, s_sum);
     const float inv = tot > 0.f ? 1.f / sqrtf(tot) : 0.f;
     for (int h = threadIdx.x; h < H; h += blockDim.x) dst[h] = __float2bfloat16_rn(__bfloat162float(src[h]) * inv);
 }

@@ -117,22 +117,29 @@ def test_topk_matches_oracle(R, V, k):
         assert torch.equal(v.cpu().double(), vals)
 
 
-def test_embed_rows_and_invalid_token():
+@pytest.mark.parametrize("H,offset", [(4096, 0), (1001, 0), (8200, 0), (4096, 1)],
+                         ids=["vector", "odd_width", "wide", "unaligned"])
+def test_embed_rows_and_invalid_token(H, offset):
+    """Rows of whole 16-byte chunks up to 8192 wide take the kernel's one-read
+    vector path; an odd width, a wider row or a weight not 16-byte aligned
+    (offset by one element) the element loop."""
     g = torch.Generator().manual_seed(9)
-    V, H = 5000, 4096
+    V = 5000
     w = rand((V, H), g)
     w[11] = 0
     toks = torch.tensor([4, 4999, 0, 11, 4, 2500], dtype=torch.int32)
     ref = oracle.embed_rows(w, toks)
     e = torch.empty((len(toks), H), dtype=BF, device=DEV)
     st = torch.zeros(1, dtype=torch.int32, device=DEV)
-    pkg.clover_embed_rows(w.to(DEV), toks.to(DEV), e, status=st)
+    w_dev = torch.empty(V * H + offset, dtype=BF, device=DEV)[offset:].view(V, H)
+    w_dev.copy_(w)
+    pkg.clover_embed_rows(w_dev, toks.to(DEV), e, status=st)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     assert ((e.cpu().double() - ref).abs() <= (2.0 ** -8) * ref.abs() + 1e-6).all()
     bad = toks.clone()
     bad[2] = V
-    pkg.clover_embed_rows(w.to(DEV), bad.to(DEV), e, status=st)
+    pkg.clover_embed_rows(w_dev, bad.to(DEV), e, status=st)
     torch.cuda.synchronize()
     assert int(st.item()) & 1 and (e[2] == 0).all()
 
