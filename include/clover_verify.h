@@ -328,6 +328,21 @@ CLOVER_API clover_status clover_linear(const void *x, const void *w, const void 
                                    int32_t *status, void *stream);
 
 /*
+ * clover_linear with launch flags (clover_linear is this call with flags 0).
+ * CLOVER_LINEAR_PDL: the layer is launched as a programmatic dependent of the
+ * kernel before it in the stream.  Its set-up and the weight tiles of its
+ * first pipeline stages are requested before that kernel completes; x, res,
+ * out, the workspace and the status word are touched only after it does.  The
+ * caller states that the kernel before it does not write w (the layers of a
+ * head step: each reads the activations the one before writes, never a
+ * weight).  Any other flag bit -> CLOVER_ERR_INVALID_ARG.
+ */
+#define CLOVER_LINEAR_PDL 1u
+CLOVER_API clover_status clover_linear_ex(const void *x, const void *w, const void *res, void *out,
+                                      int R, int N, int K, int mode, unsigned flags, void *workspace,
+                                      size_t ws_bytes, int32_t *status, void *stream);
+
+/*
  * The regressive connection's embedding (Section 3.4): e[r] = w[t[r]] / ||w[t[r]]||_2
  * (the token's row of the LM-head weight, normalised), w [V,H], tokens [R]
  * int32, e [R,H] bf16.  A token outside [0, V) -> CLOVER_ERR_INVALID_ARG

@@ -40,6 +40,7 @@ EXPORTS = (
     "clover_kv_commit_paged",
     "clover_linear_workspace_size",
     "clover_linear",
+    "clover_linear_ex",
     "clover_embed_rows",
     "clover_topk_workspace_size",
     "clover_topk",
@@ -61,6 +62,8 @@ LINEAR_F32 = 0
 LINEAR_BF16 = 1
 LINEAR_RES_SILU = 2
 LINEAR_RES = 3
+# Launch flag of clover_linear_ex (CLOVER_LINEAR_PDL).
+LINEAR_PDL = 1
 
 # Bytes of the static scratch buffer behind clover_verify_attn_noalloc
 # (CLOVER_NOALLOC_SCRATCH_BYTES in include/clover_verify.h).
@@ -143,6 +146,8 @@ def load(build_if_missing: bool = False):
         lib.clover_linear_workspace_size.restype = Z
         lib.clover_linear.argtypes = [P, P, P, P, I, I, I, I, P, Z, P, P]
         lib.clover_linear.restype = I
+        lib.clover_linear_ex.argtypes = [P, P, P, P, I, I, I, I, ctypes.c_uint, P, Z, P, P]
+        lib.clover_linear_ex.restype = I
         lib.clover_embed_rows.argtypes = [P, P, P, I, I, I, P, P]
         lib.clover_embed_rows.restype = I
         lib.clover_topk_workspace_size.argtypes = [I, I, I]

@@ -437,11 +437,13 @@ def clover_linear_workspace_size(R, N, K) -> int:
     return int(_lib.load().clover_linear_workspace_size(R, N, K))
 
 
-def clover_linear(x, w, out, res=None, mode="bf16", workspace=None, status=None, stream=None):
+def clover_linear(x, w, out, res=None, mode="bf16", workspace=None, status=None, stream=None, pdl=False):
     """out = x . w^T (fp32 accumulation) with the epilogue `mode`: "f32" (fp32
     out), "bf16", "res_silu" (res + silu(.)), "res" (res + .); x [R,K], w [N,K],
     res/out [R,N].  With a workspace of clover_linear_workspace_size bytes a
-    layer with few weight tiles splits K over more CTAs."""
+    layer with few weight tiles splits K over more CTAs.  pdl=True launches it
+    as a programmatic dependent of the kernel before it in the stream
+    (clover_linear_ex with CLOVER_LINEAR_PDL: that kernel must not write w)."""
     code = _LINEAR_MODES[mode]
     R, K = x.shape
     N = w.shape[0]
@@ -454,8 +456,9 @@ def clover_linear(x, w, out, res=None, mode="bf16", workspace=None, status=None,
         _check(status, (1,), torch.int32, "status")
     _dev(x, w, out, res if code >= 2 else None, workspace, status)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    rc = _lib.load().clover_linear(_ptr(x), _ptr(w), _ptr(res if code >= 2 else None), _ptr(out), R, N, K, code,
-                                   _ptr(workspace), ws_bytes, _ptr(status), _stream(stream))
+    rc = _lib.load().clover_linear_ex(_ptr(x), _ptr(w), _ptr(res if code >= 2 else None), _ptr(out), R, N, K, code,
+                                      _lib.LINEAR_PDL if pdl else 0, _ptr(workspace), ws_bytes, _ptr(status),
+                                      _stream(stream))
     if rc != OK:
         raise CloverError(rc, "clover_linear")
 
@@ -522,11 +525,13 @@ class DraftHead:
 
     def run(self, h, tokens, w_lm, w_v, w_o, w_1, stream=None):
         st = dict(status=self.status, stream=stream)
+        # each layer a programmatic dependent of the kernel before it: its
+        # set-up and first weight tiles overlap that kernel's end
         clover_embed_rows(w_lm, tokens, self.e, **st)
-        clover_linear(self.e, w_v, self.v, mode="bf16", workspace=self.ws_lin, **st)
-        clover_linear(self.v, w_o, self.h, res=h, mode="res", workspace=self.ws_lin, **st)
-        clover_linear(self.h, w_1, self.z, res=self.h, mode="res_silu", workspace=self.ws_lin, **st)
-        clover_linear(self.z, w_lm, self.logits, mode="f32", **st)
+        clover_linear(self.e, w_v, self.v, mode="bf16", workspace=self.ws_lin, pdl=True, **st)
+        clover_linear(self.v, w_o, self.h, res=h, mode="res", workspace=self.ws_lin, pdl=True, **st)
+        clover_linear(self.h, w_1, self.z, res=self.h, mode="res_silu", workspace=self.ws_lin, pdl=True, **st)
+        clover_linear(self.z, w_lm, self.logits, mode="f32", pdl=True, **st)
         clover_topk(self.logits, self.k, self.values, self.indices, self.ws, **st)
 
 

@@ -21,7 +21,7 @@ void accept_plan(int B, int T, int V, int dtype, bool typical, int resident, int
 size_t accept_workspace_bytes(int B, int T, int V, int dtype);
 size_t accept_typical_workspace_bytes(int B, int T, int V, int dtype);
 cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
-                             void *workspace, size_t ws_bytes, int32_t *status, cudaStream_t stream);
+                             void *workspace, size_t ws_bytes, int32_t *status, bool pdl, cudaStream_t stream);
 size_t linear_workspace_bytes(int R, int N, int K);
 size_t topk_workspace_bytes(int R, int V, int k);
 int topk_max_k();
@@ -563,7 +563,13 @@ size_t clover_linear_workspace_size(int R, int N, int K) {
 
 clover_status clover_linear(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
                             void *workspace, size_t ws_bytes, int32_t *status, void *stream) {
+    return clover_linear_ex(x, w, res, out, R, N, K, mode, 0u, workspace, ws_bytes, status, stream);
+}
+
+clover_status clover_linear_ex(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
+                               unsigned flags, void *workspace, size_t ws_bytes, int32_t *status, void *stream) {
     const NvtxRange nvtx_range("clover_linear");
+    if (flags & ~CLOVER_LINEAR_PDL) return CLOVER_ERR_INVALID_ARG;
     if (R < 0 || N < 1 || K < 64 || K % 64 != 0) return CLOVER_ERR_INVALID_ARG;
     if (mode < CLOVER_LINEAR_F32 || mode > CLOVER_LINEAR_RES) return CLOVER_ERR_INVALID_ARG;
     const bool with_res = mode == CLOVER_LINEAR_RES_SILU || mode == CLOVER_LINEAR_RES;
@@ -574,7 +580,7 @@ clover_status clover_linear(const void *x, const void *w, const void *res, void 
         return CLOVER_ERR_INVALID_ARG;
     if (workspace && !aligned16(workspace)) return CLOVER_ERR_INVALID_ARG;
     return from_cuda(launch_linear_tc(x, w, with_res ? res : nullptr, out, R, N, K, mode, workspace, ws_bytes, status,
-                                      static_cast<cudaStream_t>(stream)));
+                                      (flags & CLOVER_LINEAR_PDL) != 0, static_cast<cudaStream_t>(stream)));
 }
 
 clover_status clover_embed_rows(const void *w, const int32_t *tokens, void *e, int R, int V, int H, int32_t *status,

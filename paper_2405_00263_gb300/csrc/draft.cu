@@ -153,6 +153,9 @@ __device__ __forceinline__ float block_sum(float s, float *s_sum) {
 // plain element loop.
 __global__ void __launch_bounds__(256) embed_rows_kernel(const __nv_bfloat16 *w, const int32_t *tokens,
                                                          __nv_bfloat16 *e, int V, int H, int32_t *status) {
+    // a linear layer queued behind this call as a programmatic dependent may
+    // start its set-up now; it waits for this grid before it reads e
+    allow_dependent_launch();
     __shared__ float s_sum[8];
     const int r = blockIdx.x;
     const int t = __ldg(tokens + r);

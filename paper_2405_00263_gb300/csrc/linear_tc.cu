@@ -15,6 +15,14 @@
 // columns of the two weight tiles and of x), warp 1 issues the MMAs (two
 // accumulators), warps 2-5 read the accumulators and write y.  Every wait is
 // bounded; a wait that gives up sets CLOVER_ERR_TIMEOUT and the CTA winds down.
+//
+// Programmatic dependent launch: every CTA lets a dependent grid launch as soon
+// as it starts, and waits for the grid it depends on (griddepcontrol.wait)
+// only before its first touch of x, res, out or the workspace: the weight
+// tiles of the first stages are requested before that wait (the weight is
+// never written by the kernel before it), so a layer's set-up and first
+// weight loads overlap the end of the layer before it.  Launched without the
+// attribute the wait returns at once.
 #include "common.cuh"
 #include "tc_ptx.cuh"
 #include "tmap_host.cuh"
@@ -78,6 +86,7 @@ __global__ void __launch_bounds__(kThreadsL, 1)
     linear_tc_kernel(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_x,
                      const LinArgs a) {
     using S = LinSmem;
+    allow_dependent_launch();
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     uint64_t *full = reinterpret_cast<uint64_t *>(sm + S::bar_off);
@@ -130,12 +139,24 @@ __global__ void __launch_bounds__(kThreadsL, 1)
     if (warp == kProducer && lane == 0) {
         prefetch_tensormap(&tm_w);
         prefetch_tensormap(&tm_x);
+        // the x chunks of the first stages wait for the prerequisite grid
+        // (which writes x); their weight tiles are requested before it
+        int pend_c[kStages];
+        int n_pend = 0;
+        bool waited = false;
+        auto release_x = [&]() {
+            wait_prerequisite_grids();
+            for (int i = 0; i < n_pend; ++i)
+                tma_load_3d(sm + i * S::stage_bytes + 2 * S::w_bytes, &tm_x, &full[i], pend_c[i] * LK, 0, 0);
+            waited = true;
+        };
         int it = 0;
         for (int t = t0; t < t1 && !*s_abort; t += 2) {
             const bool two = t + 1 < t1;
             const uint32_t bytes = (uint32_t)((two ? 2 : 1) * S::w_bytes + a.Rp * LK * 2);
             for (int c = c_lo; c < c_hi; ++c, ++it) {
                 const int s = it % kStages;
+                if (it >= kStages && !waited) release_x();
                 if (!mbar_wait(&empty[s], ((it / kStages) - 1) & 1, kWaitL)) {
                     *s_abort = 1;
                     break;
@@ -144,10 +165,12 @@ __global__ void __launch_bounds__(kThreadsL, 1)
                 mbar_arrive_expect_tx(&full[s], bytes);
                 tma_load_3d(st, &tm_w, &full[s], c * LK, t * LM, 0);
                 if (two) tma_load_3d(st + S::w_bytes, &tm_w, &full[s], c * LK, (t + 1) * LM, 0);
-                tma_load_3d(st + 2 * S::w_bytes, &tm_x, &full[s], c * LK, 0, 0);
+                if (waited) tma_load_3d(st + 2 * S::w_bytes, &tm_x, &full[s], c * LK, 0, 0);
+                else pend_c[n_pend++] = c;            // stage s == n_pend here (it < kStages)
                 issued = it + 1;
             }
         }
+        if (!waited) release_x();
     }
 
     if (warp == kMma && lane == 0) {
@@ -192,6 +215,8 @@ __global__ void __launch_bounds__(kThreadsL, 1)
     }
 
     if (warp >= 2) {
+        // res, out, the partials and the counters after the prerequisite grid
+        wait_prerequisite_grids();
         // warp w reads TMEM lanes 32 (w % 4) .. +31: weight rows m of the tile
         const int quad = warp & 3;
         const int m = quad * 32 + lane;
@@ -330,7 +355,7 @@ size_t linear_workspace_bytes(int R, int N, int K) {
 // linear_workspace_bytes(R, N, K) bytes (zero-filled before first use) the
 // plan's K split is used; without one, none.
 cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void *out, int R, int N, int K, int mode,
-                             void *workspace, size_t ws_bytes, int32_t *status, cudaStream_t stream) {
+                             void *workspace, size_t ws_bytes, int32_t *status, bool pdl, cudaStream_t stream) {
     static unsigned long long done[64];
     static int sms[64];
     cudaError_t err = ensure_smem_attr(linear_tc_kernel, LinSmem::alloc, done);
@@ -370,7 +395,17 @@ cudaError_t launch_linear_tc(const void *x, const void *w, const void *res, void
                                  : nullptr;
         a.status = status;
         const int grid = n_split > 1 ? n_pairs * n_split : min(n_sm, n_tiles);
-        linear_tc_kernel<<<grid, kThreadsL, LinSmem::alloc, stream>>>(tw, tx, a);
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(grid, 1, 1);
+        cfg.blockDim = dim3(kThreadsL, 1, 1);
+        cfg.dynamicSmemBytes = LinSmem::alloc;
+        cfg.stream = stream;
+        cudaLaunchAttribute attr;
+        attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr.val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = &attr;
+        cfg.numAttrs = pdl ? 1 : 0;
+        if ((err = cudaLaunchKernelEx(&cfg, linear_tc_kernel, tw, tx, a)) != cudaSuccess) return err;
         if ((err = cudaGetLastError()) != cudaSuccess) return err;
     }
     return cudaSuccess;

@@ -229,6 +229,10 @@ def test_draft_host_validation(lib):
     assert lin(mode=2) == 1 and lin(mode=3) == 1             # residual modes need res
     assert lin(x=72) == 1 and lin(out=136) == 1              # 16-byte alignment
     assert lin(R=0) == 0
+    lin_ex = lambda flags, R=4, K=64: lib.clover_linear_ex(P(64), P(64), None, P(128), R, 128, K, 1, flags, None, 0,
+                                                           None, None)
+    assert lin_ex(2) == 1 and lin_ex(0xFFFFFFFE) == 1        # unknown flag bits
+    assert lin_ex(1, K=96) == 1 and lin_ex(1, R=0) == 0      # the same checks as clover_linear
     assert lib.clover_topk_workspace_size(3, 1000, 8) == 8 * 3 * 1 * 8 + 4 * 3
     assert lib.clover_topk_workspace_size(3, 125696, 8) == 8 * 3 * 16 * 8 + 4 * 3
     assert lib.clover_topk_workspace_size(1, 100, 33) == 0 and lib.clover_topk_workspace_size(1, 4, 5) == 0

@@ -200,3 +200,49 @@ def test_draft_head_step_against_exact_arithmetic(R, H, V, k):
         got = head.indices[r].cpu().long()
         kth = ex["top_values"][r, -1]
         assert (ex["logits"][r, got] >= kth - 2 * E[r].max()).all()
+
+
+@pytest.mark.parametrize("R", [4, 16, 40, 300])
+def test_linear_chain_programmatic_launch_equals_ordinary(R):
+    """Three dependent layers (x -> y1 -> y2 -> y3, the K-split 4096 x 4096
+    shape up to 32 rows, unsplit above, two launches at 300 rows), each later
+    layer launched as a programmatic dependent of the one before, eagerly and
+    as a replayed CUDA graph: the same bytes as ordinary launches (the same
+    plan and summation order), so no layer read its input or wrote its
+    partials before the layer before it had finished."""
+    g = torch.Generator().manual_seed(77 + R)
+    H = 4096
+    x = rand((R, H), g).to(DEV)
+    ws_ = [rand((H, H), g, std=H ** -0.5).to(DEV) for _ in range(3)]
+    ws = torch.zeros(max(16, pkg.clover_linear_workspace_size(R, H, H)), dtype=torch.uint8, device=DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+
+    def chain(pdl, outs):
+        pkg.clover_linear(x, ws_[0], outs[0], mode="bf16", workspace=ws, status=st)
+        pkg.clover_linear(outs[0], ws_[1], outs[1], res=outs[0], mode="res", workspace=ws, status=st, pdl=pdl)
+        pkg.clover_linear(outs[1], ws_[2], outs[2], res=outs[1], mode="res_silu", workspace=ws, status=st, pdl=pdl)
+
+    ref = [torch.empty((R, H), dtype=BF, device=DEV) for _ in range(3)]
+    chain(False, ref)
+    got = [torch.full((R, H), float("nan"), dtype=BF, device=DEV) for _ in range(3)]
+    chain(True, got)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    for a, b in zip(got, ref):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    stream = torch.cuda.Stream()
+    for o in got:
+        o.fill_(float("nan"))
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for _ in range(3):
+            chain(True, got)
+    graph.replay()
+    graph.replay()
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    for a, b in zip(got, ref):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    if R <= 40:                     # the first layer against the oracle (the others are pinned elsewhere)
+        want = oracle.linear(x.cpu(), ws_[0].cpu())
+        assert ((ref[0].cpu().double() - want).abs() <= linear_tol(x.cpu(), ws_[0].cpu(), want, True)).all()
