@@ -22,7 +22,7 @@
  *                         tree slots (an engine step the paper leaves implicit);
  *   clover_verify_attn_paged, clover_kv_commit_paged
  *                         the attention and the commit on a paged KV cache;
- *   clover_linear, clover_embed_rows, clover_topk
+ *   clover_linear(_ex), clover_embed_rows, clover_topk
  *                         the draft side: the dense layers of a Clover head,
  *                         the LM-head row embedding and the top-k of its
  *                         logits (Section 3).
