@@ -8,7 +8,9 @@
 // chunk's k best keys in k rounds of a block-wide max, each thread proposing
 // its best key not yet taken; it writes them to the workspace, and the CTA that
 // finishes a row's last chunk (an arrival counter) selects the row's k best
-// among the chunks' the same way and resets the counter.
+// among the chunks' the same way and resets the counter.  In the chunk phase a
+// thread keeps its 32 values as 32-bit order bits and its best one between
+// rounds: only the thread whose key won a round looks through its values again.
 #include "common.cuh"
 
 namespace clover {
@@ -91,13 +93,43 @@ __global__ void __launch_bounds__(kTkThreads) topk_kernel(const TopkArgs a) {
     const int c = blockIdx.y;
     const float *row = a.x + (size_t)r * a.V;
     const int lo = c * kTkChunk;
-    uint64_t keys[kTkPer];
+    // value j of this thread is element lo + threadIdx.x + j * kTkThreads; its
+    // order bits, 0 for none (below every value's, so never proposed)
+    uint32_t ob[kTkPer];
 #pragma unroll
     for (int j = 0; j < kTkPer; ++j) {
         const int v = lo + threadIdx.x + j * kTkThreads;
-        keys[j] = v < a.V ? tk_key(__ldcs(row + v), (uint32_t)v) : 0ull;
+        ob[j] = v < a.V ? tk_order_bits(__ldcs(row + v)) : 0u;
     }
-    tk_select<kTkPer>(keys, a.k, s_out, s_red);
+    // the thread's best value not yet taken: the largest order bits, the
+    // smallest j (so the smallest index) among equal ones
+    uint32_t bv = 0u;
+    int bj = -1;
+    auto rescan = [&]() {
+        bv = 0u;
+        bj = -1;
+#pragma unroll
+        for (int j = 0; j < kTkPer; ++j)
+            if (ob[j] > bv) {
+                bv = ob[j];
+                bj = j;
+            }
+    };
+    rescan();
+    for (int i = 0; i < a.k; ++i) {
+        const uint64_t key = bj >= 0 ? (static_cast<uint64_t>(bv) << 32) |
+                                           static_cast<uint64_t>(0xFFFFFFFFu - (uint32_t)(lo + threadIdx.x + bj * kTkThreads))
+                                     : 0ull;
+        const uint64_t m = tk_block_max(key, s_red);
+        // keys are distinct (their indices are), so one thread owns the winner
+        if (bj >= 0 && key == m) {
+#pragma unroll
+            for (int j = 0; j < kTkPer; ++j)
+                if (j == bj) ob[j] = 0u;
+            rescan();
+        }
+        if (threadIdx.x == 0) s_out[i] = m;
+    }
     if (threadIdx.x == 0) {
         unsigned long long *dst = a.cand + ((size_t)r * a.n_chunks + c) * a.k;
         for (int j = 0; j < a.k; ++j) dst[j] = s_out[j];
