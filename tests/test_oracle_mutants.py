@@ -188,3 +188,68 @@ def test_unmutated_copy_passes_every_pin(libs, monkeypatch):
 @pytest.mark.parametrize("name,areas", [(m[0], m[3]) for m in MUTANTS], ids=[m[0] for m in MUTANTS])
 def test_pins_reject_planted_mistake(name, areas, libs, monkeypatch):
     assert failing_pins(libs[name], areas, monkeypatch), f"no pin of {areas} rejects the mutant {name}"
+
+
+# ---------------------------------------------------------------------------
+# The oracle's Python compositions (oracle/__init__.py): one slip in a
+# function's source, the function rebuilt from it beside the real one and
+# swapped in for it.
+# ---------------------------------------------------------------------------
+
+HEAD = ("test_head_step",)
+
+# name, the oracle function, the source text replaced (once in that function), its replacement, the pin areas
+PY_MUTANTS = [
+    ("verify_step_without_append", "verify_step",
+     '    append_tree_kv(inp["k_new"], inp["v_new"], k_cache, v_cache, cache_len)\n', "", ("test_verify_step",)),
+    ("head_step_residual_dropped", "clover_head_step", "    h1 = h.double() + d\n", "    h1 = d\n", HEAD),
+    ("head_step_decoder_weights_swapped", "clover_head_step",
+     "    a = linear(e.to(bf), w_v)\n    d = linear(a.to(bf), w_o)\n",
+     "    a = linear(e.to(bf), w_o)\n    d = linear(a.to(bf), w_v)\n", HEAD),
+    ("head_step_mlp_residual_from_input", "clover_head_step", "res=h1.to(bf), act=1)", "res=h.to(bf), act=1)", HEAD),
+    ("head_step_lm_head_before_mlp", "clover_head_step", "    logits = linear(z.to(bf), w_lm)\n",
+     "    logits = linear(h1.to(bf), w_lm)\n", HEAD),
+]
+
+
+def rebuild(fn_name: str, old: str = "", new: str = ""):
+    """The oracle function `fn_name` defined again from its source, with `old`
+    replaced by `new` when given, over a copy of the oracle module's globals
+    (so that it calls the real library functions)."""
+    import inspect
+    src = inspect.getsource(getattr(oracle, fn_name))
+    if old:
+        assert src.count(old) == 1, f"the mutation site must occur exactly once in {fn_name}: {old!r}"
+        src = src.replace(old, new)
+    ns = dict(vars(oracle))
+    exec(compile(src, oracle.__file__, "exec"), ns)
+    return ns[fn_name]
+
+
+def failing_pins_py(fn_name, fn, areas, monkeypatch) -> list[str]:
+    failed = []
+    with monkeypatch.context() as m:
+        m.setattr(oracle, fn_name, fn)
+        for name, pin, kw in pin_cases(areas):
+            try:
+                pin(**kw)
+            except pytest.skip.Exception:
+                continue
+            except (Exception, pytest.fail.Exception):
+                failed.append(f"{name}{kw or ''}")
+    return failed
+
+
+def test_unmutated_python_compositions_pass_their_pins(monkeypatch):
+    """The control: each function rebuilt from its unchanged source passes
+    every pin of its areas."""
+    for fn_name in sorted({m[1] for m in PY_MUTANTS}):
+        areas = tuple(sorted({a for _, f, _, _, ar in PY_MUTANTS if f == fn_name for a in ar}))
+        assert sum(1 for _ in pin_cases(areas)) > 0
+        assert failing_pins_py(fn_name, rebuild(fn_name), areas, monkeypatch) == []
+
+
+@pytest.mark.parametrize("name,fn_name,old,new,areas", PY_MUTANTS, ids=[m[0] for m in PY_MUTANTS])
+def test_pins_reject_planted_composition_mistake(name, fn_name, old, new, areas, monkeypatch):
+    fn = rebuild(fn_name, old, new)
+    assert failing_pins_py(fn_name, fn, areas, monkeypatch), f"no pin of {areas} rejects the mutant {name}"
