@@ -202,6 +202,9 @@ HEAD = ("test_head_step",)
 PY_MUTANTS = [
     ("verify_step_without_append", "verify_step",
      '    append_tree_kv(inp["k_new"], inp["v_new"], k_cache, v_cache, cache_len)\n', "", ("test_verify_step",)),
+    ("verify_step_typical_outputs_swapped", "verify_step",
+     '        amax, path, alen, bonus = r["argmax"], r["path"], r["accept_len"], r["bonus"]\n',
+     '        amax, path, alen, bonus = r["argmax"], r["path"], r["accept_len"], r["argmax"][:, 0]\n', ("test_verify_step",)),
     ("head_step_residual_dropped", "clover_head_step", "    h1 = h.double() + d\n", "    h1 = d\n", HEAD),
     ("head_step_decoder_weights_swapped", "clover_head_step",
      "    a = linear(e.to(bf), w_v)\n    d = linear(a.to(bf), w_o)\n",

@@ -570,6 +570,25 @@ def test_verify_step_tiny_invariants():
     assert torch.equal(r["v_cache"][0, :, L:L + a], t["v_new"][0, p].permute(1, 0, 2))
 
 
+def test_verify_step_typical_at_small_temperature_is_greedy():
+    """The whole step under typical acceptance at temperature 1e-3: every
+    argmax candidate has probability ~1 (the logits' top gap is far above the
+    temperature) and every other candidate ~0, so with epsilon = delta = 0.3
+    exactly the argmax children pass and the step equals the greedy step
+    (siblings are distinct by construction)."""
+    w = workloads.get("tiny_f32")
+    t = workloads.make(w)
+    top2 = t["logits"].double().topk(2, dim=-1).values
+    assert (top2[..., 0] - top2[..., 1]).min() > 0.05
+    g = oracle.verify_step(t)
+    ty = oracle.verify_step(t, typical=(1e-3, 0.3, 0.3))
+    for key in ("out", "argmax", "path", "accept_len", "bonus", "src_index", "cache_len"):
+        assert torch.equal(ty[key], g[key]), key
+    a = int(g["accept_len"][0])
+    L = int(t["cache_len"][0])
+    assert torch.equal(ty["k_cache"][0, :, :L + a], g["k_cache"][0, :, :L + a])
+
+
 # ---------------------------------------------------------------------------
 # A6: typical acceptance (the sampling-side acceptance rule)
 # ---------------------------------------------------------------------------
