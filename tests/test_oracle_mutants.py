@@ -212,6 +212,11 @@ PY_MUTANTS = [
     ("head_step_mlp_residual_from_input", "clover_head_step", "res=h1.to(bf), act=1)", "res=h.to(bf), act=1)", HEAD),
     ("head_step_lm_head_before_mlp", "clover_head_step", "    logits = linear(z.to(bf), w_lm)\n",
      "    logits = linear(h1.to(bf), w_lm)\n", HEAD),
+    # the fp64 statement of the head step (the reference of the rounding bound)
+    ("exact_step_silu_sign", "clover_head_step_exact", "u / (1.0 + torch.exp(-u))", "u / (1.0 + torch.exp(u))", HEAD),
+    ("exact_step_weight_transposed", "clover_head_step_exact", "    a = e @ W_v.T\n", "    a = e @ W_v\n", HEAD),
+    ("exact_step_mlp_residual_dropped", "clover_head_step_exact", "    z = h1 + u / (1.0 + torch.exp(-u))\n",
+     "    z = u / (1.0 + torch.exp(-u))\n", HEAD),
 ]
 
 
